@@ -1,0 +1,247 @@
+"""PalQuant CPU oracle -- test infrastructure only.
+
+A plain, slow, obviously correct CPU statement of the PalQuant layer (Hu et al.,
+arXiv 2208.01944): group-wise activation quantisation (Sec. 3.2, Eq. 2), the
+B-bit group convolution of parallel low-precision quantisation (Sec. 4.1), the
+de-quantising rescale with the output scale alpha (Sec. 3.2), the cyclic
+permutation of the cyclic shuffle (Sec. 4.2, Eq. 6-8) and requantisation for the
+next layer.  The arithmetic lives in ``palquant_oracle.c`` (int64 nested loops,
+fp32 decisions made exactly as written there); this module only builds that file
+with gcc and marshals numpy arrays to it.
+
+Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  It imports nothing from the GPU library and
+the GPU library imports nothing from it.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "palquant_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_SO = os.path.join(_BUILD, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+# Compiler flags: no contraction of a*b+c into fused multiply-adds and no fast
+# math, so every fp32 decision is one IEEE round-to-nearest operation.
+CFLAGS = ["-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fopenmp", "-fPIC", "-shared"]
+
+
+def build(force: bool = False, src: str = _SRC, out: str = _SO) -> str:
+    """Compile the oracle C file into a shared library (gcc) and return its path."""
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    if force or not os.path.exists(out) or os.path.getmtime(out) < os.path.getmtime(src):
+        tmp = out + ".tmp%d" % os.getpid()
+        subprocess.check_call(["gcc", *CFLAGS, "-o", tmp, src, "-lm"])
+        os.replace(tmp, out)
+    return out
+
+
+_I64 = ctypes.c_int64
+_I32 = ctypes.c_int
+_P = ctypes.c_void_p
+
+
+def _declare(lib):
+    lib.oracle_num_threads.restype = _I32
+    lib.oracle_set_num_threads.argtypes = [_I32]
+    lib.oracle_quantize_act.argtypes = [_P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _P]
+    lib.oracle_quantize_weights.argtypes = [_P, _P, _I32, _I32, _I32, _I32, _I32, _I32, _P]
+    lib.oracle_group_conv.restype = _I64
+    lib.oracle_group_conv.argtypes = [_P, _P, _P, _I64, _I64, _I64] + [_I32] * 7
+    lib.oracle_group_conv_pixels.argtypes = [_P, _P, _P, _P, _I64, _I64, _I64, _I64] + [_I32] * 7
+    lib.oracle_group_perm.restype = _I32
+    lib.oracle_group_perm.argtypes = [_I32, _I32, _I32, _P, _P]
+    lib.oracle_epilogue.restype = _I32
+    lib.oracle_epilogue.argtypes = [_P, _I64, _I32, _I32, _P, _P, _I32, _I32, _P, _P, _I32, _I32, _P, _P, _P]
+    lib.oracle_act_step.argtypes = [_P, _I64, _I64, _I64, _I32, _I32, _I32, _P]
+    lib.oracle_weight_step.argtypes = [_P, _I32, _I64, _I32, _P]
+    lib.oracle_inv_step.restype = ctypes.c_float
+    lib.oracle_inv_step.argtypes = [ctypes.c_float]
+    lib.oracle_epilogue_scales.restype = _I32
+    lib.oracle_epilogue_scales.argtypes = [_I32, _P, _P, ctypes.c_double, _P, _I32, _I32, _P, _P, _P]
+    return lib
+
+
+def lib():
+    """The loaded oracle library (built on first use)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            _lib = _declare(ctypes.CDLL(build()))
+        return _lib
+
+
+def load_variant(path: str):
+    """Load another build of the oracle source (used by the mutation tests)."""
+    return _declare(ctypes.CDLL(path))
+
+
+def _ptr(a: np.ndarray | None):
+    if a is None:
+        return None
+    assert a.flags["C_CONTIGUOUS"], "oracle arrays must be C-contiguous"
+    return a.ctypes.data
+
+
+def _f32(a):
+    return np.ascontiguousarray(np.asarray(a, dtype=np.float32))
+
+
+def out_dim(n: int, k: int, s: int, p: int) -> int:
+    return (n + 2 * p - k) // s + 1
+
+
+def num_threads(L=None) -> int:
+    return (L or lib()).oracle_num_threads()
+
+
+def set_num_threads(n: int, L=None) -> None:
+    (L or lib()).oracle_set_num_threads(int(n))
+
+
+def quantize_act(x: np.ndarray, G: int, bits: int, inv_s, L=None) -> np.ndarray:
+    """Eq. 2 per group: codes = clamp(rint(x * inv_s[g]), 0, 2^bits - 1); x is NHWC fp32."""
+    L = L or lib()
+    x = _f32(x)
+    N, H, W, C = x.shape
+    assert C % G == 0
+    inv_s = _f32(inv_s)
+    assert inv_s.shape == (G,)
+    q = np.empty(x.shape, dtype=np.uint8)
+    L.oracle_quantize_act(_ptr(x), _ptr(q), N, H, W, G, C // G, bits, _ptr(inv_s))
+    return q
+
+
+def quantize_weights(w: np.ndarray, bits: int, inv_sw, L=None) -> np.ndarray:
+    """Signed codes clamp(rint(w * inv_sw[g]), -2^(b-1), 2^(b-1)-1); w is [G,Cout_g,kh,kw,Cin_g]."""
+    L = L or lib()
+    w = _f32(w)
+    G, Co, kh, kw, Ci = w.shape
+    inv_sw = _f32(inv_sw)
+    assert inv_sw.shape == (G,)
+    wq = np.empty(w.shape, dtype=np.int8)
+    L.oracle_quantize_weights(_ptr(w), _ptr(wq), G, Co, kh, kw, Ci, bits, _ptr(inv_sw))
+    return wq
+
+
+def group_conv(q: np.ndarray, wq: np.ndarray, stride: int, pad: int, L=None) -> np.ndarray:
+    """B-bit group convolution (Sec. 4.1) in int64: returns acc [N,Ho,Wo,G*Cout_g]."""
+    L = L or lib()
+    q = np.ascontiguousarray(q, dtype=np.uint8)
+    wq = np.ascontiguousarray(wq, dtype=np.int8)
+    N, H, W, C = q.shape
+    G, Co, kh, kw, Ci = wq.shape
+    assert C == G * Ci
+    Ho, Wo = out_dim(H, kh, stride, pad), out_dim(W, kw, stride, pad)
+    acc = np.empty((N, Ho, Wo, G * Co), dtype=np.int64)
+    L.oracle_group_conv(_ptr(q), _ptr(wq), _ptr(acc), N, H, W, G, Ci, Co, kh, kw, stride, pad)
+    return acc
+
+
+def group_conv_pixels(q: np.ndarray, wq: np.ndarray, stride: int, pad: int, pix: np.ndarray, L=None) -> np.ndarray:
+    """The group convolution at selected output pixels (flat index (n*Ho+oh)*Wo+ow)."""
+    L = L or lib()
+    q = np.ascontiguousarray(q, dtype=np.uint8)
+    wq = np.ascontiguousarray(wq, dtype=np.int8)
+    pix = np.ascontiguousarray(pix, dtype=np.int64)
+    N, H, W, C = q.shape
+    G, Co, kh, kw, Ci = wq.shape
+    acc = np.empty((pix.shape[0], G * Co), dtype=np.int64)
+    L.oracle_group_conv_pixels(_ptr(q), _ptr(wq), _ptr(acc), _ptr(pix), pix.shape[0], N, H, W, G, Ci, Co, kh, kw, stride, pad)
+    return acc
+
+
+def group_perm(G: int, kind: int = 1, shift: int = 1, perm=None, L=None) -> np.ndarray:
+    """Destination group of every source group (Eq. 6 for kind 1, shift 1)."""
+    L = L or lib()
+    p = None if perm is None else np.ascontiguousarray(perm, dtype=np.int32)
+    dst = np.empty(G, dtype=np.int32)
+    rc = L.oracle_group_perm(G, kind, shift, _ptr(p), _ptr(dst))
+    if rc != 0:
+        raise ValueError("shuffle spec is not a permutation")
+    return dst
+
+
+def epilogue(acc: np.ndarray, G: int, m_out, m_req=None, kind: int = 1, shift: int = 1, perm=None,
+             shortcut: np.ndarray | None = None, relu: bool = True, bits_out: int = 2, L=None):
+    """Rescale, optional shortcut add, ReLU, output permutation and requantisation.
+
+    acc is [..., G*Cout_g] int64; returns (acc_out int32, y_out fp32, q_out uint8) in the
+    permuted channel order (q_out is None when m_req is None)."""
+    L = L or lib()
+    acc = np.ascontiguousarray(acc, dtype=np.int64)
+    shape = acc.shape
+    C = shape[-1]
+    Co = C // G
+    npix = acc.size // C
+    m_out = _f32(m_out)
+    m_req_a = None if m_req is None else _f32(m_req)
+    p = None if perm is None else np.ascontiguousarray(perm, dtype=np.int32)
+    sc = None if shortcut is None else _f32(shortcut)
+    if sc is not None:
+        assert sc.shape == shape
+    acc_out = np.empty(shape, dtype=np.int32)
+    y_out = np.empty(shape, dtype=np.float32)
+    q_out = None if m_req_a is None else np.empty(shape, dtype=np.uint8)
+    rc = L.oracle_epilogue(_ptr(acc), npix, G, Co, _ptr(m_out), _ptr(m_req_a), kind, shift, _ptr(p), _ptr(sc),
+                           int(bool(relu)), bits_out, _ptr(acc_out), _ptr(y_out), _ptr(q_out))
+    if rc != 0:
+        raise ValueError("oracle epilogue rejected its input (|acc| >= 2^24 or bad shuffle)")
+    return acc_out, y_out, q_out
+
+
+def act_step(x: np.ndarray, G: int, bits: int, L=None) -> np.ndarray:
+    """LSQ step initialisation per group: 2*mean(x_g)/sqrt(2^b-1), mean in double."""
+    L = L or lib()
+    x = _f32(x)
+    N, H, W, C = x.shape
+    s = np.empty(G, dtype=np.float32)
+    L.oracle_act_step(_ptr(x), N, H, W, G, C // G, bits, _ptr(s))
+    return s
+
+
+def weight_step(w: np.ndarray, bits: int, L=None) -> np.ndarray:
+    """LSQ step initialisation per group: 2*mean|w_g|/sqrt(2^(b-1)-1), mean in double."""
+    L = L or lib()
+    w = _f32(w)
+    G = w.shape[0]
+    s = np.empty(G, dtype=np.float32)
+    L.oracle_weight_step(_ptr(w), G, w.size // G, bits, _ptr(s))
+    return s
+
+
+def inv_step(s) -> np.ndarray:
+    """fl(1/s) computed in double, the multiplier both implementations use."""
+    L = lib()
+    return np.array([L.oracle_inv_step(float(v)) for v in np.asarray(s, dtype=np.float32)], dtype=np.float32)
+
+
+def epilogue_scales(s_w, s_a, s_next=None, alpha: float = 1.0, kind: int = 1, shift: int = 1, perm=None, L=None):
+    """(m_out, m_req): fl(s_w s_a alpha) and fl(s_w s_a alpha / s_next[dst(g)])."""
+    L = L or lib()
+    s_w, s_a = _f32(s_w), _f32(s_a)
+    G = s_w.shape[0]
+    sn = None if s_next is None else _f32(s_next)
+    p = None if perm is None else np.ascontiguousarray(perm, dtype=np.int32)
+    m_out = np.empty(G, dtype=np.float32)
+    m_req = np.empty(G, dtype=np.float32)
+    rc = L.oracle_epilogue_scales(G, _ptr(s_w), _ptr(s_a), float(alpha), _ptr(sn), kind, shift, _ptr(p), _ptr(m_out), _ptr(m_req))
+    if rc != 0:
+        raise ValueError("bad shuffle spec")
+    return m_out, (m_req if sn is not None else None)
+
+
+def layer(x_codes: np.ndarray, wq: np.ndarray, stride: int, pad: int, m_out, m_req=None, kind: int = 1,
+          shift: int = 1, perm=None, shortcut=None, relu: bool = True, bits_out: int = 2, L=None):
+    """One PalQuant layer on codes: group conv then the epilogue.  Returns (acc, y, q)."""
+    G = wq.shape[0]
+    acc = group_conv(x_codes, wq, stride, pad, L=L)
+    return epilogue(acc, G, m_out, m_req, kind, shift, perm, shortcut, relu, bits_out, L=L)
