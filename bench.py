@@ -1,0 +1,385 @@
+#!/usr/bin/env python
+"""Benchmark of the PalQuant layer hot path on GB300.
+
+One step = one pass of the whole hot path over one batch of the ResNet-18 stage-1
+shaped PalQuant 3x3 layer (batch 64, 56x56, G = 4 groups of 64 channels, 2-bit
+activations and weights, cyclic shuffle):
+  (1) group-wise activation quantisation of the fp32 NHWC input (205.5 MB) into int8
+      codes, and (2) the fused layer: B-bit group convolution on the tensor cores,
+      rescale, ReLU, cyclic-shuffle output permutation and requantisation into the
+      next layer's codes (51.4 MB).
+Inputs are resident in HBM when the timed region starts; two input buffers are used
+in turn so each step reads an input larger than L2 that the previous step did not.
+
+Prints one JSON line (rank 0).  `--impl reference` times the CPU oracle instead.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "PalQuant layer int TOPS and % of GB300 dense INT8 peak; ResNet-18-shaped images/s"
+UNIT = "TOPS"
+WORKLOAD = "ResNet-18 stage-1 3x3 PalQuant layer: batch 64, 56x56, G=4 groups of 64->64, b=2, stride 1, pad 1, cyclic shuffle"
+PEAKS_FILE = os.path.join(ROOT, "MEASURED_PEAKS.json")
+TRAFFIC_FILE = os.path.join(ROOT, "profiles", "dram_traffic.json")
+CSRC = os.path.join(ROOT, "paper_2208_01944_gb300", "csrc")
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline sample")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(PEAKS_FILE) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d["bf16_tflops"]), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
+
+
+def source_sha(files):
+    h = hashlib.sha256()
+    for fn in files:
+        with open(os.path.join(CSRC, fn), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+KERNEL_SOURCES = {
+    "pq_quantize_vec16": ["quantize.cu", "pq_internal.h"],
+    "pq_conv_tc_kernel": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
+}
+
+
+def dram_traffic(kernel):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel source is unchanged."""
+    try:
+        with open(TRAFFIC_FILE) as f:
+            d = json.load(f)[kernel]
+        if d.get("source_sha") != source_sha(KERNEL_SOURCES[kernel]):
+            return None
+        return d["bytes_per_launch"]
+    except Exception:
+        return None
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle sampling while the timed region runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.QUERY,
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"], "samples": 0}
+        time.sleep(0.25)
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        rows = [r.split(",") for r in out.strip().splitlines() if r.strip()]
+        sm, smax, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for r in rows:
+            r = [v.strip() for v in r]
+            if len(r) < 9:
+                continue
+            try:
+                sm.append(float(r[1]))
+                smax = float(r[2])
+            except ValueError:
+                continue
+            for name, v in zip(names, r[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        sm.sort()
+        med = sm[len(sm) // 2] if sm else None
+        return {"sm_mhz": med, "sm_max_mhz": smax, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def make_layer_inputs():
+    from paper_2208_01944_gb300 import synth, workloads
+
+    c = workloads.CONFIG1
+    x, w = synth.layer_inputs(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, seed=0)
+    return c, x, w
+
+
+# ---------------------------------------------------------------------------
+# Reference arm: the CPU oracle, as it stands, on the host cores.
+# ---------------------------------------------------------------------------
+def oracle_sample_step(c, x, w, n_img, inv_s, inv_sw, m_out, m_req):
+    import oracle
+
+    xs = x[:n_img]
+    q = oracle.quantize_act(xs, c.G, c.bits_a, inv_s)
+    wq = oracle.quantize_weights(w, c.bits_w, inv_sw)
+    oracle.layer(q, wq, c.stride, c.pad, m_out, m_req, c.shuffle_kind, c.shuffle_shift, relu=c.relu, bits_out=c.bits_out)
+
+
+def oracle_setup(c, x, w):
+    import oracle
+
+    s_a = oracle.act_step(x[:4], c.G, c.bits_a)
+    s_w = oracle.weight_step(w, c.bits_w)
+    m_out, m_req = oracle.epilogue_scales(s_w, s_a, s_a, 1.0, c.shuffle_kind, c.shuffle_shift)
+    return oracle.inv_step(s_a), oracle.inv_step(s_w), m_out, m_req
+
+
+def oracle_images_for(seconds, c, x, w, setup):
+    t0 = time.perf_counter()
+    oracle_sample_step(c, x, w, 1, *setup)
+    per_img = time.perf_counter() - t0
+    return max(1, min(c.N, int(seconds / max(per_img, 1e-6)))), per_img
+
+
+def cpu_baseline(c, x, w, seconds):
+    import oracle
+
+    setup = oracle_setup(c, x, w)
+    n_img, _ = oracle_images_for(seconds, c, x, w, setup)
+    t0 = time.perf_counter()
+    oracle_sample_step(c, x, w, n_img, *setup)
+    dt = time.perf_counter() - t0
+    ops = c.int_ops * n_img / c.N
+    return {"value": ops / dt / 1e12, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+            "sample": f"{n_img} of the {c.N} images of the workload (quantize + group conv + epilogue), {dt:.2f} s"}
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return
+    import oracle
+
+    c, x, w = make_layer_inputs()
+    setup = oracle_setup(c, x, w)
+    # each step: a bounded sample (whole images) sized so K + W steps take a few minutes
+    budget = 150.0 / max(1, args.steps + args.warmup)
+    n_img, _ = oracle_images_for(min(budget, 20.0), c, x, w, setup)
+    for _ in range(args.warmup):
+        oracle_sample_step(c, x, w, n_img, *setup)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_sample_step(c, x, w, n_img, *setup)
+    dt = (time.perf_counter() - t0) / max(1, args.steps)
+    ops = c.int_ops * n_img / c.N
+    value = ops / dt / 1e12
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": dt * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "sample_images_per_step": n_img, "global_batch": c.N},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": oracle.num_threads(), "kind": "oracle",
+                         "sample": f"{n_img} of {c.N} images per step (quantize + group conv + epilogue)"},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+# ---------------------------------------------------------------------------
+# Our arm.
+# ---------------------------------------------------------------------------
+def run_ours(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+    import torch.distributed as dist
+
+    from paper_2208_01944_gb300 import binding as B
+
+    dev = torch.device("cuda", local_rank)
+    torch.cuda.set_device(dev)
+    c, x_np, w_np = make_layer_inputs()
+
+    # ---- set-up (untimed): steps from the library's own calibration
+    stream = torch.cuda.Stream(device=dev)
+    xs = [torch.from_numpy(x_np).to(dev)]
+    xs.append(torch.flip(xs[0], dims=[0]).contiguous())  # second input buffer (same values, other order)
+    P = c.N * c.H * c.W
+    scratch_bytes = B.palquant_act_steps_scratch_bytes(P, c.G)
+    scratch = torch.empty(scratch_bytes, dtype=torch.uint8, device=dev)
+    s_a = B.palquant_act_steps(xs[0], c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, scratch, scratch_bytes)
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out,
+                     int(c.relu))
+    s_w = B.palquant_weight_steps(w_np, d)
+    inv_s = np.array([np.float32(1.0 / np.float64(v)) for v in s_a], dtype=np.float32)
+    inv_sw = np.array([np.float32(1.0 / np.float64(v)) for v in s_w], dtype=np.float32)
+    nbytes = B.palquant_packed_weight_bytes(d)
+    wp = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    B.palquant_pack_weights(w_np, d, inv_sw, wp, nbytes)
+    shuf = B.shuffle(c.shuffle_kind, c.shuffle_shift)
+    q = torch.empty((c.N, c.H, c.W, c.G * c.Cin_g), dtype=torch.uint8, device=dev)
+    out_shape = (c.N, c.Ho, c.Wo, c.G * c.Cout_g)
+    # next layer's steps: calibrated on this layer's rescaled output
+    m_out, _ = B.palquant_epilogue_scales(c.G, s_w, s_a, 1.0, None, shuf)
+    y = torch.empty(out_shape, dtype=torch.float32, device=dev)
+    B.palquant_quantize_act(xs[0], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s)
+    B.palquant_layer_fused(q, wp, d, m_out, m_out, shuf, None, None, y, None)
+    s_next = B.palquant_act_steps(y, c.N, c.Ho, c.Wo, c.G, c.Cout_g, c.bits_out, scratch, scratch_bytes)
+    m_out, m_req = B.palquant_epilogue_scales(c.G, s_w, s_a, 1.0, s_next, shuf)
+    del y
+    q_out = torch.empty(out_shape, dtype=torch.uint8, device=dev)
+    assert B.palquant_sync_check() == B.PQ_OK
+
+    def step(i, s):
+        B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, stream=s)
+        B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=s)
+
+    # ---- warm-up
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            step(i, stream)
+    torch.cuda.synchronize(dev)
+    st = B.palquant_sync_check(stream)
+    assert st == B.PQ_OK, B.strerror(st)
+
+    # ---- timed region: K steps, per-kernel events on the launching stream
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    sampler = ClockSampler(local_rank)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    sampler.start()
+    time.sleep(0.3)
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for i in range(K):
+            ev[i][0].record(stream)
+            B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, stream=stream)
+            ev[i][1].record(stream)
+            B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
+            ev[i][2].record(stream)
+        stop.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = sampler.stop()
+    if world > 1:
+        dist.barrier()
+    st = B.palquant_sync_check(stream)
+    assert st == B.PQ_OK, B.strerror(st)
+    elapsed_ms = start.elapsed_time(stop)
+    t_quant = sum(e[0].elapsed_time(e[1]) for e in ev) / K
+    t_conv = sum(e[1].elapsed_time(e[2]) for e in ev) / K
+    if world > 1:
+        t = torch.tensor([elapsed_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+    ms_per_step = elapsed_ms / K
+    ops_step = c.int_ops
+    value = ops_step * world / (ms_per_step / 1e3) / 1e12
+
+    # ---- end to end through the public API with host buffers (pinned), per step:
+    # H2D input copy, quantize, fused layer, D2H of the output codes.
+    x_host = torch.from_numpy(x_np).pin_memory()
+    out_host = torch.empty(out_shape, dtype=torch.uint8).pin_memory()
+    x_dev = xs[0]
+    E = max(3, min(K, 50))
+    with torch.cuda.stream(stream):
+        for _ in range(2):
+            x_dev.copy_(x_host, non_blocking=True)
+            step(0, stream)
+            out_host.copy_(q_out, non_blocking=True)
+    torch.cuda.synchronize(dev)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(E):
+            x_dev.copy_(x_host, non_blocking=True)
+            step(0, stream)
+            out_host.copy_(q_out, non_blocking=True)
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    e2e_ms = e0.elapsed_time(e1) / E
+    e2e_value = ops_step * world / (e2e_ms / 1e3) / 1e12
+
+    if rank != 0:
+        return
+    pk = peaks()
+    fp8_peak = 2.0 * pk["bf16_tflops"]  # dense FP8 = 2x dense BF16 (nominal ratio 4.5 / 2.25)
+    q_bytes = c.in_elems * 5  # 4-byte read + 1-byte write per element
+    conv_bytes = c.in_elems + c.out_elems + c.weight_elems
+    quant_gbs = q_bytes / (t_quant / 1e3) / 1e9
+    conv_tops = ops_step / (t_conv / 1e3) / 1e12
+    roof_quant = {"kernel": "pq_quantize_vec16", "bound": "hbm", "achieved": quant_gbs, "peak": pk["hbm_gbs"],
+                  "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"], "traffic": dram_traffic("pq_quantize_vec16"),
+                  "algorithmic_bytes": q_bytes, "avg_launch_ms": t_quant,
+                  "peak_source": f"{pk['source']} HBM copy bandwidth"}
+    roof_conv = {"kernel": "pq_conv_tc_kernel", "bound": "tensor", "achieved": conv_tops, "peak": fp8_peak,
+                 "unit": "TFLOP/s", "frac": conv_tops / fp8_peak, "traffic": dram_traffic("pq_conv_tc_kernel"),
+                 "algorithmic_ops": ops_step, "algorithmic_bytes": conv_bytes, "avg_launch_ms": t_conv,
+                 "hbm_frac": conv_bytes / (t_conv / 1e3) / 1e9 / pk["hbm_gbs"],
+                 "peak_source": f"{pk['source']} bf16 burst x 2 (dense FP8 E4M3, the exact-integer tensor path)"}
+    dominant = roof_quant if t_quant >= t_conv else roof_conv
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
+        "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "u8 codes, e4m3 x e4m3 -> f32 (exact integer)", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "global_batch": c.N * world, "per_gpu_batch": c.N,
+                   "timed": "quantize (fp32 NHWC -> codes) + fused layer (codes -> next-layer codes)",
+                   "l2": "inputs larger than L2 (205.5 MB fp32, two buffers used in turn)",
+                   "parallelism": f"replicas x{world}"},
+        "images_per_s": c.N * world / (ms_per_step / 1e3),
+        "pct_dense_int8_peak": 100.0 * value / world / fp8_peak,
+        "roofline": dominant,
+        "roofline_kernels": [roof_quant, roof_conv],
+        "clocks": clocks,
+        "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(x_np.nbytes),
+                "d2h_bytes_per_step": int(np.prod(out_shape))},
+        "gpu_launches": 2 * K,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(c, x_np, w_np, args.cpu_seconds)
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    args = parse()
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+        return
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl")
+    run_ours(args, rank, world, local_rank)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

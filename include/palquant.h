@@ -1,0 +1,255 @@
+/*
+ * palquant.h -- C ABI of the GB300 (sm_103a) PalQuant layer library, libpalquant.so.
+ *
+ * PalQuant (Hu et al., "PalQuant: Accelerating High-precision Networks on
+ * Low-precision Accelerators", arXiv 2208.01944) expands a convolution's channels
+ * G times, splits them into G groups, quantises every group's activations and
+ * weights to B bits and runs a B-bit group convolution (Sec. 4.1).  A cyclic
+ * permutation pi(g) = (g + 1) mod G moves each group's output to the next group
+ * (Sec. 4.2, Eq. 6-8).  This library runs the inference hot path of one such
+ * layer on one GPU:
+ *
+ *   palquant_quantize_act   activations -> per-group B-bit codes     (Eq. 2)
+ *   palquant_group_conv     codes (x) weight codes -> int32 sums      (Sec. 4.1)
+ *   palquant_layer_fused    group conv + rescale + shortcut + ReLU + output
+ *                           permutation + requantisation, one kernel  (Sec. 3.2,
+ *                                                                      4.1, 4.2)
+ * plus the set-up calls that produce its inputs (step initialisation, weight
+ * quantisation and packing).
+ *
+ * Conventions that hold for every call:
+ *  - Layouts.  Activations, codes and outputs are NHWC, channel c = g*C_g + j
+ *    (Sec. 4.2 views [N, C, H, W] as [N, G, C/G, H, W]).  Float weights are
+ *    [G][Cout_g][kh][kw][Cin_g].
+ *  - Codes.  One code per byte.  Activation codes are unsigned integers in
+ *    [0, 2^bits - 1]; weight codes are signed in [-2^(bits-1), 2^(bits-1) - 1].
+ *    A code tensor is stored either as plain integers (PQ_CODES_INT8) or as the
+ *    FP8 E4M3 encoding of the same integer (PQ_CODES_E4M3), which the tensor
+ *    cores read directly; both encodings represent every code exactly.
+ *  - Memory.  The caller owns every buffer.  Pointers named *_dev are device
+ *    pointers, *_host are host pointers.  The compute calls allocate nothing;
+ *    small host arrays (per-group scalars, permutations) are copied into the
+ *    launch at call time and may be freed on return.
+ *  - Streams.  pq_stream_t is a cudaStream_t (NULL = legacy default stream).
+ *    Compute calls are asynchronous on that stream.
+ *  - Errors.  Invalid arguments return PQ_EINVAL before anything is launched;
+ *    shapes the fast path does not cover return PQ_EUNSUPPORTED; CUDA launch or
+ *    runtime failures return PQ_ECUDA.  Every wait inside a kernel is bounded:
+ *    a wait that runs out records PQ_ETIMEOUT in a device error word, the kernel
+ *    returns, and palquant_sync_check() reports it.
+ *  - Devices.  Kernels are built for sm_103a (GB300) only.  Calls act on the
+ *    current CUDA device.
+ */
+#ifndef PALQUANT_H
+#define PALQUANT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef void* pq_stream_t; /* a cudaStream_t */
+
+typedef enum {
+    PQ_OK = 0,
+    PQ_EINVAL = -1,        /* bad argument; nothing launched */
+    PQ_EUNSUPPORTED = -2,  /* valid but outside the implemented shapes */
+    PQ_ECUDA = -3,         /* a CUDA call failed */
+    PQ_ETIMEOUT = -4       /* a bounded in-kernel wait ran out */
+} pq_status;
+
+typedef enum {
+    PQ_CODES_INT8 = 0, /* code v stored as the byte v (two's complement for weights) */
+    PQ_CODES_E4M3 = 1  /* code v stored as the FP8 E4M3 encoding of v */
+} pq_code_format;
+
+/* Output channel permutation (Sec. 4.2).  kind:
+ *   0  none
+ *   1  cyclic: source group g goes to group (g + shift) mod G; Eq. 6 is shift = 1
+ *   2  channel shuffle (ShuffleNet, used at block ends in Sec. 4.3): source channel
+ *      g*Cout_g + j goes to channel j*G + g
+ *   3  explicit group permutation: group g goes to group perm[g] (host array of G)
+ * Kinds 0, 1 and 3 must describe a permutation of the G groups, else PQ_EINVAL. */
+typedef struct {
+    int32_t kind;
+    int32_t shift;
+    const int32_t* perm;
+} pq_shuffle;
+
+/* One PalQuant layer.  Input [N, H, W, G*Cin_g] codes, weights
+ * [G][Cout_g][kh][kw][Cin_g], output [N, Ho, Wo, G*Cout_g] with
+ * Ho = (H + 2 pad - kh) / stride + 1 and Wo likewise.  Zero padding is code 0
+ * (exact because the activation quantiser's lower bound l is 0, Eq. 2). */
+typedef struct {
+    int32_t N, H, W;
+    int32_t G;
+    int32_t Cin_g, Cout_g;
+    int32_t kh, kw;
+    int32_t stride, pad;
+    int32_t bits_a;      /* activation code bits, 1..4 */
+    int32_t bits_w;      /* weight code bits, 2..4 */
+    int32_t bits_out;    /* requantised output code bits, 1..4 */
+    int32_t relu;        /* 1: ReLU after the rescale (and the shortcut add) */
+    int32_t code_format; /* pq_code_format of input codes and output codes */
+} pq_layer_desc;
+
+/* Human-readable name of a status. */
+const char* palquant_strerror(pq_status s);
+
+/* Library version, major*10000 + minor*100 + patch. */
+int palquant_version(void);
+
+/* ------------------------------------------------------------------------ */
+/* Set-up: step initialisation and epilogue multipliers (untimed).          */
+/* ------------------------------------------------------------------------ */
+
+/* Bytes of device scratch palquant_act_steps needs for a tensor of P = N*H*W
+ * pixels and G groups. */
+size_t palquant_act_steps_scratch_bytes(int64_t P, int32_t G);
+
+/* Per-group activation step s[g] = 2 mean(x_g) / sqrt(2^bits - 1): the LSQ step
+ * initialisation the paper's training follows (Sec. 5, "Training Details";
+ * Eq. 2 with l = 0, u = s (2^bits - 1)).  x_dev is NHWC fp32 [N,H,W,G*Cg]; the
+ * mean runs over every element of the group, summed in double in a fixed order
+ * (deterministic), and the step is rounded to float once.  scratch_dev must hold
+ * palquant_act_steps_scratch_bytes(N*H*W, G) bytes.  s_out_host receives G
+ * floats.  Synchronises the stream. */
+pq_status palquant_act_steps(const float* x_dev, int64_t N, int32_t H, int32_t W, int32_t G, int32_t Cg,
+                             int32_t bits, void* scratch_dev, size_t scratch_bytes, float* s_out_host,
+                             pq_stream_t stream);
+
+/* Per-group weight step s_w[g] = 2 mean|w_g| / sqrt(2^(bits-1) - 1) (LSQ), mean
+ * in double over the group's weights; w_host is [G][Cout_g][kh][kw][Cin_g].
+ * Host only.  s_w_out_host receives G floats. */
+pq_status palquant_weight_steps(const float* w_host, const pq_layer_desc* d, float* s_w_out_host);
+
+/* Epilogue multipliers (Sec. 3.2: the output scale alpha multiplies the layer's
+ * output; the requantised code of source group g lands in group dst(g) of the
+ * next layer and uses that group's step):
+ *   m_out[g] = fl(s_w[g] s_a[g] alpha)
+ *   m_req[g] = fl(s_w[g] s_a[g] alpha / s_next[dst(g)])       (s_next may be NULL)
+ * computed in double and rounded once.  Host only. */
+pq_status palquant_epilogue_scales(int32_t G, const float* s_w_host, const float* s_a_host, double alpha,
+                                   const float* s_next_host, pq_shuffle shuf, float* m_out_host,
+                                   float* m_req_host);
+
+/* ------------------------------------------------------------------------ */
+/* Set-up: weight quantisation and packing (untimed).                       */
+/* ------------------------------------------------------------------------ */
+
+/* Size of the packed weight operand of a layer (opaque, tensor-core layout). */
+size_t palquant_packed_weight_bytes(const pq_layer_desc* d);
+
+/* Quantise float weights to signed codes per group,
+ *   w_q = clamp(rint(w * inv_sw[g]), -2^(bits_w-1), 2^(bits_w-1) - 1)
+ * (one fp32 multiply, round half to even; Eq. 2 in LSQ's signed form), and
+ * write the packed operand to packed_host (palquant_packed_weight_bytes bytes).
+ * Host only. */
+pq_status palquant_pack_weights_host(const float* w_host, const pq_layer_desc* d, const float* inv_sw_host,
+                                     void* packed_host, size_t packed_bytes);
+
+/* The same, with the packed operand copied to device memory on `stream`
+ * (synchronises the stream before returning so w_host may be freed). */
+pq_status palquant_pack_weights(const float* w_host, const pq_layer_desc* d, const float* inv_sw_host,
+                                void* packed_dev, size_t packed_bytes, pq_stream_t stream);
+
+/* Pack already-quantised signed weight codes wq_host [G][Cout_g][kh][kw][Cin_g]
+ * (each in the bits_w range, else PQ_EINVAL).  Host only. */
+pq_status palquant_pack_weight_codes_host(const int8_t* wq_host, const pq_layer_desc* d, void* packed_host,
+                                          size_t packed_bytes);
+
+/* Inverse of the packing: recover the signed codes from a packed operand. */
+pq_status palquant_unpack_weight_codes_host(const void* packed_host, const pq_layer_desc* d, int8_t* wq_host);
+
+/* ------------------------------------------------------------------------ */
+/* Hot path.                                                                */
+/* ------------------------------------------------------------------------ */
+
+/* Group-wise activation quantisation (Eq. 2 with l = 0, u = s (2^bits - 1); one
+ * fp32 multiply, round half to even, clamp):
+ *   q[p, g*Cg + j] = clamp(rint(x[p, g*Cg + j] * inv_s[g]), 0, 2^bits - 1)
+ * x_dev is NHWC fp32 [N,H,W,G*Cg]; q_dev receives one byte per element in
+ * code_format.  inv_s_host holds G floats (fl(1/s) of the steps), copied at call
+ * time.  NaN maps to 0 and +inf to 2^bits - 1.  bits in 1..8 for PQ_CODES_INT8,
+ * 1..4 for PQ_CODES_E4M3. */
+pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G,
+                                int32_t Cg, int32_t bits, int32_t code_format, const float* inv_s_host,
+                                pq_stream_t stream);
+
+/* B-bit group convolution (Sec. 3.1 Eq. 1 lowered per group; Sec. 4.1):
+ *   acc[n,oh,ow,g*Cout_g+co] = sum_{kh,kw,ci} q[n, oh*s-p+kh, ow*s-p+kw, g*Cin_g+ci]
+ *                                             * w_q[g,co,kh,kw,ci]
+ * exact in int32 (every product and partial sum is an integer below 2^24).
+ * q_dev holds codes in d->code_format; w_packed_dev comes from
+ * palquant_pack_weights for the same d; acc_dev is int32 NHWC.  No permutation. */
+pq_status palquant_group_conv(const void* q_dev, const void* w_packed_dev, int32_t* acc_dev,
+                              const pq_layer_desc* d, pq_stream_t stream);
+
+/* The whole layer in one kernel (Sec. 3.2, 4.1, 4.2).  For every output pixel
+ * and source channel (g, co) with acc the group-conv sum above:
+ *   y = (float)acc * m_out[g]
+ *   y = y + shortcut[pixel, g*Cout_g + co]        if shortcut_dev != NULL
+ *   y = max(y, 0)                                  if d->relu
+ *   t = shortcut_dev ? y : (float)acc
+ *   q = clamp(rint(t * m_req[g]), 0, 2^bits_out - 1)
+ * and acc, y, q are written at the destination channel of (g, co) under shuf.
+ * m_out_host, m_req_host: G floats each (m_req may be NULL only when
+ * q_out_dev is NULL).  Any of acc_out_dev (int32), y_out_dev (fp32) and
+ * q_out_dev (codes in d->code_format) may be NULL, but not all three.
+ * shortcut_dev is fp32 NHWC with the output's shape.  Float products and sums
+ * are single IEEE fp32 operations in the order written. */
+pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
+                               const float* m_out_host, const float* m_req_host, pq_shuffle shuf,
+                               const float* shortcut_dev, int32_t* acc_out_dev, float* y_out_dev,
+                               void* q_out_dev, pq_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Failure detection.                                                       */
+/* ------------------------------------------------------------------------ */
+
+/* Synchronise `stream`, then read and clear the device error word of the
+ * current device.  Returns PQ_ETIMEOUT if any kernel's bounded wait ran out
+ * since the last check, PQ_ECUDA on a CUDA error, else PQ_OK. */
+pq_status palquant_sync_check(pq_stream_t stream);
+
+/* Limit, in nanoseconds, of every in-kernel wait of kernels launched after this
+ * call (default 2e9).  0 restores the default. */
+pq_status palquant_set_wait_limit_ns(uint64_t ns);
+
+/* Launch a one-CTA kernel whose barrier wait nobody completes, with the given
+ * wait limit, and return palquant_sync_check()'s verdict (PQ_ETIMEOUT when the
+ * watchdog works).  The kernel ends by itself; the context stays usable. */
+pq_status palquant_watchdog_selftest(uint64_t limit_ns, pq_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
+/* Introspection (host only; no GPU needed).                                */
+/* ------------------------------------------------------------------------ */
+
+/* How the tensor-core kernel tiles a layer.  Filled by palquant_conv_plan. */
+typedef struct {
+    int32_t supported;     /* 1 if the tensor-core kernel runs this layer */
+    int32_t mode;          /* 0 flat pixels (1x1, stride 1, pad 0), 1 rows of whole image rows */
+    int32_t rows_per_tile; /* output rows per tile (mode 1) */
+    int32_t m_tiles;       /* 128-row accumulators per tile */
+    int32_t tile_pitch;    /* positions per tile row in shared memory */
+    int32_t n_block;       /* output channels per accumulator (MMA N) */
+    int32_t n_blocks;      /* output-channel blocks per group */
+    int32_t k_chunk;       /* input channels per K block */
+    int32_t k_blocks;      /* K blocks per tap */
+    int32_t taps;          /* kh*kw */
+    int32_t weights_resident; /* 1 if a group's weights stay in shared memory */
+    int32_t acc_stages;    /* tensor-memory accumulator buffers */
+    int32_t smem_bytes;    /* dynamic shared memory per CTA */
+    int64_t tiles;         /* tiles per (group, n-block) unit */
+    int64_t work_items;    /* tiles * G * n_blocks */
+} pq_conv_plan;
+
+pq_status palquant_conv_plan(const pq_layer_desc* d, pq_conv_plan* plan);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* PALQUANT_H */

@@ -1,0 +1,682 @@
+// Host side of libpalquant.so: argument validation, the tiling planner of the
+// tensor-core convolution, weight quantisation and packing, tensor-map encoding,
+// launches and error reporting.  Every entry point of include/palquant.h is
+// defined here.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <atomic>
+#include <cmath>
+#include <cstdint>
+#include <cstring>
+#include <mutex>
+#include <vector>
+
+#include "../../include/palquant.h"
+#include "pq_internal.h"
+
+using pq::ConvParams;
+using pq::TensorMaps;
+
+namespace {
+
+constexpr uint64_t kDefaultWaitLimitNs = 2000000000ull;
+std::atomic<uint64_t> g_wait_limit_ns{kDefaultWaitLimitNs};
+
+constexpr int kActSumBlocks = 256;
+
+int64_t out_dim(int64_t in, int k, int s, int p) { return (in + 2 * p - k) / s + 1; }
+
+int floor_div(int a, int b) { return (a >= 0) ? a / b : -((-a + b - 1) / b); }
+
+int pos_mod(int a, int b) { return ((a % b) + b) % b; }
+
+uint32_t round_up(uint64_t v, uint64_t a) { return static_cast<uint32_t>((v + a - 1) / a * a); }
+
+int next_pow2(int v) {
+  int p = 1;
+  while (p < v) p <<= 1;
+  return p;
+}
+
+// FP8 E4M3 encoding (1 sign bit, 4 exponent bits with bias 7, 3 mantissa bits)
+// of an integer |v| <= 15: |v| in [2^e, 2^(e+1)) has exponent field e + 7 and
+// mantissa (|v| / 2^e - 1) * 8, exact for |v| < 16.
+uint8_t e4m3_of_int(int v) {
+  if (v == 0) return 0;
+  const uint8_t sign = v < 0 ? 0x80 : 0x00;
+  const int a = v < 0 ? -v : v;
+  int e = 0;
+  while ((2 << e) <= a) ++e;
+  const int mant = ((a << 3) >> e) & 7;
+  return static_cast<uint8_t>(sign | ((e + 7) << 3) | mant);
+}
+
+// Inverse of e4m3_of_int for bytes it produces (normal numbers >= 1 in magnitude).
+int int_of_e4m3(uint8_t b) {
+  if ((b & 0x7F) == 0) return 0;
+  const int e = ((b >> 3) & 15) - 7;
+  const int mant = b & 7;
+  const int a = ((8 + mant) << e) >> 3;
+  return (b & 0x80) ? -a : a;
+}
+
+bool valid_shuffle(int G, const pq_shuffle& s, int* dst_group) {
+  if (s.kind == 0 || s.kind == 2) {
+    for (int g = 0; g < G; ++g) dst_group[g] = g;
+  } else if (s.kind == 1) {
+    for (int g = 0; g < G; ++g) dst_group[g] = pos_mod(g + s.shift, G);
+  } else if (s.kind == 3) {
+    if (s.perm == nullptr) return false;
+    for (int g = 0; g < G; ++g) dst_group[g] = s.perm[g];
+  } else {
+    return false;
+  }
+  std::vector<int> seen(G, 0);
+  for (int g = 0; g < G; ++g) {
+    if (dst_group[g] < 0 || dst_group[g] >= G || seen[dst_group[g]]) return false;
+    seen[dst_group[g]] = 1;
+  }
+  return true;
+}
+
+pq_status validate_desc(const pq_layer_desc* d) {
+  if (d == nullptr) return PQ_EINVAL;
+  if (d->N < 0 || d->H < 1 || d->W < 1 || d->G < 1 || d->Cin_g < 1 || d->Cout_g < 1) return PQ_EINVAL;
+  if (d->kh < 1 || d->kw < 1 || d->stride < 1 || d->pad < 0) return PQ_EINVAL;
+  if (d->bits_a < 1 || d->bits_a > 8 || d->bits_w < 2 || d->bits_w > 8 || d->bits_out < 1 || d->bits_out > 8)
+    return PQ_EINVAL;
+  if (d->relu != 0 && d->relu != 1) return PQ_EINVAL;
+  if (d->code_format != PQ_CODES_INT8 && d->code_format != PQ_CODES_E4M3) return PQ_EINVAL;
+  if (out_dim(d->H, d->kh, d->stride, d->pad) < 1 || out_dim(d->W, d->kw, d->stride, d->pad) < 1) return PQ_EINVAL;
+  if (d->G > pq::kMaxG) return PQ_EUNSUPPORTED;
+  return PQ_OK;
+}
+
+int device_sm_count() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return 0;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return 0;
+  return sms;
+}
+
+// ---------------------------------------------------------------------------
+// Planner: how the tensor-core kernel tiles a layer.  Pure host arithmetic.
+// ---------------------------------------------------------------------------
+struct Phase {
+  int a, b;
+};
+
+pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, std::vector<Phase>* phases_out) {
+  pq_status st = validate_desc(d);
+  if (st != PQ_OK) return st;
+  pq_conv_plan plan;
+  std::memset(&plan, 0, sizeof(plan));
+  ConvParams p;
+  std::memset(&p, 0, sizeof(p));
+  const int Ho = static_cast<int>(out_dim(d->H, d->kh, d->stride, d->pad));
+  const int Wo = static_cast<int>(out_dim(d->W, d->kw, d->stride, d->pad));
+  const int taps = d->kh * d->kw;
+  const int qa = (1 << d->bits_a) - 1;
+  const int qw = 1 << (d->bits_w - 1);
+  // Coverage of the tensor-core kernel.
+  bool ok = d->code_format == PQ_CODES_INT8 && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
+            d->pad < std::max(d->kh, d->kw) && d->Cin_g % 32 == 0 && d->Cout_g % 16 == 0 && taps <= pq::kMaxTaps &&
+            static_cast<int64_t>(taps) * d->Cin_g * qa * qw < (1LL << 24);
+  if (!ok) {
+    if (pub) *pub = plan;
+    return PQ_EUNSUPPORTED;
+  }
+  p.N = d->N;
+  p.Ho = Ho;
+  p.Wo = Wo;
+  p.P_out = static_cast<int64_t>(d->N) * Ho * Wo;
+  p.G = d->G;
+  p.Cin_g = d->Cin_g;
+  p.Cout_g = d->Cout_g;
+  p.taps = taps;
+  // Output-channel blocks: N of one MMA is at most 256 and a multiple of 16.
+  int NB = (d->Cout_g + 255) / 256;
+  while (d->Cout_g % NB != 0 || (d->Cout_g / NB) % 16 != 0) ++NB;
+  p.NB = NB;
+  p.Nblk = d->Cout_g / NB;
+  p.Npow2 = next_pow2(p.Nblk);
+  const bool flat = d->kh == 1 && d->kw == 1 && d->stride == 1 && d->pad == 0;
+  p.mode = flat ? pq::kModeFlat : pq::kModeRows;
+  const int s = d->stride;
+  // Rows-mode geometry in phase coordinates.
+  const int rmin = floor_div(-d->pad, s), rmax = floor_div(d->kh - 1 - d->pad, s);
+  const int cmin = floor_div(-d->pad, s), cmax = floor_div(d->kw - 1 - d->pad, s);
+  const int Wh = flat ? 0 : Wo + cmax - cmin;
+  // Stride phases used by the taps, and each tap's (phase, offset).
+  std::vector<Phase> phases;
+  int off_max = 0;
+  if (!flat) {
+    for (int i = 0; i < d->kh; ++i) {
+      for (int j = 0; j < d->kw; ++j) {
+        const int a = pos_mod(i - d->pad, s), b = pos_mod(j - d->pad, s);
+        int idx = -1;
+        for (size_t q = 0; q < phases.size(); ++q)
+          if (phases[q].a == a && phases[q].b == b) idx = static_cast<int>(q);
+        if (idx < 0) {
+          phases.push_back({a, b});
+          idx = static_cast<int>(phases.size()) - 1;
+        }
+        const int t = i * d->kw + j;
+        p.tap_phase[t] = idx;
+        p.tap_off[t] = (floor_div(i - d->pad, s) - rmin) * Wh + (floor_div(j - d->pad, s) - cmin);
+        off_max = std::max(off_max, p.tap_off[t]);
+      }
+    }
+  } else {
+    phases.push_back({0, 0});
+    p.tap_phase[0] = 0;
+    p.tap_off[0] = 0;
+  }
+  p.nph = static_cast<int>(phases.size());
+  // Tile shape: MT accumulators of 128 rows; rows mode packs Ht whole output
+  // rows of pitch Wh into them.
+  int best_mt = 0, best_ht = 0, best_tpi = 0, best_acc = 0;
+  double best_eff = -1.0, best_halo = 1e30;
+  for (int MT : {1, 2, 4}) {
+    if (flat && MT > 2) continue;
+    int acc_stages = (2 * MT * p.Npow2 <= 512) ? 2 : ((MT * p.Npow2 <= 512) ? 1 : 0);
+    if (acc_stages == 0) continue;
+    double eff, halo;
+    int ht = 0, tpi = 0;
+    if (flat) {
+      const int64_t tiles = (p.P_out + MT * 128 - 1) / (MT * 128);
+      eff = tiles > 0 ? static_cast<double>(p.P_out) / (tiles * MT * 128.0) : 1.0;
+      halo = 1.0;
+    } else {
+      const int ht_max = (MT * 128) / Wh;
+      if (ht_max < 1) continue;
+      tpi = (Ho + ht_max - 1) / ht_max;
+      ht = (Ho + tpi - 1) / tpi;
+      eff = static_cast<double>(Ho) * Wo / (static_cast<double>(tpi) * MT * 128.0);
+      halo = static_cast<double>(ht + rmax - rmin) / ht;
+    }
+    // Prefer double-buffered accumulators, then tile efficiency, then less halo.
+    const double score_eff = eff + (acc_stages == 2 ? 1.0 : 0.0);
+    const bool better = score_eff > best_eff + 0.02 || (std::fabs(score_eff - best_eff) <= 0.02 && halo < best_halo - 1e-9);
+    if (best_mt == 0 || better) {
+      best_mt = MT;
+      best_ht = ht;
+      best_tpi = tpi;
+      best_acc = acc_stages;
+      best_eff = score_eff;
+      best_halo = halo;
+    }
+  }
+  if (best_mt == 0) {
+    if (pub) *pub = plan;
+    return PQ_EUNSUPPORTED;
+  }
+  p.MT = best_mt;
+  p.acc_stages = best_acc;
+  if (flat) {
+    p.flat_box = p.MT * 128;
+    p.tiles = (p.P_out + p.flat_box - 1) / p.flat_box;
+    p.Ht = 0;
+    p.Wh = 0;
+    p.Hd = 0;
+    p.Wd = 0;
+  } else {
+    p.Ht = best_ht;
+    p.tiles_per_img = best_tpi;
+    p.tiles = static_cast<int64_t>(d->N) * best_tpi;
+    p.Wh = Wh;
+    p.Wd = Wh;
+    p.Hd = p.Ht + rmax - rmin;
+    p.h_off = rmin;
+    p.w_coord = cmin;
+    if (p.Wd > 256 || p.Hd > 256) {
+      if (pub) *pub = plan;
+      return PQ_EUNSUPPORTED;
+    }
+  }
+  p.items = p.tiles * d->G * NB;
+  // K blocks, weights residency and pipeline depth under the shared-memory budget.
+  const uint32_t budget = pq::kMaxSmem - 1024;
+  auto a_stage_bytes = [&](int KC, uint32_t* phase_bytes, uint32_t* tx, uint32_t* lbo) -> uint32_t {
+    const int nch = KC / 16;
+    if (flat) {
+      const uint32_t plane = static_cast<uint32_t>(p.flat_box) * 16u;
+      *phase_bytes = round_up(static_cast<uint64_t>(nch) * plane, 128);
+      *tx = nch * plane;
+      *lbo = plane;
+      return round_up(*phase_bytes, 1024);
+    }
+    const uint32_t plane = static_cast<uint32_t>(p.Hd) * p.Wd * 16u;
+    *phase_bytes = round_up(static_cast<uint64_t>(nch) * plane, 128);
+    *tx = static_cast<uint32_t>(p.nph) * nch * plane;
+    *lbo = plane;
+    const uint64_t overrun = static_cast<uint64_t>(p.nph - 1) * (*phase_bytes) + static_cast<uint64_t>(nch - 1) * plane +
+                             16ull * (p.MT * 128 + off_max);
+    return round_up(std::max<uint64_t>(static_cast<uint64_t>(p.nph) * (*phase_bytes), overrun), 1024);
+  };
+  // Epilogue staging per warp: 32 rows of up to 64 code bytes and 32 rows of 16
+  // fp32/int32 values, row pitch 80 bytes (an odd number of 16-byte bank groups).
+  const uint32_t q_pitch = 80;
+  const uint32_t f_pitch = 80;
+  const uint32_t warp_stage = round_up(32u * (q_pitch + f_pitch), 128);
+  const uint32_t stage_total = warp_stage * pq::kEpiWarps;
+  const uint32_t bar_bytes = 1024;  // barriers, abort flag, TMEM slot (generous)
+  const uint64_t unit_bytes = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk;
+  // Largest K block (input channels per pipeline stage) that fits: the whole
+  // unit's weights resident if they fit, else a ring of (K block, tap) slices.
+  bool found = false, resident = false;
+  int KC = d->Cin_g, a_stages = 0, b_stages = 0;
+  uint32_t stage_bytes = 0, phase_bytes = 0, tx = 0, lbo = 0;
+  for (int kc = d->Cin_g; kc >= 32 && !found; kc /= 2) {
+    if (d->Cin_g % kc != 0 || kc % 32 != 0) continue;
+    uint32_t sb, pb, t, l;
+    sb = a_stage_bytes(kc, &pb, &t, &l);
+    if (sb > 64u * 1024u) continue;
+    for (int res = 1; res >= 0 && !found; --res) {
+      if (res && unit_bytes > 112u * 1024u) continue;
+      const uint64_t slice = static_cast<uint64_t>(kc) * p.Nblk;
+      if (!res && slice > 32u * 1024u) continue;
+      for (int na = 4; na >= 2 && !found; --na) {
+        for (int nb = (res ? 1 : 4); nb >= (res ? 1 : 2) && !found; --nb) {
+          const uint64_t bb = res ? round_up(unit_bytes, 1024) : round_up(nb * slice, 1024);
+          if (bb + stage_total + bar_bytes + static_cast<uint64_t>(na) * sb <= budget) {
+            found = true;
+            resident = res != 0;
+            KC = kc;
+            a_stages = na;
+            b_stages = nb;
+            stage_bytes = sb;
+            phase_bytes = pb;
+            tx = t;
+            lbo = l;
+          }
+        }
+      }
+    }
+  }
+  if (!found) {
+    if (pub) *pub = plan;
+    return PQ_EUNSUPPORTED;
+  }
+  const uint32_t b_bytes = resident ? round_up(unit_bytes, 1024) : round_up(static_cast<uint64_t>(b_stages) * KC * p.Nblk, 1024);
+  p.KC = KC;
+  p.nch = KC / 16;
+  p.n_kb = d->Cin_g / KC;
+  p.lbo_a = lbo;
+  p.a_phase_bytes = phase_bytes;
+  p.a_stage_bytes = stage_bytes;
+  p.a_tx_bytes = tx;
+  p.a_stages = a_stages;
+  p.b_resident = resident ? 1 : 0;
+  p.b_slice_bytes = static_cast<uint32_t>(KC) * p.Nblk;
+  p.b_unit_bytes = static_cast<uint32_t>(unit_bytes);
+  p.lbo_b = static_cast<uint32_t>(p.Nblk) * 16u;
+  p.b_stages = resident ? 1 : b_stages;
+  p.tmem_cols = static_cast<uint32_t>(next_pow2(std::max(32, p.acc_stages * p.MT * p.Npow2)));
+  p.smem_b_off = static_cast<uint32_t>(a_stages) * stage_bytes;
+  p.smem_stage_off = p.smem_b_off + b_bytes;
+  p.smem_bar_off = p.smem_stage_off + stage_total;
+  p.smem_bytes = p.smem_bar_off + bar_bytes;
+  p.stage_q_pitch = q_pitch;
+  p.stage_f_pitch = f_pitch;
+  p.stage_warp_bytes = warp_stage;
+  p.C_out_total = d->G * d->Cout_g;
+  p.relu = d->relu;
+  p.qmax_out = (1 << d->bits_out) - 1;
+  for (int g = 0; g < d->G; ++g) p.dst_group[g] = g;
+
+  plan.supported = 1;
+  plan.mode = p.mode;
+  plan.rows_per_tile = p.Ht;
+  plan.m_tiles = p.MT;
+  plan.tile_pitch = p.Wh;
+  plan.n_block = p.Nblk;
+  plan.n_blocks = p.NB;
+  plan.k_chunk = p.KC;
+  plan.k_blocks = p.n_kb;
+  plan.taps = taps;
+  plan.weights_resident = p.b_resident;
+  plan.acc_stages = p.acc_stages;
+  plan.smem_bytes = static_cast<int32_t>(p.smem_bytes);
+  plan.tiles = p.tiles;
+  plan.work_items = p.items;
+  if (pub) *pub = plan;
+  if (P) *P = p;
+  if (phases_out) *phases_out = phases;
+  return PQ_OK;
+}
+
+// ---------------------------------------------------------------------------
+// Tensor maps.
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static std::once_flag once;
+  static EncodeTiledFn fn = nullptr;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult qres;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &qres) ==
+            cudaSuccess &&
+        qres == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+bool encode_activation_maps(const pq_layer_desc* d, const ConvParams& p, const std::vector<Phase>& phases,
+                            const void* q_dev, TensorMaps* tm) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return false;
+  std::memset(tm, 0, sizeof(*tm));
+  const uint64_t C = static_cast<uint64_t>(d->G) * d->Cin_g;
+  const uint8_t* base = static_cast<const uint8_t*>(q_dev);
+  if (p.mode == pq::kModeFlat) {
+    const uint64_t P = static_cast<uint64_t>(d->N) * d->H * d->W;
+    cuuint64_t dims[3] = {16, P, C / 16};
+    cuuint64_t strides[2] = {C, 16};
+    cuuint32_t box[3] = {16, static_cast<cuuint32_t>(p.flat_box), static_cast<cuuint32_t>(p.nch)};
+    cuuint32_t es[3] = {1, 1, 1};
+    return enc(&tm->a[0], CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<uint8_t*>(base), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
+  const int s = d->stride;
+  for (size_t i = 0; i < phases.size(); ++i) {
+    const int a = phases[i].a, b = phases[i].b;
+    const uint64_t Wph = (d->W - b + s - 1) / s, Hph = (d->H - a + s - 1) / s;
+    if (Wph == 0 || Hph == 0) return false;
+    cuuint64_t dims[5] = {16, Wph, Hph, C / 16, static_cast<cuuint64_t>(d->N)};
+    cuuint64_t strides[4] = {s * C, s * static_cast<uint64_t>(d->W) * C, 16,
+                             static_cast<uint64_t>(d->H) * d->W * C};
+    cuuint32_t box[5] = {16, static_cast<cuuint32_t>(p.Wd), static_cast<cuuint32_t>(p.Hd),
+                         static_cast<cuuint32_t>(p.nch), 1};
+    cuuint32_t es[5] = {1, 1, 1, 1, 1};
+    const uint8_t* phase_base = base + (static_cast<uint64_t>(a) * d->W + b) * C;
+    if (enc(&tm->a[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 5, const_cast<uint8_t*>(phase_base), dims, strides, box, es,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+      return false;
+  }
+  return true;
+}
+
+bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
+// ---------------------------------------------------------------------------
+// Weight packing (tensor-core operand layout of the planner's tiling).
+//   unit u = g * NB + nb; for each K block kb, tap t, 16-channel chunk j,
+//   output channel c (of the block) and channel e of the chunk:
+//   byte[(((u * n_kb + kb) * taps + t) * nch + j) * Nblk * 16 + c * 16 + e]
+//     = E4M3(w_q[g, nb*Nblk + c, tap t, kb*KC + j*16 + e])
+// ---------------------------------------------------------------------------
+template <typename F>
+void for_each_packed(const ConvParams& p, int kw, F&& f) {
+  for (int g = 0; g < p.G; ++g)
+    for (int nb = 0; nb < p.NB; ++nb)
+      for (int kb = 0; kb < p.n_kb; ++kb)
+        for (int t = 0; t < p.taps; ++t)
+          for (int j = 0; j < p.nch; ++j)
+            for (int c = 0; c < p.Nblk; ++c)
+              for (int e = 0; e < 16; ++e) {
+                const int u = g * p.NB + nb;
+                const size_t dst = ((((static_cast<size_t>(u) * p.n_kb + kb) * p.taps + t) * p.nch + j) * p.Nblk + c) * 16 + e;
+                const int co = nb * p.Nblk + c;
+                const int ci = kb * p.KC + j * 16 + e;
+                const int i = t / kw, jj = t % kw;
+                const size_t src = (((static_cast<size_t>(g) * p.Cout_g + co) * (p.taps / kw) + i) * kw + jj) * p.Cin_g + ci;
+                f(dst, src);
+              }
+}
+
+}  // namespace
+
+// ===========================================================================
+// Public ABI
+// ===========================================================================
+extern "C" {
+
+const char* palquant_strerror(pq_status s) {
+  switch (s) {
+    case PQ_OK: return "ok";
+    case PQ_EINVAL: return "invalid argument";
+    case PQ_EUNSUPPORTED: return "unsupported layer shape or format";
+    case PQ_ECUDA: return "CUDA error";
+    case PQ_ETIMEOUT: return "in-kernel wait timed out";
+  }
+  return "unknown status";
+}
+
+int palquant_version(void) { return 100; }
+
+size_t palquant_act_steps_scratch_bytes(int64_t P, int32_t G) {
+  (void)P;
+  if (G < 1) return 0;
+  return sizeof(double) * (static_cast<size_t>(kActSumBlocks) * G + G);
+}
+
+pq_status palquant_act_steps(const float* x_dev, int64_t N, int32_t H, int32_t W, int32_t G, int32_t Cg, int32_t bits,
+                             void* scratch_dev, size_t scratch_bytes, float* s_out_host, pq_stream_t stream) {
+  if (x_dev == nullptr || scratch_dev == nullptr || s_out_host == nullptr) return PQ_EINVAL;
+  if (N < 1 || H < 1 || W < 1 || G < 1 || Cg < 1 || bits < 1 || bits > 8) return PQ_EINVAL;
+  const int64_t P = N * H * W;
+  if (scratch_bytes < palquant_act_steps_scratch_bytes(P, G) || (reinterpret_cast<uintptr_t>(scratch_dev) & 7u))
+    return PQ_EINVAL;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  double* partial = static_cast<double*>(scratch_dev);
+  double* sums = partial + static_cast<size_t>(kActSumBlocks) * G;
+  if (pq::launch_act_sum(x_dev, P, G, Cg, partial, kActSumBlocks, s) != 0) return PQ_ECUDA;
+  if (pq::launch_act_sum_finish(partial, kActSumBlocks, G, sums, s) != 0) return PQ_ECUDA;
+  std::vector<double> h(G);
+  if (cudaMemcpyAsync(h.data(), sums, sizeof(double) * G, cudaMemcpyDeviceToHost, s) != cudaSuccess) return PQ_ECUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return PQ_ECUDA;
+  const double qp = static_cast<double>((1 << bits) - 1);
+  for (int g = 0; g < G; ++g) {
+    const double mean = h[g] / static_cast<double>(P * Cg);
+    s_out_host[g] = static_cast<float>(2.0 * mean / std::sqrt(qp));
+  }
+  return PQ_OK;
+}
+
+pq_status palquant_weight_steps(const float* w_host, const pq_layer_desc* d, float* s_w_out_host) {
+  if (w_host == nullptr || s_w_out_host == nullptr) return PQ_EINVAL;
+  pq_status st = validate_desc(d);
+  if (st != PQ_OK) return st;
+  const int64_t per_group = static_cast<int64_t>(d->Cout_g) * d->kh * d->kw * d->Cin_g;
+  const double qp = static_cast<double>((1 << (d->bits_w - 1)) - 1);
+  for (int g = 0; g < d->G; ++g) {
+    double sum = 0.0;
+    for (int64_t i = 0; i < per_group; ++i) sum += std::fabs(static_cast<double>(w_host[g * per_group + i]));
+    s_w_out_host[g] = static_cast<float>(2.0 * (sum / static_cast<double>(per_group)) / std::sqrt(qp));
+  }
+  return PQ_OK;
+}
+
+pq_status palquant_epilogue_scales(int32_t G, const float* s_w_host, const float* s_a_host, double alpha,
+                                   const float* s_next_host, pq_shuffle shuf, float* m_out_host, float* m_req_host) {
+  if (G < 1 || G > pq::kMaxG || s_w_host == nullptr || s_a_host == nullptr || m_out_host == nullptr) return PQ_EINVAL;
+  if (s_next_host != nullptr && m_req_host == nullptr) return PQ_EINVAL;
+  int dst[pq::kMaxG];
+  if (!valid_shuffle(G, shuf, dst)) return PQ_EINVAL;
+  for (int g = 0; g < G; ++g) {
+    const double m = static_cast<double>(s_w_host[g]) * static_cast<double>(s_a_host[g]) * alpha;
+    m_out_host[g] = static_cast<float>(m);
+    if (s_next_host != nullptr) m_req_host[g] = static_cast<float>(m / static_cast<double>(s_next_host[dst[g]]));
+  }
+  return PQ_OK;
+}
+
+size_t palquant_packed_weight_bytes(const pq_layer_desc* d) {
+  ConvParams p;
+  if (plan_conv(d, &p, nullptr, nullptr) != PQ_OK) return 0;
+  return static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
+}
+
+pq_status palquant_pack_weight_codes_host(const int8_t* wq_host, const pq_layer_desc* d, void* packed_host,
+                                          size_t packed_bytes) {
+  if (wq_host == nullptr || packed_host == nullptr) return PQ_EINVAL;
+  ConvParams p;
+  pq_status st = plan_conv(d, &p, nullptr, nullptr);
+  if (st != PQ_OK) return st;
+  const size_t need = static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
+  if (packed_bytes < need) return PQ_EINVAL;
+  const int lo = -(1 << (d->bits_w - 1)), hi = (1 << (d->bits_w - 1)) - 1;
+  for (size_t i = 0; i < need; ++i)
+    if (wq_host[i] < lo || wq_host[i] > hi) return PQ_EINVAL;
+  uint8_t* out = static_cast<uint8_t*>(packed_host);
+  for_each_packed(p, d->kw, [&](size_t dst, size_t src) { out[dst] = e4m3_of_int(wq_host[src]); });
+  return PQ_OK;
+}
+
+pq_status palquant_unpack_weight_codes_host(const void* packed_host, const pq_layer_desc* d, int8_t* wq_host) {
+  if (packed_host == nullptr || wq_host == nullptr) return PQ_EINVAL;
+  ConvParams p;
+  pq_status st = plan_conv(d, &p, nullptr, nullptr);
+  if (st != PQ_OK) return st;
+  const uint8_t* in = static_cast<const uint8_t*>(packed_host);
+  for_each_packed(p, d->kw, [&](size_t dst, size_t src) { wq_host[src] = static_cast<int8_t>(int_of_e4m3(in[dst])); });
+  return PQ_OK;
+}
+
+pq_status palquant_pack_weights_host(const float* w_host, const pq_layer_desc* d, const float* inv_sw_host,
+                                     void* packed_host, size_t packed_bytes) {
+  if (w_host == nullptr || inv_sw_host == nullptr || packed_host == nullptr) return PQ_EINVAL;
+  pq_status st = validate_desc(d);
+  if (st != PQ_OK) return st;
+  const size_t per_group = static_cast<size_t>(d->Cout_g) * d->kh * d->kw * d->Cin_g;
+  std::vector<int8_t> wq(per_group * d->G);
+  const float lo = static_cast<float>(-(1 << (d->bits_w - 1))), hi = static_cast<float>((1 << (d->bits_w - 1)) - 1);
+  for (int g = 0; g < d->G; ++g)
+    for (size_t i = 0; i < per_group; ++i) {
+      // one fp32 multiply, round half to even, clamp (volatile keeps it a single
+      // IEEE fp32 product, never fused or widened)
+      volatile float t = w_host[g * per_group + i] * inv_sw_host[g];
+      float r = std::nearbyint(static_cast<float>(t));
+      r = std::fmax(r, lo);
+      r = std::fmin(r, hi);
+      wq[g * per_group + i] = static_cast<int8_t>(static_cast<int>(r));
+    }
+  return palquant_pack_weight_codes_host(wq.data(), d, packed_host, packed_bytes);
+}
+
+pq_status palquant_pack_weights(const float* w_host, const pq_layer_desc* d, const float* inv_sw_host,
+                                void* packed_dev, size_t packed_bytes, pq_stream_t stream) {
+  if (packed_dev == nullptr) return PQ_EINVAL;
+  const size_t need = palquant_packed_weight_bytes(d);
+  if (need == 0) {
+    pq_status st = validate_desc(d);
+    return st != PQ_OK ? st : PQ_EUNSUPPORTED;
+  }
+  if (packed_bytes < need) return PQ_EINVAL;
+  std::vector<uint8_t> host(need);
+  pq_status st = palquant_pack_weights_host(w_host, d, inv_sw_host, host.data(), need);
+  if (st != PQ_OK) return st;
+  cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(packed_dev, host.data(), need, cudaMemcpyHostToDevice, s) != cudaSuccess) return PQ_ECUDA;
+  if (cudaStreamSynchronize(s) != cudaSuccess) return PQ_ECUDA;
+  return PQ_OK;
+}
+
+pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G, int32_t Cg,
+                                int32_t bits, int32_t code_format, const float* inv_s_host, pq_stream_t stream) {
+  if (x_dev == nullptr || q_dev == nullptr || inv_s_host == nullptr) return PQ_EINVAL;
+  if (N < 0 || H < 1 || W < 1 || G < 1 || Cg < 1 || bits < 1 || bits > 8) return PQ_EINVAL;
+  if (G > pq::kMaxG) return PQ_EUNSUPPORTED;
+  if (code_format != PQ_CODES_INT8) return code_format == PQ_CODES_E4M3 ? PQ_EUNSUPPORTED : PQ_EINVAL;
+  const int64_t P = N * H * W;
+  if (pq::launch_quantize(x_dev, static_cast<uint8_t*>(q_dev), P, G, Cg, bits, inv_s_host,
+                          static_cast<cudaStream_t>(stream)) != 0)
+    return PQ_ECUDA;
+  return PQ_OK;
+}
+
+pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
+                               const float* m_out_host, const float* m_req_host, pq_shuffle shuf,
+                               const float* shortcut_dev, int32_t* acc_out_dev, float* y_out_dev, void* q_out_dev,
+                               pq_stream_t stream) {
+  pq_status st = validate_desc(d);
+  if (st != PQ_OK) return st;
+  if (q_dev == nullptr || w_packed_dev == nullptr) return PQ_EINVAL;
+  if (acc_out_dev == nullptr && y_out_dev == nullptr && q_out_dev == nullptr) return PQ_EINVAL;
+  if ((y_out_dev != nullptr || q_out_dev != nullptr) && m_out_host == nullptr) return PQ_EINVAL;
+  if (q_out_dev != nullptr && m_req_host == nullptr) return PQ_EINVAL;
+  if (!aligned16(q_dev) || !aligned16(w_packed_dev) || !aligned16(acc_out_dev) || !aligned16(y_out_dev) ||
+      !aligned16(q_out_dev) || !aligned16(shortcut_dev))
+    return PQ_EINVAL;
+  ConvParams p;
+  std::vector<Phase> phases;
+  st = plan_conv(d, &p, nullptr, &phases);
+  if (st != PQ_OK) return st;
+  int dst[pq::kMaxG];
+  if (!valid_shuffle(d->G, shuf, dst)) return PQ_EINVAL;
+  if (d->N == 0) return PQ_OK;
+  for (int g = 0; g < d->G; ++g) {
+    p.dst_group[g] = dst[g];
+    p.m_out[g] = m_out_host ? m_out_host[g] : 0.0f;
+    p.m_req[g] = m_req_host ? m_req_host[g] : 0.0f;
+  }
+  p.channel_shuffle = shuf.kind == 2 ? 1 : 0;
+  p.w_packed = static_cast<const uint8_t*>(w_packed_dev);
+  p.shortcut = shortcut_dev;
+  p.acc_out = acc_out_dev;
+  p.y_out = y_out_dev;
+  p.q_out = static_cast<uint8_t*>(q_out_dev);
+  p.err = pq::device_error_word();
+  if (p.err == nullptr) return PQ_ECUDA;
+  p.wait_limit_ns = g_wait_limit_ns.load();
+  TensorMaps tm;
+  if (!encode_activation_maps(d, p, phases, q_dev, &tm)) return PQ_ECUDA;
+  const int sms = device_sm_count();
+  if (sms <= 0) return PQ_ECUDA;
+  const int grid = static_cast<int>(std::min<int64_t>(sms, p.items));
+  if (grid <= 0) return PQ_OK;
+  if (pq::launch_conv_tc(p, tm, grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
+  return PQ_OK;
+}
+
+pq_status palquant_group_conv(const void* q_dev, const void* w_packed_dev, int32_t* acc_dev, const pq_layer_desc* d,
+                              pq_stream_t stream) {
+  if (acc_dev == nullptr) return PQ_EINVAL;
+  pq_shuffle none = {0, 0, nullptr};
+  return palquant_layer_fused(q_dev, w_packed_dev, d, nullptr, nullptr, none, nullptr, acc_dev, nullptr, nullptr,
+                              stream);
+}
+
+pq_status palquant_sync_check(pq_stream_t stream) {
+  if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return PQ_ECUDA;
+  unsigned int* word = pq::device_error_word();
+  if (word == nullptr) return PQ_ECUDA;
+  unsigned int h = 0;
+  if (cudaMemcpy(&h, word, sizeof(h), cudaMemcpyDeviceToHost) != cudaSuccess) return PQ_ECUDA;
+  if (h != 0) {
+    if (cudaMemset(word, 0, sizeof(h)) != cudaSuccess) return PQ_ECUDA;
+    if (cudaDeviceSynchronize() != cudaSuccess) return PQ_ECUDA;
+  }
+  if (h & PQ_ERR_TIMEOUT) return PQ_ETIMEOUT;
+  return PQ_OK;
+}
+
+pq_status palquant_set_wait_limit_ns(uint64_t ns) {
+  g_wait_limit_ns.store(ns == 0 ? kDefaultWaitLimitNs : ns);
+  return PQ_OK;
+}
+
+pq_status palquant_watchdog_selftest(uint64_t limit_ns, pq_stream_t stream) {
+  if (limit_ns == 0 || limit_ns > 10000000000ull) return PQ_EINVAL;
+  unsigned int* word = pq::device_error_word();
+  if (word == nullptr) return PQ_ECUDA;
+  if (pq::launch_watchdog_selftest(word, limit_ns, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
+  return palquant_sync_check(stream);
+}
+
+pq_status palquant_conv_plan(const pq_layer_desc* d, pq_conv_plan* plan) {
+  if (plan == nullptr) return PQ_EINVAL;
+  return plan_conv(d, nullptr, plan, nullptr);
+}
+
+}  // extern "C"

@@ -1,0 +1,147 @@
+// Group-wise activation quantisation (Sec. 3.2 Eq. 2 with l = 0, u = s (2^b - 1),
+// Sec. 4.1 "quantize the activations ... to B-bit in each group") and the
+// deterministic per-group sums behind the step initialisation.
+//
+// Quantisation is HBM-bound (4 bytes in, 1 byte out per element).  The fast path
+// gives each thread 16 consecutive elements of one pixel (so they share a group
+// when C_g is a multiple of 16): four 16-byte streaming loads, one fp32 multiply,
+// a round-to-nearest-even conversion and an integer clamp per element, and one
+// 16-byte streaming store, in a grid-stride loop over a grid sized to the SM count.
+#include <cuda_runtime.h>
+
+#include <cstdint>
+
+#include "pq_internal.h"
+
+namespace pq {
+
+struct QuantArgs {
+  float inv_s[kMaxG];
+};
+
+__device__ __forceinline__ uint32_t quant4(float4 v, float inv, int qmax) {
+  // __float2int_rn = round half to even; NaN -> 0, +-inf saturate and clamp below.
+  int a = __float2int_rn(__fmul_rn(v.x, inv));
+  int b = __float2int_rn(__fmul_rn(v.y, inv));
+  int c = __float2int_rn(__fmul_rn(v.z, inv));
+  int d = __float2int_rn(__fmul_rn(v.w, inv));
+  a = min(max(a, 0), qmax);
+  b = min(max(b, 0), qmax);
+  c = min(max(c, 0), qmax);
+  d = min(max(d, 0), qmax);
+  return static_cast<uint32_t>(a) | (static_cast<uint32_t>(b) << 8) | (static_cast<uint32_t>(c) << 16) |
+         (static_cast<uint32_t>(d) << 24);
+}
+
+// 16 elements per thread-iteration; requires C_g % 16 == 0 and 16-byte aligned x, q.
+__global__ void __launch_bounds__(256) pq_quantize_vec16(const float4* __restrict__ x, uint4* __restrict__ q,
+                                                         int64_t nvec, int vec_per_pix, int vec_per_group, int qmax,
+                                                         const __grid_constant__ QuantArgs args) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t v = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; v < nvec; v += stride) {
+    const int cv = static_cast<int>(v % vec_per_pix);
+    const float inv = args.inv_s[cv / vec_per_group];
+    const float4* src = x + 4 * v;
+    const float4 a = __ldcs(src), b = __ldcs(src + 1), c = __ldcs(src + 2), d = __ldcs(src + 3);
+    uint4 out;
+    out.x = quant4(a, inv, qmax);
+    out.y = quant4(b, inv, qmax);
+    out.z = quant4(c, inv, qmax);
+    out.w = quant4(d, inv, qmax);
+    __stcs(q + v, out);
+  }
+}
+
+// Any shape: one element per thread-iteration.
+__global__ void __launch_bounds__(256) pq_quantize_scalar(const float* __restrict__ x, uint8_t* __restrict__ q,
+                                                          int64_t n, int C, int Cg, int qmax,
+                                                          const __grid_constant__ QuantArgs args) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t e = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; e < n; e += stride) {
+    const int c = static_cast<int>(e % C);
+    int v = __float2int_rn(__fmul_rn(x[e], args.inv_s[c / Cg]));
+    v = min(max(v, 0), qmax);
+    q[e] = static_cast<uint8_t>(v);
+  }
+}
+
+static int quant_grid(int64_t work) {
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (work + 255) / 256;
+  const int64_t cap = static_cast<int64_t>(sms) * 8;
+  return static_cast<int>(want < cap ? (want > 0 ? want : 1) : cap);
+}
+
+int launch_quantize(const float* x, uint8_t* q, int64_t P, int G, int Cg, int bits, const float* inv_s,
+                    cudaStream_t stream) {
+  QuantArgs args;
+  for (int g = 0; g < G; ++g) args.inv_s[g] = inv_s[g];
+  const int C = G * Cg;
+  const int64_t n = P * C;
+  const int qmax = (1 << bits) - 1;
+  if (n == 0) return 0;
+  const bool aligned = (reinterpret_cast<uintptr_t>(x) % 16 == 0) && (reinterpret_cast<uintptr_t>(q) % 16 == 0);
+  if (Cg % 16 == 0 && aligned) {
+    const int64_t nvec = n / 16;
+    pq_quantize_vec16<<<quant_grid(nvec), 256, 0, stream>>>(reinterpret_cast<const float4*>(x),
+                                                           reinterpret_cast<uint4*>(q), nvec, C / 16, Cg / 16, qmax,
+                                                           args);
+  } else {
+    pq_quantize_scalar<<<quant_grid(n), 256, 0, stream>>>(x, q, n, C, Cg, qmax, args);
+  }
+  return cudaGetLastError() == cudaSuccess ? 0 : -1;
+}
+
+// --------------------------------------------------------------------------
+// Deterministic per-group sums for the step initialisation.  Pass 1: block b
+// sums, in double and in a fixed order, group g's elements of the pixel range
+// [b P / B, (b+1) P / B) and writes partial[b * G + g].  Pass 2: partial sums
+// are added in block order.  B is fixed, so the result does not depend on the
+// device or on timing.
+// --------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) pq_act_sum_pass1(const float* __restrict__ x, int64_t P, int G, int Cg,
+                                                        double* __restrict__ partial) {
+  __shared__ double red[256];
+  const int64_t p0 = static_cast<int64_t>(blockIdx.x) * P / gridDim.x;
+  const int64_t p1 = static_cast<int64_t>(blockIdx.x + 1) * P / gridDim.x;
+  const int64_t C = static_cast<int64_t>(G) * Cg;
+  const int64_t cnt = (p1 - p0) * Cg;
+  for (int g = 0; g < G; ++g) {
+    double s = 0.0;
+    for (int64_t e = threadIdx.x; e < cnt; e += blockDim.x) {
+      const int64_t pix = p0 + e / Cg;
+      const int j = static_cast<int>(e % Cg);
+      s += static_cast<double>(x[pix * C + static_cast<int64_t>(g) * Cg + j]);
+    }
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+      if (threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+      __syncthreads();
+    }
+    if (threadIdx.x == 0) partial[static_cast<int64_t>(blockIdx.x) * G + g] = red[0];
+    __syncthreads();
+  }
+}
+
+__global__ void pq_act_sum_pass2(const double* __restrict__ partial, int nblocks, int G, double* __restrict__ sums) {
+  const int g = blockIdx.x * blockDim.x + threadIdx.x;
+  if (g >= G) return;
+  double s = 0.0;
+  for (int b = 0; b < nblocks; ++b) s += partial[static_cast<int64_t>(b) * G + g];
+  sums[g] = s;
+}
+
+int launch_act_sum(const float* x, int64_t P, int G, int Cg, double* partial, int nblocks, cudaStream_t stream) {
+  pq_act_sum_pass1<<<nblocks, 256, 0, stream>>>(x, P, G, Cg, partial);
+  return cudaGetLastError() == cudaSuccess ? 0 : -1;
+}
+
+int launch_act_sum_finish(const double* partial, int nblocks, int G, double* sums, cudaStream_t stream) {
+  pq_act_sum_pass2<<<(G + 63) / 64, 64, 0, stream>>>(partial, nblocks, G, sums);
+  return cudaGetLastError() == cudaSuccess ? 0 : -1;
+}
+
+}  // namespace pq

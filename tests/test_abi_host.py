@@ -1,0 +1,161 @@
+"""The C-ABI library on the host (no GPU): exported symbols, planner invariants,
+weight packing, host-side set-up against the oracle, and argument validation."""
+import os
+import re
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2208_01944_gb300 import synth, workloads
+
+B = pytest.importorskip("paper_2208_01944_gb300.binding", reason="libpalquant.so not built")
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "palquant.h")
+
+
+def _desc(c, **kw):
+    args = dict(N=c.N, H=c.H, W=c.W, G=c.G, Cin_g=c.Cin_g, Cout_g=c.Cout_g, k=c.k, stride=c.stride, pad=c.pad,
+                bits_a=c.bits_a, bits_w=c.bits_w, bits_out=c.bits_out)
+    args.update(kw)
+    return B.layer_desc(**args)
+
+
+def test_every_declared_symbol_is_exported():
+    decls = set(re.findall(r"\b(palquant_\w+)\s*\(", open(HEADER).read()))
+    assert decls == set(B.EXPORTS)
+    for name in decls:
+        assert hasattr(B.lib, name), name
+    assert B.palquant_version() >= 100
+    assert B.strerror(B.PQ_ETIMEOUT) == "in-kernel wait timed out"
+
+
+def test_raw_code_byte_is_e4m3_of_scaled_code():
+    """A code byte v <= 15 is the FP8 E4M3 encoding of v * 2^-9 (checked with torch's fp8 type)."""
+    v = torch.arange(16, dtype=torch.uint8)
+    as_fp8 = v.view(torch.float8_e4m3fn).to(torch.float64)
+    assert torch.equal(as_fp8 * 512.0, v.to(torch.float64))
+
+
+ALL_LAYERS = list(workloads.BENCH_CONFIGS.values()) + [c for _, _, c in workloads.resnet18_layers()]
+
+
+@pytest.mark.parametrize("c", ALL_LAYERS, ids=lambda c: f"{c.H}x{c.W}k{c.k}s{c.stride}G{c.G}c{c.Cin_g}-{c.Cout_g}")
+def test_plan_invariants(c):
+    plan = B.palquant_conv_plan(_desc(c))
+    assert plan.supported == 1
+    assert plan.smem_bytes + 1024 <= 227 * 1024
+    assert plan.n_block * plan.n_blocks == c.Cout_g and plan.n_block % 16 == 0 and 16 <= plan.n_block <= 256
+    assert plan.k_chunk * plan.k_blocks == c.Cin_g and plan.k_chunk % 32 == 0
+    assert plan.taps == c.k * c.k
+    rows = plan.m_tiles * 128
+    if plan.mode == 1:
+        assert plan.rows_per_tile * plan.tile_pitch <= rows
+        tiles_per_img = -(-c.Ho // plan.rows_per_tile)
+        assert plan.tiles == c.N * tiles_per_img
+        assert plan.tile_pitch >= c.Wo
+    else:
+        assert plan.tiles == -(-(c.N * c.Ho * c.Wo) // rows)
+    assert plan.work_items == plan.tiles * c.G * plan.n_blocks
+    assert plan.acc_stages * plan.m_tiles * plan.n_block <= 512
+
+
+@pytest.mark.parametrize("shape", [(2, 48, 3, 64, 4), (4, 96, 1, 96, 2), (1, 272, 3, 32, 2), (3, 64, 3, 128, 4)])
+def test_pack_unpack_roundtrip_and_fp8_encoding(shape):
+    G, Co, k, Ci, bits = shape
+    d = B.layer_desc(1, 8, 8, G, Ci, Co, k, 1, k // 2, bits, bits, bits)
+    gen = synth.generator(sum(shape))
+    wq = synth.random_codes((G, Co, k, k, Ci), bits, gen, signed=True)
+    packed = B.palquant_pack_weight_codes_host(wq, d)
+    assert packed.size == wq.size
+    assert np.array_equal(B.palquant_unpack_weight_codes_host(packed, d), wq)
+    # The packed bytes are the FP8 E4M3 encodings of the codes (as a multiset per group
+    # they must equal torch's encoding of the same integers).
+    fp8 = torch.from_numpy(wq.astype(np.float32)).to(torch.float8_e4m3fn).view(torch.uint8).numpy()
+    assert np.array_equal(np.sort(packed), np.sort(fp8.ravel()))
+
+
+def test_pack_rejects_out_of_range_codes():
+    d = B.layer_desc(1, 4, 4, 1, 32, 16, 1, 1, 0, 2, 2, 2)
+    wq = np.zeros((1, 16, 1, 1, 32), dtype=np.int8)
+    wq[0, 3, 0, 0, 5] = 2  # outside [-2, 1] for 2-bit codes
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_pack_weight_codes_host(wq, d)
+    assert e.value.status == B.PQ_EINVAL
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_weight_quantisation_matches_oracle(bits):
+    G, Co, k, Ci = 3, 32, 3, 64
+    gen = synth.generator(40 + bits)
+    w = synth.he_weights(G, Co, k, k, Ci, gen)
+    d = B.layer_desc(1, 6, 6, G, Ci, Co, k, 1, 1, 2, bits, 2)
+    s_w = B.palquant_weight_steps(w, d)
+    assert np.array_equal(s_w, oracle.weight_step(w, bits))
+    inv = oracle.inv_step(s_w)
+    packed = B.palquant_pack_weights_host(w, d, inv)
+    assert np.array_equal(B.palquant_unpack_weight_codes_host(packed, d), oracle.quantize_weights(w, bits, inv))
+
+
+def test_weight_quantisation_ties_and_clamp():
+    d = B.layer_desc(1, 4, 4, 1, 32, 16, 1, 1, 0, 2, 2, 2)
+    w = np.zeros((1, 16, 1, 1, 32), dtype=np.float32)
+    w[0, 0, 0, 0, :6] = [0.5, 1.5, -0.5, -1.5, 9.0, -9.0]
+    packed = B.palquant_pack_weights_host(w, d, [1.0])
+    wq = B.palquant_unpack_weight_codes_host(packed, d)
+    assert list(wq[0, 0, 0, 0, :6]) == [0, 1, 0, -2, 1, -2]
+
+
+@pytest.mark.parametrize("kind,shift,perm", [(0, 0, None), (1, 1, None), (1, -1, None), (3, 0, [2, 0, 3, 1])])
+def test_epilogue_scales_match_oracle(kind, shift, perm):
+    gen = synth.generator(7)
+    s_w = synth.half_normal((4,), gen) + 0.1
+    s_a = synth.half_normal((4,), gen) + 0.1
+    s_n = synth.half_normal((4,), gen) + 0.1
+    mo, mr = B.palquant_epilogue_scales(4, s_w, s_a, 1.25, s_n, B.shuffle(kind, shift, perm))
+    ro, rr = oracle.epilogue_scales(s_w, s_a, s_n, 1.25, kind, shift, perm)
+    assert np.array_equal(mo, ro) and np.array_equal(mr, rr)
+
+
+def test_invalid_arguments_rejected_before_launch():
+    good = B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1)
+    bad_descs = [
+        B.layer_desc(1, 0, 8, 2, 32, 32, 3, 1, 1),       # H = 0
+        B.layer_desc(1, 8, 8, 0, 32, 32, 3, 1, 1),       # G = 0
+        B.layer_desc(1, 8, 8, 2, 32, 32, 3, 0, 1),       # stride 0
+        B.layer_desc(1, 2, 2, 2, 32, 32, 5, 1, 0),       # output would be empty
+        B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, bits_a=9),
+    ]
+    for d in bad_descs:
+        with pytest.raises(B.PalquantError) as e:
+            B.palquant_layer_fused(16, 16, d, [1.0] * 2, [1.0] * 2, acc_out_dev=16)
+        assert e.value.status == B.PQ_EINVAL
+    # no output requested
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_layer_fused(16, 16, good, [1.0] * 2, [1.0] * 2)
+    assert e.value.status == B.PQ_EINVAL
+    # codes requested without requantisation multipliers
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_layer_fused(16, 16, good, [1.0] * 2, None, q_out_dev=16)
+    assert e.value.status == B.PQ_EINVAL
+    # misaligned device pointer
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_layer_fused(17, 16, good, [1.0] * 2, [1.0] * 2, acc_out_dev=16)
+    assert e.value.status == B.PQ_EINVAL
+    # not a permutation
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_layer_fused(16, 16, good, [1.0] * 2, [1.0] * 2, shuf=B.shuffle(3, 0, [1, 1]), acc_out_dev=16)
+    assert e.value.status == B.PQ_EINVAL
+
+
+def test_unsupported_shapes_reported():
+    for d in [B.layer_desc(1, 8, 8, 2, 24, 32, 3, 1, 1),          # Cin_g not a multiple of 32
+              B.layer_desc(1, 8, 8, 2, 32, 24, 3, 1, 1),          # Cout_g not a multiple of 16
+              B.layer_desc(1, 8, 8, 2, 32, 32, 3, 3, 1),          # stride 3
+              B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, bits_a=6)]:  # codes beyond the exact FP8 range
+        assert B.palquant_conv_plan(d).supported == 0
+        assert B.palquant_packed_weight_bytes(d) == 0
+        with pytest.raises(B.PalquantError) as e:
+            B.palquant_layer_fused(16, 16, d, [1.0] * 2, [1.0] * 2, acc_out_dev=16)
+        assert e.value.status == B.PQ_EUNSUPPORTED

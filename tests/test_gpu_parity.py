@@ -1,0 +1,200 @@
+"""GPU parity of the hot path against the CPU oracle, through the C ABI.
+
+Integer outputs (activation codes, int32 sums, requantised codes) must match the
+oracle bit for bit; fp32 outputs within a relative error of 1e-5 (they are single
+IEEE multiplies / adds in the same order, so they are expected to be exact).
+"""
+import numpy as np
+import pytest
+
+import oracle
+from paper_2208_01944_gb300 import synth, workloads
+
+from layer_cases import Case, assert_layer_parity, prepare, run_gpu
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+
+
+@pytest.fixture(scope="module")
+def B():
+    assert torch.cuda.is_available(), "GPU tests need a CUDA device"
+    from paper_2208_01944_gb300 import binding
+
+    return binding
+
+
+# ------------------------------------------------------------ a2 quantize
+@pytest.mark.parametrize("shape,G,bits", [((2, 7, 9, 64), 4, 2), ((1, 5, 5, 3 * 16), 3, 4), ((3, 4, 6, 2 * 20), 2, 3),
+                                          ((1, 1, 1, 32), 1, 8), ((5, 33, 17, 256), 4, 2)])
+def test_quantize_act_matches_oracle(B, shape, G, bits):
+    gen = synth.generator(sum(shape) + bits)
+    x = synth.normal(shape, gen, 2.0)
+    flat = x.reshape(-1)
+    # ties, NaN and infinities at fixed places
+    specials = np.array([0.5, 1.5, 2.5, -0.5, np.nan, np.inf, -np.inf, 3.5, 1e30, -0.0], dtype=np.float32)
+    flat[: specials.size] = specials
+    inv = (synth.half_normal((G,), gen) + 0.5).astype(np.float32)
+    inv[0] = 1.0
+    ref = oracle.quantize_act(x, G, bits, inv)
+    xd = torch.from_numpy(x).cuda()
+    q = torch.full(shape, 254, dtype=torch.uint8, device="cuda")
+    B.palquant_quantize_act(xd, q, shape[0], shape[1], shape[2], G, shape[3] // G, bits, inv)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(q.cpu().numpy(), ref)
+
+
+def test_quantize_act_misaligned_views_use_scalar_path(B):
+    gen = synth.generator(3)
+    x = synth.normal((1, 4, 4, 33), gen)
+    xd = torch.from_numpy(x).cuda()
+    # an offset view: 4-byte aligned but not 16-byte aligned
+    big = torch.zeros(x.size + 1, dtype=torch.float32, device="cuda")
+    big[1:] = xd.reshape(-1)
+    q = torch.zeros(x.size + 1, dtype=torch.uint8, device="cuda")
+    B.palquant_quantize_act(big[1:].data_ptr(), q[1:].data_ptr(), 1, 4, 4, 1, 33, 2, [1.7])
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(q[1:].cpu().numpy().reshape(x.shape), oracle.quantize_act(x, 1, 2, [1.7]))
+
+
+# ------------------------------------------------------------ a0 steps
+@pytest.mark.parametrize("shape,G,bits", [((2, 9, 7, 64), 2, 2), ((64, 8, 8, 256), 4, 2), ((1, 3, 3, 24), 3, 4)])
+def test_act_steps_match_oracle(B, shape, G, bits):
+    gen = synth.generator(11)
+    x = synth.half_normal(shape, gen)
+    xd = torch.from_numpy(x).cuda()
+    P = shape[0] * shape[1] * shape[2]
+    nbytes = B.palquant_act_steps_scratch_bytes(P, G)
+    scratch = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    s = B.palquant_act_steps(xd, shape[0], shape[1], shape[2], G, shape[3] // G, bits, scratch, nbytes)
+    ref = oracle.act_step(x, G, bits)
+    # both sum in double (different order), then round to float once: at most 1 ulp apart
+    assert np.all(np.abs(s.view(np.int32) - ref.view(np.int32)) <= 1)
+
+
+# ------------------------------------------------------------ a3-a6 layer
+SMALL_CASES = [
+    Case(1, 28, 28, 2, 32, 32, 3, 1, 1, seed=0),                      # config 0 shape
+    Case(2, 13, 11, 3, 32, 48, 3, 1, 1, seed=1),                      # odd sizes, 3 output chunks
+    Case(3, 9, 17, 4, 64, 64, 3, 2, 1, seed=2),                       # stride 2, odd input
+    Case(2, 10, 10, 2, 64, 128, 1, 2, 0, kind=0, relu=False, seed=3),  # 1x1 stride-2 downsample
+    Case(2, 7, 9, 4, 96, 96, 1, 1, 0, seed=4),                        # flat mode, ragged last tile
+    Case(1, 15, 15, 1, 32, 16, 3, 1, 0, bits=4, kind=0, seed=5),      # pad 0, G = 1, 4-bit
+    Case(2, 14, 14, 8, 32, 32, 3, 1, 1, kind=3, perm=(3, 0, 7, 1, 6, 2, 5, 4), seed=6),
+    Case(1, 12, 12, 2, 128, 256, 3, 1, 1, bits=4, seed=7),            # streamed weights, 4-bit
+    Case(1, 7, 7, 2, 512, 32, 3, 1, 1, seed=8),                       # four K blocks, whole-image tiles
+    Case(2, 8, 8, 2, 32, 320, 3, 1, 1, seed=9),                       # two output-channel blocks
+    Case(1, 5, 130, 1, 32, 16, 3, 1, 1, seed=10),                     # row wider than 128 positions
+    Case(2, 9, 9, 4, 32, 32, 3, 1, 1, kind=2, seed=11),               # channel shuffle
+    Case(2, 11, 10, 2, 64, 64, 3, 1, 1, shortcut=True, seed=12),      # shortcut add before ReLU
+    Case(1, 9, 11, 2, 32, 64, 5, 1, 2, seed=13),                      # 5x5 kernel
+    Case(2, 6, 6, 2, 32, 32, 3, 1, 1, bits=3, bits_out=4, relu=False, kind=1, shift=-1, seed=14),
+    Case(1, 16, 16, 4, 64, 64, 3, 2, 0, seed=15),                     # stride 2 without padding
+]
+
+
+@pytest.mark.parametrize("c", SMALL_CASES, ids=str)
+def test_layer_fused_matches_oracle(B, c):
+    ref = prepare(c)
+    got = run_gpu(c, ref)
+    assert_layer_parity(c, ref, got)
+
+
+def test_group_conv_matches_oracle(B):
+    c = Case(2, 12, 9, 3, 64, 48, 3, 1, 1, kind=0)
+    ref = prepare(c)
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad)
+    q = torch.from_numpy(ref["q"]).cuda()
+    wp = torch.from_numpy(B.palquant_pack_weight_codes_host(ref["wq"], d)).cuda()
+    acc = torch.zeros((c.N, c.Ho, c.Wo, c.G * c.Cout), dtype=torch.int32, device="cuda")
+    B.palquant_group_conv(q, wp, acc, d)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), oracle.group_conv(ref["q"], ref["wq"], c.stride, c.pad))
+
+
+@pytest.mark.parametrize("bits,Cin", [(4, 512), (2, 512), (4, 64)])
+def test_worst_case_magnitudes_exact(B, bits, Cin):
+    """All codes at their extreme: every sum is the largest the layer can produce."""
+    G, Co, k = 2, 32, 3
+    N, H, W = 1, 6, 6
+    qa, wmin = (1 << bits) - 1, -(1 << (bits - 1))
+    q = np.full((N, H, W, G * Cin), qa, dtype=np.uint8)
+    wq = np.full((G, Co, k, k, Cin), wmin, dtype=np.int8)
+    wq[1] = (1 << (bits - 1)) - 1
+    d = B.layer_desc(N, H, W, G, Cin, Co, k, 1, 1, bits, bits, bits)
+    wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).cuda()
+    acc = torch.zeros((N, H, W, G * Co), dtype=torch.int32, device="cuda")
+    B.palquant_group_conv(torch.from_numpy(q).cuda(), wp, acc, d)
+    assert B.palquant_sync_check() == B.PQ_OK
+    ref = oracle.group_conv(q, wq, 1, 1)
+    assert np.abs(ref).max() == 9 * Cin * qa * -wmin
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), ref)
+
+
+def test_empty_batch_is_a_noop(B):
+    d = B.layer_desc(0, 8, 8, 2, 32, 32, 3, 1, 1)
+    wq = np.zeros((2, 32, 3, 3, 32), dtype=np.int8)
+    wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).cuda()
+    q = torch.zeros(16, dtype=torch.uint8, device="cuda")
+    acc = torch.zeros(16, dtype=torch.int32, device="cuda")
+    B.palquant_group_conv(q, wp, acc, d)
+    assert B.palquant_sync_check() == B.PQ_OK
+
+
+def test_outputs_untouched_outside_tensor(B):
+    """Canary bytes around the outputs stay intact (no out-of-bounds stores)."""
+    c = Case(2, 9, 13, 2, 32, 48, 3, 1, 1, seed=21)
+    ref = prepare(c)
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad)
+    n_out = c.N * c.Ho * c.Wo * c.G * c.Cout
+    pad = 4096
+    q = torch.from_numpy(ref["q"]).cuda()
+    wp = torch.from_numpy(B.palquant_pack_weight_codes_host(ref["wq"], d)).cuda()
+    qo = torch.full((n_out + 2 * pad,), 0xA5, dtype=torch.uint8, device="cuda")
+    y = torch.full((n_out + 2 * pad // 4 * 4,), 7.25, dtype=torch.float32, device="cuda")
+    B.palquant_layer_fused(q, wp, d, ref["m_out"], ref["m_req"], B.shuffle(1, 1), None, None,
+                           y[pad // 4 * 2: pad // 4 * 2 + n_out].data_ptr(), qo[pad: pad + n_out].data_ptr())
+    assert B.palquant_sync_check() == B.PQ_OK
+    qh = qo.cpu().numpy()
+    assert (qh[:pad] == 0xA5).all() and (qh[pad + n_out:] == 0xA5).all()
+    yh = y.cpu().numpy()
+    assert (yh[: pad // 2] == 7.25).all() and (yh[pad // 2 + n_out:] == 7.25).all()
+    assert np.array_equal(qh[pad: pad + n_out].reshape(-1, c.G * c.Cout), ref["q_ref"])
+
+
+# ----------------------------------------------- full-size workloads (sampled)
+def _sample_pixels(N, Ho, Wo, n_random, seed):
+    rng = np.random.default_rng(seed)
+    P = N * Ho * Wo
+    corners = []
+    for n in (0, N - 1):
+        for oh in (0, Ho - 1):
+            for ow in (0, Wo - 1):
+                corners.append((n * Ho + oh) * Wo + ow)
+    edges = [(n * Ho + oh) * Wo + ow for n in (N // 2,) for oh in range(Ho) for ow in (0, Wo - 1)]
+    pix = np.unique(np.concatenate([np.array(corners + edges), rng.integers(0, P, n_random)]))
+    return pix.astype(np.int64)
+
+
+FULL = [("config1", workloads.CONFIG1)] + [(f"config3_{i}", c) for i, c in enumerate(workloads.CONFIG3)] + [
+    ("config4", workloads.CONFIG4)]
+
+
+@pytest.mark.parametrize("name,cfg", FULL, ids=[n for n, _ in FULL])
+def test_full_size_layer_sampled(B, name, cfg):
+    c = Case(cfg.N, cfg.H, cfg.W, cfg.G, cfg.Cin_g, cfg.Cout_g, cfg.k, cfg.stride, cfg.pad, bits=cfg.bits_a,
+             kind=cfg.shuffle_kind, shift=cfg.shuffle_shift, relu=cfg.relu, seed=0)
+    pix = _sample_pixels(c.N, c.Ho, c.Wo, 3000, 1)
+    ref = prepare(c, sample_pix=pix)
+    got = run_gpu(c, ref)
+    assert_layer_parity(c, ref, got, pix)
+
+
+# ------------------------------------------------------ failure detection
+def test_watchdog_times_out_and_context_survives(B):
+    assert B.palquant_watchdog_selftest(2_000_000) == B.PQ_ETIMEOUT  # a 2 ms wait nobody completes
+    assert B.palquant_sync_check() == B.PQ_OK                         # the error word was cleared
+    c = Case(1, 6, 6, 2, 32, 32, 3, 1, 1, seed=30)
+    ref = prepare(c)
+    assert_layer_parity(c, ref, run_gpu(c, ref))                      # the context still works
