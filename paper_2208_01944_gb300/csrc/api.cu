@@ -2,7 +2,6 @@
 // tensor-core convolution, weight quantisation and packing, tensor-map encoding,
 // launches and error reporting.  Every entry point of include/palquant.h is
 // defined here.
-#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -13,11 +12,10 @@
 #include <mutex>
 #include <vector>
 
-#include "../../include/palquant.h"
+#include "palquant.h"
 #include "pq_internal.h"
 
 using pq::ConvParams;
-using pq::TensorMaps;
 
 namespace {
 
@@ -235,22 +233,24 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
       if (pub) *pub = plan;
       return PQ_EUNSUPPORTED;
     }
+    for (size_t i = 0; i < phases.size(); ++i) {
+      p.phase_a[i] = phases[i].a;
+      p.phase_b[i] = phases[i].b;
+    }
   }
   p.items = p.tiles * d->G * NB;
   // K blocks, weights residency and pipeline depth under the shared-memory budget.
   const uint32_t budget = pq::kMaxSmem - 1024;
-  auto a_stage_bytes = [&](int KC, uint32_t* phase_bytes, uint32_t* tx, uint32_t* lbo) -> uint32_t {
+  auto a_stage_bytes = [&](int KC, uint32_t* phase_bytes, uint32_t* lbo) -> uint32_t {
     const int nch = KC / 16;
     if (flat) {
       const uint32_t plane = static_cast<uint32_t>(p.flat_box) * 16u;
       *phase_bytes = round_up(static_cast<uint64_t>(nch) * plane, 128);
-      *tx = nch * plane;
       *lbo = plane;
       return round_up(*phase_bytes, 1024);
     }
     const uint32_t plane = static_cast<uint32_t>(p.Hd) * p.Wd * 16u;
     *phase_bytes = round_up(static_cast<uint64_t>(nch) * plane, 128);
-    *tx = static_cast<uint32_t>(p.nph) * nch * plane;
     *lbo = plane;
     const uint64_t overrun = static_cast<uint64_t>(p.nph - 1) * (*phase_bytes) + static_cast<uint64_t>(nch - 1) * plane +
                              16ull * (p.MT * 128 + off_max);
@@ -260,7 +260,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // fp32/int32 values, row pitch 80 bytes (an odd number of 16-byte bank groups).
   const uint32_t q_pitch = 80;
   const uint32_t f_pitch = 80;
-  const uint32_t warp_stage = round_up(32u * (q_pitch + f_pitch), 128);
+  const uint32_t warp_stage = round_up(32u * q_pitch, 128);
   const uint32_t stage_total = warp_stage * pq::kEpiWarps;
   const uint32_t bar_bytes = 1024;  // barriers, abort flag, TMEM slot (generous)
   const uint64_t unit_bytes = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk;
@@ -268,11 +268,14 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // unit's weights resident if they fit, else a ring of (K block, tap) slices.
   bool found = false, resident = false;
   int KC = d->Cin_g, a_stages = 0, b_stages = 0;
-  uint32_t stage_bytes = 0, phase_bytes = 0, tx = 0, lbo = 0;
-  for (int kc = d->Cin_g; kc >= 32 && !found; kc /= 2) {
-    if (d->Cin_g % kc != 0 || kc % 32 != 0) continue;
-    uint32_t sb, pb, t, l;
-    sb = a_stage_bytes(kc, &pb, &t, &l);
+  uint32_t stage_bytes = 0, phase_bytes = 0, lbo = 0;
+  // K blocks of 32 * {8, 4, 3, 2, 1} channels: the MMA issue loop is compiled for
+  // these K-step counts.
+  for (int kc : {256, 128, 96, 64, 32}) {
+    if (found) break;
+    if (d->Cin_g % kc != 0) continue;
+    uint32_t sb, pb, l;
+    sb = a_stage_bytes(kc, &pb, &l);
     if (sb > 64u * 1024u) continue;
     for (int res = 1; res >= 0 && !found; --res) {
       if (res && unit_bytes > 112u * 1024u) continue;
@@ -289,7 +292,6 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
             b_stages = nb;
             stage_bytes = sb;
             phase_bytes = pb;
-            tx = t;
             lbo = l;
           }
         }
@@ -303,11 +305,17 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const uint32_t b_bytes = resident ? round_up(unit_bytes, 1024) : round_up(static_cast<uint64_t>(b_stages) * KC * p.Nblk, 1024);
   p.KC = KC;
   p.nch = KC / 16;
+  p.nch_magic = static_cast<uint32_t>(((1ull << 32) + p.nch - 1) / p.nch);
+  p.H = d->H;
+  p.W = d->W;
+  p.stride = d->stride;
+  p.C_in_total = d->G * d->Cin_g;
   p.n_kb = d->Cin_g / KC;
   p.lbo_a = lbo;
   p.a_phase_bytes = phase_bytes;
+  for (int t = 0; t < taps; ++t)
+    p.tap_a16[t] = (static_cast<uint32_t>(p.tap_phase[t]) * phase_bytes + static_cast<uint32_t>(p.tap_off[t]) * 16u) >> 4;
   p.a_stage_bytes = stage_bytes;
-  p.a_tx_bytes = tx;
   p.a_stages = a_stages;
   p.b_resident = resident ? 1 : 0;
   p.b_slice_bytes = static_cast<uint32_t>(KC) * p.Nblk;
@@ -346,64 +354,6 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   if (P) *P = p;
   if (phases_out) *phases_out = phases;
   return PQ_OK;
-}
-
-// ---------------------------------------------------------------------------
-// Tensor maps.
-// ---------------------------------------------------------------------------
-typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
-
-EncodeTiledFn encode_fn() {
-  static std::once_flag once;
-  static EncodeTiledFn fn = nullptr;
-  std::call_once(once, [] {
-    void* ptr = nullptr;
-    cudaDriverEntryPointQueryResult qres;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &qres) ==
-            cudaSuccess &&
-        qres == cudaDriverEntryPointSuccess)
-      fn = reinterpret_cast<EncodeTiledFn>(ptr);
-  });
-  return fn;
-}
-
-bool encode_activation_maps(const pq_layer_desc* d, const ConvParams& p, const std::vector<Phase>& phases,
-                            const void* q_dev, TensorMaps* tm) {
-  EncodeTiledFn enc = encode_fn();
-  if (enc == nullptr) return false;
-  std::memset(tm, 0, sizeof(*tm));
-  const uint64_t C = static_cast<uint64_t>(d->G) * d->Cin_g;
-  const uint8_t* base = static_cast<const uint8_t*>(q_dev);
-  if (p.mode == pq::kModeFlat) {
-    const uint64_t P = static_cast<uint64_t>(d->N) * d->H * d->W;
-    cuuint64_t dims[3] = {16, P, C / 16};
-    cuuint64_t strides[2] = {C, 16};
-    cuuint32_t box[3] = {16, static_cast<cuuint32_t>(p.flat_box), static_cast<cuuint32_t>(p.nch)};
-    cuuint32_t es[3] = {1, 1, 1};
-    return enc(&tm->a[0], CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<uint8_t*>(base), dims, strides, box, es,
-               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-  }
-  const int s = d->stride;
-  for (size_t i = 0; i < phases.size(); ++i) {
-    const int a = phases[i].a, b = phases[i].b;
-    const uint64_t Wph = (d->W - b + s - 1) / s, Hph = (d->H - a + s - 1) / s;
-    if (Wph == 0 || Hph == 0) return false;
-    cuuint64_t dims[5] = {16, Wph, Hph, C / 16, static_cast<cuuint64_t>(d->N)};
-    cuuint64_t strides[4] = {s * C, s * static_cast<uint64_t>(d->W) * C, 16,
-                             static_cast<uint64_t>(d->H) * d->W * C};
-    cuuint32_t box[5] = {16, static_cast<cuuint32_t>(p.Wd), static_cast<cuuint32_t>(p.Hd),
-                         static_cast<cuuint32_t>(p.nch), 1};
-    cuuint32_t es[5] = {1, 1, 1, 1, 1};
-    const uint8_t* phase_base = base + (static_cast<uint64_t>(a) * d->W + b) * C;
-    if (enc(&tm->a[i], CU_TENSOR_MAP_DATA_TYPE_UINT8, 5, const_cast<uint8_t*>(phase_base), dims, strides, box, es,
-            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
-      return false;
-  }
-  return true;
 }
 
 bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
@@ -615,10 +565,16 @@ pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, cons
   int dst[pq::kMaxG];
   if (!valid_shuffle(d->G, shuf, dst)) return PQ_EINVAL;
   if (d->N == 0) return PQ_OK;
+  // Multipliers are scaled by 2^9 inside the kernel; keep them in the range where
+  // that scaling and every product with an accumulator stay exact normal floats.
+  auto usable = [](float m) { return std::isfinite(m) && (m == 0.0f || (std::fabs(m) > 1e-30f && std::fabs(m) < 1e30f)); };
   for (int g = 0; g < d->G; ++g) {
     p.dst_group[g] = dst[g];
     p.m_out[g] = m_out_host ? m_out_host[g] : 0.0f;
     p.m_req[g] = m_req_host ? m_req_host[g] : 0.0f;
+    if (!usable(p.m_out[g]) || !usable(p.m_req[g])) return PQ_EINVAL;
+    p.m_out512[g] = p.m_out[g] * 512.0f;
+    p.m_req512[g] = p.m_req[g] * 512.0f;
   }
   p.channel_shuffle = shuf.kind == 2 ? 1 : 0;
   p.w_packed = static_cast<const uint8_t*>(w_packed_dev);
@@ -629,13 +585,12 @@ pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, cons
   p.err = pq::device_error_word();
   if (p.err == nullptr) return PQ_ECUDA;
   p.wait_limit_ns = g_wait_limit_ns.load();
-  TensorMaps tm;
-  if (!encode_activation_maps(d, p, phases, q_dev, &tm)) return PQ_ECUDA;
+  p.q_in = static_cast<const uint8_t*>(q_dev);
   const int sms = device_sm_count();
   if (sms <= 0) return PQ_ECUDA;
   const int grid = static_cast<int>(std::min<int64_t>(sms, p.items));
   if (grid <= 0) return PQ_OK;
-  if (pq::launch_conv_tc(p, tm, grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
+  if (pq::launch_conv_tc(p, grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
   return PQ_OK;
 }
 

@@ -9,28 +9,31 @@
 // all written at the destination channel of (g, co).
 //
 // How (one persistent CTA per SM, warp-specialised):
-//  * warp 0 (one lane) loads, per tile, the activation codes a tile needs with
-//    TMA straight into the tensor core's no-swizzle K-major operand layout: for
-//    each 16-byte chunk of input channels a plane of consecutive positions, one
-//    position per 16-byte row.  A "position" is a pixel of the zero-padded input
-//    tile (rows mode) or a pixel of the flattened batch (flat mode, 1x1 layers).
-//    Out-of-range pixels are zero-filled by TMA, which is exactly the zero
-//    padding (code 0).  Stride-2 layers load the four stride phases of the input
-//    through strided tensor views, so every tap is again a contiguous run of
-//    positions.
+//  * warps 2-5 copy, per tile, the activation codes the tile needs with 16-byte
+//    cp.async straight into the tensor core's no-swizzle K-major operand layout:
+//    for each 16-byte chunk of input channels a plane of consecutive positions,
+//    one position per 16-byte row.  A "position" is a pixel of the zero-padded
+//    input tile (rows mode) or a pixel of the flattened batch (flat mode, 1x1
+//    layers).  Out-of-range pixels are zero-filled, which is exactly the zero
+//    padding (code 0).  Stride-2 layers get one plane set per stride phase of
+//    the input, so every tap is again a contiguous run of positions.  (A TMA box
+//    with a 16-byte inner extent moves one element per several cycles per SM and
+//    starved the tensor core; the LSU path moves 512 bytes per warp instruction.)
 //  * The int8 codes are NOT converted: a byte v <= 15 is the FP8 E4M3 encoding of
 //    v * 2^-9 (subnormal and first binade are linear), so the tensor core reads
 //    the codes in place and every product and sum is exact in the fp32
 //    accumulator; the epilogue multiplies by 2^9 (exact).
 //  * Weights are packed on the host as E4M3 of the signed integer codes in the
-//    same layout, and either stay resident in shared memory for the CTA's whole
-//    (group, output-block) unit or stream through a ring of (K block, tap) slices.
+//    same layout; warp 0 bulk-copies them (cp.async.bulk) so they either stay
+//    resident in shared memory for the CTA's whole (group, output-block) unit or
+//    stream through a ring of (K block, tap) slices.
 //  * warp 1 (one lane) issues tcgen05.mma kind::f8f6f4 (M = 128, N = the output
 //    block): for every tap the A operand is the same planes with the start
 //    address moved by the tap's position offset (16 bytes per position), so a
 //    3x3 convolution needs no im2col copy.  Accumulators live in tensor memory,
 //    double-buffered so the epilogue of tile i overlaps the MMAs of tile i+1.
-//  * warps 2-5 read the accumulators (tcgen05.ld), apply the rescale, shortcut,
+//  * warps 6-13 (two warpgroups, each taking half of the output columns) read the
+//    accumulators (tcgen05.ld), apply the rescale, shortcut,
 //    ReLU, output permutation and requantisation in registers, stage rows in
 //    shared memory and write them with coalesced 16-byte stores.
 //  * every wait is bounded (failure detection): a wait that runs out records
@@ -55,29 +58,58 @@ struct Ring {
   }
 };
 
+// Position in the CTA's contiguous range of work items, advanced without
+// divisions (64-bit divisions per item cost every role hundreds of cycles).
 struct Item {
-  int64_t unit, tile;
+  int64_t it;   // global item index
+  int unit;     // (group, output block) unit = g * NB + nb
+  int tile;     // tile within the unit
   int g, nb;
-  int n, oh0;   // rows mode
-  int64_t p0;   // flat mode
+  int n, rb;    // rows mode: image and row block (oh0 = rb * Ht)
+  int64_t p0;   // flat mode: first pixel
+  __device__ __forceinline__ int oh0(int Ht) const { return rb * Ht; }
 };
 
-__device__ __forceinline__ Item decode_item(const ConvParams& p, int64_t it) {
+__device__ __forceinline__ Item item_begin(const ConvParams& p, int64_t it) {
   Item r;
-  r.unit = it / p.tiles;
-  r.tile = it - r.unit * p.tiles;
-  r.g = static_cast<int>(r.unit / p.NB);
-  r.nb = static_cast<int>(r.unit - static_cast<int64_t>(r.g) * p.NB);
+  r.it = it;
+  const int64_t unit = it / p.tiles;
+  r.unit = static_cast<int>(unit);
+  r.tile = static_cast<int>(it - unit * p.tiles);
+  r.g = r.unit / p.NB;
+  r.nb = r.unit - r.g * p.NB;
   if (p.mode == kModeFlat) {
-    r.p0 = r.tile * p.flat_box;
     r.n = 0;
-    r.oh0 = 0;
+    r.rb = 0;
+    r.p0 = static_cast<int64_t>(r.tile) * p.flat_box;
   } else {
-    r.n = static_cast<int>(r.tile / p.tiles_per_img);
-    r.oh0 = static_cast<int>(r.tile - static_cast<int64_t>(r.n) * p.tiles_per_img) * p.Ht;
+    r.n = r.tile / p.tiles_per_img;
+    r.rb = r.tile - r.n * p.tiles_per_img;
     r.p0 = 0;
   }
   return r;
+}
+
+__device__ __forceinline__ void item_next(const ConvParams& p, Item& r) {
+  ++r.it;
+  if (++r.tile == p.tiles) {
+    r.tile = 0;
+    r.n = 0;
+    r.rb = 0;
+    r.p0 = 0;
+    if (++r.nb == p.NB) {
+      r.nb = 0;
+      ++r.g;
+    }
+    ++r.unit;
+    return;
+  }
+  if (p.mode == kModeFlat) {
+    r.p0 += p.flat_box;
+  } else if (++r.rb == p.tiles_per_img) {
+    r.rb = 0;
+    ++r.n;
+  }
 }
 
 // Shared-memory barrier block layout (64-bit words):
@@ -98,110 +130,247 @@ struct Bars {
 };
 
 // --------------------------------------------------------------------------
-// Copy role (warp 0, lane 0).
+// Weight copy role (warp 0, lane 0): bulk copies of the packed weights, either
+// once per (group, output-block) unit (resident) or one (K block, tap) slice at
+// a time through a ring.
 // --------------------------------------------------------------------------
-__device__ void producer_role(const ConvParams& p, const TensorMaps& tm, const Bars& bars, uint32_t a_base,
-                              uint32_t b_base, int64_t it0, int64_t it1, const WaitCtx& ctx) {
-  Ring ra{0, 0, static_cast<uint32_t>(p.a_stages)};
+__device__ __forceinline__ void weights_role(const ConvParams& p, const Bars& bars, uint32_t b_base, int64_t it0, int64_t it1,
+                             const WaitCtx& ctx) {
   Ring rb{0, 0, static_cast<uint32_t>(p.b_resident ? 1 : p.b_stages)};
-  int64_t a_issued = 0, b_issued = 0;
+  int64_t b_issued = 0;
   int64_t cur_unit = -1;
   bool ok = true;
-  for (int64_t it = it0; it < it1 && ok; ++it) {
-    const Item item = decode_item(p, it);
-    if (p.b_resident && item.unit != cur_unit) {
-      if (!mbar_wait(bars.b_empty(rb.stage), rb.phase ^ 1u, ctx)) { ok = false; break; }
+  Item item = item_begin(p, it0);
+  for (int64_t it = it0; it < it1 && ok; ++it, item_next(p, item)) {
+    const int64_t unit = item.unit;
+    if (p.b_resident) {
+      if (unit == cur_unit) continue;
+      if (!mbar_wait(bars.b_empty(rb.stage), rb.phase ^ 1u, ctx)) break;
       const uint32_t bar = bars.b_full(rb.stage);
       mbar_arrive_expect_tx(bar, p.b_unit_bytes);
-      const uint8_t* src = p.w_packed + static_cast<size_t>(item.unit) * p.b_unit_bytes;
-      // Copy in pieces of at most 64 KB.
-      for (uint32_t off = 0; off < p.b_unit_bytes; off += 65536u) {
-        const uint32_t len = min(65536u, p.b_unit_bytes - off);
-        bulk_load(b_base + off, src + off, len, bar);
-      }
+      const uint8_t* src = p.w_packed + static_cast<size_t>(unit) * p.b_unit_bytes;
+      for (uint32_t off = 0; off < p.b_unit_bytes; off += 65536u)
+        bulk_load(b_base + off, src + off, min(65536u, p.b_unit_bytes - off), bar);
       rb.advance();
       ++b_issued;
-      cur_unit = item.unit;
+      cur_unit = unit;
+      continue;
     }
-    for (int kb = 0; kb < p.n_kb; ++kb) {
-      if (!mbar_wait(bars.a_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
-      const uint32_t full = bars.a_full(ra.stage);
-      mbar_arrive_expect_tx(full, p.a_tx_bytes);
-      const uint32_t dst = a_base + ra.stage * p.a_stage_bytes;
-      const int chi = (item.g * p.Cin_g + kb * p.KC) >> 4;
-      if (p.mode == kModeFlat) {
-        tma_load_3d(dst, &tm.a[0], 0, static_cast<int>(item.p0), chi, full);
-      } else {
-        for (int ph = 0; ph < p.nph; ++ph)
-          tma_load_5d(dst + ph * p.a_phase_bytes, &tm.a[ph], 0, p.w_coord, item.oh0 + p.h_off, chi, item.n, full);
-      }
-      ra.advance();
-      ++a_issued;
-      if (!p.b_resident) {
-        for (int t = 0; t < p.taps; ++t) {
-          if (!mbar_wait(bars.b_empty(rb.stage), rb.phase ^ 1u, ctx)) { ok = false; break; }
-          const uint32_t bar = bars.b_full(rb.stage);
-          mbar_arrive_expect_tx(bar, p.b_slice_bytes);
-          const size_t slice = (static_cast<size_t>(item.unit) * p.n_kb + kb) * p.taps + t;
-          bulk_load(b_base + rb.stage * p.b_slice_bytes, p.w_packed + slice * p.b_slice_bytes, p.b_slice_bytes, bar);
-          rb.advance();
-          ++b_issued;
-        }
-        if (!ok) break;
+    for (int kb = 0; kb < p.n_kb && ok; ++kb) {
+      for (int t = 0; t < p.taps; ++t) {
+        if (!mbar_wait(bars.b_empty(rb.stage), rb.phase ^ 1u, ctx)) { ok = false; break; }
+        const uint32_t bar = bars.b_full(rb.stage);
+        mbar_arrive_expect_tx(bar, p.b_slice_bytes);
+        const size_t slice = (static_cast<size_t>(unit) * p.n_kb + kb) * p.taps + t;
+        bulk_load(b_base + rb.stage * p.b_slice_bytes, p.w_packed + slice * p.b_slice_bytes, p.b_slice_bytes, bar);
+        rb.advance();
+        ++b_issued;
       }
     }
   }
-  // Drain: the last min(stages, issued) copies of each ring may still be in flight.
-  const int64_t na = p.a_stages, nbs = p.b_resident ? 1 : p.b_stages;
-  for (int64_t k = (a_issued > na ? a_issued - na : 0); k < a_issued; ++k)
-    mbar_wait_drain(bars.a_full(static_cast<int>(k % na)), static_cast<uint32_t>((k / na) & 1), ctx.limit_ns, ctx.err);
+  // Drain: the last min(stages, issued) copies may still be in flight.
+  const int64_t nbs = p.b_resident ? 1 : p.b_stages;
   for (int64_t k = (b_issued > nbs ? b_issued - nbs : 0); k < b_issued; ++k)
     mbar_wait_drain(bars.b_full(static_cast<int>(k % nbs)), static_cast<uint32_t>((k / nbs) & 1), ctx.limit_ns, ctx.err);
 }
 
 // --------------------------------------------------------------------------
+// Activation copy role (warps 2-5): 16-byte cp.async copies of the codes a tile
+// needs into the tensor core's no-swizzle K-major layout.  For each stride phase
+// and each 16-byte chunk j of the K block's input channels there is a plane of
+// Hd x Wd positions (one 16-byte row per position); a position outside the image
+// is zero-filled (src-size 0), which is the zero padding.  Flat mode is one row
+// of flat_box positions.  The (position, chunk) pattern of a plane row is the same
+// for every row, so each thread precomputes its share once.  A thread releases a
+// stage after its copies have landed (wait_group) and a proxy fence, so the
+// tensor core (async proxy) sees the data; up to `depth` newer stages per thread
+// stay in flight meanwhile.
+// --------------------------------------------------------------------------
+constexpr int kLoaders = 32 * kLoadWarps;
+constexpr int kMaxLoadEntries = 8;
+
+__device__ __forceinline__ void load_release(const Bars& bars, int64_t k, int stages) {
+  fence_proxy_async_smem();
+  mbar_arrive(bars.a_full(static_cast<int>(k % stages)));
+}
+
+__device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bars, uint32_t a_base, int64_t it0, int64_t it1,
+                            const WaitCtx& ctx) {
+  const int tid = threadIdx.x - 32 * kFirstLoadWarp;
+  const bool flat = p.mode == kModeFlat;
+  const int nch = p.nch;
+  const uint32_t plane = p.lbo_a;
+  const int64_t C = p.C_in_total;
+  const int row_len = flat ? p.flat_box : p.Wd;
+  const int per_row = row_len * nch;
+  const bool tabled = per_row <= kMaxLoadEntries * kLoaders;
+  // This thread's (position, chunk) entries of one plane row.
+  uint32_t ent_dst[kMaxLoadEntries];
+  int ent_iw0[kMaxLoadEntries], ent_jo[kMaxLoadEntries];
+  int n_ent = 0;
+#pragma unroll
+  for (int i = 0; i < kMaxLoadEntries; ++i) {
+    const int e = tid + i * kLoaders;
+    ent_dst[i] = 0;
+    ent_iw0[i] = 0;
+    ent_jo[i] = 0;
+    if (tabled && e < per_row) {
+      const int w = static_cast<int>(__umulhi(static_cast<uint32_t>(e), p.nch_magic));
+      const int j = e - w * nch;
+      ent_dst[i] = static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(w) * 16u;
+      ent_iw0[i] = flat ? w : p.stride * (p.w_coord + w);
+      ent_jo[i] = j * 16;
+      n_ent = i + 1;
+    }
+  }
+  // Per-row values that depend on the stride phase, held in registers (a
+  // dynamically indexed kernel-parameter array costs a long-latency load).
+  const int pa0 = p.phase_a[0], pa1 = p.phase_a[1], pa2 = p.phase_a[2], pa3 = p.phase_a[3];
+  const int pb0 = p.phase_b[0], pb1 = p.phase_b[1], pb2 = p.phase_b[2], pb3 = p.phase_b[3];
+  const int depth = min(2, p.a_stages - 1);
+  Ring ra{0, 0, static_cast<uint32_t>(p.a_stages)};
+  int64_t issued = 0, released = 0;
+  bool ok = true;
+  const int nph = flat ? 1 : p.nph, Hd = flat ? 1 : p.Hd;
+  Item item = item_begin(p, it0);
+  for (int64_t it = it0; it < it1 && ok; ++it, item_next(p, item)) {
+    for (int kb = 0; kb < p.n_kb; ++kb) {
+      if (!mbar_wait(bars.a_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
+      const uint32_t stage = a_base + ra.stage * p.a_stage_bytes;
+      const int ch0 = item.g * p.Cin_g + kb * p.KC;  // first input channel of the K block
+      for (int ph = 0; ph < nph; ++ph)
+      for (int r = 0; r < Hd; ++r) {
+        bool row_ok;
+        const uint8_t* row_src;
+        uint32_t row_dst;
+        int b, w_lim;
+        if (flat) {
+          row_ok = true;
+          row_src = p.q_in + item.p0 * C + ch0;
+          row_dst = stage;
+          b = 0;
+          w_lim = static_cast<int>(min(p.P_out - item.p0, static_cast<int64_t>(p.flat_box)));
+        } else {
+          const int pa = ph == 0 ? pa0 : ph == 1 ? pa1 : ph == 2 ? pa2 : pa3;
+          const int ih = p.stride * (item.oh0(p.Ht) + p.h_off + r) + pa;
+          row_ok = ih >= 0 && ih < p.H;
+          row_src = p.q_in + ((static_cast<int64_t>(item.n) * p.H + (row_ok ? ih : 0)) * p.W) * C + ch0;
+          row_dst = stage + ph * p.a_phase_bytes + static_cast<uint32_t>(r * p.Wd) * 16u;
+          b = ph == 0 ? pb0 : ph == 1 ? pb1 : ph == 2 ? pb2 : pb3;
+          w_lim = p.W;
+        }
+        if (tabled) {
+#pragma unroll
+          for (int i = 0; i < kMaxLoadEntries; ++i) {
+            if (i < n_ent) {
+              const int iw = ent_iw0[i] + b;
+              const bool valid = row_ok && iw >= 0 && iw < w_lim;
+              cp_async_16(row_dst + ent_dst[i], valid ? row_src + static_cast<int64_t>(iw) * C + ent_jo[i] : p.q_in,
+                          valid ? 16u : 0u);
+            }
+          }
+        } else {
+          for (int e = tid; e < per_row; e += kLoaders) {
+            const int w = static_cast<int>(__umulhi(static_cast<uint32_t>(e), p.nch_magic));
+            const int j = e - w * nch;
+            const int iw = (flat ? w : p.stride * (p.w_coord + w)) + b;
+            const bool valid = row_ok && iw >= 0 && iw < w_lim;
+            cp_async_16(row_dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(w) * 16u,
+                        valid ? row_src + static_cast<int64_t>(iw) * C + j * 16 : p.q_in, valid ? 16u : 0u);
+          }
+        }
+      }
+      cp_async_commit();
+      ++issued;
+      ra.advance();
+      // Release the oldest stage once only `depth` newer ones may still be pending.
+      if (issued - released > depth) {
+        if (depth >= 2) cp_async_wait<2>();
+        else cp_async_wait<1>();
+        load_release(bars, released, p.a_stages);
+        ++released;
+      }
+    }
+  }
+  cp_async_wait<0>();
+  while (released < issued) {
+    load_release(bars, released, p.a_stages);
+    ++released;
+  }
+}
+
+// --------------------------------------------------------------------------
 // Tensor-core issue role (warp 1, lane 0).
 // --------------------------------------------------------------------------
-__device__ void mma_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t b_base, uint32_t tmem_base,
-                         int64_t it0, int64_t it1, const WaitCtx& ctx) {
+template <int KSTEPS, int MT>
+__device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t b_base,
+                                         uint32_t tmem_base, const uint32_t* tap_a16, int64_t it0, int64_t it1,
+                                         const WaitCtx& ctx) {
+  // The issue loop must stay lean: one thread issues every MMA and each extra
+  // instruction, branch or long-latency load per MMA lowers tensor-core
+  // throughput directly.  So the K steps and accumulators per tap are
+  // compile-time (fully unrolled), operand addresses are 32-bit adds of
+  // 16-byte-unit offsets onto the low word of precomputed descriptors
+  // (shared-memory addresses are below 2^18, so the 14-bit address field never
+  // carries), and the per-tap offsets come from shared memory.
   Ring ra{0, 0, static_cast<uint32_t>(p.a_stages)};
   Ring rb{0, 0, static_cast<uint32_t>(p.b_resident ? 1 : p.b_stages)};
   Ring racc{0, 0, static_cast<uint32_t>(p.acc_stages)};
   const uint32_t idesc = idesc_e4m3_f32(128, p.Nblk);
-  const int ksteps = p.nch >> 1;
-  int64_t cur_unit = -1;
+  const uint64_t a_desc0 = smem_desc(a_base, p.lbo_a, 128u);
+  const uint64_t b_desc0 = smem_desc(b_base, p.lbo_b, 128u);
+  const uint64_t a_hi = a_desc0 & 0xFFFFFFFF00000000ull, b_hi = b_desc0 & 0xFFFFFFFF00000000ull;
+  const uint32_t a_lo0 = static_cast<uint32_t>(a_desc0), b_lo0 = static_cast<uint32_t>(b_desc0);
+  const uint32_t a_ks16 = (2u * p.lbo_a) >> 4, b_ks16 = (2u * p.lbo_b) >> 4;  // one K step (32 bytes of K)
+  const uint32_t a_stage16 = p.a_stage_bytes >> 4, b_slice16 = p.b_slice_bytes >> 4;
+  const int taps = p.taps, n_kb = p.n_kb;
+  const uint32_t npow2 = static_cast<uint32_t>(p.Npow2);
+  const bool resident = p.b_resident != 0;
+  const int64_t tiles = p.tiles;
+  int unit = -1;
+  int tile = static_cast<int>(it0 % tiles);
+  int unit_next = static_cast<int>(it0 / tiles);
   bool ok = true;
   for (int64_t it = it0; it < it1 && ok; ++it) {
-    const int64_t unit = it / p.tiles;
-    if (p.b_resident && unit != cur_unit) {
+    const int cur = unit_next;
+    if (++tile == tiles) {
+      tile = 0;
+      ++unit_next;
+    }
+    if (resident && cur != unit) {
       if (!mbar_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
-      cur_unit = unit;
+      unit = cur;
     }
     if (!mbar_wait(bars.acc_empty(racc.stage), racc.phase ^ 1u, ctx)) { ok = false; break; }
     tc_fence_after();
-    const uint32_t d0 = tmem_base + racc.stage * p.MT * p.Npow2;
-    for (int kb = 0; kb < p.n_kb && ok; ++kb) {
+    const uint32_t d0 = tmem_base + racc.stage * static_cast<uint32_t>(MT) * npow2;
+    for (int kb = 0; kb < n_kb && ok; ++kb) {
       if (!mbar_wait(bars.a_full(ra.stage), ra.phase, ctx)) { ok = false; break; }
       tc_fence_after();
-      const uint32_t a_stage = a_base + ra.stage * p.a_stage_bytes;
-      for (int t = 0; t < p.taps; ++t) {
-        uint32_t bslice;
-        if (p.b_resident) {
-          bslice = b_base + (kb * p.taps + t) * p.b_slice_bytes;
+      const uint32_t a_lo_stage = a_lo0 + ra.stage * a_stage16;
+      uint32_t b_lo_slice = b_lo0 + static_cast<uint32_t>(kb * taps) * b_slice16;
+      for (int t = 0; t < taps; ++t) {
+        uint32_t b_lo_tap;
+        if (resident) {
+          b_lo_tap = b_lo_slice;
+          b_lo_slice += b_slice16;
         } else {
           if (!mbar_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
           tc_fence_after();
-          bslice = b_base + rb.stage * p.b_slice_bytes;
+          b_lo_tap = b_lo0 + rb.stage * b_slice16;
         }
-        const uint32_t a_tap = a_stage + p.tap_phase[t] * p.a_phase_bytes + static_cast<uint32_t>(p.tap_off[t]) * 16u;
-        for (int ks = 0; ks < ksteps; ++ks) {
-          const uint64_t bdesc = smem_desc(bslice + 2u * ks * p.lbo_b, p.lbo_b, 128u);
-          for (int mt = 0; mt < p.MT; ++mt) {
-            const uint64_t adesc = smem_desc(a_tap + mt * 2048u + 2u * ks * p.lbo_a, p.lbo_a, 128u);
-            tc_mma_e4m3(d0 + mt * p.Npow2, adesc, bdesc, idesc, (kb | t | ks) != 0 ? 1u : 0u);
-          }
+        const uint32_t a_lo_tap = a_lo_stage + tap_a16[t];
+        const uint32_t acc0 = (kb | t) == 0 ? 0u : 1u;
+#pragma unroll
+        for (int ks = 0; ks < KSTEPS; ++ks) {
+          const uint64_t bdesc = b_hi | (b_lo_tap + static_cast<uint32_t>(ks) * b_ks16);
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt)
+            tc_mma_e4m3(d0 + static_cast<uint32_t>(mt) * npow2,
+                        a_hi | (a_lo_tap + static_cast<uint32_t>(ks) * a_ks16 + static_cast<uint32_t>(mt) * 128u), bdesc,
+                        idesc, ks == 0 ? acc0 : 1u);
         }
-        if (!p.b_resident) {
+        if (!resident) {
           tc_commit(bars.b_empty(rb.stage));
           rb.advance();
         }
@@ -213,17 +382,33 @@ __device__ void mma_role(const ConvParams& p, const Bars& bars, uint32_t a_base,
     if (!ok) break;
     tc_commit(bars.acc_full(racc.stage));
     racc.advance();
-    if (p.b_resident) {
-      const int64_t next_unit = (it + 1 < it1) ? (it + 1) / p.tiles : -1;
-      if (next_unit != unit) {
-        tc_commit(bars.b_empty(rb.stage));
-        rb.advance();
-      }
+    if (resident && (it + 1 >= it1 || unit_next != cur)) {
+      tc_commit(bars.b_empty(rb.stage));
+      rb.advance();
     }
   }
   // Drain: wait until every MMA this thread issued has completed.
   tc_commit(bars.drain());
   mbar_wait_drain(bars.drain(), 0, ctx.limit_ns, ctx.err);
+}
+
+// Dispatch to the MMA role compiled for this layer's K steps per tap and
+// accumulators per tile.
+__device__ __forceinline__ void mma_role_dispatch(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t b_base,
+                                                  uint32_t tmem_base, const uint32_t* tap_a16, int64_t it0, int64_t it1,
+                                                  const WaitCtx& ctx) {
+  const int ks = p.nch >> 1;
+#define PQ_MMA_CASE(K, M) \
+  if (ks == K && p.MT == M) return mma_role<K, M>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1, ctx);
+  PQ_MMA_CASE(1, 1) PQ_MMA_CASE(1, 2) PQ_MMA_CASE(1, 4)
+  PQ_MMA_CASE(2, 1) PQ_MMA_CASE(2, 2) PQ_MMA_CASE(2, 4)
+  PQ_MMA_CASE(3, 1) PQ_MMA_CASE(3, 2) PQ_MMA_CASE(3, 4)
+  PQ_MMA_CASE(4, 1) PQ_MMA_CASE(4, 2) PQ_MMA_CASE(4, 4)
+  PQ_MMA_CASE(8, 1) PQ_MMA_CASE(8, 2) PQ_MMA_CASE(8, 4)
+#undef PQ_MMA_CASE
+  // The planner only produces the shapes above; anything else is a planner bug.
+  atomicOr(ctx.err, PQ_ERR_TIMEOUT | PQ_ERR_MMA);
+  *ctx.abort_flag = 1;
 }
 
 // --------------------------------------------------------------------------
@@ -245,23 +430,39 @@ __device__ __forceinline__ void warp_store_rows(const uint8_t* stg, uint32_t pit
   __syncwarp();
 }
 
-__device__ void epilogue_role(const ConvParams& p, const Bars& bars, uint32_t tmem_base, uint8_t* stage_base,
+// Requantised code of t = clamp(rint(t), 0, qmax) with round-half-to-even, on the
+// FMA and integer pipes: clamping t to [-1, qmax + 1] first does not change the
+// result (rounding is monotone and the final clamp is integral), and for
+// |r| < 2^22 the fp32 sum r + 1.5 * 2^23 is rounded by the adder to the nearest
+// integer, ties to even, which then sits in the low mantissa bits.  NaN -> 0.
+__device__ __forceinline__ int requant_code(float t, float qmax_f, int qmax) {
+  const float r = fminf(fmaxf(t, -1.0f), qmax_f + 1.0f);
+  int i = __float_as_int(__fadd_rn(r, 12582912.0f)) - 0x4B400000;
+  return min(max(i, 0), qmax);
+}
+
+constexpr int kSeg = 2;  // 16-column chunks per TMEM load batch
+
+__device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& bars, uint32_t tmem_base, uint8_t* stage_base,
                               int64_t it0, int64_t it1, const WaitCtx& ctx) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int quarter = warp & 3;  // TMEM lanes this warp may access
-  uint8_t* stg_q = stage_base + (warp - 2) * p.stage_warp_bytes;
-  uint8_t* stg_f = stg_q + 32 * p.stage_q_pitch;
+  const int ew = warp - kFirstEpiWarp;  // epilogue warp index
+  const int wg = ew >> 2;             // warpgroup: which share of the output columns
+  const int quarter = warp & 3;       // TMEM lanes this warp may access
+  uint8_t* stg = stage_base + ew * p.stage_warp_bytes;
   Ring racc{0, 0, static_cast<uint32_t>(p.acc_stages)};
   const int nchunks = p.Nblk >> 4;
-  const float qmax = static_cast<float>(p.qmax_out);
-  for (int64_t it = it0; it < it1; ++it) {
-    const Item item = decode_item(p, it);
+  const int c_begin = (wg * nchunks) / kEpiGroups, c_end = ((wg + 1) * nchunks) / kEpiGroups;
+  const int qmax = p.qmax_out;
+  const float qmax_f = static_cast<float>(qmax);
+  const bool has_sc = p.shortcut != nullptr;
+  Item item = item_begin(p, it0);
+  for (int64_t it = it0; it < it1; ++it, item_next(p, item)) {
     if (!mbar_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
     tc_fence_after();
     const int g = item.g;
-    const float m_out = p.m_out[g];
-    const float m_req = p.m_req[g];
-    const int src_c0 = g * p.Cout_g + item.nb * p.Nblk;          // source channel of column 0
+    const float m_out512 = p.m_out512[g], m_req512 = p.m_req512[g], m_req = p.m_req[g];
+    const int src_c0 = g * p.Cout_g + item.nb * p.Nblk;               // source channel of column 0
     const int dst_c0 = p.dst_group[g] * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
     for (int mt = 0; mt < p.MT; ++mt) {
       const int m = mt * 128 + quarter * 32 + lane;
@@ -273,98 +474,107 @@ __device__ void epilogue_role(const ConvParams& p, const Bars& bars, uint32_t tm
       } else {
         const int r = m / p.Wh;
         const int c = m - r * p.Wh;
-        const int oh = item.oh0 + r;
+        const int oh = item.oh0(p.Ht) + r;
         valid = (r < p.Ht) && (c < p.Wo) && (oh < p.Ho);
         pix = (static_cast<long long>(item.n) * p.Ho + oh) * p.Wo + c;
       }
       const long long row_elem = valid ? pix * p.C_out_total : -1;
       const uint32_t tcol = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2 +
                             mt * p.Npow2;
-      for (int ch = 0; ch < nchunks; ++ch) {
-        uint32_t v[16];
-        tmem_ld16(tcol + ch * 16, v);
-        tmem_wait_ld();
-        float accf[16];
+      for (int seg = c_begin; seg < c_end; seg += kSeg) {
+        const int nseg = min(kSeg, c_end - seg);
+        uint32_t v[kSeg][16];
 #pragma unroll
-        for (int j = 0; j < 16; ++j) accf[j] = __uint_as_float(v[j]) * 512.0f;  // exact: codes were read as v * 2^-9
-        float sc[16];
-        if (p.shortcut != nullptr) {
-          if (valid) {
-            const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + pix * p.C_out_total + src_c0 + ch * 16);
+        for (int s = 0; s < kSeg; ++s)
+          if (s < nseg) tmem_ld16(tcol + (seg + s) * 16, v[s]);
+        tmem_wait_ld();
+        uint32_t qw[kSeg][4];
+#pragma unroll
+        for (int s = 0; s < kSeg; ++s) {
+          if (s >= nseg) continue;
+          const int ch = seg + s;
+          if (!has_sc && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle) {
+            // Timed path: codes only, t = acc * m_req = raw * (m_req * 2^9).
 #pragma unroll
             for (int j = 0; j < 4; ++j) {
-              const float4 t = s4[j];
-              sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
+              const int a = requant_code(__fmul_rn(__uint_as_float(v[s][4 * j]), m_req512), qmax_f, qmax);
+              const int b = requant_code(__fmul_rn(__uint_as_float(v[s][4 * j + 1]), m_req512), qmax_f, qmax);
+              const int c = requant_code(__fmul_rn(__uint_as_float(v[s][4 * j + 2]), m_req512), qmax_f, qmax);
+              const int d = requant_code(__fmul_rn(__uint_as_float(v[s][4 * j + 3]), m_req512), qmax_f, qmax);
+              qw[s][j] = __byte_perm(__byte_perm(a, b, 0x0040), __byte_perm(c, d, 0x0040), 0x5410);
             }
-          } else {
-#pragma unroll
-            for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
+            continue;
           }
-        }
-        float y[16];
+          float sc[16];
+          if (has_sc) {
+            if (valid) {
+              const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + pix * p.C_out_total + src_c0 + ch * 16);
 #pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          float t = __fmul_rn(accf[j], m_out);
-          if (p.shortcut != nullptr) t = __fadd_rn(t, sc[j]);
-          if (p.relu) t = fmaxf(t, 0.0f);
-          y[j] = t;
-        }
-        if (p.channel_shuffle) {
-          // Per-channel scatter (destination channel co * G + g); rarely used, unstaged.
-          if (valid) {
+              for (int j = 0; j < 4; ++j) {
+                const float4 t = s4[j];
+                sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
+              }
+            } else {
 #pragma unroll
-            for (int j = 0; j < 16; ++j) {
-              const int co = item.nb * p.Nblk + ch * 16 + j;
-              const long long o = pix * p.C_out_total + static_cast<long long>(co) * p.G + g;
-              if (p.acc_out) p.acc_out[o] = __float2int_rn(accf[j]);
-              if (p.y_out) p.y_out[o] = y[j];
-              if (p.q_out) {
-                float r = rintf(__fmul_rn(p.shortcut != nullptr ? y[j] : accf[j], m_req));
-                r = fminf(fmaxf(r, 0.0f), qmax);
-                p.q_out[o] = static_cast<uint8_t>(static_cast<int>(r));
+              for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
+            }
+          }
+          float y[16];
+          int code[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j) {
+            const float raw = __uint_as_float(v[s][j]);
+            float t = __fmul_rn(raw, m_out512);  // = (float)acc * m_out, one rounding
+            if (has_sc) t = __fadd_rn(t, sc[j]);
+            if (p.relu) t = fmaxf(t, 0.0f);
+            y[j] = t;
+            code[j] = requant_code(has_sc ? __fmul_rn(t, m_req) : __fmul_rn(raw, m_req512), qmax_f, qmax);
+          }
+          if (p.channel_shuffle) {
+            // Per-channel scatter (destination channel co * G + g); rarely used, unstaged.
+            if (valid) {
+#pragma unroll
+              for (int j = 0; j < 16; ++j) {
+                const int co = item.nb * p.Nblk + ch * 16 + j;
+                const long long o = pix * p.C_out_total + static_cast<long long>(co) * p.G + g;
+                if (p.acc_out) p.acc_out[o] = __float2int_rn(__fmul_rn(__uint_as_float(v[s][j]), 512.0f));
+                if (p.y_out) p.y_out[o] = y[j];
+                if (p.q_out) p.q_out[o] = static_cast<uint8_t>(code[j]);
               }
             }
+            continue;
           }
-          continue;
-        }
-        if (p.acc_out) {
-          uint32_t* row = reinterpret_cast<uint32_t*>(stg_f + lane * p.stage_f_pitch);
+          if (p.acc_out) {
+            uint32_t* row = reinterpret_cast<uint32_t*>(stg + lane * p.stage_q_pitch);
 #pragma unroll
-          for (int j = 0; j < 16; j += 4)
-            *reinterpret_cast<uint4*>(row + j) =
-                make_uint4(__float2int_rn(accf[j]), __float2int_rn(accf[j + 1]), __float2int_rn(accf[j + 2]),
-                           __float2int_rn(accf[j + 3]));
-          warp_store_rows(stg_f, p.stage_f_pitch, 64, reinterpret_cast<uint8_t*>(p.acc_out),
-                          row_elem < 0 ? -1 : (row_elem + dst_c0 + ch * 16) * 4, lane);
-        }
-        if (p.y_out) {
-          float* row = reinterpret_cast<float*>(stg_f + lane * p.stage_f_pitch);
-#pragma unroll
-          for (int j = 0; j < 16; j += 4) *reinterpret_cast<float4*>(row + j) = make_float4(y[j], y[j + 1], y[j + 2], y[j + 3]);
-          warp_store_rows(stg_f, p.stage_f_pitch, 64, reinterpret_cast<uint8_t*>(p.y_out),
-                          row_elem < 0 ? -1 : (row_elem + dst_c0 + ch * 16) * 4, lane);
-        }
-        if (p.q_out) {
-          uint32_t w[4];
-#pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            uint32_t packed = 0;
-#pragma unroll
-            for (int b = 0; b < 4; ++b) {
-              const float src = p.shortcut != nullptr ? y[4 * j + b] : accf[4 * j + b];
-              float r = rintf(__fmul_rn(src, m_req));
-              r = fminf(fmaxf(r, 0.0f), qmax);
-              packed |= static_cast<uint32_t>(static_cast<int>(r)) << (8 * b);
-            }
-            w[j] = packed;
+            for (int j = 0; j < 16; j += 4)
+              *reinterpret_cast<int4*>(row + j) = make_int4(
+                  __float2int_rn(__fmul_rn(__uint_as_float(v[s][j]), 512.0f)),
+                  __float2int_rn(__fmul_rn(__uint_as_float(v[s][j + 1]), 512.0f)),
+                  __float2int_rn(__fmul_rn(__uint_as_float(v[s][j + 2]), 512.0f)),
+                  __float2int_rn(__fmul_rn(__uint_as_float(v[s][j + 3]), 512.0f)));
+            warp_store_rows(stg, p.stage_q_pitch, 64, reinterpret_cast<uint8_t*>(p.acc_out),
+                            row_elem < 0 ? -1 : (row_elem + dst_c0 + ch * 16) * 4, lane);
           }
-          *reinterpret_cast<uint4*>(stg_q + lane * p.stage_q_pitch + (ch & 3) * 16) = make_uint4(w[0], w[1], w[2], w[3]);
-          // Codes go out in segments of up to 64 channels (4 chunks) per row.
-          if ((ch & 3) == 3 || ch == nchunks - 1) {
-            const int seg0 = ch & ~3;
-            warp_store_rows(stg_q, p.stage_q_pitch, (ch - seg0 + 1) * 16, p.q_out,
-                            row_elem < 0 ? -1 : row_elem + dst_c0 + seg0 * 16, lane);
+          if (p.y_out) {
+            float* row = reinterpret_cast<float*>(stg + lane * p.stage_q_pitch);
+#pragma unroll
+            for (int j = 0; j < 16; j += 4) *reinterpret_cast<float4*>(row + j) = make_float4(y[j], y[j + 1], y[j + 2], y[j + 3]);
+            warp_store_rows(stg, p.stage_q_pitch, 64, reinterpret_cast<uint8_t*>(p.y_out),
+                            row_elem < 0 ? -1 : (row_elem + dst_c0 + ch * 16) * 4, lane);
           }
+#pragma unroll
+          for (int j = 0; j < 4; ++j)
+            qw[s][j] = __byte_perm(__byte_perm(code[4 * j], code[4 * j + 1], 0x0040),
+                                   __byte_perm(code[4 * j + 2], code[4 * j + 3], 0x0040), 0x5410);
+        }
+        if (p.q_out && !p.channel_shuffle) {
+          // Codes of this segment go out as one staged row each.
+#pragma unroll
+          for (int s = 0; s < kSeg; ++s)
+            if (s < nseg)
+              *reinterpret_cast<uint4*>(stg + lane * p.stage_q_pitch + s * 16) = make_uint4(qw[s][0], qw[s][1], qw[s][2], qw[s][3]);
+          warp_store_rows(stg, p.stage_q_pitch, nseg * 16, p.q_out, row_elem < 0 ? -1 : row_elem + dst_c0 + seg * 16, lane);
         }
       }
     }
@@ -376,8 +586,7 @@ __device__ void epilogue_role(const ConvParams& p, const Bars& bars, uint32_t tm
 
 }  // namespace
 
-__global__ void __launch_bounds__(kConvThreads, 1)
-    pq_conv_tc_kernel(const __grid_constant__ ConvParams p, const __grid_constant__ TensorMaps tm) {
+__global__ void __launch_bounds__(kConvThreads, 1) pq_conv_tc_kernel(const __grid_constant__ ConvParams p) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -388,10 +597,12 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   uint8_t* bar_block = gbase + p.smem_bar_off;
   volatile int* abort_flag = reinterpret_cast<volatile int*>(bar_block + 8 * bars.words());
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar_block + 8 * bars.words() + 8);
+  uint32_t* tap_a16 = reinterpret_cast<uint32_t*>(bar_block + 8 * bars.words() + 16);  // p.taps entries
+  for (int t = threadIdx.x; t < p.taps; t += blockDim.x) tap_a16[t] = p.tap_a16[t];
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < bars.A; ++s) {
-      mbar_init(bars.a_full(s), 1);
+      mbar_init(bars.a_full(s), 32 * kLoadWarps);
       mbar_init(bars.a_empty(s), 1);
     }
     for (int s = 0; s < bars.B; ++s) {
@@ -406,9 +617,6 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     *abort_flag = 0;
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) {
-    for (int ph = 0; ph < p.nph; ++ph) prefetch_tmap(&tm.a[ph]);
-  }
   if (warp == 1) tmem_alloc(smem_u32(tmem_slot), p.tmem_cols);
   tc_fence_before();
   __syncthreads();
@@ -421,10 +629,15 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   const uint32_t b_base = base + p.smem_b_off;
 
   if (warp == 0) {
-    if (lane == 0) producer_role(p, tm, bars, a_base, b_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
-  } else if (warp == 1) {
-    if (lane == 0) mma_role(p, bars, a_base, b_base, tmem_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_MMA});
+    if (lane == 0) weights_role(p, bars, b_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
     __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0)
+      mma_role_dispatch(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1,
+                        WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_MMA});
+    __syncwarp();
+  } else if (warp < kFirstEpiWarp) {
+    loader_role(p, bars, a_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else {
     epilogue_role(p, bars, tmem_base, gbase + p.smem_stage_off, it0, it1,
                   WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_EPILOGUE});
@@ -437,7 +650,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   }
 }
 
-int launch_conv_tc(const ConvParams& p, const TensorMaps& tm, int grid, cudaStream_t stream) {
+int launch_conv_tc(const ConvParams& p, int grid, cudaStream_t stream) {
   static int attr_set_for_device[64] = {0};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return -1;
@@ -447,7 +660,7 @@ int launch_conv_tc(const ConvParams& p, const TensorMaps& tm, int grid, cudaStre
       return -1;
     attr_set_for_device[dev] = kMaxSmem;
   }
-  pq_conv_tc_kernel<<<grid, kConvThreads, need, stream>>>(p, tm);
+  pq_conv_tc_kernel<<<grid, kConvThreads, need, stream>>>(p);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }
 

@@ -1,5 +1,5 @@
-// Device-side building blocks for sm_103a: mbarriers with bounded waits, TMA and
-// bulk copies into shared memory, and the tcgen05 (5th-generation tensor core)
+// Device-side building blocks for sm_103a: mbarriers with bounded waits, bulk and
+// 16-byte asynchronous copies into shared memory, and the tcgen05 (5th-generation tensor core)
 // operations used by the PalQuant kernels.  All inline PTX is written here; the
 // kernels call these helpers only.
 #pragma once
@@ -59,18 +59,25 @@ struct WaitCtx {
   unsigned int err_bits;     // bits recorded by this role on timeout
 };
 
+// Wait limits are kept in SM clock cycles: the cycle counter costs a few cycles
+// to read, while %globaltimer reads cost on the order of a microsecond, which
+// stalled every role of the pipeline when read on each blocking wait.  The
+// conversion assumes 2.5 cycles per ns, above the highest SM clock (2.07 GHz),
+// so a limit never ends earlier than asked.
+__device__ __forceinline__ uint64_t limit_cycles(uint64_t limit_ns) { return limit_ns * 5u / 2u; }
+
 // Wait until the phase with the given parity of `bar` has completed.  Returns
 // false (after recording PQ_ERR_TIMEOUT and raising the abort flag) when the
 // wait exceeds ctx.limit_ns, or when another role of the CTA already aborted.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtx& ctx) {
   if (mbar_try_wait(bar, parity)) return true;
-  uint64_t t0 = global_timer_ns();
+  const long long t0 = clock64();
   uint32_t n = 0;
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((++n & 63u) == 0) {
       if (*ctx.abort_flag) return false;
-      if (global_timer_ns() - t0 > ctx.limit_ns) {
+      if (static_cast<uint64_t>(clock64() - t0) > limit_cycles(ctx.limit_ns)) {
         atomicOr(ctx.err, PQ_ERR_TIMEOUT | ctx.err_bits);
         *ctx.abort_flag = 1;
         return false;
@@ -81,10 +88,10 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const W
 
 // Bounded wait that ignores the abort flag (teardown: drain what is in flight).
 __device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity, uint64_t limit_ns, unsigned int* err) {
-  uint64_t t0 = global_timer_ns();
+  const long long t0 = clock64();
   uint32_t n = 0;
   while (!mbar_try_wait(bar, parity)) {
-    if ((++n & 63u) == 0 && global_timer_ns() - t0 > limit_ns) {
+    if ((++n & 63u) == 0 && static_cast<uint64_t>(clock64() - t0) > limit_cycles(limit_ns)) {
       atomicOr(err, PQ_ERR_TIMEOUT | PQ_ERR_TEARDOWN);
       return false;
     }
@@ -94,25 +101,9 @@ __device__ __forceinline__ bool mbar_wait_drain(uint32_t bar, uint32_t parity, u
 
 // ------------------------------------------------------------ async copies
 // Order this thread's generic-proxy shared-memory accesses before later
-// async-proxy (TMA / tensor core) accesses.
+// async-proxy (bulk copy / tensor core) accesses.
 __device__ __forceinline__ void fence_proxy_async_smem() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-}
-
-// Tiled TMA loads (global -> shared), completion counted on `bar` in bytes.
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const void* tmap, int c0, int c1, int c2, uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
-      : "memory");
-}
-
-__device__ __forceinline__ void tma_load_5d(uint32_t dst, const void* tmap, int c0, int c1, int c2, int c3, int c4,
-                                            uint32_t bar) {
-  asm volatile(
-      "cp.async.bulk.tensor.5d.shared::cluster.global.tile.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3, %4, %5, %6}], [%7];" ::"r"(dst),
-      "l"(reinterpret_cast<uint64_t>(tmap)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(c4), "r"(bar)
-      : "memory");
 }
 
 // Plain bulk copy of `bytes` (multiple of 16, both addresses 16-byte aligned).
@@ -122,8 +113,20 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
                : "memory");
 }
 
-__device__ __forceinline__ void prefetch_tmap(const void* tmap) {
-  asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(tmap)) : "memory");
+// 16-byte asynchronous copy global -> shared through the LSU path; src_bytes = 0
+// writes 16 zero bytes and reads nothing.
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(reinterpret_cast<uint64_t>(src)),
+               "r"(src_bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+
+// Wait until at most N of this thread's most recent copy groups are pending.
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
 // ------------------------------------------------------------------ tcgen05

@@ -2,7 +2,7 @@
 // Not part of the public ABI (see include/palquant.h).
 #pragma once
 
-#include <cuda.h>
+#include <cuda_runtime.h>
 #include <cstdint>
 
 // Bits of the device error word.
@@ -18,16 +18,15 @@ namespace pq {
 constexpr int kMaxG = 64;
 constexpr int kMaxTaps = 49;
 constexpr int kMaxPhases = 4;
-constexpr int kConvThreads = 192;  // warp 0: copies, warp 1: MMA issue + TMEM, warps 2-5: epilogue
-constexpr int kEpiWarps = 4;
+constexpr int kEpiGroups = 2;                      // epilogue warpgroups, splitting the output columns
+constexpr int kEpiWarps = 4 * kEpiGroups;
+constexpr int kLoadWarps = 4;                      // activation-operand copy warps
+constexpr int kFirstLoadWarp = 2;
+constexpr int kFirstEpiWarp = kFirstLoadWarp + kLoadWarps;
+constexpr int kConvThreads = 32 * (kFirstEpiWarp + kEpiWarps);  // warp 0 weights, 1 MMA, 2-5 loads, 6-13 epilogue
 constexpr int kMaxSmem = 227 * 1024;
 
 enum ConvMode : int { kModeFlat = 0, kModeRows = 1 };
-
-// Tensor maps of the activation operand, one per stride phase.
-struct TensorMaps {
-  CUtensorMap a[kMaxPhases];
-};
 
 // Everything the tensor-core conv kernel needs; filled by the host planner.
 struct ConvParams {
@@ -38,9 +37,13 @@ struct ConvParams {
   int G, Cin_g, Cout_g;
   int Ht;                 // output rows per tile (rows mode)
   int Wh;                 // positions per tile row in the operand planes
-  int Hd, Wd;             // box rows / columns loaded per phase
-  int h_off;              // TMA row coordinate = oh0 + h_off (phase rows)
-  int w_coord;            // TMA column coordinate (phase columns)
+  int Hd, Wd;             // plane rows / columns loaded per phase
+  int h_off;              // first plane row = phase row oh0 + h_off
+  int w_coord;            // first plane column = phase column w_coord
+  int H, W, stride;       // input geometry
+  int C_in_total;         // G * Cin_g (bytes per input pixel)
+  int phase_a[kMaxPhases], phase_b[kMaxPhases];  // stride phase (row, column) of each plane set
+  uint32_t nch_magic;     // ceil(2^32 / nch): e / nch = umulhi(e, nch_magic) for small e
   int tiles_per_img;      // rows mode
   int64_t tiles;          // tiles per (group, n-block) unit
   int64_t items;          // tiles * G * NB
@@ -48,11 +51,12 @@ struct ConvParams {
   int MT;                 // 128-row accumulators per tile
   int KC, n_kb, nch;      // channels per K block, K blocks, 16-byte chunks per K block
   int taps, nph;          // kh*kw, stride phases
-  int flat_box;           // pixels per flat-mode box (= MT * 128)
+  int flat_box;           // pixels per flat-mode tile (= MT * 128)
   int tap_phase[kMaxTaps];
   int tap_off[kMaxTaps];  // position offset of each tap in the plane
+  uint32_t tap_a16[kMaxTaps];  // stage-relative start of each tap's A operand, in 16-byte units
   uint32_t lbo_a;         // byte stride between 16-byte K chunks of the A planes
-  uint32_t a_phase_bytes, a_stage_bytes, a_tx_bytes;
+  uint32_t a_phase_bytes, a_stage_bytes;
   int a_stages;
   int b_resident;         // 1: the whole unit's weights stay in shared memory
   uint32_t b_slice_bytes; // one (K block, tap) slice: KC * Nblk bytes
@@ -64,11 +68,14 @@ struct ConvParams {
   uint32_t smem_b_off, smem_stage_off, smem_bar_off, smem_bytes;
   uint32_t stage_q_pitch, stage_f_pitch, stage_warp_bytes;
   // ---- operands
+  const uint8_t* q_in;    // activation codes, NHWC
   const uint8_t* w_packed;
   // ---- epilogue
   int C_out_total;        // G * Cout_g
-  float m_out[kMaxG];
-  float m_req[kMaxG];
+  float m_out[kMaxG];     // as given: y = (float)acc * m_out
+  float m_req[kMaxG];     // as given: applied to the shortcut sum
+  float m_out512[kMaxG];  // m_out * 2^9 (exact): applied to the raw accumulator, which holds acc * 2^-9
+  float m_req512[kMaxG];  // m_req * 2^9 (exact)
   int dst_group[kMaxG];
   int channel_shuffle;    // 1: destination channel co*G + g (per-channel scatter)
   int relu;
@@ -83,7 +90,7 @@ struct ConvParams {
 };
 
 // Host-side launch helpers implemented in the .cu files.
-int launch_conv_tc(const ConvParams& p, const TensorMaps& tm, int grid, cudaStream_t stream);
+int launch_conv_tc(const ConvParams& p, int grid, cudaStream_t stream);
 int launch_quantize(const float* x, uint8_t* q, int64_t P, int G, int Cg, int bits, const float* inv_s,
                     cudaStream_t stream);
 int launch_act_sum(const float* x, int64_t P, int G, int Cg, double* partial, int nblocks, cudaStream_t stream);
