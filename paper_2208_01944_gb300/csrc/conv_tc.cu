@@ -302,6 +302,8 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
 // --------------------------------------------------------------------------
 // Tensor-core issue role (warp 1, lane 0).
 // --------------------------------------------------------------------------
+constexpr int kUnrollTaps = 9;
+
 template <int KSTEPS, int MT>
 __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t b_base,
                                          uint32_t tmem_base, const uint32_t* tap_a16, int64_t it0, int64_t it1,
@@ -327,6 +329,9 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
   const uint32_t npow2 = static_cast<uint32_t>(p.Npow2);
   const bool resident = p.b_resident != 0;
   const int64_t tiles = p.tiles;
+  uint32_t tap_reg[kUnrollTaps];
+#pragma unroll
+  for (int t = 0; t < kUnrollTaps; ++t) tap_reg[t] = t < taps ? tap_a16[t] : 0u;
   int unit = -1;
   int tile = static_cast<int>(it0 % tiles);
   int unit_next = static_cast<int>(it0 / tiles);
@@ -348,18 +353,9 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
       if (!mbar_wait(bars.a_full(ra.stage), ra.phase, ctx)) { ok = false; break; }
       tc_fence_after();
       const uint32_t a_lo_stage = a_lo0 + ra.stage * a_stage16;
-      uint32_t b_lo_slice = b_lo0 + static_cast<uint32_t>(kb * taps) * b_slice16;
-      for (int t = 0; t < taps; ++t) {
-        uint32_t b_lo_tap;
-        if (resident) {
-          b_lo_tap = b_lo_slice;
-          b_lo_slice += b_slice16;
-        } else {
-          if (!mbar_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
-          tc_fence_after();
-          b_lo_tap = b_lo0 + rb.stage * b_slice16;
-        }
-        const uint32_t a_lo_tap = a_lo_stage + tap_a16[t];
+      const uint32_t b_lo_kb = b_lo0 + static_cast<uint32_t>(kb * taps) * b_slice16;
+      // One tap: KSTEPS x MT MMAs, fully unrolled.
+      auto issue_tap = [&](int t, uint32_t a_lo_tap, uint32_t b_lo_tap) {
         const uint32_t acc0 = (kb | t) == 0 ? 0u : 1u;
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
@@ -370,9 +366,28 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
                         a_hi | (a_lo_tap + static_cast<uint32_t>(ks) * a_ks16 + static_cast<uint32_t>(mt) * 128u), bdesc,
                         idesc, ks == 0 ? acc0 : 1u);
         }
-        if (!resident) {
-          tc_commit(bars.b_empty(rb.stage));
-          rb.advance();
+      };
+      if (resident && taps <= kUnrollTaps) {
+        // Up to 9 taps unrolled with their offsets in registers: no loads or
+        // loop branches between the MMAs of a K block.
+#pragma unroll
+        for (int t = 0; t < kUnrollTaps; ++t)
+          if (t < taps) issue_tap(t, a_lo_stage + tap_reg[t], b_lo_kb + static_cast<uint32_t>(t) * b_slice16);
+      } else {
+        for (int t = 0; t < taps; ++t) {
+          uint32_t b_lo_tap;
+          if (resident) {
+            b_lo_tap = b_lo_kb + static_cast<uint32_t>(t) * b_slice16;
+          } else {
+            if (!mbar_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
+            tc_fence_after();
+            b_lo_tap = b_lo0 + rb.stage * b_slice16;
+          }
+          issue_tap(t, a_lo_stage + tap_a16[t], b_lo_tap);
+          if (!resident) {
+            tc_commit(bars.b_empty(rb.stage));
+            rb.advance();
+          }
         }
       }
       if (!ok) break;
@@ -456,6 +471,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
   const int qmax = p.qmax_out;
   const float qmax_f = static_cast<float>(qmax);
   const bool has_sc = p.shortcut != nullptr;
+  const bool codes_only = !has_sc && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle;
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1; ++it, item_next(p, item)) {
     if (!mbar_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
@@ -493,16 +509,26 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         for (int s = 0; s < kSeg; ++s) {
           if (s >= nseg) continue;
           const int ch = seg + s;
-          if (!has_sc && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle) {
-            // Timed path: codes only, t = acc * m_req = raw * (m_req * 2^9).
+          if (codes_only) {
+            // Timed path, codes only: t = acc * m_req = raw * (m_req * 2^9),
+            // clamped to [0, Qp] in fp32 (NaN -> 0), then rounded half to even by
+            // adding 1.5 * 2^23, which leaves the code in the sum's low byte.
+            uint32_t bits[16];
 #pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const int a = requant_code(__fmul_rn(__uint_as_float(v[s][4 * j]), m_req512), qmax_f, qmax);
-              const int b = requant_code(__fmul_rn(__uint_as_float(v[s][4 * j + 1]), m_req512), qmax_f, qmax);
-              const int c = requant_code(__fmul_rn(__uint_as_float(v[s][4 * j + 2]), m_req512), qmax_f, qmax);
-              const int d = requant_code(__fmul_rn(__uint_as_float(v[s][4 * j + 3]), m_req512), qmax_f, qmax);
-              qw[s][j] = __byte_perm(__byte_perm(a, b, 0x0040), __byte_perm(c, d, 0x0040), 0x5410);
+            for (int j = 0; j < 16; j += 2) {
+              float t0, t1;
+              mul2_rn(__uint_as_float(v[s][j]), __uint_as_float(v[s][j + 1]), m_req512, t0, t1);
+              t0 = fminf(fmaxf(t0, 0.0f), qmax_f);
+              t1 = fminf(fmaxf(t1, 0.0f), qmax_f);
+              float r0, r1;
+              add2_rn(t0, t1, 12582912.0f, r0, r1);
+              bits[j] = __float_as_uint(r0);
+              bits[j + 1] = __float_as_uint(r1);
             }
+#pragma unroll
+            for (int j = 0; j < 4; ++j)
+              qw[s][j] = __byte_perm(__byte_perm(bits[4 * j], bits[4 * j + 1], 0x0040),
+                                     __byte_perm(bits[4 * j + 2], bits[4 * j + 3], 0x0040), 0x5410);
             continue;
           }
           float sc[16];

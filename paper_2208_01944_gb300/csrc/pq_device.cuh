@@ -129,6 +129,21 @@ __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
 
+// ------------------------------------------------------------ packed fp32
+// Two IEEE fp32 round-to-nearest multiplies / adds in one instruction
+// (sm_100+ f32x2 arithmetic); lane-wise identical to __fmul_rn / __fadd_rn.
+__device__ __forceinline__ void mul2_rn(float a, float b, float m, float& x, float& y) {
+  asm("{\n.reg .b64 s, t, r;\nmov.b64 s, {%2, %3};\nmov.b64 t, {%4, %4};\nmul.rn.f32x2 r, s, t;\nmov.b64 {%0, %1}, r;\n}"
+      : "=f"(x), "=f"(y)
+      : "f"(a), "f"(b), "f"(m));
+}
+
+__device__ __forceinline__ void add2_rn(float a, float b, float m, float& x, float& y) {
+  asm("{\n.reg .b64 s, t, r;\nmov.b64 s, {%2, %3};\nmov.b64 t, {%4, %4};\nadd.rn.f32x2 r, s, t;\nmov.b64 {%0, %1}, r;\n}"
+      : "=f"(x), "=f"(y)
+      : "f"(a), "f"(b), "f"(m));
+}
+
 // ------------------------------------------------------------------ tcgen05
 // Shared-memory matrix descriptor, no swizzle, K-major: core matrices of
 // 8 rows x 16 bytes; `lbo` = byte distance between core matrices adjacent in K,

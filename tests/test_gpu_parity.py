@@ -198,3 +198,34 @@ def test_watchdog_times_out_and_context_survives(B):
     c = Case(1, 6, 6, 2, 32, 32, 3, 1, 1, seed=30)
     ref = prepare(c)
     assert_layer_parity(c, ref, run_gpu(c, ref))                      # the context still works
+
+
+# ------------------------------------------- codes-only path (the timed one)
+CODES_ONLY = [
+    Case(2, 13, 11, 3, 32, 48, 3, 1, 1, seed=40),
+    Case(1, 12, 12, 2, 128, 256, 3, 1, 1, bits=4, seed=41),
+    Case(2, 7, 9, 4, 96, 96, 1, 1, 0, seed=42),
+    Case(3, 9, 17, 4, 64, 64, 3, 2, 1, seed=43),
+]
+
+
+@pytest.mark.parametrize("c", CODES_ONLY, ids=str)
+def test_layer_codes_only_matches_oracle(B, c):
+    ref = prepare(c)
+    got = run_gpu(c, ref, outputs=("q",))
+    assert_layer_parity(c, ref, got)
+
+
+@pytest.mark.parametrize("mult", [0.5, 0.25, 1.0 / 3.0])
+def test_requant_ties_round_half_even(B, mult):
+    """Multipliers that put many products exactly on .5: ties must round to even."""
+    c = Case(2, 10, 10, 2, 64, 64, 3, 1, 1, bits=4, seed=44)
+    ref = prepare(c)
+    m_req = np.full(c.G, mult, dtype=np.float32)
+    acc = oracle.group_conv(ref["q"], ref["wq"], c.stride, c.pad).reshape(-1, c.G * c.Cout)
+    _, _, q_ref = oracle.epilogue(acc, c.G, ref["m_out"], m_req, c.kind, c.shift, None, None, True, 4)
+    ref = dict(ref, m_req=m_req, q_ref=q_ref)
+    got = run_gpu(c, ref, outputs=("q",))
+    assert np.array_equal(got["q_out"], q_ref)
+    if mult == 0.5:
+        assert np.any((acc % 2 == 1) & (acc > 0)), "the case must contain ties"
