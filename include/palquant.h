@@ -120,6 +120,22 @@ pq_status palquant_act_steps(const float* x_dev, int64_t N, int32_t H, int32_t W
                              int32_t bits, void* scratch_dev, size_t scratch_bytes, float* s_out_host,
                              pq_stream_t stream);
 
+/* The same per-group activation steps as palquant_act_steps, for callers that
+ * cannot allocate device memory (for example code whose device memory is owned
+ * by a host framework, or a path whose memory budget is fixed in advance).  The
+ * paper has no counterpart: this is a deployment convenience.
+ *
+ * It allocates nothing.  Its scratch is a fixed array of 131,584 bytes in the
+ * library's own device memory (held by every GPU that loads the library until
+ * the process exits), which bounds the group count: G <= 64, else
+ * PQ_EUNSUPPORTED.  The first call on a device looks up that array's device
+ * address (make it before any stream capture).  All calls share the array and
+ * overwrite what they read, so calls that run on the GPU at the same time race
+ * and must be serialised by the caller.  Results are identical to
+ * palquant_act_steps for the same input.  Synchronises the stream. */
+pq_status palquant_act_steps_noalloc(const float* x_dev, int64_t N, int32_t H, int32_t W, int32_t G, int32_t Cg,
+                                     int32_t bits, float* s_out_host, pq_stream_t stream);
+
 /* Per-group weight step s_w[g] = 2 mean|w_g| / sqrt(2^(bits-1) - 1) (LSQ), mean
  * in double over the group's weights; w_host is [G][Cout_g][kh][kw][Cin_g].
  * Host only.  s_w_out_host receives G floats. */

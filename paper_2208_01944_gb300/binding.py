@@ -23,6 +23,7 @@ PQ_CODES_INT8, PQ_CODES_E4M3 = 0, 1
 # Every symbol include/palquant.h declares.
 EXPORTS = [
     "palquant_strerror", "palquant_version", "palquant_act_steps_scratch_bytes", "palquant_act_steps",
+    "palquant_act_steps_noalloc",
     "palquant_weight_steps", "palquant_epilogue_scales", "palquant_packed_weight_bytes",
     "palquant_pack_weights_host", "palquant_pack_weights", "palquant_pack_weight_codes_host",
     "palquant_unpack_weight_codes_host", "palquant_quantize_act", "palquant_group_conv", "palquant_layer_fused",
@@ -72,6 +73,8 @@ def _load():
     L.palquant_act_steps_scratch_bytes.argtypes = [_I64, _I32]
     L.palquant_act_steps.restype = _I32
     L.palquant_act_steps.argtypes = [_P, _I64, _I32, _I32, _I32, _I32, _I32, _P, ctypes.c_size_t, _P, _P]
+    L.palquant_act_steps_noalloc.restype = _I32
+    L.palquant_act_steps_noalloc.argtypes = [_P, _I64, _I32, _I32, _I32, _I32, _I32, _P, _P]
     L.palquant_weight_steps.restype = _I32
     L.palquant_weight_steps.argtypes = [_P, ctypes.POINTER(LayerDesc), _P]
     L.palquant_epilogue_scales.restype = _I32
@@ -172,6 +175,14 @@ def palquant_act_steps(x_dev, N, H, W, G, Cg, bits, scratch_dev, scratch_bytes, 
     out = np.empty(G, dtype=np.float32)
     _check(lib.palquant_act_steps(_ptr(x_dev), N, H, W, G, Cg, bits, _ptr(scratch_dev), scratch_bytes, _ptr(out),
                                   _stream(stream)), "palquant_act_steps")
+    return out
+
+
+def palquant_act_steps_noalloc(x_dev, N, H, W, G, Cg, bits, stream=None) -> np.ndarray:
+    """Per-group activation steps without any device allocation (fixed library scratch)."""
+    out = np.empty(G, dtype=np.float32)
+    _check(lib.palquant_act_steps_noalloc(_ptr(x_dev), N, H, W, G, Cg, bits, _ptr(out), _stream(stream)),
+           "palquant_act_steps_noalloc")
     return out
 
 
