@@ -42,7 +42,34 @@ def parse():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline sample")
+    ap.add_argument("--profile-layer", default=None, metavar="CONFIG",
+                    help="only run the fused layer of CONFIG (config0, config1, config3_0..4, config4) --reps times "
+                         "on random codes (codes out), for profilers; prints nothing else")
+    ap.add_argument("--reps", type=int, default=3)
     return ap.parse_args()
+
+
+def run_profile_layer(name: str, reps: int):
+    """The fused layer alone, for profiling: random codes and weights of the named workload."""
+    import numpy as np
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300 import synth, workloads
+
+    c = workloads.BENCH_CONFIGS[name]
+    dev = torch.device("cuda:0")
+    gen = synth.generator(0)
+    q = torch.from_numpy(synth.random_codes((c.N, c.H, c.W, c.G * c.Cin_g), c.bits_a, gen)).to(dev)
+    wq = synth.random_codes((c.G, c.Cout_g, c.k, c.k, c.Cin_g), c.bits_w, gen, signed=True)
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out)
+    wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).to(dev)
+    qo = torch.empty((c.N, c.Ho, c.Wo, c.G * c.Cout_g), dtype=torch.uint8, device=dev)
+    m = np.full(c.G, 0.01, np.float32)
+    for _ in range(reps):
+        B.palquant_layer_fused(q, wp, d, m, m, B.shuffle(c.shuffle_kind, c.shuffle_shift), None, None, None, qo)
+    st = B.palquant_sync_check()
+    assert st == B.PQ_OK, B.strerror(st)
 
 
 def peaks():
@@ -365,6 +392,9 @@ def main():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.profile_layer:
+        run_profile_layer(args.profile_layer, args.reps)
+        return
     if args.impl == "reference":
         run_reference(args, rank, world)
         return
