@@ -23,9 +23,8 @@
  *    [G][Cout_g][kh][kw][Cin_g].
  *  - Codes.  One code per byte.  Activation codes are unsigned integers in
  *    [0, 2^bits - 1]; weight codes are signed in [-2^(bits-1), 2^(bits-1) - 1].
- *    A code tensor is stored either as plain integers (PQ_CODES_INT8) or as the
- *    FP8 E4M3 encoding of the same integer (PQ_CODES_E4M3), which the tensor
- *    cores read directly; both encodings represent every code exactly.
+ *    An activation code tensor is either NHWC (PQ_CODES_INT8) or channel-blocked
+ *    (PQ_CODES_C16, see pq_code_format); both hold the same integer values.
  *  - Memory.  The caller owns every buffer.  Pointers named *_dev are device
  *    pointers, *_host are host pointers.  The compute calls allocate nothing;
  *    small host arrays (per-group scalars, permutations) are copied into the
@@ -61,8 +60,12 @@ typedef enum {
 } pq_status;
 
 typedef enum {
-    PQ_CODES_INT8 = 0, /* code v stored as the byte v (two's complement for weights) */
-    PQ_CODES_E4M3 = 1  /* code v stored as the FP8 E4M3 encoding of v */
+    PQ_CODES_INT8 = 0, /* code v stored as the byte v, NHWC: byte (((n*H + h)*W + w)*C + c) */
+    PQ_CODES_E4M3 = 1, /* reserved (PQ_EUNSUPPORTED) */
+    PQ_CODES_C16 = 2   /* code v stored as the byte v, channel-blocked in 16-channel blocks:
+                          byte ((((n*(C/16) + c/16)*H + h)*W + w)*16 + c%16).  C % 16 == 0.
+                          The tensor cores' operand layout: every run of positions of one
+                          16-channel block is contiguous.  The fastest format. */
 } pq_code_format;
 
 /* Output channel permutation (Sec. 4.2).  kind:
@@ -92,7 +95,7 @@ typedef struct {
     int32_t bits_w;      /* weight code bits, 2..4 */
     int32_t bits_out;    /* requantised output code bits, 1..4 */
     int32_t relu;        /* 1: ReLU after the rescale (and the shortcut add) */
-    int32_t code_format; /* pq_code_format of input codes and output codes */
+    int32_t code_format; /* pq_code_format (INT8 or C16) of the input codes and the output codes */
 } pq_layer_desc;
 
 /* Human-readable name of a status. */
@@ -187,9 +190,9 @@ pq_status palquant_unpack_weight_codes_host(const void* packed_host, const pq_la
  * fp32 multiply, round half to even, clamp):
  *   q[p, g*Cg + j] = clamp(rint(x[p, g*Cg + j] * inv_s[g]), 0, 2^bits - 1)
  * x_dev is NHWC fp32 [N,H,W,G*Cg]; q_dev receives one byte per element in
- * code_format.  inv_s_host holds G floats (fl(1/s) of the steps), copied at call
- * time.  NaN maps to 0 and +inf to 2^bits - 1.  bits in 1..8 for PQ_CODES_INT8,
- * 1..4 for PQ_CODES_E4M3. */
+ * code_format (PQ_CODES_INT8: NHWC; PQ_CODES_C16: channel-blocked, needs
+ * Cg % 16 == 0).  inv_s_host holds G floats (fl(1/s) of the steps), copied at
+ * call time.  NaN maps to 0 and +inf to 2^bits - 1.  bits in 1..8. */
 pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G,
                                 int32_t Cg, int32_t bits, int32_t code_format, const float* inv_s_host,
                                 pq_stream_t stream);

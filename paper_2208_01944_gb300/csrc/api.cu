@@ -2,6 +2,7 @@
 // tensor-core convolution, weight quantisation and packing, tensor-map encoding,
 // launches and error reporting.  Every entry point of include/palquant.h is
 // defined here.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -86,7 +87,8 @@ pq_status validate_desc(const pq_layer_desc* d) {
   if (d->bits_a < 1 || d->bits_a > 8 || d->bits_w < 2 || d->bits_w > 8 || d->bits_out < 1 || d->bits_out > 8)
     return PQ_EINVAL;
   if (d->relu != 0 && d->relu != 1) return PQ_EINVAL;
-  if (d->code_format != PQ_CODES_INT8 && d->code_format != PQ_CODES_E4M3) return PQ_EINVAL;
+  if (d->code_format != PQ_CODES_INT8 && d->code_format != PQ_CODES_E4M3 && d->code_format != PQ_CODES_C16)
+    return PQ_EINVAL;
   if (out_dim(d->H, d->kh, d->stride, d->pad) < 1 || out_dim(d->W, d->kw, d->stride, d->pad) < 1) return PQ_EINVAL;
   if (d->G > pq::kMaxG) return PQ_EUNSUPPORTED;
   return PQ_OK;
@@ -119,7 +121,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const int qa = (1 << d->bits_a) - 1;
   const int qw = 1 << (d->bits_w - 1);
   // Coverage of the tensor-core kernel.
-  bool ok = d->code_format == PQ_CODES_INT8 && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
+  const bool c16 = d->code_format == PQ_CODES_C16;
+  bool ok = (d->code_format == PQ_CODES_INT8 || c16) && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
             d->pad < std::max(d->kh, d->kw) && d->Cin_g % 32 == 0 && d->Cout_g % 16 == 0 && taps <= pq::kMaxTaps &&
             static_cast<int64_t>(taps) * d->Cin_g * qa * qw < (1LL << 24);
   if (!ok) {
@@ -178,14 +181,15 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   int best_mt = 0, best_ht = 0, best_tpi = 0, best_acc = 0;
   double best_eff = -1.0, best_halo = 1e30;
   for (int MT : {1, 2, 4}) {
-    if (flat && MT > 2) continue;
+    if (flat && (MT > 2 || (c16 && MT > 1))) continue;
     int acc_stages = (2 * MT * p.Npow2 <= 512) ? 2 : ((MT * p.Npow2 <= 512) ? 1 : 0);
     if (acc_stages == 0) continue;
     double eff, halo;
     int ht = 0, tpi = 0;
     if (flat) {
-      const int64_t tiles = (p.P_out + MT * 128 - 1) / (MT * 128);
-      eff = tiles > 0 ? static_cast<double>(p.P_out) / (tiles * MT * 128.0) : 1.0;
+      const int64_t hw = static_cast<int64_t>(Ho) * Wo;
+      const int64_t tiles = (hw + MT * 128 - 1) / (MT * 128);
+      eff = static_cast<double>(hw) / (tiles * MT * 128.0);
       halo = 1.0;
     } else {
       const int ht_max = (MT * 128) / Wh;
@@ -214,8 +218,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.MT = best_mt;
   p.acc_stages = best_acc;
   if (flat) {
+    // Flat tiles are runs of flat_box pixels inside one image.
     p.flat_box = p.MT * 128;
-    p.tiles = (p.P_out + p.flat_box - 1) / p.flat_box;
+    p.tiles_per_img = static_cast<int>((static_cast<int64_t>(Ho) * Wo + p.flat_box - 1) / p.flat_box);
+    p.tiles = static_cast<int64_t>(d->N) * p.tiles_per_img;
     p.Ht = 0;
     p.Wh = 0;
     p.Hd = 0;
@@ -310,6 +316,29 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.W = d->W;
   p.stride = d->stride;
   p.C_in_total = d->G * d->Cin_g;
+  p.img_pix = d->H * d->W;
+  p.codes_c16 = c16 ? 1 : 0;
+  // The A operand comes by TMA when every plane row is one contiguous run in
+  // global memory: channel-blocked codes, stride 1, rows of at most 128 positions.
+  p.a_tma = (c16 && d->stride == 1 && (flat ? p.flat_box == 128 : p.Wd <= 128)) ? 1 : 0;
+  p.a_tx_bytes = flat ? static_cast<uint32_t>(p.nch) * p.flat_box * 16u
+                      : static_cast<uint32_t>(p.nph) * p.nch * p.Hd * p.Wd * 16u;
+  {
+    const int64_t C = p.C_in_total, H = d->H, W = d->W;
+    if (c16) {
+      p.ld_pix = 16;
+      p.ld_row = W * 16;
+      p.ld_chunk = H * W * 16;
+      p.ld_img = (C / 16) * H * W * 16;
+      p.ld_c0_mul = H * W * 16;  // channel block c0/16 starts c0/16 chunks in
+    } else {
+      p.ld_pix = C;
+      p.ld_row = W * C;
+      p.ld_chunk = 16;
+      p.ld_img = H * W * C;
+      p.ld_c0_mul = 16;  // channel c0 is c0 bytes in
+    }
+  }
   p.n_kb = d->Cin_g / KC;
   p.lbo_a = lbo;
   p.a_phase_bytes = phase_bytes;
@@ -357,6 +386,55 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
 }
 
 bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
+
+// ---------------------------------------------------------------------------
+// Tensor map of channel-blocked activation codes for the TMA operand loads.
+// Element = 8 bytes, so one 16-byte position is 2 elements and a plane row of
+// Wd positions is one box row of 2 Wd elements (a contiguous run).
+// Rows mode (stride 1): dims (2W, H, C/16, N); box (2 Wd, Hd, nch, 1).
+// Flat mode: dims (2 HW, C/16, N); box (2 * 128, nch, 1).
+// Out-of-range elements are zero-filled: the zero padding.
+// ---------------------------------------------------------------------------
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static std::once_flag once;
+  static EncodeTiledFn fn = nullptr;
+  std::call_once(once, [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult qres;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &qres) ==
+            cudaSuccess &&
+        qres == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  });
+  return fn;
+}
+
+bool encode_c16_map(const pq_layer_desc* d, const ConvParams& p, const void* q_dev, CUtensorMap* map) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return false;
+  std::memset(map, 0, sizeof(*map));
+  const uint64_t C16 = static_cast<uint64_t>(d->G) * d->Cin_g / 16, H = d->H, W = d->W;
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  if (p.mode == pq::kModeFlat) {
+    cuuint64_t dims[3] = {2 * H * W, C16, static_cast<cuuint64_t>(d->N)};
+    cuuint64_t strides[2] = {H * W * 16, C16 * H * W * 16};
+    cuuint32_t box[3] = {2u * static_cast<cuuint32_t>(p.flat_box), static_cast<cuuint32_t>(p.nch), 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT64, 3, const_cast<void*>(q_dev), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
+  cuuint64_t dims[4] = {2 * W, H, C16, static_cast<cuuint64_t>(d->N)};
+  cuuint64_t strides[3] = {W * 16, H * W * 16, C16 * H * W * 16};
+  cuuint32_t box[4] = {2u * static_cast<cuuint32_t>(p.Wd), static_cast<cuuint32_t>(p.Hd),
+                       static_cast<cuuint32_t>(p.nch), 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT64, 4, const_cast<void*>(q_dev), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 // ---------------------------------------------------------------------------
 // Weight packing (tensor-core operand layout of the planner's tiling).
@@ -537,8 +615,17 @@ pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int3
   if (x_dev == nullptr || q_dev == nullptr || inv_s_host == nullptr) return PQ_EINVAL;
   if (N < 0 || H < 1 || W < 1 || G < 1 || Cg < 1 || bits < 1 || bits > 8) return PQ_EINVAL;
   if (G > pq::kMaxG) return PQ_EUNSUPPORTED;
-  if (code_format != PQ_CODES_INT8) return code_format == PQ_CODES_E4M3 ? PQ_EUNSUPPORTED : PQ_EINVAL;
+  if (code_format == PQ_CODES_E4M3) return PQ_EUNSUPPORTED;
+  if (code_format != PQ_CODES_INT8 && code_format != PQ_CODES_C16) return PQ_EINVAL;
   const int64_t P = N * H * W;
+  if (code_format == PQ_CODES_C16) {
+    if (Cg % 16 != 0) return PQ_EINVAL;
+    if (!aligned16(x_dev) || !aligned16(q_dev)) return PQ_EINVAL;
+    if (pq::launch_quantize_c16(x_dev, static_cast<uint8_t*>(q_dev), N, static_cast<int64_t>(H) * W, G, Cg, bits,
+                                inv_s_host, static_cast<cudaStream_t>(stream)) != 0)
+      return PQ_ECUDA;
+    return PQ_OK;
+  }
   if (pq::launch_quantize(x_dev, static_cast<uint8_t*>(q_dev), P, G, Cg, bits, inv_s_host,
                           static_cast<cudaStream_t>(stream)) != 0)
     return PQ_ECUDA;
@@ -590,7 +677,10 @@ pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, cons
   if (sms <= 0) return PQ_ECUDA;
   const int grid = static_cast<int>(std::min<int64_t>(sms, p.items));
   if (grid <= 0) return PQ_OK;
-  if (pq::launch_conv_tc(p, grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
+  CUtensorMap map;
+  std::memset(&map, 0, sizeof(map));
+  if (p.a_tma && !encode_c16_map(d, p, q_dev, &map)) return PQ_ECUDA;
+  if (pq::launch_conv_tc(p, map, grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
   return PQ_OK;
 }
 

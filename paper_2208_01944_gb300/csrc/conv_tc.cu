@@ -65,8 +65,7 @@ struct Item {
   int unit;     // (group, output block) unit = g * NB + nb
   int tile;     // tile within the unit
   int g, nb;
-  int n, rb;    // rows mode: image and row block (oh0 = rb * Ht)
-  int64_t p0;   // flat mode: first pixel
+  int n, rb;    // image and tile within it (rows mode: oh0 = rb * Ht; flat mode: first pixel rb * flat_box)
   __device__ __forceinline__ int oh0(int Ht) const { return rb * Ht; }
 };
 
@@ -78,15 +77,8 @@ __device__ __forceinline__ Item item_begin(const ConvParams& p, int64_t it) {
   r.tile = static_cast<int>(it - unit * p.tiles);
   r.g = r.unit / p.NB;
   r.nb = r.unit - r.g * p.NB;
-  if (p.mode == kModeFlat) {
-    r.n = 0;
-    r.rb = 0;
-    r.p0 = static_cast<int64_t>(r.tile) * p.flat_box;
-  } else {
-    r.n = r.tile / p.tiles_per_img;
-    r.rb = r.tile - r.n * p.tiles_per_img;
-    r.p0 = 0;
-  }
+  r.n = r.tile / p.tiles_per_img;
+  r.rb = r.tile - r.n * p.tiles_per_img;
   return r;
 }
 
@@ -96,7 +88,6 @@ __device__ __forceinline__ void item_next(const ConvParams& p, Item& r) {
     r.tile = 0;
     r.n = 0;
     r.rb = 0;
-    r.p0 = 0;
     if (++r.nb == p.NB) {
       r.nb = 0;
       ++r.g;
@@ -104,9 +95,7 @@ __device__ __forceinline__ void item_next(const ConvParams& p, Item& r) {
     ++r.unit;
     return;
   }
-  if (p.mode == kModeFlat) {
-    r.p0 += p.flat_box;
-  } else if (++r.rb == p.tiles_per_img) {
+  if (++r.rb == p.tiles_per_img) {
     r.rb = 0;
     ++r.n;
   }
@@ -130,21 +119,25 @@ struct Bars {
 };
 
 // --------------------------------------------------------------------------
-// Weight copy role (warp 0, lane 0): bulk copies of the packed weights, either
-// once per (group, output-block) unit (resident) or one (K block, tap) slice at
-// a time through a ring.
+// Copy role (warp 0, lane 0): bulk copies of the packed weights, either once
+// per (group, output-block) unit (resident) or one (K block, tap) slice at a
+// time through a ring; and, for channel-blocked codes at stride 1, the
+// activation operand of each stage as one TMA load (every plane row is a
+// contiguous run there).
 // --------------------------------------------------------------------------
-__device__ __forceinline__ void weights_role(const ConvParams& p, const Bars& bars, uint32_t b_base, int64_t it0, int64_t it1,
-                             const WaitCtx& ctx) {
+__device__ __forceinline__ void producer_role(const ConvParams& p, const CUtensorMap* tmA, const Bars& bars,
+                                              uint32_t a_base, uint32_t b_base, int64_t it0, int64_t it1,
+                                              const WaitCtx& ctx) {
+  Ring ra{0, 0, static_cast<uint32_t>(p.a_stages)};
   Ring rb{0, 0, static_cast<uint32_t>(p.b_resident ? 1 : p.b_stages)};
-  int64_t b_issued = 0;
+  int64_t a_issued = 0, b_issued = 0;
   int64_t cur_unit = -1;
+  const bool a_tma = p.a_tma != 0, flat = p.mode == kModeFlat;
   bool ok = true;
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1 && ok; ++it, item_next(p, item)) {
     const int64_t unit = item.unit;
-    if (p.b_resident) {
-      if (unit == cur_unit) continue;
+    if (p.b_resident && unit != cur_unit) {
       if (!mbar_wait(bars.b_empty(rb.stage), rb.phase ^ 1u, ctx)) break;
       const uint32_t bar = bars.b_full(rb.stage);
       mbar_arrive_expect_tx(bar, p.b_unit_bytes);
@@ -154,9 +147,23 @@ __device__ __forceinline__ void weights_role(const ConvParams& p, const Bars& ba
       rb.advance();
       ++b_issued;
       cur_unit = unit;
-      continue;
     }
+    if (!a_tma && p.b_resident) continue;
     for (int kb = 0; kb < p.n_kb && ok; ++kb) {
+      if (a_tma) {
+        if (!mbar_wait(bars.a_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
+        const uint32_t full = bars.a_full(ra.stage);
+        mbar_arrive_expect_tx(full, p.a_tx_bytes);
+        const uint32_t dst = a_base + ra.stage * p.a_stage_bytes;
+        const int chi = (item.g * p.Cin_g + kb * p.KC) >> 4;
+        if (flat)
+          tma_load_3d(dst, tmA, 2 * item.rb * p.flat_box, chi, item.n, full);
+        else
+          tma_load_4d(dst, tmA, 2 * p.w_coord, item.oh0(p.Ht) + p.h_off, chi, item.n, full);
+        ra.advance();
+        ++a_issued;
+      }
+      if (p.b_resident) continue;
       for (int t = 0; t < p.taps; ++t) {
         if (!mbar_wait(bars.b_empty(rb.stage), rb.phase ^ 1u, ctx)) { ok = false; break; }
         const uint32_t bar = bars.b_full(rb.stage);
@@ -168,8 +175,10 @@ __device__ __forceinline__ void weights_role(const ConvParams& p, const Bars& ba
       }
     }
   }
-  // Drain: the last min(stages, issued) copies may still be in flight.
-  const int64_t nbs = p.b_resident ? 1 : p.b_stages;
+  // Drain: the last min(stages, issued) copies of each ring may still be in flight.
+  const int64_t na = p.a_stages, nbs = p.b_resident ? 1 : p.b_stages;
+  for (int64_t k = (a_issued > na ? a_issued - na : 0); k < a_issued; ++k)
+    mbar_wait_drain(bars.a_full(static_cast<int>(k % na)), static_cast<uint32_t>((k / na) & 1), ctx.limit_ns, ctx.err);
   for (int64_t k = (b_issued > nbs ? b_issued - nbs : 0); k < b_issued; ++k)
     mbar_wait_drain(bars.b_full(static_cast<int>(k % nbs)), static_cast<uint32_t>((k / nbs) & 1), ctx.limit_ns, ctx.err);
 }
@@ -196,17 +205,18 @@ __device__ __forceinline__ void load_release(const Bars& bars, int64_t k, int st
 
 __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bars, uint32_t a_base, int64_t it0, int64_t it1,
                             const WaitCtx& ctx) {
+  if (p.a_tma) return;  // warp 0 loads the operand with TMA
   const int tid = threadIdx.x - 32 * kFirstLoadWarp;
   const bool flat = p.mode == kModeFlat;
   const int nch = p.nch;
   const uint32_t plane = p.lbo_a;
-  const int64_t C = p.C_in_total;
+  const int64_t ld_pix = p.ld_pix, ld_chunk = p.ld_chunk;
   const int row_len = flat ? p.flat_box : p.Wd;
   const int per_row = row_len * nch;
   const bool tabled = per_row <= kMaxLoadEntries * kLoaders;
   // This thread's (position, chunk) entries of one plane row.
   uint32_t ent_dst[kMaxLoadEntries];
-  int ent_iw0[kMaxLoadEntries], ent_jo[kMaxLoadEntries];
+  int ent_iw0[kMaxLoadEntries], ent_jo[kMaxLoadEntries];  // ent_jo: the entry's 16-channel chunk
   int n_ent = 0;
 #pragma unroll
   for (int i = 0; i < kMaxLoadEntries; ++i) {
@@ -219,7 +229,7 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
       const int j = e - w * nch;
       ent_dst[i] = static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(w) * 16u;
       ent_iw0[i] = flat ? w : p.stride * (p.w_coord + w);
-      ent_jo[i] = j * 16;
+      ent_jo[i] = j;
       n_ent = i + 1;
     }
   }
@@ -238,6 +248,7 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
       if (!mbar_wait(bars.a_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
       const uint32_t stage = a_base + ra.stage * p.a_stage_bytes;
       const int ch0 = item.g * p.Cin_g + kb * p.KC;  // first input channel of the K block
+      const uint8_t* img_src = p.q_in + item.n * p.ld_img + static_cast<int64_t>(ch0) * p.ld_c0_mul / 16;
       for (int ph = 0; ph < nph; ++ph)
       for (int r = 0; r < Hd; ++r) {
         bool row_ok;
@@ -245,16 +256,17 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
         uint32_t row_dst;
         int b, w_lim;
         if (flat) {
+          const int p0 = item.rb * p.flat_box;  // first pixel of the tile in its image
           row_ok = true;
-          row_src = p.q_in + item.p0 * C + ch0;
+          row_src = img_src + static_cast<int64_t>(p0) * ld_pix;
           row_dst = stage;
           b = 0;
-          w_lim = static_cast<int>(min(p.P_out - item.p0, static_cast<int64_t>(p.flat_box)));
+          w_lim = min(p.img_pix - p0, p.flat_box);
         } else {
           const int pa = ph == 0 ? pa0 : ph == 1 ? pa1 : ph == 2 ? pa2 : pa3;
           const int ih = p.stride * (item.oh0(p.Ht) + p.h_off + r) + pa;
           row_ok = ih >= 0 && ih < p.H;
-          row_src = p.q_in + ((static_cast<int64_t>(item.n) * p.H + (row_ok ? ih : 0)) * p.W) * C + ch0;
+          row_src = img_src + (row_ok ? ih : 0) * p.ld_row;
           row_dst = stage + ph * p.a_phase_bytes + static_cast<uint32_t>(r * p.Wd) * 16u;
           b = ph == 0 ? pb0 : ph == 1 ? pb1 : ph == 2 ? pb2 : pb3;
           w_lim = p.W;
@@ -265,7 +277,7 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
             if (i < n_ent) {
               const int iw = ent_iw0[i] + b;
               const bool valid = row_ok && iw >= 0 && iw < w_lim;
-              cp_async_16(row_dst + ent_dst[i], valid ? row_src + static_cast<int64_t>(iw) * C + ent_jo[i] : p.q_in,
+              cp_async_16(row_dst + ent_dst[i], valid ? row_src + iw * ld_pix + ent_jo[i] * ld_chunk : p.q_in,
                           valid ? 16u : 0u);
             }
           }
@@ -276,7 +288,7 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
             const int iw = (flat ? w : p.stride * (p.w_coord + w)) + b;
             const bool valid = row_ok && iw >= 0 && iw < w_lim;
             cp_async_16(row_dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(w) * 16u,
-                        valid ? row_src + static_cast<int64_t>(iw) * C + j * 16 : p.q_in, valid ? 16u : 0u);
+                        valid ? row_src + iw * ld_pix + j * ld_chunk : p.q_in, valid ? 16u : 0u);
           }
         }
       }
@@ -472,6 +484,9 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
   const float qmax_f = static_cast<float>(qmax);
   const bool has_sc = p.shortcut != nullptr;
   const bool codes_only = !has_sc && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle;
+  const bool c16 = p.codes_c16 != 0;
+  const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
+  const long long c16_out = p.C_out_total / 16;
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1; ++it, item_next(p, item)) {
     if (!mbar_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
@@ -482,19 +497,22 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
     const int dst_c0 = p.dst_group[g] * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
     for (int mt = 0; mt < p.MT; ++mt) {
       const int m = mt * 128 + quarter * 32 + lane;
-      long long pix;
+      int pos;  // output pixel within its image
       bool valid;
       if (p.mode == kModeFlat) {
-        pix = item.p0 + m;
-        valid = pix < p.P_out;
+        pos = item.rb * p.flat_box + m;
+        valid = m < p.flat_box && pos < p.img_pix;
       } else {
         const int r = m / p.Wh;
         const int c = m - r * p.Wh;
         const int oh = item.oh0(p.Ht) + r;
         valid = (r < p.Ht) && (c < p.Wo) && (oh < p.Ho);
-        pix = (static_cast<long long>(item.n) * p.Ho + oh) * p.Wo + c;
+        pos = oh * p.Wo + c;
       }
+      const long long pix = static_cast<long long>(item.n) * hw_out + pos;
       const long long row_elem = valid ? pix * p.C_out_total : -1;
+      // Channel-blocked output codes: 16-channel block k of this pixel at c16_row + k * hw_out * 16.
+      const long long c16_row = (static_cast<long long>(item.n) * c16_out * hw_out + pos) * 16;
       const uint32_t tcol = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2 +
                             mt * p.Npow2;
       for (int seg = c_begin; seg < c_end; seg += kSeg) {
@@ -565,7 +583,10 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
                 const long long o = pix * p.C_out_total + static_cast<long long>(co) * p.G + g;
                 if (p.acc_out) p.acc_out[o] = __float2int_rn(__fmul_rn(__uint_as_float(v[s][j]), 512.0f));
                 if (p.y_out) p.y_out[o] = y[j];
-                if (p.q_out) p.q_out[o] = static_cast<uint8_t>(code[j]);
+                if (p.q_out) {
+                  const long long dc = static_cast<long long>(co) * p.G + g;
+                  p.q_out[c16 ? c16_row + (dc >> 4) * hw_out * 16 + (dc & 15) : o] = static_cast<uint8_t>(code[j]);
+                }
               }
             }
             continue;
@@ -595,12 +616,24 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
                                    __byte_perm(code[4 * j + 2], code[4 * j + 3], 0x0040), 0x5410);
         }
         if (p.q_out && !p.channel_shuffle) {
-          // Codes of this segment go out as one staged row each.
+          if (c16) {
+            // Channel-blocked codes: lanes hold consecutive pixels, so each
+            // 16-byte store of the warp lands next to its neighbours'.
+            if (valid) {
 #pragma unroll
-          for (int s = 0; s < kSeg; ++s)
-            if (s < nseg)
-              *reinterpret_cast<uint4*>(stg + lane * p.stage_q_pitch + s * 16) = make_uint4(qw[s][0], qw[s][1], qw[s][2], qw[s][3]);
-          warp_store_rows(stg, p.stage_q_pitch, nseg * 16, p.q_out, row_elem < 0 ? -1 : row_elem + dst_c0 + seg * 16, lane);
+              for (int s = 0; s < kSeg; ++s)
+                if (s < nseg)
+                  *reinterpret_cast<uint4*>(p.q_out + c16_row + ((dst_c0 >> 4) + seg + s) * hw_out * 16) =
+                      make_uint4(qw[s][0], qw[s][1], qw[s][2], qw[s][3]);
+            }
+          } else {
+            // NHWC codes of this segment go out as one staged row each.
+#pragma unroll
+            for (int s = 0; s < kSeg; ++s)
+              if (s < nseg)
+                *reinterpret_cast<uint4*>(stg + lane * p.stage_q_pitch + s * 16) = make_uint4(qw[s][0], qw[s][1], qw[s][2], qw[s][3]);
+            warp_store_rows(stg, p.stage_q_pitch, nseg * 16, p.q_out, row_elem < 0 ? -1 : row_elem + dst_c0 + seg * 16, lane);
+          }
         }
       }
     }
@@ -612,7 +645,8 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
 
 }  // namespace
 
-__global__ void __launch_bounds__(kConvThreads, 1) pq_conv_tc_kernel(const __grid_constant__ ConvParams p) {
+__global__ void __launch_bounds__(kConvThreads, 1)
+    pq_conv_tc_kernel(const __grid_constant__ ConvParams p, const __grid_constant__ CUtensorMap tmA) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -628,7 +662,7 @@ __global__ void __launch_bounds__(kConvThreads, 1) pq_conv_tc_kernel(const __gri
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < bars.A; ++s) {
-      mbar_init(bars.a_full(s), 32 * kLoadWarps);
+      mbar_init(bars.a_full(s), p.a_tma ? 1 : 32 * kLoadWarps);
       mbar_init(bars.a_empty(s), 1);
     }
     for (int s = 0; s < bars.B; ++s) {
@@ -655,7 +689,10 @@ __global__ void __launch_bounds__(kConvThreads, 1) pq_conv_tc_kernel(const __gri
   const uint32_t b_base = base + p.smem_b_off;
 
   if (warp == 0) {
-    if (lane == 0) weights_role(p, bars, b_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
+    if (lane == 0) {
+      if (p.a_tma) prefetch_tmap(&tmA);
+      producer_role(p, &tmA, bars, a_base, b_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
+    }
     __syncwarp();
   } else if (warp == 1) {
     if (lane == 0)
@@ -676,7 +713,7 @@ __global__ void __launch_bounds__(kConvThreads, 1) pq_conv_tc_kernel(const __gri
   }
 }
 
-int launch_conv_tc(const ConvParams& p, int grid, cudaStream_t stream) {
+int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream) {
   static int attr_set_for_device[64] = {0};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return -1;
@@ -686,7 +723,7 @@ int launch_conv_tc(const ConvParams& p, int grid, cudaStream_t stream) {
       return -1;
     attr_set_for_device[dev] = kMaxSmem;
   }
-  pq_conv_tc_kernel<<<grid, kConvThreads, need, stream>>>(p);
+  pq_conv_tc_kernel<<<grid, kConvThreads, need, stream>>>(p, tma_a);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }
 

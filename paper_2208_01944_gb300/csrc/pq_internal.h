@@ -2,6 +2,7 @@
 // Not part of the public ABI (see include/palquant.h).
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 #include <cstdint>
 
@@ -42,6 +43,14 @@ struct ConvParams {
   int w_coord;            // first plane column = phase column w_coord
   int H, W, stride;       // input geometry
   int C_in_total;         // G * Cin_g (bytes per input pixel)
+  int img_pix;            // H * W (flat mode tiles stay inside one image)
+  int codes_c16;          // 1: input and output codes in the channel-blocked layout [N][C/16][H][W][16]
+  int a_tma;              // 1: warp 0 loads the A operand with one TMA per stage (channel-blocked codes, stride 1)
+  uint32_t a_tx_bytes;    // bytes one A stage receives (TMA mode)
+  // Activation copy addressing (cp.async mode), in bytes: code (n, ih, iw, c0 + 16 j) of the
+  // K block starting at channel c0 sits at n*ld_img + ih*ld_row + iw*ld_pix + ld_c0(c0) + j*ld_chunk,
+  // with ld_c0(c0) = c0 * ld_c0_mul / 16.
+  int64_t ld_img, ld_row, ld_pix, ld_chunk, ld_c0_mul;
   int phase_a[kMaxPhases], phase_b[kMaxPhases];  // stride phase (row, column) of each plane set
   uint32_t nch_magic;     // ceil(2^32 / nch): e / nch = umulhi(e, nch_magic) for small e
   int tiles_per_img;      // rows mode
@@ -90,7 +99,9 @@ struct ConvParams {
 };
 
 // Host-side launch helpers implemented in the .cu files.
-int launch_conv_tc(const ConvParams& p, int grid, cudaStream_t stream);
+int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream);
+int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G, int Cg, int bits, const float* inv_s,
+                        cudaStream_t stream);
 int launch_quantize(const float* x, uint8_t* q, int64_t P, int G, int Cg, int bits, const float* inv_s,
                     cudaStream_t stream);
 int launch_act_sum(const float* x, int64_t P, int G, int Cg, double* partial, int nblocks, cudaStream_t stream);

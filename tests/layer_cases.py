@@ -78,8 +78,15 @@ def prepare(c: Case, sample_pix: np.ndarray | None = None):
                 m_out=m_out, m_req=m_req, acc_ref=a_ref, y_ref=y_ref, q_ref=q_ref)
 
 
-def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q")):
-    """Quantise and run the fused layer on the GPU through the C ABI."""
+def c16_to_nhwc(a: np.ndarray, N: int, H: int, W: int, C: int) -> np.ndarray:
+    """Channel-blocked codes [N][C/16][H][W][16] -> NHWC (a pure permutation of bytes)."""
+    return np.ascontiguousarray(a.reshape(N, C // 16, H, W, 16).transpose(0, 2, 3, 1, 4).reshape(N, H, W, C))
+
+
+def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q"), fmt: int = 0):
+    """Quantise and run the fused layer on the GPU through the C ABI.  fmt is the
+    code format of the activation and output codes (0 NHWC, 2 channel-blocked);
+    returned codes are always NHWC."""
     import torch
 
     from paper_2208_01944_gb300 import binding as B
@@ -87,8 +94,9 @@ def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q")):
     dev = torch.device("cuda:0")
     x = torch.from_numpy(ref["x"]).to(dev)
     q = torch.empty(x.shape, dtype=torch.uint8, device=dev)
-    B.palquant_quantize_act(x, q, c.N, c.H, c.W, c.G, c.Cin, c.bits, ref["inv_s"])
-    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad, c.bits, c.bits, c.bo, int(c.relu))
+    B.palquant_quantize_act(x, q, c.N, c.H, c.W, c.G, c.Cin, c.bits, ref["inv_s"], code_format=fmt)
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad, c.bits, c.bits, c.bo, int(c.relu),
+                     code_format=fmt)
     nbytes = B.palquant_packed_weight_bytes(d)
     wp = torch.empty(nbytes, dtype=torch.uint8, device=dev)
     B.palquant_pack_weights(ref["w"], d, ref["inv_sw"], wp, nbytes)
@@ -100,13 +108,19 @@ def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q")):
     B.palquant_layer_fused(q, wp, d, ref["m_out"], ref["m_req"], B.shuffle(c.kind, c.shift, c.perm), sc, acc, y, qo)
     st = B.palquant_sync_check()
     assert st == B.PQ_OK, B.strerror(st)
-    out = dict(q=q.cpu().numpy())
+    qh = q.cpu().numpy()
+    if fmt == B.PQ_CODES_C16:
+        qh = c16_to_nhwc(qh, c.N, c.H, c.W, c.G * c.Cin)
+    out = dict(q=qh)
     if acc is not None:
         out["acc"] = acc.cpu().numpy().reshape(-1, c.G * c.Cout)
     if y is not None:
         out["y"] = y.cpu().numpy().reshape(-1, c.G * c.Cout)
     if qo is not None:
-        out["q_out"] = qo.cpu().numpy().reshape(-1, c.G * c.Cout)
+        qoh = qo.cpu().numpy()
+        if fmt == B.PQ_CODES_C16:
+            qoh = c16_to_nhwc(qoh, c.N, c.Ho, c.Wo, c.G * c.Cout)
+        out["q_out"] = qoh.reshape(-1, c.G * c.Cout)
     return out
 
 

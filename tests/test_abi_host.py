@@ -56,7 +56,7 @@ def test_plan_invariants(c):
         assert plan.tiles == c.N * tiles_per_img
         assert plan.tile_pitch >= c.Wo
     else:
-        assert plan.tiles == -(-(c.N * c.Ho * c.Wo) // rows)
+        assert plan.tiles == c.N * -(-(c.Ho * c.Wo) // rows)  # flat tiles stay inside one image
     assert plan.work_items == plan.tiles * c.G * plan.n_blocks
     assert plan.acc_stages * plan.m_tiles * plan.n_block <= 512
 

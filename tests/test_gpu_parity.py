@@ -94,11 +94,31 @@ SMALL_CASES = [
 ]
 
 
+FORMATS = [0, 2]  # NHWC codes, channel-blocked codes
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=["nhwc", "c16"])
 @pytest.mark.parametrize("c", SMALL_CASES, ids=str)
-def test_layer_fused_matches_oracle(B, c):
+def test_layer_fused_matches_oracle(B, c, fmt):
     ref = prepare(c)
-    got = run_gpu(c, ref)
+    got = run_gpu(c, ref, fmt=fmt)
     assert_layer_parity(c, ref, got)
+
+
+@pytest.mark.parametrize("shape,G,bits", [((2, 7, 9, 64), 4, 2), ((3, 5, 6, 3 * 16), 3, 4), ((1, 1, 1, 32), 1, 8)])
+def test_quantize_act_c16_matches_oracle(B, shape, G, bits):
+    from layer_cases import c16_to_nhwc
+
+    gen = synth.generator(sum(shape) + 7)
+    x = synth.normal(shape, gen, 2.0)
+    x.reshape(-1)[:6] = np.array([0.5, 1.5, 2.5, np.nan, np.inf, -np.inf], dtype=np.float32)
+    inv = (synth.half_normal((G,), gen) + 0.5).astype(np.float32)
+    xd = torch.from_numpy(x).cuda()
+    q = torch.full(shape, 254, dtype=torch.uint8, device="cuda")
+    B.palquant_quantize_act(xd, q, shape[0], shape[1], shape[2], G, shape[3] // G, bits, inv, code_format=B.PQ_CODES_C16)
+    assert B.palquant_sync_check() == B.PQ_OK
+    got = c16_to_nhwc(q.cpu().numpy(), *shape)
+    assert np.array_equal(got, oracle.quantize_act(x, G, bits, inv))
 
 
 def test_group_conv_matches_oracle(B):
@@ -181,13 +201,25 @@ FULL = [("config1", workloads.CONFIG1)] + [(f"config3_{i}", c) for i, c in enume
     ("config4", workloads.CONFIG4)]
 
 
+@pytest.mark.parametrize("fmt", FORMATS, ids=["nhwc", "c16"])
 @pytest.mark.parametrize("name,cfg", FULL, ids=[n for n, _ in FULL])
-def test_full_size_layer_sampled(B, name, cfg):
+def test_full_size_layer_sampled(B, name, cfg, fmt):
     c = Case(cfg.N, cfg.H, cfg.W, cfg.G, cfg.Cin_g, cfg.Cout_g, cfg.k, cfg.stride, cfg.pad, bits=cfg.bits_a,
              kind=cfg.shuffle_kind, shift=cfg.shuffle_shift, relu=cfg.relu, seed=0)
     pix = _sample_pixels(c.N, c.Ho, c.Wo, 3000, 1)
     ref = prepare(c, sample_pix=pix)
-    got = run_gpu(c, ref)
+    got = run_gpu(c, ref, fmt=fmt)
+    assert_layer_parity(c, ref, got, pix)
+
+
+@pytest.mark.parametrize("name,cfg", FULL, ids=[n for n, _ in FULL])
+def test_full_size_codes_only_c16_sampled(B, name, cfg):
+    """The benchmarked configuration: channel-blocked codes in and out, codes only."""
+    c = Case(cfg.N, cfg.H, cfg.W, cfg.G, cfg.Cin_g, cfg.Cout_g, cfg.k, cfg.stride, cfg.pad, bits=cfg.bits_a,
+             kind=cfg.shuffle_kind, shift=cfg.shuffle_shift, relu=cfg.relu, seed=0)
+    pix = _sample_pixels(c.N, c.Ho, c.Wo, 3000, 2)
+    ref = prepare(c, sample_pix=pix)
+    got = run_gpu(c, ref, outputs=("q",), fmt=2)
     assert_layer_parity(c, ref, got, pix)
 
 
@@ -209,10 +241,11 @@ CODES_ONLY = [
 ]
 
 
+@pytest.mark.parametrize("fmt", FORMATS, ids=["nhwc", "c16"])
 @pytest.mark.parametrize("c", CODES_ONLY, ids=str)
-def test_layer_codes_only_matches_oracle(B, c):
+def test_layer_codes_only_matches_oracle(B, c, fmt):
     ref = prepare(c)
-    got = run_gpu(c, ref, outputs=("q",))
+    got = run_gpu(c, ref, outputs=("q",), fmt=fmt)
     assert_layer_parity(c, ref, got)
 
 
