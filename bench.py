@@ -4,10 +4,11 @@
 One step = one pass of the whole hot path over one batch of the ResNet-18 stage-1
 shaped PalQuant 3x3 layer (batch 64, 56x56, G = 4 groups of 64 channels, 2-bit
 activations and weights, cyclic shuffle):
-  (1) group-wise activation quantisation of the fp32 NHWC input (205.5 MB) into int8
-      codes, and (2) the fused layer: B-bit group convolution on the tensor cores,
-      rescale, ReLU, cyclic-shuffle output permutation and requantisation into the
-      next layer's codes (51.4 MB).
+  (1) group-wise activation quantisation of the fp32 NHWC input (205.5 MB) into one
+      byte per code in the channel-blocked layout the tensor cores read, and (2) the
+      fused layer: B-bit group convolution on the tensor cores, rescale, ReLU,
+      cyclic-shuffle output permutation and requantisation into the next layer's
+      codes (51.4 MB, same layout).
 Inputs are resident in HBM when the timed region starts; two input buffers are used
 in turn so each step reads an input larger than L2 that the previous step did not.
 
@@ -62,7 +63,8 @@ def run_profile_layer(name: str, reps: int):
     gen = synth.generator(0)
     q = torch.from_numpy(synth.random_codes((c.N, c.H, c.W, c.G * c.Cin_g), c.bits_a, gen)).to(dev)
     wq = synth.random_codes((c.G, c.Cout_g, c.k, c.k, c.Cin_g), c.bits_w, gen, signed=True)
-    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out)
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out,
+                     code_format=B.PQ_CODES_C16)
     wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).to(dev)
     qo = torch.empty((c.N, c.Ho, c.Wo, c.G * c.Cout_g), dtype=torch.uint8, device=dev)
     m = np.full(c.G, 0.01, np.float32)
@@ -90,7 +92,7 @@ def source_sha(files):
 
 
 KERNEL_SOURCES = {
-    "pq_quantize_vec16": ["quantize.cu", "pq_internal.h"],
+    "pq_quantize_c16": ["quantize.cu", "pq_internal.h"],
     "pq_conv_tc_kernel": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
 }
 
@@ -253,8 +255,9 @@ def run_ours(args, rank, world, local_rank):
     scratch_bytes = B.palquant_act_steps_scratch_bytes(P, c.G)
     scratch = torch.empty(scratch_bytes, dtype=torch.uint8, device=dev)
     s_a = B.palquant_act_steps(xs[0], c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, scratch, scratch_bytes)
+    fmt = B.PQ_CODES_C16
     d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out,
-                     int(c.relu))
+                     int(c.relu), code_format=fmt)
     s_w = B.palquant_weight_steps(w_np, d)
     inv_s = np.array([np.float32(1.0 / np.float64(v)) for v in s_a], dtype=np.float32)
     inv_sw = np.array([np.float32(1.0 / np.float64(v)) for v in s_w], dtype=np.float32)
@@ -267,7 +270,7 @@ def run_ours(args, rank, world, local_rank):
     # next layer's steps: calibrated on this layer's rescaled output
     m_out, _ = B.palquant_epilogue_scales(c.G, s_w, s_a, 1.0, None, shuf)
     y = torch.empty(out_shape, dtype=torch.float32, device=dev)
-    B.palquant_quantize_act(xs[0], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s)
+    B.palquant_quantize_act(xs[0], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt)
     B.palquant_layer_fused(q, wp, d, m_out, m_out, shuf, None, None, y, None)
     s_next = B.palquant_act_steps(y, c.N, c.Ho, c.Wo, c.G, c.Cout_g, c.bits_out, scratch, scratch_bytes)
     m_out, m_req = B.palquant_epilogue_scales(c.G, s_w, s_a, 1.0, s_next, shuf)
@@ -276,7 +279,7 @@ def run_ours(args, rank, world, local_rank):
     assert B.palquant_sync_check() == B.PQ_OK
 
     def step(i, s):
-        B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, stream=s)
+        B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt, stream=s)
         B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=s)
 
     # ---- warm-up
@@ -301,7 +304,8 @@ def run_ours(args, rank, world, local_rank):
         start.record(stream)
         for i in range(K):
             ev[i][0].record(stream)
-            B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, stream=stream)
+            B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt,
+                                    stream=stream)
             ev[i][1].record(stream)
             B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
             ev[i][2].record(stream)
@@ -355,8 +359,8 @@ def run_ours(args, rank, world, local_rank):
     conv_bytes = c.in_elems + c.out_elems + c.weight_elems
     quant_gbs = q_bytes / (t_quant / 1e3) / 1e9
     conv_tops = ops_step / (t_conv / 1e3) / 1e12
-    roof_quant = {"kernel": "pq_quantize_vec16", "bound": "hbm", "achieved": quant_gbs, "peak": pk["hbm_gbs"],
-                  "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"], "traffic": dram_traffic("pq_quantize_vec16"),
+    roof_quant = {"kernel": "pq_quantize_c16", "bound": "hbm", "achieved": quant_gbs, "peak": pk["hbm_gbs"],
+                  "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"], "traffic": dram_traffic("pq_quantize_c16"),
                   "algorithmic_bytes": q_bytes, "avg_launch_ms": t_quant,
                   "peak_source": f"{pk['source']} HBM copy bandwidth"}
     roof_conv = {"kernel": "pq_conv_tc_kernel", "bound": "tensor", "achieved": conv_tops, "peak": fp8_peak,
@@ -371,6 +375,7 @@ def run_ours(args, rank, world, local_rank):
         "dtype": "u8 codes, e4m3 x e4m3 -> f32 (exact integer)", "data": "synthetic",
         "config": {"workload": WORKLOAD, "global_batch": c.N * world, "per_gpu_batch": c.N,
                    "timed": "quantize (fp32 NHWC -> codes) + fused layer (codes -> next-layer codes)",
+                   "code_layout": "channel-blocked [N][C/16][H][W][16], one byte per code",
                    "l2": "inputs larger than L2 (205.5 MB fp32, two buffers used in turn)",
                    "parallelism": f"replicas x{world}"},
         "images_per_s": c.N * world / (ms_per_step / 1e3),

@@ -267,7 +267,9 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const uint32_t q_pitch = 80;
   const uint32_t f_pitch = 80;
   const uint32_t warp_stage = round_up(32u * q_pitch, 128);
-  const uint32_t stage_total = warp_stage * pq::kEpiWarps;
+  // Staging for every warp that can run the epilogue (the copy warps join it when
+  // TMA loads the activation operand).
+  const uint32_t stage_total = warp_stage * (pq::kEpiWarps + pq::kLoadWarps);
   const uint32_t bar_bytes = 1024;  // barriers, abort flag, TMEM slot (generous)
   const uint64_t unit_bytes = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk;
   // Largest K block (input channels per pipeline stage) that fits: the whole

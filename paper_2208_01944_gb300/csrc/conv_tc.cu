@@ -468,173 +468,250 @@ __device__ __forceinline__ int requant_code(float t, float qmax_f, int qmax) {
   return min(max(i, 0), qmax);
 }
 
-constexpr int kSeg = 2;  // 16-column chunks per TMEM load batch
+// Item-level constants of the epilogue.
+struct EpiItem {
+  uint32_t tbase;        // TMEM address of accumulator 0, this warp's lanes
+  float m_out512, m_req512, m_req;
+  int g, src_c0, dst_c0;
+  int n, rb, oh0;
+  int nb;
+};
 
-__device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& bars, uint32_t tmem_base, uint8_t* stage_base,
-                              int64_t it0, int64_t it1, const WaitCtx& ctx) {
+// Output pixel (within its image) of accumulator row m, and whether it exists.
+__device__ __forceinline__ int epi_pos(const ConvParams& p, const EpiItem& e, int m, bool& valid) {
+  if (p.mode == kModeFlat) {
+    const int pos = e.rb * p.flat_box + m;
+    valid = m < p.flat_box && pos < p.img_pix;
+    return pos;
+  }
+  const int r = m / p.Wh;
+  const int c = m - r * p.Wh;
+  const int oh = e.oh0 + r;
+  valid = (r < p.Ht) && (c < p.Wo) && (oh < p.Ho);
+  return oh * p.Wo + c;
+}
+
+// Codes-only unit (the timed path): t = acc * m_req = raw * (m_req * 2^9),
+// clamped to [0, Qp] in fp32 (NaN -> 0), then rounded half to even by adding
+// 1.5 * 2^23, which leaves the code in the sum's low byte.
+__device__ __forceinline__ uint4 epi_codes16(const uint32_t (&v)[16], float m_req512, float qmax_f) {
+  uint32_t bits[16];
+#pragma unroll
+  for (int j = 0; j < 16; j += 2) {
+    float t0, t1;
+    mul2_rn(__uint_as_float(v[j]), __uint_as_float(v[j + 1]), m_req512, t0, t1);
+    t0 = fminf(fmaxf(t0, 0.0f), qmax_f);
+    t1 = fminf(fmaxf(t1, 0.0f), qmax_f);
+    float r0, r1;
+    add2_rn(t0, t1, 12582912.0f, r0, r1);
+    bits[j] = __float_as_uint(r0);
+    bits[j + 1] = __float_as_uint(r1);
+  }
+  uint4 w;
+  w.x = __byte_perm(__byte_perm(bits[0], bits[1], 0x0040), __byte_perm(bits[2], bits[3], 0x0040), 0x5410);
+  w.y = __byte_perm(__byte_perm(bits[4], bits[5], 0x0040), __byte_perm(bits[6], bits[7], 0x0040), 0x5410);
+  w.z = __byte_perm(__byte_perm(bits[8], bits[9], 0x0040), __byte_perm(bits[10], bits[11], 0x0040), 0x5410);
+  w.w = __byte_perm(__byte_perm(bits[12], bits[13], 0x0040), __byte_perm(bits[14], bits[15], 0x0040), 0x5410);
+  return w;
+}
+
+// Store 16 codes of 16-column chunk `ch` of the row (output pixel pos).
+__device__ __forceinline__ void epi_store_codes(const ConvParams& p, const EpiItem& e, uint8_t* stg, int lane, bool valid,
+                                                int pos, int ch, uint4 w) {
+  const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
+  if (p.codes_c16) {
+    // Channel-blocked codes: lanes hold consecutive pixels, so each 16-byte
+    // store of the warp lands next to its neighbours'.
+    if (valid) {
+      const long long blk = (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (e.dst_c0 >> 4) + ch) * hw_out + pos;
+      *reinterpret_cast<uint4*>(p.q_out + blk * 16) = w;
+    }
+  } else {
+    // NHWC: staged, then 16-byte rows written by the warp.
+    *reinterpret_cast<uint4*>(stg + lane * p.stage_q_pitch) = w;
+    const long long pix = static_cast<long long>(e.n) * hw_out + pos;
+    warp_store_rows(stg, p.stage_q_pitch, 16, p.q_out, valid ? pix * p.C_out_total + e.dst_c0 + ch * 16 : -1, lane);
+  }
+}
+
+// General unit: int32 sums, fp32 outputs (with the shortcut) and codes, or the
+// per-channel scatter of the channel shuffle.
+__device__ __noinline__ void epi_general16(const ConvParams& p, const EpiItem& e, uint8_t* stg, int lane, int m, int ch,
+                                           const uint32_t* v) {
+  bool valid;
+  const int pos = epi_pos(p, e, m, valid);
+  const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
+  const long long pix = static_cast<long long>(e.n) * hw_out + pos;
+  const long long row_elem = valid ? pix * p.C_out_total : -1;
+  const bool has_sc = p.shortcut != nullptr;
+  const int qmax = p.qmax_out;
+  const float qmax_f = static_cast<float>(qmax);
+  float sc[16];
+  if (has_sc) {
+    if (valid) {
+      const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + pix * p.C_out_total + e.src_c0 + ch * 16);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float4 t = s4[j];
+        sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
+      }
+    } else {
+#pragma unroll
+      for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
+    }
+  }
+  float y[16];
+  int code[16];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) {
+    const float raw = __uint_as_float(v[j]);
+    float t = __fmul_rn(raw, e.m_out512);  // = (float)acc * m_out, one rounding
+    if (has_sc) t = __fadd_rn(t, sc[j]);
+    if (p.relu) t = fmaxf(t, 0.0f);
+    y[j] = t;
+    code[j] = requant_code(has_sc ? __fmul_rn(t, e.m_req) : __fmul_rn(raw, e.m_req512), qmax_f, qmax);
+  }
+  if (p.channel_shuffle) {
+    // Per-channel scatter (destination channel co * G + g); rarely used, unstaged.
+    if (valid) {
+      for (int j = 0; j < 16; ++j) {
+        const int co = e.nb * p.Nblk + ch * 16 + j;
+        const long long dc = static_cast<long long>(co) * p.G + e.g;
+        const long long o = pix * p.C_out_total + dc;
+        if (p.acc_out) p.acc_out[o] = __float2int_rn(__fmul_rn(__uint_as_float(v[j]), 512.0f));
+        if (p.y_out) p.y_out[o] = y[j];
+        if (p.q_out) {
+          const long long c16o = (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (dc >> 4)) * hw_out + pos;
+          p.q_out[p.codes_c16 ? c16o * 16 + (dc & 15) : o] = static_cast<uint8_t>(code[j]);
+        }
+      }
+    }
+    return;
+  }
+  if (p.acc_out) {
+    uint32_t* row = reinterpret_cast<uint32_t*>(stg + lane * p.stage_q_pitch);
+    for (int j = 0; j < 16; j += 4)
+      *reinterpret_cast<int4*>(row + j) =
+          make_int4(__float2int_rn(__fmul_rn(__uint_as_float(v[j]), 512.0f)),
+                    __float2int_rn(__fmul_rn(__uint_as_float(v[j + 1]), 512.0f)),
+                    __float2int_rn(__fmul_rn(__uint_as_float(v[j + 2]), 512.0f)),
+                    __float2int_rn(__fmul_rn(__uint_as_float(v[j + 3]), 512.0f)));
+    warp_store_rows(stg, p.stage_q_pitch, 64, reinterpret_cast<uint8_t*>(p.acc_out),
+                    row_elem < 0 ? -1 : (row_elem + e.dst_c0 + ch * 16) * 4, lane);
+  }
+  if (p.y_out) {
+    float* row = reinterpret_cast<float*>(stg + lane * p.stage_q_pitch);
+    for (int j = 0; j < 16; j += 4) *reinterpret_cast<float4*>(row + j) = make_float4(y[j], y[j + 1], y[j + 2], y[j + 3]);
+    warp_store_rows(stg, p.stage_q_pitch, 64, reinterpret_cast<uint8_t*>(p.y_out),
+                    row_elem < 0 ? -1 : (row_elem + e.dst_c0 + ch * 16) * 4, lane);
+  }
+  if (p.q_out) {
+    uint4 w;
+    w.x = __byte_perm(__byte_perm(code[0], code[1], 0x0040), __byte_perm(code[2], code[3], 0x0040), 0x5410);
+    w.y = __byte_perm(__byte_perm(code[4], code[5], 0x0040), __byte_perm(code[6], code[7], 0x0040), 0x5410);
+    w.z = __byte_perm(__byte_perm(code[8], code[9], 0x0040), __byte_perm(code[10], code[11], 0x0040), 0x5410);
+    w.w = __byte_perm(__byte_perm(code[12], code[13], 0x0040), __byte_perm(code[14], code[15], 0x0040), 0x5410);
+    epi_store_codes(p, e, stg, lane, valid, pos, ch, w);
+  }
+}
+
+// The epilogue's work per tile is a list of units, one per (accumulator mt,
+// 16-column chunk); epilogue warpgroup wg of n_groups takes units wg,
+// wg + n_groups, ...  Each warp handles the 32 TMEM lanes (rows) it may access.
+// On the codes-only path the TMEM loads are double-buffered: the next unit's
+// load is in flight while the current one is computed and stored.
+__device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& bars, uint32_t tmem_base,
+                                              uint8_t* stage_base, int first_warp, int n_groups, int64_t it0,
+                                              int64_t it1, const WaitCtx& ctx) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int ew = warp - kFirstEpiWarp;  // epilogue warp index
-  const int wg = ew >> 2;             // warpgroup: which share of the output columns
-  const int quarter = warp & 3;       // TMEM lanes this warp may access
+  const int ew = warp - first_warp;  // epilogue warp index
+  const int wg = ew >> 2;            // warpgroup
+  const int quarter = warp & 3;      // TMEM lanes this warp may access
   uint8_t* stg = stage_base + ew * p.stage_warp_bytes;
   Ring racc{0, 0, static_cast<uint32_t>(p.acc_stages)};
   const int nchunks = p.Nblk >> 4;
-  const int c_begin = (wg * nchunks) / kEpiGroups, c_end = ((wg + 1) * nchunks) / kEpiGroups;
-  const int qmax = p.qmax_out;
-  const float qmax_f = static_cast<float>(qmax);
-  const bool has_sc = p.shortcut != nullptr;
-  const bool codes_only = !has_sc && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle;
-  const bool c16 = p.codes_c16 != 0;
-  const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
-  const long long c16_out = p.C_out_total / 16;
+  const int n_units = p.MT * nchunks;
+  const float qmax_f = static_cast<float>(p.qmax_out);
+  const bool codes_only = p.shortcut == nullptr && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle;
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1; ++it, item_next(p, item)) {
     if (!mbar_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
     tc_fence_after();
-    const int g = item.g;
-    const float m_out512 = p.m_out512[g], m_req512 = p.m_req512[g], m_req = p.m_req[g];
-    const int src_c0 = g * p.Cout_g + item.nb * p.Nblk;               // source channel of column 0
-    const int dst_c0 = p.dst_group[g] * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
-    for (int mt = 0; mt < p.MT; ++mt) {
-      const int m = mt * 128 + quarter * 32 + lane;
-      int pos;  // output pixel within its image
-      bool valid;
-      if (p.mode == kModeFlat) {
-        pos = item.rb * p.flat_box + m;
-        valid = m < p.flat_box && pos < p.img_pix;
-      } else {
-        const int r = m / p.Wh;
-        const int c = m - r * p.Wh;
-        const int oh = item.oh0(p.Ht) + r;
-        valid = (r < p.Ht) && (c < p.Wo) && (oh < p.Ho);
-        pos = oh * p.Wo + c;
-      }
-      const long long pix = static_cast<long long>(item.n) * hw_out + pos;
-      const long long row_elem = valid ? pix * p.C_out_total : -1;
-      // Channel-blocked output codes: 16-channel block k of this pixel at c16_row + k * hw_out * 16.
-      const long long c16_row = (static_cast<long long>(item.n) * c16_out * hw_out + pos) * 16;
-      const uint32_t tcol = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2 +
-                            mt * p.Npow2;
-      for (int seg = c_begin; seg < c_end; seg += kSeg) {
-        const int nseg = min(kSeg, c_end - seg);
-        uint32_t v[kSeg][16];
-#pragma unroll
-        for (int s = 0; s < kSeg; ++s)
-          if (s < nseg) tmem_ld16(tcol + (seg + s) * 16, v[s]);
+    EpiItem e;
+    e.g = item.g;
+    e.nb = item.nb;
+    e.n = item.n;
+    e.rb = item.rb;
+    e.oh0 = item.oh0(p.Ht);
+    e.m_out512 = p.m_out512[e.g];
+    e.m_req512 = p.m_req512[e.g];
+    e.m_req = p.m_req[e.g];
+    e.src_c0 = e.g * p.Cout_g + item.nb * p.Nblk;               // source channel of column 0
+    e.dst_c0 = p.dst_group[e.g] * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
+    e.tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2;
+    if (codes_only && p.codes_c16) {
+      // Channel-blocked codes only (the timed path).  A warp's units run in
+      // increasing (mt, ch) order; the destination of this lane's row is
+      // computed once per accumulator, and 16-channel block ch of that row lies
+      // ch * H_out * W_out * 16 bytes further on.
+      const long long chunk_bytes = static_cast<long long>(p.Ho) * p.Wo * 16;
+      uint8_t* const blk0 = p.q_out + (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (e.dst_c0 >> 4)) * chunk_bytes;
+      const int m_lane = quarter * 32 + lane;
+      const int MT = p.MT;
+      auto row_ptr = [&](int mt) -> uint8_t* {
+        if (mt >= MT) return nullptr;
+        bool valid;
+        const int pos = epi_pos(p, e, mt * 128 + m_lane, valid);
+        return valid ? blk0 + static_cast<long long>(pos) * 16 : nullptr;
+      };
+      auto step = [&](int& mt, int& ch) {
+        ch += n_groups;
+        while (ch >= nchunks) {
+          ch -= nchunks;
+          ++mt;
+        }
+      };
+      auto col = [&](int mt, int ch) { return e.tbase + static_cast<uint32_t>(mt) * p.Npow2 + ch * 16; };
+      uint32_t va[16], vb[16];
+      int c_mt = 0, c_ch = wg - n_groups;
+      step(c_mt, c_ch);
+      uint8_t* c_row = row_ptr(c_mt);
+      if (c_mt < MT) {
+        tmem_ld16(col(c_mt, c_ch), va);
         tmem_wait_ld();
-        uint32_t qw[kSeg][4];
-#pragma unroll
-        for (int s = 0; s < kSeg; ++s) {
-          if (s >= nseg) continue;
-          const int ch = seg + s;
-          if (codes_only) {
-            // Timed path, codes only: t = acc * m_req = raw * (m_req * 2^9),
-            // clamped to [0, Qp] in fp32 (NaN -> 0), then rounded half to even by
-            // adding 1.5 * 2^23, which leaves the code in the sum's low byte.
-            uint32_t bits[16];
-#pragma unroll
-            for (int j = 0; j < 16; j += 2) {
-              float t0, t1;
-              mul2_rn(__uint_as_float(v[s][j]), __uint_as_float(v[s][j + 1]), m_req512, t0, t1);
-              t0 = fminf(fmaxf(t0, 0.0f), qmax_f);
-              t1 = fminf(fmaxf(t1, 0.0f), qmax_f);
-              float r0, r1;
-              add2_rn(t0, t1, 12582912.0f, r0, r1);
-              bits[j] = __float_as_uint(r0);
-              bits[j + 1] = __float_as_uint(r1);
-            }
-#pragma unroll
-            for (int j = 0; j < 4; ++j)
-              qw[s][j] = __byte_perm(__byte_perm(bits[4 * j], bits[4 * j + 1], 0x0040),
-                                     __byte_perm(bits[4 * j + 2], bits[4 * j + 3], 0x0040), 0x5410);
-            continue;
-          }
-          float sc[16];
-          if (has_sc) {
-            if (valid) {
-              const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + pix * p.C_out_total + src_c0 + ch * 16);
-#pragma unroll
-              for (int j = 0; j < 4; ++j) {
-                const float4 t = s4[j];
-                sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
-              }
-            } else {
-#pragma unroll
-              for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
-            }
-          }
-          float y[16];
-          int code[16];
-#pragma unroll
-          for (int j = 0; j < 16; ++j) {
-            const float raw = __uint_as_float(v[s][j]);
-            float t = __fmul_rn(raw, m_out512);  // = (float)acc * m_out, one rounding
-            if (has_sc) t = __fadd_rn(t, sc[j]);
-            if (p.relu) t = fmaxf(t, 0.0f);
-            y[j] = t;
-            code[j] = requant_code(has_sc ? __fmul_rn(t, m_req) : __fmul_rn(raw, m_req512), qmax_f, qmax);
-          }
-          if (p.channel_shuffle) {
-            // Per-channel scatter (destination channel co * G + g); rarely used, unstaged.
-            if (valid) {
-#pragma unroll
-              for (int j = 0; j < 16; ++j) {
-                const int co = item.nb * p.Nblk + ch * 16 + j;
-                const long long o = pix * p.C_out_total + static_cast<long long>(co) * p.G + g;
-                if (p.acc_out) p.acc_out[o] = __float2int_rn(__fmul_rn(__uint_as_float(v[s][j]), 512.0f));
-                if (p.y_out) p.y_out[o] = y[j];
-                if (p.q_out) {
-                  const long long dc = static_cast<long long>(co) * p.G + g;
-                  p.q_out[c16 ? c16_row + (dc >> 4) * hw_out * 16 + (dc & 15) : o] = static_cast<uint8_t>(code[j]);
-                }
-              }
-            }
-            continue;
-          }
-          if (p.acc_out) {
-            uint32_t* row = reinterpret_cast<uint32_t*>(stg + lane * p.stage_q_pitch);
-#pragma unroll
-            for (int j = 0; j < 16; j += 4)
-              *reinterpret_cast<int4*>(row + j) = make_int4(
-                  __float2int_rn(__fmul_rn(__uint_as_float(v[s][j]), 512.0f)),
-                  __float2int_rn(__fmul_rn(__uint_as_float(v[s][j + 1]), 512.0f)),
-                  __float2int_rn(__fmul_rn(__uint_as_float(v[s][j + 2]), 512.0f)),
-                  __float2int_rn(__fmul_rn(__uint_as_float(v[s][j + 3]), 512.0f)));
-            warp_store_rows(stg, p.stage_q_pitch, 64, reinterpret_cast<uint8_t*>(p.acc_out),
-                            row_elem < 0 ? -1 : (row_elem + dst_c0 + ch * 16) * 4, lane);
-          }
-          if (p.y_out) {
-            float* row = reinterpret_cast<float*>(stg + lane * p.stage_q_pitch);
-#pragma unroll
-            for (int j = 0; j < 16; j += 4) *reinterpret_cast<float4*>(row + j) = make_float4(y[j], y[j + 1], y[j + 2], y[j + 3]);
-            warp_store_rows(stg, p.stage_q_pitch, 64, reinterpret_cast<uint8_t*>(p.y_out),
-                            row_elem < 0 ? -1 : (row_elem + dst_c0 + ch * 16) * 4, lane);
-          }
-#pragma unroll
-          for (int j = 0; j < 4; ++j)
-            qw[s][j] = __byte_perm(__byte_perm(code[4 * j], code[4 * j + 1], 0x0040),
-                                   __byte_perm(code[4 * j + 2], code[4 * j + 3], 0x0040), 0x5410);
+      }
+      // Unrolled by two so both buffers stay in registers; the next unit's TMEM
+      // load is in flight while the current one is converted and stored.
+      while (c_mt < MT) {
+        int n_mt = c_mt, n_ch = c_ch;
+        step(n_mt, n_ch);
+        if (n_mt < MT) tmem_ld16(col(n_mt, n_ch), vb);
+        {
+          const uint4 w = epi_codes16(va, e.m_req512, qmax_f);
+          if (c_row) *reinterpret_cast<uint4*>(c_row + c_ch * chunk_bytes) = w;
         }
-        if (p.q_out && !p.channel_shuffle) {
-          if (c16) {
-            // Channel-blocked codes: lanes hold consecutive pixels, so each
-            // 16-byte store of the warp lands next to its neighbours'.
-            if (valid) {
-#pragma unroll
-              for (int s = 0; s < kSeg; ++s)
-                if (s < nseg)
-                  *reinterpret_cast<uint4*>(p.q_out + c16_row + ((dst_c0 >> 4) + seg + s) * hw_out * 16) =
-                      make_uint4(qw[s][0], qw[s][1], qw[s][2], qw[s][3]);
-            }
-          } else {
-            // NHWC codes of this segment go out as one staged row each.
-#pragma unroll
-            for (int s = 0; s < kSeg; ++s)
-              if (s < nseg)
-                *reinterpret_cast<uint4*>(stg + lane * p.stage_q_pitch + s * 16) = make_uint4(qw[s][0], qw[s][1], qw[s][2], qw[s][3]);
-            warp_store_rows(stg, p.stage_q_pitch, nseg * 16, p.q_out, row_elem < 0 ? -1 : row_elem + dst_c0 + seg * 16, lane);
-          }
+        tmem_wait_ld();
+        if (n_mt >= MT) break;
+        uint8_t* n_row = n_mt == c_mt ? c_row : row_ptr(n_mt);
+        int m2 = n_mt, c2 = n_ch;
+        step(m2, c2);
+        if (m2 < MT) tmem_ld16(col(m2, c2), va);
+        {
+          const uint4 w = epi_codes16(vb, e.m_req512, qmax_f);
+          if (n_row) *reinterpret_cast<uint4*>(n_row + n_ch * chunk_bytes) = w;
         }
+        tmem_wait_ld();
+        c_row = m2 == n_mt ? n_row : row_ptr(m2);
+        c_mt = m2;
+        c_ch = c2;
+      }
+    } else {
+      for (int u = wg; u < n_units; u += n_groups) {
+        const int mt = u / nchunks, ch = u - mt * nchunks;
+        uint32_t v[16];
+        tmem_ld16(e.tbase + mt * p.Npow2 + ch * 16, v);
+        tmem_wait_ld();
+        epi_general16(p, e, stg, lane, mt * 128 + quarter * 32 + lane, ch, v);
       }
     }
     tc_fence_before();
@@ -671,7 +748,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(bars.acc_full(s), 1);
-      mbar_init(bars.acc_empty(s), kEpiWarps * 32);
+      mbar_init(bars.acc_empty(s), (p.a_tma ? kEpiWarps + kLoadWarps : kEpiWarps) * 32);
     }
     mbar_init(bars.drain(), 1);
     *abort_flag = 0;
@@ -699,10 +776,12 @@ __global__ void __launch_bounds__(kConvThreads, 1)
       mma_role_dispatch(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1,
                         WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_MMA});
     __syncwarp();
-  } else if (warp < kFirstEpiWarp) {
+  } else if (warp < kFirstEpiWarp && !p.a_tma) {
     loader_role(p, bars, a_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else {
-    epilogue_role(p, bars, tmem_base, gbase + p.smem_stage_off, it0, it1,
+    // With TMA loading the activations, the copy warps form a third epilogue warpgroup.
+    const int first = p.a_tma ? kFirstLoadWarp : kFirstEpiWarp;
+    epilogue_role(p, bars, tmem_base, gbase + p.smem_stage_off, first, p.a_tma ? kEpiGroups + 1 : kEpiGroups, it0, it1,
                   WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_EPILOGUE});
   }
   tc_fence_before();
