@@ -312,21 +312,29 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
 }
 
 // --------------------------------------------------------------------------
-// Tensor-core issue role (warp 1, lane 0).
+// Tensor-core issue role (warp 1).
 // --------------------------------------------------------------------------
+// Wait taken by every lane of a converged warp; the lanes agree on the outcome.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const WaitCtx& ctx) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, ctx));
+}
+
 constexpr int kUnrollTaps = 9;
 
 template <int KSTEPS, int MT>
 __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t b_base,
                                          uint32_t tmem_base, const uint32_t* tap_a16, int64_t it0, int64_t it1,
                                          const WaitCtx& ctx) {
-  // The issue loop must stay lean: one thread issues every MMA and each extra
-  // instruction, branch or long-latency load per MMA lowers tensor-core
-  // throughput directly.  So the K steps and accumulators per tap are
-  // compile-time (fully unrolled), operand addresses are 32-bit adds of
-  // 16-byte-unit offsets onto the low word of precomputed descriptors
-  // (shared-memory addresses are below 2^18, so the 14-bit address field never
-  // carries), and the per-tap offsets come from shared memory.
+  // The issue loop must stay lean: the whole warp runs it converged and one
+  // elected lane issues each MMA; every extra instruction, branch or
+  // long-latency load per MMA lowers tensor-core throughput directly, the more
+  // so as the epilogue warps compete for the same schedulers.  So the K steps
+  // and accumulators per tap are compile-time (fully unrolled), operand
+  // addresses are 32-bit adds of 16-byte-unit offsets onto the low word of
+  // precomputed descriptors (shared-memory addresses are below 2^18, so the
+  // 14-bit address field never carries), and the per-tap offsets sit in
+  // registers.  Waits are taken by all lanes and agreed on with a vote, so the
+  // warp stays converged even when a wait times out.
   Ring ra{0, 0, static_cast<uint32_t>(p.a_stages)};
   Ring rb{0, 0, static_cast<uint32_t>(p.b_resident ? 1 : p.b_stages)};
   Ring racc{0, 0, static_cast<uint32_t>(p.acc_stages)};
@@ -355,14 +363,14 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
       ++unit_next;
     }
     if (resident && cur != unit) {
-      if (!mbar_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
+      if (!warp_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
       unit = cur;
     }
-    if (!mbar_wait(bars.acc_empty(racc.stage), racc.phase ^ 1u, ctx)) { ok = false; break; }
+    if (!warp_wait(bars.acc_empty(racc.stage), racc.phase ^ 1u, ctx)) { ok = false; break; }
     tc_fence_after();
     const uint32_t d0 = tmem_base + racc.stage * static_cast<uint32_t>(MT) * npow2;
     for (int kb = 0; kb < n_kb && ok; ++kb) {
-      if (!mbar_wait(bars.a_full(ra.stage), ra.phase, ctx)) { ok = false; break; }
+      if (!warp_wait(bars.a_full(ra.stage), ra.phase, ctx)) { ok = false; break; }
       tc_fence_after();
       const uint32_t a_lo_stage = a_lo0 + ra.stage * a_stage16;
       const uint32_t b_lo_kb = b_lo0 + static_cast<uint32_t>(kb * taps) * b_slice16;
@@ -374,7 +382,7 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
           const uint64_t bdesc = b_hi | (b_lo_tap + static_cast<uint32_t>(ks) * b_ks16);
 #pragma unroll
           for (int mt = 0; mt < MT; ++mt)
-            tc_mma_e4m3(d0 + static_cast<uint32_t>(mt) * npow2,
+            tc_mma_e4m3_warp(d0 + static_cast<uint32_t>(mt) * npow2,
                         a_hi | (a_lo_tap + static_cast<uint32_t>(ks) * a_ks16 + static_cast<uint32_t>(mt) * 128u), bdesc,
                         idesc, ks == 0 ? acc0 : 1u);
         }
@@ -391,31 +399,31 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
           if (resident) {
             b_lo_tap = b_lo_kb + static_cast<uint32_t>(t) * b_slice16;
           } else {
-            if (!mbar_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
+            if (!warp_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
             tc_fence_after();
             b_lo_tap = b_lo0 + rb.stage * b_slice16;
           }
           issue_tap(t, a_lo_stage + tap_a16[t], b_lo_tap);
           if (!resident) {
-            tc_commit(bars.b_empty(rb.stage));
+            tc_commit_warp(bars.b_empty(rb.stage));
             rb.advance();
           }
         }
       }
       if (!ok) break;
-      tc_commit(bars.a_empty(ra.stage));
+      tc_commit_warp(bars.a_empty(ra.stage));
       ra.advance();
     }
     if (!ok) break;
-    tc_commit(bars.acc_full(racc.stage));
+    tc_commit_warp(bars.acc_full(racc.stage));
     racc.advance();
     if (resident && (it + 1 >= it1 || unit_next != cur)) {
-      tc_commit(bars.b_empty(rb.stage));
+      tc_commit_warp(bars.b_empty(rb.stage));
       rb.advance();
     }
   }
-  // Drain: wait until every MMA this thread issued has completed.
-  tc_commit(bars.drain());
+  // Drain: wait until every MMA this warp issued has completed.
+  tc_commit_warp(bars.drain());
   mbar_wait_drain(bars.drain(), 0, ctx.limit_ns, ctx.err);
 }
 
@@ -536,7 +544,7 @@ __device__ __forceinline__ void epi_store_codes(const ConvParams& p, const EpiIt
 
 // General unit: int32 sums, fp32 outputs (with the shortcut) and codes, or the
 // per-channel scatter of the channel shuffle.
-__device__ __noinline__ void epi_general16(const ConvParams& p, const EpiItem& e, uint8_t* stg, int lane, int m, int ch,
+__device__ __forceinline__ void epi_general16(const ConvParams& p, const EpiItem& e, uint8_t* stg, int lane, int m, int ch,
                                            const uint32_t* v) {
   bool valid;
   const int pos = epi_pos(p, e, m, valid);
@@ -772,9 +780,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     }
     __syncwarp();
   } else if (warp == 1) {
-    if (lane == 0)
-      mma_role_dispatch(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1,
-                        WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_MMA});
+    mma_role_dispatch(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1,
+                      WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_MMA});
     __syncwarp();
   } else if (warp < kFirstEpiWarp && !p.a_tma) {
     loader_role(p, bars, a_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
