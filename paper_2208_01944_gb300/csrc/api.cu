@@ -178,37 +178,40 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.nph = static_cast<int>(phases.size());
   // Tile shape: MT accumulators of 128 rows; rows mode packs Ht whole output
   // rows of pitch Wh into them.
+  //
+  // Choice of MT: a work item costs a fixed overhead (waits, commits, the
+  // epilogue's per-item set-up) plus, per 128-row accumulator, the larger of its
+  // MMA time and its epilogue time, so few large items beat many small ones
+  // even at some cost in padded rows.  Model (per SM): an M=128, K=32 FP8 MMA
+  // takes max(32 + N/4, N/2) cycles (shared-memory operand reads at 128 B per
+  // cycle, tensor rate), the epilogue about 0.07 ns per accumulator value and an
+  // item 500 ns of overhead.  Double-buffered accumulators come first.
+  const double ns_per_clk = 1.0 / 1.9;
+  const double mma_ns = std::max(32.0 + p.Npow2 / 4.0, p.Npow2 / 2.0) * ns_per_clk;
+  const double slot_ns = std::max(static_cast<double>(p.taps) * (d->Cin_g / 32) * mma_ns, 128.0 * p.Npow2 * 0.07);
   int best_mt = 0, best_ht = 0, best_tpi = 0, best_acc = 0;
-  double best_eff = -1.0, best_halo = 1e30;
+  double best_cost = 0.0;
   for (int MT : {1, 2, 4}) {
     if (flat && (MT > 2 || (c16 && MT > 1))) continue;
     int acc_stages = (2 * MT * p.Npow2 <= 512) ? 2 : ((MT * p.Npow2 <= 512) ? 1 : 0);
     if (acc_stages == 0) continue;
-    double eff, halo;
     int ht = 0, tpi = 0;
     if (flat) {
-      const int64_t hw = static_cast<int64_t>(Ho) * Wo;
-      const int64_t tiles = (hw + MT * 128 - 1) / (MT * 128);
-      eff = static_cast<double>(hw) / (tiles * MT * 128.0);
-      halo = 1.0;
+      tpi = static_cast<int>((static_cast<int64_t>(Ho) * Wo + MT * 128 - 1) / (MT * 128));
     } else {
       const int ht_max = (MT * 128) / Wh;
       if (ht_max < 1) continue;
       tpi = (Ho + ht_max - 1) / ht_max;
       ht = (Ho + tpi - 1) / tpi;
-      eff = static_cast<double>(Ho) * Wo / (static_cast<double>(tpi) * MT * 128.0);
-      halo = static_cast<double>(ht + rmax - rmin) / ht;
     }
-    // Prefer double-buffered accumulators, then tile efficiency, then less halo.
-    const double score_eff = eff + (acc_stages == 2 ? 1.0 : 0.0);
-    const bool better = score_eff > best_eff + 0.02 || (std::fabs(score_eff - best_eff) <= 0.02 && halo < best_halo - 1e-9);
-    if (best_mt == 0 || better) {
+    const double cost = static_cast<double>(tpi) * (500.0 + MT * slot_ns);
+    const bool better = best_mt == 0 || acc_stages > best_acc || (acc_stages == best_acc && cost < best_cost * 0.98);
+    if (better) {
       best_mt = MT;
       best_ht = ht;
       best_tpi = tpi;
       best_acc = acc_stages;
-      best_eff = score_eff;
-      best_halo = halo;
+      best_cost = cost;
     }
   }
   if (best_mt == 0) {

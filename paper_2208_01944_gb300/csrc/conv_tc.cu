@@ -380,11 +380,16 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
 #pragma unroll
         for (int ks = 0; ks < KSTEPS; ++ks) {
           const uint64_t bdesc = b_hi | (b_lo_tap + static_cast<uint32_t>(ks) * b_ks16);
-#pragma unroll
-          for (int mt = 0; mt < MT; ++mt)
-            tc_mma_e4m3_warp(d0 + static_cast<uint32_t>(mt) * npow2,
-                        a_hi | (a_lo_tap + static_cast<uint32_t>(ks) * a_ks16 + static_cast<uint32_t>(mt) * 128u), bdesc,
-                        idesc, ks == 0 ? acc0 : 1u);
+          const uint32_t a_lo = a_lo_tap + static_cast<uint32_t>(ks) * a_ks16;
+          const uint32_t acc = ks == 0 ? acc0 : 1u;
+          if constexpr (MT == 4) {
+            tc_mma4_e4m3_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u),
+                              a_hi | (a_lo + 256u), a_hi | (a_lo + 384u), bdesc, idesc, acc);
+          } else if constexpr (MT == 2) {
+            tc_mma2_e4m3_warp(d0, d0 + npow2, a_hi | a_lo, a_hi | (a_lo + 128u), bdesc, idesc, acc);
+          } else {
+            tc_mma_e4m3_warp(d0, a_hi | a_lo, bdesc, idesc, acc);
+          }
         }
       };
       if (resident && taps <= kUnrollTaps) {

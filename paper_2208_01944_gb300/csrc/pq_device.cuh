@@ -214,6 +214,30 @@ __device__ __forceinline__ void tc_mma_e4m3_warp(uint32_t d_tmem, uint64_t a_des
       : "memory");
 }
 
+// MT MMAs sharing one B operand and accumulate flag, one election for the group.
+__device__ __forceinline__ void tc_mma2_e4m3_warp(uint32_t d0, uint32_t d1, uint64_t a0, uint64_t a1, uint64_t b_desc,
+                                                  uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p, e;\nelect.sync _|e, 0xffffffff;\nsetp.ne.b32 p, %6, 0;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %2, %4, %5, p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%1], %3, %4, %5, p;\n}" ::"r"(d0),
+      "r"(d1), "l"(a0), "l"(a1), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_mma4_e4m3_warp(uint32_t d0, uint32_t d1, uint32_t d2, uint32_t d3, uint64_t a0,
+                                                  uint64_t a1, uint64_t a2, uint64_t a3, uint64_t b_desc,
+                                                  uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p, e;\nelect.sync _|e, 0xffffffff;\nsetp.ne.b32 p, %10, 0;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %4, %8, %9, p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%1], %5, %8, %9, p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%2], %6, %8, %9, p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%3], %7, %8, %9, p;\n}" ::"r"(d0),
+      "r"(d1), "r"(d2), "r"(d3), "l"(a0), "l"(a1), "l"(a2), "l"(a3), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 __device__ __forceinline__ void tc_commit_warp(uint32_t bar) {
   asm volatile(
       "{\n.reg .pred e;\nelect.sync _|e, 0xffffffff;\n"
