@@ -50,8 +50,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   return ok != 0;
 }
 
-// Shared state every role of a CTA consults while waiting: a CTA-wide abort
-// flag (set by whichever role times out first) and the wait limit.
+// As mbar_try_wait, but the thread may stay suspended (without taking issue
+// slots) for up to `suspend_ns` while the phase is incomplete; it resumes as
+// soon as the phase completes.
+__device__ __forceinline__ bool mbar_try_wait_suspend(uint32_t bar, uint32_t parity, uint32_t suspend_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n.reg .pred p;\n"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
+      "selp.u32 %0, 1, 0, p;\n}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(suspend_ns)
+      : "memory");
+  return ok != 0;
+}
+
 struct WaitCtx {
   volatile int* abort_flag;  // shared memory
   unsigned int* err;         // device error word (global)
@@ -66,22 +79,24 @@ struct WaitCtx {
 // so a limit never ends earlier than asked.
 __device__ __forceinline__ uint64_t limit_cycles(uint64_t limit_ns) { return limit_ns * 5u / 2u; }
 
+// Suspension per try_wait of a blocking wait: waiting warps leave the issue
+// slots to working ones, and the abort flag and the limit are still checked
+// every few microseconds.
+constexpr uint32_t kSuspendNs = 4000;
+
 // Wait until the phase with the given parity of `bar` has completed.  Returns
 // false (after recording PQ_ERR_TIMEOUT and raising the abort flag) when the
 // wait exceeds ctx.limit_ns, or when another role of the CTA already aborted.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const WaitCtx& ctx) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
-  uint32_t n = 0;
   while (true) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((++n & 63u) == 0) {
-      if (*ctx.abort_flag) return false;
-      if (static_cast<uint64_t>(clock64() - t0) > limit_cycles(ctx.limit_ns)) {
-        atomicOr(ctx.err, PQ_ERR_TIMEOUT | ctx.err_bits);
-        *ctx.abort_flag = 1;
-        return false;
-      }
+    if (mbar_try_wait_suspend(bar, parity, kSuspendNs)) return true;
+    if (*ctx.abort_flag) return false;
+    if (static_cast<uint64_t>(clock64() - t0) > limit_cycles(ctx.limit_ns)) {
+      atomicOr(ctx.err, PQ_ERR_TIMEOUT | ctx.err_bits);
+      *ctx.abort_flag = 1;
+      return false;
     }
   }
 }
