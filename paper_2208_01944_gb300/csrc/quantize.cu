@@ -65,29 +65,39 @@ __global__ void __launch_bounds__(256) pq_quantize_scalar(const float* __restric
   }
 }
 
-// Channel-blocked output [N][C/16][HW][16]: grid.y walks the (image, 16-channel
-// block) planes, grid.x the pixels of a plane.  A thread reads one pixel's 16
-// channels (64 bytes of the NHWC input) and writes their 16 codes; consecutive
-// threads take consecutive pixels, so the 16-byte stores of a warp are contiguous.
-__global__ void __launch_bounds__(256) pq_quantize_c16(const float4* __restrict__ x, uint4* __restrict__ q,
-                                                       int64_t planes, int64_t HW, int C16, int blocks_per_group,
-                                                       int qmax, const __grid_constant__ QuantArgs args) {
-  for (int64_t plane = blockIdx.y; plane < planes; plane += gridDim.y) {
-    const int64_t n = plane / C16;
-    const int j = static_cast<int>(plane - n * C16);
-    const float inv = args.inv_s[j / blocks_per_group];
-    const float4* src_img = x + (n * HW * C16 + j) * 4;  // pixel hw of this block at src_img + hw * C16 * 4
-    uint4* dst = q + plane * HW;
-    for (int64_t hw = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; hw < HW;
-         hw += static_cast<int64_t>(gridDim.x) * blockDim.x) {
-      const float4* s4 = src_img + hw * C16 * 4;
+// Channel-blocked output [N][C/16][HW][16].  A warp takes 8 consecutive pixels
+// x 4 consecutive 16-channel blocks of one image: lane (p, j) reads the 64 bytes
+// of its pixel's block (the warp reads 8 runs of 256 contiguous bytes) and writes
+// the block's 16 codes (the warp writes 4 runs of 128 contiguous bytes, one per
+// block).  Consecutive warps take the next 4 blocks of the same pixels, so whole
+// pixel rows are read by neighbouring warps at about the same time.  A grid of a
+// few blocks per SM, striding over the (image, pixel group, block group) units,
+// keeps enough loads in flight for the HBM bandwidth.
+__global__ void __launch_bounds__(256) pq_quantize_c16(const float4* __restrict__ x, uint4* __restrict__ q, int64_t N,
+                                                       int64_t HW, int C16, int blocks_per_group, int qmax,
+                                                       const __grid_constant__ QuantArgs args) {
+  const int lane = threadIdx.x & 31;
+  const int jj = lane & 3, pp = lane >> 2;
+  const int64_t pix_groups = (HW + 7) / 8;
+  const int jgroups = (C16 + 3) / 4;
+  const int64_t units = N * pix_groups * jgroups;
+  const int64_t wstride = static_cast<int64_t>(gridDim.x) * (blockDim.x >> 5);
+  for (int64_t u = static_cast<int64_t>(blockIdx.x) * (blockDim.x >> 5) + (threadIdx.x >> 5); u < units; u += wstride) {
+    const int jg = static_cast<int>(u % jgroups);
+    const int64_t r = u / jgroups;
+    const int64_t n = r / pix_groups;
+    const int64_t hw = (r - n * pix_groups) * 8 + pp;
+    const int j = jg * 4 + jj;
+    if (hw < HW && j < C16) {
+      const float inv = args.inv_s[j / blocks_per_group];
+      const float4* s4 = x + ((n * HW + hw) * C16 + j) * 4;
       const float4 a = __ldcs(s4), b = __ldcs(s4 + 1), c = __ldcs(s4 + 2), d = __ldcs(s4 + 3);
       uint4 out;
       out.x = quant4(a, inv, qmax);
       out.y = quant4(b, inv, qmax);
       out.z = quant4(c, inv, qmax);
       out.w = quant4(d, inv, qmax);
-      __stcs(dst + hw, out);
+      __stcs(q + (n * C16 + j) * HW + hw, out);
     }
   }
 }
@@ -97,12 +107,16 @@ int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G
   QuantArgs args;
   for (int g = 0; g < G; ++g) args.inv_s[g] = inv_s[g];
   const int C16 = G * Cg / 16;
-  const int64_t planes = N * C16;
-  if (planes == 0 || HW == 0) return 0;
-  const unsigned gy = static_cast<unsigned>(planes < 65535 ? planes : 65535);
-  const unsigned gx = static_cast<unsigned>((HW + 255) / 256);
-  pq_quantize_c16<<<dim3(gx, gy), 256, 0, stream>>>(reinterpret_cast<const float4*>(x), reinterpret_cast<uint4*>(q),
-                                                     planes, HW, C16, Cg / 16, (1 << bits) - 1, args);
+  if (N == 0 || HW == 0) return 0;
+  const int64_t warps = N * ((HW + 7) / 8) * ((C16 + 3) / 4);
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int64_t want = (warps + 7) / 8;  // 8 warps per block
+  const int64_t cap = static_cast<int64_t>(sms) * 4;
+  const unsigned grid = static_cast<unsigned>(want < cap ? want : cap);
+  pq_quantize_c16<<<grid, 256, 0, stream>>>(reinterpret_cast<const float4*>(x), reinterpret_cast<uint4*>(q), N, HW, C16,
+                                            Cg / 16, (1 << bits) - 1, args);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }
 

@@ -105,7 +105,9 @@ def test_layer_fused_matches_oracle(B, c, fmt):
     assert_layer_parity(c, ref, got)
 
 
-@pytest.mark.parametrize("shape,G,bits", [((2, 7, 9, 64), 4, 2), ((3, 5, 6, 3 * 16), 3, 4), ((1, 1, 1, 32), 1, 8)])
+@pytest.mark.parametrize("shape,G,bits", [((2, 7, 9, 64), 4, 2), ((3, 5, 6, 3 * 16), 3, 4), ((1, 1, 1, 32), 1, 8),
+                                         # several 256-channel ranges and ragged pixel tiles; a ragged range
+                                         ((2, 11, 13, 768), 4, 2), ((1, 40, 40, 400), 5, 3)])
 def test_quantize_act_c16_matches_oracle(B, shape, G, bits):
     from layer_cases import c16_to_nhwc
 
