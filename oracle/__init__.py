@@ -67,6 +67,10 @@ def _declare(lib):
     lib.oracle_inv_step.argtypes = [ctypes.c_float]
     lib.oracle_epilogue_scales.restype = _I32
     lib.oracle_epilogue_scales.argtypes = [_I32, _P, _P, ctypes.c_double, _P, _I32, _I32, _P, _P, _P]
+    lib.oracle_conv2d_f32.argtypes = [_P, _P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _I32, _I32, _I32]
+    lib.oracle_maxpool_f32.argtypes = [_P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _I32]
+    lib.oracle_avgpool_f32.argtypes = [_P, _P, _I64, _I64, _I64, _I32]
+    lib.oracle_linear_f32.argtypes = [_P, _P, _P, _I64, _I32, _I32]
     return lib
 
 
@@ -245,3 +249,49 @@ def layer(x_codes: np.ndarray, wq: np.ndarray, stride: int, pad: int, m_out, m_r
     G = wq.shape[0]
     acc = group_conv(x_codes, wq, stride, pad, L=L)
     return epilogue(acc, G, m_out, m_req, kind, shift, perm, shortcut, relu, bits_out, L=L)
+
+
+# ---------------------------------------------------------------------------
+# Full-precision layers around the PalQuant body (the paper keeps the first and
+# last layers in full precision, Sec. 5).  Fixed summation orders, see the C file.
+# ---------------------------------------------------------------------------
+def conv2d_f32(x: np.ndarray, w: np.ndarray, stride: int, pad: int, relu: bool = False, L=None) -> np.ndarray:
+    """NHWC fp32 convolution, w [Cout,k,k,Cin]; fmaf over (kh, kw, ci) in order."""
+    L = L or lib()
+    x, w = _f32(x), _f32(w)
+    N, H, W, Ci = x.shape
+    Co, k, k2, Ci2 = w.shape
+    assert k == k2 and Ci == Ci2
+    Ho, Wo = out_dim(H, k, stride, pad), out_dim(W, k, stride, pad)
+    y = np.empty((N, Ho, Wo, Co), dtype=np.float32)
+    L.oracle_conv2d_f32(_ptr(x), _ptr(w), _ptr(y), N, H, W, Ci, Co, k, stride, pad, int(bool(relu)))
+    return y
+
+
+def maxpool_f32(x: np.ndarray, k: int, stride: int, pad: int, L=None) -> np.ndarray:
+    L = L or lib()
+    x = _f32(x)
+    N, H, W, C = x.shape
+    y = np.empty((N, out_dim(H, k, stride, pad), out_dim(W, k, stride, pad), C), dtype=np.float32)
+    L.oracle_maxpool_f32(_ptr(x), _ptr(y), N, H, W, C, k, stride, pad)
+    return y
+
+
+def avgpool_f32(x: np.ndarray, L=None) -> np.ndarray:
+    L = L or lib()
+    x = _f32(x)
+    N, H, W, C = x.shape
+    y = np.empty((N, C), dtype=np.float32)
+    L.oracle_avgpool_f32(_ptr(x), _ptr(y), N, H, W, C)
+    return y
+
+
+def linear_f32(x: np.ndarray, w: np.ndarray, L=None) -> np.ndarray:
+    L = L or lib()
+    x, w = _f32(x), _f32(w)
+    N, Ci = x.shape
+    Co = w.shape[0]
+    assert w.shape == (Co, Ci)
+    y = np.empty((N, Co), dtype=np.float32)
+    L.oracle_linear_f32(_ptr(x), _ptr(w), _ptr(y), N, Ci, Co)
+    return y

@@ -39,6 +39,18 @@
  *   oracle_weight_step       pinned (half-normal / Gaussian closed forms,
  *                            statistical)
  *   oracle_epilogue_scales   pinned (hand cases)
+ *   oracle_conv2d_f32,
+ *   oracle_maxpool_f32,
+ *   oracle_avgpool_f32,
+ *   oracle_linear_f32        pinned (float64 library convolution / pooling /
+ *                            matmul within the fp32 error bound; hand cases;
+ *                            max pooling exactly)
+ *
+ * The full-precision functions serve the ResNet-18-shaped network around the
+ * PalQuant layers (the paper keeps the first and the last layer in full
+ * precision, Sec. 5).  Each sums in one fixed order with one fused
+ * multiply-add per term (fmaf, a single IEEE rounding), so that the values
+ * feeding the next quantiser are defined to the bit.
  */
 #include <math.h>
 #include <stdint.h>
@@ -323,4 +335,92 @@ int oracle_epilogue_scales(int G, const float* s_w, const float* s_a, double alp
         if (s_next) m_req[g] = (float)(m / (double)s_next[dst_group[g]]);
     }
     return 0;
+}
+
+/* ---------------------------------------------------------------------- */
+/* Full-precision layers around the PalQuant body (Sec. 5: the first and  */
+/* the last layer are not quantised).                                      */
+/* ---------------------------------------------------------------------- */
+
+/* Direct NHWC convolution, weights [Cout][k][k][Cin]: every output starts
+ * from 0 and adds fmaf(x, w, acc) over (kh, kw, ci) in that order, skipping
+ * taps outside the image (zero padding); optional ReLU (fmaxf, NaN -> 0). */
+void oracle_conv2d_f32(const float* x, const float* w, float* y, int64_t N, int64_t H, int64_t W, int Cin,
+                       int Cout, int k, int s, int p, int relu) {
+    const int64_t Ho = out_dim(H, k, s, p), Wo = out_dim(W, k, s, p);
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int64_t n = 0; n < N; ++n) {
+        for (int64_t oh = 0; oh < Ho; ++oh) {
+            for (int64_t ow = 0; ow < Wo; ++ow) {
+                for (int co = 0; co < Cout; ++co) {
+                    float acc = 0.0f;
+                    for (int kh = 0; kh < k; ++kh) {
+                        const int64_t ih = oh * s - p + kh;
+                        if (ih < 0 || ih >= H) continue;
+                        for (int kw = 0; kw < k; ++kw) {
+                            const int64_t iw = ow * s - p + kw;
+                            if (iw < 0 || iw >= W) continue;
+                            const float* xp = x + ((n * H + ih) * W + iw) * Cin;
+                            const float* wp = w + (((int64_t)co * k + kh) * k + kw) * Cin;
+                            for (int ci = 0; ci < Cin; ++ci) acc = fmaf(xp[ci], wp[ci], acc);
+                        }
+                    }
+                    if (relu) acc = fmaxf(acc, 0.0f);
+                    y[((n * Ho + oh) * Wo + ow) * Cout + co] = acc;
+                }
+            }
+        }
+    }
+}
+
+/* Max pooling over the in-image taps of each k x k window (padding taps are
+ * ignored), taken with fmaxf in (kh, kw) order starting from -infinity. */
+void oracle_maxpool_f32(const float* x, float* y, int64_t N, int64_t H, int64_t W, int C, int k, int s, int p) {
+    const int64_t Ho = out_dim(H, k, s, p), Wo = out_dim(W, k, s, p);
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int64_t n = 0; n < N; ++n) {
+        for (int64_t oh = 0; oh < Ho; ++oh) {
+            for (int64_t ow = 0; ow < Wo; ++ow) {
+                for (int c = 0; c < C; ++c) {
+                    float m = -INFINITY;
+                    for (int kh = 0; kh < k; ++kh) {
+                        const int64_t ih = oh * s - p + kh;
+                        if (ih < 0 || ih >= H) continue;
+                        for (int kw = 0; kw < k; ++kw) {
+                            const int64_t iw = ow * s - p + kw;
+                            if (iw < 0 || iw >= W) continue;
+                            m = fmaxf(m, x[((n * H + ih) * W + iw) * C + c]);
+                        }
+                    }
+                    y[((n * Ho + oh) * Wo + ow) * C + c] = m;
+                }
+            }
+        }
+    }
+}
+
+/* Global average pooling: the sum over (h, w) in storage order from 0, then
+ * one division by H * W. */
+void oracle_avgpool_f32(const float* x, float* y, int64_t N, int64_t H, int64_t W, int C) {
+#pragma omp parallel for schedule(static)
+    for (int64_t n = 0; n < N; ++n) {
+        for (int c = 0; c < C; ++c) {
+            float acc = 0.0f;
+            for (int64_t i = 0; i < H * W; ++i) acc = acc + x[(n * H * W + i) * C + c];
+            y[n * C + c] = acc / (float)(H * W);
+        }
+    }
+}
+
+/* Fully connected layer without bias, weights [Cout][Cin]: each output is
+ * fmaf(x_i, w_oi, acc) over i in order from 0. */
+void oracle_linear_f32(const float* x, const float* w, float* y, int64_t N, int Cin, int Cout) {
+#pragma omp parallel for collapse(2) schedule(static)
+    for (int64_t n = 0; n < N; ++n) {
+        for (int o = 0; o < Cout; ++o) {
+            float acc = 0.0f;
+            for (int i = 0; i < Cin; ++i) acc = fmaf(x[n * Cin + i], w[(int64_t)o * Cin + i], acc);
+            y[n * Cout + o] = acc;
+        }
+    }
 }

@@ -56,3 +56,30 @@ def random_codes(shape, bits: int, gen: torch.Generator, signed: bool = False) -
         lo, hi = -(1 << (bits - 1)), (1 << (bits - 1))
         return torch.randint(lo, hi, tuple(shape), generator=gen, dtype=torch.int16).numpy().astype(np.int8)
     return torch.randint(0, 1 << bits, tuple(shape), generator=gen, dtype=torch.int16).numpy().astype(np.uint8)
+
+
+def resnet18_inputs(N: int, H: int = 224, W: int = 224, G: int = 2, widths=(64, 128, 256, 512), classes: int = 1000,
+                    seed: int = 0):
+    """(x, params) for the ResNet-18-shaped PalQuant network.
+
+    x: images N(0, 1), NHWC [N, H, W, 3].  params: name -> fp32 weights, drawn after x
+    in this order: "stem" [G*widths[0], 7, 7, 3] N(0, 2/147); then for stage s = 1..4
+    and block b = 1, 2: "s{s}b{b}.conv1" [G, w, 3, 3, cin], "s{s}b{b}.conv2"
+    [G, w, 3, 3, w] and, in the first block of stages 2-4 (stride 2, channels change),
+    "s{s}b{b}.down" [G, w, 1, 1, cin], all He-initialised per group (w = widths[s-1],
+    cin = the block's per-group input width); last "fc" [classes, G*widths[-1]]
+    N(0, 1/fan_in)."""
+    gen = generator(seed)
+    x = normal((N, H, W, 3), gen)
+    params = {"stem": normal((G * widths[0], 7, 7, 3), gen, math.sqrt(2.0 / 147.0))}
+    cin = widths[0]
+    for s, w in enumerate(widths):
+        for b in range(2):
+            name = f"s{s + 1}b{b + 1}"
+            params[name + ".conv1"] = he_weights(G, w, 3, 3, cin, gen)
+            params[name + ".conv2"] = he_weights(G, w, 3, 3, w, gen)
+            if s > 0 and b == 0:
+                params[name + ".down"] = he_weights(G, w, 1, 1, cin, gen)
+            cin = w
+    params["fc"] = normal((classes, G * widths[-1]), gen, math.sqrt(1.0 / (G * widths[-1])))
+    return x, params
