@@ -243,6 +243,41 @@ pq_status palquant_set_wait_limit_ns(uint64_t ns);
 pq_status palquant_watchdog_selftest(uint64_t limit_ns, pq_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
+/* Full-precision layers around the PalQuant body of a network.  The paper   */
+/* keeps the first and the last layer in full precision (Sec. 5); these are  */
+/* not part of the PalQuant method itself.  Each output is summed in one     */
+/* fixed order, with one fused multiply-add (a single IEEE rounding) per     */
+/* term, so values do not depend on the launch shape.  All tensors are fp32  */
+/* device buffers owned by the caller; calls are asynchronous on `stream`.   */
+/* ------------------------------------------------------------------------ */
+
+/* Direct convolution: x NHWC [N,H,W,Cin], w [Cout][k][k][Cin], y NHWC
+ * [N,Ho,Wo,Cout] (16-byte aligned) with Ho = (H + 2 pad - k) / stride + 1.
+ * y[n,oh,ow,co] = fma-sum over (kh, kw, ci) in that order, starting from 0, of
+ * x[n, oh*stride - pad + kh, ow*stride - pad + kw, ci] * w[co,kh,kw,ci], taps
+ * outside the image skipped (zero padding); then max(y, 0) if relu.  Cout must
+ * be a multiple of 16; pad < k.  PQ_EINVAL otherwise. */
+pq_status palquant_conv2d_f32(const float* x_dev, const float* w_dev, float* y_dev, int64_t N, int32_t H, int32_t W,
+                              int32_t Cin, int32_t Cout, int32_t k, int32_t stride, int32_t pad, int32_t relu,
+                              pq_stream_t stream);
+
+/* Max pooling, NHWC: y[n,oh,ow,c] = max over the in-image taps of the k x k
+ * window at (oh*stride - pad, ow*stride - pad) (padding taps are ignored);
+ * pad < k. */
+pq_status palquant_maxpool2d_f32(const float* x_dev, float* y_dev, int64_t N, int32_t H, int32_t W, int32_t C,
+                                 int32_t k, int32_t stride, int32_t pad, pq_stream_t stream);
+
+/* Global average pooling: y[n,c] = (sum over h, w in storage order of
+ * x[n,h,w,c]) / (H W), x NHWC, y [N,C]. */
+pq_status palquant_avgpool_f32(const float* x_dev, float* y_dev, int64_t N, int32_t H, int32_t W, int32_t C,
+                               pq_stream_t stream);
+
+/* Fully connected layer without bias: y[n,o] = fma-sum over i in order of
+ * x[n,i] w[o,i]; x [N,Cin], w [Cout][Cin], y [N,Cout]. */
+pq_status palquant_linear_f32(const float* x_dev, const float* w_dev, float* y_dev, int64_t N, int32_t Cin,
+                              int32_t Cout, pq_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
 /* Introspection (host only; no GPU needed).                                */
 /* ------------------------------------------------------------------------ */
 

@@ -28,6 +28,7 @@ EXPORTS = [
     "palquant_pack_weights_host", "palquant_pack_weights", "palquant_pack_weight_codes_host",
     "palquant_unpack_weight_codes_host", "palquant_quantize_act", "palquant_group_conv", "palquant_layer_fused",
     "palquant_sync_check", "palquant_set_wait_limit_ns", "palquant_watchdog_selftest", "palquant_conv_plan",
+    "palquant_conv2d_f32", "palquant_maxpool2d_f32", "palquant_avgpool_f32", "palquant_linear_f32",
 ]
 
 
@@ -103,6 +104,12 @@ def _load():
     L.palquant_watchdog_selftest.argtypes = [ctypes.c_uint64, _P]
     L.palquant_conv_plan.restype = _I32
     L.palquant_conv_plan.argtypes = [ctypes.POINTER(LayerDesc), ctypes.POINTER(ConvPlan)]
+    for name, args in (("palquant_conv2d_f32", [_P, _P, _P, _I64] + [_I32] * 8 + [_P]),
+                       ("palquant_maxpool2d_f32", [_P, _P, _I64] + [_I32] * 6 + [_P]),
+                       ("palquant_avgpool_f32", [_P, _P, _I64, _I32, _I32, _I32, _P]),
+                       ("palquant_linear_f32", [_P, _P, _P, _I64, _I32, _I32, _P])):
+        getattr(L, name).restype = _I32
+        getattr(L, name).argtypes = args
     return L
 
 
@@ -278,3 +285,23 @@ def palquant_conv_plan(d: LayerDesc) -> ConvPlan:
     if st not in (PQ_OK, PQ_EUNSUPPORTED):
         raise PalquantError(st, "palquant_conv_plan")
     return plan
+
+
+# Full-precision layers around the PalQuant body (first and last layers of a network).
+def palquant_conv2d_f32(x_dev, w_dev, y_dev, N, H, W, Cin, Cout, k, stride, pad, relu=False, stream=None):
+    _check(lib.palquant_conv2d_f32(_ptr(x_dev), _ptr(w_dev), _ptr(y_dev), N, H, W, Cin, Cout, k, stride, pad,
+                                   int(bool(relu)), _stream(stream)), "palquant_conv2d_f32")
+
+
+def palquant_maxpool2d_f32(x_dev, y_dev, N, H, W, C, k, stride, pad, stream=None):
+    _check(lib.palquant_maxpool2d_f32(_ptr(x_dev), _ptr(y_dev), N, H, W, C, k, stride, pad, _stream(stream)),
+           "palquant_maxpool2d_f32")
+
+
+def palquant_avgpool_f32(x_dev, y_dev, N, H, W, C, stream=None):
+    _check(lib.palquant_avgpool_f32(_ptr(x_dev), _ptr(y_dev), N, H, W, C, _stream(stream)), "palquant_avgpool_f32")
+
+
+def palquant_linear_f32(x_dev, w_dev, y_dev, N, Cin, Cout, stream=None):
+    _check(lib.palquant_linear_f32(_ptr(x_dev), _ptr(w_dev), _ptr(y_dev), N, Cin, Cout, _stream(stream)),
+           "palquant_linear_f32")

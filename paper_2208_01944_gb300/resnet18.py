@@ -1,0 +1,238 @@
+"""ResNet-18-shaped PalQuant network on one GPU, driven through the C ABI.
+
+The paper evaluates PalQuant on ResNet-18 (Sec. 5): every body convolution becomes a
+PalQuant layer with G groups of B-bit codes (Sec. 4.1), a cyclic permutation moves
+each block's output groups on (Sec. 4.2, Eq. 6-8), and the first and last layers stay
+in full precision (Sec. 5).  The paper's network figure is not available; this driver
+takes the following reading:
+
+* stem: 7x7 stride-2 pad-3 fp32 convolution (3 -> G*w_1 channels) + ReLU, then 3x3
+  stride-2 pad-1 max pooling; the pooled tensor is quantised once into codes;
+* four stages of two basic blocks (per-group widths w_1..w_4).  In block (X, Q):
+    conv1  PalQuant 3x3 (stride 2 in the first block of stages 2-4), ReLU, no
+           permutation, codes out (requantised with conv2's input steps);
+    down   (first block of stages 2-4) PalQuant 1x1 with the block's stride on Q,
+           no ReLU, no permutation, fp32 out: the shortcut;
+    conv2  PalQuant 3x3 on conv1's codes + shortcut (down's output, else X), ReLU,
+           cyclic permutation; fp32 out (the next block's X) and, fused in the same
+           epilogue, the next block's codes (multiplier fl(1/s) of the destination
+           group's input step);
+* global average pooling and an fp32 FC layer.
+
+Every step runs in the library's kernels; this module only owns buffers, derives
+per-layer multipliers through palquant_epilogue_scales and launches the calls on one
+stream, with no host synchronisation inside forward() (which can be captured in a
+CUDA graph).  Codes between layers use the channel-blocked layout (PQ_CODES_C16).
+"""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+from . import binding as B
+
+
+def _out(n: int, k: int, s: int, p: int) -> int:
+    return (n + 2 * p - k) // s + 1
+
+
+class PalQuantResNet18:
+    def __init__(self, params: dict, N: int, H: int = 224, W: int = 224, G: int = 2, widths=(64, 128, 256, 512),
+                 classes: int = 1000, bits: int = 2, device="cuda:0", stream: torch.cuda.Stream | None = None):
+        self.dev = torch.device(device)
+        self.N, self.H, self.W, self.G, self.bits, self.classes = N, H, W, G, bits, classes
+        self.stream = stream or torch.cuda.Stream(device=self.dev)
+        fmt = B.PQ_CODES_C16
+        f32 = dict(dtype=torch.float32, device=self.dev)
+        u8 = dict(dtype=torch.uint8, device=self.dev)
+        self.params = params
+        C0 = G * widths[0]
+        self.Hs, self.Ws = _out(H, 7, 2, 3), _out(W, 7, 2, 3)
+        self.Hp, self.Wp = _out(self.Hs, 3, 2, 1), _out(self.Ws, 3, 2, 1)
+        self.C0 = C0
+        self.w_stem = torch.from_numpy(np.ascontiguousarray(params["stem"])).to(self.dev)
+        self.w_fc = torch.from_numpy(np.ascontiguousarray(params["fc"])).to(self.dev)
+        self.stem_out = torch.empty((N, self.Hs, self.Ws, C0), **f32)
+        self.pool = torch.empty((N, self.Hp, self.Wp, C0), **f32)
+        self.in_codes = torch.empty((N, self.Hp, self.Wp, C0), **u8)
+        self.blocks = []
+        Hc, Wc, cin = self.Hp, self.Wp, widths[0]
+        for s, w in enumerate(widths):
+            for b in range(2):
+                name = f"s{s + 1}b{b + 1}"
+                stride = 2 if (s > 0 and b == 0) else 1
+                Ho, Wo = _out(Hc, 3, stride, 1), _out(Wc, 3, stride, 1)
+                blk = dict(name=name, stride=stride, cin=cin, w=w, H=Hc, W=Wc, Ho=Ho, Wo=Wo,
+                           down=(name + ".down") in params)
+                blk["d1"] = B.layer_desc(N, Hc, Wc, G, cin, w, 3, stride, 1, bits, bits, bits, 1, code_format=fmt)
+                blk["d2"] = B.layer_desc(N, Ho, Wo, G, w, w, 3, 1, 1, bits, bits, bits, 1, code_format=fmt)
+                if blk["down"]:
+                    blk["dd"] = B.layer_desc(N, Hc, Wc, G, cin, w, 1, stride, 0, bits, bits, bits, 0, code_format=fmt)
+                    blk["down_out"] = torch.empty((N, Ho, Wo, G * w), **f32)
+                blk["mid_codes"] = torch.empty((N, Ho, Wo, G * w), **u8)
+                blk["out"] = torch.empty((N, Ho, Wo, G * w), **f32)
+                blk["out_codes"] = torch.empty((N, Ho, Wo, G * w), **u8)
+                for key, d in (("wp1", blk["d1"]), ("wp2", blk["d2"])) + ((("wpd", blk["dd"]),) if blk["down"] else ()):
+                    blk[key] = torch.empty(B.palquant_packed_weight_bytes(d), **u8)
+                self.blocks.append(blk)
+                Hc, Wc, cin = Ho, Wo, w
+        self.Hl, self.Wl, self.Cl = Hc, Wc, G * cin
+        self.avg = torch.empty((N, self.Cl), **f32)
+        self.logits = torch.empty((N, classes), **f32)
+        self.no_shuffle = B.shuffle(0, 0)
+        self.cyclic = B.shuffle(1, 1)
+        self.ones = np.ones(G, dtype=np.float32)
+        self.steps = None
+        self.graph = None
+
+    # --------------------------------------------------------------- set-up
+    def _inv(self, s, shuf=None):
+        """fl(1/s[dst(g)]) per source group g, computed by the library in double."""
+        return B.palquant_epilogue_scales(self.G, self.ones, self.ones, 1.0, s, shuf or self.no_shuffle)[1]
+
+    def _act_steps(self, t: torch.Tensor, Cg: int) -> np.ndarray:
+        N, H, W, C = t.shape
+        nbytes = B.palquant_act_steps_scratch_bytes(N * H * W, self.G)
+        scratch = torch.empty(nbytes, dtype=torch.uint8, device=self.dev)
+        return B.palquant_act_steps(t, N, H, W, self.G, Cg, self.bits, scratch, nbytes, stream=self.stream)
+
+    def calibrate(self, x_dev: torch.Tensor) -> dict:
+        """Steps of every PalQuant layer from one fp32 pass over x (LSQ initialisation:
+        weights from their own values, activations from the tensor entering the layer)."""
+        G, bits, st = self.G, self.bits, {}
+        s = self.stream
+        self._stem(x_dev)
+        first = self.blocks[0]["name"]
+        st[first + ".in"] = self._act_steps(self.pool, self.C0 // G)
+        for i, blk in enumerate(self.blocks):
+            n = blk["name"]
+            st[n + ".conv1.w"] = B.palquant_weight_steps(self.params[n + ".conv1"], blk["d1"])
+            st[n + ".conv2.w"] = B.palquant_weight_steps(self.params[n + ".conv2"], blk["d2"])
+            if blk["down"]:
+                st[n + ".down.w"] = B.palquant_weight_steps(self.params[n + ".down"], blk["dd"])
+        # activation steps layer by layer: each needs the previous layers' codes
+        self.steps = st
+        for i, blk in enumerate(self.blocks):
+            n = blk["name"]
+            self._pack(blk, st)
+            self._scales(blk, st)
+            if i == 0:
+                B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, G, self.C0 // G, bits,
+                                        self._inv(st[n + ".in"]), code_format=B.PQ_CODES_C16, stream=s)
+            q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]
+            m_out1, _ = B.palquant_epilogue_scales(G, st[n + ".conv1.w"], st[n + ".in"], 1.0, None, self.no_shuffle)
+            y1 = torch.empty((self.N, blk["Ho"], blk["Wo"], G * blk["w"]), dtype=torch.float32, device=self.dev)
+            B.palquant_layer_fused(q_in, blk["wp1"], blk["d1"], m_out1, None, self.no_shuffle, None, None, y1, None,
+                                   stream=s)
+            st[n + ".mid"] = self._act_steps(y1, blk["w"])
+            del y1
+            self._scales(blk, st)
+            self._block_front(blk, q_in)
+            if i + 1 < len(self.blocks):
+                self._conv2(blk, None)  # fp32 output only
+                nxt = self.blocks[i + 1]["name"] + ".in"
+                st[nxt] = self._act_steps(blk["out"], blk["w"])
+                # the next block's codes, as forward() fuses them into conv2
+                self._conv2(blk, self._inv(st[nxt], self.cyclic))
+        self.set_steps(st)
+        return st
+
+    def _pack(self, blk, st):
+        """Quantise and pack the block's weights with their steps (synchronous)."""
+        n = blk["name"]
+        for key, d, wname in (("wp1", blk["d1"], ".conv1"), ("wp2", blk["d2"], ".conv2")) + \
+                ((("wpd", blk["dd"], ".down"),) if blk["down"] else ()):
+            B.palquant_pack_weights(self.params[n + wname], d, self._inv(st[n + wname + ".w"]), blk[key],
+                                    blk[key].numel(), stream=self.stream)
+
+    def _scales(self, blk, st):
+        """Epilogue multipliers of the block's layers from the steps known so far."""
+        n, G = blk["name"], self.G
+        blk["m_out1"], blk["m_req1"] = B.palquant_epilogue_scales(G, st[n + ".conv1.w"], st[n + ".in"], 1.0,
+                                                                  st.get(n + ".mid"), self.no_shuffle)
+        if blk["down"]:
+            blk["m_outd"], _ = B.palquant_epilogue_scales(G, st[n + ".down.w"], st[n + ".in"], 1.0, None,
+                                                          self.no_shuffle)
+        if n + ".mid" in st:
+            blk["m_out2"], _ = B.palquant_epilogue_scales(G, st[n + ".conv2.w"], st[n + ".mid"], 1.0, None, self.cyclic)
+
+    def set_steps(self, steps: dict):
+        """Pack every layer's weights and derive the epilogue multipliers from `steps`."""
+        self.steps = dict(steps)
+        for i, blk in enumerate(self.blocks):
+            self._pack(blk, self.steps)
+            self._scales(blk, self.steps)
+            nxt = self.blocks[i + 1]["name"] + ".in" if i + 1 < len(self.blocks) else None
+            # conv2's codes land in group dst(g) of the next block: multiplier fl(1/s_next[dst(g)])
+            blk["m_req2"] = None if nxt is None else self._inv(self.steps[nxt], self.cyclic)
+        self.inv_in = self._inv(self.steps[self.blocks[0]["name"] + ".in"])
+        self.stream.synchronize()
+        self.graph = None
+
+    # --------------------------------------------------------------- forward
+    def _stem(self, x_dev):
+        s = self.stream
+        B.palquant_conv2d_f32(x_dev, self.w_stem, self.stem_out, self.N, self.H, self.W, 3, self.C0, 7, 2, 3, relu=True,
+                              stream=s)
+        B.palquant_maxpool2d_f32(self.stem_out, self.pool, self.N, self.Hs, self.Ws, self.C0, 3, 2, 1, stream=s)
+
+    def _block_front(self, blk, q_in):
+        s = self.stream
+        B.palquant_layer_fused(q_in, blk["wp1"], blk["d1"], blk["m_out1"], blk["m_req1"], self.no_shuffle, None, None,
+                               None, blk["mid_codes"], stream=s)
+        if blk["down"]:
+            B.palquant_layer_fused(q_in, blk["wpd"], blk["dd"], blk["m_outd"], None, self.no_shuffle, None, None,
+                                   blk["down_out"], None, stream=s)
+
+    def _conv2(self, blk, m_req2):
+        i = self.blocks.index(blk)
+        shortcut = blk["down_out"] if blk["down"] else (self.pool if i == 0 else self.blocks[i - 1]["out"])
+        B.palquant_layer_fused(blk["mid_codes"], blk["wp2"], blk["d2"], blk["m_out2"], m_req2, self.cyclic, shortcut,
+                               None, blk["out"], None if m_req2 is None else blk["out_codes"], stream=self.stream)
+
+    def forward(self, x_dev: torch.Tensor) -> torch.Tensor:
+        """Logits [N, classes] for images x_dev (NHWC fp32 [N, H, W, 3] on the device);
+        asynchronous on self.stream."""
+        if self.steps is None:
+            raise RuntimeError("calibrate() or set_steps() first")
+        s = self.stream
+        self._stem(x_dev)
+        B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, self.G, self.C0 // self.G,
+                                self.bits, self.inv_in, code_format=B.PQ_CODES_C16, stream=s)
+        for i, blk in enumerate(self.blocks):
+            q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]
+            self._block_front(blk, q_in)
+            self._conv2(blk, blk["m_req2"])
+        last = self.blocks[-1]["out"]
+        B.palquant_avgpool_f32(last, self.avg, self.N, self.Hl, self.Wl, self.Cl, stream=s)
+        B.palquant_linear_f32(self.avg, self.w_fc, self.logits, self.N, self.Cl, self.classes, stream=s)
+        return self.logits
+
+    def capture(self, x_dev: torch.Tensor):
+        """Capture forward(x_dev) into a CUDA graph (replayed by replay())."""
+        self.forward(x_dev)  # warm-up outside capture (first-call set-up in the library)
+        self.stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=self.stream):
+            self.forward(x_dev)
+        self.graph = g
+        return g
+
+    def replay(self):
+        self.graph.replay()
+        return self.logits
+
+    def launches_per_forward(self) -> int:
+        """Kernels one forward launches: stem conv, max pooling, quantiser, per block
+        conv1 (+ down) + conv2, average pooling, FC."""
+        return 3 + sum(3 if b["down"] else 2 for b in self.blocks) + 2
+
+    def body_int_ops(self) -> int:
+        """Integer operations (2 per MAC) of the PalQuant layers of one forward."""
+        G, N, ops = self.G, self.N, 0
+        for b in self.blocks:
+            ops += 2 * N * b["Ho"] * b["Wo"] * G * b["w"] * 9 * b["cin"]
+            ops += 2 * N * b["Ho"] * b["Wo"] * G * b["w"] * 9 * b["w"]
+            if b["down"]:
+                ops += 2 * N * b["Ho"] * b["Wo"] * G * b["w"] * b["cin"]
+        return ops

@@ -1,0 +1,97 @@
+"""The ResNet-18-shaped PalQuant network on the GPU against the oracle network.
+
+Both sides receive the same seeded images and weights and the oracle's calibrated
+steps; every intermediate tensor is compared: full-precision stem and pooling outputs
+and logits bit for bit (fixed summation order on both sides), all codes bit for bit,
+and the blocks' fp32 outputs bit for bit (one fp32 multiply and one add per value).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle.resnet as OR
+from layer_cases import c16_to_nhwc
+from paper_2208_01944_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+
+def _codes(t):
+    N, H, W, C = t.shape
+    return c16_to_nhwc(t.cpu().numpy(), N, H, W, C)
+
+
+def _compare(net, r):
+    assert np.array_equal(net.stem_out.cpu().numpy(), r["stem"]), "stem"
+    assert np.array_equal(net.pool.cpu().numpy(), r["pool"]), "max pooling"
+    assert np.array_equal(_codes(net.in_codes), r[net.blocks[0]["name"] + ".in_codes"]), "input codes"
+    for i, blk in enumerate(net.blocks):
+        n = blk["name"]
+        assert np.array_equal(_codes(blk["mid_codes"]), r[n + ".mid_codes"]), n + " conv1 codes"
+        if blk["down"]:
+            assert np.array_equal(blk["down_out"].cpu().numpy(), r[n + ".down"]), n + " downsample"
+        assert np.array_equal(blk["out"].cpu().numpy(), r[n + ".out"]), n + " block output"
+        if i + 1 < len(net.blocks):
+            assert np.array_equal(_codes(blk["out_codes"]), r[n + ".out_codes"]), n + " next-block codes"
+    assert np.array_equal(net.avg.cpu().numpy(), r["avg"]), "average pooling"
+    assert np.array_equal(net.logits.cpu().numpy(), r["logits"]), "logits"
+
+
+@pytest.mark.parametrize("N,H,widths,classes,seed", [(2, 32, (32, 32, 32, 32), 10, 1),
+                                                     (3, 64, (32, 64, 32, 64), 16, 2)])
+def test_small_network_matches_oracle(N, H, widths, classes, seed):
+    from paper_2208_01944_gb300.resnet18 import PalQuantResNet18
+
+    x, params = synth.resnet18_inputs(N, H, H, 2, widths, classes, seed=seed)
+    steps = OR.calibrate(x, params, 2, 2)
+    r = OR.forward(x, params, 2, 2, steps)
+    net = PalQuantResNet18(params, N, H, H, 2, widths, classes, 2)
+    net.set_steps(steps)
+    xd = torch.from_numpy(x).cuda()
+    net.forward(xd)
+    net.stream.synchronize()
+    from paper_2208_01944_gb300 import binding as B
+    assert B.palquant_sync_check() == B.PQ_OK
+    _compare(net, r)
+
+
+def test_resnet18_224_matches_oracle():
+    """The full ResNet-18 shape (224x224 input, per-group widths 64/128/256/512, G = 2,
+    1000 classes) on one image, and the CUDA-graph replay of the same forward."""
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300.resnet18 import PalQuantResNet18
+
+    x, params = synth.resnet18_inputs(1, seed=0)
+    steps = OR.calibrate(x, params, 2, 2)
+    r = OR.forward(x, params, 2, 2, steps)
+    net = PalQuantResNet18(params, 1)
+    net.set_steps(steps)
+    xd = torch.from_numpy(x).cuda()
+    net.forward(xd)
+    net.stream.synchronize()
+    assert B.palquant_sync_check() == B.PQ_OK
+    _compare(net, r)
+    net.logits.zero_()
+    net.capture(xd)
+    net.replay()
+    net.stream.synchronize()
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(net.logits.cpu().numpy(), r["logits"])
+
+
+def test_device_calibration_close_to_oracle():
+    """The library's own step initialisation (device sums) on the same network: the
+    first block's input steps and every weight step within one float ulp of the oracle's."""
+    from paper_2208_01944_gb300.resnet18 import PalQuantResNet18
+
+    x, params = synth.resnet18_inputs(2, 32, 32, 2, (32, 32, 32, 32), 10, seed=3)
+    ref = OR.calibrate(x, params, 2, 2)
+    net = PalQuantResNet18(params, 2, 32, 32, 2, (32, 32, 32, 32), 10, 2)
+    got = net.calibrate(torch.from_numpy(x).cuda())
+    assert set(got) == set(ref)
+    keys = ["s1b1.in"] + [k for k in ref if k.endswith(".w")]
+    for k in keys:
+        d = np.abs(got[k].view(np.int32).astype(np.int64) - ref[k].view(np.int32).astype(np.int64))
+        assert np.all(d <= 1), k
+    for k in ref:
+        assert np.allclose(got[k], ref[k], rtol=1e-3), k
