@@ -47,6 +47,9 @@ def parse():
                     help="only run the fused layer of CONFIG (config0, config1, config3_0..4, config4) --reps times "
                          "on random codes (codes out), for profilers; prints nothing else")
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--no-resnet", action="store_true", help="skip the ResNet-18-shaped network measurement")
+    ap.add_argument("--resnet-batch", type=int, default=128)
+    ap.add_argument("--resnet-reps", type=int, default=20)
     return ap.parse_args()
 
 
@@ -234,6 +237,69 @@ def run_reference(args, rank, world):
 
 
 # ---------------------------------------------------------------------------
+# The ResNet-18-shaped network (config 2): images/s of the whole forward.
+# ---------------------------------------------------------------------------
+def measure_resnet18(dev, world, args):
+    """Forward of the ResNet-18-shaped PalQuant network (224x224, G = 2, b = 2, per-group
+    widths 64/128/256/512, fp32 stem and FC) on a batch of synthetic images, replayed
+    from CUDA graphs; two input batches (154 MB together, more than L2) alternate."""
+    import numpy as np
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300 import synth
+    from paper_2208_01944_gb300.resnet18 import PalQuantResNet18
+
+    N = args.resnet_batch
+    x_np, params = synth.resnet18_inputs(N, seed=0)
+    net = PalQuantResNet18(params, N, device=dev)
+    xs = [torch.from_numpy(x_np).to(dev)]
+    xs.append(torch.flip(xs[0], dims=[0]).contiguous())
+    net.calibrate(xs[0])  # step initialisation, untimed
+    graphs = [net.capture(x) for x in xs]
+    for i in range(3):
+        net.replay(graphs[i & 1])
+    torch.cuda.synchronize(dev)
+    R = args.resnet_reps
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(net.stream)
+    for i in range(R):
+        net.replay(graphs[i & 1])
+    e1.record(net.stream)
+    torch.cuda.synchronize(dev)
+    st = B.palquant_sync_check(net.stream)
+    assert st == B.PQ_OK, B.strerror(st)
+    ms = e0.elapsed_time(e1) / R
+    out = {"workload": "ResNet-18-shaped PalQuant forward: batch %d, 224x224x3 N(0,1) images, G=2, b=2, per-group widths "
+                       "64/128/256/512, fp32 7x7 stem + max pooling and fp32 FC, cyclic shuffle after each block" % N,
+           "images_per_s": N * world / (ms / 1e3), "ms_per_batch": ms, "batch_per_gpu": N, "reps": R,
+           "palquant_body_tops": net.body_int_ops() * world / (ms / 1e3) / 1e12,
+           "timed": "CUDA-graph replay of the whole forward (stem, pooling, quantiser, 20 PalQuant layers, pooling, FC)",
+           "gpu_launches_per_forward": net.launches_per_forward(), "data": "synthetic"}
+    # where the time goes: one eager forward with events between its stages
+    marks = []
+    net.forward(xs[0], marks)
+    torch.cuda.synchronize(dev)
+    out["stages_ms"] = {name: marks[i - 1][1].elapsed_time(ev) for i, (name, ev) in enumerate(marks) if i > 0}
+    del graphs, net
+    torch.cuda.empty_cache()
+    if not args.no_cpu_baseline:
+        import time
+
+        import oracle
+        import oracle.resnet as OR
+
+        x1, p1 = synth.resnet18_inputs(1, seed=0)
+        steps = OR.calibrate(x1, p1, 2, 2)
+        t0 = time.perf_counter()
+        OR.forward(x1, p1, 2, 2, steps)
+        dt = time.perf_counter() - t0
+        out["cpu_baseline"] = {"value": 1.0 / dt, "unit": "images/s", "cores": oracle.num_threads(), "kind": "oracle",
+                               "sample": f"1 image, forward with given steps, {dt:.2f} s"}
+    return out
+
+
+# ---------------------------------------------------------------------------
 # Our arm.
 # ---------------------------------------------------------------------------
 def run_ours(args, rank, world, local_rank):
@@ -311,11 +377,12 @@ def run_ours(args, rank, world, local_rank):
             ev[i][2].record(stream)
         stop.record(stream)
     torch.cuda.synchronize(dev)
+    st = B.palquant_sync_check(stream)
+    assert st == B.PQ_OK, B.strerror(st)
+    resnet = None if args.no_resnet else measure_resnet18(dev, world, args)
     clocks = sampler.stop()
     if world > 1:
         dist.barrier()
-    st = B.palquant_sync_check(stream)
-    assert st == B.PQ_OK, B.strerror(st)
     elapsed_ms = start.elapsed_time(stop)
     t_quant = sum(e[0].elapsed_time(e[1]) for e in ev) / K
     t_conv = sum(e[1].elapsed_time(e[2]) for e in ev) / K
@@ -387,6 +454,8 @@ def run_ours(args, rank, world, local_rank):
                 "d2h_bytes_per_step": int(np.prod(out_shape))},
         "gpu_launches": 2 * K,
     }
+    if resnet is not None:
+        line["resnet18"] = resnet
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(c, x_np, w_np, args.cpu_seconds)
     print(json.dumps(line), flush=True)

@@ -190,22 +190,36 @@ class PalQuantResNet18:
         B.palquant_layer_fused(blk["mid_codes"], blk["wp2"], blk["d2"], blk["m_out2"], m_req2, self.cyclic, shortcut,
                                None, blk["out"], None if m_req2 is None else blk["out_codes"], stream=self.stream)
 
-    def forward(self, x_dev: torch.Tensor) -> torch.Tensor:
+    def forward(self, x_dev: torch.Tensor, marks: list | None = None) -> torch.Tensor:
         """Logits [N, classes] for images x_dev (NHWC fp32 [N, H, W, 3] on the device);
-        asynchronous on self.stream."""
+        asynchronous on self.stream.  With `marks`, a CUDA event recorded on the stream
+        after each stage is appended as (stage name, event)."""
         if self.steps is None:
             raise RuntimeError("calibrate() or set_steps() first")
         s = self.stream
+
+        def mark(name):
+            if marks is not None:
+                ev = torch.cuda.Event(enable_timing=True)
+                ev.record(s)
+                marks.append((name, ev))
+
+        mark("start")
         self._stem(x_dev)
+        mark("stem conv + max pooling (fp32)")
         B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, self.G, self.C0 // self.G,
                                 self.bits, self.inv_in, code_format=B.PQ_CODES_C16, stream=s)
+        mark("input quantiser")
         for i, blk in enumerate(self.blocks):
             q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]
             self._block_front(blk, q_in)
+            mark(blk["name"] + " conv1" + (" + down" if blk["down"] else ""))
             self._conv2(blk, blk["m_req2"])
+            mark(blk["name"] + " conv2")
         last = self.blocks[-1]["out"]
         B.palquant_avgpool_f32(last, self.avg, self.N, self.Hl, self.Wl, self.Cl, stream=s)
         B.palquant_linear_f32(self.avg, self.w_fc, self.logits, self.N, self.Cl, self.classes, stream=s)
+        mark("average pooling + FC (fp32)")
         return self.logits
 
     def capture(self, x_dev: torch.Tensor):
@@ -218,8 +232,10 @@ class PalQuantResNet18:
         self.graph = g
         return g
 
-    def replay(self):
-        self.graph.replay()
+    def replay(self, graph=None):
+        """Replay a captured forward on self.stream (the last capture by default)."""
+        with torch.cuda.stream(self.stream):
+            (graph or self.graph).replay()
         return self.logits
 
     def launches_per_forward(self) -> int:

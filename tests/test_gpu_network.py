@@ -95,3 +95,53 @@ def test_device_calibration_close_to_oracle():
         assert np.all(d <= 1), k
     for k in ref:
         assert np.allclose(got[k], ref[k], rtol=1e-3), k
+
+
+# ------------------------------------------------------------ full-precision layers alone
+@pytest.mark.parametrize("shape,Cout,k,s,p,relu", [
+    ((2, 37, 29, 3), 64, 7, 2, 3, True),     # the stem kernel, ragged tiles
+    ((1, 224, 224, 3), 128, 7, 2, 3, True),  # the network's stem shape
+    ((2, 9, 11, 5), 32, 3, 1, 1, False),     # the generic kernel, weights in shared memory
+    ((1, 12, 10, 64), 48, 5, 2, 2, True),    # the generic kernel, weights from global memory
+])
+def test_conv2d_f32_matches_oracle(shape, Cout, k, s, p, relu):
+    import oracle
+    from paper_2208_01944_gb300 import binding as B
+
+    gen = synth.generator(sum(shape) + Cout)
+    x = synth.normal(shape, gen)
+    w = synth.normal((Cout, k, k, shape[3]), gen, 0.2)
+    ref = oracle.conv2d_f32(x, w, s, p, relu)
+    y = torch.empty(ref.shape, dtype=torch.float32, device="cuda")
+    B.palquant_conv2d_f32(torch.from_numpy(x).cuda(), torch.from_numpy(w).cuda(), y, shape[0], shape[1], shape[2],
+                          shape[3], Cout, k, s, p, relu)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(y.cpu().numpy(), ref)
+
+
+def test_pooling_and_linear_match_oracle():
+    import oracle
+    from paper_2208_01944_gb300 import binding as B
+
+    gen = synth.generator(21)
+    x = synth.normal((3, 13, 11, 24), gen)
+    ref = oracle.maxpool_f32(x, 3, 2, 1)
+    y = torch.empty(ref.shape, dtype=torch.float32, device="cuda")
+    B.palquant_maxpool2d_f32(torch.from_numpy(x).cuda(), y, 3, 13, 11, 24, 3, 2, 1)
+    assert np.array_equal(y.cpu().numpy(), ref)
+    x5 = synth.normal((2, 7, 9, 5), gen)  # channels not a multiple of 4: the scalar kernel
+    ref5 = oracle.maxpool_f32(x5, 3, 2, 1)
+    y5 = torch.empty(ref5.shape, dtype=torch.float32, device="cuda")
+    B.palquant_maxpool2d_f32(torch.from_numpy(x5).cuda(), y5, 2, 7, 9, 5, 3, 2, 1)
+    assert np.array_equal(y5.cpu().numpy(), ref5)
+    ref = oracle.avgpool_f32(x)
+    y = torch.empty(ref.shape, dtype=torch.float32, device="cuda")
+    B.palquant_avgpool_f32(torch.from_numpy(x).cuda(), y, 3, 13, 11, 24)
+    assert np.array_equal(y.cpu().numpy(), ref)
+    v = synth.normal((13, 100), gen)
+    w = synth.normal((1000, 100), gen)
+    ref = oracle.linear_f32(v, w)
+    y = torch.empty(ref.shape, dtype=torch.float32, device="cuda")
+    B.palquant_linear_f32(torch.from_numpy(v).cuda(), torch.from_numpy(w).cuda(), y, 13, 100, 1000)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(y.cpu().numpy(), ref)
