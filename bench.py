@@ -50,6 +50,8 @@ def parse():
     ap.add_argument("--no-resnet", action="store_true", help="skip the ResNet-18-shaped network measurement")
     ap.add_argument("--resnet-batch", type=int, default=128)
     ap.add_argument("--resnet-reps", type=int, default=20)
+    ap.add_argument("--no-layers", action="store_true", help="skip the per-config layer measurements")
+    ap.add_argument("--layer-reps", type=int, default=50)
     return ap.parse_args()
 
 
@@ -110,6 +112,25 @@ def dram_traffic(kernel):
         return d["bytes_per_launch"]
     except Exception:
         return None
+
+
+def max_over_ranks(x: float, world: int, device="cpu") -> float:
+    """The largest of the ranks' values of x (a time), all_reduce(MAX) over the
+    process group (NCCL on the GPU, gloo on the CPU); x itself with one rank."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([float(x)], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, world: int, ms: float) -> float:
+    """Units per second of the whole job: every rank processed `units_per_rank` in
+    `ms` (the slowest rank's time), weak scaling."""
+    return units_per_rank * world / (ms / 1e3)
 
 
 class ClockSampler:
@@ -237,6 +258,89 @@ def run_reference(args, rank, world):
 
 
 # ---------------------------------------------------------------------------
+# The single-layer configs (0, 1, the b/G sweep 3, the 1x1 layer 4) and the
+# quantiser alone: per-launch device time of the fused layer, codes in and out.
+# ---------------------------------------------------------------------------
+L2_BYTES = 126 * 1024 * 1024
+
+
+def measure_layer_configs(dev, args):
+    """Each config's fused layer in timed mode (channel-blocked codes in, codes out)
+    and the quantiser on the config-1 and config-4 inputs.  Input/output buffer sets
+    rotate so that the bytes one pass touches total at least 2x L2; CUDA events on the
+    launching stream bracket `reps` launches after 3 warm-up launches."""
+    import numpy as np
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300 import synth, workloads
+
+    pk = peaks()
+    fp8_peak = 2.0 * pk["bf16_tflops"]
+    stream = torch.cuda.Stream(device=dev)
+    fmt = B.PQ_CODES_C16
+    out = {}
+    reps = args.layer_reps
+
+    def timed(launch, n_sets):
+        with torch.cuda.stream(stream):
+            for i in range(3):
+                launch(i % n_sets)
+        torch.cuda.synchronize(dev)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for i in range(reps):
+                launch(i % n_sets)
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        st = B.palquant_sync_check(stream)
+        assert st == B.PQ_OK, B.strerror(st)
+        return e0.elapsed_time(e1) / reps
+
+    for name, c in workloads.BENCH_CONFIGS.items():
+        gen = synth.generator(0)
+        per_set = c.in_elems + c.out_elems
+        n_sets = max(1, min(16, -(-2 * L2_BYTES // per_set)))
+        q = torch.from_numpy(synth.random_codes((c.N, c.H, c.W, c.G * c.Cin_g), c.bits_a, gen)).to(dev)
+        qs = [q] + [q.clone() for _ in range(n_sets - 1)]
+        wq = synth.random_codes((c.G, c.Cout_g, c.k, c.k, c.Cin_g), c.bits_w, gen, signed=True)
+        d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out,
+                         int(c.relu), code_format=fmt)
+        wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).to(dev)
+        qo = [torch.empty((c.N, c.Ho, c.Wo, c.G * c.Cout_g), dtype=torch.uint8, device=dev) for _ in range(n_sets)]
+        m = np.full(c.G, 0.01, np.float32)
+        shuf = B.shuffle(c.shuffle_kind, c.shuffle_shift)
+        ms = timed(lambda i: B.palquant_layer_fused(qs[i], wp, d, m, m, shuf, None, None, None, qo[i], stream=stream),
+                   n_sets)
+        byt = c.in_elems + c.out_elems + c.weight_elems
+        tops = c.int_ops / (ms / 1e3) / 1e12
+        plan = B.palquant_conv_plan(d).as_dict()
+        out[name] = {"shape": c.name, "us": ms * 1e3, "tops": tops, "frac_fp8_peak": tops / fp8_peak,
+                     "algorithmic_gbs": byt / (ms / 1e3) / 1e9, "frac_hbm": byt / (ms / 1e3) / 1e9 / pk["hbm_gbs"],
+                     "buffer_sets": n_sets, "plan": {k: plan[k] for k in ("m_tiles", "n_block", "k_chunk",
+                                                                         "weights_resident", "work_items")}}
+        del qs, qo, q, wp
+    for name in ("config1", "config4"):
+        c = workloads.BENCH_CONFIGS[name]
+        shape = (c.N, c.H, c.W, c.G * c.Cin_g)
+        per_set = c.in_elems * 5
+        n_sets = max(1, min(8, -(-2 * L2_BYTES // per_set)))
+        x = torch.randn(shape, device=dev).abs_()
+        xs = [x] + [x.clone() for _ in range(n_sets - 1)]
+        qq = [torch.empty(shape, dtype=torch.uint8, device=dev) for _ in range(n_sets)]
+        inv = np.full(c.G, 1.3, np.float32)
+        ms = timed(lambda i: B.palquant_quantize_act(xs[i], qq[i], c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv,
+                                                     code_format=fmt, stream=stream), n_sets)
+        gbs = per_set / (ms / 1e3) / 1e9
+        out["quantize_" + name] = {"shape": f"{c.N}x{c.H}x{c.W}x{c.G * c.Cin_g} fp32 -> channel-blocked codes",
+                                   "us": ms * 1e3, "gbs": gbs, "frac_hbm": gbs / pk["hbm_gbs"], "buffer_sets": n_sets}
+        del xs, qq, x
+    torch.cuda.empty_cache()
+    return out
+
+
+# ---------------------------------------------------------------------------
 # The ResNet-18-shaped network (config 2): images/s of the whole forward.
 # ---------------------------------------------------------------------------
 def measure_resnet18(dev, world, args):
@@ -269,11 +373,11 @@ def measure_resnet18(dev, world, args):
     torch.cuda.synchronize(dev)
     st = B.palquant_sync_check(net.stream)
     assert st == B.PQ_OK, B.strerror(st)
-    ms = e0.elapsed_time(e1) / R
+    ms = max_over_ranks(e0.elapsed_time(e1) / R, world, dev)
     out = {"workload": "ResNet-18-shaped PalQuant forward: batch %d, 224x224x3 N(0,1) images, G=2, b=2, per-group widths "
                        "64/128/256/512, fp32 7x7 stem + max pooling and fp32 FC, cyclic shuffle after each block" % N,
-           "images_per_s": N * world / (ms / 1e3), "ms_per_batch": ms, "batch_per_gpu": N, "reps": R,
-           "palquant_body_tops": net.body_int_ops() * world / (ms / 1e3) / 1e12,
+           "images_per_s": whole_job_rate(N, world, ms), "ms_per_batch": ms, "batch_per_gpu": N, "reps": R,
+           "palquant_body_tops": whole_job_rate(net.body_int_ops(), world, ms) / 1e12,
            "timed": "CUDA-graph replay of the whole forward (stem, pooling, quantiser, 20 PalQuant layers, pooling, FC)",
            "gpu_launches_per_forward": net.launches_per_forward(), "data": "synthetic"}
     # where the time goes: one eager forward with events between its stages
@@ -283,7 +387,7 @@ def measure_resnet18(dev, world, args):
     out["stages_ms"] = {name: marks[i - 1][1].elapsed_time(ev) for i, (name, ev) in enumerate(marks) if i > 0}
     del graphs, net
     torch.cuda.empty_cache()
-    if not args.no_cpu_baseline:
+    if not args.no_cpu_baseline and world == 1:
         import time
 
         import oracle
@@ -380,19 +484,17 @@ def run_ours(args, rank, world, local_rank):
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
     resnet = None if args.no_resnet else measure_resnet18(dev, world, args)
+    layers = None if args.no_layers else measure_layer_configs(dev, args)
     clocks = sampler.stop()
     if world > 1:
         dist.barrier()
     elapsed_ms = start.elapsed_time(stop)
     t_quant = sum(e[0].elapsed_time(e[1]) for e in ev) / K
     t_conv = sum(e[1].elapsed_time(e[2]) for e in ev) / K
-    if world > 1:
-        t = torch.tensor([elapsed_ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(elapsed_ms, world, dev)
     ms_per_step = elapsed_ms / K
     ops_step = c.int_ops
-    value = ops_step * world / (ms_per_step / 1e3) / 1e12
+    value = whole_job_rate(ops_step, world, ms_per_step) / 1e12
 
     # ---- end to end through the public API with host buffers (pinned), per step:
     # H2D input copy, quantize, fused layer, D2H of the output codes.
@@ -415,8 +517,8 @@ def run_ours(args, rank, world, local_rank):
             out_host.copy_(q_out, non_blocking=True)
         e1.record(stream)
     torch.cuda.synchronize(dev)
-    e2e_ms = e0.elapsed_time(e1) / E
-    e2e_value = ops_step * world / (e2e_ms / 1e3) / 1e12
+    e2e_ms = max_over_ranks(e0.elapsed_time(e1) / E, world, dev)
+    e2e_value = whole_job_rate(ops_step, world, e2e_ms) / 1e12
 
     if rank != 0:
         return
@@ -445,7 +547,7 @@ def run_ours(args, rank, world, local_rank):
                    "code_layout": "channel-blocked [N][C/16][H][W][16], one byte per code",
                    "l2": "inputs larger than L2 (205.5 MB fp32, two buffers used in turn)",
                    "parallelism": f"replicas x{world}"},
-        "images_per_s": c.N * world / (ms_per_step / 1e3),
+        "images_per_s": whole_job_rate(c.N, world, ms_per_step),
         "pct_dense_int8_peak": 100.0 * value / world / fp8_peak,
         "roofline": dominant,
         "roofline_kernels": [roof_quant, roof_conv],
@@ -456,7 +558,9 @@ def run_ours(args, rank, world, local_rank):
     }
     if resnet is not None:
         line["resnet18"] = resnet
-    if not args.no_cpu_baseline:
+    if layers is not None:
+        line["layers"] = layers
+    if not args.no_cpu_baseline and world == 1:
         line["cpu_baseline"] = cpu_baseline(c, x_np, w_np, args.cpu_seconds)
     print(json.dumps(line), flush=True)
 

@@ -1,0 +1,68 @@
+"""The benchmark's multi-rank host logic on CPU processes (gloo, world size 2).
+
+The path shards by batch with no exchange step (replicas), so the only cross-rank
+work is the timing: every rank's time is reduced with MAX and the whole-job rate
+counts every rank's units.  The reference arm runs on rank 0 only.
+"""
+import os
+import socket
+import sys
+
+import pytest
+import torch.multiprocessing as mp
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def _free_port() -> int:
+    with socket.socket() as s:
+        s.bind(("127.0.0.1", 0))
+        return s.getsockname()[1]
+
+
+def _rank_main(rank, world, port, times, out):
+    import torch.distributed as dist
+
+    sys.path.insert(0, ROOT)
+    import bench
+
+    os.environ["MASTER_ADDR"] = "127.0.0.1"
+    os.environ["MASTER_PORT"] = str(port)
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        t = bench.max_over_ranks(times[rank], world, "cpu")
+        out[rank] = (t, bench.whole_job_rate(64, world, t))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_max_over_ranks_and_rate_gloo_world2():
+    world = 2
+    times = [3.0, 5.0]
+    with mp.Manager() as m:
+        out = m.dict()
+        mp.spawn(_rank_main, args=(world, _free_port(), times, out), nprocs=world, join=True)
+        res = dict(out)
+    for rank in range(world):
+        t, rate = res[rank]
+        assert t == 5.0  # the slowest rank's time, on every rank
+        assert rate == pytest.approx(64 * 2 / 5e-3)
+
+
+def test_single_rank_is_identity():
+    sys.path.insert(0, ROOT)
+    import bench
+
+    assert bench.max_over_ranks(7.5, 1) == 7.5
+    assert bench.whole_job_rate(10, 1, 2.0) == pytest.approx(5000.0)
+
+
+def test_reference_arm_runs_on_rank0_only(capsys):
+    sys.path.insert(0, ROOT)
+    import bench
+
+    class Args:
+        steps, warmup, gpus = 1, 0, 2
+
+    assert bench.run_reference(Args(), 1, 2) is None  # rank 1: no work, no output
+    assert capsys.readouterr().out == ""
