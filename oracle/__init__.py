@@ -295,3 +295,32 @@ def linear_f32(x: np.ndarray, w: np.ndarray, L=None) -> np.ndarray:
     y = np.empty((N, Co), dtype=np.float32)
     L.oracle_linear_f32(_ptr(x), _ptr(w), _ptr(y), N, Ci, Co)
     return y
+
+
+# ---------------------------------------------------------------------------
+# Cyclic shuffle module (Sec. 4.2, Eq. 9-10): Y = CyclicPermute(X) by Eq. 8,
+# Z = X + Conv1x1(Y) with the 1x1 convolution a PalQuant group convolution.
+# ---------------------------------------------------------------------------
+def permute_groups(t: np.ndarray, G: int, shift: int = 1, L=None) -> np.ndarray:
+    """Eq. 8 on the channel axis of an NHWC tensor: Y[..., pi(i) block] = X[..., i block],
+    pi(i) = (i + shift) mod G (Eq. 6 for shift 1)."""
+    dst = group_perm(G, 1, shift, L=L)
+    C = t.shape[-1]
+    Cg = C // G
+    y = np.empty_like(t)
+    for i in range(G):
+        y[..., dst[i] * Cg:(dst[i] + 1) * Cg] = t[..., i * Cg:(i + 1) * Cg]
+    return y
+
+
+def cyclic_shuffle_module(x: np.ndarray, q: np.ndarray, wq: np.ndarray, m_out, m_req=None, shift: int = 1,
+                          relu: bool = False, bits_out: int = 2, L=None):
+    """Z = X + Conv1x1(CyclicPermute(X)) on a quantised layer: the codes q of X are
+    permuted by Eq. 8, convolved by the 1x1 group convolution wq [G, C_g, 1, 1, C_g],
+    rescaled by m_out and added to the fp32 X (Eq. 10), optional ReLU; with m_req, the
+    codes of Z for the next layer (requantised from the sum).  Returns (z, codes or None)."""
+    G = wq.shape[0]
+    y = permute_groups(q, G, shift, L=L)
+    acc = group_conv(y, wq, 1, 0, L=L)
+    _, z, codes = epilogue(acc, G, m_out, m_req, 0, 0, None, x, relu, bits_out, L=L)
+    return z, codes

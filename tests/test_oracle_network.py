@@ -221,3 +221,51 @@ def test_fp32_mutation_is_caught(name, tmp_path):
     path.write_text(src.replace(old, new, 1))
     so = oracle.build(force=True, src=str(path), out=str(tmp_path / "libmut.so"))
     assert not _fp32_pins_pass(oracle.load_variant(so)), f"mutation {name} not caught"
+
+
+# ------------------------------------------------------------ cyclic shuffle module (Eq. 9-10)
+def test_permute_groups_is_eq8():
+    x = np.arange(2 * 3 * 12, dtype=np.float32).reshape(2, 3, 12)
+    y = oracle.permute_groups(x, 4, 1)
+    # Y[:, pi(i)] = X[:, i] with pi(i) = (i + 1) mod 4: group 0 lands in group 1, group 3 in group 0
+    assert np.array_equal(y[..., 3:6], x[..., 0:3]) and np.array_equal(y[..., 0:3], x[..., 9:12])
+    assert np.array_equal(y, np.roll(x.reshape(2, 3, 4, 3), 1, axis=2).reshape(x.shape))
+    assert np.array_equal(oracle.permute_groups(y, 4, -1), x)
+
+
+@pytest.mark.parametrize("G,Cg", [(2, 32), (4, 16), (3, 32)])
+def test_cyclic_shuffle_module_rederived(G, Cg):
+    """Z = X + Conv1x1(CyclicPermute(X)) recomputed with numpy's roll and torch's
+    float64 grouped convolution of the integer codes (exact), one fp32 multiply and
+    one fp32 add."""
+    gen = synth.generator(G * Cg)
+    x = synth.half_normal((2, 5, 6, G * Cg), gen)
+    q = oracle.quantize_act(x, G, 2, np.full(G, 1.7, np.float32))
+    wq = synth.random_codes((G, Cg, 1, 1, Cg), 2, gen, signed=True)
+    m_out = (np.arange(G, dtype=np.float32) + 1) * np.float32(0.03)
+    inv_next = np.full(G, 1.3, np.float32)
+    z, codes = oracle.cyclic_shuffle_module(x, q, wq, m_out, inv_next, 1)
+    rolled = np.roll(q.reshape(2, 5, 6, G, Cg), 1, axis=3).reshape(q.shape)
+    acc = torch_group_conv_f64(rolled, wq, 1, 0)
+    y = (acc.astype(np.float32).reshape(2, 5, 6, G, Cg) * m_out[:, None]).reshape(acc.shape)
+    assert np.array_equal(z, y + x)
+    assert np.array_equal(codes, oracle.quantize_act(z, G, 2, inv_next))
+
+
+@pytest.mark.parametrize("G", [2, 3, 4, 5])
+def test_prop1_G_minus_1_modules_reach_every_group(G):
+    """Prop. 1: after G-1 cyclic shuffle modules every group holds information from
+    every group.  Only group s of the input is non-zero and all weights are positive:
+    after k modules exactly the groups s, s+1, ..., s+k (mod G) are non-zero."""
+    Cg = 16
+    wq = np.ones((G, Cg, 1, 1, Cg), dtype=np.int8)
+    m_out = np.full(G, 0.1, np.float32)  # large enough that a reached group quantises to a non-zero code
+    inv = np.ones(G, np.float32)
+    for s in range(G):
+        x = np.zeros((1, 2, 2, G * Cg), dtype=np.float32)
+        x[..., s * Cg:(s + 1) * Cg] = 2.0
+        for k in range(1, G):
+            q = oracle.quantize_act(x, G, 2, inv)
+            x, _ = oracle.cyclic_shuffle_module(x, q, wq, m_out, None, 1)
+            live = {g for g in range(G) if np.any(x[..., g * Cg:(g + 1) * Cg] != 0)}
+            assert live == {(s + j) % G for j in range(k + 1)}, (G, s, k, live)
