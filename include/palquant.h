@@ -224,6 +224,23 @@ pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, cons
                                const float* shortcut_dev, int32_t* acc_out_dev, float* y_out_dev,
                                void* q_out_dev, pq_stream_t stream);
 
+/* Cyclic shuffle module (Sec. 4.2, Eq. 9-10), fused into one kernel:
+ *   Y = CyclicPermute(X):  Y[:, pi(i)] = X[:, i] with pi(i) = (i + shift) mod G (Eq. 8,
+ *                          group-level; Eq. 6 for shift = 1)
+ *   Z = X + Conv1x1(Y)     the 1x1 B-bit group convolution of the permuted codes,
+ *                          rescaled (m_out), plus the fp32 X, then ReLU if d->relu.
+ * The permutation is not a data movement: conv group g reads input group
+ * pi^-1(g) = (g - shift) mod G.  q_dev holds X's codes in d->code_format;
+ * x_dev is X in fp32 NHWC (the short-cut); z_out_dev (fp32 NHWC, nullable)
+ * receives Z and q_out_dev (nullable, d->code_format) Z's codes for the next
+ * layer, clamp(rint(z * m_req[g]), 0, 2^bits_out - 1) (m_req is then the next
+ * layer's fl(1/s) of group g, no permutation after the module).  d must be a
+ * 1x1, stride-1, pad-0 layer with Cin_g == Cout_g (PQ_EINVAL otherwise); at
+ * least one output.  Other conventions as palquant_layer_fused. */
+pq_status palquant_cyclic_shuffle_module(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
+                                         const float* m_out_host, const float* m_req_host, int32_t shift,
+                                         const float* x_dev, float* z_out_dev, void* q_out_dev, pq_stream_t stream);
+
 /* ------------------------------------------------------------------------ */
 /* Failure detection.                                                       */
 /* ------------------------------------------------------------------------ */

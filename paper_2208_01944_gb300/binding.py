@@ -29,6 +29,7 @@ EXPORTS = [
     "palquant_unpack_weight_codes_host", "palquant_quantize_act", "palquant_group_conv", "palquant_layer_fused",
     "palquant_sync_check", "palquant_set_wait_limit_ns", "palquant_watchdog_selftest", "palquant_conv_plan",
     "palquant_conv2d_f32", "palquant_maxpool2d_f32", "palquant_avgpool_f32", "palquant_linear_f32",
+    "palquant_cyclic_shuffle_module",
 ]
 
 
@@ -104,6 +105,8 @@ def _load():
     L.palquant_watchdog_selftest.argtypes = [ctypes.c_uint64, _P]
     L.palquant_conv_plan.restype = _I32
     L.palquant_conv_plan.argtypes = [ctypes.POINTER(LayerDesc), ctypes.POINTER(ConvPlan)]
+    L.palquant_cyclic_shuffle_module.restype = _I32
+    L.palquant_cyclic_shuffle_module.argtypes = [_P, _P, ctypes.POINTER(LayerDesc), _P, _P, _I32, _P, _P, _P, _P]
     for name, args in (("palquant_conv2d_f32", [_P, _P, _P, _I64] + [_I32] * 8 + [_P]),
                        ("palquant_maxpool2d_f32", [_P, _P, _I64] + [_I32] * 6 + [_P]),
                        ("palquant_avgpool_f32", [_P, _P, _I64, _I32, _I32, _I32, _P]),
@@ -265,6 +268,15 @@ def palquant_layer_fused(q_dev, w_packed_dev, d: LayerDesc, m_out, m_req=None, s
     _check(lib.palquant_layer_fused(_ptr(q_dev), _ptr(w_packed_dev), ctypes.byref(d), _ptr(mo), _ptr(mr),
                                     shuf or shuffle(1, 1), _ptr(shortcut_dev), _ptr(acc_out_dev), _ptr(y_out_dev),
                                     _ptr(q_out_dev), _stream(stream)), "palquant_layer_fused")
+
+
+def palquant_cyclic_shuffle_module(q_dev, w_packed_dev, d: LayerDesc, m_out, m_req=None, shift=1, x_dev=None,
+                                   z_out_dev=None, q_out_dev=None, stream=None):
+    mo = None if m_out is None else _f32(m_out)
+    mr = None if m_req is None else _f32(m_req)
+    _check(lib.palquant_cyclic_shuffle_module(_ptr(q_dev), _ptr(w_packed_dev), ctypes.byref(d), _ptr(mo), _ptr(mr),
+                                              int(shift), _ptr(x_dev), _ptr(z_out_dev), _ptr(q_out_dev),
+                                              _stream(stream)), "palquant_cyclic_shuffle_module")
 
 
 def palquant_sync_check(stream=None) -> int:

@@ -368,6 +368,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.relu = d->relu;
   p.qmax_out = (1 << d->bits_out) - 1;
   for (int g = 0; g < d->G; ++g) p.dst_group[g] = g;
+  for (int g = 0; g < d->G; ++g) p.src_group[g] = g;
 
   plan.supported = 1;
   plan.mode = p.mode;
@@ -465,6 +466,59 @@ void for_each_packed(const ConvParams& p, int kw, F&& f) {
                 const size_t src = (((static_cast<size_t>(g) * p.Cout_g + co) * (p.taps / kw) + i) * kw + jj) * p.Cin_g + ci;
                 f(dst, src);
               }
+}
+
+pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
+                           const float* m_out_host, const float* m_req_host, pq_shuffle shuf,
+                           const float* shortcut_dev, int32_t* acc_out_dev, float* y_out_dev, void* q_out_dev,
+                           const int* src_group, pq_stream_t stream) {
+  pq_status st = validate_desc(d);
+  if (st != PQ_OK) return st;
+  if (q_dev == nullptr || w_packed_dev == nullptr) return PQ_EINVAL;
+  if (acc_out_dev == nullptr && y_out_dev == nullptr && q_out_dev == nullptr) return PQ_EINVAL;
+  if ((y_out_dev != nullptr || q_out_dev != nullptr) && m_out_host == nullptr) return PQ_EINVAL;
+  if (q_out_dev != nullptr && m_req_host == nullptr) return PQ_EINVAL;
+  if (!aligned16(q_dev) || !aligned16(w_packed_dev) || !aligned16(acc_out_dev) || !aligned16(y_out_dev) ||
+      !aligned16(q_out_dev) || !aligned16(shortcut_dev))
+    return PQ_EINVAL;
+  ConvParams p;
+  std::vector<Phase> phases;
+  st = plan_conv(d, &p, nullptr, &phases);
+  if (st != PQ_OK) return st;
+  int dst[pq::kMaxG];
+  if (!valid_shuffle(d->G, shuf, dst)) return PQ_EINVAL;
+  if (d->N == 0) return PQ_OK;
+  // Multipliers are scaled by 2^9 inside the kernel; keep them in the range where
+  // that scaling and every product with an accumulator stay exact normal floats.
+  auto usable = [](float m) { return std::isfinite(m) && (m == 0.0f || (std::fabs(m) > 1e-30f && std::fabs(m) < 1e30f)); };
+  for (int g = 0; g < d->G; ++g) {
+    p.dst_group[g] = dst[g];
+    p.src_group[g] = src_group ? src_group[g] : g;
+    p.m_out[g] = m_out_host ? m_out_host[g] : 0.0f;
+    p.m_req[g] = m_req_host ? m_req_host[g] : 0.0f;
+    if (!usable(p.m_out[g]) || !usable(p.m_req[g])) return PQ_EINVAL;
+    p.m_out512[g] = p.m_out[g] * 512.0f;
+    p.m_req512[g] = p.m_req[g] * 512.0f;
+  }
+  p.channel_shuffle = shuf.kind == 2 ? 1 : 0;
+  p.w_packed = static_cast<const uint8_t*>(w_packed_dev);
+  p.shortcut = shortcut_dev;
+  p.acc_out = acc_out_dev;
+  p.y_out = y_out_dev;
+  p.q_out = static_cast<uint8_t*>(q_out_dev);
+  p.err = pq::device_error_word();
+  if (p.err == nullptr) return PQ_ECUDA;
+  p.wait_limit_ns = g_wait_limit_ns.load();
+  p.q_in = static_cast<const uint8_t*>(q_dev);
+  const int sms = device_sm_count();
+  if (sms <= 0) return PQ_ECUDA;
+  const int grid = static_cast<int>(std::min<int64_t>(sms, p.items));
+  if (grid <= 0) return PQ_OK;
+  CUtensorMap map;
+  std::memset(&map, 0, sizeof(map));
+  if (p.a_tma && !encode_c16_map(d, p, q_dev, &map)) return PQ_ECUDA;
+  if (pq::launch_conv_tc(p, map, grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
+  return PQ_OK;
 }
 
 }  // namespace
@@ -641,52 +695,25 @@ pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, cons
                                const float* m_out_host, const float* m_req_host, pq_shuffle shuf,
                                const float* shortcut_dev, int32_t* acc_out_dev, float* y_out_dev, void* q_out_dev,
                                pq_stream_t stream) {
+  return layer_fused_impl(q_dev, w_packed_dev, d, m_out_host, m_req_host, shuf, shortcut_dev, acc_out_dev, y_out_dev,
+                          q_out_dev, nullptr, stream);
+}
+
+pq_status palquant_cyclic_shuffle_module(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
+                                         const float* m_out_host, const float* m_req_host, int32_t shift,
+                                         const float* x_dev, float* z_out_dev, void* q_out_dev, pq_stream_t stream) {
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
-  if (q_dev == nullptr || w_packed_dev == nullptr) return PQ_EINVAL;
-  if (acc_out_dev == nullptr && y_out_dev == nullptr && q_out_dev == nullptr) return PQ_EINVAL;
-  if ((y_out_dev != nullptr || q_out_dev != nullptr) && m_out_host == nullptr) return PQ_EINVAL;
-  if (q_out_dev != nullptr && m_req_host == nullptr) return PQ_EINVAL;
-  if (!aligned16(q_dev) || !aligned16(w_packed_dev) || !aligned16(acc_out_dev) || !aligned16(y_out_dev) ||
-      !aligned16(q_out_dev) || !aligned16(shortcut_dev))
-    return PQ_EINVAL;
-  ConvParams p;
-  std::vector<Phase> phases;
-  st = plan_conv(d, &p, nullptr, &phases);
-  if (st != PQ_OK) return st;
-  int dst[pq::kMaxG];
-  if (!valid_shuffle(d->G, shuf, dst)) return PQ_EINVAL;
-  if (d->N == 0) return PQ_OK;
-  // Multipliers are scaled by 2^9 inside the kernel; keep them in the range where
-  // that scaling and every product with an accumulator stay exact normal floats.
-  auto usable = [](float m) { return std::isfinite(m) && (m == 0.0f || (std::fabs(m) > 1e-30f && std::fabs(m) < 1e30f)); };
-  for (int g = 0; g < d->G; ++g) {
-    p.dst_group[g] = dst[g];
-    p.m_out[g] = m_out_host ? m_out_host[g] : 0.0f;
-    p.m_req[g] = m_req_host ? m_req_host[g] : 0.0f;
-    if (!usable(p.m_out[g]) || !usable(p.m_req[g])) return PQ_EINVAL;
-    p.m_out512[g] = p.m_out[g] * 512.0f;
-    p.m_req512[g] = p.m_req[g] * 512.0f;
-  }
-  p.channel_shuffle = shuf.kind == 2 ? 1 : 0;
-  p.w_packed = static_cast<const uint8_t*>(w_packed_dev);
-  p.shortcut = shortcut_dev;
-  p.acc_out = acc_out_dev;
-  p.y_out = y_out_dev;
-  p.q_out = static_cast<uint8_t*>(q_out_dev);
-  p.err = pq::device_error_word();
-  if (p.err == nullptr) return PQ_ECUDA;
-  p.wait_limit_ns = g_wait_limit_ns.load();
-  p.q_in = static_cast<const uint8_t*>(q_dev);
-  const int sms = device_sm_count();
-  if (sms <= 0) return PQ_ECUDA;
-  const int grid = static_cast<int>(std::min<int64_t>(sms, p.items));
-  if (grid <= 0) return PQ_OK;
-  CUtensorMap map;
-  std::memset(&map, 0, sizeof(map));
-  if (p.a_tma && !encode_c16_map(d, p, q_dev, &map)) return PQ_ECUDA;
-  if (pq::launch_conv_tc(p, map, grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
-  return PQ_OK;
+  if (d->kh != 1 || d->kw != 1 || d->stride != 1 || d->pad != 0 || d->Cin_g != d->Cout_g) return PQ_EINVAL;
+  if (x_dev == nullptr || (z_out_dev == nullptr && q_out_dev == nullptr)) return PQ_EINVAL;
+  // Eq. 8: Y[:, pi(i)] = X[:, i] with pi(i) = (i + shift) mod G, so conv group g reads
+  // input group pi^-1(g) = (g - shift) mod G.
+  int src[pq::kMaxG];
+  if (d->G > pq::kMaxG) return PQ_EUNSUPPORTED;
+  for (int g = 0; g < d->G; ++g) src[g] = pos_mod(g - shift, d->G);
+  pq_shuffle none = {0, 0, nullptr};
+  return layer_fused_impl(q_dev, w_packed_dev, d, m_out_host, m_req_host, none, x_dev, nullptr, z_out_dev, q_out_dev,
+                          src, stream);
 }
 
 pq_status palquant_group_conv(const void* q_dev, const void* w_packed_dev, int32_t* acc_dev, const pq_layer_desc* d,

@@ -155,7 +155,7 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
         const uint32_t full = bars.a_full(ra.stage);
         mbar_arrive_expect_tx(full, p.a_tx_bytes);
         const uint32_t dst = a_base + ra.stage * p.a_stage_bytes;
-        const int chi = (item.g * p.Cin_g + kb * p.KC) >> 4;
+        const int chi = (p.src_group[item.g] * p.Cin_g + kb * p.KC) >> 4;
         if (flat)
           tma_load_3d(dst, tmA, 2 * item.rb * p.flat_box, chi, item.n, full);
         else
@@ -247,7 +247,7 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
     for (int kb = 0; kb < p.n_kb; ++kb) {
       if (!mbar_wait(bars.a_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
       const uint32_t stage = a_base + ra.stage * p.a_stage_bytes;
-      const int ch0 = item.g * p.Cin_g + kb * p.KC;  // first input channel of the K block
+      const int ch0 = p.src_group[item.g] * p.Cin_g + kb * p.KC;  // first input channel of the K block
       const uint8_t* img_src = p.q_in + item.n * p.ld_img + static_cast<int64_t>(ch0) * p.ld_c0_mul / 16;
       for (int ph = 0; ph < nph; ++ph)
       for (int r = 0; r < Hd; ++r) {

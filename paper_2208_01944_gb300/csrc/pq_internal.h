@@ -86,6 +86,7 @@ struct ConvParams {
   float m_out512[kMaxG];  // m_out * 2^9 (exact): applied to the raw accumulator, which holds acc * 2^-9
   float m_req512[kMaxG];  // m_req * 2^9 (exact)
   int dst_group[kMaxG];
+  int src_group[kMaxG];  // input group read by conv group g (identity, or the module's Eq. 8 permutation)
   int channel_shuffle;    // 1: destination channel co*G + g (per-channel scatter)
   int relu;
   int qmax_out;
