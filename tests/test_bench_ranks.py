@@ -39,7 +39,7 @@ def _rank_main(rank, world, port, times, out):
 def test_max_over_ranks_and_rate_gloo_world2():
     world = 2
     times = [3.0, 5.0]
-    with mp.Manager() as m:
+    with mp.get_context("spawn").Manager() as m:
         out = m.dict()
         mp.spawn(_rank_main, args=(world, _free_port(), times, out), nprocs=world, join=True)
         res = dict(out)

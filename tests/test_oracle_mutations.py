@@ -38,6 +38,9 @@ MUTATIONS = {
     # the shortcut added after the ReLU
     "shortcut_after_relu": ("if (shortcut) y = y + shortcut[p * C + src];\n                if (relu) y = fmaxf(y, 0.0f);",
                             "if (relu) y = fmaxf(y, 0.0f);\n                if (shortcut) y = y + shortcut[p * C + src];"),
+    # channel shuffle as the identity instead of ShuffleNet's transpose
+    "channel_shuffle_identity": ("if (kind == 2) return (int64_t)co * G + g;",
+                                 "if (kind == 2) return (int64_t)g * Cout_g + co;"),
     # step from the mean without the factor 2
     "act_step_factor": ("s_out[g] = (float)(2.0 * mean / sqrt(qp));\n    }\n}\n\nvoid oracle_weight_step",
                         "s_out[g] = (float)(mean / sqrt(qp));\n    }\n}\n\nvoid oracle_weight_step"),
@@ -71,6 +74,11 @@ def _pins_pass(L) -> bool:
         a, y, qq = oracle.epilogue(np.array([[4, -8]], dtype=np.int64), 1, [0.25], [2.0], kind=0,
                                    shortcut=np.array([[0.5, 1.0]], dtype=np.float32), relu=True, L=L)
         if list(y[0]) != [1.5, 0.0] or list(qq[0]) != [3, 0]:
+            return False
+        # channel shuffle: ShuffleNet's reshape / transpose
+        acc = np.arange(12, dtype=np.int64).reshape(1, 12)
+        _, y2, _ = oracle.epilogue(acc, 3, [1.0, 1.0, 1.0], None, kind=2, relu=False, L=L)
+        if list(y2[0]) != [float(v) for v in np.arange(12).reshape(3, 4).T.ravel()]:
             return False
         # constant-tensor step closed form
         c = np.full((1, 2, 2, 4), 1.5, dtype=np.float32)

@@ -332,3 +332,16 @@ def test_layer_op_counts():
     assert c1.int_ops == 2 * 64 * 56 * 56 * 4 * 64 * 9 * 64
     assert abs(c1.int_ops - 59.19e9) / 59.19e9 < 1e-3
     assert abs(workloads.CONFIG4.int_ops - 3.70e9) / 3.70e9 < 2e-3
+
+
+@pytest.mark.parametrize("G,Co", [(2, 3), (4, 2), (3, 5)])
+def test_epilogue_channel_shuffle_is_shufflenet_transpose(G, Co):
+    """The channel shuffle (ShuffleNet's reshape to [G, C/G], transpose, flatten) that the
+    paper pairs with the cyclic shuffle (Sec. 4.3), written with torch's reshape/transpose."""
+    gen = synth.generator(G * 7 + Co)
+    acc = torch.randint(-50, 50, (2, 3, G * Co), generator=gen).numpy().astype(np.int64)
+    a0, y0, _ = oracle.epilogue(acc, G, np.full(G, 0.5, np.float32), kind=0)
+    a2, y2, _ = oracle.epilogue(acc, G, np.full(G, 0.5, np.float32), kind=2)
+    for ref, got in ((a0, a2), (y0, y2)):
+        t = torch.from_numpy(ref).reshape(2, 3, G, Co).transpose(2, 3).reshape(ref.shape).numpy()
+        assert np.array_equal(t, got)
