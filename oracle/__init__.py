@@ -324,3 +324,43 @@ def cyclic_shuffle_module(x: np.ndarray, q: np.ndarray, wq: np.ndarray, m_out, m
     acc = group_conv(y, wq, 1, 0, L=L)
     _, z, codes = epilogue(acc, G, m_out, m_req, 0, 0, None, x, relu, bits_out, L=L)
     return z, codes
+
+
+# ---------------------------------------------------------------------------
+# Bit-level decomposition (Sec. 3.3, Eq. 4): an M-bit layer run as G^2 B-bit
+# products, G = ceil(M / B), shifted and summed:
+#   Y = sum_i sum_j X_i W_j^T 2^((i + j) B)
+# with X_i, W_j the B-bit slices of the M-bit codes.
+# ---------------------------------------------------------------------------
+def bit_slices_act(q: np.ndarray, bits_m: int, bits_b: int) -> list:
+    """Unsigned M-bit codes -> [X_0, ..., X_{G-1}], x = sum_i X_i 2^(i B), X_i in [0, 2^B - 1]."""
+    G = -(-bits_m // bits_b)
+    q = np.asarray(q).astype(np.int64)
+    return [((q >> (i * bits_b)) & ((1 << bits_b) - 1)).astype(np.uint8) for i in range(G)]
+
+
+def bit_slices_weights(wq: np.ndarray, bits_m: int, bits_b: int) -> list:
+    """Signed M-bit codes -> [W_0, ..., W_{G-1}], w = sum_j W_j 2^(j B): the lower slices
+    unsigned in [0, 2^B - 1], the top slice the signed remainder (two's complement)."""
+    G = -(-bits_m // bits_b)
+    w = np.asarray(wq).astype(np.int64)
+    out = []
+    for j in range(G):
+        if j < G - 1:
+            out.append(((w >> (j * bits_b)) & ((1 << bits_b) - 1)).astype(np.int8))
+        else:
+            out.append((w >> (j * bits_b)).astype(np.int8))  # arithmetic shift keeps the sign
+    return out
+
+
+def bitsplit_conv(q: np.ndarray, wq: np.ndarray, stride: int, pad: int, bits_m: int, bits_b: int, L=None) -> np.ndarray:
+    """Eq. 4: the M-bit convolution as G^2 B-bit convolutions, each shifted by 2^((i+j)B)
+    and summed (int64)."""
+    xs = bit_slices_act(q, bits_m, bits_b)
+    ws = bit_slices_weights(wq, bits_m, bits_b)
+    acc = None
+    for i, xi in enumerate(xs):
+        for j, wj in enumerate(ws):
+            part = group_conv(xi, wj, stride, pad, L=L) << ((i + j) * bits_b)
+            acc = part if acc is None else acc + part
+    return acc
