@@ -260,6 +260,48 @@ pq_status palquant_set_wait_limit_ns(uint64_t ns);
 pq_status palquant_watchdog_selftest(uint64_t limit_ns, pq_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
+/* Bit-level decomposition (Sec. 3.3, Eq. 4): the baseline PalQuant is        */
+/* compared with.  An M-bit layer on B-bit hardware runs as the G^2 products  */
+/* of B-bit slices, G = ceil(M / B), each shifted by 2^((i + j) B):           */
+/*   Y = sum_i sum_j X_i W_j^T 2^((i + j) B)                                 */
+/* with x = sum_i X_i 2^(iB), X_i in [0, 2^B - 1], and w = sum_j W_j 2^(jB),   */
+/* the lower weight slices unsigned B-bit and the top one the signed rest.     */
+/* Here the G^2 products form the K dimension of one tensor-core pass: the    */
+/* input channels are the slice pairs (i, j), block (i Gw + j) carrying X_i,   */
+/* and the packed weight block (i, j) holds 2^((i+j)B) W_j.  The result equals */
+/* palquant_group_conv of the M-bit layer exactly.                             */
+/*                                                                            */
+/* d describes the M-bit layer (bits_a = M_a, bits_w = M_w, one group:        */
+/* d->G == 1, codes one per byte, G * Cin_g % 16 == 0).  bits_b in 1..4.      */
+/* Shapes whose shifted weight slices are not exact E4M3 values (beyond      */
+/* (2^B - 1) 2^((Ga - 1 + Gw - 1) B) = 448, e.g. 6-bit on 2-bit hardware) or   */
+/* whose M-bit sums could reach 2^24 return PQ_EUNSUPPORTED.                   */
+/* ------------------------------------------------------------------------ */
+
+/* The decomposed layer's descriptor: Cin_g multiplied by Ga Gw, bits_a = B. */
+pq_status palquant_bitsplit_desc(const pq_layer_desc* d, int32_t bits_b, pq_layer_desc* out);
+
+/* Bytes of the slice buffer (N H W Ga Gw Cin_g); 0 if unsupported. */
+size_t palquant_bitsplit_scratch_bytes(const pq_layer_desc* d, int32_t bits_b);
+
+/* Pack the decomposed weights from the M-bit signed codes wq_host
+ * ([G][Cout_g][kh][kw][Cin_g], in [-2^(M_w-1), 2^(M_w-1) - 1], else PQ_EINVAL)
+ * into packed_host (palquant_packed_weight_bytes of the decomposed
+ * descriptor).  Host only. */
+pq_status palquant_bitsplit_pack_weight_codes_host(const int8_t* wq_host, const pq_layer_desc* d, int32_t bits_b,
+                                                   void* packed_host, size_t packed_bytes);
+
+/* Slice the M-bit activation codes q_dev (d->code_format) into xs_dev (same
+ * format, the decomposed layer's input; xs_bytes >= the scratch size). */
+pq_status palquant_bitsplit_act(const void* q_dev, void* xs_dev, size_t xs_bytes, const pq_layer_desc* d,
+                                int32_t bits_b, pq_stream_t stream);
+
+/* Eq. 4 end to end: palquant_bitsplit_act into xs_dev, then the decomposed
+ * convolution into acc_dev (int32 NHWC, as palquant_group_conv of d). */
+pq_status palquant_bitsplit_conv(const void* q_dev, void* xs_dev, size_t xs_bytes, const void* w_packed_dev,
+                                 int32_t* acc_dev, const pq_layer_desc* d, int32_t bits_b, pq_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
 /* Full-precision layers around the PalQuant body of a network.  The paper   */
 /* keeps the first and the last layer in full precision (Sec. 5); these are  */
 /* not part of the PalQuant method itself.  Each output is summed in one     */

@@ -29,7 +29,8 @@ EXPORTS = [
     "palquant_unpack_weight_codes_host", "palquant_quantize_act", "palquant_group_conv", "palquant_layer_fused",
     "palquant_sync_check", "palquant_set_wait_limit_ns", "palquant_watchdog_selftest", "palquant_conv_plan",
     "palquant_conv2d_f32", "palquant_maxpool2d_f32", "palquant_avgpool_f32", "palquant_linear_f32",
-    "palquant_cyclic_shuffle_module",
+    "palquant_cyclic_shuffle_module", "palquant_bitsplit_desc", "palquant_bitsplit_scratch_bytes",
+    "palquant_bitsplit_pack_weight_codes_host", "palquant_bitsplit_act", "palquant_bitsplit_conv",
 ]
 
 
@@ -105,6 +106,16 @@ def _load():
     L.palquant_watchdog_selftest.argtypes = [ctypes.c_uint64, _P]
     L.palquant_conv_plan.restype = _I32
     L.palquant_conv_plan.argtypes = [ctypes.POINTER(LayerDesc), ctypes.POINTER(ConvPlan)]
+    L.palquant_bitsplit_desc.restype = _I32
+    L.palquant_bitsplit_desc.argtypes = [ctypes.POINTER(LayerDesc), _I32, ctypes.POINTER(LayerDesc)]
+    L.palquant_bitsplit_scratch_bytes.restype = ctypes.c_size_t
+    L.palquant_bitsplit_scratch_bytes.argtypes = [ctypes.POINTER(LayerDesc), _I32]
+    L.palquant_bitsplit_pack_weight_codes_host.restype = _I32
+    L.palquant_bitsplit_pack_weight_codes_host.argtypes = [_P, ctypes.POINTER(LayerDesc), _I32, _P, ctypes.c_size_t]
+    L.palquant_bitsplit_act.restype = _I32
+    L.palquant_bitsplit_act.argtypes = [_P, _P, ctypes.c_size_t, ctypes.POINTER(LayerDesc), _I32, _P]
+    L.palquant_bitsplit_conv.restype = _I32
+    L.palquant_bitsplit_conv.argtypes = [_P, _P, ctypes.c_size_t, _P, _P, ctypes.POINTER(LayerDesc), _I32, _P]
     L.palquant_cyclic_shuffle_module.restype = _I32
     L.palquant_cyclic_shuffle_module.argtypes = [_P, _P, ctypes.POINTER(LayerDesc), _P, _P, _I32, _P, _P, _P, _P]
     for name, args in (("palquant_conv2d_f32", [_P, _P, _P, _I64] + [_I32] * 8 + [_P]),
@@ -317,3 +328,33 @@ def palquant_avgpool_f32(x_dev, y_dev, N, H, W, C, stream=None):
 def palquant_linear_f32(x_dev, w_dev, y_dev, N, Cin, Cout, stream=None):
     _check(lib.palquant_linear_f32(_ptr(x_dev), _ptr(w_dev), _ptr(y_dev), N, Cin, Cout, _stream(stream)),
            "palquant_linear_f32")
+
+
+# Bit-level decomposition (Eq. 4): the baseline PalQuant is compared with.
+def palquant_bitsplit_desc(d: LayerDesc, bits_b: int) -> LayerDesc:
+    out = LayerDesc()
+    _check(lib.palquant_bitsplit_desc(ctypes.byref(d), bits_b, ctypes.byref(out)), "palquant_bitsplit_desc")
+    return out
+
+
+def palquant_bitsplit_scratch_bytes(d: LayerDesc, bits_b: int) -> int:
+    return lib.palquant_bitsplit_scratch_bytes(ctypes.byref(d), bits_b)
+
+
+def palquant_bitsplit_pack_weight_codes_host(wq_host, d: LayerDesc, bits_b: int) -> np.ndarray:
+    n = palquant_packed_weight_bytes(palquant_bitsplit_desc(d, bits_b))
+    out = np.empty(n, dtype=np.uint8)
+    wq = np.ascontiguousarray(wq_host, dtype=np.int8)
+    _check(lib.palquant_bitsplit_pack_weight_codes_host(_ptr(wq), ctypes.byref(d), bits_b, _ptr(out), n),
+           "palquant_bitsplit_pack_weight_codes_host")
+    return out
+
+
+def palquant_bitsplit_act(q_dev, xs_dev, xs_bytes, d: LayerDesc, bits_b: int, stream=None):
+    _check(lib.palquant_bitsplit_act(_ptr(q_dev), _ptr(xs_dev), xs_bytes, ctypes.byref(d), bits_b, _stream(stream)),
+           "palquant_bitsplit_act")
+
+
+def palquant_bitsplit_conv(q_dev, xs_dev, xs_bytes, w_packed_dev, acc_dev, d: LayerDesc, bits_b: int, stream=None):
+    _check(lib.palquant_bitsplit_conv(_ptr(q_dev), _ptr(xs_dev), xs_bytes, _ptr(w_packed_dev), _ptr(acc_dev),
+                                      ctypes.byref(d), bits_b, _stream(stream)), "palquant_bitsplit_conv")

@@ -724,6 +724,119 @@ pq_status palquant_group_conv(const void* q_dev, const void* w_packed_dev, int32
                               stream);
 }
 
+// ---------------------------------------------------------------------------
+// Bit-level decomposition (Sec. 3.3, Eq. 4).
+// ---------------------------------------------------------------------------
+namespace {
+int ceil_div(int a, int b) { return (a + b - 1) / b; }
+
+// The decomposed layer: K blocks (i, j) for i < Ga activation slices, j < Gw
+// weight slices; PQ_OK only when every shifted weight slice value is an exact
+// E4M3 number and the M-bit products stay exact in fp32.
+pq_status bitsplit_layer(const pq_layer_desc* d, int bits_b, pq_layer_desc* out, int* ga, int* gw) {
+  pq_status st = validate_desc(d);
+  if (st != PQ_OK) return st;
+  if (bits_b < 1 || bits_b > 4) return PQ_EINVAL;
+  const int Ga = ceil_div(d->bits_a, bits_b), Gw = ceil_div(d->bits_w, bits_b);
+  // (i+1) B <= 8 keeps the byte-wise slicing exact; the largest shifted weight
+  // slice is (2^B - 1) 2^((Ga-1 + Gw-1) B) (E4M3 holds integers m 2^k with
+  // m < 16 up to 448).
+  if (Ga * bits_b > 8) return PQ_EUNSUPPORTED;
+  const int64_t wmax = ((1LL << bits_b) - 1) << ((Ga - 1 + Gw - 1) * bits_b);
+  if (wmax > 448) return PQ_EUNSUPPORTED;
+  const int64_t taps = static_cast<int64_t>(d->kh) * d->kw;
+  if (taps * d->Cin_g * ((1LL << d->bits_a) - 1) * (1LL << (d->bits_w - 1)) >= (1LL << 24)) return PQ_EUNSUPPORTED;
+  *out = *d;
+  out->Cin_g = d->Cin_g * Ga * Gw;
+  out->bits_a = bits_b;
+  out->bits_w = bits_b < 2 ? 2 : bits_b;
+  *ga = Ga;
+  *gw = Gw;
+  return PQ_OK;
+}
+}  // namespace
+
+pq_status palquant_bitsplit_desc(const pq_layer_desc* d, int32_t bits_b, pq_layer_desc* out) {
+  if (out == nullptr) return PQ_EINVAL;
+  int Ga, Gw;
+  pq_layer_desc t;
+  pq_status st = bitsplit_layer(d, bits_b, &t, &Ga, &Gw);
+  if (st != PQ_OK) return st;
+  ConvParams p;
+  st = plan_conv(&t, &p, nullptr, nullptr);
+  if (st != PQ_OK) return st;
+  *out = t;
+  return PQ_OK;
+}
+
+size_t palquant_bitsplit_scratch_bytes(const pq_layer_desc* d, int32_t bits_b) {
+  pq_layer_desc t;
+  if (palquant_bitsplit_desc(d, bits_b, &t) != PQ_OK) return 0;
+  return static_cast<size_t>(t.N) * t.H * t.W * t.G * t.Cin_g;
+}
+
+pq_status palquant_bitsplit_pack_weight_codes_host(const int8_t* wq_host, const pq_layer_desc* d, int32_t bits_b,
+                                                   void* packed_host, size_t packed_bytes) {
+  if (wq_host == nullptr || packed_host == nullptr) return PQ_EINVAL;
+  int Ga, Gw;
+  pq_layer_desc t;
+  pq_status st = bitsplit_layer(d, bits_b, &t, &Ga, &Gw);
+  if (st != PQ_OK) return st;
+  ConvParams p;
+  st = plan_conv(&t, &p, nullptr, nullptr);
+  if (st != PQ_OK) return st;
+  const size_t need = static_cast<size_t>(t.G) * t.Cout_g * t.kh * t.kw * t.Cin_g;
+  if (packed_bytes < need) return PQ_EINVAL;
+  const int lo = -(1 << (d->bits_w - 1)), hi = (1 << (d->bits_w - 1)) - 1;
+  const size_t n_codes = static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
+  for (size_t i = 0; i < n_codes; ++i)
+    if (wq_host[i] < lo || wq_host[i] > hi) return PQ_EINVAL;
+  // Weight block (i, j) holds 2^((i+j)B) w_j (w_j: slice j of w, the lower
+  // slices unsigned B-bit, the top one the signed rest), encoded as E4M3 (exact:
+  // bitsplit_layer bounded the magnitude).
+  uint8_t* out = static_cast<uint8_t*>(packed_host);
+  const int Cin_t = t.Cin_g;
+  for_each_packed(p, t.kw, [&](size_t dst, size_t src) {
+    const size_t r = src / Cin_t;
+    const int k = static_cast<int>(src - r * Cin_t);
+    const int blk = k / d->Cin_g, c = k - blk * d->Cin_g;
+    const int i = blk / Gw, j = blk - i * Gw;
+    const int w = wq_host[r * d->Cin_g + c];
+    const int wj = (j < Gw - 1) ? ((w >> (j * bits_b)) & ((1 << bits_b) - 1)) : (w >> (j * bits_b));
+    out[dst] = e4m3_of_int(wj * (1 << ((i + j) * bits_b)));
+  });
+  return PQ_OK;
+}
+
+pq_status palquant_bitsplit_act(const void* q_dev, void* xs_dev, size_t xs_bytes, const pq_layer_desc* d,
+                                int32_t bits_b, pq_stream_t stream) {
+  if (q_dev == nullptr || xs_dev == nullptr || !aligned16(q_dev) || !aligned16(xs_dev)) return PQ_EINVAL;
+  int Ga, Gw;
+  pq_layer_desc t;
+  pq_status st = bitsplit_layer(d, bits_b, &t, &Ga, &Gw);
+  if (st != PQ_OK) return st;
+  const int C = d->G * d->Cin_g;
+  if (C % 16 != 0) return PQ_EUNSUPPORTED;
+  if (xs_bytes < palquant_bitsplit_scratch_bytes(d, bits_b)) return PQ_EINVAL;
+  if (d->N == 0) return PQ_OK;
+  if (d->G != 1) return PQ_EUNSUPPORTED;  // one group: the M-bit layer of Eq. 4
+  return pq::launch_bitsplit_act(static_cast<const uint8_t*>(q_dev), static_cast<uint8_t*>(xs_dev), d->N,
+                                 static_cast<int64_t>(d->H) * d->W, C, Ga, Gw, bits_b,
+                                 d->code_format == PQ_CODES_C16 ? 1 : 0, static_cast<cudaStream_t>(stream)) == 0
+             ? PQ_OK
+             : PQ_ECUDA;
+}
+
+pq_status palquant_bitsplit_conv(const void* q_dev, void* xs_dev, size_t xs_bytes, const void* w_packed_dev,
+                                 int32_t* acc_dev, const pq_layer_desc* d, int32_t bits_b, pq_stream_t stream) {
+  pq_layer_desc t;
+  pq_status st = palquant_bitsplit_desc(d, bits_b, &t);
+  if (st != PQ_OK) return st;
+  st = palquant_bitsplit_act(q_dev, xs_dev, xs_bytes, d, bits_b, stream);
+  if (st != PQ_OK) return st;
+  return palquant_group_conv(xs_dev, w_packed_dev, acc_dev, &t, stream);
+}
+
 pq_status palquant_sync_check(pq_stream_t stream) {
   if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return PQ_ECUDA;
   unsigned int* word = pq::device_error_word();

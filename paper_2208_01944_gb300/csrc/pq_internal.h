@@ -101,6 +101,8 @@ struct ConvParams {
 
 // Host-side launch helpers implemented in the .cu files.
 int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream);
+int launch_bitsplit_act(const uint8_t* q, uint8_t* xs, int64_t N, int64_t HW, int C, int Ga, int Gw, int B, int c16,
+                        cudaStream_t stream);
 int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G, int Cg, int bits, const float* inv_s,
                         cudaStream_t stream);
 int launch_quantize(const float* x, uint8_t* q, int64_t P, int G, int Cg, int bits, const float* inv_s,

@@ -159,3 +159,35 @@ def test_unsupported_shapes_reported():
         with pytest.raises(B.PalquantError) as e:
             B.palquant_layer_fused(16, 16, d, [1.0] * 2, [1.0] * 2, acc_out_dev=16)
         assert e.value.status == B.PQ_EUNSUPPORTED
+
+
+@pytest.mark.parametrize("M,Bb", [(4, 2), (3, 2), (4, 1)])  # shifted values within int8 for the unpacker
+def test_bitsplit_weight_blocks_are_shifted_slices(M, Bb):
+    """Eq. 4's weight side: block (i, j) of the decomposed weights is 2^((i+j)B) W_j,
+    W_j the oracle's slices of the M-bit codes."""
+    d = B.layer_desc(1, 8, 8, 1, 32, 16, 3, 1, 1, M, M, 2)
+    gen = synth.generator(M * 3 + Bb)
+    wq = synth.random_codes((1, 16, 3, 3, 32), M, gen, signed=True)
+    B_bits = Bb
+    t = B.palquant_bitsplit_desc(d, B_bits)
+    Ga = Gw = -(-M // B_bits)
+    assert t.Cin_g == 32 * Ga * Gw and t.bits_a == B_bits
+    packed = B.palquant_bitsplit_pack_weight_codes_host(wq, d, B_bits)
+    vals = B.palquant_unpack_weight_codes_host(packed, t).astype(np.int64)  # [1,16,3,3,Ga*Gw*32]
+    ws = oracle.bit_slices_weights(wq, M, B_bits)
+    for i in range(Ga):
+        for j in range(Gw):
+            blk = vals[..., (i * Gw + j) * 32:(i * Gw + j + 1) * 32]
+            assert np.array_equal(blk, ws[j].astype(np.int64) << ((i + j) * B_bits))
+
+
+def test_bitsplit_unsupported_shapes():
+    # 6-bit on 2-bit hardware: shifted slices reach 3 * 2^8, beyond exact E4M3
+    d = B.layer_desc(1, 8, 8, 1, 32, 16, 3, 1, 1, 6, 6, 2)
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_bitsplit_desc(d, 2)
+    assert e.value.status == B.PQ_EUNSUPPORTED
+    assert B.palquant_bitsplit_scratch_bytes(d, 2) == 0
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_bitsplit_desc(B.layer_desc(1, 8, 8, 1, 32, 16, 3, 1, 1, 4, 4, 2), 5)
+    assert e.value.status == B.PQ_EINVAL
