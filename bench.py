@@ -321,6 +321,7 @@ def measure_layer_configs(dev, args):
                      "buffer_sets": n_sets, "plan": {k: plan[k] for k in ("m_tiles", "n_block", "k_chunk",
                                                                          "weights_resident", "work_items")}}
         del qs, qo, q, wp
+    out["table2_4bit_on_2bit"] = measure_bitsplit_vs_palquant(dev, stream, timed, pk, fp8_peak)
     for name in ("config1", "config4"):
         c = workloads.BENCH_CONFIGS[name]
         shape = (c.N, c.H, c.W, c.G * c.Cin_g)
@@ -338,6 +339,65 @@ def measure_layer_configs(dev, args):
         del xs, qq, x
     torch.cuda.empty_cache()
     return out
+
+
+def measure_bitsplit_vs_palquant(dev, stream, timed, pk, fp8_peak):
+    """The GPU analogue of the paper's Table 2 comparison on one 3x3 layer shape
+    (batch 128, 28x28, per-group width C = 256): a 4-bit layer C -> C run on 2-bit
+    operands by bit-level decomposition (Eq. 4: slice kernel + one pass over the 4
+    shifted 2-bit products), the same 4-bit layer run directly (GB300's FP8 tensor
+    cores take 4-bit codes natively), and the PalQuant layer that replaces it (G = 2
+    groups of C -> C at 2 bits, Sec. 4.1).  All produce next-layer codes."""
+    import numpy as np
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300 import synth
+
+    N, H, C, k = 128, 28, 256, 3
+    fmt = B.PQ_CODES_C16
+    gen = synth.generator(5)
+    res = {"shape": f"{N}x{H}x{H}, 3x3, C={C} per group, codes in and out"}
+    m1 = np.full(1, 0.01, np.float32)
+    # direct 4-bit and decomposed (one group, C -> C)
+    d4 = B.layer_desc(N, H, H, 1, C, C, k, 1, 1, 4, 4, 4, 1, code_format=fmt)
+    R = 5  # rotating input / output sets: each pass touches more than L2
+    q4 = [torch.from_numpy(synth.random_codes((N, H, H, C), 4, gen)).to(dev) for _ in range(R)]
+    w4 = synth.random_codes((1, C, k, k, C), 4, gen, signed=True)
+    wp4 = torch.from_numpy(B.palquant_pack_weight_codes_host(w4, d4)).to(dev)
+    qo = [torch.empty((N, H, H, C), dtype=torch.uint8, device=dev) for _ in range(R)]
+    none = B.shuffle(0, 0)
+    ms_direct = timed(lambda i: B.palquant_layer_fused(q4[i], wp4, d4, m1, m1, none, None, None, None, qo[i],
+                                                       stream=stream), R)
+    t = B.palquant_bitsplit_desc(d4, 2)
+    wps = torch.from_numpy(B.palquant_bitsplit_pack_weight_codes_host(w4, d4, 2)).to(dev)
+    xs_bytes = B.palquant_bitsplit_scratch_bytes(d4, 2)
+    xs = torch.empty(xs_bytes, dtype=torch.uint8, device=dev)
+
+    def split_run(i):
+        B.palquant_bitsplit_act(q4[i], xs, xs_bytes, d4, 2, stream=stream)
+        B.palquant_layer_fused(xs, wps, t, m1, m1, none, None, None, None, qo[i], stream=stream)
+
+    ms_split = timed(split_run, R)
+    # PalQuant: 2 groups of C -> C at 2 bits (2C channels), cyclic shuffle
+    dp = B.layer_desc(N, H, H, 2, C, C, k, 1, 1, 2, 2, 2, 1, code_format=fmt)
+    qp = [torch.from_numpy(synth.random_codes((N, H, H, 2 * C), 2, gen)).to(dev) for _ in range(R)]
+    wpq = synth.random_codes((2, C, k, k, C), 2, gen, signed=True)
+    wpp = torch.from_numpy(B.palquant_pack_weight_codes_host(wpq, dp)).to(dev)
+    qop = [torch.empty((N, H, H, 2 * C), dtype=torch.uint8, device=dev) for _ in range(R)]
+    m2 = np.full(2, 0.01, np.float32)
+    ms_pal = timed(lambda i: B.palquant_layer_fused(qp[i], wpp, dp, m2, m2, B.shuffle(1, 1), None, None, None, qop[i],
+                                                    stream=stream), R)
+    ops4 = 2 * N * H * H * C * k * k * C
+    res.update({
+        "direct_4bit_us": ms_direct * 1e3,
+        "bit_decomposed_4bit_on_2bit_us": ms_split * 1e3,
+        "palquant_2bit_G2_us": ms_pal * 1e3,
+        "speedup_palquant_vs_bit_decomposed": ms_split / ms_pal,
+        "int_ops": {"direct_4bit": ops4, "bit_decomposed_2bit_products": 4 * ops4, "palquant_G2": 2 * ops4},
+        "note": "the 4 products of Eq. 4 form one tensor-core pass (K = 4C) after a slice kernel",
+    })
+    return res
 
 
 # ---------------------------------------------------------------------------
