@@ -23,8 +23,9 @@
  *    [G][Cout_g][kh][kw][Cin_g].
  *  - Codes.  One code per byte.  Activation codes are unsigned integers in
  *    [0, 2^bits - 1]; weight codes are signed in [-2^(bits-1), 2^(bits-1) - 1].
- *    An activation code tensor is either NHWC (PQ_CODES_INT8) or channel-blocked
- *    (PQ_CODES_C16, see pq_code_format); both hold the same integer values.
+ *    An activation code tensor is NHWC (PQ_CODES_INT8), channel-blocked
+ *    (PQ_CODES_C16) or channel-blocked with 2-bit codes packed four to a byte
+ *    (PQ_CODES_C16P2), see pq_code_format; all hold the same integer values.
  *  - Memory.  The caller owns every buffer.  Pointers named *_dev are device
  *    pointers, *_host are host pointers.  The compute calls allocate nothing;
  *    small host arrays (per-group scalars, permutations) are copied into the
@@ -62,10 +63,16 @@ typedef enum {
 typedef enum {
     PQ_CODES_INT8 = 0, /* code v stored as the byte v, NHWC: byte (((n*H + h)*W + w)*C + c) */
     PQ_CODES_E4M3 = 1, /* reserved (PQ_EUNSUPPORTED) */
-    PQ_CODES_C16 = 2   /* code v stored as the byte v, channel-blocked in 16-channel blocks:
+    PQ_CODES_C16 = 2,  /* code v stored as the byte v, channel-blocked in 16-channel blocks:
                           byte ((((n*(C/16) + c/16)*H + h)*W + w)*16 + c%16).  C % 16 == 0.
                           The tensor cores' operand layout: every run of positions of one
-                          16-channel block is contiguous.  The fastest format. */
+                          16-channel block is contiguous. */
+    PQ_CODES_C16P2 = 3 /* 2-bit codes packed four to a byte, channel-blocked: the 16 codes of
+                          a position and 16-channel block form one little-endian 32-bit word
+                          at byte ((((n*(C/16) + c/16)*H + h)*W + w)*4), code of channel c at
+                          bits 2 (c % 16).  bits <= 2, C % 16 == 0; as a layer input it needs
+                          stride 1 and W % 4 == 0 (H W % 4 == 0 for 1x1 layers).  A quarter
+                          of the bytes of PQ_CODES_C16. */
 } pq_code_format;
 
 /* Output channel permutation (Sec. 4.2).  kind:
@@ -191,7 +198,8 @@ pq_status palquant_unpack_weight_codes_host(const void* packed_host, const pq_la
  *   q[p, g*Cg + j] = clamp(rint(x[p, g*Cg + j] * inv_s[g]), 0, 2^bits - 1)
  * x_dev is NHWC fp32 [N,H,W,G*Cg]; q_dev receives one byte per element in
  * code_format (PQ_CODES_INT8: NHWC; PQ_CODES_C16: channel-blocked, needs
- * Cg % 16 == 0).  inv_s_host holds G floats (fl(1/s) of the steps), copied at
+ * Cg % 16 == 0; PQ_CODES_C16P2: channel-blocked 2-bit codes four to a byte,
+ * needs Cg % 16 == 0 and bits <= 2).  inv_s_host holds G floats (fl(1/s) of the steps), copied at
  * call time.  NaN maps to 0 and +inf to 2^bits - 1.  bits in 1..8. */
 pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G,
                                 int32_t Cg, int32_t bits, int32_t code_format, const float* inv_s_host,

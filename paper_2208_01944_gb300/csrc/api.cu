@@ -87,7 +87,8 @@ pq_status validate_desc(const pq_layer_desc* d) {
   if (d->bits_a < 1 || d->bits_a > 8 || d->bits_w < 2 || d->bits_w > 8 || d->bits_out < 1 || d->bits_out > 8)
     return PQ_EINVAL;
   if (d->relu != 0 && d->relu != 1) return PQ_EINVAL;
-  if (d->code_format != PQ_CODES_INT8 && d->code_format != PQ_CODES_E4M3 && d->code_format != PQ_CODES_C16)
+  if (d->code_format != PQ_CODES_INT8 && d->code_format != PQ_CODES_E4M3 && d->code_format != PQ_CODES_C16 &&
+      d->code_format != PQ_CODES_C16P2)
     return PQ_EINVAL;
   if (out_dim(d->H, d->kh, d->stride, d->pad) < 1 || out_dim(d->W, d->kw, d->stride, d->pad) < 1) return PQ_EINVAL;
   if (d->G > pq::kMaxG) return PQ_EUNSUPPORTED;
@@ -121,8 +122,14 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const int qa = (1 << d->bits_a) - 1;
   const int qw = 1 << (d->bits_w - 1);
   // Coverage of the tensor-core kernel.
-  const bool c16 = d->code_format == PQ_CODES_C16;
-  bool ok = (d->code_format == PQ_CODES_INT8 || c16) && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
+  const bool p2 = d->code_format == PQ_CODES_C16P2;
+  const bool c16 = d->code_format == PQ_CODES_C16 || p2;  // channel-blocked (bytes or packed)
+  // Packed 2-bit codes: 2-bit input and output codes, stride 1, and 16-byte aligned
+  // rows (1x1: image planes) for the TMA loads of the packed tile.
+  const bool flat_shape = d->kh == 1 && d->kw == 1 && d->stride == 1 && d->pad == 0;
+  const bool p2_ok = !p2 || (d->bits_a <= 2 && d->bits_out <= 2 && d->stride == 1 &&
+                             (flat_shape ? (static_cast<int64_t>(d->H) * d->W) % 4 == 0 : d->W % 4 == 0));
+  bool ok = (d->code_format == PQ_CODES_INT8 || c16) && p2_ok && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
             d->pad < std::max(d->kh, d->kw) && d->Cin_g % 32 == 0 && d->Cout_g % 16 == 0 && taps <= pq::kMaxTaps &&
             static_cast<int64_t>(taps) * d->Cin_g * qa * qw < (1LL << 24);
   if (!ok) {
@@ -275,6 +282,21 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const uint32_t stage_total = warp_stage * (pq::kEpiWarps + pq::kLoadWarps);
   const uint32_t bar_bytes = 1024;  // barriers, abort flag, TMEM slot (generous)
   const uint64_t unit_bytes = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk;
+  // Packed codes: a staging stage per operand stage holding the TMA box of 32-bit
+  // words (rows start at the tile's first position rounded down to a multiple of
+  // 4, the TMA's 16-byte alignment of the innermost coordinate).
+  const int pk_x0 = flat ? 0 : static_cast<int>(std::floor(p.w_coord / 4.0)) * 4;
+  const int pk_off = flat ? 0 : p.w_coord - pk_x0;
+  const int pk_box_w = flat ? p.flat_box : static_cast<int>(round_up(static_cast<uint64_t>(p.Wd + pk_off), 4));
+  if (p2 && pk_box_w > 256) {
+    if (pub) *pub = plan;
+    return PQ_EUNSUPPORTED;
+  }
+  auto pk_stage_bytes = [&](int KC) -> uint32_t {
+    if (!p2) return 0;
+    const uint64_t rows = flat ? 1 : p.Hd;
+    return round_up(static_cast<uint64_t>(pk_box_w) * rows * (KC / 16) * 4, 1024);
+  };
   // Largest K block (input channels per pipeline stage) that fits: the whole
   // unit's weights resident if they fit, else a ring of (K block, tap) slices.
   bool found = false, resident = false;
@@ -295,7 +317,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
       for (int na = 4; na >= 2 && !found; --na) {
         for (int nb = (res ? 1 : 4); nb >= (res ? 1 : 2) && !found; --nb) {
           const uint64_t bb = res ? round_up(unit_bytes, 1024) : round_up(nb * slice, 1024);
-          if (bb + stage_total + bar_bytes + static_cast<uint64_t>(na) * sb <= budget) {
+          if (bb + stage_total + bar_bytes + static_cast<uint64_t>(na) * (sb + pk_stage_bytes(kc)) <= budget) {
             found = true;
             resident = res != 0;
             KC = kc;
@@ -323,11 +345,17 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.C_in_total = d->G * d->Cin_g;
   p.img_pix = d->H * d->W;
   p.codes_c16 = c16 ? 1 : 0;
+  p.codes_p2 = p2 ? 1 : 0;
+  p.a_unpack = p2 ? 1 : 0;
+  p.pk_box_w = pk_box_w;
+  p.pk_off = pk_off;
+  p.pk_stage_bytes = pk_stage_bytes(KC);
   // The A operand comes by TMA when every plane row is one contiguous run in
   // global memory: channel-blocked codes, stride 1, rows of at most 128 positions.
-  p.a_tma = (c16 && d->stride == 1 && (flat ? p.flat_box == 128 : p.Wd <= 128)) ? 1 : 0;
-  p.a_tx_bytes = flat ? static_cast<uint32_t>(p.nch) * p.flat_box * 16u
-                      : static_cast<uint32_t>(p.nph) * p.nch * p.Hd * p.Wd * 16u;
+  p.a_tma = (p2 || (c16 && d->stride == 1 && (flat ? p.flat_box == 128 : p.Wd <= 128))) ? 1 : 0;
+  p.a_tx_bytes = p2 ? static_cast<uint32_t>(p.nch) * pk_box_w * (flat ? 1 : p.Hd) * 4u
+                 : flat ? static_cast<uint32_t>(p.nch) * p.flat_box * 16u
+                        : static_cast<uint32_t>(p.nph) * p.nch * p.Hd * p.Wd * 16u;
   {
     const int64_t C = p.C_in_total, H = d->H, W = d->W;
     if (c16) {
@@ -359,7 +387,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.tmem_cols = static_cast<uint32_t>(next_pow2(std::max(32, p.acc_stages * p.MT * p.Npow2)));
   p.smem_b_off = static_cast<uint32_t>(a_stages) * stage_bytes;
   p.smem_stage_off = p.smem_b_off + b_bytes;
-  p.smem_bar_off = p.smem_stage_off + stage_total;
+  p.smem_pk_off = p.smem_stage_off + stage_total;  // packed staging ring (a_stages x pk_stage_bytes)
+  p.smem_bar_off = p.smem_pk_off + static_cast<uint32_t>(a_stages) * p.pk_stage_bytes;
   p.smem_bytes = p.smem_bar_off + bar_bytes;
   p.stage_q_pitch = q_pitch;
   p.stage_f_pitch = f_pitch;
@@ -425,6 +454,24 @@ bool encode_c16_map(const pq_layer_desc* d, const ConvParams& p, const void* q_d
   std::memset(map, 0, sizeof(*map));
   const uint64_t C16 = static_cast<uint64_t>(d->G) * d->Cin_g / 16, H = d->H, W = d->W;
   cuuint32_t es[4] = {1, 1, 1, 1};
+  if (p.codes_p2) {
+    // Packed codes: one 32-bit word per (position, 16-channel block).
+    if (p.mode == pq::kModeFlat) {
+      cuuint64_t dims[3] = {H * W, C16, static_cast<cuuint64_t>(d->N)};
+      cuuint64_t strides[2] = {H * W * 4, C16 * H * W * 4};
+      cuuint32_t box[3] = {static_cast<cuuint32_t>(p.pk_box_w), static_cast<cuuint32_t>(p.nch), 1};
+      return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT32, 3, const_cast<void*>(q_dev), dims, strides, box, es,
+                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+    }
+    cuuint64_t dims[4] = {W, H, C16, static_cast<cuuint64_t>(d->N)};
+    cuuint64_t strides[3] = {W * 4, H * W * 4, C16 * H * W * 4};
+    cuuint32_t box[4] = {static_cast<cuuint32_t>(p.pk_box_w), static_cast<cuuint32_t>(p.Hd),
+                         static_cast<cuuint32_t>(p.nch), 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT32, 4, const_cast<void*>(q_dev), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
   if (p.mode == pq::kModeFlat) {
     cuuint64_t dims[3] = {2 * H * W, C16, static_cast<cuuint64_t>(d->N)};
     cuuint64_t strides[2] = {H * W * 16, C16 * H * W * 16};
@@ -501,6 +548,8 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
     p.m_req512[g] = p.m_req[g] * 512.0f;
   }
   p.channel_shuffle = shuf.kind == 2 ? 1 : 0;
+  // A per-channel scatter cannot write single 2-bit codes into packed bytes.
+  if (p.channel_shuffle && p.codes_p2 && q_out_dev != nullptr) return PQ_EUNSUPPORTED;
   p.w_packed = static_cast<const uint8_t*>(w_packed_dev);
   p.shortcut = shortcut_dev;
   p.acc_out = acc_out_dev;
@@ -675,13 +724,14 @@ pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int3
   if (N < 0 || H < 1 || W < 1 || G < 1 || Cg < 1 || bits < 1 || bits > 8) return PQ_EINVAL;
   if (G > pq::kMaxG) return PQ_EUNSUPPORTED;
   if (code_format == PQ_CODES_E4M3) return PQ_EUNSUPPORTED;
-  if (code_format != PQ_CODES_INT8 && code_format != PQ_CODES_C16) return PQ_EINVAL;
+  if (code_format != PQ_CODES_INT8 && code_format != PQ_CODES_C16 && code_format != PQ_CODES_C16P2) return PQ_EINVAL;
   const int64_t P = N * H * W;
-  if (code_format == PQ_CODES_C16) {
+  if (code_format == PQ_CODES_C16 || code_format == PQ_CODES_C16P2) {
     if (Cg % 16 != 0) return PQ_EINVAL;
+    if (code_format == PQ_CODES_C16P2 && bits > 2) return PQ_EINVAL;
     if (!aligned16(x_dev) || !aligned16(q_dev)) return PQ_EINVAL;
     if (pq::launch_quantize_c16(x_dev, static_cast<uint8_t*>(q_dev), N, static_cast<int64_t>(H) * W, G, Cg, bits,
-                                inv_s_host, static_cast<cudaStream_t>(stream)) != 0)
+                                inv_s_host, code_format == PQ_CODES_C16P2, static_cast<cudaStream_t>(stream)) != 0)
       return PQ_ECUDA;
     return PQ_OK;
   }
@@ -818,6 +868,7 @@ pq_status palquant_bitsplit_act(const void* q_dev, void* xs_dev, size_t xs_bytes
   const int C = d->G * d->Cin_g;
   if (C % 16 != 0) return PQ_EUNSUPPORTED;
   if (xs_bytes < palquant_bitsplit_scratch_bytes(d, bits_b)) return PQ_EINVAL;
+  if (d->code_format == PQ_CODES_C16P2) return PQ_EUNSUPPORTED;  // M-bit codes are one per byte
   if (d->N == 0) return PQ_OK;
   if (d->G != 1) return PQ_EUNSUPPORTED;  // one group: the M-bit layer of Eq. 4
   return pq::launch_bitsplit_act(static_cast<const uint8_t*>(q_dev), static_cast<uint8_t*>(xs_dev), d->N,

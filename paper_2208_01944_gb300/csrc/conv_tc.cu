@@ -104,7 +104,8 @@ __device__ __forceinline__ void item_next(const ConvParams& p, Item& r) {
 // Shared-memory barrier block layout (64-bit words):
 //   [0, A)           a_full       [A, 2A)        a_empty
 //   [2A, 2A+B)       b_full       [2A+B, 2A+2B)  b_empty
-//   +0,+1 acc_full, +2,+3 acc_empty, +4 drain, then int abort flag, u32 TMEM base.
+//   +0,+1 acc_full, +2,+3 acc_empty, +4 drain, then A pk_full and A pk_empty
+//   (packed codes only), then int abort flag, u32 TMEM base.
 struct Bars {
   uint32_t base;
   int A, B;
@@ -115,7 +116,10 @@ struct Bars {
   __device__ uint32_t acc_full(int s) const { return base + 8u * (2 * A + 2 * B + s); }
   __device__ uint32_t acc_empty(int s) const { return base + 8u * (2 * A + 2 * B + 2 + s); }
   __device__ uint32_t drain() const { return base + 8u * (2 * A + 2 * B + 4); }
-  __device__ uint32_t words() const { return 2 * A + 2 * B + 5; }
+  // packed-code staging ring (one stage per operand stage)
+  __device__ uint32_t pk_full(int s) const { return base + 8u * (2 * A + 2 * B + 5 + s); }
+  __device__ uint32_t pk_empty(int s) const { return base + 8u * (3 * A + 2 * B + 5 + s); }
+  __device__ uint32_t words() const { return 4 * A + 2 * B + 5; }
 };
 
 // --------------------------------------------------------------------------
@@ -126,8 +130,8 @@ struct Bars {
 // contiguous run there).
 // --------------------------------------------------------------------------
 __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtensorMap* tmA, const Bars& bars,
-                                              uint32_t a_base, uint32_t b_base, int64_t it0, int64_t it1,
-                                              const WaitCtx& ctx) {
+                                              uint32_t a_base, uint32_t b_base, uint32_t pk_base, int64_t it0,
+                                              int64_t it1, const WaitCtx& ctx) {
   Ring ra{0, 0, static_cast<uint32_t>(p.a_stages)};
   Ring rb{0, 0, static_cast<uint32_t>(p.b_resident ? 1 : p.b_stages)};
   int64_t a_issued = 0, b_issued = 0;
@@ -150,7 +154,21 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
     }
     if (!a_tma && p.b_resident) continue;
     for (int kb = 0; kb < p.n_kb && ok; ++kb) {
-      if (a_tma) {
+      if (a_tma && p.a_unpack) {
+        // Packed codes: the box of 32-bit words into the staging ring; the copy
+        // warps unpack it into the operand stage.
+        if (!mbar_wait(bars.pk_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
+        const uint32_t full = bars.pk_full(ra.stage);
+        mbar_arrive_expect_tx(full, p.a_tx_bytes);
+        const uint32_t dst = pk_base + ra.stage * p.pk_stage_bytes;
+        const int chi = (p.src_group[item.g] * p.Cin_g + kb * p.KC) >> 4;
+        if (flat)
+          tma_load_3d(dst, tmA, item.rb * p.flat_box, chi, item.n, full);
+        else
+          tma_load_4d(dst, tmA, p.w_coord - p.pk_off, item.oh0(p.Ht) + p.h_off, chi, item.n, full);
+        ra.advance();
+        ++a_issued;
+      } else if (a_tma) {
         if (!mbar_wait(bars.a_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
         const uint32_t full = bars.a_full(ra.stage);
         mbar_arrive_expect_tx(full, p.a_tx_bytes);
@@ -178,7 +196,8 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
   // Drain: the last min(stages, issued) copies of each ring may still be in flight.
   const int64_t na = p.a_stages, nbs = p.b_resident ? 1 : p.b_stages;
   for (int64_t k = (a_issued > na ? a_issued - na : 0); k < a_issued; ++k)
-    mbar_wait_drain(bars.a_full(static_cast<int>(k % na)), static_cast<uint32_t>((k / na) & 1), ctx.limit_ns, ctx.err);
+    mbar_wait_drain(p.a_unpack ? bars.pk_full(static_cast<int>(k % na)) : bars.a_full(static_cast<int>(k % na)),
+                    static_cast<uint32_t>((k / na) & 1), ctx.limit_ns, ctx.err);
   for (int64_t k = (b_issued > nbs ? b_issued - nbs : 0); k < b_issued; ++k)
     mbar_wait_drain(bars.b_full(static_cast<int>(k % nbs)), static_cast<uint32_t>((k / nbs) & 1), ctx.limit_ns, ctx.err);
 }
@@ -308,6 +327,56 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
   while (released < issued) {
     load_release(bars, released, p.a_stages);
     ++released;
+  }
+}
+
+// --------------------------------------------------------------------------
+// Unpack role for packed 2-bit codes (warps 2-5): each staged TMA box of
+// 32-bit words (16 codes of one position and 16-channel chunk) is expanded into
+// the operand stage, one byte per code.  A staged row of chunk j and tile row r
+// holds pk_box_w words starting pk_off positions left of the tile's first
+// position (the TMA start is rounded down to 16 bytes); positions outside the
+// image were zero-filled by the TMA unit, which is the zero padding.  Warp wi
+// takes rows wi, wi + 4, ... and its lanes consecutive positions, so the 4-byte
+// reads and 16-byte writes of shared memory are conflict-free.  The stage is
+// released to the tensor core after a proxy fence (generic writes, async-proxy
+// reads), and the staging stage back to the producer.
+// --------------------------------------------------------------------------
+__device__ __forceinline__ void unpack_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t pk_base,
+                                            int64_t it0, int64_t it1, const WaitCtx& ctx) {
+  const int tid = threadIdx.x - 32 * kFirstLoadWarp;
+  const int wi = tid >> 5, lane = tid & 31;
+  const bool flat = p.mode == kModeFlat;
+  const int row_len = flat ? p.flat_box : p.Wd;
+  const int n_rows = p.nch * (flat ? 1 : p.Hd);
+  const int Hd = flat ? 1 : p.Hd;
+  const uint32_t plane = p.lbo_a;  // bytes between 16-channel chunks of the operand stage
+  Ring r{0, 0, static_cast<uint32_t>(p.a_stages)};
+  bool ok = true;
+  for (int64_t it = it0; it < it1 && ok; ++it) {
+    for (int kb = 0; kb < p.n_kb; ++kb) {
+      if (!mbar_wait(bars.pk_full(r.stage), r.phase, ctx)) { ok = false; break; }
+      if (!mbar_wait(bars.a_empty(r.stage), r.phase ^ 1u, ctx)) { ok = false; break; }
+      const uint32_t src = pk_base + r.stage * p.pk_stage_bytes;
+      const uint32_t dst = a_base + r.stage * p.a_stage_bytes;
+      for (int row = wi; row < n_rows; row += kLoadWarps) {
+        const int j = row / Hd, rr = row - j * Hd;
+        const uint32_t srow = src + static_cast<uint32_t>(row * p.pk_box_w + p.pk_off) * 4u;
+        const uint32_t drow = dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(rr * row_len) * 16u;
+        for (int w = lane; w < row_len; w += 32) {
+          uint32_t v;
+          asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(srow + static_cast<uint32_t>(w) * 4u) : "memory");
+          const uint4 u = unpack2_word(v);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(drow + static_cast<uint32_t>(w) * 16u),
+                       "r"(u.x), "r"(u.y), "r"(u.z), "r"(u.w)
+                       : "memory");
+        }
+      }
+      fence_proxy_async_smem();
+      mbar_arrive(bars.a_full(r.stage));
+      mbar_arrive(bars.pk_empty(r.stage));
+      r.advance();
+    }
   }
 }
 
@@ -528,16 +597,25 @@ __device__ __forceinline__ uint4 epi_codes16(const uint32_t (&v)[16], float m_re
   return w;
 }
 
+// 16 codes (one per byte of w) to global memory: as they are, or packed four to
+// a byte (channel-blocked 2-bit layout).
+__device__ __forceinline__ void store_codes16(uint8_t* dst, uint4 w, int packed2) {
+  if (packed2)
+    *reinterpret_cast<uint32_t*>(dst) = pack2_word(w);
+  else
+    *reinterpret_cast<uint4*>(dst) = w;
+}
+
 // Store 16 codes of 16-column chunk `ch` of the row (output pixel pos).
 __device__ __forceinline__ void epi_store_codes(const ConvParams& p, const EpiItem& e, uint8_t* stg, int lane, bool valid,
                                                 int pos, int ch, uint4 w) {
   const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
   if (p.codes_c16) {
-    // Channel-blocked codes: lanes hold consecutive pixels, so each 16-byte
-    // store of the warp lands next to its neighbours'.
+    // Channel-blocked codes: lanes hold consecutive pixels, so each store of the
+    // warp lands next to its neighbours'.
     if (valid) {
       const long long blk = (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (e.dst_c0 >> 4) + ch) * hw_out + pos;
-      *reinterpret_cast<uint4*>(p.q_out + blk * 16) = w;
+      store_codes16(p.q_out + blk * (p.codes_p2 ? 4 : 16), w, p.codes_p2);
     }
   } else {
     // NHWC: staged, then 16-byte rows written by the warp.
@@ -667,7 +745,8 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
       // increasing (mt, ch) order; the destination of this lane's row is
       // computed once per accumulator, and 16-channel block ch of that row lies
       // ch * H_out * W_out * 16 bytes further on.
-      const long long chunk_bytes = static_cast<long long>(p.Ho) * p.Wo * 16;
+      const int code_bytes = p.codes_p2 ? 4 : 16;  // bytes per (position, 16-channel chunk)
+      const long long chunk_bytes = static_cast<long long>(p.Ho) * p.Wo * code_bytes;
       uint8_t* const blk0 = p.q_out + (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (e.dst_c0 >> 4)) * chunk_bytes;
       const int m_lane = quarter * 32 + lane;
       const int MT = p.MT;
@@ -675,7 +754,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         if (mt >= MT) return nullptr;
         bool valid;
         const int pos = epi_pos(p, e, mt * 128 + m_lane, valid);
-        return valid ? blk0 + static_cast<long long>(pos) * 16 : nullptr;
+        return valid ? blk0 + static_cast<long long>(pos) * code_bytes : nullptr;
       };
       auto step = [&](int& mt, int& ch) {
         ch += n_groups;
@@ -701,7 +780,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         if (n_mt < MT) tmem_ld16(col(n_mt, n_ch), vb);
         {
           const uint4 w = epi_codes16(va, e.m_req512, qmax_f);
-          if (c_row) *reinterpret_cast<uint4*>(c_row + c_ch * chunk_bytes) = w;
+          if (c_row) store_codes16(c_row + c_ch * chunk_bytes, w, p.codes_p2);
         }
         tmem_wait_ld();
         if (n_mt >= MT) break;
@@ -711,7 +790,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         if (m2 < MT) tmem_ld16(col(m2, c2), va);
         {
           const uint4 w = epi_codes16(vb, e.m_req512, qmax_f);
-          if (n_row) *reinterpret_cast<uint4*>(n_row + n_ch * chunk_bytes) = w;
+          if (n_row) store_codes16(n_row + n_ch * chunk_bytes, w, p.codes_p2);
         }
         tmem_wait_ld();
         c_row = m2 == n_mt ? n_row : row_ptr(m2);
@@ -752,8 +831,12 @@ __global__ void __launch_bounds__(kConvThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < bars.A; ++s) {
-      mbar_init(bars.a_full(s), p.a_tma ? 1 : 32 * kLoadWarps);
+      mbar_init(bars.a_full(s), (p.a_tma && !p.a_unpack) ? 1 : 32 * kLoadWarps);
       mbar_init(bars.a_empty(s), 1);
+      if (p.a_unpack) {
+        mbar_init(bars.pk_full(s), 1);
+        mbar_init(bars.pk_empty(s), 32 * kLoadWarps);
+      }
     }
     for (int s = 0; s < bars.B; ++s) {
       mbar_init(bars.b_full(s), 1);
@@ -761,7 +844,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     }
     for (int s = 0; s < 2; ++s) {
       mbar_init(bars.acc_full(s), 1);
-      mbar_init(bars.acc_empty(s), (p.a_tma ? kEpiWarps + kLoadWarps : kEpiWarps) * 32);
+      mbar_init(bars.acc_empty(s), ((p.a_tma && !p.a_unpack) ? kEpiWarps + kLoadWarps : kEpiWarps) * 32);
     }
     mbar_init(bars.drain(), 1);
     *abort_flag = 0;
@@ -781,7 +864,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   if (warp == 0) {
     if (lane == 0) {
       if (p.a_tma) prefetch_tmap(&tmA);
-      producer_role(p, &tmA, bars, a_base, b_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
+      producer_role(p, &tmA, bars, a_base, b_base, base + p.smem_pk_off, it0, it1,
+                    WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
     }
     __syncwarp();
   } else if (warp == 1) {
@@ -790,10 +874,15 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     __syncwarp();
   } else if (warp < kFirstEpiWarp && !p.a_tma) {
     loader_role(p, bars, a_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
+  } else if (warp < kFirstEpiWarp && p.a_unpack) {
+    unpack_role(p, bars, a_base, base + p.smem_pk_off, it0, it1,
+                WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else {
-    // With TMA loading the activations, the copy warps form a third epilogue warpgroup.
-    const int first = p.a_tma ? kFirstLoadWarp : kFirstEpiWarp;
-    epilogue_role(p, bars, tmem_base, gbase + p.smem_stage_off, first, p.a_tma ? kEpiGroups + 1 : kEpiGroups, it0, it1,
+    // With TMA loading the activations as they are, the copy warps form a third
+    // epilogue warpgroup.
+    const bool third = p.a_tma && !p.a_unpack;
+    const int first = third ? kFirstLoadWarp : kFirstEpiWarp;
+    epilogue_role(p, bars, tmem_base, gbase + p.smem_stage_off, first, third ? kEpiGroups + 1 : kEpiGroups, it0, it1,
                   WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_EPILOGUE});
   }
   tc_fence_before();

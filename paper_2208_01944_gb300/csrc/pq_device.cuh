@@ -179,6 +179,32 @@ __device__ __forceinline__ void add2_rn(float a, float b, float m, float& x, flo
       : "f"(a), "f"(b), "f"(m));
 }
 
+// ------------------------------------------------------------- packed codes
+// Sixteen 2-bit codes (one per byte of w, each <= 3) packed into one 32-bit word,
+// code k at bits 2k: the product of a byte quadruple with 2^24 + 2^18 + 2^12 + 2^6
+// moves byte k's value to bits 24 + 2k without carries (every partial product
+// occupies its own bit pair), and the top byte holds the four codes.
+__device__ __forceinline__ uint32_t pack2_quad(uint32_t x) { return (x * 0x01041040u) >> 24; }
+
+__device__ __forceinline__ uint32_t pack2_word(uint4 w) {
+  return pack2_quad(w.x) | (pack2_quad(w.y) << 8) | (pack2_quad(w.z) << 16) | (pack2_quad(w.w) << 24);
+}
+
+// Inverse: the 16 codes of a packed word, one per byte.  Even codes sit in the
+// low two bits of the nibbles of (v & 0x33333333), odd codes in those of
+// ((v >> 2) & 0x33333333); byte permutes interleave them back in order.
+__device__ __forceinline__ uint4 unpack2_word(uint32_t v) {
+  const uint32_t e = v & 0x33333333u, o = (v >> 2) & 0x33333333u;
+  const uint32_t e_lo = e & 0x0F0F0F0Fu, e_hi = (e >> 4) & 0x0F0F0F0Fu;  // codes 0,4,8,12 | 2,6,10,14
+  const uint32_t o_lo = o & 0x0F0F0F0Fu, o_hi = (o >> 4) & 0x0F0F0F0Fu;  // codes 1,5,9,13 | 3,7,11,15
+  const uint32_t a = __byte_perm(e_lo, o_lo, 0x5140);  // 0 1 4 5
+  const uint32_t b = __byte_perm(e_hi, o_hi, 0x5140);  // 2 3 6 7
+  const uint32_t c = __byte_perm(e_lo, o_lo, 0x7362);  // 8 9 12 13
+  const uint32_t d = __byte_perm(e_hi, o_hi, 0x7362);  // 10 11 14 15
+  return make_uint4(__byte_perm(a, b, 0x5410), __byte_perm(a, b, 0x7632), __byte_perm(c, d, 0x5410),
+                    __byte_perm(c, d, 0x7632));
+}
+
 // ------------------------------------------------------------------ tcgen05
 // Shared-memory matrix descriptor, no swizzle, K-major: core matrices of
 // 8 rows x 16 bytes; `lbo` = byte distance between core matrices adjacent in K,

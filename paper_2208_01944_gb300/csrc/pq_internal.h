@@ -45,6 +45,13 @@ struct ConvParams {
   int C_in_total;         // G * Cin_g (bytes per input pixel)
   int img_pix;            // H * W (flat mode tiles stay inside one image)
   int codes_c16;          // 1: input and output codes in the channel-blocked layout [N][C/16][H][W][16]
+  int codes_p2;           // 1: channel-blocked 2-bit codes packed four to a byte ([N][C/16][H][W][4 B])
+  // Packed activations come by TMA into a staging ring and the copy warps unpack
+  // them into the operand stages (a_unpack = 1): staged rows of pk_box_w 32-bit
+  // words starting pk_off words left of the tile's first position.
+  int a_unpack;
+  int pk_box_w, pk_off;
+  uint32_t pk_stage_bytes, smem_pk_off;
   int a_tma;              // 1: warp 0 loads the A operand with one TMA per stage (channel-blocked codes, stride 1)
   uint32_t a_tx_bytes;    // bytes one A stage receives (TMA mode)
   // Activation copy addressing (cp.async mode), in bytes: code (n, ih, iw, c0 + 16 j) of the
@@ -104,7 +111,7 @@ int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cuda
 int launch_bitsplit_act(const uint8_t* q, uint8_t* xs, int64_t N, int64_t HW, int C, int Ga, int Gw, int B, int c16,
                         cudaStream_t stream);
 int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G, int Cg, int bits, const float* inv_s,
-                        cudaStream_t stream);
+                        bool packed2, cudaStream_t stream);
 int launch_quantize(const float* x, uint8_t* q, int64_t P, int G, int Cg, int bits, const float* inv_s,
                     cudaStream_t stream);
 int launch_act_sum(const float* x, int64_t P, int G, int Cg, double* partial, int nblocks, cudaStream_t stream);

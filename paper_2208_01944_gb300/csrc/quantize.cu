@@ -12,6 +12,7 @@
 #include <cstdint>
 
 #include "pq_internal.h"
+#include "pq_device.cuh"
 
 namespace pq {
 
@@ -73,7 +74,8 @@ __global__ void __launch_bounds__(256) pq_quantize_scalar(const float* __restric
 // pixel rows are read by neighbouring warps at about the same time.  A grid of a
 // few blocks per SM, striding over the (image, pixel group, block group) units,
 // keeps enough loads in flight for the HBM bandwidth.
-__global__ void __launch_bounds__(256) pq_quantize_c16(const float4* __restrict__ x, uint4* __restrict__ q, int64_t N,
+template <bool PACK2>
+__global__ void __launch_bounds__(256) pq_quantize_c16(const float4* __restrict__ x, void* __restrict__ q, int64_t N,
                                                        int64_t HW, int C16, int blocks_per_group, int qmax,
                                                        const __grid_constant__ QuantArgs args) {
   const int lane = threadIdx.x & 31;
@@ -97,13 +99,16 @@ __global__ void __launch_bounds__(256) pq_quantize_c16(const float4* __restrict_
       out.y = quant4(b, inv, qmax);
       out.z = quant4(c, inv, qmax);
       out.w = quant4(d, inv, qmax);
-      __stcs(q + (n * C16 + j) * HW + hw, out);
+      if (PACK2)
+        __stcs(static_cast<uint32_t*>(q) + (n * C16 + j) * HW + hw, pack2_word(out));
+      else
+        __stcs(static_cast<uint4*>(q) + (n * C16 + j) * HW + hw, out);
     }
   }
 }
 
 int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G, int Cg, int bits, const float* inv_s,
-                        cudaStream_t stream) {
+                        bool packed2, cudaStream_t stream) {
   QuantArgs args;
   for (int g = 0; g < G; ++g) args.inv_s[g] = inv_s[g];
   const int C16 = G * Cg / 16;
@@ -115,8 +120,12 @@ int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G
   const int64_t want = (warps + 7) / 8;  // 8 warps per block
   const int64_t cap = static_cast<int64_t>(sms) * 4;
   const unsigned grid = static_cast<unsigned>(want < cap ? want : cap);
-  pq_quantize_c16<<<grid, 256, 0, stream>>>(reinterpret_cast<const float4*>(x), reinterpret_cast<uint4*>(q), N, HW, C16,
-                                            Cg / 16, (1 << bits) - 1, args);
+  if (packed2)
+    pq_quantize_c16<true><<<grid, 256, 0, stream>>>(reinterpret_cast<const float4*>(x), q, N, HW, C16, Cg / 16,
+                                                    (1 << bits) - 1, args);
+  else
+    pq_quantize_c16<false><<<grid, 256, 0, stream>>>(reinterpret_cast<const float4*>(x), q, N, HW, C16, Cg / 16,
+                                                     (1 << bits) - 1, args);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }
 

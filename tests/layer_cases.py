@@ -83,6 +83,34 @@ def c16_to_nhwc(a: np.ndarray, N: int, H: int, W: int, C: int) -> np.ndarray:
     return np.ascontiguousarray(a.reshape(N, C // 16, H, W, 16).transpose(0, 2, 3, 1, 4).reshape(N, H, W, C))
 
 
+def c16p2_to_nhwc(a: np.ndarray, N: int, H: int, W: int, C: int) -> np.ndarray:
+    """Packed channel-blocked 2-bit codes (little-endian 32-bit word per position and
+    16-channel block, code of channel c at bits 2 (c % 16)) -> NHWC, one code per byte."""
+    words = np.ascontiguousarray(a).view(np.uint32).reshape(N, C // 16, H, W)
+    codes = (words[..., None] >> (2 * np.arange(16, dtype=np.uint32))) & 3
+    return np.ascontiguousarray(codes.astype(np.uint8).transpose(0, 2, 3, 1, 4).reshape(N, H, W, C))
+
+
+def to_format(codes_nhwc: np.ndarray, fmt: int) -> np.ndarray:
+    """NHWC codes -> the given code format's bytes (0 NHWC, 2 channel-blocked, 3 packed)."""
+    N, H, W, C = codes_nhwc.shape
+    blk = codes_nhwc.reshape(N, H, W, C // 16, 16).transpose(0, 3, 1, 2, 4)
+    if fmt == 2:
+        return np.ascontiguousarray(blk).reshape(-1)
+    if fmt == 3:
+        w = (blk.astype(np.uint32) << (2 * np.arange(16, dtype=np.uint32))).sum(axis=-1).astype(np.uint32)
+        return np.ascontiguousarray(w).view(np.uint8).reshape(-1)
+    return np.ascontiguousarray(codes_nhwc).reshape(-1)
+
+
+def from_format(raw: np.ndarray, fmt: int, N: int, H: int, W: int, C: int) -> np.ndarray:
+    if fmt == 2:
+        return c16_to_nhwc(raw, N, H, W, C)
+    if fmt == 3:
+        return c16p2_to_nhwc(raw, N, H, W, C)
+    return np.ascontiguousarray(raw).reshape(N, H, W, C)
+
+
 def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q"), fmt: int = 0):
     """Quantise and run the fused layer on the GPU through the C ABI.  fmt is the
     code format of the activation and output codes (0 NHWC, 2 channel-blocked);
@@ -93,7 +121,8 @@ def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q"), fmt: int = 0):
 
     dev = torch.device("cuda:0")
     x = torch.from_numpy(ref["x"]).to(dev)
-    q = torch.empty(x.shape, dtype=torch.uint8, device=dev)
+    nq = x.numel() // (4 if fmt == B.PQ_CODES_C16P2 else 1)
+    q = torch.empty(nq, dtype=torch.uint8, device=dev)
     B.palquant_quantize_act(x, q, c.N, c.H, c.W, c.G, c.Cin, c.bits, ref["inv_s"], code_format=fmt)
     d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad, c.bits, c.bits, c.bo, int(c.relu),
                      code_format=fmt)
@@ -103,23 +132,20 @@ def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q"), fmt: int = 0):
     shape = (c.N, c.Ho, c.Wo, c.G * c.Cout)
     acc = torch.full(shape, -7, dtype=torch.int32, device=dev) if "acc" in outputs else None
     y = torch.full(shape, float("nan"), dtype=torch.float32, device=dev) if "y" in outputs else None
-    qo = torch.full(shape, 255, dtype=torch.uint8, device=dev) if "q" in outputs else None
+    nqo = int(np.prod(shape)) // (4 if fmt == B.PQ_CODES_C16P2 else 1)
+    qo = torch.full((nqo,), 255, dtype=torch.uint8, device=dev) if "q" in outputs else None
     sc = None if ref["shortcut"] is None else torch.from_numpy(ref["shortcut"]).to(dev)
     B.palquant_layer_fused(q, wp, d, ref["m_out"], ref["m_req"], B.shuffle(c.kind, c.shift, c.perm), sc, acc, y, qo)
     st = B.palquant_sync_check()
     assert st == B.PQ_OK, B.strerror(st)
-    qh = q.cpu().numpy()
-    if fmt == B.PQ_CODES_C16:
-        qh = c16_to_nhwc(qh, c.N, c.H, c.W, c.G * c.Cin)
+    qh = from_format(q.cpu().numpy(), fmt, c.N, c.H, c.W, c.G * c.Cin)
     out = dict(q=qh)
     if acc is not None:
         out["acc"] = acc.cpu().numpy().reshape(-1, c.G * c.Cout)
     if y is not None:
         out["y"] = y.cpu().numpy().reshape(-1, c.G * c.Cout)
     if qo is not None:
-        qoh = qo.cpu().numpy()
-        if fmt == B.PQ_CODES_C16:
-            qoh = c16_to_nhwc(qoh, c.N, c.Ho, c.Wo, c.G * c.Cout)
+        qoh = from_format(qo.cpu().numpy(), fmt, c.N, c.Ho, c.Wo, c.G * c.Cout)
         out["q_out"] = qoh.reshape(-1, c.G * c.Cout)
     return out
 

@@ -191,3 +191,35 @@ def test_bitsplit_unsupported_shapes():
     with pytest.raises(B.PalquantError) as e:
         B.palquant_bitsplit_desc(B.layer_desc(1, 8, 8, 1, 32, 16, 3, 1, 1, 4, 4, 2), 5)
     assert e.value.status == B.PQ_EINVAL
+
+
+def test_packed_codes_layout_rules():
+    """Packed 2-bit codes: 2-bit codes only, stride 1, rows of whole 16-byte multiples."""
+    P2 = B.PQ_CODES_C16P2
+    ok = B.palquant_conv_plan(B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=P2))
+    assert ok.supported == 1
+    for d in [B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 4, 4, 4, code_format=P2),   # 4-bit codes
+              B.layer_desc(1, 8, 8, 2, 32, 32, 3, 2, 1, 2, 2, 2, code_format=P2),   # stride 2
+              B.layer_desc(1, 8, 10, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=P2),  # W % 4 != 0
+              B.layer_desc(1, 3, 3, 2, 32, 32, 1, 1, 0, 2, 2, 2, code_format=P2)]:  # 1x1, H W % 4 != 0
+        assert B.palquant_conv_plan(d).supported == 0
+    # a per-channel scatter cannot write packed codes
+    d = B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=P2)
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_layer_fused(16, 16, d, [1.0] * 2, [1.0] * 2, shuf=B.shuffle(2, 0), q_out_dev=16)
+    assert e.value.status == B.PQ_EUNSUPPORTED
+
+
+def test_packed_code_helpers_roundtrip():
+    from layer_cases import c16p2_to_nhwc, from_format, to_format
+
+    gen = synth.generator(77)
+    q = synth.random_codes((2, 3, 4, 32), 2, gen)
+    raw = to_format(q, 3)
+    assert raw.size == q.size // 4
+    assert np.array_equal(c16p2_to_nhwc(raw, 2, 3, 4, 32), q)
+    assert np.array_equal(from_format(to_format(q, 2), 2, 2, 3, 4, 32), q)
+    # code of channel c at bits 2 (c % 16) of its block's little-endian word
+    one = np.zeros((1, 1, 1, 16), np.uint8)
+    one[0, 0, 0, 5] = 3
+    assert int(to_format(one, 3).view(np.uint32)[0]) == 3 << 10

@@ -264,3 +264,60 @@ def test_requant_ties_round_half_even(B, mult):
     assert np.array_equal(got["q_out"], q_ref)
     if mult == 0.5:
         assert np.any((acc % 2 == 1) & (acc > 0)), "the case must contain ties"
+
+
+# ------------------------------------ packed 2-bit channel-blocked codes (format 3)
+P2_CASES = [
+    Case(1, 28, 28, 2, 32, 32, 3, 1, 1, seed=50),
+    Case(2, 12, 16, 3, 32, 48, 3, 1, 1, seed=51),                     # 3 output chunks
+    Case(2, 8, 8, 4, 96, 96, 1, 1, 0, seed=52),                       # flat, one partial tile
+    Case(2, 14, 14, 4, 96, 96, 1, 1, 0, seed=53),                     # flat, ragged second tile
+    Case(1, 12, 12, 2, 128, 256, 3, 1, 1, seed=54),                   # streamed weights
+    Case(1, 8, 8, 2, 512, 32, 3, 1, 1, seed=55),                      # four K blocks
+    Case(2, 8, 8, 2, 32, 320, 3, 1, 1, seed=56),                      # two output-channel blocks
+    Case(1, 5, 132, 1, 32, 16, 3, 1, 1, seed=57),                     # rows wider than 128 positions
+    Case(2, 12, 8, 2, 64, 64, 3, 1, 1, shortcut=True, seed=58),       # shortcut add
+    Case(1, 9, 12, 2, 32, 64, 5, 1, 2, seed=59),                      # 5x5, pad 2 (staging offset 2)
+    Case(1, 16, 16, 1, 32, 16, 3, 1, 0, kind=0, seed=60),             # pad 0 (offset 0)
+    Case(2, 8, 12, 8, 32, 32, 3, 1, 1, kind=3, perm=(3, 0, 7, 1, 6, 2, 5, 4), seed=61),
+    Case(2, 6, 8, 2, 32, 32, 3, 1, 1, relu=False, kind=1, shift=-1, seed=62),
+]
+
+
+@pytest.mark.parametrize("c", P2_CASES, ids=str)
+def test_layer_fused_packed_codes_matches_oracle(B, c):
+    ref = prepare(c)
+    got = run_gpu(c, ref, fmt=B.PQ_CODES_C16P2)
+    assert_layer_parity(c, ref, got)
+
+
+@pytest.mark.parametrize("c", P2_CASES[:6], ids=str)
+def test_layer_codes_only_packed_matches_oracle(B, c):
+    ref = prepare(c)
+    got = run_gpu(c, ref, outputs=("q",), fmt=B.PQ_CODES_C16P2)
+    assert_layer_parity(c, ref, got)
+
+
+@pytest.mark.parametrize("name,cfg", [(n, c) for n, c in FULL if c.bits_a <= 2], ids=lambda v: v if isinstance(v, str) else "")
+def test_full_size_codes_only_packed_sampled(B, name, cfg):
+    c = Case(cfg.N, cfg.H, cfg.W, cfg.G, cfg.Cin_g, cfg.Cout_g, cfg.k, cfg.stride, cfg.pad, bits=cfg.bits_a,
+             kind=cfg.shuffle_kind, shift=cfg.shuffle_shift, relu=cfg.relu, seed=0)
+    pix = _sample_pixels(c.N, c.Ho, c.Wo, 3000, 3)
+    ref = prepare(c, sample_pix=pix)
+    got = run_gpu(c, ref, outputs=("q",), fmt=B.PQ_CODES_C16P2)
+    assert_layer_parity(c, ref, got, pix)
+
+
+@pytest.mark.parametrize("shape,G,bits", [((2, 7, 9, 64), 4, 2), ((1, 5, 6, 48), 3, 1), ((2, 11, 13, 768), 4, 2)])
+def test_quantize_act_packed_matches_oracle(B, shape, G, bits):
+    from layer_cases import c16p2_to_nhwc
+
+    gen = synth.generator(sum(shape) + 9)
+    x = synth.normal(shape, gen, 2.0)
+    x.reshape(-1)[:6] = np.array([0.5, 1.5, 2.5, np.nan, np.inf, -np.inf], dtype=np.float32)
+    inv = (synth.half_normal((G,), gen) + 0.5).astype(np.float32)
+    q = torch.full((int(np.prod(shape)) // 4,), 254, dtype=torch.uint8, device="cuda")
+    B.palquant_quantize_act(torch.from_numpy(x).cuda(), q, shape[0], shape[1], shape[2], G, shape[3] // G, bits, inv,
+                            code_format=B.PQ_CODES_C16P2)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(c16p2_to_nhwc(q.cpu().numpy(), *shape), oracle.quantize_act(x, G, bits, inv))
