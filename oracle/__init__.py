@@ -67,6 +67,7 @@ def _declare(lib):
     lib.oracle_inv_step.argtypes = [ctypes.c_float]
     lib.oracle_epilogue_scales.restype = _I32
     lib.oracle_epilogue_scales.argtypes = [_I32, _P, _P, ctypes.c_double, _P, _I32, _I32, _P, _P, _P]
+    lib.oracle_quantize_weights_odd.argtypes = [_P, _P, _I32, _I64, _I32, _P]
     lib.oracle_conv2d_f32.argtypes = [_P, _P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _I32, _I32, _I32]
     lib.oracle_maxpool_f32.argtypes = [_P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _I32]
     lib.oracle_avgpool_f32.argtypes = [_P, _P, _I64, _I64, _I64, _I32]
@@ -364,3 +365,16 @@ def bitsplit_conv(q: np.ndarray, wq: np.ndarray, stride: int, pad: int, bits_m: 
             part = group_conv(xi, wj, stride, pad, L=L) << ((i + j) * bits_b)
             acc = part if acc is None else acc + part
     return acc
+
+
+def quantize_weights_odd(w: np.ndarray, bits: int, u, L=None) -> np.ndarray:
+    """The paper's weight quantiser (Eq. 2, Eq. 3's weight form): odd integer codes
+    2 x_q - (2^b - 1), x_q = clamp(rint((w + u[g]) * fl((2^b-1) / (2 u[g]))), 0, 2^b - 1)."""
+    L = L or lib()
+    w = _f32(w)
+    u = _f32(u)
+    G = w.shape[0]
+    assert u.shape == (G,)
+    wq = np.empty(w.shape, dtype=np.int8)
+    L.oracle_quantize_weights_odd(_ptr(w), _ptr(wq), G, w.size // G, bits, _ptr(u))
+    return wq

@@ -30,6 +30,8 @@
  *   oracle_quantize_act      pinned (hand rounding cases, code range, closed
  *                            forms)
  *   oracle_quantize_weights  pinned (hand cases, code range)
+ *   oracle_quantize_weights_odd  pinned (hand cases, odd levels, monotone,
+ *                            the clip bounds)
  *   oracle_group_conv        pinned (float64 library convolution on codes,
  *                            brute-force dequantised conv, 1x1 = matmul,
  *                            all-max closed form, G = 1 case)
@@ -121,6 +123,27 @@ void oracle_quantize_weights(const float* w, int8_t* wq, int G, int Cout_g, int 
             r = fmaxf(r, (float)qmin);
             r = fminf(r, (float)qmax);
             wq[g * per_group + i] = (int8_t)(int)r;
+        }
+    }
+}
+
+/* The paper's own weight quantiser (Sec. 3.2, Eq. 2 with the de-quantised form
+ * 2 (x_q / (2^b - 1) - 0.5) of Eq. 3 for weights): with the clip range
+ * [l, u] = [-u, u], x_n = clip((w + u) / (2 u), 0, 1), x_q = round((2^b - 1) x_n),
+ * and the weight enters the convolution as the odd integer 2 x_q - (2^b - 1)
+ * (levels -3, -1, 1, 3 at b = 2; the de-quantised weight is that integer times
+ * u / (2^b - 1)).  In fp32: one add, one multiply by k[g] = fl((2^b - 1) / (2 u[g]))
+ * (computed in double), round half to even, clamp. */
+void oracle_quantize_weights_odd(const float* w, int8_t* wq, int G, int64_t per_group, int bits, const float* u) {
+    const int qp = (1 << bits) - 1;
+    for (int g = 0; g < G; ++g) {
+        const float k = (float)((double)qp / (2.0 * (double)u[g]));
+        for (int64_t i = 0; i < per_group; ++i) {
+            float t = (w[g * per_group + i] + u[g]) * k;
+            float r = rintf(t);
+            r = fmaxf(r, 0.0f);
+            r = fminf(r, (float)qp);
+            wq[g * per_group + i] = (int8_t)(2 * (int)r - qp);
         }
     }
 }

@@ -41,6 +41,11 @@ MUTATIONS = {
     # channel shuffle as the identity instead of ShuffleNet's transpose
     "channel_shuffle_identity": ("if (kind == 2) return (int64_t)co * G + g;",
                                  "if (kind == 2) return (int64_t)g * Cout_g + co;"),
+    # odd weight levels without the factor 2
+    "odd_levels_unscaled": ("wq[g * per_group + i] = (int8_t)(2 * (int)r - qp);",
+                            "wq[g * per_group + i] = (int8_t)((int)r - qp);"),
+    # the clip range shifted by u twice
+    "odd_levels_shift": ("float t = (w[g * per_group + i] + u[g]) * k;", "float t = (w[g * per_group + i] + 2.0f * u[g]) * k;"),
     # step from the mean without the factor 2
     "act_step_factor": ("s_out[g] = (float)(2.0 * mean / sqrt(qp));\n    }\n}\n\nvoid oracle_weight_step",
                         "s_out[g] = (float)(mean / sqrt(qp));\n    }\n}\n\nvoid oracle_weight_step"),
@@ -74,6 +79,10 @@ def _pins_pass(L) -> bool:
         a, y, qq = oracle.epilogue(np.array([[4, -8]], dtype=np.int64), 1, [0.25], [2.0], kind=0,
                                    shortcut=np.array([[0.5, 1.0]], dtype=np.float32), relu=True, L=L)
         if list(y[0]) != [1.5, 0.0] or list(qq[0]) != [3, 0]:
+            return False
+        # the paper's odd weight levels
+        wo = np.array([-2.0, -0.5, 0.0, 0.5, 1.0], np.float32).reshape(1, 1, 1, 1, -1)
+        if list(oracle.quantize_weights_odd(wo, 2, [1.0], L=L).ravel()) != [-3, -1, 1, 1, 3]:
             return False
         # channel shuffle: ShuffleNet's reshape / transpose
         acc = np.arange(12, dtype=np.int64).reshape(1, 12)

@@ -345,3 +345,27 @@ def test_epilogue_channel_shuffle_is_shufflenet_transpose(G, Co):
     for ref, got in ((a0, a2), (y0, y2)):
         t = torch.from_numpy(ref).reshape(2, 3, G, Co).transpose(2, 3).reshape(ref.shape).numpy()
         assert np.array_equal(t, got)
+
+
+# ------------------------------------------------ the paper's odd weight levels
+def test_odd_weight_levels_hand_cases():
+    # b = 2, u = 1: k = 3 / 2; t = (w + 1) * 1.5
+    w = np.array([-2.0, -1.0, -0.5, -1.0 / 3.0, 0.0, 0.2, 1.0 / 3.0, 0.5, 1.0, 5.0], dtype=np.float32)
+    got = oracle.quantize_weights_odd(w.reshape(1, 1, 1, 1, -1), 2, [1.0]).ravel()
+    # t: -1.5 0 0.75 1.0 1.5 1.8 2.0 2.25 3 9 -> x_q 0 0 1 1 2 2 2 2 3 3 -> 2 x_q - 3
+    assert list(got) == [-3, -3, -1, -1, 1, 1, 1, 1, 3, 3]
+
+
+@pytest.mark.parametrize("bits", [2, 3, 4])
+def test_odd_weight_levels_range_and_monotone(bits):
+    gen = synth.generator(bits + 100)
+    w = synth.normal((2, 4, 3, 3, 16), gen, 0.3)
+    u = np.array([0.4, 0.7], np.float32)
+    wq = oracle.quantize_weights_odd(w, bits, u)
+    qp = (1 << bits) - 1
+    assert np.all(np.abs(wq) <= qp) and np.all(wq % 2 != 0)  # odd levels in [-Qp, Qp]
+    for g in range(2):
+        order = np.argsort(w[g].ravel(), kind="stable")
+        assert np.all(np.diff(wq[g].ravel()[order].astype(int)) >= 0)
+        # outside the clip range the extreme levels
+        assert np.all(wq[g][w[g] >= u[g]] == qp) and np.all(wq[g][w[g] <= -u[g]] == -qp)
