@@ -176,6 +176,19 @@ size_t palquant_packed_weight_bytes(const pq_layer_desc* d);
 pq_status palquant_pack_weights_host(const float* w_host, const pq_layer_desc* d, const float* inv_sw_host,
                                      void* packed_host, size_t packed_bytes);
 
+/* The paper's own weight quantiser (Sec. 3.2: Eq. 2 with the clip range
+ * [-u[g], u[g]] and Eq. 3's de-quantised weight 2 (x_q / (2^b - 1) - 0.5)):
+ *   x_q = clamp(rint((w + u[g]) * k[g]), 0, 2^b - 1), k[g] = fl((2^b - 1) / (2 u[g])),
+ *   code = 2 x_q - (2^b - 1)
+ * (one fp32 add and one fp32 multiply), i.e. the odd levels -3, -1, 1, 3 at
+ * b = 2 instead of the LSQ range [-2^(b-1), 2^(b-1) - 1]; the de-quantised
+ * weight is code * u[g] / (2^b - 1), so its epilogue scale uses
+ * s_w = u / (2^b - 1).  Packed like palquant_pack_weights_host (same size).
+ * u_host: G positive floats.  PQ_EUNSUPPORTED when the larger codes could
+ * make a sum reach 2^24.  Host only. */
+pq_status palquant_pack_weights_odd_host(const float* w_host, const pq_layer_desc* d, const float* u_host,
+                                        void* packed_host, size_t packed_bytes);
+
 /* The same, with the packed operand copied to device memory on `stream`
  * (synchronises the stream before returning so w_host may be freed). */
 pq_status palquant_pack_weights(const float* w_host, const pq_layer_desc* d, const float* inv_sw_host,

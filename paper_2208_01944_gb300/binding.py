@@ -31,6 +31,7 @@ EXPORTS = [
     "palquant_conv2d_f32", "palquant_maxpool2d_f32", "palquant_avgpool_f32", "palquant_linear_f32",
     "palquant_cyclic_shuffle_module", "palquant_bitsplit_desc", "palquant_bitsplit_scratch_bytes",
     "palquant_bitsplit_pack_weight_codes_host", "palquant_bitsplit_act", "palquant_bitsplit_conv",
+    "palquant_pack_weights_odd_host",
 ]
 
 
@@ -106,6 +107,8 @@ def _load():
     L.palquant_watchdog_selftest.argtypes = [ctypes.c_uint64, _P]
     L.palquant_conv_plan.restype = _I32
     L.palquant_conv_plan.argtypes = [ctypes.POINTER(LayerDesc), ctypes.POINTER(ConvPlan)]
+    L.palquant_pack_weights_odd_host.restype = _I32
+    L.palquant_pack_weights_odd_host.argtypes = [_P, ctypes.POINTER(LayerDesc), _P, _P, ctypes.c_size_t]
     L.palquant_bitsplit_desc.restype = _I32
     L.palquant_bitsplit_desc.argtypes = [ctypes.POINTER(LayerDesc), _I32, ctypes.POINTER(LayerDesc)]
     L.palquant_bitsplit_scratch_bytes.restype = ctypes.c_size_t
@@ -358,3 +361,15 @@ def palquant_bitsplit_act(q_dev, xs_dev, xs_bytes, d: LayerDesc, bits_b: int, st
 def palquant_bitsplit_conv(q_dev, xs_dev, xs_bytes, w_packed_dev, acc_dev, d: LayerDesc, bits_b: int, stream=None):
     _check(lib.palquant_bitsplit_conv(_ptr(q_dev), _ptr(xs_dev), xs_bytes, _ptr(w_packed_dev), _ptr(acc_dev),
                                       ctypes.byref(d), bits_b, _stream(stream)), "palquant_bitsplit_conv")
+
+
+def palquant_pack_weights_odd_host(w_host, d: LayerDesc, u) -> np.ndarray:
+    """The paper's odd-level weight quantiser (clip range [-u, u]) and packing."""
+    n = palquant_packed_weight_bytes(d)
+    if n == 0:
+        raise PalquantError(PQ_EUNSUPPORTED, "palquant_packed_weight_bytes")
+    out = np.empty(n, dtype=np.uint8)
+    w, uu = _f32(w_host), _f32(u)
+    _check(lib.palquant_pack_weights_odd_host(_ptr(w), ctypes.byref(d), _ptr(uu), _ptr(out), n),
+           "palquant_pack_weights_odd_host")
+    return out

@@ -700,6 +700,38 @@ pq_status palquant_pack_weights_host(const float* w_host, const pq_layer_desc* d
   return palquant_pack_weight_codes_host(wq.data(), d, packed_host, packed_bytes);
 }
 
+pq_status palquant_pack_weights_odd_host(const float* w_host, const pq_layer_desc* d, const float* u_host,
+                                        void* packed_host, size_t packed_bytes) {
+  if (w_host == nullptr || u_host == nullptr || packed_host == nullptr) return PQ_EINVAL;
+  ConvParams p;
+  pq_status st = plan_conv(d, &p, nullptr, nullptr);
+  if (st != PQ_OK) return st;
+  const size_t per_group = static_cast<size_t>(d->Cout_g) * d->kh * d->kw * d->Cin_g;
+  const size_t need = per_group * d->G;
+  if (packed_bytes < need) return PQ_EINVAL;
+  const int qp = (1 << d->bits_w) - 1;
+  // the odd levels reach 2^b - 1 in magnitude: keep every sum exact in fp32
+  const int64_t taps = static_cast<int64_t>(d->kh) * d->kw;
+  if (qp > 15 || taps * d->Cin_g * ((1LL << d->bits_a) - 1) * qp >= (1LL << 24)) return PQ_EUNSUPPORTED;
+  std::vector<int8_t> wq(need);
+  for (int g = 0; g < d->G; ++g) {
+    if (!(u_host[g] > 0.0f) || !std::isfinite(u_host[g])) return PQ_EINVAL;
+    const float k = static_cast<float>(static_cast<double>(qp) / (2.0 * static_cast<double>(u_host[g])));
+    for (size_t i = 0; i < per_group; ++i) {
+      // one fp32 add and one fp32 multiply (volatile: never fused or widened)
+      volatile float a = w_host[g * per_group + i] + u_host[g];
+      volatile float t = a * k;
+      float r = std::nearbyint(static_cast<float>(t));
+      r = std::fmax(r, 0.0f);
+      r = std::fmin(r, static_cast<float>(qp));
+      wq[g * per_group + i] = static_cast<int8_t>(2 * static_cast<int>(r) - qp);
+    }
+  }
+  uint8_t* out = static_cast<uint8_t*>(packed_host);
+  for_each_packed(p, d->kw, [&](size_t dst, size_t src) { out[dst] = e4m3_of_int(wq[src]); });
+  return PQ_OK;
+}
+
 pq_status palquant_pack_weights(const float* w_host, const pq_layer_desc* d, const float* inv_sw_host,
                                 void* packed_dev, size_t packed_bytes, pq_stream_t stream) {
   if (packed_dev == nullptr) return PQ_EINVAL;

@@ -223,3 +223,14 @@ def test_packed_code_helpers_roundtrip():
     one = np.zeros((1, 1, 1, 16), np.uint8)
     one[0, 0, 0, 5] = 3
     assert int(to_format(one, 3).view(np.uint32)[0]) == 3 << 10
+
+
+@pytest.mark.parametrize("bits", [2, 3])
+def test_odd_level_weights_match_oracle(bits):
+    gen = synth.generator(bits + 60)
+    G, Co, k, Ci = 2, 32, 3, 64
+    w = synth.he_weights(G, Co, k, k, Ci, gen)
+    u = (2.0 * np.abs(w).reshape(G, -1).mean(axis=1)).astype(np.float32)
+    d = B.layer_desc(1, 6, 6, G, Ci, Co, k, 1, 1, 2, bits, 2)
+    packed = B.palquant_pack_weights_odd_host(w, d, u)
+    assert np.array_equal(B.palquant_unpack_weight_codes_host(packed, d), oracle.quantize_weights_odd(w, bits, u))

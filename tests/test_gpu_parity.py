@@ -321,3 +321,36 @@ def test_quantize_act_packed_matches_oracle(B, shape, G, bits):
                             code_format=B.PQ_CODES_C16P2)
     assert B.palquant_sync_check() == B.PQ_OK
     assert np.array_equal(c16p2_to_nhwc(q.cpu().numpy(), *shape), oracle.quantize_act(x, G, bits, inv))
+
+
+# ---------------------------------------- the paper's odd weight levels (Eq. 2-3)
+@pytest.mark.parametrize("fmt", FORMATS, ids=["nhwc", "c16"])
+@pytest.mark.parametrize("bits_w", [2, 3])
+def test_layer_with_odd_weight_levels_matches_oracle(B, fmt, bits_w):
+    from layer_cases import from_format
+
+    N, H, W, G, Ci, Co = 2, 12, 10, 2, 64, 48
+    gen = synth.generator(70 + bits_w)
+    x = synth.half_normal((N, H, W, G * Ci), gen)
+    w = synth.he_weights(G, Co, 3, 3, Ci, gen)
+    s_a = oracle.act_step(x, G, 2)
+    inv_s = oracle.inv_step(s_a)
+    u = (2.0 * np.abs(w).reshape(G, -1).mean(axis=1)).astype(np.float32)
+    s_w = (u.astype(np.float64) / ((1 << bits_w) - 1)).astype(np.float32)  # de-quantised weight = code * s_w
+    q = oracle.quantize_act(x, G, 2, inv_s)
+    wq = oracle.quantize_weights_odd(w, bits_w, u)
+    m_out, m_req = oracle.epilogue_scales(s_w, s_a, s_a, 1.0, 1, 1)
+    acc = oracle.group_conv(q, wq, 1, 1).reshape(-1, G * Co)
+    a_ref, y_ref, q_ref = oracle.epilogue(acc, G, m_out, m_req, 1, 1, None, None, True, 2)
+    d = B.layer_desc(N, H, W, G, Ci, Co, 3, 1, 1, 2, bits_w, 2, 1, code_format=fmt)
+    wp = torch.from_numpy(B.palquant_pack_weights_odd_host(w, d, u)).cuda()
+    qd = torch.empty(x.size, dtype=torch.uint8, device="cuda")
+    B.palquant_quantize_act(torch.from_numpy(x).cuda(), qd, N, H, W, G, Ci, 2, inv_s, code_format=fmt)
+    ad = torch.empty((N * H * W, G * Co), dtype=torch.int32, device="cuda")
+    yd = torch.empty((N * H * W, G * Co), dtype=torch.float32, device="cuda")
+    qo = torch.empty(N * H * W * G * Co, dtype=torch.uint8, device="cuda")
+    B.palquant_layer_fused(qd, wp, d, m_out, m_req, B.shuffle(1, 1), None, ad, yd, qo)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(ad.cpu().numpy(), a_ref)
+    assert np.array_equal(yd.cpu().numpy(), y_ref)
+    assert np.array_equal(from_format(qo.cpu().numpy(), fmt, N, H, W, G * Co).reshape(-1, G * Co), q_ref)
