@@ -47,6 +47,8 @@ def parse():
                     help="only run the fused layer of CONFIG (config0, config1, config3_0..4, config4) --reps times "
                          "on random codes (codes out), for profilers; prints nothing else")
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--profile-format", default="c16", choices=["c16", "f4"],
+                    help="code format of --profile-layer: one code per byte, or packed FP4 nibbles")
     ap.add_argument("--no-resnet", action="store_true", help="skip the ResNet-18-shaped network measurement")
     ap.add_argument("--resnet-batch", type=int, default=128)
     ap.add_argument("--resnet-reps", type=int, default=20)
@@ -55,7 +57,7 @@ def parse():
     return ap.parse_args()
 
 
-def run_profile_layer(name: str, reps: int):
+def run_profile_layer(name: str, reps: int, fmt_name: str = "c16"):
     """The fused layer alone, for profiling: random codes and weights of the named workload."""
     import numpy as np
     import torch
@@ -66,12 +68,17 @@ def run_profile_layer(name: str, reps: int):
     c = workloads.BENCH_CONFIGS[name]
     dev = torch.device("cuda:0")
     gen = synth.generator(0)
-    q = torch.from_numpy(synth.random_codes((c.N, c.H, c.W, c.G * c.Cin_g), c.bits_a, gen)).to(dev)
+    f4 = fmt_name == "f4"
+    if f4:  # two random codes per byte, one per nibble
+        lo = synth.random_codes((c.in_elems // 2,), c.bits_a, gen)
+        q = torch.from_numpy(lo | (synth.random_codes((c.in_elems // 2,), c.bits_a, gen) << 4)).to(dev)
+    else:
+        q = torch.from_numpy(synth.random_codes((c.N, c.H, c.W, c.G * c.Cin_g), c.bits_a, gen)).to(dev)
     wq = synth.random_codes((c.G, c.Cout_g, c.k, c.k, c.Cin_g), c.bits_w, gen, signed=True)
     d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out,
-                     code_format=B.PQ_CODES_C16)
+                     code_format=B.PQ_CODES_C32F4 if f4 else B.PQ_CODES_C16)
     wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).to(dev)
-    qo = torch.empty((c.N, c.Ho, c.Wo, c.G * c.Cout_g), dtype=torch.uint8, device=dev)
+    qo = torch.empty(c.out_elems // (2 if f4 else 1), dtype=torch.uint8, device=dev)
     m = np.full(c.G, 0.01, np.float32)
     for _ in range(reps):
         B.palquant_layer_fused(q, wp, d, m, m, B.shuffle(c.shuffle_kind, c.shuffle_shift), None, None, None, qo)
@@ -631,7 +638,7 @@ def main():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.profile_layer:
-        run_profile_layer(args.profile_layer, args.reps)
+        run_profile_layer(args.profile_layer, args.reps, args.profile_format)
         return
     if args.impl == "reference":
         run_reference(args, rank, world)

@@ -67,12 +67,20 @@ typedef enum {
                           byte ((((n*(C/16) + c/16)*H + h)*W + w)*16 + c%16).  C % 16 == 0.
                           The tensor cores' operand layout: every run of positions of one
                           16-channel block is contiguous. */
-    PQ_CODES_C16P2 = 3 /* 2-bit codes packed four to a byte, channel-blocked: the 16 codes of
+    PQ_CODES_C16P2 = 3, /* 2-bit codes packed four to a byte, channel-blocked: the 16 codes of
                           a position and 16-channel block form one little-endian 32-bit word
                           at byte ((((n*(C/16) + c/16)*H + h)*W + w)*4), code of channel c at
                           bits 2 (c % 16).  bits <= 2, C % 16 == 0; as a layer input it needs
                           stride 1 and W % 4 == 0 (H W % 4 == 0 for 1x1 layers).  A quarter
                           of the bytes of PQ_CODES_C16. */
+    PQ_CODES_C32F4 = 4  /* 2-bit codes as packed FP4: two to a byte, channel-blocked in
+                          32-channel blocks of 16 bytes per position; code of channel c in the
+                          4 bits at byte ((((n*(C/32) + c/32)*H + h)*W + w)*16 + (c%32)/2),
+                          low nibble for even c, high nibble for odd c.  A code v <= 3 is the
+                          FP4 E2M1 encoding of v/2, so the layer's block-scaled FP4 tensor-core
+                          path reads it in place.  bits <= 2, C % 32 == 0; as a layer format it
+                          also needs Cin_g % 64 == 0, Cout_g % 32 == 0, bits_w <= 3, and no
+                          channel shuffle.  Half the bytes of PQ_CODES_C16. */
 } pq_code_format;
 
 /* Output channel permutation (Sec. 4.2).  kind:
@@ -102,7 +110,7 @@ typedef struct {
     int32_t bits_w;      /* weight code bits, 2..4 */
     int32_t bits_out;    /* requantised output code bits, 1..4 */
     int32_t relu;        /* 1: ReLU after the rescale (and the shortcut add) */
-    int32_t code_format; /* pq_code_format (INT8 or C16) of the input codes and the output codes */
+    int32_t code_format; /* pq_code_format of the input codes and the output codes */
 } pq_layer_desc;
 
 /* Human-readable name of a status. */
@@ -212,7 +220,8 @@ pq_status palquant_unpack_weight_codes_host(const void* packed_host, const pq_la
  * x_dev is NHWC fp32 [N,H,W,G*Cg]; q_dev receives one byte per element in
  * code_format (PQ_CODES_INT8: NHWC; PQ_CODES_C16: channel-blocked, needs
  * Cg % 16 == 0; PQ_CODES_C16P2: channel-blocked 2-bit codes four to a byte,
- * needs Cg % 16 == 0 and bits <= 2).  inv_s_host holds G floats (fl(1/s) of the steps), copied at
+ * needs Cg % 16 == 0 and bits <= 2; PQ_CODES_C32F4: 2-bit codes two to a byte
+ * in 32-channel blocks, needs Cg % 16 == 0, G*Cg % 32 == 0 and bits <= 2).  inv_s_host holds G floats (fl(1/s) of the steps), copied at
  * call time.  NaN maps to 0 and +inf to 2^bits - 1.  bits in 1..8. */
 pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G,
                                 int32_t Cg, int32_t bits, int32_t code_format, const float* inv_s_host,

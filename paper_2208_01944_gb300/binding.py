@@ -18,7 +18,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libpalquant.so")
 
 PQ_OK, PQ_EINVAL, PQ_EUNSUPPORTED, PQ_ECUDA, PQ_ETIMEOUT = 0, -1, -2, -3, -4
-PQ_CODES_INT8, PQ_CODES_E4M3, PQ_CODES_C16, PQ_CODES_C16P2 = 0, 1, 2, 3
+PQ_CODES_INT8, PQ_CODES_E4M3, PQ_CODES_C16, PQ_CODES_C16P2, PQ_CODES_C32F4 = 0, 1, 2, 3, 4
 
 # Every symbol include/palquant.h declares.
 EXPORTS = [

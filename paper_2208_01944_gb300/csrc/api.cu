@@ -88,7 +88,7 @@ pq_status validate_desc(const pq_layer_desc* d) {
     return PQ_EINVAL;
   if (d->relu != 0 && d->relu != 1) return PQ_EINVAL;
   if (d->code_format != PQ_CODES_INT8 && d->code_format != PQ_CODES_E4M3 && d->code_format != PQ_CODES_C16 &&
-      d->code_format != PQ_CODES_C16P2)
+      d->code_format != PQ_CODES_C16P2 && d->code_format != PQ_CODES_C32F4)
     return PQ_EINVAL;
   if (out_dim(d->H, d->kh, d->stride, d->pad) < 1 || out_dim(d->W, d->kw, d->stride, d->pad) < 1) return PQ_EINVAL;
   if (d->G > pq::kMaxG) return PQ_EUNSUPPORTED;
@@ -123,13 +123,19 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const int qw = 1 << (d->bits_w - 1);
   // Coverage of the tensor-core kernel.
   const bool p2 = d->code_format == PQ_CODES_C16P2;
-  const bool c16 = d->code_format == PQ_CODES_C16 || p2;  // channel-blocked (bytes or packed)
+  const bool f4 = d->code_format == PQ_CODES_C32F4;
+  const bool c16 = d->code_format == PQ_CODES_C16 || p2 || f4;  // channel-blocked (bytes or packed)
+  // FP4 nibbles: 16-byte chunks of 32 channels and 64 channels per MMA K step;
+  // E2M1 holds the codes v / 2 for v <= 3 and the weights -4..4.
+  const int cpb = f4 ? 2 : 1;  // channels per byte of the operands
+  const bool f4_ok = !f4 || (d->bits_a <= 2 && d->bits_out <= 2 && d->bits_w <= 3 && d->Cin_g % 64 == 0 &&
+                             d->Cout_g % 32 == 0);
   // Packed 2-bit codes: 2-bit input and output codes, stride 1, and 16-byte aligned
   // rows (1x1: image planes) for the TMA loads of the packed tile.
   const bool flat_shape = d->kh == 1 && d->kw == 1 && d->stride == 1 && d->pad == 0;
   const bool p2_ok = !p2 || (d->bits_a <= 2 && d->bits_out <= 2 && d->stride == 1 &&
                              (flat_shape ? (static_cast<int64_t>(d->H) * d->W) % 4 == 0 : d->W % 4 == 0));
-  bool ok = (d->code_format == PQ_CODES_INT8 || c16) && p2_ok && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
+  bool ok = (d->code_format == PQ_CODES_INT8 || c16) && p2_ok && f4_ok && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
             d->pad < std::max(d->kh, d->kw) && d->Cin_g % 32 == 0 && d->Cout_g % 16 == 0 && taps <= pq::kMaxTaps &&
             static_cast<int64_t>(taps) * d->Cin_g * qa * qw < (1LL << 24);
   if (!ok) {
@@ -145,7 +151,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.Cout_g = d->Cout_g;
   p.taps = taps;
   // Output-channel blocks: N of one MMA is at most 256 and a multiple of 16.
-  int NB = (d->Cout_g + 255) / 256;
+  // FP4 keeps N <= 128 so that two accumulators and the 32 scale-factor columns
+  // fit the 512 TMEM columns.
+  const int n_max = f4 ? 128 : 256;
+  int NB = (d->Cout_g + n_max - 1) / n_max;
   while (d->Cout_g % NB != 0 || (d->Cout_g / NB) % 16 != 0) ++NB;
   p.NB = NB;
   p.Nblk = d->Cout_g / NB;
@@ -190,17 +199,20 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // epilogue's per-item set-up) plus, per 128-row accumulator, the larger of its
   // MMA time and its epilogue time, so few large items beat many small ones
   // even at some cost in padded rows.  Model (per SM): an M=128, K=32 FP8 MMA
-  // takes max(32 + N/4, N/2) cycles (shared-memory operand reads at 128 B per
-  // cycle, tensor rate), the epilogue about 0.07 ns per accumulator value and an
-  // item 500 ns of overhead.  Double-buffered accumulators come first.
+  // (or K=64 FP4 MMA, the same 32 bytes of K) takes max(32 + N/4, N/2) cycles
+  // (shared-memory operand reads at 128 B per cycle, tensor rate), the epilogue
+  // about 0.07 ns per accumulator value and an item 500 ns of overhead.
+  // Double-buffered accumulators come first.
   const double ns_per_clk = 1.0 / 1.9;
   const double mma_ns = std::max(32.0 + p.Npow2 / 4.0, p.Npow2 / 2.0) * ns_per_clk;
-  const double slot_ns = std::max(static_cast<double>(p.taps) * (d->Cin_g / 32) * mma_ns, 128.0 * p.Npow2 * 0.07);
+  const double slot_ns =
+      std::max(static_cast<double>(p.taps) * (d->Cin_g / (32 * cpb)) * mma_ns, 128.0 * p.Npow2 * 0.07);
+  const int tmem_avail = f4 ? 512 - 32 : 512;  // FP4: 32 columns hold the scale factors
   int best_mt = 0, best_ht = 0, best_tpi = 0, best_acc = 0;
   double best_cost = 0.0;
   for (int MT : {1, 2, 4}) {
     if (flat && (MT > 2 || (c16 && MT > 1))) continue;
-    int acc_stages = (2 * MT * p.Npow2 <= 512) ? 2 : ((MT * p.Npow2 <= 512) ? 1 : 0);
+    int acc_stages = (2 * MT * p.Npow2 <= tmem_avail) ? 2 : ((MT * p.Npow2 <= tmem_avail) ? 1 : 0);
     if (acc_stages == 0) continue;
     int ht = 0, tpi = 0;
     if (flat) {
@@ -258,7 +270,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // K blocks, weights residency and pipeline depth under the shared-memory budget.
   const uint32_t budget = pq::kMaxSmem - 1024;
   auto a_stage_bytes = [&](int KC, uint32_t* phase_bytes, uint32_t* lbo) -> uint32_t {
-    const int nch = KC / 16;
+    const int nch = KC / (16 * cpb);
     if (flat) {
       const uint32_t plane = static_cast<uint32_t>(p.flat_box) * 16u;
       *phase_bytes = round_up(static_cast<uint64_t>(nch) * plane, 128);
@@ -281,7 +293,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // TMA loads the activation operand).
   const uint32_t stage_total = warp_stage * (pq::kEpiWarps + pq::kLoadWarps);
   const uint32_t bar_bytes = 1024;  // barriers, abort flag, TMEM slot (generous)
-  const uint64_t unit_bytes = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk;
+  const uint64_t unit_bytes = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk / cpb;
   // Packed codes: a staging stage per operand stage holding the TMA box of 32-bit
   // words (rows start at the tile's first position rounded down to a multiple of
   // 4, the TMA's 16-byte alignment of the innermost coordinate).
@@ -302,17 +314,18 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   bool found = false, resident = false;
   int KC = d->Cin_g, a_stages = 0, b_stages = 0;
   uint32_t stage_bytes = 0, phase_bytes = 0, lbo = 0;
-  // K blocks of 32 * {8, 4, 3, 2, 1} channels: the MMA issue loop is compiled for
-  // these K-step counts.
-  for (int kc : {256, 128, 96, 64, 32}) {
+  // K blocks of {8, 4, 3, 2, 1} MMA K steps (32 channels each, 64 for FP4): the
+  // MMA issue loop is compiled for these K-step counts.
+  for (int kc1 : {256, 128, 96, 64, 32}) {
     if (found) break;
+    const int kc = kc1 * cpb;
     if (d->Cin_g % kc != 0) continue;
     uint32_t sb, pb, l;
     sb = a_stage_bytes(kc, &pb, &l);
     if (sb > 64u * 1024u) continue;
     for (int res = 1; res >= 0 && !found; --res) {
       if (res && unit_bytes > 112u * 1024u) continue;
-      const uint64_t slice = static_cast<uint64_t>(kc) * p.Nblk;
+      const uint64_t slice = static_cast<uint64_t>(kc) * p.Nblk / cpb;
       if (!res && slice > 32u * 1024u) continue;
       for (int na = 4; na >= 2 && !found; --na) {
         for (int nb = (res ? 1 : 4); nb >= (res ? 1 : 2) && !found; --nb) {
@@ -335,9 +348,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
     if (pub) *pub = plan;
     return PQ_EUNSUPPORTED;
   }
-  const uint32_t b_bytes = resident ? round_up(unit_bytes, 1024) : round_up(static_cast<uint64_t>(b_stages) * KC * p.Nblk, 1024);
+  const uint32_t b_bytes =
+      resident ? round_up(unit_bytes, 1024) : round_up(static_cast<uint64_t>(b_stages) * KC * p.Nblk / cpb, 1024);
   p.KC = KC;
-  p.nch = KC / 16;
+  p.nch = KC / (16 * cpb);
   p.nch_magic = static_cast<uint32_t>(((1ull << 32) + p.nch - 1) / p.nch);
   p.H = d->H;
   p.W = d->W;
@@ -346,6 +360,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.img_pix = d->H * d->W;
   p.codes_c16 = c16 ? 1 : 0;
   p.codes_p2 = p2 ? 1 : 0;
+  p.codes_f4 = f4 ? 1 : 0;
+  p.chunk_shift = f4 ? 5 : 4;
   p.a_unpack = p2 ? 1 : 0;
   p.pk_box_w = pk_box_w;
   p.pk_off = pk_off;
@@ -359,11 +375,12 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   {
     const int64_t C = p.C_in_total, H = d->H, W = d->W;
     if (c16) {
+      // 16-byte chunks of 16 channels (32 for FP4 nibbles)
       p.ld_pix = 16;
       p.ld_row = W * 16;
       p.ld_chunk = H * W * 16;
-      p.ld_img = (C / 16) * H * W * 16;
-      p.ld_c0_mul = H * W * 16;  // channel block c0/16 starts c0/16 chunks in
+      p.ld_img = (C / (16 * cpb)) * H * W * 16;
+      p.ld_c0_mul = H * W * 16 / cpb;  // channel block c0/16 (c0/32) starts that many chunks in
     } else {
       p.ld_pix = C;
       p.ld_row = W * C;
@@ -380,11 +397,15 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.a_stage_bytes = stage_bytes;
   p.a_stages = a_stages;
   p.b_resident = resident ? 1 : 0;
-  p.b_slice_bytes = static_cast<uint32_t>(KC) * p.Nblk;
+  p.b_slice_bytes = static_cast<uint32_t>(KC) * p.Nblk / cpb;
   p.b_unit_bytes = static_cast<uint32_t>(unit_bytes);
   p.lbo_b = static_cast<uint32_t>(p.Nblk) * 16u;
   p.b_stages = resident ? 1 : b_stages;
-  p.tmem_cols = static_cast<uint32_t>(next_pow2(std::max(32, p.acc_stages * p.MT * p.Npow2)));
+  {
+    const int acc_cols = std::max(32, p.acc_stages * p.MT * p.Npow2);
+    p.sf_col = static_cast<uint32_t>(round_up(acc_cols, 32));  // FP4 scale factors after the accumulators
+    p.tmem_cols = static_cast<uint32_t>(next_pow2(f4 ? static_cast<int>(p.sf_col) + 32 : acc_cols));
+  }
   p.smem_b_off = static_cast<uint32_t>(a_stages) * stage_bytes;
   p.smem_stage_off = p.smem_b_off + b_bytes;
   p.smem_pk_off = p.smem_stage_off + stage_total;  // packed staging ring (a_stages x pk_stage_bytes)
@@ -452,7 +473,8 @@ bool encode_c16_map(const pq_layer_desc* d, const ConvParams& p, const void* q_d
   EncodeTiledFn enc = encode_fn();
   if (enc == nullptr) return false;
   std::memset(map, 0, sizeof(*map));
-  const uint64_t C16 = static_cast<uint64_t>(d->G) * d->Cin_g / 16, H = d->H, W = d->W;
+  // 16-byte chunks per position: C/16, or C/32 for FP4 nibbles
+  const uint64_t C16 = static_cast<uint64_t>(d->G) * d->Cin_g / (p.codes_f4 ? 32 : 16), H = d->H, W = d->W;
   cuuint32_t es[4] = {1, 1, 1, 1};
   if (p.codes_p2) {
     // Packed codes: one 32-bit word per (position, 16-channel block).
@@ -491,28 +513,65 @@ bool encode_c16_map(const pq_layer_desc* d, const ConvParams& p, const void* q_d
 
 // ---------------------------------------------------------------------------
 // Weight packing (tensor-core operand layout of the planner's tiling).
-//   unit u = g * NB + nb; for each K block kb, tap t, 16-channel chunk j,
-//   output channel c (of the block) and channel e of the chunk:
-//   byte[(((u * n_kb + kb) * taps + t) * nch + j) * Nblk * 16 + c * 16 + e]
-//     = E4M3(w_q[g, nb*Nblk + c, tap t, kb*KC + j*16 + e])
+//   unit u = g * NB + nb; for each K block kb, tap t, 16-byte chunk j,
+//   output channel c (of the block) and channel e of the chunk (E = 16
+//   channels per chunk, 32 for FP4):
+//   element[(((u * n_kb + kb) * taps + t) * nch + j) * Nblk * E + c * E + e]
+//     = w_q[g, nb*Nblk + c, tap t, kb*KC + j*E + e]
+//   as an E4M3 byte, or (FP4) an E2M1 nibble, element 2i in the low nibble of
+//   byte i and element 2i+1 in the high one.
 // ---------------------------------------------------------------------------
 template <typename F>
 void for_each_packed(const ConvParams& p, int kw, F&& f) {
+  const int E = 16 << (p.chunk_shift - 4);
   for (int g = 0; g < p.G; ++g)
     for (int nb = 0; nb < p.NB; ++nb)
       for (int kb = 0; kb < p.n_kb; ++kb)
         for (int t = 0; t < p.taps; ++t)
           for (int j = 0; j < p.nch; ++j)
             for (int c = 0; c < p.Nblk; ++c)
-              for (int e = 0; e < 16; ++e) {
+              for (int e = 0; e < E; ++e) {
                 const int u = g * p.NB + nb;
-                const size_t dst = ((((static_cast<size_t>(u) * p.n_kb + kb) * p.taps + t) * p.nch + j) * p.Nblk + c) * 16 + e;
+                const size_t dst = ((((static_cast<size_t>(u) * p.n_kb + kb) * p.taps + t) * p.nch + j) * p.Nblk + c) * E + e;
                 const int co = nb * p.Nblk + c;
-                const int ci = kb * p.KC + j * 16 + e;
+                const int ci = kb * p.KC + j * E + e;
                 const int i = t / kw, jj = t % kw;
                 const size_t src = (((static_cast<size_t>(g) * p.Cout_g + co) * (p.taps / kw) + i) * kw + jj) * p.Cin_g + ci;
                 f(dst, src);
               }
+}
+
+// E2M1 nibble of an integer weight code in [-4, 4]: the magnitudes 0..4 are the
+// E2M1 values 0, 1.0, 2.0, 3.0, 4.0 (nibbles 0, 2, 4, 5, 6), bit 3 the sign.
+uint8_t e2m1_of_int(int v) {
+  static const uint8_t mag[5] = {0, 2, 4, 5, 6};
+  const int a = v < 0 ? -v : v;
+  return static_cast<uint8_t>(mag[a] | (v < 0 ? 8 : 0));
+}
+
+// Inverse of e2m1_of_int (nibbles it does not produce read as -128).
+int int_of_e2m1(uint8_t b) {
+  static const int val[8] = {0, -128, 1, -128, 2, 3, 4, -128};
+  const int m = val[b & 7];
+  return (b & 8) && m != -128 ? -m : m;
+}
+
+// Bytes of the packed weight operand: one per code, or one per two (FP4).
+size_t packed_weight_bytes_of(const pq_layer_desc* d, const ConvParams& p) {
+  const size_t elems = static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
+  return p.codes_f4 ? elems / 2 : elems;
+}
+
+// Write the signed codes wq [G][Cout_g][kh][kw][Cin_g] in the operand layout.
+void pack_codes(const ConvParams& p, const pq_layer_desc* d, const int8_t* wq, uint8_t* out) {
+  if (p.codes_f4) {
+    std::memset(out, 0, packed_weight_bytes_of(d, p));
+    for_each_packed(p, d->kw, [&](size_t dst, size_t src) {
+      out[dst >> 1] = static_cast<uint8_t>(out[dst >> 1] | (e2m1_of_int(wq[src]) << (4 * (dst & 1))));
+    });
+  } else {
+    for_each_packed(p, d->kw, [&](size_t dst, size_t src) { out[dst] = e4m3_of_int(wq[src]); });
+  }
 }
 
 pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
@@ -549,7 +608,7 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
   }
   p.channel_shuffle = shuf.kind == 2 ? 1 : 0;
   // A per-channel scatter cannot write single 2-bit codes into packed bytes.
-  if (p.channel_shuffle && p.codes_p2 && q_out_dev != nullptr) return PQ_EUNSUPPORTED;
+  if (p.channel_shuffle && (p.codes_p2 || p.codes_f4) && q_out_dev != nullptr) return PQ_EUNSUPPORTED;
   p.w_packed = static_cast<const uint8_t*>(w_packed_dev);
   p.shortcut = shortcut_dev;
   p.acc_out = acc_out_dev;
@@ -650,7 +709,7 @@ pq_status palquant_epilogue_scales(int32_t G, const float* s_w_host, const float
 size_t palquant_packed_weight_bytes(const pq_layer_desc* d) {
   ConvParams p;
   if (plan_conv(d, &p, nullptr, nullptr) != PQ_OK) return 0;
-  return static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
+  return packed_weight_bytes_of(d, p);
 }
 
 pq_status palquant_pack_weight_codes_host(const int8_t* wq_host, const pq_layer_desc* d, void* packed_host,
@@ -659,13 +718,12 @@ pq_status palquant_pack_weight_codes_host(const int8_t* wq_host, const pq_layer_
   ConvParams p;
   pq_status st = plan_conv(d, &p, nullptr, nullptr);
   if (st != PQ_OK) return st;
-  const size_t need = static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
-  if (packed_bytes < need) return PQ_EINVAL;
+  const size_t elems = static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
+  if (packed_bytes < packed_weight_bytes_of(d, p)) return PQ_EINVAL;
   const int lo = -(1 << (d->bits_w - 1)), hi = (1 << (d->bits_w - 1)) - 1;
-  for (size_t i = 0; i < need; ++i)
+  for (size_t i = 0; i < elems; ++i)
     if (wq_host[i] < lo || wq_host[i] > hi) return PQ_EINVAL;
-  uint8_t* out = static_cast<uint8_t*>(packed_host);
-  for_each_packed(p, d->kw, [&](size_t dst, size_t src) { out[dst] = e4m3_of_int(wq_host[src]); });
+  pack_codes(p, d, wq_host, static_cast<uint8_t*>(packed_host));
   return PQ_OK;
 }
 
@@ -675,7 +733,12 @@ pq_status palquant_unpack_weight_codes_host(const void* packed_host, const pq_la
   pq_status st = plan_conv(d, &p, nullptr, nullptr);
   if (st != PQ_OK) return st;
   const uint8_t* in = static_cast<const uint8_t*>(packed_host);
-  for_each_packed(p, d->kw, [&](size_t dst, size_t src) { wq_host[src] = static_cast<int8_t>(int_of_e4m3(in[dst])); });
+  if (p.codes_f4)
+    for_each_packed(p, d->kw, [&](size_t dst, size_t src) {
+      wq_host[src] = static_cast<int8_t>(int_of_e2m1(static_cast<uint8_t>(in[dst >> 1] >> (4 * (dst & 1)))));
+    });
+  else
+    for_each_packed(p, d->kw, [&](size_t dst, size_t src) { wq_host[src] = static_cast<int8_t>(int_of_e4m3(in[dst])); });
   return PQ_OK;
 }
 
@@ -708,11 +771,13 @@ pq_status palquant_pack_weights_odd_host(const float* w_host, const pq_layer_des
   if (st != PQ_OK) return st;
   const size_t per_group = static_cast<size_t>(d->Cout_g) * d->kh * d->kw * d->Cin_g;
   const size_t need = per_group * d->G;
-  if (packed_bytes < need) return PQ_EINVAL;
+  if (packed_bytes < packed_weight_bytes_of(d, p)) return PQ_EINVAL;
   const int qp = (1 << d->bits_w) - 1;
-  // the odd levels reach 2^b - 1 in magnitude: keep every sum exact in fp32
+  // the odd levels reach 2^b - 1 in magnitude: keep every sum exact in fp32 (and,
+  // for FP4 operands, every level an E2M1 value: b <= 2)
   const int64_t taps = static_cast<int64_t>(d->kh) * d->kw;
   if (qp > 15 || taps * d->Cin_g * ((1LL << d->bits_a) - 1) * qp >= (1LL << 24)) return PQ_EUNSUPPORTED;
+  if (p.codes_f4 && qp > 3) return PQ_EUNSUPPORTED;
   std::vector<int8_t> wq(need);
   for (int g = 0; g < d->G; ++g) {
     if (!(u_host[g] > 0.0f) || !std::isfinite(u_host[g])) return PQ_EINVAL;
@@ -727,8 +792,7 @@ pq_status palquant_pack_weights_odd_host(const float* w_host, const pq_layer_des
       wq[g * per_group + i] = static_cast<int8_t>(2 * static_cast<int>(r) - qp);
     }
   }
-  uint8_t* out = static_cast<uint8_t*>(packed_host);
-  for_each_packed(p, d->kw, [&](size_t dst, size_t src) { out[dst] = e4m3_of_int(wq[src]); });
+  pack_codes(p, d, wq.data(), static_cast<uint8_t*>(packed_host));
   return PQ_OK;
 }
 
@@ -756,14 +820,18 @@ pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int3
   if (N < 0 || H < 1 || W < 1 || G < 1 || Cg < 1 || bits < 1 || bits > 8) return PQ_EINVAL;
   if (G > pq::kMaxG) return PQ_EUNSUPPORTED;
   if (code_format == PQ_CODES_E4M3) return PQ_EUNSUPPORTED;
-  if (code_format != PQ_CODES_INT8 && code_format != PQ_CODES_C16 && code_format != PQ_CODES_C16P2) return PQ_EINVAL;
+  if (code_format != PQ_CODES_INT8 && code_format != PQ_CODES_C16 && code_format != PQ_CODES_C16P2 &&
+      code_format != PQ_CODES_C32F4)
+    return PQ_EINVAL;
   const int64_t P = N * H * W;
-  if (code_format == PQ_CODES_C16 || code_format == PQ_CODES_C16P2) {
+  if (code_format != PQ_CODES_INT8) {
     if (Cg % 16 != 0) return PQ_EINVAL;
-    if (code_format == PQ_CODES_C16P2 && bits > 2) return PQ_EINVAL;
+    if ((code_format == PQ_CODES_C16P2 || code_format == PQ_CODES_C32F4) && bits > 2) return PQ_EINVAL;
+    if (code_format == PQ_CODES_C32F4 && (static_cast<int64_t>(G) * Cg) % 32 != 0) return PQ_EINVAL;
     if (!aligned16(x_dev) || !aligned16(q_dev)) return PQ_EINVAL;
+    const int pack = code_format == PQ_CODES_C16P2 ? 1 : (code_format == PQ_CODES_C32F4 ? 2 : 0);
     if (pq::launch_quantize_c16(x_dev, static_cast<uint8_t*>(q_dev), N, static_cast<int64_t>(H) * W, G, Cg, bits,
-                                inv_s_host, code_format == PQ_CODES_C16P2, static_cast<cudaStream_t>(stream)) != 0)
+                                inv_s_host, pack, static_cast<cudaStream_t>(stream)) != 0)
       return PQ_ECUDA;
     return PQ_OK;
   }
@@ -819,6 +887,8 @@ pq_status bitsplit_layer(const pq_layer_desc* d, int bits_b, pq_layer_desc* out,
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
   if (bits_b < 1 || bits_b > 4) return PQ_EINVAL;
+  // the M-bit input codes and the shifted weight slices are one per byte
+  if (d->code_format == PQ_CODES_C16P2 || d->code_format == PQ_CODES_C32F4) return PQ_EUNSUPPORTED;
   const int Ga = ceil_div(d->bits_a, bits_b), Gw = ceil_div(d->bits_w, bits_b);
   // (i+1) B <= 8 keeps the byte-wise slicing exact; the largest shifted weight
   // slice is (2^B - 1) 2^((Ga-1 + Gw-1) B) (E4M3 holds integers m 2^k with

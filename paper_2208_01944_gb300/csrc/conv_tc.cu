@@ -173,7 +173,7 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
         const uint32_t full = bars.a_full(ra.stage);
         mbar_arrive_expect_tx(full, p.a_tx_bytes);
         const uint32_t dst = a_base + ra.stage * p.a_stage_bytes;
-        const int chi = (p.src_group[item.g] * p.Cin_g + kb * p.KC) >> 4;
+        const int chi = (p.src_group[item.g] * p.Cin_g + kb * p.KC) >> p.chunk_shift;
         if (flat)
           tma_load_3d(dst, tmA, 2 * item.rb * p.flat_box, chi, item.n, full);
         else
@@ -390,7 +390,7 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const W
 
 constexpr int kUnrollTaps = 9;
 
-template <int KSTEPS, int MT>
+template <int KSTEPS, int MT, bool F4>
 __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t b_base,
                                          uint32_t tmem_base, const uint32_t* tap_a16, int64_t it0, int64_t it1,
                                          const WaitCtx& ctx) {
@@ -407,7 +407,10 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
   Ring ra{0, 0, static_cast<uint32_t>(p.a_stages)};
   Ring rb{0, 0, static_cast<uint32_t>(p.b_resident ? 1 : p.b_stages)};
   Ring racc{0, 0, static_cast<uint32_t>(p.acc_stages)};
-  const uint32_t idesc = idesc_e4m3_f32(128, p.Nblk);
+  const uint32_t idesc = F4 ? idesc_mxf4_f32(128, p.Nblk) : idesc_e4m3_f32(128, p.Nblk);
+  // FP4: scale factors of A and B (all 2^-4, so a product is v/2 * w * 2^-8 =
+  // v * w * 2^-9, the same raw accumulator as the FP8 path).
+  const uint32_t sfa = tmem_base + p.sf_col, sfb = tmem_base + p.sf_col + 16u;
   const uint64_t a_desc0 = smem_desc(a_base, p.lbo_a, 128u);
   const uint64_t b_desc0 = smem_desc(b_base, p.lbo_b, 128u);
   const uint64_t a_hi = a_desc0 & 0xFFFFFFFF00000000ull, b_hi = b_desc0 & 0xFFFFFFFF00000000ull;
@@ -451,7 +454,16 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
           const uint64_t bdesc = b_hi | (b_lo_tap + static_cast<uint32_t>(ks) * b_ks16);
           const uint32_t a_lo = a_lo_tap + static_cast<uint32_t>(ks) * a_ks16;
           const uint32_t acc = ks == 0 ? acc0 : 1u;
-          if constexpr (MT == 4) {
+          if constexpr (F4) {
+            if constexpr (MT == 4) {
+              tc_mma4_f4_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u),
+                              a_hi | (a_lo + 256u), a_hi | (a_lo + 384u), bdesc, idesc, sfa, sfb, acc);
+            } else if constexpr (MT == 2) {
+              tc_mma2_f4_warp(d0, d0 + npow2, a_hi | a_lo, a_hi | (a_lo + 128u), bdesc, idesc, sfa, sfb, acc);
+            } else {
+              tc_mma_f4_warp(d0, a_hi | a_lo, bdesc, idesc, sfa, sfb, acc);
+            }
+          } else if constexpr (MT == 4) {
             tc_mma4_e4m3_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u),
                               a_hi | (a_lo + 256u), a_hi | (a_lo + 384u), bdesc, idesc, acc);
           } else if constexpr (MT == 2) {
@@ -506,9 +518,13 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
 __device__ __forceinline__ void mma_role_dispatch(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t b_base,
                                                   uint32_t tmem_base, const uint32_t* tap_a16, int64_t it0, int64_t it1,
                                                   const WaitCtx& ctx) {
-  const int ks = p.nch >> 1;
-#define PQ_MMA_CASE(K, M) \
-  if (ks == K && p.MT == M) return mma_role<K, M>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1, ctx);
+  const int ks = p.nch >> 1;  // one MMA takes 32 bytes of K: 32 FP8 or 64 FP4 channels
+  const bool f4 = p.codes_f4 != 0;
+#define PQ_MMA_CASE(K, M)                                                                                   \
+  if (ks == K && p.MT == M) {                                                                               \
+    if (f4) return mma_role<K, M, true>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1, ctx);        \
+    return mma_role<K, M, false>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1, ctx);              \
+  }
   PQ_MMA_CASE(1, 1) PQ_MMA_CASE(1, 2) PQ_MMA_CASE(1, 4)
   PQ_MMA_CASE(2, 1) PQ_MMA_CASE(2, 2) PQ_MMA_CASE(2, 4)
   PQ_MMA_CASE(3, 1) PQ_MMA_CASE(3, 2) PQ_MMA_CASE(3, 4)
@@ -597,13 +613,27 @@ __device__ __forceinline__ uint4 epi_codes16(const uint32_t (&v)[16], float m_re
   return w;
 }
 
-// 16 codes (one per byte of w) to global memory: as they are, or packed four to
-// a byte (channel-blocked 2-bit layout).
-__device__ __forceinline__ void store_codes16(uint8_t* dst, uint4 w, int packed2) {
-  if (packed2)
+// Code packing of the channel-blocked output: 0 one code per byte, 1 four 2-bit
+// codes per byte, 2 two FP4 nibbles per byte.
+__device__ __forceinline__ int codes_pack(const ConvParams& p) { return p.codes_p2 ? 1 : (p.codes_f4 ? 2 : 0); }
+
+// 16 codes (one per byte of w) to global memory: as they are (16 bytes), packed
+// four to a byte (4 bytes) or two to a byte (8 bytes, half of a 32-channel row).
+__device__ __forceinline__ void store_codes16(uint8_t* dst, uint4 w, int pack) {
+  if (pack == 1)
     *reinterpret_cast<uint32_t*>(dst) = pack2_word(w);
+  else if (pack == 2)
+    *reinterpret_cast<uint2*>(dst) = pack4_word(w);
   else
     *reinterpret_cast<uint4*>(dst) = w;
+}
+
+// Byte offset of the 16 codes of output pixel pos (in its image n) and the
+// 16-channel chunk k = channel / 16, channel-blocked.
+__device__ __forceinline__ long long codes_offset(const ConvParams& p, int pack, int n, long long hw_out, int pos, int k) {
+  if (pack == 2)
+    return ((static_cast<long long>(n) * (p.C_out_total >> 5) + (k >> 1)) * hw_out + pos) * 16 + (k & 1) * 8;
+  return ((static_cast<long long>(n) * (p.C_out_total >> 4) + k) * hw_out + pos) * (pack ? 4 : 16);
 }
 
 // Store 16 codes of 16-column chunk `ch` of the row (output pixel pos).
@@ -614,8 +644,8 @@ __device__ __forceinline__ void epi_store_codes(const ConvParams& p, const EpiIt
     // Channel-blocked codes: lanes hold consecutive pixels, so each store of the
     // warp lands next to its neighbours'.
     if (valid) {
-      const long long blk = (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (e.dst_c0 >> 4) + ch) * hw_out + pos;
-      store_codes16(p.q_out + blk * (p.codes_p2 ? 4 : 16), w, p.codes_p2);
+      const int pack = codes_pack(p);
+      store_codes16(p.q_out + codes_offset(p, pack, e.n, hw_out, pos, (e.dst_c0 >> 4) + ch), w, pack);
     }
   } else {
     // NHWC: staged, then 16-byte rows written by the warp.
@@ -745,9 +775,20 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
       // increasing (mt, ch) order; the destination of this lane's row is
       // computed once per accumulator, and 16-channel block ch of that row lies
       // ch * H_out * W_out * 16 bytes further on.
-      const int code_bytes = p.codes_p2 ? 4 : 16;  // bytes per (position, 16-channel chunk)
+      // FP4 nibbles: 32-channel blocks of 16 bytes per position, a chunk writes
+      // one half of its block's row.
+      const int pack = codes_pack(p);
+      const int code_bytes = pack == 1 ? 4 : 16;  // bytes per position of a channel block
       const long long chunk_bytes = static_cast<long long>(p.Ho) * p.Wo * code_bytes;
-      uint8_t* const blk0 = p.q_out + (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (e.dst_c0 >> 4)) * chunk_bytes;
+      const int k0 = e.dst_c0 >> 4;
+      uint8_t* const blk0 =
+          p.q_out + (pack == 2 ? static_cast<long long>(e.n) * (p.C_out_total >> 5) * chunk_bytes
+                               : (static_cast<long long>(e.n) * (p.C_out_total >> 4) + k0) * chunk_bytes);
+      auto coff = [&](int ch) -> long long {
+        if (pack != 2) return ch * chunk_bytes;
+        const int k = k0 + ch;
+        return (k >> 1) * chunk_bytes + (k & 1) * 8;
+      };
       const int m_lane = quarter * 32 + lane;
       const int MT = p.MT;
       auto row_ptr = [&](int mt) -> uint8_t* {
@@ -780,7 +821,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         if (n_mt < MT) tmem_ld16(col(n_mt, n_ch), vb);
         {
           const uint4 w = epi_codes16(va, e.m_req512, qmax_f);
-          if (c_row) store_codes16(c_row + c_ch * chunk_bytes, w, p.codes_p2);
+          if (c_row) store_codes16(c_row + coff(c_ch), w, pack);
         }
         tmem_wait_ld();
         if (n_mt >= MT) break;
@@ -790,7 +831,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         if (m2 < MT) tmem_ld16(col(m2, c2), va);
         {
           const uint4 w = epi_codes16(vb, e.m_req512, qmax_f);
-          if (n_row) store_codes16(n_row + n_ch * chunk_bytes, w, p.codes_p2);
+          if (n_row) store_codes16(n_row + coff(n_ch), w, pack);
         }
         tmem_wait_ld();
         c_row = m2 == n_mt ? n_row : row_ptr(m2);
@@ -855,6 +896,19 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  if (p.codes_f4) {
+    // Block scale factors of the FP4 MMAs: 32 columns of every lane set to 2^-4
+    // (UE8M0 byte 123); warps 2-5 cover the four lane quarters.
+    if (warp >= kFirstLoadWarp && warp < kFirstLoadWarp + 4) {
+      const uint32_t t = tmem_base + (static_cast<uint32_t>((warp & 3) * 32) << 16) + p.sf_col;
+#pragma unroll
+      for (int c = 0; c < 32; c += 8) tmem_st8_fill(t + c, 0x7B7B7B7Bu);
+      tmem_wait_st();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+  }
 
   const int64_t it0 = static_cast<int64_t>(blockIdx.x) * p.items / gridDim.x;
   const int64_t it1 = static_cast<int64_t>(blockIdx.x + 1) * p.items / gridDim.x;

@@ -279,6 +279,67 @@ __device__ __forceinline__ void tc_mma4_e4m3_warp(uint32_t d0, uint32_t d1, uint
       : "memory");
 }
 
+// Instruction descriptor of kind::mxf4 (block-scaled, packed E2M1 A and B, two
+// per byte), UE8M0 scale factors (scale-factor IDs 0), fp32 accumulator, both
+// operands K-major, dense K = 64.
+__host__ __device__ constexpr uint32_t idesc_mxf4_f32(int M, int N) {
+  return (1u << 7) | (1u << 10)                    // A, B: E2M1
+         | (static_cast<uint32_t>(N >> 3) << 17)   // N / 8
+         | (1u << 23)                              // scale factors UE8M0
+         | (static_cast<uint32_t>(M >> 4) << 24);  // M / 16
+}
+
+// Block-scaled FP4 forms of the whole-warp MMAs: `sfa`, `sfb` are the tensor-
+// memory addresses of the A and B scale factors (one per 32 K elements).
+__device__ __forceinline__ void tc_mma_f4_warp(uint32_t d_tmem, uint64_t a_desc, uint64_t b_desc, uint32_t idesc,
+                                               uint32_t sfa, uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p, e;\nelect.sync _|e, 0xffffffff;\nsetp.ne.b32 p, %6, 0;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], %1, %2, %3, [%4], [%5], p;\n}" ::"r"(
+          d_tmem),
+      "l"(a_desc), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_mma2_f4_warp(uint32_t d0, uint32_t d1, uint64_t a0, uint64_t a1, uint64_t b_desc,
+                                                uint32_t idesc, uint32_t sfa, uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p, e;\nelect.sync _|e, 0xffffffff;\nsetp.ne.b32 p, %8, 0;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], %2, %4, %5, [%6], [%7], p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%1], %3, %4, %5, [%6], [%7], p;\n}" ::"r"(d0),
+      "r"(d1), "l"(a0), "l"(a1), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_mma4_f4_warp(uint32_t d0, uint32_t d1, uint32_t d2, uint32_t d3, uint64_t a0,
+                                                uint64_t a1, uint64_t a2, uint64_t a3, uint64_t b_desc, uint32_t idesc,
+                                                uint32_t sfa, uint32_t sfb, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p, e;\nelect.sync _|e, 0xffffffff;\nsetp.ne.b32 p, %12, 0;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], %4, %8, %9, [%10], [%11], p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%1], %5, %8, %9, [%10], [%11], p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%2], %6, %8, %9, [%10], [%11], p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%3], %7, %8, %9, [%10], [%11], p;\n}" ::"r"(d0),
+      "r"(d1), "r"(d2), "r"(d3), "l"(a0), "l"(a1), "l"(a2), "l"(a3), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb),
+      "r"(accumulate)
+      : "memory");
+}
+
+// Eight 32-bit columns of this warp's 32 tensor-memory lanes set to `v`.
+__device__ __forceinline__ void tmem_st8_fill(uint32_t taddr, uint32_t v) {
+  asm volatile("tcgen05.st.sync.aligned.32x32b.x8.b32 [%0], {%1, %1, %1, %1, %1, %1, %1, %1};" ::"r"(taddr), "r"(v)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// Sixteen 4-bit codes (one per byte of w, each <= 15) packed two to a byte, code
+// k in the low nibble of byte k / 2 when k is even and the high nibble when odd.
+__device__ __forceinline__ uint32_t pack4_pair(uint32_t a, uint32_t b) {
+  const uint32_t ta = (a | (a >> 4)) & 0x00FF00FFu, tb = (b | (b >> 4)) & 0x00FF00FFu;
+  return __byte_perm(ta, tb, 0x6420);
+}
+__device__ __forceinline__ uint2 pack4_word(uint4 w) { return make_uint2(pack4_pair(w.x, w.y), pack4_pair(w.z, w.w)); }
+
 __device__ __forceinline__ void tc_commit_warp(uint32_t bar) {
   asm volatile(
       "{\n.reg .pred e;\nelect.sync _|e, 0xffffffff;\n"

@@ -46,6 +46,11 @@ struct ConvParams {
   int img_pix;            // H * W (flat mode tiles stay inside one image)
   int codes_c16;          // 1: input and output codes in the channel-blocked layout [N][C/16][H][W][16]
   int codes_p2;           // 1: channel-blocked 2-bit codes packed four to a byte ([N][C/16][H][W][4 B])
+  // 1: 2-bit codes as packed FP4 (E2M1) nibbles, [N][C/32][H][W][16 B], read by the
+  // block-scaled FP4 MMA; one 16-byte chunk then holds 32 channels.
+  int codes_f4;
+  int chunk_shift;        // log2(channels per 16-byte chunk): 4, or 5 for FP4 codes
+  uint32_t sf_col;        // FP4: first TMEM column of the (uniform) block scale factors
   // Packed activations come by TMA into a staging ring and the copy warps unpack
   // them into the operand stages (a_unpack = 1): staged rows of pk_box_w 32-bit
   // words starting pk_off words left of the tile's first position.
@@ -110,8 +115,10 @@ struct ConvParams {
 int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream);
 int launch_bitsplit_act(const uint8_t* q, uint8_t* xs, int64_t N, int64_t HW, int C, int Ga, int Gw, int B, int c16,
                         cudaStream_t stream);
+// pack: 0 one code per byte [N][C/16][HW][16]; 1 four 2-bit codes per byte
+// [N][C/16][HW][4 B]; 2 two 4-bit codes per byte [N][C/32][HW][16 B].
 int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G, int Cg, int bits, const float* inv_s,
-                        bool packed2, cudaStream_t stream);
+                        int pack, cudaStream_t stream);
 int launch_quantize(const float* x, uint8_t* q, int64_t P, int G, int Cg, int bits, const float* inv_s,
                     cudaStream_t stream);
 int launch_act_sum(const float* x, int64_t P, int G, int Cg, double* partial, int nblocks, cudaStream_t stream);

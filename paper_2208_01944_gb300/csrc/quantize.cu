@@ -74,7 +74,9 @@ __global__ void __launch_bounds__(256) pq_quantize_scalar(const float* __restric
 // pixel rows are read by neighbouring warps at about the same time.  A grid of a
 // few blocks per SM, striding over the (image, pixel group, block group) units,
 // keeps enough loads in flight for the HBM bandwidth.
-template <bool PACK2>
+// PACK = 1: the block's codes packed four to a 32-bit word; PACK = 2: two to a
+// byte (8 bytes, half of the 16-byte row of its 32-channel block).
+template <int PACK>
 __global__ void __launch_bounds__(256) pq_quantize_c16(const float4* __restrict__ x, void* __restrict__ q, int64_t N,
                                                        int64_t HW, int C16, int blocks_per_group, int qmax,
                                                        const __grid_constant__ QuantArgs args) {
@@ -99,8 +101,10 @@ __global__ void __launch_bounds__(256) pq_quantize_c16(const float4* __restrict_
       out.y = quant4(b, inv, qmax);
       out.z = quant4(c, inv, qmax);
       out.w = quant4(d, inv, qmax);
-      if (PACK2)
+      if (PACK == 1)
         __stcs(static_cast<uint32_t*>(q) + (n * C16 + j) * HW + hw, pack2_word(out));
+      else if (PACK == 2)
+        __stcs(static_cast<uint2*>(q) + ((n * (C16 >> 1) + (j >> 1)) * HW + hw) * 2 + (j & 1), pack4_word(out));
       else
         __stcs(static_cast<uint4*>(q) + (n * C16 + j) * HW + hw, out);
     }
@@ -108,7 +112,7 @@ __global__ void __launch_bounds__(256) pq_quantize_c16(const float4* __restrict_
 }
 
 int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G, int Cg, int bits, const float* inv_s,
-                        bool packed2, cudaStream_t stream) {
+                        int pack, cudaStream_t stream) {
   QuantArgs args;
   for (int g = 0; g < G; ++g) args.inv_s[g] = inv_s[g];
   const int C16 = G * Cg / 16;
@@ -120,12 +124,14 @@ int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G
   const int64_t want = (warps + 7) / 8;  // 8 warps per block
   const int64_t cap = static_cast<int64_t>(sms) * 4;
   const unsigned grid = static_cast<unsigned>(want < cap ? want : cap);
-  if (packed2)
-    pq_quantize_c16<true><<<grid, 256, 0, stream>>>(reinterpret_cast<const float4*>(x), q, N, HW, C16, Cg / 16,
-                                                    (1 << bits) - 1, args);
+  const float4* xv = reinterpret_cast<const float4*>(x);
+  const int qmax = (1 << bits) - 1;
+  if (pack == 1)
+    pq_quantize_c16<1><<<grid, 256, 0, stream>>>(xv, q, N, HW, C16, Cg / 16, qmax, args);
+  else if (pack == 2)
+    pq_quantize_c16<2><<<grid, 256, 0, stream>>>(xv, q, N, HW, C16, Cg / 16, qmax, args);
   else
-    pq_quantize_c16<false><<<grid, 256, 0, stream>>>(reinterpret_cast<const float4*>(x), q, N, HW, C16, Cg / 16,
-                                                     (1 << bits) - 1, args);
+    pq_quantize_c16<0><<<grid, 256, 0, stream>>>(xv, q, N, HW, C16, Cg / 16, qmax, args);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }
 

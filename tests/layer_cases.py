@@ -91,9 +91,21 @@ def c16p2_to_nhwc(a: np.ndarray, N: int, H: int, W: int, C: int) -> np.ndarray:
     return np.ascontiguousarray(codes.astype(np.uint8).transpose(0, 2, 3, 1, 4).reshape(N, H, W, C))
 
 
+def c32f4_to_nhwc(a: np.ndarray, N: int, H: int, W: int, C: int) -> np.ndarray:
+    """FP4 nibble codes [N][C/32][H][W][16 bytes], channel 2i of a block in the low
+    nibble of byte i and 2i+1 in the high nibble -> NHWC, one code per byte."""
+    b = np.ascontiguousarray(a).reshape(N, C // 32, H, W, 16)
+    codes = np.stack([b & 15, b >> 4], axis=-1).reshape(N, C // 32, H, W, 32)
+    return np.ascontiguousarray(codes.astype(np.uint8).transpose(0, 2, 3, 1, 4).reshape(N, H, W, C))
+
+
 def to_format(codes_nhwc: np.ndarray, fmt: int) -> np.ndarray:
-    """NHWC codes -> the given code format's bytes (0 NHWC, 2 channel-blocked, 3 packed)."""
+    """NHWC codes -> the given code format's bytes (0 NHWC, 2 channel-blocked, 3 packed
+    2-bit, 4 FP4 nibbles)."""
     N, H, W, C = codes_nhwc.shape
+    if fmt == 4:
+        blk = codes_nhwc.reshape(N, H, W, C // 32, 16, 2).transpose(0, 3, 1, 2, 4, 5).astype(np.uint8)
+        return np.ascontiguousarray(blk[..., 0] | (blk[..., 1] << 4)).reshape(-1)
     blk = codes_nhwc.reshape(N, H, W, C // 16, 16).transpose(0, 3, 1, 2, 4)
     if fmt == 2:
         return np.ascontiguousarray(blk).reshape(-1)
@@ -108,7 +120,14 @@ def from_format(raw: np.ndarray, fmt: int, N: int, H: int, W: int, C: int) -> np
         return c16_to_nhwc(raw, N, H, W, C)
     if fmt == 3:
         return c16p2_to_nhwc(raw, N, H, W, C)
+    if fmt == 4:
+        return c32f4_to_nhwc(raw, N, H, W, C)
     return np.ascontiguousarray(raw).reshape(N, H, W, C)
+
+
+def code_bytes(n_codes: int, fmt: int) -> int:
+    """Bytes of n_codes codes in a code format."""
+    return n_codes // {3: 4, 4: 2}.get(fmt, 1)
 
 
 def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q"), fmt: int = 0):
@@ -121,7 +140,7 @@ def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q"), fmt: int = 0):
 
     dev = torch.device("cuda:0")
     x = torch.from_numpy(ref["x"]).to(dev)
-    nq = x.numel() // (4 if fmt == B.PQ_CODES_C16P2 else 1)
+    nq = code_bytes(x.numel(), fmt)
     q = torch.empty(nq, dtype=torch.uint8, device=dev)
     B.palquant_quantize_act(x, q, c.N, c.H, c.W, c.G, c.Cin, c.bits, ref["inv_s"], code_format=fmt)
     d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad, c.bits, c.bits, c.bo, int(c.relu),
@@ -132,7 +151,7 @@ def run_gpu(c: Case, ref: dict, outputs=("acc", "y", "q"), fmt: int = 0):
     shape = (c.N, c.Ho, c.Wo, c.G * c.Cout)
     acc = torch.full(shape, -7, dtype=torch.int32, device=dev) if "acc" in outputs else None
     y = torch.full(shape, float("nan"), dtype=torch.float32, device=dev) if "y" in outputs else None
-    nqo = int(np.prod(shape)) // (4 if fmt == B.PQ_CODES_C16P2 else 1)
+    nqo = code_bytes(int(np.prod(shape)), fmt)
     qo = torch.full((nqo,), 255, dtype=torch.uint8, device=dev) if "q" in outputs else None
     sc = None if ref["shortcut"] is None else torch.from_numpy(ref["shortcut"]).to(dev)
     B.palquant_layer_fused(q, wp, d, ref["m_out"], ref["m_req"], B.shuffle(c.kind, c.shift, c.perm), sc, acc, y, qo)

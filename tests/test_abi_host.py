@@ -234,3 +234,99 @@ def test_odd_level_weights_match_oracle(bits):
     d = B.layer_desc(1, 6, 6, G, Ci, Co, k, 1, 1, 2, bits, 2)
     packed = B.palquant_pack_weights_odd_host(w, d, u)
     assert np.array_equal(B.palquant_unpack_weight_codes_host(packed, d), oracle.quantize_weights_odd(w, bits, u))
+
+
+# --------------------------------------------- packed FP4 codes (format 4)
+def _e2m1_value(nib):
+    """E2M1 by its definition: sign bit 3, exponent bits 2-1 (bias 1), mantissa bit 0;
+    exponent 0 is subnormal (m * 0.5)."""
+    nib = np.asarray(nib, dtype=np.int64)
+    s = np.where(nib & 8, -1.0, 1.0)
+    e, m = (nib >> 1) & 3, nib & 1
+    mag = np.where(e == 0, m * 0.5, (1.0 + m / 2.0) * 2.0 ** (e - 1))
+    return s * mag
+
+
+def test_fp4_nibble_of_code_is_e2m1_of_half_code():
+    """An activation code v <= 3 stored as the nibble v reads as v / 2 in E2M1, and
+    the weight codes -4..4 all have exact E2M1 encodings."""
+    v = np.arange(4)
+    assert np.array_equal(_e2m1_value(v), v / 2.0)
+    vals = _e2m1_value(np.arange(16))
+    for w in range(-4, 5):
+        assert w in vals
+    # the block scale 2^-4 on both operands turns (v/2) * w into v * w * 2^-9
+    assert (0.5 * 2.0 ** -4) * 2.0 ** -4 == 2.0 ** -9
+
+
+@pytest.mark.parametrize("shape", [(2, 64, 3, 64, 2), (4, 96, 1, 128, 3), (1, 288, 3, 64, 2), (2, 32, 3, 192, 3)])
+def test_fp4_pack_unpack_roundtrip_and_e2m1_encoding(shape):
+    G, Co, k, Ci, bits_w = shape
+    d = B.layer_desc(1, 8, 8, G, Ci, Co, k, 1, k // 2, 2, bits_w, 2, code_format=B.PQ_CODES_C32F4)
+    gen = synth.generator(sum(shape) + 5)
+    wq = synth.random_codes((G, Co, k, k, Ci), bits_w, gen, signed=True)
+    packed = B.palquant_pack_weight_codes_host(wq, d)
+    assert packed.size == wq.size // 2
+    assert np.array_equal(B.palquant_unpack_weight_codes_host(packed, d), wq)
+    nibbles = np.stack([packed & 15, packed >> 4], axis=-1).ravel()
+    assert np.array_equal(np.sort(_e2m1_value(nibbles)), np.sort(wq.ravel().astype(np.float64)))
+
+
+def test_fp4_layout_rules():
+    F4 = B.PQ_CODES_C32F4
+    ok = B.palquant_conv_plan(B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 3, 2, code_format=F4))
+    assert ok.supported == 1 and ok.k_chunk % 64 == 0
+    for d in [B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 3, 2, 2, code_format=F4),   # 3-bit activations
+              B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 4, 2, code_format=F4),   # 4-bit weights
+              B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 2, 3, code_format=F4),   # 3-bit output codes
+              B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=F4),   # Cin_g % 64 != 0
+              B.layer_desc(1, 8, 8, 2, 64, 48, 3, 1, 1, 2, 2, 2, code_format=F4)]:  # Cout_g % 32 != 0
+        assert B.palquant_conv_plan(d).supported == 0
+    d = B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 2, 2, code_format=F4)
+    with pytest.raises(B.PalquantError) as e:   # a per-channel scatter cannot write nibbles
+        B.palquant_layer_fused(16, 16, d, [1.0] * 2, [1.0] * 2, shuf=B.shuffle(2, 0), q_out_dev=16)
+    assert e.value.status == B.PQ_EUNSUPPORTED
+    with pytest.raises(B.PalquantError) as e:   # bit-decomposed slices are one per byte
+        B.palquant_bitsplit_desc(d, 1)
+    assert e.value.status == B.PQ_EUNSUPPORTED
+    w = np.zeros((2, 32, 3, 3, 64), np.float32)
+    with pytest.raises(B.PalquantError) as e:   # odd levels +-5, +-7 are not E2M1 values
+        B.palquant_pack_weights_odd_host(w, B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 3, 2, code_format=F4),
+                                         [1.0, 1.0])
+    assert e.value.status == B.PQ_EUNSUPPORTED
+    with pytest.raises(B.PalquantError) as e:   # the quantiser's FP4 output holds 2-bit codes
+        B.palquant_quantize_act(16, 16, 1, 4, 4, 2, 32, 3, [1.0, 1.0], code_format=F4)
+    assert e.value.status == B.PQ_EINVAL
+
+
+F4_LAYERS = [c for c in ALL_LAYERS if c.bits_a <= 2 and c.bits_out <= 2 and c.bits_w <= 3 and c.Cin_g % 64 == 0
+             and c.Cout_g % 32 == 0]
+
+
+@pytest.mark.parametrize("c", F4_LAYERS, ids=lambda c: f"{c.H}x{c.W}k{c.k}s{c.stride}G{c.G}c{c.Cin_g}-{c.Cout_g}")
+def test_fp4_plan_invariants(c):
+    plan = B.palquant_conv_plan(_desc(c, code_format=B.PQ_CODES_C32F4))
+    assert plan.supported == 1
+    assert plan.smem_bytes + 1024 <= 227 * 1024
+    assert plan.n_block * plan.n_blocks == c.Cout_g and plan.n_block % 16 == 0 and plan.n_block <= 128
+    assert plan.k_chunk * plan.k_blocks == c.Cin_g and plan.k_chunk % 64 == 0
+    # accumulators and the 32 scale-factor columns share the 512 TMEM columns
+    npow2 = 1 << (plan.n_block - 1).bit_length()
+    assert plan.acc_stages * plan.m_tiles * npow2 + 32 <= 512
+
+
+def test_fp4_code_helpers_roundtrip():
+    from layer_cases import c32f4_to_nhwc, code_bytes, from_format, to_format
+
+    gen = synth.generator(78)
+    q = synth.random_codes((2, 3, 4, 64), 2, gen)
+    raw = to_format(q, 4)
+    assert raw.size == code_bytes(q.size, 4) == q.size // 2
+    assert np.array_equal(c32f4_to_nhwc(raw, 2, 3, 4, 64), q)
+    assert np.array_equal(from_format(raw, 4, 2, 3, 4, 64), q)
+    # channel c of a position: byte (c % 32) / 2 of its block's 16-byte row, low
+    # nibble for even c; the second 32-channel block lies H*W*16 bytes further on
+    one = np.zeros((1, 2, 1, 64), np.uint8)
+    one[0, 1, 0, 32 + 7] = 3
+    r = to_format(one, 4)
+    assert np.flatnonzero(r).tolist() == [2 * 16 + 16 + 3] and r[2 * 16 + 16 + 3] == 3 << 4

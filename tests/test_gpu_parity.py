@@ -354,3 +354,117 @@ def test_layer_with_odd_weight_levels_matches_oracle(B, fmt, bits_w):
     assert np.array_equal(ad.cpu().numpy(), a_ref)
     assert np.array_equal(yd.cpu().numpy(), y_ref)
     assert np.array_equal(from_format(qo.cpu().numpy(), fmt, N, H, W, G * Co).reshape(-1, G * Co), q_ref)
+
+
+# --------------------------- packed FP4 codes (format 4, block-scaled FP4 MMA)
+F4_CASES = [
+    Case(1, 28, 28, 2, 64, 32, 3, 1, 1, seed=80),
+    Case(2, 13, 11, 3, 64, 96, 3, 1, 1, seed=81),                     # odd sizes, six 16-column chunks
+    Case(3, 9, 17, 4, 64, 64, 3, 2, 1, seed=82),                      # stride 2 (copy warps)
+    Case(2, 10, 10, 2, 64, 128, 1, 2, 0, kind=0, relu=False, seed=83),  # 1x1 stride-2 downsample
+    Case(2, 7, 9, 4, 128, 96, 1, 1, 0, seed=84),                      # flat mode, ragged last tile
+    Case(2, 14, 14, 8, 64, 32, 3, 1, 1, kind=3, perm=(3, 0, 7, 1, 6, 2, 5, 4), seed=85),
+    Case(1, 12, 12, 2, 128, 256, 3, 1, 1, seed=86),                   # two output-channel blocks of 128
+    Case(1, 7, 7, 2, 1024, 32, 3, 1, 1, seed=87),                     # two K blocks, whole-image tiles
+    Case(2, 8, 8, 2, 64, 320, 3, 1, 1, seed=88),                      # 80-column blocks: half-row stores
+    Case(1, 5, 130, 1, 64, 32, 3, 1, 1, seed=89),                     # rows wider than 128 positions
+    Case(2, 11, 10, 2, 64, 64, 3, 1, 1, shortcut=True, seed=90),      # shortcut add before ReLU
+    Case(1, 9, 11, 2, 64, 64, 5, 1, 2, seed=91),                      # 5x5 kernel
+    Case(2, 6, 6, 2, 64, 32, 3, 1, 1, bits_out=1, relu=False, kind=1, shift=-1, seed=92),
+    Case(1, 16, 16, 4, 64, 64, 3, 2, 0, seed=93),                     # stride 2 without padding
+    Case(2, 8, 8, 2, 256, 256, 3, 1, 1, seed=94),                     # 256 channels per group
+    Case(1, 10, 10, 2, 192, 64, 3, 1, 1, seed=95),                    # three K steps per tap
+]
+
+
+@pytest.mark.parametrize("c", F4_CASES, ids=str)
+def test_layer_fused_fp4_codes_matches_oracle(B, c):
+    ref = prepare(c)
+    got = run_gpu(c, ref, fmt=B.PQ_CODES_C32F4)
+    assert_layer_parity(c, ref, got)
+
+
+@pytest.mark.parametrize("c", F4_CASES, ids=str)
+def test_layer_codes_only_fp4_matches_oracle(B, c):
+    ref = prepare(c)
+    got = run_gpu(c, ref, outputs=("q",), fmt=B.PQ_CODES_C32F4)
+    assert_layer_parity(c, ref, got)
+
+
+F4_FULL = [(n, c) for n, c in FULL if c.bits_a <= 2 and c.Cin_g % 64 == 0 and c.Cout_g % 32 == 0]
+
+
+@pytest.mark.parametrize("name,cfg", F4_FULL, ids=[n for n, _ in F4_FULL])
+def test_full_size_codes_only_fp4_sampled(B, name, cfg):
+    c = Case(cfg.N, cfg.H, cfg.W, cfg.G, cfg.Cin_g, cfg.Cout_g, cfg.k, cfg.stride, cfg.pad, bits=cfg.bits_a,
+             kind=cfg.shuffle_kind, shift=cfg.shuffle_shift, relu=cfg.relu, seed=0)
+    pix = _sample_pixels(c.N, c.Ho, c.Wo, 3000, 4)
+    ref = prepare(c, sample_pix=pix)
+    got = run_gpu(c, ref, outputs=("q",), fmt=B.PQ_CODES_C32F4)
+    assert_layer_parity(c, ref, got, pix)
+
+
+@pytest.mark.parametrize("bits_w,Cin", [(3, 1024), (2, 1024), (3, 64)])
+def test_fp4_worst_case_magnitudes_exact(B, bits_w, Cin):
+    """Activation codes all 3, weight codes all at an extreme (-4 with 3 bits): the
+    largest sums the FP4 path can produce, exact."""
+    G, Co, k, N, H, W = 2, 32, 3, 1, 6, 6
+    from layer_cases import to_format
+
+    q = np.full((N, H, W, G * Cin), 3, dtype=np.uint8)
+    wq = np.full((G, Co, k, k, Cin), -(1 << (bits_w - 1)), dtype=np.int8)
+    wq[1] = (1 << (bits_w - 1)) - 1
+    d = B.layer_desc(N, H, W, G, Cin, Co, k, 1, 1, 2, bits_w, 2, code_format=B.PQ_CODES_C32F4)
+    wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).cuda()
+    acc = torch.zeros((N, H, W, G * Co), dtype=torch.int32, device="cuda")
+    B.palquant_group_conv(torch.from_numpy(to_format(q, 4)).cuda(), wp, acc, d)
+    assert B.palquant_sync_check() == B.PQ_OK
+    ref = oracle.group_conv(q, wq, 1, 1)
+    assert np.abs(ref).max() == 9 * Cin * 3 * (1 << (bits_w - 1))
+    assert np.array_equal(acc.cpu().numpy().astype(np.int64), ref)
+
+
+@pytest.mark.parametrize("shape,G,bits", [((2, 7, 9, 64), 4, 2), ((1, 5, 6, 96), 3, 1), ((2, 11, 13, 768), 4, 2),
+                                          ((3, 4, 5, 32), 2, 2)])
+def test_quantize_act_fp4_matches_oracle(B, shape, G, bits):
+    from layer_cases import c32f4_to_nhwc
+
+    gen = synth.generator(sum(shape) + 13)
+    x = synth.normal(shape, gen, 2.0)
+    x.reshape(-1)[:6] = np.array([0.5, 1.5, 2.5, np.nan, np.inf, -np.inf], dtype=np.float32)
+    inv = (synth.half_normal((G,), gen) + 0.5).astype(np.float32)
+    q = torch.full((int(np.prod(shape)) // 2,), 254, dtype=torch.uint8, device="cuda")
+    B.palquant_quantize_act(torch.from_numpy(x).cuda(), q, shape[0], shape[1], shape[2], G, shape[3] // G, bits, inv,
+                            code_format=B.PQ_CODES_C32F4)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(c32f4_to_nhwc(q.cpu().numpy(), *shape), oracle.quantize_act(x, G, bits, inv))
+
+
+def test_layer_fp4_with_odd_weight_levels_matches_oracle(B):
+    from layer_cases import from_format
+
+    N, H, W, G, Ci, Co = 2, 12, 10, 2, 64, 64
+    gen = synth.generator(75)
+    x = synth.half_normal((N, H, W, G * Ci), gen)
+    w = synth.he_weights(G, Co, 3, 3, Ci, gen)
+    s_a = oracle.act_step(x, G, 2)
+    inv_s = oracle.inv_step(s_a)
+    u = (2.0 * np.abs(w).reshape(G, -1).mean(axis=1)).astype(np.float32)
+    s_w = (u.astype(np.float64) / 3.0).astype(np.float32)
+    q = oracle.quantize_act(x, G, 2, inv_s)
+    wq = oracle.quantize_weights_odd(w, 2, u)
+    m_out, m_req = oracle.epilogue_scales(s_w, s_a, s_a, 1.0, 1, 1)
+    acc = oracle.group_conv(q, wq, 1, 1).reshape(-1, G * Co)
+    a_ref, y_ref, q_ref = oracle.epilogue(acc, G, m_out, m_req, 1, 1, None, None, True, 2)
+    d = B.layer_desc(N, H, W, G, Ci, Co, 3, 1, 1, 2, 2, 2, 1, code_format=B.PQ_CODES_C32F4)
+    wp = torch.from_numpy(B.palquant_pack_weights_odd_host(w, d, u)).cuda()
+    qd = torch.empty(x.size // 2, dtype=torch.uint8, device="cuda")
+    B.palquant_quantize_act(torch.from_numpy(x).cuda(), qd, N, H, W, G, Ci, 2, inv_s, code_format=B.PQ_CODES_C32F4)
+    ad = torch.empty((N * H * W, G * Co), dtype=torch.int32, device="cuda")
+    yd = torch.empty((N * H * W, G * Co), dtype=torch.float32, device="cuda")
+    qo = torch.empty(N * H * W * G * Co // 2, dtype=torch.uint8, device="cuda")
+    B.palquant_layer_fused(qd, wp, d, m_out, m_req, B.shuffle(1, 1), None, ad, yd, qo)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(ad.cpu().numpy(), a_ref)
+    assert np.array_equal(yd.cpu().numpy(), y_ref)
+    assert np.array_equal(from_format(qo.cpu().numpy(), 4, N, H, W, G * Co).reshape(-1, G * Co), q_ref)
