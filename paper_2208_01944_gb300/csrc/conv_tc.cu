@@ -104,7 +104,7 @@ __device__ __forceinline__ void item_next(const ConvParams& p, Item& r) {
 // Shared-memory barrier block layout (64-bit words):
 //   [0, A)           a_full       [A, 2A)        a_empty
 //   [2A, 2A+B)       b_full       [2A+B, 2A+2B)  b_empty
-//   +0,+1 acc_full, +2,+3 acc_empty, +4 drain, then A pk_full and A pk_empty
+//   +0..+3 acc_full, +4..+7 acc_empty (kMaxAccStages), +8 drain, then A pk_full and A pk_empty
 //   (packed codes only), then int abort flag, u32 TMEM base.
 struct Bars {
   uint32_t base;
@@ -114,13 +114,20 @@ struct Bars {
   __device__ uint32_t b_full(int s) const { return base + 8u * (2 * A + s); }
   __device__ uint32_t b_empty(int s) const { return base + 8u * (2 * A + B + s); }
   __device__ uint32_t acc_full(int s) const { return base + 8u * (2 * A + 2 * B + s); }
-  __device__ uint32_t acc_empty(int s) const { return base + 8u * (2 * A + 2 * B + 2 + s); }
-  __device__ uint32_t drain() const { return base + 8u * (2 * A + 2 * B + 4); }
+  __device__ uint32_t acc_empty(int s) const { return base + 8u * (2 * A + 2 * B + kMaxAccStages + s); }
+  __device__ uint32_t drain() const { return base + 8u * (2 * A + 2 * B + 2 * kMaxAccStages); }
   // packed-code staging ring (one stage per operand stage)
-  __device__ uint32_t pk_full(int s) const { return base + 8u * (2 * A + 2 * B + 5 + s); }
-  __device__ uint32_t pk_empty(int s) const { return base + 8u * (3 * A + 2 * B + 5 + s); }
-  __device__ uint32_t words() const { return 4 * A + 2 * B + 5; }
+  __device__ uint32_t pk_full(int s) const { return base + 8u * (2 * A + 2 * B + 2 * kMaxAccStages + 1 + s); }
+  __device__ uint32_t pk_empty(int s) const { return base + 8u * (3 * A + 2 * B + 2 * kMaxAccStages + 1 + s); }
+  __device__ uint32_t words() const { return 4 * A + 2 * B + 2 * kMaxAccStages + 1; }
 };
+
+// Wait taken by every lane of a converged warp; the lanes agree on the outcome,
+// so the warp stays converged (for warp barriers and per-warp arrivals) even when
+// a wait times out.
+__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const WaitCtx& ctx) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, ctx));
+}
 
 // --------------------------------------------------------------------------
 // Copy role (warp 0, lane 0): bulk copies of the packed weights, either once
@@ -217,9 +224,12 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
 constexpr int kLoaders = 32 * kLoadWarps;
 constexpr int kMaxLoadEntries = 8;
 
+// Every thread's copies of the stage have landed (its wait_group); after the
+// proxy fence and a warp barrier one lane arrives for the warp.
 __device__ __forceinline__ void load_release(const Bars& bars, int64_t k, int stages) {
   fence_proxy_async_smem();
-  mbar_arrive(bars.a_full(static_cast<int>(k % stages)));
+  __syncwarp();
+  if ((threadIdx.x & 31) == 0) mbar_arrive(bars.a_full(static_cast<int>(k % stages)));
 }
 
 __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bars, uint32_t a_base, int64_t it0, int64_t it1,
@@ -264,7 +274,7 @@ __device__ __forceinline__ void loader_role(const ConvParams& p, const Bars& bar
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1 && ok; ++it, item_next(p, item)) {
     for (int kb = 0; kb < p.n_kb; ++kb) {
-      if (!mbar_wait(bars.a_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
+      if (!warp_wait(bars.a_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
       const uint32_t stage = a_base + ra.stage * p.a_stage_bytes;
       const int ch0 = p.src_group[item.g] * p.Cin_g + kb * p.KC;  // first input channel of the K block
       const uint8_t* img_src = p.q_in + item.n * p.ld_img + static_cast<int64_t>(ch0) * p.ld_c0_mul / 16;
@@ -355,8 +365,8 @@ __device__ __forceinline__ void unpack_role(const ConvParams& p, const Bars& bar
   bool ok = true;
   for (int64_t it = it0; it < it1 && ok; ++it) {
     for (int kb = 0; kb < p.n_kb; ++kb) {
-      if (!mbar_wait(bars.pk_full(r.stage), r.phase, ctx)) { ok = false; break; }
-      if (!mbar_wait(bars.a_empty(r.stage), r.phase ^ 1u, ctx)) { ok = false; break; }
+      if (!warp_wait(bars.pk_full(r.stage), r.phase, ctx)) { ok = false; break; }
+      if (!warp_wait(bars.a_empty(r.stage), r.phase ^ 1u, ctx)) { ok = false; break; }
       const uint32_t src = pk_base + r.stage * p.pk_stage_bytes;
       const uint32_t dst = a_base + r.stage * p.a_stage_bytes;
       for (int row = wi; row < n_rows; row += kLoadWarps) {
@@ -373,8 +383,11 @@ __device__ __forceinline__ void unpack_role(const ConvParams& p, const Bars& bar
         }
       }
       fence_proxy_async_smem();
-      mbar_arrive(bars.a_full(r.stage));
-      mbar_arrive(bars.pk_empty(r.stage));
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(bars.a_full(r.stage));
+        mbar_arrive(bars.pk_empty(r.stage));
+      }
       r.advance();
     }
   }
@@ -383,10 +396,6 @@ __device__ __forceinline__ void unpack_role(const ConvParams& p, const Bars& bar
 // --------------------------------------------------------------------------
 // Tensor-core issue role (warp 1).
 // --------------------------------------------------------------------------
-// Wait taken by every lane of a converged warp; the lanes agree on the outcome.
-__device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, const WaitCtx& ctx) {
-  return __all_sync(0xffffffffu, mbar_wait(bar, parity, ctx));
-}
 
 constexpr int kUnrollTaps = 9;
 
@@ -756,7 +765,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
   const bool codes_only = p.shortcut == nullptr && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle;
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1; ++it, item_next(p, item)) {
-    if (!mbar_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
+    if (!warp_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
     tc_fence_after();
     EpiItem e;
     e.g = item.g;
@@ -770,7 +779,56 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
     e.src_c0 = e.g * p.Cout_g + item.nb * p.Nblk;               // source channel of column 0
     e.dst_c0 = p.dst_group[e.g] * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
     e.tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2;
-    if (codes_only && p.codes_c16) {
+    if (codes_only && p.codes_f4 && (p.Nblk & 31) == 0) {
+      // FP4 nibbles, units of 32 columns: a lane's 32 codes are one whole 16-byte
+      // row of a 32-channel block, so a unit costs one store instruction (the
+      // epilogue's time goes mostly to store instructions, not bytes).
+      const int nb32 = p.Nblk >> 5;
+      const long long blk_bytes = static_cast<long long>(p.Ho) * p.Wo * 16;
+      uint8_t* const blk0 =
+          p.q_out + (static_cast<long long>(e.n) * (p.C_out_total >> 5) + (e.dst_c0 >> 5)) * blk_bytes;
+      const int m_lane = quarter * 32 + lane;
+      const int MT = p.MT;
+      auto row_ptr = [&](int mt) -> uint8_t* {
+        if (mt >= MT) return nullptr;
+        bool valid;
+        const int pos = epi_pos(p, e, mt * 128 + m_lane, valid);
+        return valid ? blk0 + static_cast<long long>(pos) * 16 : nullptr;
+      };
+      auto step = [&](int& mt, int& b) {
+        b += n_groups;
+        while (b >= nb32) {
+          b -= nb32;
+          ++mt;
+        }
+      };
+      auto col = [&](int mt, int b) { return e.tbase + static_cast<uint32_t>(mt) * p.Npow2 + b * 32; };
+      // Two 16-column buffers: the unit's first half (va) is converted while its
+      // second half (vb) loads, and the next unit's first half loads while the
+      // second half is converted and the row is stored.
+      uint32_t va[16], vb[16];
+      int c_mt = 0, c_b = wg - n_groups;
+      step(c_mt, c_b);
+      uint8_t* c_row = row_ptr(c_mt);
+      if (c_mt < MT) {
+        tmem_ld16(col(c_mt, c_b), va);
+        tmem_wait_ld();
+      }
+      while (c_mt < MT) {
+        tmem_ld16(col(c_mt, c_b) + 16, vb);
+        const uint2 lo = pack4_word(epi_codes16(va, e.m_req512, qmax_f));
+        tmem_wait_ld();
+        int n_mt = c_mt, n_b = c_b;
+        step(n_mt, n_b);
+        if (n_mt < MT) tmem_ld16(col(n_mt, n_b), va);
+        const uint2 hi = pack4_word(epi_codes16(vb, e.m_req512, qmax_f));
+        tmem_wait_ld();  // before the store: a TMEM-load wait right after a store stalls on the store
+        if (c_row) *reinterpret_cast<uint4*>(c_row + c_b * blk_bytes) = make_uint4(lo.x, lo.y, hi.x, hi.y);
+        c_row = n_mt == c_mt ? c_row : row_ptr(n_mt);
+        c_mt = n_mt;
+        c_b = n_b;
+      }
+    } else if (codes_only && p.codes_c16) {
       // Channel-blocked codes only (the timed path).  A warp's units run in
       // increasing (mt, ch) order; the destination of this lane's row is
       // computed once per accumulator, and 16-channel block ch of that row lies
@@ -821,9 +879,9 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         if (n_mt < MT) tmem_ld16(col(n_mt, n_ch), vb);
         {
           const uint4 w = epi_codes16(va, e.m_req512, qmax_f);
+          tmem_wait_ld();  // before the store: a TMEM-load wait right after a store stalls on the store
           if (c_row) store_codes16(c_row + coff(c_ch), w, pack);
         }
-        tmem_wait_ld();
         if (n_mt >= MT) break;
         uint8_t* n_row = n_mt == c_mt ? c_row : row_ptr(n_mt);
         int m2 = n_mt, c2 = n_ch;
@@ -831,9 +889,9 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         if (m2 < MT) tmem_ld16(col(m2, c2), va);
         {
           const uint4 w = epi_codes16(vb, e.m_req512, qmax_f);
+          tmem_wait_ld();
           if (n_row) store_codes16(n_row + coff(n_ch), w, pack);
         }
-        tmem_wait_ld();
         c_row = m2 == n_mt ? n_row : row_ptr(m2);
         c_mt = m2;
         c_ch = c2;
@@ -847,8 +905,12 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         epi_general16(p, e, stg, lane, mt * 128 + quarter * 32 + lane, ch, v);
       }
     }
+    // One arrival per warp: the warp's tensor-memory reads are complete (each
+    // thread waited for its loads) and ordered before the arrive by the fence
+    // and the warp barrier.
     tc_fence_before();
-    mbar_arrive(bars.acc_empty(racc.stage));
+    __syncwarp();
+    if (lane == 0) mbar_arrive(bars.acc_empty(racc.stage));
     racc.advance();
   }
 }
@@ -872,20 +934,20 @@ __global__ void __launch_bounds__(kConvThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < bars.A; ++s) {
-      mbar_init(bars.a_full(s), (p.a_tma && !p.a_unpack) ? 1 : 32 * kLoadWarps);
+      mbar_init(bars.a_full(s), (p.a_tma && !p.a_unpack) ? 1 : kLoadWarps);  // TMA, or one arrival per copy warp
       mbar_init(bars.a_empty(s), 1);
       if (p.a_unpack) {
         mbar_init(bars.pk_full(s), 1);
-        mbar_init(bars.pk_empty(s), 32 * kLoadWarps);
+        mbar_init(bars.pk_empty(s), kLoadWarps);
       }
     }
     for (int s = 0; s < bars.B; ++s) {
       mbar_init(bars.b_full(s), 1);
       mbar_init(bars.b_empty(s), 1);
     }
-    for (int s = 0; s < 2; ++s) {
+    for (int s = 0; s < p.acc_stages; ++s) {
       mbar_init(bars.acc_full(s), 1);
-      mbar_init(bars.acc_empty(s), ((p.a_tma && !p.a_unpack) ? kEpiWarps + kLoadWarps : kEpiWarps) * 32);
+      mbar_init(bars.acc_empty(s), (p.a_tma && !p.a_unpack) ? kEpiWarps + kLoadWarps : kEpiWarps);  // one per warp
     }
     mbar_init(bars.drain(), 1);
     *abort_flag = 0;

@@ -19,6 +19,7 @@ namespace pq {
 constexpr int kMaxG = 64;
 constexpr int kMaxTaps = 49;
 constexpr int kMaxPhases = 4;
+constexpr int kMaxAccStages = 4;                   // TMEM accumulator ring depth at most
 constexpr int kEpiGroups = 2;                      // epilogue warpgroups, splitting the output columns
 constexpr int kEpiWarps = 4 * kEpiGroups;
 constexpr int kLoadWarps = 4;                      // activation-operand copy warps
@@ -84,7 +85,7 @@ struct ConvParams {
   uint32_t b_unit_bytes;  // taps * Cin_g * Nblk
   uint32_t lbo_b;         // Nblk * 16
   int b_stages;           // ring stages when streamed
-  int acc_stages;         // TMEM accumulator buffers
+  int acc_stages;         // TMEM accumulator buffers (ring of 1..kMaxAccStages)
   uint32_t tmem_cols;
   uint32_t smem_b_off, smem_stage_off, smem_bar_off, smem_bytes;
   uint32_t stage_q_pitch, stage_f_pitch, stage_warp_bytes;
