@@ -284,6 +284,7 @@ def measure_layer_configs(dev, args):
 
     pk = peaks()
     fp8_peak = 2.0 * pk["bf16_tflops"]
+    fp4_peak = 6.0 * pk["bf16_tflops"]
     stream = torch.cuda.Stream(device=dev)
     fmt = B.PQ_CODES_C16
     out = {}
@@ -328,6 +329,29 @@ def measure_layer_configs(dev, args):
                      "buffer_sets": n_sets, "plan": {k: plan[k] for k in ("m_tiles", "n_block", "k_chunk",
                                                                          "weights_resident", "work_items")}}
         del qs, qo, q, wp
+        # the same layer with packed FP4 codes (block-scaled FP4 tensor path), where it applies
+        d4 = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w,
+                          c.bits_out, int(c.relu), code_format=B.PQ_CODES_C32F4)
+        if B.palquant_conv_plan(d4).supported:
+            nin, nout = c.in_elems // 2, c.out_elems // 2
+            n4 = max(1, min(16, -(-2 * L2_BYTES // (nin + nout))))
+            lo = synth.random_codes((nin,), c.bits_a, gen)
+            q4 = torch.from_numpy(lo | (synth.random_codes((nin,), c.bits_a, gen) << 4)).to(dev)
+            q4s = [q4] + [q4.clone() for _ in range(n4 - 1)]
+            wp4 = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d4)).to(dev)
+            qo4 = [torch.empty(nout, dtype=torch.uint8, device=dev) for _ in range(n4)]
+            ms4 = timed(lambda i: B.palquant_layer_fused(q4s[i], wp4, d4, m, m, shuf, None, None, None, qo4[i],
+                                                         stream=stream), n4)
+            tops4 = c.int_ops / (ms4 / 1e3) / 1e12
+            byt4 = nin + nout + c.weight_elems // 2
+            plan4 = B.palquant_conv_plan(d4).as_dict()
+            out[name + "_fp4"] = {"shape": c.name + ", packed FP4 codes", "us": ms4 * 1e3, "tops": tops4,
+                                  "frac_fp4_peak": tops4 / fp4_peak, "frac_fp8_peak": tops4 / fp8_peak,
+                                  "algorithmic_gbs": byt4 / (ms4 / 1e3) / 1e9,
+                                  "frac_hbm": byt4 / (ms4 / 1e3) / 1e9 / pk["hbm_gbs"], "buffer_sets": n4,
+                                  "plan": {k: plan4[k] for k in ("m_tiles", "n_block", "k_chunk", "weights_resident",
+                                                                  "work_items")}}
+            del q4s, qo4, q4, wp4
     out["table2_4bit_on_2bit"] = measure_bitsplit_vs_palquant(dev, stream, timed, pk, fp8_peak)
     for name in ("config1", "config4"):
         c = workloads.BENCH_CONFIGS[name]
@@ -343,7 +367,14 @@ def measure_layer_configs(dev, args):
         gbs = per_set / (ms / 1e3) / 1e9
         out["quantize_" + name] = {"shape": f"{c.N}x{c.H}x{c.W}x{c.G * c.Cin_g} fp32 -> channel-blocked codes",
                                    "us": ms * 1e3, "gbs": gbs, "frac_hbm": gbs / pk["hbm_gbs"], "buffer_sets": n_sets}
-        del xs, qq, x
+        qq4 = [torch.empty(c.in_elems // 2, dtype=torch.uint8, device=dev) for _ in range(n_sets)]
+        ms4 = timed(lambda i: B.palquant_quantize_act(xs[i], qq4[i], c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv,
+                                                      code_format=B.PQ_CODES_C32F4, stream=stream), n_sets)
+        b4 = c.in_elems * 4 + c.in_elems // 2
+        out["quantize_" + name + "_fp4"] = {"shape": f"{c.N}x{c.H}x{c.W}x{c.G * c.Cin_g} fp32 -> packed FP4 codes",
+                                            "us": ms4 * 1e3, "gbs": b4 / (ms4 / 1e3) / 1e9,
+                                            "frac_hbm": b4 / (ms4 / 1e3) / 1e9 / pk["hbm_gbs"], "buffer_sets": n_sets}
+        del xs, qq, x, qq4
     torch.cuda.empty_cache()
     return out
 
@@ -446,7 +477,9 @@ def measure_resnet18(dev, world, args):
            "images_per_s": whole_job_rate(N, world, ms), "ms_per_batch": ms, "batch_per_gpu": N, "reps": R,
            "palquant_body_tops": whole_job_rate(net.body_int_ops(), world, ms) / 1e12,
            "timed": "CUDA-graph replay of the whole forward (stem, pooling, quantiser, 20 PalQuant layers, pooling, FC)",
-           "gpu_launches_per_forward": net.launches_per_forward(), "data": "synthetic"}
+           "gpu_launches_per_forward": net.launches_per_forward(), "data": "synthetic",
+           "code_layout": ("packed FP4 nibbles [N][C/32][H][W][16 B] between layers" if net.fmt == B.PQ_CODES_C32F4
+                           else "channel-blocked [N][C/16][H][W][16], one byte per code")}
     # where the time goes: one eager forward with events between its stages
     marks = []
     net.forward(xs[0], marks)
@@ -468,6 +501,80 @@ def measure_resnet18(dev, world, args):
         out["cpu_baseline"] = {"value": 1.0 / dt, "unit": "images/s", "cores": oracle.num_threads(), "kind": "oracle",
                                "sample": f"1 image, forward with given steps, {dt:.2f} s"}
     return out
+
+
+def measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf, K, world):
+    """The same step (quantise + fused layer, same steps and multipliers) with the
+    codes as packed FP4 nibbles (PQ_CODES_C32F4) and the block-scaled FP4 tensor-core
+    path: K timed steps after 3 warm-up steps, per-kernel CUDA events."""
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+
+    fmt = B.PQ_CODES_C32F4
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out,
+                     int(c.relu), code_format=fmt)
+    nbytes = B.palquant_packed_weight_bytes(d)
+    wp = torch.empty(nbytes, dtype=torch.uint8, device=dev)
+    B.palquant_pack_weights(w_np, d, inv_sw, wp, nbytes)
+    q = torch.empty(c.in_elems // 2, dtype=torch.uint8, device=dev)
+    q_out = torch.empty(c.out_elems // 2, dtype=torch.uint8, device=dev)
+
+    def launch(i):
+        B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt,
+                                stream=stream)
+        B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for i in range(3):
+            launch(i)
+    torch.cuda.synchronize(dev)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for i in range(K):
+            ev[i][0].record(stream)
+            B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt,
+                                    stream=stream)
+            ev[i][1].record(stream)
+            B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
+            ev[i][2].record(stream)
+        stop.record(stream)
+    torch.cuda.synchronize(dev)
+    st = B.palquant_sync_check(stream)
+    assert st == B.PQ_OK, B.strerror(st)
+    return {"ms_per_step": max_over_ranks(start.elapsed_time(stop) / K, world, dev),
+            "t_quant": sum(e[0].elapsed_time(e[1]) for e in ev) / K,
+            "t_conv": sum(e[1].elapsed_time(e[2]) for e in ev) / K}
+
+
+def fp4_summary(r, c, pk, world):
+    """The FP4 step's throughput and the rooflines of its two kernels.  The layer's
+    tensor instructions are FP4 (kind::mxf4), so its compute peak is the dense FP4
+    rate: the measured bf16 burst x 6 (nominal 13.5 / 2.25 PFLOP/s); its bytes are
+    half those of one code per byte."""
+    fp4_peak = 6.0 * pk["bf16_tflops"]
+    q_bytes = c.in_elems * 4 + c.in_elems // 2
+    conv_bytes = c.in_elems // 2 + c.out_elems // 2 + c.weight_elems // 2
+    conv_tops = c.int_ops / (r["t_conv"] / 1e3) / 1e12
+    quant_gbs = q_bytes / (r["t_quant"] / 1e3) / 1e9
+    conv_gbs = conv_bytes / (r["t_conv"] / 1e3) / 1e9
+    return {
+        "value": whole_job_rate(c.int_ops, world, r["ms_per_step"]) / 1e12, "unit": UNIT,
+        "ms_per_step": r["ms_per_step"],
+        "code_layout": "packed FP4 nibbles [N][C/32][H][W][16 B], two 2-bit codes per byte",
+        "dtype": "2-bit codes as FP4 e2m1 x e2m1 weights, block scales 2^-4 -> f32 (exact integer)",
+        "roofline_kernels": [
+            {"kernel": "pq_quantize_c16<FP4 nibbles>", "bound": "hbm", "achieved": quant_gbs, "peak": pk["hbm_gbs"],
+             "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"], "traffic": None, "algorithmic_bytes": q_bytes,
+             "avg_launch_ms": r["t_quant"], "peak_source": f"{pk['source']} HBM copy bandwidth"},
+            {"kernel": "pq_conv_tc_kernel<FP4>", "bound": "tensor", "achieved": conv_tops, "peak": fp4_peak,
+             "unit": "TFLOP/s", "frac": conv_tops / fp4_peak, "traffic": None, "algorithmic_ops": c.int_ops,
+             "algorithmic_bytes": conv_bytes, "avg_launch_ms": r["t_conv"], "hbm_frac": conv_gbs / pk["hbm_gbs"],
+             "peak_source": f"{pk['source']} bf16 burst x 6 (dense FP4, nominal 13.5 / 2.25 PFLOP/s)"}],
+        "gpu_launches": 2,
+    }
 
 
 # ---------------------------------------------------------------------------
@@ -550,6 +657,7 @@ def run_ours(args, rank, world, local_rank):
     torch.cuda.synchronize(dev)
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
+    fp4 = measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf, K, world)
     resnet = None if args.no_resnet else measure_resnet18(dev, world, args)
     layers = None if args.no_layers else measure_layer_configs(dev, args)
     clocks = sampler.stop()
@@ -623,6 +731,7 @@ def run_ours(args, rank, world, local_rank):
                 "d2h_bytes_per_step": int(np.prod(out_shape))},
         "gpu_launches": 2 * K,
     }
+    line["fp4_step"] = fp4_summary(fp4, c, pk, world)
     if resnet is not None:
         line["resnet18"] = resnet
     if layers is not None:

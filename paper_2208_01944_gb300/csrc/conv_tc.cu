@@ -523,17 +523,14 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
 }
 
 // Dispatch to the MMA role compiled for this layer's K steps per tap and
-// accumulators per tile.
+// accumulators per tile (and operand type: F4 for packed FP4 codes).
+template <bool F4>
 __device__ __forceinline__ void mma_role_dispatch(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t b_base,
                                                   uint32_t tmem_base, const uint32_t* tap_a16, int64_t it0, int64_t it1,
                                                   const WaitCtx& ctx) {
   const int ks = p.nch >> 1;  // one MMA takes 32 bytes of K: 32 FP8 or 64 FP4 channels
-  const bool f4 = p.codes_f4 != 0;
-#define PQ_MMA_CASE(K, M)                                                                                   \
-  if (ks == K && p.MT == M) {                                                                               \
-    if (f4) return mma_role<K, M, true>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1, ctx);        \
-    return mma_role<K, M, false>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1, ctx);              \
-  }
+#define PQ_MMA_CASE(K, M) \
+  if (ks == K && p.MT == M) return mma_role<K, M, F4>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1, ctx);
   PQ_MMA_CASE(1, 1) PQ_MMA_CASE(1, 2) PQ_MMA_CASE(1, 4)
   PQ_MMA_CASE(2, 1) PQ_MMA_CASE(2, 2) PQ_MMA_CASE(2, 4)
   PQ_MMA_CASE(3, 1) PQ_MMA_CASE(3, 2) PQ_MMA_CASE(3, 4)
@@ -750,6 +747,7 @@ __device__ __forceinline__ void epi_general16(const ConvParams& p, const EpiItem
 // wg + n_groups, ...  Each warp handles the 32 TMEM lanes (rows) it may access.
 // On the codes-only path the TMEM loads are double-buffered: the next unit's
 // load is in flight while the current one is computed and stored.
+template <bool F4>
 __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& bars, uint32_t tmem_base,
                                               uint8_t* stage_base, int first_warp, int n_groups, int64_t it0,
                                               int64_t it1, const WaitCtx& ctx) {
@@ -779,7 +777,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
     e.src_c0 = e.g * p.Cout_g + item.nb * p.Nblk;               // source channel of column 0
     e.dst_c0 = p.dst_group[e.g] * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
     e.tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2;
-    if (codes_only && p.codes_f4 && (p.Nblk & 31) == 0) {
+    if (F4 && codes_only && (p.Nblk & 31) == 0) {
       // FP4 nibbles, units of 32 columns: a lane's 32 codes are one whole 16-byte
       // row of a 32-channel block, so a unit costs one store instruction (the
       // epilogue's time goes mostly to store instructions, not bytes).
@@ -917,6 +915,10 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
 
 }  // namespace
 
+// One instance per operand type (F4: packed FP4 codes and block-scaled FP4 MMAs;
+// else one code per byte or packed 2-bit codes, FP8 MMAs), so that each carries
+// only its own MMA loops and epilogue paths (a smaller instruction footprint).
+template <bool F4>
 __global__ void __launch_bounds__(kConvThreads, 1)
     pq_conv_tc_kernel(const __grid_constant__ ConvParams p, const __grid_constant__ CUtensorMap tmA) {
   extern __shared__ uint8_t smem_raw[];
@@ -958,7 +960,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  if (p.codes_f4) {
+  if (F4) {
     // Block scale factors of the FP4 MMAs: 32 columns of every lane set to 2^-4
     // (UE8M0 byte 123); warps 2-5 cover the four lane quarters.
     if (warp >= kFirstLoadWarp && warp < kFirstLoadWarp + 4) {
@@ -985,7 +987,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     }
     __syncwarp();
   } else if (warp == 1) {
-    mma_role_dispatch(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1,
+    mma_role_dispatch<F4>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1,
                       WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_MMA});
     __syncwarp();
   } else if (warp < kFirstEpiWarp && !p.a_tma) {
@@ -998,7 +1000,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     // epilogue warpgroup.
     const bool third = p.a_tma && !p.a_unpack;
     const int first = third ? kFirstLoadWarp : kFirstEpiWarp;
-    epilogue_role(p, bars, tmem_base, gbase + p.smem_stage_off, first, third ? kEpiGroups + 1 : kEpiGroups, it0, it1,
+    epilogue_role<F4>(p, bars, tmem_base, gbase + p.smem_stage_off, first, third ? kEpiGroups + 1 : kEpiGroups, it0, it1,
                   WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_EPILOGUE});
   }
   tc_fence_before();
@@ -1010,16 +1012,22 @@ __global__ void __launch_bounds__(kConvThreads, 1)
 }
 
 int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream) {
-  static int attr_set_for_device[64] = {0};
+  static int attr_set_for_device[2][64] = {{0}};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return -1;
   const int need = static_cast<int>(p.smem_bytes) + 1024;
-  if (dev < 64 && attr_set_for_device[dev] < need) {
-    if (cudaFuncSetAttribute(pq_conv_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) != cudaSuccess)
-      return -1;
-    attr_set_for_device[dev] = kMaxSmem;
+  const int f4 = p.codes_f4 ? 1 : 0;
+  if (dev < 64 && attr_set_for_device[f4][dev] < need) {
+    const cudaError_t e =
+        f4 ? cudaFuncSetAttribute(pq_conv_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem)
+           : cudaFuncSetAttribute(pq_conv_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+    if (e != cudaSuccess) return -1;
+    attr_set_for_device[f4][dev] = kMaxSmem;
   }
-  pq_conv_tc_kernel<<<grid, kConvThreads, need, stream>>>(p, tma_a);
+  if (f4)
+    pq_conv_tc_kernel<true><<<grid, kConvThreads, need, stream>>>(p, tma_a);
+  else
+    pq_conv_tc_kernel<false><<<grid, kConvThreads, need, stream>>>(p, tma_a);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }
 

@@ -22,7 +22,11 @@ takes the following reading:
 Every step runs in the library's kernels; this module only owns buffers, derives
 per-layer multipliers through palquant_epilogue_scales and launches the calls on one
 stream, with no host synchronisation inside forward() (which can be captured in a
-CUDA graph).  Codes between layers use the channel-blocked layout (PQ_CODES_C16).
+CUDA graph).  Codes between layers are packed FP4 nibbles (PQ_CODES_C32F4, the
+block-scaled FP4 tensor-core path) when the codes have at most 2 bits and every
+per-group width is a multiple of 64, else one code per byte, channel-blocked
+(PQ_CODES_C16); code_format chooses explicitly.  A code tensor is held as
+[N, H, W, C] bytes, or [N, H, W, C/2] for FP4 nibbles.
 """
 from __future__ import annotations
 
@@ -38,11 +42,18 @@ def _out(n: int, k: int, s: int, p: int) -> int:
 
 class PalQuantResNet18:
     def __init__(self, params: dict, N: int, H: int = 224, W: int = 224, G: int = 2, widths=(64, 128, 256, 512),
-                 classes: int = 1000, bits: int = 2, device="cuda:0", stream: torch.cuda.Stream | None = None):
+                 classes: int = 1000, bits: int = 2, device="cuda:0", stream: torch.cuda.Stream | None = None,
+                 code_format: int | None = None):
         self.dev = torch.device(device)
         self.N, self.H, self.W, self.G, self.bits, self.classes = N, H, W, G, bits, classes
         self.stream = stream or torch.cuda.Stream(device=self.dev)
-        fmt = B.PQ_CODES_C16
+        if code_format is None:
+            f4_ok = bits <= 2 and all(w % 64 == 0 for w in widths)
+            code_format = B.PQ_CODES_C32F4 if f4_ok else B.PQ_CODES_C16
+        if code_format not in (B.PQ_CODES_C16, B.PQ_CODES_C32F4):
+            raise ValueError("code_format must be PQ_CODES_C16 or PQ_CODES_C32F4")
+        self.fmt = fmt = code_format
+        per_byte = 2 if fmt == B.PQ_CODES_C32F4 else 1  # codes per byte
         f32 = dict(dtype=torch.float32, device=self.dev)
         u8 = dict(dtype=torch.uint8, device=self.dev)
         self.params = params
@@ -54,7 +65,7 @@ class PalQuantResNet18:
         self.w_fc = torch.from_numpy(np.ascontiguousarray(params["fc"])).to(self.dev)
         self.stem_out = torch.empty((N, self.Hs, self.Ws, C0), **f32)
         self.pool = torch.empty((N, self.Hp, self.Wp, C0), **f32)
-        self.in_codes = torch.empty((N, self.Hp, self.Wp, C0), **u8)
+        self.in_codes = torch.empty((N, self.Hp, self.Wp, C0 // per_byte), **u8)
         self.blocks = []
         Hc, Wc, cin = self.Hp, self.Wp, widths[0]
         for s, w in enumerate(widths):
@@ -69,9 +80,9 @@ class PalQuantResNet18:
                 if blk["down"]:
                     blk["dd"] = B.layer_desc(N, Hc, Wc, G, cin, w, 1, stride, 0, bits, bits, bits, 0, code_format=fmt)
                     blk["down_out"] = torch.empty((N, Ho, Wo, G * w), **f32)
-                blk["mid_codes"] = torch.empty((N, Ho, Wo, G * w), **u8)
+                blk["mid_codes"] = torch.empty((N, Ho, Wo, G * w // per_byte), **u8)
                 blk["out"] = torch.empty((N, Ho, Wo, G * w), **f32)
-                blk["out_codes"] = torch.empty((N, Ho, Wo, G * w), **u8)
+                blk["out_codes"] = torch.empty((N, Ho, Wo, G * w // per_byte), **u8)
                 for key, d in (("wp1", blk["d1"]), ("wp2", blk["d2"])) + ((("wpd", blk["dd"]),) if blk["down"] else ()):
                     blk[key] = torch.empty(B.palquant_packed_weight_bytes(d), **u8)
                 self.blocks.append(blk)
@@ -118,7 +129,7 @@ class PalQuantResNet18:
             self._scales(blk, st)
             if i == 0:
                 B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, G, self.C0 // G, bits,
-                                        self._inv(st[n + ".in"]), code_format=B.PQ_CODES_C16, stream=s)
+                                        self._inv(st[n + ".in"]), code_format=self.fmt, stream=s)
             q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]
             m_out1, _ = B.palquant_epilogue_scales(G, st[n + ".conv1.w"], st[n + ".in"], 1.0, None, self.no_shuffle)
             y1 = torch.empty((self.N, blk["Ho"], blk["Wo"], G * blk["w"]), dtype=torch.float32, device=self.dev)
@@ -208,7 +219,7 @@ class PalQuantResNet18:
         self._stem(x_dev)
         mark("stem conv + max pooling (fp32)")
         B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, self.G, self.C0 // self.G,
-                                self.bits, self.inv_in, code_format=B.PQ_CODES_C16, stream=s)
+                                self.bits, self.inv_in, code_format=self.fmt, stream=s)
         mark("input quantiser")
         for i, blk in enumerate(self.blocks):
             q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]

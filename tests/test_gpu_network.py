@@ -10,42 +10,46 @@ import pytest
 import torch
 
 import oracle.resnet as OR
-from layer_cases import c16_to_nhwc
+from layer_cases import from_format
 from paper_2208_01944_gb300 import synth
 
 pytestmark = pytest.mark.gpu
 
 
-def _codes(t):
+def _codes(t, fmt):
     N, H, W, C = t.shape
-    return c16_to_nhwc(t.cpu().numpy(), N, H, W, C)
+    return from_format(t.cpu().numpy(), fmt, N, H, W, C * (2 if fmt == 4 else 1))
 
 
 def _compare(net, r):
+    f = net.fmt
     assert np.array_equal(net.stem_out.cpu().numpy(), r["stem"]), "stem"
     assert np.array_equal(net.pool.cpu().numpy(), r["pool"]), "max pooling"
-    assert np.array_equal(_codes(net.in_codes), r[net.blocks[0]["name"] + ".in_codes"]), "input codes"
+    assert np.array_equal(_codes(net.in_codes, f), r[net.blocks[0]["name"] + ".in_codes"]), "input codes"
     for i, blk in enumerate(net.blocks):
         n = blk["name"]
-        assert np.array_equal(_codes(blk["mid_codes"]), r[n + ".mid_codes"]), n + " conv1 codes"
+        assert np.array_equal(_codes(blk["mid_codes"], f), r[n + ".mid_codes"]), n + " conv1 codes"
         if blk["down"]:
             assert np.array_equal(blk["down_out"].cpu().numpy(), r[n + ".down"]), n + " downsample"
         assert np.array_equal(blk["out"].cpu().numpy(), r[n + ".out"]), n + " block output"
         if i + 1 < len(net.blocks):
-            assert np.array_equal(_codes(blk["out_codes"]), r[n + ".out_codes"]), n + " next-block codes"
+            assert np.array_equal(_codes(blk["out_codes"], f), r[n + ".out_codes"]), n + " next-block codes"
     assert np.array_equal(net.avg.cpu().numpy(), r["avg"]), "average pooling"
     assert np.array_equal(net.logits.cpu().numpy(), r["logits"]), "logits"
 
 
-@pytest.mark.parametrize("N,H,widths,classes,seed", [(2, 32, (32, 32, 32, 32), 10, 1),
-                                                     (3, 64, (32, 64, 32, 64), 16, 2)])
-def test_small_network_matches_oracle(N, H, widths, classes, seed):
+@pytest.mark.parametrize("N,H,widths,classes,seed,fmt", [(2, 32, (32, 32, 32, 32), 10, 1, 2),
+                                                         (3, 64, (32, 64, 32, 64), 16, 2, 2),
+                                                         (2, 48, (64, 64, 128, 64), 12, 4, 4),   # FP4 codes
+                                                         (2, 48, (64, 64, 128, 64), 12, 4, 2)])
+def test_small_network_matches_oracle(N, H, widths, classes, seed, fmt):
     from paper_2208_01944_gb300.resnet18 import PalQuantResNet18
 
     x, params = synth.resnet18_inputs(N, H, H, 2, widths, classes, seed=seed)
     steps = OR.calibrate(x, params, 2, 2)
     r = OR.forward(x, params, 2, 2, steps)
-    net = PalQuantResNet18(params, N, H, H, 2, widths, classes, 2)
+    net = PalQuantResNet18(params, N, H, H, 2, widths, classes, 2, code_format=fmt)
+    assert net.fmt == fmt
     net.set_steps(steps)
     xd = torch.from_numpy(x).cuda()
     net.forward(xd)
@@ -64,19 +68,22 @@ def test_resnet18_224_matches_oracle():
     x, params = synth.resnet18_inputs(1, seed=0)
     steps = OR.calibrate(x, params, 2, 2)
     r = OR.forward(x, params, 2, 2, steps)
-    net = PalQuantResNet18(params, 1)
-    net.set_steps(steps)
     xd = torch.from_numpy(x).cuda()
-    net.forward(xd)
-    net.stream.synchronize()
-    assert B.palquant_sync_check() == B.PQ_OK
-    _compare(net, r)
-    net.logits.zero_()
-    net.capture(xd)
-    net.replay()
-    net.stream.synchronize()
-    assert B.palquant_sync_check() == B.PQ_OK
-    assert np.array_equal(net.logits.cpu().numpy(), r["logits"])
+    for fmt in (B.PQ_CODES_C32F4, B.PQ_CODES_C16):  # the default (FP4 nibbles), and one code per byte
+        net = PalQuantResNet18(params, 1, code_format=None if fmt == B.PQ_CODES_C32F4 else fmt)
+        assert net.fmt == fmt
+        net.set_steps(steps)
+        net.forward(xd)
+        net.stream.synchronize()
+        assert B.palquant_sync_check() == B.PQ_OK
+        _compare(net, r)
+        net.logits.zero_()
+        net.capture(xd)
+        net.replay()
+        net.stream.synchronize()
+        assert B.palquant_sync_check() == B.PQ_OK
+        assert np.array_equal(net.logits.cpu().numpy(), r["logits"])
+        del net
 
 
 def test_device_calibration_close_to_oracle():
