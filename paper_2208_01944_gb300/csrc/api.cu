@@ -353,6 +353,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.KC = KC;
   p.nch = KC / (16 * cpb);
   p.nch_magic = static_cast<uint32_t>(((1ull << 32) + p.nch - 1) / p.nch);
+  p.wh_magic = p.Wh > 0 ? static_cast<uint32_t>(((1ull << 32) + p.Wh - 1) / p.Wh) : 0u;
   p.H = d->H;
   p.W = d->W;
   p.stride = d->stride;

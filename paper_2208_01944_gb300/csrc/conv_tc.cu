@@ -588,7 +588,7 @@ __device__ __forceinline__ int epi_pos(const ConvParams& p, const EpiItem& e, in
     valid = m < p.flat_box && pos < p.img_pix;
     return pos;
   }
-  const int r = m / p.Wh;
+  const int r = static_cast<int>(__umulhi(static_cast<uint32_t>(m), p.wh_magic));  // m / Wh
   const int c = m - r * p.Wh;
   const int oh = e.oh0 + r;
   valid = (r < p.Ht) && (c < p.Wo) && (oh < p.Ho);
@@ -761,8 +761,20 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
   const int n_units = p.MT * nchunks;
   const float qmax_f = static_cast<float>(p.qmax_out);
   const bool codes_only = p.shortcut == nullptr && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle;
+  // The group's multipliers and destination stay in registers while consecutive
+  // items share the group (items run group by group); a dynamically indexed
+  // kernel-parameter array costs a long-latency constant load.
+  int cur_g = -1, dst_g = 0;
+  float g_m_out512 = 0.0f, g_m_req512 = 0.0f, g_m_req = 0.0f;
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1; ++it, item_next(p, item)) {
+    if (item.g != cur_g) {
+      cur_g = item.g;
+      g_m_out512 = p.m_out512[cur_g];
+      g_m_req512 = p.m_req512[cur_g];
+      g_m_req = p.m_req[cur_g];
+      dst_g = p.dst_group[cur_g];
+    }
     if (!warp_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
     tc_fence_after();
     EpiItem e;
@@ -771,11 +783,11 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
     e.n = item.n;
     e.rb = item.rb;
     e.oh0 = item.oh0(p.Ht);
-    e.m_out512 = p.m_out512[e.g];
-    e.m_req512 = p.m_req512[e.g];
-    e.m_req = p.m_req[e.g];
-    e.src_c0 = e.g * p.Cout_g + item.nb * p.Nblk;               // source channel of column 0
-    e.dst_c0 = p.dst_group[e.g] * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
+    e.m_out512 = g_m_out512;
+    e.m_req512 = g_m_req512;
+    e.m_req = g_m_req;
+    e.src_c0 = e.g * p.Cout_g + item.nb * p.Nblk;     // source channel of column 0
+    e.dst_c0 = dst_g * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
     e.tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2;
     if (F4 && codes_only && (p.Nblk & 31) == 0) {
       // FP4 nibbles, units of 32 columns: a lane's 32 codes are one whole 16-byte

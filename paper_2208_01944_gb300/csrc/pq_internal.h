@@ -66,6 +66,7 @@ struct ConvParams {
   int64_t ld_img, ld_row, ld_pix, ld_chunk, ld_c0_mul;
   int phase_a[kMaxPhases], phase_b[kMaxPhases];  // stride phase (row, column) of each plane set
   uint32_t nch_magic;     // ceil(2^32 / nch): e / nch = umulhi(e, nch_magic) for small e
+  uint32_t wh_magic;      // ceil(2^32 / Wh) (rows mode): m / Wh = umulhi(m, wh_magic) for m < 2^24
   int tiles_per_img;      // rows mode
   int64_t tiles;          // tiles per (group, n-block) unit
   int64_t items;          // tiles * G * NB
