@@ -196,21 +196,32 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // rows of pitch Wh into them.
   //
   // Choice of MT: a work item costs a fixed overhead (waits, commits, the
-  // epilogue's per-item set-up) plus, per 128-row accumulator, the larger of its
-  // MMA time and its epilogue time, so few large items beat many small ones
-  // even at some cost in padded rows.  Model (per SM): an M=128, K=32 FP8 MMA
-  // (or K=64 FP4 MMA, the same 32 bytes of K) takes max(32 + N/4, N/2) cycles
-  // (shared-memory operand reads at 128 B per cycle, tensor rate), the epilogue
-  // about 0.07 ns per accumulator value and an item 500 ns of overhead.
-  // Double-buffered accumulators come first.
+  // epilogue's per-item set-up) plus the larger of its MMA time and its
+  // epilogue time, so few large items beat many small ones even at some cost in
+  // padded rows.  Model (per SM, measured): an M=128, K=32 FP8 MMA (or K=64 FP4
+  // MMA, the same 32 bytes of K) takes max(32 + N/4, N/2) cycles (shared-memory
+  // operand reads at 128 B per cycle, tensor rate); the epilogue splits a tile
+  // into units of 16 accumulator columns (32 for FP4 codes) x 128 rows, each
+  // taking one warpgroup about 430 ns (550 ns for a 32-column FP4 unit), and its
+  // warpgroups (three when TMA loads the operand, else two) take the units in
+  // turn, so an uneven split costs a whole unit; an item costs 500 ns of
+  // overhead; weights too large to stay in shared memory are streamed again for
+  // every item, from L2 at about 40 B/ns per SM when all SMs stream (config 3,
+  // b=2, G=4: 147 KB per item).  Double-buffered accumulators come first.
   const double ns_per_clk = 1.0 / 1.9;
   const double mma_ns = std::max(32.0 + p.Npow2 / 4.0, p.Npow2 / 2.0) * ns_per_clk;
-  const double slot_ns =
-      std::max(static_cast<double>(p.taps) * (d->Cin_g / (32 * cpb)) * mma_ns, 128.0 * p.Npow2 * 0.07);
+  const double mma_acc_ns = static_cast<double>(p.taps) * (d->Cin_g / (32 * cpb)) * mma_ns;  // one accumulator
+  const bool tma_operand = c16 && d->stride == 1 && (flat || Wh <= 128);
+  const int epi_groups = tma_operand ? pq::kEpiGroups + 1 : pq::kEpiGroups;
+  const int unit_cols = (f4 && p.Nblk % 32 == 0) ? 32 : 16;
+  const int units_per_acc = p.Nblk / unit_cols;
+  const double unit_ns = unit_cols == 32 ? 550.0 : 430.0;
+  const double w_unit_bytes = static_cast<double>(p.taps) * d->Cin_g * p.Nblk / cpb;
+  const double w_stream_ns = w_unit_bytes > 112.0 * 1024.0 ? w_unit_bytes / 40.0 : 0.0;  // per item
   const int tmem_avail = f4 ? 512 - 32 : 512;  // FP4: 32 columns hold the scale factors
   int best_mt = 0, best_ht = 0, best_tpi = 0, best_acc = 0;
   double best_cost = 0.0;
-  for (int MT : {1, 2, 4}) {
+  for (int MT : {1, 2, 3, 4}) {
     if (flat && (MT > 2 || (c16 && MT > 1))) continue;
     int acc_stages = (2 * MT * p.Npow2 <= tmem_avail) ? 2 : ((MT * p.Npow2 <= tmem_avail) ? 1 : 0);
     if (acc_stages == 0) continue;
@@ -223,7 +234,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
       tpi = (Ho + ht_max - 1) / ht_max;
       ht = (Ho + tpi - 1) / tpi;
     }
-    const double cost = static_cast<double>(tpi) * (500.0 + MT * slot_ns);
+    const int units = MT * units_per_acc;
+    const double epi_ns = ((units + epi_groups - 1) / epi_groups) * unit_ns;
+    const double mma_side = std::max(MT * mma_acc_ns, w_stream_ns);
+    const double cost = static_cast<double>(tpi) * (500.0 + std::max(mma_side, epi_ns));
     const bool better = best_mt == 0 || acc_stages > best_acc || (acc_stages == best_acc && cost < best_cost * 0.98);
     if (better) {
       best_mt = MT;

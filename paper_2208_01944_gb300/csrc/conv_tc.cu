@@ -467,6 +467,9 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
             if constexpr (MT == 4) {
               tc_mma4_f4_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u),
                               a_hi | (a_lo + 256u), a_hi | (a_lo + 384u), bdesc, idesc, sfa, sfb, acc);
+            } else if constexpr (MT == 3) {
+              tc_mma3_f4_warp(d0, d0 + npow2, d0 + 2 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u), a_hi | (a_lo + 256u),
+                              bdesc, idesc, sfa, sfb, acc);
             } else if constexpr (MT == 2) {
               tc_mma2_f4_warp(d0, d0 + npow2, a_hi | a_lo, a_hi | (a_lo + 128u), bdesc, idesc, sfa, sfb, acc);
             } else {
@@ -475,6 +478,9 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
           } else if constexpr (MT == 4) {
             tc_mma4_e4m3_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u),
                               a_hi | (a_lo + 256u), a_hi | (a_lo + 384u), bdesc, idesc, acc);
+          } else if constexpr (MT == 3) {
+            tc_mma3_e4m3_warp(d0, d0 + npow2, d0 + 2 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u), a_hi | (a_lo + 256u),
+                              bdesc, idesc, acc);
           } else if constexpr (MT == 2) {
             tc_mma2_e4m3_warp(d0, d0 + npow2, a_hi | a_lo, a_hi | (a_lo + 128u), bdesc, idesc, acc);
           } else {
@@ -531,11 +537,11 @@ __device__ __forceinline__ void mma_role_dispatch(const ConvParams& p, const Bar
   const int ks = p.nch >> 1;  // one MMA takes 32 bytes of K: 32 FP8 or 64 FP4 channels
 #define PQ_MMA_CASE(K, M) \
   if (ks == K && p.MT == M) return mma_role<K, M, F4>(p, bars, a_base, b_base, tmem_base, tap_a16, it0, it1, ctx);
-  PQ_MMA_CASE(1, 1) PQ_MMA_CASE(1, 2) PQ_MMA_CASE(1, 4)
-  PQ_MMA_CASE(2, 1) PQ_MMA_CASE(2, 2) PQ_MMA_CASE(2, 4)
-  PQ_MMA_CASE(3, 1) PQ_MMA_CASE(3, 2) PQ_MMA_CASE(3, 4)
-  PQ_MMA_CASE(4, 1) PQ_MMA_CASE(4, 2) PQ_MMA_CASE(4, 4)
-  PQ_MMA_CASE(8, 1) PQ_MMA_CASE(8, 2) PQ_MMA_CASE(8, 4)
+  PQ_MMA_CASE(1, 1) PQ_MMA_CASE(1, 2) PQ_MMA_CASE(1, 3) PQ_MMA_CASE(1, 4)
+  PQ_MMA_CASE(2, 1) PQ_MMA_CASE(2, 2) PQ_MMA_CASE(2, 3) PQ_MMA_CASE(2, 4)
+  PQ_MMA_CASE(3, 1) PQ_MMA_CASE(3, 2) PQ_MMA_CASE(3, 3) PQ_MMA_CASE(3, 4)
+  PQ_MMA_CASE(4, 1) PQ_MMA_CASE(4, 2) PQ_MMA_CASE(4, 3) PQ_MMA_CASE(4, 4)
+  PQ_MMA_CASE(8, 1) PQ_MMA_CASE(8, 2) PQ_MMA_CASE(8, 3) PQ_MMA_CASE(8, 4)
 #undef PQ_MMA_CASE
   // The planner only produces the shapes above; anything else is a planner bug.
   atomicOr(ctx.err, PQ_ERR_TIMEOUT | PQ_ERR_MMA);

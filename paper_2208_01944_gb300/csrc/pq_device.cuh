@@ -266,6 +266,17 @@ __device__ __forceinline__ void tc_mma2_e4m3_warp(uint32_t d0, uint32_t d1, uint
       : "memory");
 }
 
+__device__ __forceinline__ void tc_mma3_e4m3_warp(uint32_t d0, uint32_t d1, uint32_t d2, uint64_t a0, uint64_t a1,
+                                                  uint64_t a2, uint64_t b_desc, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p, e;\nelect.sync _|e, 0xffffffff;\nsetp.ne.b32 p, %8, 0;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%0], %3, %6, %7, p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%1], %4, %6, %7, p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::f8f6f4 [%2], %5, %6, %7, p;\n}" ::"r"(d0),
+      "r"(d1), "r"(d2), "l"(a0), "l"(a1), "l"(a2), "l"(b_desc), "r"(idesc), "r"(accumulate)
+      : "memory");
+}
+
 __device__ __forceinline__ void tc_mma4_e4m3_warp(uint32_t d0, uint32_t d1, uint32_t d2, uint32_t d3, uint64_t a0,
                                                   uint64_t a1, uint64_t a2, uint64_t a3, uint64_t b_desc,
                                                   uint32_t idesc, uint32_t accumulate) {
@@ -308,6 +319,18 @@ __device__ __forceinline__ void tc_mma2_f4_warp(uint32_t d0, uint32_t d1, uint64
       "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], %2, %4, %5, [%6], [%7], p;\n"
       "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%1], %3, %4, %5, [%6], [%7], p;\n}" ::"r"(d0),
       "r"(d1), "l"(a0), "l"(a1), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
+      : "memory");
+}
+
+__device__ __forceinline__ void tc_mma3_f4_warp(uint32_t d0, uint32_t d1, uint32_t d2, uint64_t a0, uint64_t a1,
+                                                uint64_t a2, uint64_t b_desc, uint32_t idesc, uint32_t sfa, uint32_t sfb,
+                                                uint32_t accumulate) {
+  asm volatile(
+      "{\n.reg .pred p, e;\nelect.sync _|e, 0xffffffff;\nsetp.ne.b32 p, %10, 0;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%0], %3, %6, %7, [%8], [%9], p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%1], %4, %6, %7, [%8], [%9], p;\n"
+      "@e tcgen05.mma.cta_group::1.kind::mxf4.block_scale.scale_vec::2X [%2], %5, %6, %7, [%8], [%9], p;\n}" ::"r"(d0),
+      "r"(d1), "r"(d2), "l"(a0), "l"(a1), "l"(a2), "l"(b_desc), "r"(idesc), "r"(sfa), "r"(sfb), "r"(accumulate)
       : "memory");
 }
 

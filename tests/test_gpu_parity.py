@@ -91,6 +91,9 @@ SMALL_CASES = [
     Case(1, 9, 11, 2, 32, 64, 5, 1, 2, seed=13),                      # 5x5 kernel
     Case(2, 6, 6, 2, 32, 32, 3, 1, 1, bits=3, bits_out=4, relu=False, kind=1, shift=-1, seed=14),
     Case(1, 16, 16, 4, 64, 64, 3, 2, 0, seed=15),                     # stride 2 without padding
+    Case(2, 36, 40, 2, 64, 64, 3, 1, 1, shortcut=True, seed=16),      # three accumulators per tile (c16)
+    Case(1, 30, 20, 2, 64, 64, 3, 1, 1, seed=17),                     # three accumulators, ragged last tile
+    Case(1, 40, 30, 2, 64, 64, 3, 2, 1, seed=18),                     # three accumulators, stride 2
 ]
 
 
@@ -374,6 +377,9 @@ F4_CASES = [
     Case(1, 16, 16, 4, 64, 64, 3, 2, 0, seed=93),                     # stride 2 without padding
     Case(2, 8, 8, 2, 256, 256, 3, 1, 1, seed=94),                     # 256 channels per group
     Case(1, 10, 10, 2, 192, 64, 3, 1, 1, seed=95),                    # three K steps per tap
+    Case(2, 36, 40, 2, 64, 64, 3, 1, 1, shortcut=True, seed=96),      # three accumulators per tile
+    Case(1, 40, 30, 2, 64, 64, 3, 2, 1, seed=97),                     # three accumulators, stride 2
+    Case(2, 20, 42, 2, 128, 64, 3, 1, 1, seed=98),                    # three accumulators, two K steps
 ]
 
 
