@@ -222,7 +222,9 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   int best_mt = 0, best_ht = 0, best_tpi = 0, best_acc = 0;
   double best_cost = 0.0;
   for (int MT : {1, 2, 3, 4}) {
-    if (flat && (MT > 2 || (c16 && MT > 1))) continue;
+    // flat tiles: up to two accumulators (by TMA, one 128-position box each); the
+    // packed 2-bit path stages one box
+    if (flat && (MT > 2 || (p2 && MT > 1))) continue;
     int acc_stages = (2 * MT * p.Npow2 <= tmem_avail) ? 2 : ((MT * p.Npow2 <= tmem_avail) ? 1 : 0);
     if (acc_stages == 0) continue;
     int ht = 0, tpi = 0;
@@ -285,6 +287,12 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const uint32_t budget = pq::kMaxSmem - 1024;
   auto a_stage_bytes = [&](int KC, uint32_t* phase_bytes, uint32_t* lbo) -> uint32_t {
     const int nch = KC / (16 * cpb);
+    if (flat && c16 && !p2) {
+      // TMA: per accumulator a region of nch planes of 128 positions (one box)
+      *lbo = 128u * 16u;
+      *phase_bytes = static_cast<uint32_t>(p.MT) * nch * 2048u;
+      return round_up(*phase_bytes, 1024);
+    }
     if (flat) {
       const uint32_t plane = static_cast<uint32_t>(p.flat_box) * 16u;
       *phase_bytes = round_up(static_cast<uint64_t>(nch) * plane, 128);
@@ -383,7 +391,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.pk_stage_bytes = pk_stage_bytes(KC);
   // The A operand comes by TMA when every plane row is one contiguous run in
   // global memory: channel-blocked codes, stride 1, rows of at most 128 positions.
-  p.a_tma = (p2 || (c16 && d->stride == 1 && (flat ? p.flat_box == 128 : p.Wd <= 128))) ? 1 : 0;
+  p.a_tma = (p2 || (c16 && d->stride == 1 && (flat ? p.flat_box <= 256 : p.Wd <= 128))) ? 1 : 0;
+  p.a_mt16 = (flat && c16 && !p2) ? static_cast<uint32_t>(p.nch) * 128u : 128u;
   p.a_tx_bytes = p2 ? static_cast<uint32_t>(p.nch) * pk_box_w * (flat ? 1 : p.Hd) * 4u
                  : flat ? static_cast<uint32_t>(p.nch) * p.flat_box * 16u
                         : static_cast<uint32_t>(p.nph) * p.nch * p.Hd * p.Wd * 16u;
@@ -512,7 +521,7 @@ bool encode_c16_map(const pq_layer_desc* d, const ConvParams& p, const void* q_d
   if (p.mode == pq::kModeFlat) {
     cuuint64_t dims[3] = {2 * H * W, C16, static_cast<cuuint64_t>(d->N)};
     cuuint64_t strides[2] = {H * W * 16, C16 * H * W * 16};
-    cuuint32_t box[3] = {2u * static_cast<cuuint32_t>(p.flat_box), static_cast<cuuint32_t>(p.nch), 1};
+    cuuint32_t box[3] = {2u * 128u, static_cast<cuuint32_t>(p.nch), 1};  // one accumulator's 128 positions
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT64, 3, const_cast<void*>(q_dev), dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;

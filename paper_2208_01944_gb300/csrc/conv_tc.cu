@@ -181,10 +181,14 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
         mbar_arrive_expect_tx(full, p.a_tx_bytes);
         const uint32_t dst = a_base + ra.stage * p.a_stage_bytes;
         const int chi = (p.src_group[item.g] * p.Cin_g + kb * p.KC) >> p.chunk_shift;
-        if (flat)
-          tma_load_3d(dst, tmA, 2 * item.rb * p.flat_box, chi, item.n, full);
-        else
+        if (flat) {
+          // one box of 128 positions per accumulator, each into its own region
+          for (int mt = 0; mt < p.MT; ++mt)
+            tma_load_3d(dst + static_cast<uint32_t>(mt) * (p.a_mt16 << 4), tmA, 2 * (item.rb * p.flat_box + mt * 128),
+                        chi, item.n, full);
+        } else {
           tma_load_4d(dst, tmA, 2 * p.w_coord, item.oh0(p.Ht) + p.h_off, chi, item.n, full);
+        }
         ra.advance();
         ++a_issued;
       }
@@ -426,6 +430,7 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
   const uint32_t a_lo0 = static_cast<uint32_t>(a_desc0), b_lo0 = static_cast<uint32_t>(b_desc0);
   const uint32_t a_ks16 = (2u * p.lbo_a) >> 4, b_ks16 = (2u * p.lbo_b) >> 4;  // one K step (32 bytes of K)
   const uint32_t a_stage16 = p.a_stage_bytes >> 4, b_slice16 = p.b_slice_bytes >> 4;
+  const uint32_t amt = p.a_mt16;  // A operand of accumulator mt starts mt * amt 16-byte units in
   const int taps = p.taps, n_kb = p.n_kb;
   const uint32_t npow2 = static_cast<uint32_t>(p.Npow2);
   const bool resident = p.b_resident != 0;
@@ -465,24 +470,24 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
           const uint32_t acc = ks == 0 ? acc0 : 1u;
           if constexpr (F4) {
             if constexpr (MT == 4) {
-              tc_mma4_f4_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u),
-                              a_hi | (a_lo + 256u), a_hi | (a_lo + 384u), bdesc, idesc, sfa, sfb, acc);
+              tc_mma4_f4_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + amt),
+                              a_hi | (a_lo + 2u * amt), a_hi | (a_lo + 3u * amt), bdesc, idesc, sfa, sfb, acc);
             } else if constexpr (MT == 3) {
-              tc_mma3_f4_warp(d0, d0 + npow2, d0 + 2 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u), a_hi | (a_lo + 256u),
+              tc_mma3_f4_warp(d0, d0 + npow2, d0 + 2 * npow2, a_hi | a_lo, a_hi | (a_lo + amt), a_hi | (a_lo + 2u * amt),
                               bdesc, idesc, sfa, sfb, acc);
             } else if constexpr (MT == 2) {
-              tc_mma2_f4_warp(d0, d0 + npow2, a_hi | a_lo, a_hi | (a_lo + 128u), bdesc, idesc, sfa, sfb, acc);
+              tc_mma2_f4_warp(d0, d0 + npow2, a_hi | a_lo, a_hi | (a_lo + amt), bdesc, idesc, sfa, sfb, acc);
             } else {
               tc_mma_f4_warp(d0, a_hi | a_lo, bdesc, idesc, sfa, sfb, acc);
             }
           } else if constexpr (MT == 4) {
-            tc_mma4_e4m3_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u),
-                              a_hi | (a_lo + 256u), a_hi | (a_lo + 384u), bdesc, idesc, acc);
+            tc_mma4_e4m3_warp(d0, d0 + npow2, d0 + 2 * npow2, d0 + 3 * npow2, a_hi | a_lo, a_hi | (a_lo + amt),
+                              a_hi | (a_lo + 2u * amt), a_hi | (a_lo + 3u * amt), bdesc, idesc, acc);
           } else if constexpr (MT == 3) {
-            tc_mma3_e4m3_warp(d0, d0 + npow2, d0 + 2 * npow2, a_hi | a_lo, a_hi | (a_lo + 128u), a_hi | (a_lo + 256u),
+            tc_mma3_e4m3_warp(d0, d0 + npow2, d0 + 2 * npow2, a_hi | a_lo, a_hi | (a_lo + amt), a_hi | (a_lo + 2u * amt),
                               bdesc, idesc, acc);
           } else if constexpr (MT == 2) {
-            tc_mma2_e4m3_warp(d0, d0 + npow2, a_hi | a_lo, a_hi | (a_lo + 128u), bdesc, idesc, acc);
+            tc_mma2_e4m3_warp(d0, d0 + npow2, a_hi | a_lo, a_hi | (a_lo + amt), bdesc, idesc, acc);
           } else {
             tc_mma_e4m3_warp(d0, a_hi | a_lo, bdesc, idesc, acc);
           }

@@ -79,6 +79,8 @@ struct ConvParams {
   int tap_off[kMaxTaps];  // position offset of each tap in the plane
   uint32_t tap_a16[kMaxTaps];  // stage-relative start of each tap's A operand, in 16-byte units
   uint32_t lbo_a;         // byte stride between 16-byte K chunks of the A planes
+  uint32_t a_mt16;        // 16-byte units between the A operands of consecutive accumulators:
+                          // 128 (one plane of positions), or nch * 128 (flat TMA: a box region each)
   uint32_t a_phase_bytes, a_stage_bytes;
   int a_stages;
   int b_resident;         // 1: the whole unit's weights stay in shared memory

@@ -94,6 +94,8 @@ SMALL_CASES = [
     Case(2, 36, 40, 2, 64, 64, 3, 1, 1, shortcut=True, seed=16),      # three accumulators per tile (c16)
     Case(1, 30, 20, 2, 64, 64, 3, 1, 1, seed=17),                     # three accumulators, ragged last tile
     Case(1, 40, 30, 2, 64, 64, 3, 2, 1, seed=18),                     # three accumulators, stride 2
+    Case(2, 20, 20, 2, 64, 64, 1, 1, 0, seed=19),                     # flat, two boxes per tile, ragged
+    Case(2, 17, 17, 2, 64, 64, 1, 1, 0, shortcut=True, seed=20),      # flat, second box wholly past the image
 ]
 
 
@@ -243,6 +245,7 @@ CODES_ONLY = [
     Case(1, 12, 12, 2, 128, 256, 3, 1, 1, bits=4, seed=41),
     Case(2, 7, 9, 4, 96, 96, 1, 1, 0, seed=42),
     Case(3, 9, 17, 4, 64, 64, 3, 2, 1, seed=43),
+    Case(2, 17, 17, 4, 96, 96, 1, 1, 0, seed=45),                     # flat, two boxes per tile
 ]
 
 
@@ -380,6 +383,8 @@ F4_CASES = [
     Case(2, 36, 40, 2, 64, 64, 3, 1, 1, shortcut=True, seed=96),      # three accumulators per tile
     Case(1, 40, 30, 2, 64, 64, 3, 2, 1, seed=97),                     # three accumulators, stride 2
     Case(2, 20, 42, 2, 128, 64, 3, 1, 1, seed=98),                    # three accumulators, two K steps
+    Case(2, 20, 20, 2, 64, 64, 1, 1, 0, seed=99),                     # flat, two boxes per tile
+    Case(2, 17, 17, 2, 128, 64, 1, 1, 0, seed=100),                   # flat, second box wholly past the image
 ]
 
 
