@@ -587,6 +587,7 @@ __device__ __forceinline__ int requant_code(float t, float qmax_f, int qmax) {
 struct EpiItem {
   uint32_t tbase;        // TMEM address of accumulator 0, this warp's lanes
   float m_out512, m_req512, m_req;
+  float m_sat;           // m_req512 / 2^b_out (codes-only conversion)
   int g, src_c0, dst_c0;
   int n, rb, oh0;
   int nb;
@@ -606,27 +607,30 @@ __device__ __forceinline__ int epi_pos(const ConvParams& p, const EpiItem& e, in
   return oh * p.Wo + c;
 }
 
-// Codes-only unit (the timed path): t = acc * m_req = raw * (m_req * 2^9),
-// clamped to [0, Qp] in fp32 (NaN -> 0), then rounded half to even by adding
-// 1.5 * 2^23, which leaves the code in the sum's low byte.
-__device__ __forceinline__ uint4 epi_codes16(const uint32_t (&v)[16], float m_req512, float qmax_f) {
-  uint32_t bits[16];
+// Codes-only unit (the timed path): the codes clamp(rint(t), 0, Qp) of
+// t = acc * m_req = raw * (m_req * 2^9), Qp = 2^b - 1, as
+//   c = sat(raw * m_sat), m_sat = m_req * 2^9 / 2^b (a power-of-two scaling, so
+//       c = clamp(t, 0, 2^b) / 2^b exactly; NaN -> 0);
+//   r = c * 2^b + 1.5 * 2^23, one rounding half to even: the low 16 bits of r
+//       hold k = rint(clamp(t, 0, 2^b)), in [0, 2^b];
+//   code = min(k, Qp), two 16-bit halves per instruction.
+// Clamping to [0, 2^b] before rounding and to Qp after it equals clamping the
+// rounded value to [0, Qp] (integer bounds, monotone rounding).
+__device__ __forceinline__ uint4 epi_codes16(const uint32_t (&v)[16], float m_sat, float two_b, uint32_t qmax2) {
+  uint32_t h[8];
 #pragma unroll
   for (int j = 0; j < 16; j += 2) {
-    float t0, t1;
-    mul2_rn(__uint_as_float(v[j]), __uint_as_float(v[j + 1]), m_req512, t0, t1);
-    t0 = fminf(fmaxf(t0, 0.0f), qmax_f);
-    t1 = fminf(fmaxf(t1, 0.0f), qmax_f);
+    const float c0 = mul_sat(__uint_as_float(v[j]), m_sat);
+    const float c1 = mul_sat(__uint_as_float(v[j + 1]), m_sat);
     float r0, r1;
-    add2_rn(t0, t1, 12582912.0f, r0, r1);
-    bits[j] = __float_as_uint(r0);
-    bits[j + 1] = __float_as_uint(r1);
+    fma2_rn(c0, c1, two_b, 12582912.0f, r0, r1);
+    h[j >> 1] = __vimin_s16x2_relu(__byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x5410), qmax2);
   }
   uint4 w;
-  w.x = __byte_perm(__byte_perm(bits[0], bits[1], 0x0040), __byte_perm(bits[2], bits[3], 0x0040), 0x5410);
-  w.y = __byte_perm(__byte_perm(bits[4], bits[5], 0x0040), __byte_perm(bits[6], bits[7], 0x0040), 0x5410);
-  w.z = __byte_perm(__byte_perm(bits[8], bits[9], 0x0040), __byte_perm(bits[10], bits[11], 0x0040), 0x5410);
-  w.w = __byte_perm(__byte_perm(bits[12], bits[13], 0x0040), __byte_perm(bits[14], bits[15], 0x0040), 0x5410);
+  w.x = __byte_perm(h[0], h[1], 0x6420);
+  w.y = __byte_perm(h[2], h[3], 0x6420);
+  w.z = __byte_perm(h[4], h[5], 0x6420);
+  w.w = __byte_perm(h[6], h[7], 0x6420);
   return w;
 }
 
@@ -776,7 +780,10 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
   // items share the group (items run group by group); a dynamically indexed
   // kernel-parameter array costs a long-latency constant load.
   int cur_g = -1, dst_g = 0;
-  float g_m_out512 = 0.0f, g_m_req512 = 0.0f, g_m_req = 0.0f;
+  float g_m_out512 = 0.0f, g_m_req512 = 0.0f, g_m_req = 0.0f, g_m_sat = 0.0f;
+  const float two_b = static_cast<float>(p.qmax_out + 1);  // 2^b_out
+  const float inv_two_b = 1.0f / two_b;                     // exact: a power of two
+  const uint32_t qmax2 = static_cast<uint32_t>(p.qmax_out) * 0x00010001u;
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1; ++it, item_next(p, item)) {
     if (item.g != cur_g) {
@@ -784,6 +791,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
       g_m_out512 = p.m_out512[cur_g];
       g_m_req512 = p.m_req512[cur_g];
       g_m_req = p.m_req[cur_g];
+      g_m_sat = __fmul_rn(g_m_req512, inv_two_b);
       dst_g = p.dst_group[cur_g];
     }
     if (!warp_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
@@ -797,6 +805,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
     e.m_out512 = g_m_out512;
     e.m_req512 = g_m_req512;
     e.m_req = g_m_req;
+    e.m_sat = g_m_sat;
     e.src_c0 = e.g * p.Cout_g + item.nb * p.Nblk;     // source channel of column 0
     e.dst_c0 = dst_g * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
     e.tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2;
@@ -837,12 +846,12 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
       }
       while (c_mt < MT) {
         tmem_ld16(col(c_mt, c_b) + 16, vb);
-        const uint2 lo = pack4_word(epi_codes16(va, e.m_req512, qmax_f));
+        const uint2 lo = pack4_word(epi_codes16(va, e.m_sat, two_b, qmax2));
         tmem_wait_ld();
         int n_mt = c_mt, n_b = c_b;
         step(n_mt, n_b);
         if (n_mt < MT) tmem_ld16(col(n_mt, n_b), va);
-        const uint2 hi = pack4_word(epi_codes16(vb, e.m_req512, qmax_f));
+        const uint2 hi = pack4_word(epi_codes16(vb, e.m_sat, two_b, qmax2));
         tmem_wait_ld();  // before the store: a TMEM-load wait right after a store stalls on the store
         if (c_row) *reinterpret_cast<uint4*>(c_row + c_b * blk_bytes) = make_uint4(lo.x, lo.y, hi.x, hi.y);
         c_row = n_mt == c_mt ? c_row : row_ptr(n_mt);
@@ -887,35 +896,26 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
       uint32_t va[16], vb[16];
       int c_mt = 0, c_ch = wg - n_groups;
       step(c_mt, c_ch);
-      uint8_t* c_row = row_ptr(c_mt);
-      if (c_mt < MT) {
-        tmem_ld16(col(c_mt, c_ch), va);
-        tmem_wait_ld();
-      }
-      // Unrolled by two so both buffers stay in registers; the next unit's TMEM
-      // load is in flight while the current one is converted and stored.
+      // Units in pairs: both TMEM loads in flight together, one wait, then both
+      // conversions in one stretch of code (independent work the scheduler can
+      // interleave) and two stores.
       while (c_mt < MT) {
         int n_mt = c_mt, n_ch = c_ch;
         step(n_mt, n_ch);
-        if (n_mt < MT) tmem_ld16(col(n_mt, n_ch), vb);
-        {
-          const uint4 w = epi_codes16(va, e.m_req512, qmax_f);
-          tmem_wait_ld();  // before the store: a TMEM-load wait right after a store stalls on the store
-          if (c_row) store_codes16(c_row + coff(c_ch), w, pack);
-        }
-        if (n_mt >= MT) break;
-        uint8_t* n_row = n_mt == c_mt ? c_row : row_ptr(n_mt);
-        int m2 = n_mt, c2 = n_ch;
-        step(m2, c2);
-        if (m2 < MT) tmem_ld16(col(m2, c2), va);
-        {
-          const uint4 w = epi_codes16(vb, e.m_req512, qmax_f);
-          tmem_wait_ld();
-          if (n_row) store_codes16(n_row + coff(n_ch), w, pack);
-        }
-        c_row = m2 == n_mt ? n_row : row_ptr(m2);
-        c_mt = m2;
-        c_ch = c2;
+        const bool two = n_mt < MT;
+        tmem_ld16(col(c_mt, c_ch), va);
+        if (two) tmem_ld16(col(n_mt, n_ch), vb);
+        uint8_t* c_row = row_ptr(c_mt);
+        uint8_t* n_row = two ? (n_mt == c_mt ? c_row : row_ptr(n_mt)) : nullptr;
+        tmem_wait_ld();
+        const uint4 w0 = epi_codes16(va, e.m_sat, two_b, qmax2);
+        const uint4 w1 = epi_codes16(vb, e.m_sat, two_b, qmax2);
+        if (c_row) store_codes16(c_row + coff(c_ch), w0, pack);
+        if (n_row) store_codes16(n_row + coff(n_ch), w1, pack);
+        if (!two) break;
+        step(n_mt, n_ch);
+        c_mt = n_mt;
+        c_ch = n_ch;
       }
     } else {
       for (int u = wg; u < n_units; u += n_groups) {

@@ -179,6 +179,21 @@ __device__ __forceinline__ void add2_rn(float a, float b, float m, float& x, flo
       : "f"(a), "f"(b), "f"(m));
 }
 
+// x = fl(a * b) clamped to [0, 1] (saturation; NaN -> +0).
+__device__ __forceinline__ float mul_sat(float a, float b) {
+  float x;
+  asm("mul.rn.sat.f32 %0, %1, %2;" : "=f"(x) : "f"(a), "f"(b));
+  return x;
+}
+
+// (x, y) = (fl(a * m + c), fl(b * m + c)), each one rounding (packed fp32 FMA).
+__device__ __forceinline__ void fma2_rn(float a, float b, float m, float c, float& x, float& y) {
+  asm("{\n.reg .b64 s, t, u, r;\nmov.b64 s, {%2, %3};\nmov.b64 t, {%4, %4};\nmov.b64 u, {%5, %5};\n"
+      "fma.rn.f32x2 r, s, t, u;\nmov.b64 {%0, %1}, r;\n}"
+      : "=f"(x), "=f"(y)
+      : "f"(a), "f"(b), "f"(m), "f"(c));
+}
+
 // ------------------------------------------------------------- packed codes
 // Sixteen 2-bit codes (one per byte of w, each <= 3) packed into one 32-bit word,
 // code k at bits 2k: the product of a byte quadruple with 2^24 + 2^18 + 2^12 + 2^6

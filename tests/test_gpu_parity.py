@@ -257,19 +257,24 @@ def test_layer_codes_only_matches_oracle(B, c, fmt):
     assert_layer_parity(c, ref, got)
 
 
-@pytest.mark.parametrize("mult", [0.5, 0.25, 1.0 / 3.0])
-def test_requant_ties_round_half_even(B, mult):
-    """Multipliers that put many products exactly on .5: ties must round to even."""
-    c = Case(2, 10, 10, 2, 64, 64, 3, 1, 1, bits=4, seed=44)
+@pytest.mark.parametrize("fmt,bits", [(0, 4), (2, 4), (2, 1), (4, 2)], ids=["nhwc4", "c16_4", "c16_1", "fp4_2"])
+@pytest.mark.parametrize("mult", [0.5, 0.25, 1.0 / 3.0, 1e4, -0.5, 1e-3])
+def test_requant_ties_round_half_even(B, mult, fmt, bits):
+    """Multipliers that put many products exactly on .5 (ties must round to even),
+    that saturate every positive sum, that make every product negative, and that
+    round almost everything to 0; codes only, in every code format."""
+    c = Case(2, 10, 10, 2, 64, 64, 3, 1, 1, bits=bits if bits > 1 else 2, bits_out=bits, seed=44)
     ref = prepare(c)
-    m_req = np.full(c.G, mult, dtype=np.float32)
+    m_req = np.array([mult, mult * 0.75], dtype=np.float32)
     acc = oracle.group_conv(ref["q"], ref["wq"], c.stride, c.pad).reshape(-1, c.G * c.Cout)
-    _, _, q_ref = oracle.epilogue(acc, c.G, ref["m_out"], m_req, c.kind, c.shift, None, None, True, 4)
+    _, _, q_ref = oracle.epilogue(acc, c.G, ref["m_out"], m_req, c.kind, c.shift, None, None, True, bits)
     ref = dict(ref, m_req=m_req, q_ref=q_ref)
-    got = run_gpu(c, ref, outputs=("q",))
+    got = run_gpu(c, ref, outputs=("q",), fmt=fmt)
     assert np.array_equal(got["q_out"], q_ref)
     if mult == 0.5:
         assert np.any((acc % 2 == 1) & (acc > 0)), "the case must contain ties"
+    if mult == 1e4:
+        assert np.any(q_ref == (1 << bits) - 1) and np.any(acc > 0)
 
 
 # ------------------------------------ packed 2-bit channel-blocked codes (format 3)
