@@ -104,8 +104,10 @@ def source_sha(files):
 
 
 KERNEL_SOURCES = {
-    "pq_quantize_c16": ["quantize.cu", "pq_internal.h"],
+    "pq_quantize_c16": ["quantize.cu", "pq_device.cuh", "pq_internal.h"],
     "pq_conv_tc_kernel": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
+    "pq_quantize_c16<FP4 nibbles>": ["quantize.cu", "pq_device.cuh", "pq_internal.h"],
+    "pq_conv_tc_kernel<FP4>": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
 }
 
 
@@ -567,10 +569,12 @@ def fp4_summary(r, c, pk, world):
         "dtype": "2-bit codes as FP4 e2m1 x e2m1 weights, block scales 2^-4 -> f32 (exact integer)",
         "roofline_kernels": [
             {"kernel": "pq_quantize_c16<FP4 nibbles>", "bound": "hbm", "achieved": quant_gbs, "peak": pk["hbm_gbs"],
-             "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"], "traffic": None, "algorithmic_bytes": q_bytes,
+             "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"],
+             "traffic": dram_traffic("pq_quantize_c16<FP4 nibbles>"), "algorithmic_bytes": q_bytes,
              "avg_launch_ms": r["t_quant"], "peak_source": f"{pk['source']} HBM copy bandwidth"},
             {"kernel": "pq_conv_tc_kernel<FP4>", "bound": "tensor", "achieved": conv_tops, "peak": fp4_peak,
-             "unit": "TFLOP/s", "frac": conv_tops / fp4_peak, "traffic": None, "algorithmic_ops": c.int_ops,
+             "unit": "TFLOP/s", "frac": conv_tops / fp4_peak, "traffic": dram_traffic("pq_conv_tc_kernel<FP4>"),
+             "algorithmic_ops": c.int_ops,
              "algorithmic_bytes": conv_bytes, "avg_launch_ms": r["t_conv"], "hbm_frac": conv_gbs / pk["hbm_gbs"],
              "peak_source": f"{pk['source']} bf16 burst x 6 (dense FP4, nominal 13.5 / 2.25 PFLOP/s)"}],
         "gpu_launches": 2,
