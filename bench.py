@@ -47,6 +47,9 @@ def parse():
                     help="only run the fused layer of CONFIG (config0, config1, config3_0..4, config4) --reps times "
                          "on random codes (codes out), for profilers; prints nothing else")
     ap.add_argument("--reps", type=int, default=3)
+    ap.add_argument("--profile-stem", type=int, default=0, metavar="N",
+                    help="only run the network's fp32 7x7 stem convolution on N 224x224 images --reps times, "
+                         "for profilers; prints nothing else")
     ap.add_argument("--profile-format", default="c16", choices=["c16", "f4"],
                     help="code format of --profile-layer: one code per byte, or packed FP4 nibbles")
     ap.add_argument("--no-resnet", action="store_true", help="skip the ResNet-18-shaped network measurement")
@@ -82,6 +85,25 @@ def run_profile_layer(name: str, reps: int, fmt_name: str = "c16"):
     m = np.full(c.G, 0.01, np.float32)
     for _ in range(reps):
         B.palquant_layer_fused(q, wp, d, m, m, B.shuffle(c.shuffle_kind, c.shuffle_shift), None, None, None, qo)
+    st = B.palquant_sync_check()
+    assert st == B.PQ_OK, B.strerror(st)
+
+
+def run_profile_stem(N: int, reps: int):
+    """The network's stem alone (7x7 stride-2 pad-3 fp32 convolution 3 -> 128 channels
+    + ReLU) on N synthetic 224x224 images, for profiling."""
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300 import synth
+
+    dev = torch.device("cuda:0")
+    x, params = synth.resnet18_inputs(N, seed=0)
+    xd = torch.from_numpy(x).to(dev)
+    wd = torch.from_numpy(params["stem"]).to(dev)
+    y = torch.empty((N, 112, 112, wd.shape[0]), dtype=torch.float32, device=dev)
+    for _ in range(reps):
+        B.palquant_conv2d_f32(xd, wd, y, N, 224, 224, 3, wd.shape[0], 7, 2, 3, relu=True)
     st = B.palquant_sync_check()
     assert st == B.PQ_OK, B.strerror(st)
 
@@ -752,6 +774,9 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.profile_layer:
         run_profile_layer(args.profile_layer, args.reps, args.profile_format)
+        return
+    if args.profile_stem:
+        run_profile_stem(args.profile_stem, args.reps)
         return
     if args.impl == "reference":
         run_reference(args, rank, world)

@@ -154,9 +154,11 @@ __global__ void __launch_bounds__(256, 2) pq_stem7x7s2_kernel(const float* __res
   };
   int64_t t = blockIdx.x;
   if (t < n_tiles) load_tile(t, 0);
+  // transposed to [term][Cout]: consecutive threads write consecutive words
+  // (conflict-free) and gather from the [Cout][term] weights through L2
   for (int i = threadIdx.x; i < kStemTerms * Cout; i += blockDim.x) {
-    const int co = i / kStemTerms, r = i - co * kStemTerms;
-    ws[r * Cout + co] = w[i];
+    const int r = i / Cout, co = i - r * Cout;
+    ws[i] = w[co * kStemTerms + r];
   }
   const int cg = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int ohl = lane >> 2, owl = (lane & 3) * 4;
