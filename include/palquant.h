@@ -254,6 +254,21 @@ pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, cons
                                const float* shortcut_dev, int32_t* acc_out_dev, float* y_out_dev,
                                void* q_out_dev, pq_stream_t stream);
 
+/* The activation quantiser and the whole layer in one kernel (Sec. 3.2 Eq. 2,
+ * then as palquant_layer_fused): the layer's input is the fp32 NHWC activation
+ * tensor x_dev [N, H, W, G*Cin_g] instead of codes, quantised as it is loaded,
+ *   q[p, g*Cin_g + j] = clamp(rint(x[p, g*Cin_g + j] * inv_s[g]), 0, 2^bits_a - 1)
+ * (one fp32 multiply, round half to even, NaN -> 0; the codes palquant_quantize_act
+ * produces), so the codes never pass through memory.  inv_s_host: G floats
+ * (fl(1/s) of the input steps, >= 0), copied at call time.  Everything else as
+ * palquant_layer_fused: w_packed_dev comes from palquant_pack_weights for the same
+ * d, whose code_format (PQ_CODES_INT8 or PQ_CODES_C16) is the output codes'.
+ * Needs stride 1 and 16-byte aligned x_dev; other shapes return PQ_EUNSUPPORTED. */
+pq_status palquant_quantize_layer_fused(const float* x_dev, const float* inv_s_host, const void* w_packed_dev,
+                                        const pq_layer_desc* d, const float* m_out_host, const float* m_req_host,
+                                        pq_shuffle shuf, const float* shortcut_dev, int32_t* acc_out_dev,
+                                        float* y_out_dev, void* q_out_dev, pq_stream_t stream);
+
 /* Cyclic shuffle module (Sec. 4.2, Eq. 9-10), fused into one kernel:
  *   Y = CyclicPermute(X):  Y[:, pi(i)] = X[:, i] with pi(i) = (i + shift) mod G (Eq. 8,
  *                          group-level; Eq. 6 for shift = 1)

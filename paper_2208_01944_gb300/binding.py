@@ -27,6 +27,7 @@ EXPORTS = [
     "palquant_weight_steps", "palquant_epilogue_scales", "palquant_packed_weight_bytes",
     "palquant_pack_weights_host", "palquant_pack_weights", "palquant_pack_weight_codes_host",
     "palquant_unpack_weight_codes_host", "palquant_quantize_act", "palquant_group_conv", "palquant_layer_fused",
+    "palquant_quantize_layer_fused",
     "palquant_sync_check", "palquant_set_wait_limit_ns", "palquant_watchdog_selftest", "palquant_conv_plan",
     "palquant_conv2d_f32", "palquant_maxpool2d_f32", "palquant_avgpool_f32", "palquant_linear_f32",
     "palquant_cyclic_shuffle_module", "palquant_bitsplit_desc", "palquant_bitsplit_scratch_bytes",
@@ -99,6 +100,9 @@ def _load():
     L.palquant_group_conv.argtypes = [_P, _P, _P, ctypes.POINTER(LayerDesc), _P]
     L.palquant_layer_fused.restype = _I32
     L.palquant_layer_fused.argtypes = [_P, _P, ctypes.POINTER(LayerDesc), _P, _P, Shuffle, _P, _P, _P, _P, _P]
+    L.palquant_quantize_layer_fused.restype = _I32
+    L.palquant_quantize_layer_fused.argtypes = [_P, _P, _P, ctypes.POINTER(LayerDesc), _P, _P, Shuffle, _P, _P, _P, _P,
+                                                _P]
     L.palquant_sync_check.restype = _I32
     L.palquant_sync_check.argtypes = [_P]
     L.palquant_set_wait_limit_ns.restype = _I32
@@ -282,6 +286,17 @@ def palquant_layer_fused(q_dev, w_packed_dev, d: LayerDesc, m_out, m_req=None, s
     _check(lib.palquant_layer_fused(_ptr(q_dev), _ptr(w_packed_dev), ctypes.byref(d), _ptr(mo), _ptr(mr),
                                     shuf or shuffle(1, 1), _ptr(shortcut_dev), _ptr(acc_out_dev), _ptr(y_out_dev),
                                     _ptr(q_out_dev), _stream(stream)), "palquant_layer_fused")
+
+
+def palquant_quantize_layer_fused(x_dev, inv_s, w_packed_dev, d: LayerDesc, m_out, m_req=None, shuf=None,
+                                  shortcut_dev=None, acc_out_dev=None, y_out_dev=None, q_out_dev=None, stream=None):
+    inv = _f32(inv_s)
+    mo = None if m_out is None else _f32(m_out)
+    mr = None if m_req is None else _f32(m_req)
+    _check(lib.palquant_quantize_layer_fused(_ptr(x_dev), _ptr(inv), _ptr(w_packed_dev), ctypes.byref(d), _ptr(mo),
+                                             _ptr(mr), shuf or shuffle(1, 1), _ptr(shortcut_dev), _ptr(acc_out_dev),
+                                             _ptr(y_out_dev), _ptr(q_out_dev), _stream(stream)),
+           "palquant_quantize_layer_fused")
 
 
 def palquant_cyclic_shuffle_module(q_dev, w_packed_dev, d: LayerDesc, m_out, m_req=None, shift=1, x_dev=None,

@@ -109,7 +109,10 @@ struct Phase {
   int a, b;
 };
 
-pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, std::vector<Phase>* phases_out) {
+// quant_in: the layer's input is fp32 NHWC activations, quantised on load (the
+// copy warps quantise TMA-staged 32-channel fp32 boxes into the operand stages).
+pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, std::vector<Phase>* phases_out,
+                    bool quant_in = false) {
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
   pq_conv_plan plan;
@@ -135,7 +138,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const bool flat_shape = d->kh == 1 && d->kw == 1 && d->stride == 1 && d->pad == 0;
   const bool p2_ok = !p2 || (d->bits_a <= 2 && d->bits_out <= 2 && d->stride == 1 &&
                              (flat_shape ? (static_cast<int64_t>(d->H) * d->W) % 4 == 0 : d->W % 4 == 0));
-  bool ok = (d->code_format == PQ_CODES_INT8 || c16) && p2_ok && f4_ok && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
+  // Quantise-on-load: stride 1, byte codes out (NHWC or channel-blocked), 32-channel
+  // K blocks, fp32 rows of 16-byte multiples for the TMA.
+  const bool quant_ok = !quant_in || (d->stride == 1 && !p2 && !f4 && (d->G * d->Cin_g) % 4 == 0);
+  bool ok = (d->code_format == PQ_CODES_INT8 || c16) && p2_ok && f4_ok && quant_ok && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
             d->pad < std::max(d->kh, d->kw) && d->Cin_g % 32 == 0 && d->Cout_g % 16 == 0 && taps <= pq::kMaxTaps &&
             static_cast<int64_t>(taps) * d->Cin_g * qa * qw < (1LL << 24);
   if (!ok) {
@@ -211,7 +217,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const double ns_per_clk = 1.0 / 1.9;
   const double mma_ns = std::max(32.0 + p.Npow2 / 4.0, p.Npow2 / 2.0) * ns_per_clk;
   const double mma_acc_ns = static_cast<double>(p.taps) * (d->Cin_g / (32 * cpb)) * mma_ns;  // one accumulator
-  const bool tma_operand = c16 && d->stride == 1 && (flat || Wh <= 128);
+  // (quantise-on-load keeps the copy warps busy converting: two epilogue groups)
+  const bool tma_operand = !quant_in && c16 && d->stride == 1 && (flat || Wh <= 128);
   const int epi_groups = tma_operand ? pq::kEpiGroups + 1 : pq::kEpiGroups;
   const int unit_cols = (f4 && p.Nblk % 32 == 0) ? 32 : 16;
   const int units_per_acc = p.Nblk / unit_cols;
@@ -224,7 +231,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   for (int MT : {1, 2, 3, 4}) {
     // flat tiles: up to two accumulators (by TMA, one 128-position box each); the
     // packed 2-bit path stages one box
-    if (flat && (MT > 2 || (p2 && MT > 1))) continue;
+    if (flat && (MT > 2 || ((p2 || quant_in) && MT > 1))) continue;
     int acc_stages = (2 * MT * p.Npow2 <= tmem_avail) ? 2 : ((MT * p.Npow2 <= tmem_avail) ? 1 : 0);
     if (acc_stages == 0) continue;
     int ht = 0, tpi = 0;
@@ -235,6 +242,17 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
       if (ht_max < 1) continue;
       tpi = (Ho + ht_max - 1) / ht_max;
       ht = (Ho + tpi - 1) / tpi;
+    }
+    if (quant_in) {
+      // two fp32 staging stages (128 bytes per position) and two operand stages
+      // (32 bytes per position) must fit beside the weights (resident, or a
+      // two-slice ring) and the epilogue staging
+      const uint64_t npos = flat ? 128u : static_cast<uint64_t>(ht + rmax - rmin) * Wh;
+      const uint64_t w_unit = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk;
+      const uint64_t w_min = w_unit <= 112u * 1024u ? round_up(w_unit, 1024) : 2ull * round_up(32ull * p.Nblk, 1024);
+      const uint64_t need = 2ull * (round_up(npos * 128, 1024) + round_up(npos * 32, 1024)) + w_min +
+                            pq::kEpiWarps * 2560ull + 1024;
+      if (need > pq::kMaxSmem - 1024) continue;
     }
     const int units = MT * units_per_acc;
     const double epi_ns = ((units + epi_groups - 1) / epi_groups) * unit_ns;
@@ -311,9 +329,11 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const uint32_t q_pitch = 80;
   const uint32_t f_pitch = 80;
   const uint32_t warp_stage = round_up(32u * q_pitch, 128);
-  // Staging for every warp that can run the epilogue (the copy warps join it when
-  // TMA loads the activation operand).
-  const uint32_t stage_total = warp_stage * (pq::kEpiWarps + pq::kLoadWarps);
+  // Staging for every warp that runs the epilogue: the copy warps join it only when
+  // TMA loads the activation operand as it is (not unpacked, not quantised).
+  const bool third_group =
+      !quant_in && !p2 && c16 && d->stride == 1 && (flat ? p.flat_box <= 256 : p.Wd <= 128);
+  const uint32_t stage_total = warp_stage * (third_group ? pq::kEpiWarps + pq::kLoadWarps : pq::kEpiWarps);
   const uint32_t bar_bytes = 1024;  // barriers, abort flag, TMEM slot (generous)
   const uint64_t unit_bytes = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk / cpb;
   // Packed codes: a staging stage per operand stage holding the TMA box of 32-bit
@@ -327,6 +347,11 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
     return PQ_EUNSUPPORTED;
   }
   auto pk_stage_bytes = [&](int KC) -> uint32_t {
+    if (quant_in) {
+      // fp32 box of KC channels x all positions of the stage (128-byte rows)
+      const uint64_t npos = flat ? static_cast<uint64_t>(p.flat_box) : static_cast<uint64_t>(p.Hd) * p.Wd;
+      return round_up(npos * KC * 4, 1024);
+    }
     if (!p2) return 0;
     const uint64_t rows = flat ? 1 : p.Hd;
     return round_up(static_cast<uint64_t>(pk_box_w) * rows * (KC / 16) * 4, 1024);
@@ -340,6 +365,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // MMA issue loop is compiled for these K-step counts.
   for (int kc1 : {256, 128, 96, 64, 32}) {
     if (found) break;
+    if (quant_in && kc1 != 32) continue;  // one 128-byte fp32 row per position
     const int kc = kc1 * cpb;
     if (d->Cin_g % kc != 0) continue;
     uint32_t sb, pb, l;
@@ -386,14 +412,16 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.codes_f4 = f4 ? 1 : 0;
   p.chunk_shift = f4 ? 5 : 4;
   p.a_unpack = p2 ? 1 : 0;
+  p.a_quant = quant_in ? 1 : 0;
   p.pk_box_w = pk_box_w;
   p.pk_off = pk_off;
   p.pk_stage_bytes = pk_stage_bytes(KC);
   // The A operand comes by TMA when every plane row is one contiguous run in
   // global memory: channel-blocked codes, stride 1, rows of at most 128 positions.
-  p.a_tma = (p2 || (c16 && d->stride == 1 && (flat ? p.flat_box <= 256 : p.Wd <= 128))) ? 1 : 0;
-  p.a_mt16 = (flat && c16 && !p2) ? static_cast<uint32_t>(p.nch) * 128u : 128u;
-  p.a_tx_bytes = p2 ? static_cast<uint32_t>(p.nch) * pk_box_w * (flat ? 1 : p.Hd) * 4u
+  p.a_tma = (quant_in || p2 || (c16 && d->stride == 1 && (flat ? p.flat_box <= 256 : p.Wd <= 128))) ? 1 : 0;
+  p.a_mt16 = (flat && c16 && !p2 && !quant_in) ? static_cast<uint32_t>(p.nch) * 128u : 128u;
+  p.a_tx_bytes = quant_in ? static_cast<uint32_t>(KC) * 4u * (flat ? p.flat_box : p.Hd * p.Wd)
+                 : p2 ? static_cast<uint32_t>(p.nch) * pk_box_w * (flat ? 1 : p.Hd) * 4u
                  : flat ? static_cast<uint32_t>(p.nch) * p.flat_box * 16u
                         : static_cast<uint32_t>(p.nph) * p.nch * p.Hd * p.Wd * 16u;
   {
@@ -535,13 +563,41 @@ bool encode_c16_map(const pq_layer_desc* d, const ConvParams& p, const void* q_d
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Tensor map of fp32 NHWC activations for quantise-on-load: boxes of 32 channels
+// (128 bytes, swizzled 128B so the copy warps read them without bank conflicts)
+// x Wd positions x Hd rows (rows mode), or x 128 positions (flat mode, HW as one
+// dimension).  Out-of-range positions are zero-filled: code 0, the zero padding.
+bool encode_f32_map(const pq_layer_desc* d, const ConvParams& p, const void* x_dev, CUtensorMap* map) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return false;
+  std::memset(map, 0, sizeof(*map));
+  const uint64_t C = static_cast<uint64_t>(d->G) * d->Cin_g, H = d->H, W = d->W;
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  if (p.mode == pq::kModeFlat) {
+    cuuint64_t dims[3] = {C, H * W, static_cast<cuuint64_t>(d->N)};
+    cuuint64_t strides[2] = {C * 4, H * W * C * 4};
+    cuuint32_t box[3] = {32u, static_cast<cuuint32_t>(p.flat_box), 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(x_dev), dims, strides, box, es,
+               CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+  }
+  cuuint64_t dims[4] = {C, W, H, static_cast<cuuint64_t>(d->N)};
+  cuuint64_t strides[3] = {C * 4, W * C * 4, H * W * C * 4};
+  cuuint32_t box[4] = {32u, static_cast<cuuint32_t>(p.Wd), static_cast<cuuint32_t>(p.Hd), 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<void*>(x_dev), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 // ---------------------------------------------------------------------------
 // Weight packing (tensor-core operand layout of the planner's tiling).
-//   unit u = g * NB + nb; for each K block kb, tap t, 16-byte chunk j,
-//   output channel c (of the block) and channel e of the chunk (E = 16
-//   channels per chunk, 32 for FP4):
-//   element[(((u * n_kb + kb) * taps + t) * nch + j) * Nblk * E + c * E + e]
-//     = w_q[g, nb*Nblk + c, tap t, kb*KC + j*E + e]
+//   unit u = g * NB + nb; for each tap t, 16-byte chunk J of the input channels
+//   (J = kb * nch + j for K block kb), output channel c (of the block) and
+//   channel e of the chunk (E = 16 channels per chunk, 32 for FP4):
+//   element[(((u * taps + t) * NCH + J) * Nblk + c) * E + e]
+//     = w_q[g, nb*Nblk + c, tap t, J*E + e],   NCH = Cin_g / E
+//   so a (K block, tap) slice is one contiguous run whatever the K blocking
+//   (the same packing serves every tiling of the layer).
 //   as an E4M3 byte, or (FP4) an E2M1 nibble, element 2i in the low nibble of
 //   byte i and element 2i+1 in the high one.
 // ---------------------------------------------------------------------------
@@ -556,7 +612,8 @@ void for_each_packed(const ConvParams& p, int kw, F&& f) {
             for (int c = 0; c < p.Nblk; ++c)
               for (int e = 0; e < E; ++e) {
                 const int u = g * p.NB + nb;
-                const size_t dst = ((((static_cast<size_t>(u) * p.n_kb + kb) * p.taps + t) * p.nch + j) * p.Nblk + c) * E + e;
+                const size_t dst =
+                    ((((static_cast<size_t>(u) * p.taps + t) * p.n_kb + kb) * p.nch + j) * p.Nblk + c) * E + e;
                 const int co = nb * p.Nblk + c;
                 const int ci = kb * p.KC + j * E + e;
                 const int i = t / kw, jj = t % kw;
@@ -598,10 +655,12 @@ void pack_codes(const ConvParams& p, const pq_layer_desc* d, const int8_t* wq, u
   }
 }
 
+// inv_s_in (host, G floats, or NULL): q_dev is fp32 NHWC activations quantised on
+// load with these reciprocal steps instead of codes.
 pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
                            const float* m_out_host, const float* m_req_host, pq_shuffle shuf,
                            const float* shortcut_dev, int32_t* acc_out_dev, float* y_out_dev, void* q_out_dev,
-                           const int* src_group, pq_stream_t stream) {
+                           const int* src_group, pq_stream_t stream, const float* inv_s_in = nullptr) {
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
   if (q_dev == nullptr || w_packed_dev == nullptr) return PQ_EINVAL;
@@ -613,8 +672,20 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
     return PQ_EINVAL;
   ConvParams p;
   std::vector<Phase> phases;
-  st = plan_conv(d, &p, nullptr, &phases);
+  st = plan_conv(d, &p, nullptr, &phases, inv_s_in != nullptr);
   if (st != PQ_OK) return st;
+  if (inv_s_in != nullptr) {
+    // reciprocal steps scaled by 2^-b (exact: a power of two) for the saturating form
+    const float inv_two_b = 1.0f / static_cast<float>(1 << d->bits_a);
+    for (int g = 0; g < d->G; ++g) {
+      if (!std::isfinite(inv_s_in[g]) || !(inv_s_in[g] >= 0.0f) || (inv_s_in[g] != 0.0f && inv_s_in[g] < 1e-30f) ||
+          inv_s_in[g] > 1e30f)
+        return PQ_EINVAL;
+      p.q_inv_sat[g] = inv_s_in[g] * inv_two_b;
+    }
+    p.q_two_b = static_cast<float>(1 << d->bits_a);
+    p.q_qmax2 = static_cast<uint32_t>((1 << d->bits_a) - 1) * 0x00010001u;
+  }
   int dst[pq::kMaxG];
   if (!valid_shuffle(d->G, shuf, dst)) return PQ_EINVAL;
   if (d->N == 0) return PQ_OK;
@@ -648,7 +719,11 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
   if (grid <= 0) return PQ_OK;
   CUtensorMap map;
   std::memset(&map, 0, sizeof(map));
-  if (p.a_tma && !encode_c16_map(d, p, q_dev, &map)) return PQ_ECUDA;
+  if (p.a_quant) {
+    if (!encode_f32_map(d, p, q_dev, &map)) return PQ_ECUDA;
+  } else if (p.a_tma && !encode_c16_map(d, p, q_dev, &map)) {
+    return PQ_ECUDA;
+  }
   if (pq::launch_conv_tc(p, map, grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
   return PQ_OK;
 }
@@ -871,6 +946,15 @@ pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, cons
                                pq_stream_t stream) {
   return layer_fused_impl(q_dev, w_packed_dev, d, m_out_host, m_req_host, shuf, shortcut_dev, acc_out_dev, y_out_dev,
                           q_out_dev, nullptr, stream);
+}
+
+pq_status palquant_quantize_layer_fused(const float* x_dev, const float* inv_s_host, const void* w_packed_dev,
+                                        const pq_layer_desc* d, const float* m_out_host, const float* m_req_host,
+                                        pq_shuffle shuf, const float* shortcut_dev, int32_t* acc_out_dev,
+                                        float* y_out_dev, void* q_out_dev, pq_stream_t stream) {
+  if (inv_s_host == nullptr) return PQ_EINVAL;
+  return layer_fused_impl(x_dev, w_packed_dev, d, m_out_host, m_req_host, shuf, shortcut_dev, acc_out_dev, y_out_dev,
+                          q_out_dev, nullptr, stream, inv_s_host);
 }
 
 pq_status palquant_cyclic_shuffle_module(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,

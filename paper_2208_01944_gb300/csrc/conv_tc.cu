@@ -161,7 +161,21 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
     }
     if (!a_tma && p.b_resident) continue;
     for (int kb = 0; kb < p.n_kb && ok; ++kb) {
-      if (a_tma && p.a_unpack) {
+      if (a_tma && p.a_quant) {
+        // fp32 activations: a box of 32 channels (one 128-byte swizzled row per
+        // position) into the staging ring; the copy warps quantise it.
+        if (!mbar_wait(bars.pk_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
+        const uint32_t full = bars.pk_full(ra.stage);
+        mbar_arrive_expect_tx(full, p.a_tx_bytes);
+        const uint32_t dst = pk_base + ra.stage * p.pk_stage_bytes;
+        const int ch0 = p.src_group[item.g] * p.Cin_g + kb * p.KC;
+        if (flat)
+          tma_load_3d(dst, tmA, ch0, item.rb * p.flat_box, item.n, full);
+        else
+          tma_load_4d(dst, tmA, ch0, p.w_coord, item.oh0(p.Ht) + p.h_off, item.n, full);
+        ra.advance();
+        ++a_issued;
+      } else if (a_tma && p.a_unpack) {
         // Packed codes: the box of 32-bit words into the staging ring; the copy
         // warps unpack it into the operand stage.
         if (!mbar_wait(bars.pk_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
@@ -197,7 +211,7 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
         if (!mbar_wait(bars.b_empty(rb.stage), rb.phase ^ 1u, ctx)) { ok = false; break; }
         const uint32_t bar = bars.b_full(rb.stage);
         mbar_arrive_expect_tx(bar, p.b_slice_bytes);
-        const size_t slice = (static_cast<size_t>(unit) * p.n_kb + kb) * p.taps + t;
+        const size_t slice = (static_cast<size_t>(unit) * p.taps + t) * p.n_kb + kb;  // tap-major packing
         bulk_load(b_base + rb.stage * p.b_slice_bytes, p.w_packed + slice * p.b_slice_bytes, p.b_slice_bytes, bar);
         rb.advance();
         ++b_issued;
@@ -207,7 +221,7 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
   // Drain: the last min(stages, issued) copies of each ring may still be in flight.
   const int64_t na = p.a_stages, nbs = p.b_resident ? 1 : p.b_stages;
   for (int64_t k = (a_issued > na ? a_issued - na : 0); k < a_issued; ++k)
-    mbar_wait_drain(p.a_unpack ? bars.pk_full(static_cast<int>(k % na)) : bars.a_full(static_cast<int>(k % na)),
+    mbar_wait_drain((p.a_unpack || p.a_quant) ? bars.pk_full(static_cast<int>(k % na)) : bars.a_full(static_cast<int>(k % na)),
                     static_cast<uint32_t>((k / na) & 1), ctx.limit_ns, ctx.err);
   for (int64_t k = (b_issued > nbs ? b_issued - nbs : 0); k < b_issued; ++k)
     mbar_wait_drain(bars.b_full(static_cast<int>(k % nbs)), static_cast<uint32_t>((k / nbs) & 1), ctx.limit_ns, ctx.err);
@@ -430,6 +444,7 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
   const uint32_t a_lo0 = static_cast<uint32_t>(a_desc0), b_lo0 = static_cast<uint32_t>(b_desc0);
   const uint32_t a_ks16 = (2u * p.lbo_a) >> 4, b_ks16 = (2u * p.lbo_b) >> 4;  // one K step (32 bytes of K)
   const uint32_t a_stage16 = p.a_stage_bytes >> 4, b_slice16 = p.b_slice_bytes >> 4;
+  const uint32_t b_tap16 = static_cast<uint32_t>(p.n_kb) * b_slice16;  // one tap of all K blocks
   const uint32_t amt = p.a_mt16;  // A operand of accumulator mt starts mt * amt 16-byte units in
   const int taps = p.taps, n_kb = p.n_kb;
   const uint32_t npow2 = static_cast<uint32_t>(p.Npow2);
@@ -459,7 +474,8 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
       if (!warp_wait(bars.a_full(ra.stage), ra.phase, ctx)) { ok = false; break; }
       tc_fence_after();
       const uint32_t a_lo_stage = a_lo0 + ra.stage * a_stage16;
-      const uint32_t b_lo_kb = b_lo0 + static_cast<uint32_t>(kb * taps) * b_slice16;
+      // packed weights are tap-major: tap t of K block kb is slice t * n_kb + kb
+      const uint32_t b_lo_kb = b_lo0 + static_cast<uint32_t>(kb) * b_slice16;
       // One tap: KSTEPS x MT MMAs, fully unrolled.
       auto issue_tap = [&](int t, uint32_t a_lo_tap, uint32_t b_lo_tap) {
         const uint32_t acc0 = (kb | t) == 0 ? 0u : 1u;
@@ -498,12 +514,12 @@ __device__ __forceinline__ void mma_role(const ConvParams& p, const Bars& bars, 
         // loop branches between the MMAs of a K block.
 #pragma unroll
         for (int t = 0; t < kUnrollTaps; ++t)
-          if (t < taps) issue_tap(t, a_lo_stage + tap_reg[t], b_lo_kb + static_cast<uint32_t>(t) * b_slice16);
+          if (t < taps) issue_tap(t, a_lo_stage + tap_reg[t], b_lo_kb + static_cast<uint32_t>(t) * b_tap16);
       } else {
         for (int t = 0; t < taps; ++t) {
           uint32_t b_lo_tap;
           if (resident) {
-            b_lo_tap = b_lo_kb + static_cast<uint32_t>(t) * b_slice16;
+            b_lo_tap = b_lo_kb + static_cast<uint32_t>(t) * b_tap16;
           } else {
             if (!warp_wait(bars.b_full(rb.stage), rb.phase, ctx)) { ok = false; break; }
             tc_fence_after();
@@ -655,6 +671,64 @@ __device__ __forceinline__ long long codes_offset(const ConvParams& p, int pack,
   if (pack == 2)
     return ((static_cast<long long>(n) * (p.C_out_total >> 5) + (k >> 1)) * hw_out + pos) * 16 + (k & 1) * 8;
   return ((static_cast<long long>(n) * (p.C_out_total >> 4) + k) * hw_out + pos) * (pack ? 4 : 16);
+}
+
+// --------------------------------------------------------------------------
+// Quantise-on-load role (warps 2-5): each staged box holds, per position of the
+// stage, the 32 fp32 activations of the K block as one 128-byte row, swizzled
+// 128B (16-byte chunk c of row r at chunk c ^ (r & 7), the rows' bank groups
+// spread).  Thread items are (position, 16-channel half): four 16-byte reads,
+// the codes clamp(rint(x * fl(1/s)), 0, Qp) of the input group (one fp32
+// multiply, the saturating form of the epilogue's conversion, NaN -> 0), one
+// 16-byte write to the operand plane of the half.  Positions outside the image
+// were zero-filled by the TMA unit: code 0, the zero padding.
+// --------------------------------------------------------------------------
+__device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t st_base,
+                                           int64_t it0, int64_t it1, const WaitCtx& ctx) {
+  const int tid = threadIdx.x - 32 * kFirstLoadWarp;
+  const int lane = tid & 31;
+  const int npos = p.mode == kModeFlat ? p.flat_box : p.Hd * p.Wd;
+  const int n_items = 2 * npos;
+  const uint32_t plane = p.lbo_a;
+  const float two_b = p.q_two_b;
+  const uint32_t qmax2 = p.q_qmax2;
+  Ring r{0, 0, static_cast<uint32_t>(p.a_stages)};
+  bool ok = true;
+  Item item = item_begin(p, it0);
+  for (int64_t it = it0; it < it1 && ok; ++it, item_next(p, item)) {
+    const float m_sat = p.q_inv_sat[p.src_group[item.g]];
+    for (int kb = 0; kb < p.n_kb; ++kb) {
+      if (!warp_wait(bars.pk_full(r.stage), r.phase, ctx)) { ok = false; break; }
+      if (!warp_wait(bars.a_empty(r.stage), r.phase ^ 1u, ctx)) { ok = false; break; }
+      const uint32_t src = st_base + r.stage * p.pk_stage_bytes;
+      const uint32_t dst = a_base + r.stage * p.a_stage_bytes;
+      for (int e = tid; e < n_items; e += 32 * kLoadWarps) {
+        const int pos = e >> 1, half = e & 1;
+        const uint32_t row = src + static_cast<uint32_t>(pos) * 128u;
+        uint32_t v[16];
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const uint32_t a = row + ((static_cast<uint32_t>(4 * half + k) ^ static_cast<uint32_t>(pos & 7)) << 4);
+          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                       : "=r"(v[4 * k]), "=r"(v[4 * k + 1]), "=r"(v[4 * k + 2]), "=r"(v[4 * k + 3])
+                       : "r"(a)
+                       : "memory");
+        }
+        const uint4 w = epi_codes16(v, m_sat, two_b, qmax2);
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst + static_cast<uint32_t>(half) * plane +
+                                                                          static_cast<uint32_t>(pos) * 16u),
+                     "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
+                     : "memory");
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(bars.a_full(r.stage));
+        mbar_arrive(bars.pk_empty(r.stage));
+      }
+      r.advance();
+    }
+  }
 }
 
 // Store 16 codes of 16-column chunk `ch` of the row (output pixel pos).
@@ -959,9 +1033,10 @@ __global__ void __launch_bounds__(kConvThreads, 1)
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < bars.A; ++s) {
-      mbar_init(bars.a_full(s), (p.a_tma && !p.a_unpack) ? 1 : kLoadWarps);  // TMA, or one arrival per copy warp
+      // TMA, or one arrival per copy warp
+      mbar_init(bars.a_full(s), (p.a_tma && !p.a_unpack && !p.a_quant) ? 1 : kLoadWarps);
       mbar_init(bars.a_empty(s), 1);
-      if (p.a_unpack) {
+      if (p.a_unpack || p.a_quant) {
         mbar_init(bars.pk_full(s), 1);
         mbar_init(bars.pk_empty(s), kLoadWarps);
       }
@@ -972,7 +1047,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     }
     for (int s = 0; s < p.acc_stages; ++s) {
       mbar_init(bars.acc_full(s), 1);
-      mbar_init(bars.acc_empty(s), (p.a_tma && !p.a_unpack) ? kEpiWarps + kLoadWarps : kEpiWarps);  // one per warp
+      mbar_init(bars.acc_empty(s),
+                (p.a_tma && !p.a_unpack && !p.a_quant) ? kEpiWarps + kLoadWarps : kEpiWarps);  // one per warp
     }
     mbar_init(bars.drain(), 1);
     *abort_flag = 0;
@@ -1015,13 +1091,16 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     __syncwarp();
   } else if (warp < kFirstEpiWarp && !p.a_tma) {
     loader_role(p, bars, a_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
+  } else if (warp < kFirstEpiWarp && p.a_quant) {
+    quant_role(p, bars, a_base, base + p.smem_pk_off, it0, it1,
+               WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else if (warp < kFirstEpiWarp && p.a_unpack) {
     unpack_role(p, bars, a_base, base + p.smem_pk_off, it0, it1,
                 WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else {
     // With TMA loading the activations as they are, the copy warps form a third
     // epilogue warpgroup.
-    const bool third = p.a_tma && !p.a_unpack;
+    const bool third = p.a_tma && !p.a_unpack && !p.a_quant;
     const int first = third ? kFirstLoadWarp : kFirstEpiWarp;
     epilogue_role<F4>(p, bars, tmem_base, gbase + p.smem_stage_off, first, third ? kEpiGroups + 1 : kEpiGroups, it0, it1,
                   WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_EPILOGUE});

@@ -56,6 +56,14 @@ struct ConvParams {
   // them into the operand stages (a_unpack = 1): staged rows of pk_box_w 32-bit
   // words starting pk_off words left of the tile's first position.
   int a_unpack;
+  // Quantise-on-load (a_quant = 1): the input is fp32 NHWC; TMA stages boxes of 32
+  // channels x all positions of a stage (128-byte rows, 128-byte swizzle) into the
+  // staging ring and the copy warps quantise them into the operand stage:
+  // code = min(rint(sat(x * q_inv_sat[g]) * 2^b), Qp), q_inv_sat = fl(1/s) / 2^b.
+  int a_quant;
+  float q_inv_sat[kMaxG];
+  float q_two_b;
+  uint32_t q_qmax2;  // Qp in both 16-bit halves
   int pk_box_w, pk_off;
   uint32_t pk_stage_bytes, smem_pk_off;
   int a_tma;              // 1: warp 0 loads the A operand with one TMA per stage (channel-blocked codes, stride 1)

@@ -330,3 +330,26 @@ def test_fp4_code_helpers_roundtrip():
     one[0, 1, 0, 32 + 7] = 3
     r = to_format(one, 4)
     assert np.flatnonzero(r).tolist() == [2 * 16 + 16 + 3] and r[2 * 16 + 16 + 3] == 3 << 4
+
+
+def test_quantize_layer_fused_rules():
+    """Quantise-on-load covers stride-1 layers with byte codes out; the reciprocal
+    steps are required and must be finite and non-negative."""
+    d = B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C16)
+    for bad in [B.layer_desc(1, 8, 8, 2, 32, 32, 3, 2, 1, 2, 2, 2, code_format=B.PQ_CODES_C16),    # stride 2
+                B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C16P2),  # packed codes
+                B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C32F4)]:  # FP4 codes
+        with pytest.raises(B.PalquantError) as e:
+            B.palquant_quantize_layer_fused(16, [1.0, 1.0], 16, bad, [1.0] * 2, [1.0] * 2, q_out_dev=16)
+        assert e.value.status == B.PQ_EUNSUPPORTED
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_quantize_layer_fused(16, [1.0, float("nan")], 16, d, [1.0] * 2, [1.0] * 2, q_out_dev=16)
+    assert e.value.status == B.PQ_EINVAL
+    with pytest.raises(B.PalquantError) as e:
+        B.palquant_quantize_layer_fused(16, [1.0, -2.0], 16, d, [1.0] * 2, [1.0] * 2, q_out_dev=16)
+    assert e.value.status == B.PQ_EINVAL
+    # one packing serves both the plain layer and quantise-on-load (tap-major layout)
+    gen = synth.generator(9)
+    wq = synth.random_codes((2, 32, 3, 3, 64), 2, gen, signed=True)
+    d2 = B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C16)
+    assert np.array_equal(B.palquant_unpack_weight_codes_host(B.palquant_pack_weight_codes_host(wq, d2), d2), wq)

@@ -484,3 +484,87 @@ def test_layer_fp4_with_odd_weight_levels_matches_oracle(B):
     assert np.array_equal(ad.cpu().numpy(), a_ref)
     assert np.array_equal(yd.cpu().numpy(), y_ref)
     assert np.array_equal(from_format(qo.cpu().numpy(), 4, N, H, W, G * Co).reshape(-1, G * Co), q_ref)
+
+
+# ------------------------------- quantiser fused into the layer (fp32 in, codes out)
+QF_CASES = [
+    Case(1, 28, 28, 2, 32, 32, 3, 1, 1, seed=110),                    # config 0 shape
+    Case(2, 13, 11, 3, 32, 48, 3, 1, 1, seed=111),                    # odd sizes, three output chunks
+    Case(2, 7, 9, 4, 96, 96, 1, 1, 0, seed=112),                      # flat, ragged last tile
+    Case(2, 20, 20, 2, 64, 64, 1, 1, 0, seed=113),                    # flat, several tiles
+    Case(1, 12, 12, 2, 128, 256, 3, 1, 1, seed=114),                  # four K blocks, two output blocks
+    Case(1, 7, 7, 2, 256, 32, 3, 1, 1, seed=115),                     # eight K blocks, whole-image tiles
+    Case(2, 11, 10, 2, 64, 64, 3, 1, 1, shortcut=True, seed=116),     # shortcut add before ReLU
+    Case(1, 9, 11, 2, 32, 64, 5, 1, 2, seed=117),                     # 5x5 kernel
+    Case(1, 16, 16, 1, 32, 16, 3, 1, 0, bits=4, kind=0, seed=118),    # pad 0, G = 1, 4-bit
+    Case(2, 14, 14, 8, 32, 32, 3, 1, 1, kind=3, perm=(3, 0, 7, 1, 6, 2, 5, 4), seed=119),
+    Case(2, 6, 6, 2, 32, 32, 3, 1, 1, bits=3, bits_out=4, relu=False, kind=1, shift=-1, seed=120),
+    Case(1, 5, 130, 1, 32, 16, 3, 1, 1, seed=121),                    # rows wider than 128 positions
+    Case(2, 36, 40, 2, 64, 64, 3, 1, 1, seed=122),                    # several row tiles per image
+]
+
+
+def _run_quant_fused(B, c, ref, fmt, outputs=("acc", "y", "q")):
+    from layer_cases import code_bytes, from_format
+
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad, c.bits, c.bits, c.bo, int(c.relu),
+                     code_format=fmt)
+    nbytes = B.palquant_packed_weight_bytes(d)
+    wp = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    B.palquant_pack_weights(ref["w"], d, ref["inv_sw"], wp, nbytes)
+    shape = (c.N, c.Ho, c.Wo, c.G * c.Cout)
+    acc = torch.full(shape, -7, dtype=torch.int32, device="cuda") if "acc" in outputs else None
+    y = torch.full(shape, float("nan"), dtype=torch.float32, device="cuda") if "y" in outputs else None
+    qo = torch.full((code_bytes(int(np.prod(shape)), fmt),), 255, dtype=torch.uint8, device="cuda")
+    sc = None if ref["shortcut"] is None else torch.from_numpy(ref["shortcut"]).cuda()
+    B.palquant_quantize_layer_fused(torch.from_numpy(ref["x"]).cuda(), ref["inv_s"], wp, d, ref["m_out"],
+                                    ref["m_req"], B.shuffle(c.kind, c.shift, c.perm), sc, acc, y, qo)
+    st = B.palquant_sync_check()
+    assert st == B.PQ_OK, B.strerror(st)
+    out = dict(q=ref["q"])  # the input codes never leave the kernel
+    if acc is not None:
+        out["acc"] = acc.cpu().numpy().reshape(-1, c.G * c.Cout)
+    if y is not None:
+        out["y"] = y.cpu().numpy().reshape(-1, c.G * c.Cout)
+    out["q_out"] = from_format(qo.cpu().numpy(), fmt, c.N, c.Ho, c.Wo, c.G * c.Cout).reshape(-1, c.G * c.Cout)
+    return out
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=["nhwc", "c16"])
+@pytest.mark.parametrize("c", QF_CASES, ids=str)
+def test_quantize_layer_fused_matches_oracle(B, c, fmt):
+    """Quantise-on-load: the same int32 sums, fp32 outputs and codes as the oracle's
+    quantiser followed by its layer."""
+    ref = prepare(c)
+    assert_layer_parity(c, ref, _run_quant_fused(B, c, ref, fmt))
+
+
+@pytest.mark.parametrize("c", QF_CASES[:6], ids=str)
+def test_quantize_layer_fused_codes_only(B, c):
+    ref = prepare(c)
+    assert_layer_parity(c, ref, _run_quant_fused(B, c, ref, 2, outputs=("q",)))
+
+
+def test_quantize_layer_fused_special_inputs(B):
+    """Inputs exactly on rounding ties, NaN, +-inf and negative values quantise as the
+    oracle's quantiser does (NaN -> 0, +inf -> Qp, ties to even)."""
+    c = Case(2, 10, 12, 2, 64, 32, 3, 1, 1, bits=2, seed=123)
+    ref = prepare(c)
+    x = ref["x"].copy()
+    flat = x.reshape(-1)
+    rng = np.random.default_rng(5)
+    idx = rng.choice(flat.size, 400, replace=False)
+    inv = ref["inv_s"]
+    g_of = (np.arange(flat.size) % (c.G * c.Cin)) // c.Cin
+    ties = (rng.integers(0, 4, idx.size) + 0.5).astype(np.float32)
+    flat[idx[:200]] = ties[:200] / inv[g_of[idx[:200]]]  # x * inv_s lands on (or next to) a tie
+    flat[idx[200:250]] = np.nan
+    flat[idx[250:300]] = np.inf
+    flat[idx[300:350]] = -np.inf
+    flat[idx[350:]] = -rng.random(50).astype(np.float32)
+    q = oracle.quantize_act(x, c.G, c.bits, inv)
+    wq = ref["wq"]
+    acc = oracle.group_conv(q, wq, c.stride, c.pad).reshape(-1, c.G * c.Cout)
+    a_ref, y_ref, q_ref = oracle.epilogue(acc, c.G, ref["m_out"], ref["m_req"], c.kind, c.shift, None, None, True, c.bo)
+    ref2 = dict(ref, x=x, q=q, acc_ref=a_ref, y_ref=y_ref, q_ref=q_ref)
+    assert_layer_parity(c, ref2, _run_quant_fused(B, c, ref2, 2))
