@@ -50,8 +50,9 @@ def parse():
     ap.add_argument("--profile-stem", type=int, default=0, metavar="N",
                     help="only run the network's fp32 7x7 stem convolution on N 224x224 images --reps times, "
                          "for profilers; prints nothing else")
-    ap.add_argument("--profile-format", default="c16", choices=["c16", "f4"],
-                    help="code format of --profile-layer: one code per byte, or packed FP4 nibbles")
+    ap.add_argument("--profile-format", default="c16", choices=["c16", "f4", "f32"],
+                    help="input of --profile-layer: codes one per byte, packed FP4 nibbles, or fp32 activations "
+                         "quantised on load (the benchmark step)")
     ap.add_argument("--no-resnet", action="store_true", help="skip the ResNet-18-shaped network measurement")
     ap.add_argument("--resnet-batch", type=int, default=128)
     ap.add_argument("--resnet-reps", type=int, default=20)
@@ -72,6 +73,21 @@ def run_profile_layer(name: str, reps: int, fmt_name: str = "c16"):
     dev = torch.device("cuda:0")
     gen = synth.generator(0)
     f4 = fmt_name == "f4"
+    if fmt_name == "f32":  # fp32 activations, quantised on load: the benchmark step
+        x = torch.from_numpy(synth.half_normal((c.N, c.H, c.W, c.G * c.Cin_g), gen)).to(dev)
+        wq = synth.random_codes((c.G, c.Cout_g, c.k, c.k, c.Cin_g), c.bits_w, gen, signed=True)
+        d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w,
+                         c.bits_out, code_format=B.PQ_CODES_C16)
+        wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).to(dev)
+        qo = torch.empty(c.out_elems, dtype=torch.uint8, device=dev)
+        m = np.full(c.G, 0.01, np.float32)
+        inv = np.full(c.G, 1.3, np.float32)
+        for _ in range(reps):
+            B.palquant_quantize_layer_fused(x, inv, wp, d, m, m, B.shuffle(c.shuffle_kind, c.shuffle_shift), None,
+                                            None, None, qo)
+        st = B.palquant_sync_check()
+        assert st == B.PQ_OK, B.strerror(st)
+        return
     if f4:  # two random codes per byte, one per nibble
         lo = synth.random_codes((c.in_elems // 2,), c.bits_a, gen)
         q = torch.from_numpy(lo | (synth.random_codes((c.in_elems // 2,), c.bits_a, gen) << 4)).to(dev)
@@ -126,6 +142,7 @@ def source_sha(files):
 
 
 KERNEL_SOURCES = {
+    "pq_conv_tc_kernel<quantise-on-load>": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
     "pq_quantize_c16": ["quantize.cu", "pq_device.cuh", "pq_internal.h"],
     "pq_conv_tc_kernel": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
     "pq_quantize_c16<FP4 nibbles>": ["quantize.cu", "pq_device.cuh", "pq_internal.h"],
@@ -527,6 +544,69 @@ def measure_resnet18(dev, world, args):
     return out
 
 
+def measure_unfused_step(dev, stream, c, xs, q, inv_s, wp, d, m_out, m_req, shuf, q_out, K, world):
+    """The same step as two launches (the quantiser writing codes, then the layer
+    reading them back): K timed steps after 3 warm-up steps, per-kernel events."""
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+
+    fmt = B.PQ_CODES_C16
+
+    def launch(i):
+        B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt,
+                                stream=stream)
+        B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
+
+    with torch.cuda.stream(stream):
+        for i in range(3):
+            launch(i)
+    torch.cuda.synchronize(dev)
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for i in range(K):
+            ev[i][0].record(stream)
+            B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt,
+                                    stream=stream)
+            ev[i][1].record(stream)
+            B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
+            ev[i][2].record(stream)
+        stop.record(stream)
+    torch.cuda.synchronize(dev)
+    st = B.palquant_sync_check(stream)
+    assert st == B.PQ_OK, B.strerror(st)
+    return {"ms_per_step": max_over_ranks(start.elapsed_time(stop) / K, world, dev),
+            "t_quant": sum(e[0].elapsed_time(e[1]) for e in ev) / K,
+            "t_conv": sum(e[1].elapsed_time(e[2]) for e in ev) / K}
+
+
+def unfused_summary(r, c, pk, world):
+    """The two-launch step's throughput and the rooflines of its kernels."""
+    fp8_peak = 2.0 * pk["bf16_tflops"]
+    q_bytes = c.in_elems * 5  # 4-byte read + 1-byte write per element
+    conv_bytes = c.in_elems + c.out_elems + c.weight_elems
+    quant_gbs = q_bytes / (r["t_quant"] / 1e3) / 1e9
+    conv_tops = c.int_ops / (r["t_conv"] / 1e3) / 1e12
+    return {
+        "value": whole_job_rate(c.int_ops, world, r["ms_per_step"]) / 1e12, "unit": UNIT,
+        "ms_per_step": r["ms_per_step"],
+        "timed": "quantiser (fp32 NHWC -> codes) + layer (codes -> next-layer codes), two launches",
+        "roofline_kernels": [
+            {"kernel": "pq_quantize_c16", "bound": "hbm", "achieved": quant_gbs, "peak": pk["hbm_gbs"],
+             "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"], "traffic": dram_traffic("pq_quantize_c16"),
+             "algorithmic_bytes": q_bytes, "avg_launch_ms": r["t_quant"],
+             "peak_source": f"{pk['source']} HBM copy bandwidth"},
+            {"kernel": "pq_conv_tc_kernel", "bound": "tensor", "achieved": conv_tops, "peak": fp8_peak,
+             "unit": "TFLOP/s", "frac": conv_tops / fp8_peak, "traffic": dram_traffic("pq_conv_tc_kernel"),
+             "algorithmic_ops": c.int_ops, "algorithmic_bytes": conv_bytes, "avg_launch_ms": r["t_conv"],
+             "hbm_frac": conv_bytes / (r["t_conv"] / 1e3) / 1e9 / pk["hbm_gbs"],
+             "peak_source": f"{pk['source']} bf16 burst x 2 (dense FP8 E4M3, the exact-integer tensor path)"}],
+        "gpu_launches": 2,
+    }
+
+
 def measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf, K, world):
     """The same step (quantise + fused layer, same steps and multipliers) with the
     codes as packed FP4 nibbles (PQ_CODES_C32F4) and the block-scaled FP4 tensor-core
@@ -649,8 +729,9 @@ def run_ours(args, rank, world, local_rank):
     assert B.palquant_sync_check() == B.PQ_OK
 
     def step(i, s):
-        B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt, stream=s)
-        B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=s)
+        # the whole hot path in one launch: quantise on load, group conv, rescale,
+        # ReLU, cyclic remap, requantise
+        B.palquant_quantize_layer_fused(xs[i & 1], inv_s, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=s)
 
     # ---- warm-up
     with torch.cuda.stream(stream):
@@ -660,9 +741,9 @@ def run_ours(args, rank, world, local_rank):
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
 
-    # ---- timed region: K steps, per-kernel events on the launching stream
+    # ---- timed region: K steps, per-launch events on the launching stream
     K = args.steps
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local_rank)
     if world > 1:
@@ -674,15 +755,13 @@ def run_ours(args, rank, world, local_rank):
         start.record(stream)
         for i in range(K):
             ev[i][0].record(stream)
-            B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt,
-                                    stream=stream)
+            step(i, stream)
             ev[i][1].record(stream)
-            B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
-            ev[i][2].record(stream)
         stop.record(stream)
     torch.cuda.synchronize(dev)
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
+    unfused = measure_unfused_step(dev, stream, c, xs, q, inv_s, wp, d, m_out, m_req, shuf, q_out, K, world)
     fp4 = measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf, K, world)
     resnet = None if args.no_resnet else measure_resnet18(dev, world, args)
     layers = None if args.no_layers else measure_layer_configs(dev, args)
@@ -690,15 +769,14 @@ def run_ours(args, rank, world, local_rank):
     if world > 1:
         dist.barrier()
     elapsed_ms = start.elapsed_time(stop)
-    t_quant = sum(e[0].elapsed_time(e[1]) for e in ev) / K
-    t_conv = sum(e[1].elapsed_time(e[2]) for e in ev) / K
+    t_step = sum(e[0].elapsed_time(e[1]) for e in ev) / K
     elapsed_ms = max_over_ranks(elapsed_ms, world, dev)
     ms_per_step = elapsed_ms / K
     ops_step = c.int_ops
     value = whole_job_rate(ops_step, world, ms_per_step) / 1e12
 
     # ---- end to end through the public API with host buffers (pinned), per step:
-    # H2D input copy, quantize, fused layer, D2H of the output codes.
+    # H2D input copy, the fused quantiser + layer, D2H of the output codes.
     x_host = torch.from_numpy(x_np).pin_memory()
     out_host = torch.empty(out_shape, dtype=torch.uint8).pin_memory()
     x_dev = xs[0]
@@ -725,38 +803,33 @@ def run_ours(args, rank, world, local_rank):
         return
     pk = peaks()
     fp8_peak = 2.0 * pk["bf16_tflops"]  # dense FP8 = 2x dense BF16 (nominal ratio 4.5 / 2.25)
-    q_bytes = c.in_elems * 5  # 4-byte read + 1-byte write per element
-    conv_bytes = c.in_elems + c.out_elems + c.weight_elems
-    quant_gbs = q_bytes / (t_quant / 1e3) / 1e9
-    conv_tops = ops_step / (t_conv / 1e3) / 1e12
-    roof_quant = {"kernel": "pq_quantize_c16", "bound": "hbm", "achieved": quant_gbs, "peak": pk["hbm_gbs"],
-                  "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"], "traffic": dram_traffic("pq_quantize_c16"),
-                  "algorithmic_bytes": q_bytes, "avg_launch_ms": t_quant,
-                  "peak_source": f"{pk['source']} HBM copy bandwidth"}
-    roof_conv = {"kernel": "pq_conv_tc_kernel", "bound": "tensor", "achieved": conv_tops, "peak": fp8_peak,
-                 "unit": "TFLOP/s", "frac": conv_tops / fp8_peak, "traffic": dram_traffic("pq_conv_tc_kernel"),
-                 "algorithmic_ops": ops_step, "algorithmic_bytes": conv_bytes, "avg_launch_ms": t_conv,
-                 "hbm_frac": conv_bytes / (t_conv / 1e3) / 1e9 / pk["hbm_gbs"],
-                 "peak_source": f"{pk['source']} bf16 burst x 2 (dense FP8 E4M3, the exact-integer tensor path)"}
-    dominant = roof_quant if t_quant >= t_conv else roof_conv
+    step_bytes = c.in_elems * 4 + c.out_elems + c.weight_elems  # fp32 in, codes out, weights
+    step_gbs = step_bytes / (t_step / 1e3) / 1e9
+    step_tops = ops_step / (t_step / 1e3) / 1e12
+    roof_step = {"kernel": "pq_conv_tc_kernel (quantise on load)", "bound": "hbm", "achieved": step_gbs,
+                 "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": step_gbs / pk["hbm_gbs"],
+                 "traffic": dram_traffic("pq_conv_tc_kernel<quantise-on-load>"), "algorithmic_bytes": step_bytes,
+                 "algorithmic_ops": ops_step, "avg_launch_ms": t_step, "tensor_tops": step_tops,
+                 "tensor_frac": step_tops / fp8_peak, "peak_source": f"{pk['source']} HBM copy bandwidth"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "u8 codes, e4m3 x e4m3 -> f32 (exact integer)", "data": "synthetic",
+        "dtype": "fp32 activations -> u8 codes, e4m3 x e4m3 -> f32 (exact integer)", "data": "synthetic",
         "config": {"workload": WORKLOAD, "global_batch": c.N * world, "per_gpu_batch": c.N,
-                   "timed": "quantize (fp32 NHWC -> codes) + fused layer (codes -> next-layer codes)",
-                   "code_layout": "channel-blocked [N][C/16][H][W][16], one byte per code",
+                   "timed": "one launch per step: quantiser fused into the layer (fp32 NHWC -> next-layer codes)",
+                   "code_layout": "output codes channel-blocked [N][C/16][H][W][16], one byte per code",
                    "l2": "inputs larger than L2 (205.5 MB fp32, two buffers used in turn)",
                    "parallelism": f"replicas x{world}"},
         "images_per_s": whole_job_rate(c.N, world, ms_per_step),
         "pct_dense_int8_peak": 100.0 * value / world / fp8_peak,
-        "roofline": dominant,
-        "roofline_kernels": [roof_quant, roof_conv],
+        "roofline": roof_step,
+        "roofline_kernels": [roof_step],
         "clocks": clocks,
         "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": int(x_np.nbytes),
                 "d2h_bytes_per_step": int(np.prod(out_shape))},
-        "gpu_launches": 2 * K,
+        "gpu_launches": K,
     }
+    line["unfused_step"] = unfused_summary(unfused, c, pk, world)
     line["fp4_step"] = fp4_summary(fp4, c, pk, world)
     if resnet is not None:
         line["resnet18"] = resnet
