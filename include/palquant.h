@@ -262,8 +262,9 @@ pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, cons
  * produces), so the codes never pass through memory.  inv_s_host: G floats
  * (fl(1/s) of the input steps, >= 0), copied at call time.  Everything else as
  * palquant_layer_fused: w_packed_dev comes from palquant_pack_weights for the same
- * d, whose code_format (PQ_CODES_INT8 or PQ_CODES_C16) is the output codes'.
- * Needs stride 1 and 16-byte aligned x_dev; other shapes return PQ_EUNSUPPORTED. */
+ * d, whose code_format (PQ_CODES_INT8, PQ_CODES_C16, or PQ_CODES_C32F4 with its
+ * constraints) is the output codes'.  Needs stride 1 and 16-byte aligned x_dev;
+ * other shapes return PQ_EUNSUPPORTED. */
 pq_status palquant_quantize_layer_fused(const float* x_dev, const float* inv_s_host, const void* w_packed_dev,
                                         const pq_layer_desc* d, const float* m_out_host, const float* m_req_host,
                                         pq_shuffle shuf, const float* shortcut_dev, int32_t* acc_out_dev,

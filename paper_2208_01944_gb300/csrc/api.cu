@@ -138,9 +138,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const bool flat_shape = d->kh == 1 && d->kw == 1 && d->stride == 1 && d->pad == 0;
   const bool p2_ok = !p2 || (d->bits_a <= 2 && d->bits_out <= 2 && d->stride == 1 &&
                              (flat_shape ? (static_cast<int64_t>(d->H) * d->W) % 4 == 0 : d->W % 4 == 0));
-  // Quantise-on-load: stride 1, byte codes out (NHWC or channel-blocked), 32-channel
-  // K blocks, fp32 rows of 16-byte multiples for the TMA.
-  const bool quant_ok = !quant_in || (d->stride == 1 && !p2 && !f4 && (d->G * d->Cin_g) % 4 == 0);
+  // Quantise-on-load: stride 1, codes out one per byte (NHWC or channel-blocked) or
+  // as FP4 nibbles, K blocks of one MMA K step (32 channels, 64 for FP4: two 32-channel
+  // fp32 boxes), fp32 rows of 16-byte multiples for the TMA.
+  const bool quant_ok = !quant_in || (d->stride == 1 && !p2 && (d->G * d->Cin_g) % 4 == 0);
   bool ok = (d->code_format == PQ_CODES_INT8 || c16) && p2_ok && f4_ok && quant_ok && d->bits_a <= 4 && d->bits_w <= 4 && d->stride <= 2 &&
             d->pad < std::max(d->kh, d->kw) && d->Cin_g % 32 == 0 && d->Cout_g % 16 == 0 && taps <= pq::kMaxTaps &&
             static_cast<int64_t>(taps) * d->Cin_g * qa * qw < (1LL << 24);
@@ -248,9 +249,9 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
       // (32 bytes per position) must fit beside the weights (resident, or a
       // two-slice ring) and the epilogue staging
       const uint64_t npos = flat ? 128u : static_cast<uint64_t>(ht + rmax - rmin) * Wh;
-      const uint64_t w_unit = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk;
+      const uint64_t w_unit = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk / cpb;
       const uint64_t w_min = w_unit <= 112u * 1024u ? round_up(w_unit, 1024) : 2ull * round_up(32ull * p.Nblk, 1024);
-      const uint64_t need = 2ull * (round_up(npos * 128, 1024) + round_up(npos * 32, 1024)) + w_min +
+      const uint64_t need = 2ull * (cpb * round_up(npos * 128, 1024) + round_up(npos * 32, 1024)) + w_min +
                             pq::kEpiWarps * 2560ull + 1024;
       if (need > pq::kMaxSmem - 1024) continue;
     }
@@ -348,9 +349,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   }
   auto pk_stage_bytes = [&](int KC) -> uint32_t {
     if (quant_in) {
-      // fp32 box of KC channels x all positions of the stage (128-byte rows)
+      // KC/32 fp32 boxes of 32 channels x all positions of the stage (128-byte rows),
+      // each starting on a 1024-byte swizzle atom
       const uint64_t npos = flat ? static_cast<uint64_t>(p.flat_box) : static_cast<uint64_t>(p.Hd) * p.Wd;
-      return round_up(npos * KC * 4, 1024);
+      return static_cast<uint32_t>(KC / 32) * round_up(npos * 128, 1024);
     }
     if (!p2) return 0;
     const uint64_t rows = flat ? 1 : p.Hd;
@@ -365,7 +367,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // MMA issue loop is compiled for these K-step counts.
   for (int kc1 : {256, 128, 96, 64, 32}) {
     if (found) break;
-    if (quant_in && kc1 != 32) continue;  // one 128-byte fp32 row per position
+    // at most four 32-channel fp32 boxes per stage, a power-of-two chunk count
+    if (quant_in && (kc1 > 128 || kc1 == 96)) continue;
     const int kc = kc1 * cpb;
     if (d->Cin_g % kc != 0) continue;
     uint32_t sb, pb, l;
@@ -413,6 +416,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.chunk_shift = f4 ? 5 : 4;
   p.a_unpack = p2 ? 1 : 0;
   p.a_quant = quant_in ? 1 : 0;
+  p.q_box_bytes = quant_in ? round_up(static_cast<uint64_t>(flat ? p.flat_box : p.Hd * p.Wd) * 128, 1024) : 0;
   p.pk_box_w = pk_box_w;
   p.pk_off = pk_off;
   p.pk_stage_bytes = pk_stage_bytes(KC);

@@ -169,10 +169,14 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
         mbar_arrive_expect_tx(full, p.a_tx_bytes);
         const uint32_t dst = pk_base + ra.stage * p.pk_stage_bytes;
         const int ch0 = p.src_group[item.g] * p.Cin_g + kb * p.KC;
-        if (flat)
-          tma_load_3d(dst, tmA, ch0, item.rb * p.flat_box, item.n, full);
-        else
-          tma_load_4d(dst, tmA, ch0, p.w_coord, item.oh0(p.Ht) + p.h_off, item.n, full);
+        // one box per 32 channels of the K block, each on a 1024-byte swizzle atom
+        for (int b = 0; b < (p.KC >> 5); ++b) {
+          const uint32_t db = dst + static_cast<uint32_t>(b) * p.q_box_bytes;
+          if (flat)
+            tma_load_3d(db, tmA, ch0 + 32 * b, item.rb * p.flat_box, item.n, full);
+          else
+            tma_load_4d(db, tmA, ch0 + 32 * b, p.w_coord, item.oh0(p.Ht) + p.h_off, item.n, full);
+        }
         ra.advance();
         ++a_issued;
       } else if (a_tma && p.a_unpack) {
@@ -683,12 +687,17 @@ __device__ __forceinline__ long long codes_offset(const ConvParams& p, int pack,
 // 16-byte write to the operand plane of the half.  Positions outside the image
 // were zero-filled by the TMA unit: code 0, the zero padding.
 // --------------------------------------------------------------------------
+template <bool F4>
 __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t st_base,
                                            int64_t it0, int64_t it1, const WaitCtx& ctx) {
   const int tid = threadIdx.x - 32 * kFirstLoadWarp;
   const int lane = tid & 31;
   const int npos = p.mode == kModeFlat ? p.flat_box : p.Hd * p.Wd;
-  const int n_items = 2 * npos;
+  const uint32_t box_bytes = p.q_box_bytes;  // one 32-channel fp32 box (1024-byte aligned)
+  // items (position, chunk j): nch 16-byte chunks of the operand per position
+  // (16 channels each, 32 for FP4); nch is a power of two
+  const int lg_nch = __ffs(p.nch) - 1;
+  const int n_items = npos << lg_nch;
   const uint32_t plane = p.lbo_a;
   const float two_b = p.q_two_b;
   const uint32_t qmax2 = p.q_qmax2;
@@ -703,22 +712,45 @@ __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars
       const uint32_t src = st_base + r.stage * p.pk_stage_bytes;
       const uint32_t dst = a_base + r.stage * p.a_stage_bytes;
       for (int e = tid; e < n_items; e += 32 * kLoadWarps) {
-        const int pos = e >> 1, half = e & 1;
-        const uint32_t row = src + static_cast<uint32_t>(pos) * 128u;
-        uint32_t v[16];
+        const int pos = e >> lg_nch, j = e & (p.nch - 1);
+        const uint32_t out = dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(pos) * 16u;
+        if (F4) {
+          // FP4 nibbles: chunk j is box j, the whole 128-byte row: 32 codes packed
+          // two to a byte
+          const uint32_t row = src + static_cast<uint32_t>(j) * box_bytes + static_cast<uint32_t>(pos) * 128u;
+          uint32_t v[16];
+          uint2 packed[2];
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const uint32_t a = row + ((static_cast<uint32_t>(4 * half + k) ^ static_cast<uint32_t>(pos & 7)) << 4);
-          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
-                       : "=r"(v[4 * k]), "=r"(v[4 * k + 1]), "=r"(v[4 * k + 2]), "=r"(v[4 * k + 3])
-                       : "r"(a)
+          for (int h = 0; h < 2; ++h) {
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const uint32_t a = row + ((static_cast<uint32_t>(4 * h + k) ^ static_cast<uint32_t>(pos & 7)) << 4);
+              asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                           : "=r"(v[4 * k]), "=r"(v[4 * k + 1]), "=r"(v[4 * k + 2]), "=r"(v[4 * k + 3])
+                           : "r"(a)
+                           : "memory");
+            }
+            packed[h] = pack4_word(epi_codes16(v, m_sat, two_b, qmax2));
+          }
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(out), "r"(packed[0].x), "r"(packed[0].y),
+                       "r"(packed[1].x), "r"(packed[1].y)
+                       : "memory");
+        } else {
+          // byte codes: chunk j is the 16-channel half j & 1 of box j >> 1
+          const uint32_t row = src + static_cast<uint32_t>(j >> 1) * box_bytes + static_cast<uint32_t>(pos) * 128u;
+          uint32_t v[16];
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const uint32_t a = row + ((static_cast<uint32_t>(4 * (j & 1) + k) ^ static_cast<uint32_t>(pos & 7)) << 4);
+            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(v[4 * k]), "=r"(v[4 * k + 1]), "=r"(v[4 * k + 2]), "=r"(v[4 * k + 3])
+                         : "r"(a)
+                         : "memory");
+          }
+          const uint4 w = epi_codes16(v, m_sat, two_b, qmax2);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(out), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
                        : "memory");
         }
-        const uint4 w = epi_codes16(v, m_sat, two_b, qmax2);
-        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(dst + static_cast<uint32_t>(half) * plane +
-                                                                          static_cast<uint32_t>(pos) * 16u),
-                     "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
-                     : "memory");
       }
       fence_proxy_async_smem();
       __syncwarp();
@@ -1092,7 +1124,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   } else if (warp < kFirstEpiWarp && !p.a_tma) {
     loader_role(p, bars, a_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else if (warp < kFirstEpiWarp && p.a_quant) {
-    quant_role(p, bars, a_base, base + p.smem_pk_off, it0, it1,
+    quant_role<F4>(p, bars, a_base, base + p.smem_pk_off, it0, it1,
                WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else if (warp < kFirstEpiWarp && p.a_unpack) {
     unpack_role(p, bars, a_base, base + p.smem_pk_off, it0, it1,

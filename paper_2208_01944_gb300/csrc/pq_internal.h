@@ -64,6 +64,7 @@ struct ConvParams {
   float q_inv_sat[kMaxG];
   float q_two_b;
   uint32_t q_qmax2;  // Qp in both 16-bit halves
+  uint32_t q_box_bytes;  // staging bytes per 32-channel box (a multiple of 1024: the 128B swizzle atom)
   int pk_box_w, pk_off;
   uint32_t pk_stage_bytes, smem_pk_off;
   int a_tma;              // 1: warp 0 loads the A operand with one TMA per stage (channel-blocked codes, stride 1)

@@ -333,12 +333,12 @@ def test_fp4_code_helpers_roundtrip():
 
 
 def test_quantize_layer_fused_rules():
-    """Quantise-on-load covers stride-1 layers with byte codes out; the reciprocal
-    steps are required and must be finite and non-negative."""
+    """Quantise-on-load covers stride-1 layers with byte or FP4 codes out; the
+    reciprocal steps are required and must be finite and non-negative."""
     d = B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C16)
     for bad in [B.layer_desc(1, 8, 8, 2, 32, 32, 3, 2, 1, 2, 2, 2, code_format=B.PQ_CODES_C16),    # stride 2
                 B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C16P2),  # packed codes
-                B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C32F4)]:  # FP4 codes
+                B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C32F4)]:  # FP4, Cin_g 32
         with pytest.raises(B.PalquantError) as e:
             B.palquant_quantize_layer_fused(16, [1.0, 1.0], 16, bad, [1.0] * 2, [1.0] * 2, q_out_dev=16)
         assert e.value.status == B.PQ_EUNSUPPORTED

@@ -539,6 +539,25 @@ def test_quantize_layer_fused_matches_oracle(B, c, fmt):
     assert_layer_parity(c, ref, _run_quant_fused(B, c, ref, fmt))
 
 
+QF_F4_CASES = [
+    Case(1, 28, 28, 2, 64, 32, 3, 1, 1, seed=130),
+    Case(2, 13, 11, 3, 64, 96, 3, 1, 1, seed=131),                    # odd sizes
+    Case(2, 7, 9, 4, 128, 96, 1, 1, 0, seed=132),                     # flat, ragged last tile
+    Case(1, 12, 12, 2, 128, 256, 3, 1, 1, seed=133),                  # two K blocks, two output blocks
+    Case(2, 11, 10, 2, 64, 64, 3, 1, 1, shortcut=True, seed=134),     # shortcut add before ReLU
+    Case(2, 14, 14, 8, 64, 32, 3, 1, 1, kind=3, perm=(3, 0, 7, 1, 6, 2, 5, 4), seed=135),
+    Case(2, 36, 40, 2, 64, 64, 3, 1, 1, seed=136),                    # several row tiles per image
+    Case(2, 6, 6, 2, 64, 32, 3, 1, 1, bits_out=1, relu=False, kind=1, shift=-1, seed=137),
+]
+
+
+@pytest.mark.parametrize("c", QF_F4_CASES, ids=str)
+def test_quantize_layer_fused_fp4_matches_oracle(B, c):
+    """Quantise-on-load into packed FP4 operands (block-scaled FP4 MMAs), FP4 codes out."""
+    ref = prepare(c)
+    assert_layer_parity(c, ref, _run_quant_fused(B, c, ref, B.PQ_CODES_C32F4))
+
+
 @pytest.mark.parametrize("c", QF_CASES[:6], ids=str)
 def test_quantize_layer_fused_codes_only(B, c):
     ref = prepare(c)
