@@ -145,8 +145,7 @@ KERNEL_SOURCES = {
     "pq_conv_tc_kernel<quantise-on-load>": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
     "pq_quantize_c16": ["quantize.cu", "pq_device.cuh", "pq_internal.h"],
     "pq_conv_tc_kernel": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
-    "pq_quantize_c16<FP4 nibbles>": ["quantize.cu", "pq_device.cuh", "pq_internal.h"],
-    "pq_conv_tc_kernel<FP4>": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
+    "pq_conv_tc_kernel<FP4, quantise-on-load>": ["conv_tc.cu", "pq_device.cuh", "pq_internal.h"],
 }
 
 
@@ -608,9 +607,10 @@ def unfused_summary(r, c, pk, world):
 
 
 def measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf, K, world):
-    """The same step (quantise + fused layer, same steps and multipliers) with the
-    codes as packed FP4 nibbles (PQ_CODES_C32F4) and the block-scaled FP4 tensor-core
-    path: K timed steps after 3 warm-up steps, per-kernel CUDA events."""
+    """The same step (the quantiser fused into the layer, same steps and
+    multipliers) with packed FP4 operands and output codes (PQ_CODES_C32F4, the
+    block-scaled FP4 tensor path): K timed steps after 3 warm-up steps, events
+    around each launch."""
     import torch
 
     from paper_2208_01944_gb300 import binding as B
@@ -621,65 +621,54 @@ def measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf
     nbytes = B.palquant_packed_weight_bytes(d)
     wp = torch.empty(nbytes, dtype=torch.uint8, device=dev)
     B.palquant_pack_weights(w_np, d, inv_sw, wp, nbytes)
-    q = torch.empty(c.in_elems // 2, dtype=torch.uint8, device=dev)
     q_out = torch.empty(c.out_elems // 2, dtype=torch.uint8, device=dev)
 
     def launch(i):
-        B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt,
-                                stream=stream)
-        B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
+        B.palquant_quantize_layer_fused(xs[i & 1], inv_s, wp, d, m_out, m_req, shuf, None, None, None, q_out,
+                                        stream=stream)
 
     with torch.cuda.stream(stream):
         for i in range(3):
             launch(i)
     torch.cuda.synchronize(dev)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         start.record(stream)
         for i in range(K):
             ev[i][0].record(stream)
-            B.palquant_quantize_act(xs[i & 1], q, c.N, c.H, c.W, c.G, c.Cin_g, c.bits_a, inv_s, code_format=fmt,
-                                    stream=stream)
+            launch(i)
             ev[i][1].record(stream)
-            B.palquant_layer_fused(q, wp, d, m_out, m_req, shuf, None, None, None, q_out, stream=stream)
-            ev[i][2].record(stream)
         stop.record(stream)
     torch.cuda.synchronize(dev)
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
     return {"ms_per_step": max_over_ranks(start.elapsed_time(stop) / K, world, dev),
-            "t_quant": sum(e[0].elapsed_time(e[1]) for e in ev) / K,
-            "t_conv": sum(e[1].elapsed_time(e[2]) for e in ev) / K}
+            "t_step": sum(e[0].elapsed_time(e[1]) for e in ev) / K}
 
 
 def fp4_summary(r, c, pk, world):
-    """The FP4 step's throughput and the rooflines of its two kernels.  The layer's
-    tensor instructions are FP4 (kind::mxf4), so its compute peak is the dense FP4
-    rate: the measured bf16 burst x 6 (nominal 13.5 / 2.25 PFLOP/s); its bytes are
-    half those of one code per byte."""
+    """The FP4 step's throughput and the roofline of its one kernel: HBM-bound on
+    the fp32 input and the nibble codes out; its tensor instructions are FP4
+    (kind::mxf4), whose dense peak is the measured bf16 burst x 6 (nominal 13.5 /
+    2.25 PFLOP/s)."""
     fp4_peak = 6.0 * pk["bf16_tflops"]
-    q_bytes = c.in_elems * 4 + c.in_elems // 2
-    conv_bytes = c.in_elems // 2 + c.out_elems // 2 + c.weight_elems // 2
-    conv_tops = c.int_ops / (r["t_conv"] / 1e3) / 1e12
-    quant_gbs = q_bytes / (r["t_quant"] / 1e3) / 1e9
-    conv_gbs = conv_bytes / (r["t_conv"] / 1e3) / 1e9
+    step_bytes = c.in_elems * 4 + c.out_elems // 2 + c.weight_elems // 2
+    gbs = step_bytes / (r["t_step"] / 1e3) / 1e9
+    tops = c.int_ops / (r["t_step"] / 1e3) / 1e12
     return {
         "value": whole_job_rate(c.int_ops, world, r["ms_per_step"]) / 1e12, "unit": UNIT,
         "ms_per_step": r["ms_per_step"],
+        "timed": "one launch per step: quantiser fused into the layer, packed FP4 operands and codes",
         "code_layout": "packed FP4 nibbles [N][C/32][H][W][16 B], two 2-bit codes per byte",
-        "dtype": "2-bit codes as FP4 e2m1 x e2m1 weights, block scales 2^-4 -> f32 (exact integer)",
+        "dtype": "fp32 activations -> 2-bit codes as FP4 e2m1 x e2m1 weights, block scales 2^-4 -> f32 (exact)",
         "roofline_kernels": [
-            {"kernel": "pq_quantize_c16<FP4 nibbles>", "bound": "hbm", "achieved": quant_gbs, "peak": pk["hbm_gbs"],
-             "unit": "GB/s", "frac": quant_gbs / pk["hbm_gbs"],
-             "traffic": dram_traffic("pq_quantize_c16<FP4 nibbles>"), "algorithmic_bytes": q_bytes,
-             "avg_launch_ms": r["t_quant"], "peak_source": f"{pk['source']} HBM copy bandwidth"},
-            {"kernel": "pq_conv_tc_kernel<FP4>", "bound": "tensor", "achieved": conv_tops, "peak": fp4_peak,
-             "unit": "TFLOP/s", "frac": conv_tops / fp4_peak, "traffic": dram_traffic("pq_conv_tc_kernel<FP4>"),
-             "algorithmic_ops": c.int_ops,
-             "algorithmic_bytes": conv_bytes, "avg_launch_ms": r["t_conv"], "hbm_frac": conv_gbs / pk["hbm_gbs"],
-             "peak_source": f"{pk['source']} bf16 burst x 6 (dense FP4, nominal 13.5 / 2.25 PFLOP/s)"}],
-        "gpu_launches": 2,
+            {"kernel": "pq_conv_tc_kernel<FP4> (quantise on load)", "bound": "hbm", "achieved": gbs,
+             "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": gbs / pk["hbm_gbs"],
+             "traffic": dram_traffic("pq_conv_tc_kernel<FP4, quantise-on-load>"), "algorithmic_bytes": step_bytes,
+             "algorithmic_ops": c.int_ops, "avg_launch_ms": r["t_step"], "tensor_tops": tops,
+             "tensor_frac_fp4": tops / fp4_peak, "peak_source": f"{pk['source']} HBM copy bandwidth"}],
+        "gpu_launches": 1,
     }
 
 
