@@ -111,8 +111,11 @@ struct Phase {
 
 // quant_in: the layer's input is fp32 NHWC activations, quantised on load (the
 // copy warps quantise TMA-staged 32-channel fp32 boxes into the operand stages).
+// direct_out: the call writes channel-blocked codes only (no int32 or fp32
+// outputs), which the epilogue stores straight from registers, so the plan
+// reserves no per-warp staging for it.
 pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, std::vector<Phase>* phases_out,
-                    bool quant_in = false) {
+                    bool quant_in = false, bool direct_out = false) {
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
   pq_conv_plan plan;
@@ -252,7 +255,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
       const uint64_t w_unit = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk / cpb;
       const uint64_t w_min = w_unit <= 112u * 1024u ? round_up(w_unit, 1024) : 2ull * round_up(32ull * p.Nblk, 1024);
       const uint64_t need = 2ull * (cpb * round_up(npos * 128, 1024) + round_up(npos * 32, 1024)) + w_min +
-                            pq::kEpiWarps * 2560ull + 1024;
+                            (direct_out ? 0ull : pq::kEpiWarps * 2560ull) + 1024;
       if (need > pq::kMaxSmem - 1024) continue;
     }
     const int units = MT * units_per_acc;
@@ -334,7 +337,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // TMA loads the activation operand as it is (not unpacked, not quantised).
   const bool third_group =
       !quant_in && !p2 && c16 && d->stride == 1 && (flat ? p.flat_box <= 256 : p.Wd <= 128);
-  const uint32_t stage_total = warp_stage * (third_group ? pq::kEpiWarps + pq::kLoadWarps : pq::kEpiWarps);
+  const uint32_t stage_total =
+      direct_out ? 0u : warp_stage * (third_group ? pq::kEpiWarps + pq::kLoadWarps : pq::kEpiWarps);
   const uint32_t bar_bytes = 1024;  // barriers, abort flag, TMEM slot (generous)
   const uint64_t unit_bytes = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk / cpb;
   // Packed codes: a staging stage per operand stage holding the TMA box of 32-bit
@@ -676,7 +680,10 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
     return PQ_EINVAL;
   ConvParams p;
   std::vector<Phase> phases;
-  st = plan_conv(d, &p, nullptr, &phases, inv_s_in != nullptr);
+  // Channel-blocked codes as the only output are stored from registers (the
+  // per-channel scatter of the channel shuffle is unstaged too).
+  const bool direct_out = acc_out_dev == nullptr && y_out_dev == nullptr && d->code_format != PQ_CODES_INT8;
+  st = plan_conv(d, &p, nullptr, &phases, inv_s_in != nullptr, direct_out);
   if (st != PQ_OK) return st;
   if (inv_s_in != nullptr) {
     // reciprocal steps scaled by 2^-b (exact: a power of two) for the saturating form

@@ -681,11 +681,12 @@ __device__ __forceinline__ long long codes_offset(const ConvParams& p, int pack,
 // Quantise-on-load role (warps 2-5): each staged box holds, per position of the
 // stage, the 32 fp32 activations of the K block as one 128-byte row, swizzled
 // 128B (16-byte chunk c of row r at chunk c ^ (r & 7), the rows' bank groups
-// spread).  Thread items are (position, 16-channel half): four 16-byte reads,
+// spread).  Thread items are (position, box): eight 16-byte reads of the row,
 // the codes clamp(rint(x * fl(1/s)), 0, Qp) of the input group (one fp32
-// multiply, the saturating form of the epilogue's conversion, NaN -> 0), one
-// 16-byte write to the operand plane of the half.  Positions outside the image
-// were zero-filled by the TMA unit: code 0, the zero padding.
+// multiply, the saturating form of the epilogue's conversion, NaN -> 0), and
+// 16-byte writes to the operand planes: one per 16-channel half for byte codes,
+// one for the row's 32 FP4 nibbles.  Positions outside the image were
+// zero-filled by the TMA unit: code 0, the zero padding.
 // --------------------------------------------------------------------------
 template <bool F4>
 __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t st_base,
@@ -694,10 +695,10 @@ __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars
   const int lane = tid & 31;
   const int npos = p.mode == kModeFlat ? p.flat_box : p.Hd * p.Wd;
   const uint32_t box_bytes = p.q_box_bytes;  // one 32-channel fp32 box (1024-byte aligned)
-  // items (position, chunk j): nch 16-byte chunks of the operand per position
-  // (16 channels each, 32 for FP4); nch is a power of two
-  const int lg_nch = __ffs(p.nch) - 1;
-  const int n_items = npos << lg_nch;
+  // items (position, box j): one 128-byte row of 32 channels each; the stage
+  // holds KC / 32 boxes, a power of two
+  const int lg_nbox = __ffs(p.KC >> 5) - 1;
+  const int n_items = npos << lg_nbox;
   const uint32_t plane = p.lbo_a;
   const float two_b = p.q_two_b;
   const uint32_t qmax2 = p.q_qmax2;
@@ -712,12 +713,12 @@ __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars
       const uint32_t src = st_base + r.stage * p.pk_stage_bytes;
       const uint32_t dst = a_base + r.stage * p.a_stage_bytes;
       for (int e = tid; e < n_items; e += 32 * kLoadWarps) {
-        const int pos = e >> lg_nch, j = e & (p.nch - 1);
-        const uint32_t out = dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(pos) * 16u;
+        const int pos = e >> lg_nbox, j = e & ((1 << lg_nbox) - 1);
+        const uint32_t row = src + static_cast<uint32_t>(j) * box_bytes + static_cast<uint32_t>(pos) * 128u;
         if (F4) {
-          // FP4 nibbles: chunk j is box j, the whole 128-byte row: 32 codes packed
+          // FP4 nibbles: operand chunk j is box j, the whole row: 32 codes packed
           // two to a byte
-          const uint32_t row = src + static_cast<uint32_t>(j) * box_bytes + static_cast<uint32_t>(pos) * 128u;
+          const uint32_t out = dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(pos) * 16u;
           uint32_t v[16];
           uint2 packed[2];
 #pragma unroll
@@ -736,19 +737,30 @@ __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars
                        "r"(packed[1].x), "r"(packed[1].y)
                        : "memory");
         } else {
-          // byte codes: chunk j is the 16-channel half j & 1 of box j >> 1
-          const uint32_t row = src + static_cast<uint32_t>(j >> 1) * box_bytes + static_cast<uint32_t>(pos) * 128u;
-          uint32_t v[16];
+          // byte codes: the row's two 16-channel halves are operand chunks 2j and
+          // 2j + 1 (all eight reads issued before the conversions)
+          const uint32_t out = dst + static_cast<uint32_t>(2 * j) * plane + static_cast<uint32_t>(pos) * 16u;
+          uint32_t v[16], u[16];
 #pragma unroll
           for (int k = 0; k < 4; ++k) {
-            const uint32_t a = row + ((static_cast<uint32_t>(4 * (j & 1) + k) ^ static_cast<uint32_t>(pos & 7)) << 4);
+            const uint32_t a = row + ((static_cast<uint32_t>(k) ^ static_cast<uint32_t>(pos & 7)) << 4);
+            const uint32_t b = row + ((static_cast<uint32_t>(4 + k) ^ static_cast<uint32_t>(pos & 7)) << 4);
             asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
                          : "=r"(v[4 * k]), "=r"(v[4 * k + 1]), "=r"(v[4 * k + 2]), "=r"(v[4 * k + 3])
                          : "r"(a)
                          : "memory");
+            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(u[4 * k]), "=r"(u[4 * k + 1]), "=r"(u[4 * k + 2]), "=r"(u[4 * k + 3])
+                         : "r"(b)
+                         : "memory");
           }
-          const uint4 w = epi_codes16(v, m_sat, two_b, qmax2);
-          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(out), "r"(w.x), "r"(w.y), "r"(w.z), "r"(w.w)
+          const uint4 w0 = epi_codes16(v, m_sat, two_b, qmax2);
+          const uint4 w1 = epi_codes16(u, m_sat, two_b, qmax2);
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(out), "r"(w0.x), "r"(w0.y), "r"(w0.z),
+                       "r"(w0.w)
+                       : "memory");
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(out + plane), "r"(w1.x), "r"(w1.y), "r"(w1.z),
+                       "r"(w1.w)
                        : "memory");
         }
       }

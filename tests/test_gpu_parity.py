@@ -558,10 +558,37 @@ def test_quantize_layer_fused_fp4_matches_oracle(B, c):
     assert_layer_parity(c, ref, _run_quant_fused(B, c, ref, B.PQ_CODES_C32F4))
 
 
-@pytest.mark.parametrize("c", QF_CASES[:6], ids=str)
+@pytest.mark.parametrize("c", QF_CASES, ids=str)
 def test_quantize_layer_fused_codes_only(B, c):
+    """Channel-blocked codes as the only output: the plan reserves no epilogue
+    staging and takes larger tiles than with int32 / fp32 outputs."""
     ref = prepare(c)
     assert_layer_parity(c, ref, _run_quant_fused(B, c, ref, 2, outputs=("q",)))
+
+
+@pytest.mark.parametrize("c", QF_F4_CASES, ids=str)
+def test_quantize_layer_fused_fp4_codes_only(B, c):
+    ref = prepare(c)
+    assert_layer_parity(c, ref, _run_quant_fused(B, c, ref, B.PQ_CODES_C32F4, outputs=("q",)))
+
+
+QF_FULL = [(n, c) for n, c in FULL if c.stride == 1]
+
+
+@pytest.mark.parametrize("fmt", [2, 4], ids=["c16", "fp4"])
+@pytest.mark.parametrize("name,cfg", QF_FULL, ids=[n for n, _ in QF_FULL])
+def test_full_size_quantize_layer_fused_sampled(B, name, cfg, fmt):
+    """The benchmarked step at full size, as the benchmark launches it: fp32
+    activations in, the next layer's codes out (codes only), sampled pixels
+    against the oracle's quantiser followed by its layer."""
+    if fmt == 4 and (cfg.bits_a > 2 or cfg.Cin_g % 64 or cfg.Cout_g % 32 or cfg.shuffle_kind == 2):
+        pytest.skip("outside the packed-FP4 format")
+    c = Case(cfg.N, cfg.H, cfg.W, cfg.G, cfg.Cin_g, cfg.Cout_g, cfg.k, cfg.stride, cfg.pad, bits=cfg.bits_a,
+             kind=cfg.shuffle_kind, shift=cfg.shuffle_shift, relu=cfg.relu, seed=0)
+    pix = _sample_pixels(c.N, c.Ho, c.Wo, 3000, 3)
+    ref = prepare(c, sample_pix=pix)
+    got = _run_quant_fused(B, c, ref, fmt, outputs=("q",))
+    assert_layer_parity(c, ref, got, pix)
 
 
 def test_quantize_layer_fused_special_inputs(B):
