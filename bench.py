@@ -609,8 +609,8 @@ def unfused_summary(r, c, pk, world):
 def measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf, K, world):
     """The same step (the quantiser fused into the layer, same steps and
     multipliers) with packed FP4 operands and output codes (PQ_CODES_C32F4, the
-    block-scaled FP4 tensor path): K timed steps after 3 warm-up steps, events
-    around each launch."""
+    block-scaled FP4 tensor path): K timed steps after 3 warm-up steps, one
+    launch each, timed as a region (average launch duration = region / K)."""
     import torch
 
     from paper_2208_01944_gb300 import binding as B
@@ -631,20 +631,17 @@ def measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf
         for i in range(3):
             launch(i)
     torch.cuda.synchronize(dev)
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         start.record(stream)
         for i in range(K):
-            ev[i][0].record(stream)
             launch(i)
-            ev[i][1].record(stream)
         stop.record(stream)
     torch.cuda.synchronize(dev)
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
-    return {"ms_per_step": max_over_ranks(start.elapsed_time(stop) / K, world, dev),
-            "t_step": sum(e[0].elapsed_time(e[1]) for e in ev) / K}
+    t = start.elapsed_time(stop) / K
+    return {"ms_per_step": max_over_ranks(t, world, dev), "t_step": t}
 
 
 def fp4_summary(r, c, pk, world):
@@ -730,9 +727,10 @@ def run_ours(args, rank, world, local_rank):
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
 
-    # ---- timed region: K steps, per-launch events on the launching stream
+    # ---- timed region: K steps (one launch each) between two events on the
+    # launching stream; the step's average launch duration is the region / K
+    # (launch gaps included), with no events between the launches
     K = args.steps
-    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     sampler = ClockSampler(local_rank)
     if world > 1:
@@ -743,9 +741,7 @@ def run_ours(args, rank, world, local_rank):
     with torch.cuda.stream(stream):
         start.record(stream)
         for i in range(K):
-            ev[i][0].record(stream)
             step(i, stream)
-            ev[i][1].record(stream)
         stop.record(stream)
     torch.cuda.synchronize(dev)
     st = B.palquant_sync_check(stream)
@@ -758,7 +754,7 @@ def run_ours(args, rank, world, local_rank):
     if world > 1:
         dist.barrier()
     elapsed_ms = start.elapsed_time(stop)
-    t_step = sum(e[0].elapsed_time(e[1]) for e in ev) / K
+    t_step = elapsed_ms / K
     elapsed_ms = max_over_ranks(elapsed_ms, world, dev)
     ms_per_step = elapsed_ms / K
     ops_step = c.int_ops
