@@ -68,6 +68,8 @@ def _declare(lib):
     lib.oracle_epilogue_scales.restype = _I32
     lib.oracle_epilogue_scales.argtypes = [_I32, _P, _P, ctypes.c_double, _P, _I32, _I32, _P, _P, _P]
     lib.oracle_quantize_weights_odd.argtypes = [_P, _P, _I32, _I64, _I32, _P]
+    lib.oracle_fake_quant_fwd.argtypes = [_P, _P, _I64, _I32, _I64, _I32, _I32, _P, _P]
+    lib.oracle_fake_quant_bwd.argtypes = [_P, _P, _P, _P, _P, _I64, _I32, _I64, _I32, _I32, _P, _P]
     lib.oracle_conv2d_f32.argtypes = [_P, _P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _I32, _I32, _I32]
     lib.oracle_maxpool_f32.argtypes = [_P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _I32]
     lib.oracle_avgpool_f32.argtypes = [_P, _P, _I64, _I64, _I64, _I32]
@@ -378,3 +380,32 @@ def quantize_weights_odd(w: np.ndarray, bits: int, u, L=None) -> np.ndarray:
     wq = np.empty(w.shape, dtype=np.int8)
     L.oracle_quantize_weights_odd(_ptr(w), _ptr(wq), G, w.size // G, bits, _ptr(u))
     return wq
+
+
+def fake_quant_forward(x: np.ndarray, G: int, bits: int, kind: int, l, u, L=None) -> np.ndarray:
+    """Quantisation-aware training forward (Eq. 2-3 with learned bounds l, u per
+    group; kind 0 activations in [0, 1], kind 1 weights in [-1, 1]).  x: [..., G*Cg]."""
+    L = L or lib()
+    x = _f32(x)
+    l, u = _f32(l), _f32(u)
+    C = x.shape[-1]
+    assert C % G == 0 and l.shape == (G,) and u.shape == (G,)
+    out = np.empty_like(x)
+    L.oracle_fake_quant_fwd(_ptr(x), _ptr(out), x.size // C, G, C // G, bits, kind, _ptr(l), _ptr(u))
+    return out
+
+
+def fake_quant_backward(x: np.ndarray, dy: np.ndarray, G: int, bits: int, kind: int, l, u, L=None):
+    """Its straight-through backward: (dx fp32, dl [G] float64, du [G] float64)."""
+    L = L or lib()
+    x, dy = _f32(x), _f32(dy)
+    l, u = _f32(l), _f32(u)
+    assert x.shape == dy.shape
+    C = x.shape[-1]
+    assert C % G == 0 and l.shape == (G,) and u.shape == (G,)
+    dx = np.empty_like(x)
+    dl = np.empty(G, dtype=np.float64)
+    du = np.empty(G, dtype=np.float64)
+    L.oracle_fake_quant_bwd(_ptr(x), _ptr(dy), _ptr(dx), _ptr(dl), _ptr(du), x.size // C, G, C // G, bits, kind,
+                            _ptr(l), _ptr(u))
+    return dx, dl, du

@@ -46,6 +46,19 @@ MUTATIONS = {
                             "wq[g * per_group + i] = (int8_t)((int)r - qp);"),
     # the clip range shifted by u twice
     "odd_levels_shift": ("float t = (w[g * per_group + i] + u[g]) * k;", "float t = (w[g * per_group + i] + 2.0f * u[g]) * k;"),
+    # quantisation-aware training: weights de-quantised without the factor 2
+    "qat_weight_factor": ("xhat[i] = kind ? 2.0f * (v - 0.5f) : v;", "xhat[i] = kind ? (v - 0.5f) : v;"),
+    # rounding half up instead of half to even
+    "qat_round_half_up": ("float xq = rintf(xn * qp);", "float xq = floorf(xn * qp + 0.5f);"),
+    # the straight-through gradient also at the clip bounds
+    "qat_inside_inclusive": ("if (t > 0.0f && t < 1.0f) {", "if (t >= 0.0f && t <= 1.0f) {"),
+    # the gradient of u with the wrong sign
+    "qat_du_sign": ("du[g] = -c / (rd * rd) * sb;", "du[g] = c / (rd * rd) * sb;"),
+    # the gradient of l measured from the wrong bound
+    "qat_dl_bound": ("sa += (double)dy[i] * ((double)x[i] - (double)u[g]);",
+                     "sa += (double)dy[i] * ((double)x[i] - (double)l[g]);"),
+    # the input gradient without the de-quantisation factor
+    "qat_dx_factor": ("const float k = (float)c / r;", "const float k = 1.0f / r;"),
     # step from the mean without the factor 2
     "act_step_factor": ("s_out[g] = (float)(2.0 * mean / sqrt(qp));\n    }\n}\n\nvoid oracle_weight_step",
                         "s_out[g] = (float)(mean / sqrt(qp));\n    }\n}\n\nvoid oracle_weight_step"),
@@ -88,6 +101,24 @@ def _pins_pass(L) -> bool:
         acc = np.arange(12, dtype=np.int64).reshape(1, 12)
         _, y2, _ = oracle.epilogue(acc, 3, [1.0, 1.0, 1.0], None, kind=2, relu=False, L=L)
         if list(y2[0]) != [float(v) for v in np.arange(12).reshape(3, 4).T.ravel()]:
+            return False
+        # quantisation-aware training: forward hand cases (both kinds, a shifted grid)
+        xq = np.array([[0.5, 1.0, 2.0, 3.5, 4.0, 5.0, -1.0]], np.float32)
+        third = np.float32(1) / np.float32(3)
+        if list(oracle.fake_quant_forward(xq, 1, 2, 0, [0.0], [4.0], L=L)[0]) != \
+                [0.0, third, np.float32(2) / np.float32(3), 1.0, 1.0, 1.0, 0.0]:
+            return False
+        if list(oracle.fake_quant_forward(xq, 1, 2, 1, [0.0], [4.0], L=L)[0][[0, 3, 6]]) != [-1.0, 1.0, -1.0]:
+            return False
+        if list(oracle.fake_quant_forward(np.array([[-0.5, 0.0, 0.5]], np.float32), 1, 1, 0, [-2.0], [2.0],
+                                          L=L)[0]) != [0.0, 0.0, 1.0]:
+            return False
+        # backward hand cases (the bound t = 1 is outside; weights carry the factor 2)
+        dx, dl, du = oracle.fake_quant_backward(xq, np.ones_like(xq), 1, 2, 0, [0.0], [4.0], L=L)
+        if list(dx[0]) != [0.25, 0.25, 0.25, 0.25, 0.0, 0.0, 0.0] or dl[0] != -9.0 / 16 or du[0] != -7.0 / 16:
+            return False
+        dx, dl, du = oracle.fake_quant_backward(xq, np.ones_like(xq), 1, 2, 1, [0.0], [4.0], L=L)
+        if list(dx[0][:4]) != [0.5] * 4 or dl[0] != -18.0 / 16 or du[0] != -14.0 / 16:
             return False
         # constant-tensor step closed form
         c = np.full((1, 2, 2, 4), 1.5, dtype=np.float32)
