@@ -143,27 +143,29 @@ void oracle_quantize_weights(const float* w, int8_t* wq, int G, int Cout_g, int 
 /* Quantisation-aware training forward (Sec. 3.2 Eq. 2-3; Sec. 5: the bounds l,
  * u are learned, the rounding is passed by the straight-through estimator).
  * x is [P][G*Cg], group g = channel / Cg, bounds l[g] < u[g].  Per element, in
- * fp32 with one IEEE rounding per operation:
- *   t = (x - l) / (u - l),  x_n = min(max(t, 0), 1)  (NaN -> 0),
- *   x_q = rint(x_n * (2^b - 1))                      (half to even),
- *   kind 0 (activations): x_hat = x_q / (2^b - 1)            in [0, 1]
- *   kind 1 (weights):     x_hat = 2 * (x_q / (2^b - 1) - 0.5) in [-1, 1]
+ * fp32 with one IEEE rounding per operation, the divisions taken as multiplies
+ * by fp32 reciprocals (as the inference quantiser takes x / s as x * fl(1/s)):
+ *   t = (x - l) * fl(1 / fl(u - l)),  x_n = min(max(t, 0), 1)  (NaN -> 0),
+ *   x_q = rint(x_n * (2^b - 1))                                (half to even),
+ *   kind 0 (activations): x_hat = x_q * fl(1 / (2^b - 1))            in [0, 1]
+ *   kind 1 (weights):     x_hat = 2 * (x_q * fl(1 / (2^b - 1)) - 0.5) in [-1, 1]
  * (Eq. 3 printed with its two cases swapped; activations are the non-negative
  * ones.) */
-static float fq_t(float x, float l, float r) { return (x - l) / r; }
+static float fq_t(float x, float l, float inv_r) { return (x - l) * inv_r; }
 
 void oracle_fake_quant_fwd(const float* x, float* xhat, int64_t P, int G, int64_t Cg, int bits, int kind,
                            const float* l, const float* u) {
     const float qp = (float)((1 << bits) - 1);
+    const float inv_qp = 1.0f / qp;
     const int64_t C = (int64_t)G * Cg;
     for (int64_t p = 0; p < P; ++p) {
         for (int g = 0; g < G; ++g) {
-            const float r = u[g] - l[g];
+            const float inv_r = 1.0f / (u[g] - l[g]);
             for (int64_t j = 0; j < Cg; ++j) {
                 const int64_t i = p * C + (int64_t)g * Cg + j;
-                float xn = fminf(fmaxf(fq_t(x[i], l[g], r), 0.0f), 1.0f);
+                float xn = fminf(fmaxf(fq_t(x[i], l[g], inv_r), 0.0f), 1.0f);
                 float xq = rintf(xn * qp);
-                float v = xq / qp;
+                float v = xq * inv_qp;
                 xhat[i] = kind ? 2.0f * (v - 0.5f) : v;
             }
         }
@@ -173,7 +175,7 @@ void oracle_fake_quant_fwd(const float* x, float* xhat, int64_t P, int G, int64_
 /* Its backward with the straight-through estimator: the rounding passes the
  * gradient unchanged, the clip does not (zero outside 0 < t < 1).  With the
  * de-quantisation factor c = 1 (activations) or 2 (weights) and r = u - l:
- *   dx     = dy * fl(c / r)                     (fp32, elements with 0 < t < 1; else 0)
+ *   dx     = dy * c * fl(1 / fl(r))             (fp32, elements with 0 < t < 1; else 0)
  *   dl[g]  = c / r^2 * sum over those elements of group g of dy * (x - u)
  *   du[g]  = -c / r^2 * sum over those elements of group g of dy * (x - l)
  * (d t / d l = (x - u) / r^2, d t / d u = -(x - l) / r^2), the sums and the
@@ -185,14 +187,14 @@ void oracle_fake_quant_bwd(const float* x, const float* dy, float* dx, double* d
     const int64_t C = (int64_t)G * Cg;
     const double c = kind ? 2.0 : 1.0;
     for (int g = 0; g < G; ++g) {
-        const float r = u[g] - l[g];
-        const float k = (float)c / r;
+        const float inv_r = 1.0f / (u[g] - l[g]);
+        const float k = (float)c * inv_r;
         const double rd = (double)u[g] - (double)l[g];
         double sa = 0.0, sb = 0.0;
         for (int64_t p = 0; p < P; ++p) {
             for (int64_t j = 0; j < Cg; ++j) {
                 const int64_t i = p * C + (int64_t)g * Cg + j;
-                const float t = fq_t(x[i], l[g], r);
+                const float t = fq_t(x[i], l[g], inv_r);
                 if (t > 0.0f && t < 1.0f) {
                     dx[i] = dy[i] * k;
                     sa += (double)dy[i] * ((double)x[i] - (double)u[g]);

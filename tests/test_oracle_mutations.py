@@ -58,7 +58,7 @@ MUTATIONS = {
     "qat_dl_bound": ("sa += (double)dy[i] * ((double)x[i] - (double)u[g]);",
                      "sa += (double)dy[i] * ((double)x[i] - (double)l[g]);"),
     # the input gradient without the de-quantisation factor
-    "qat_dx_factor": ("const float k = (float)c / r;", "const float k = 1.0f / r;"),
+    "qat_dx_factor": ("const float k = (float)c * inv_r;", "const float k = inv_r;"),
     # step from the mean without the factor 2
     "act_step_factor": ("s_out[g] = (float)(2.0 * mean / sqrt(qp));\n    }\n}\n\nvoid oracle_weight_step",
                         "s_out[g] = (float)(mean / sqrt(qp));\n    }\n}\n\nvoid oracle_weight_step"),
