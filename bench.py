@@ -416,7 +416,44 @@ def measure_layer_configs(dev, args):
                                             "frac_hbm": b4 / (ms4 / 1e3) / 1e9 / pk["hbm_gbs"], "buffer_sets": n_sets}
         del xs, qq, x, qq4
     torch.cuda.empty_cache()
+    out.update(measure_qat(dev, stream, timed, pk))
     return out
+
+
+def measure_qat(dev, stream, timed, pk):
+    """Quantisation-aware training of the quantiser on the config-1 activation
+    tensor (64x56x56x256 fp32, G = 4, learned bounds l, u per group): the forward
+    (8 bytes per element) and the straight-through backward with the gradients of l
+    and u (12 bytes per element); each tensor is larger than L2, two sets rotate."""
+    import numpy as np
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300 import workloads
+
+    c = workloads.CONFIG1
+    P, G, Cg = c.N * c.H * c.W, c.G, c.Cin_g
+    n = P * G * Cg
+    l = np.full(G, 0.05, np.float32)
+    u = np.full(G, 2.0, np.float32)
+    xs = [torch.randn((P, G * Cg), device=dev).abs_() for _ in range(2)]
+    dys = [torch.randn((P, G * Cg), device=dev) for _ in range(2)]
+    outs = [torch.empty((P, G * Cg), device=dev) for _ in range(2)]
+    dl = torch.empty(G, dtype=torch.float64, device=dev)
+    du = torch.empty(G, dtype=torch.float64, device=dev)
+    sb = B.palquant_fake_quant_scratch_bytes(P, G, Cg)
+    scratch = torch.empty(sb, dtype=torch.uint8, device=dev)
+    ms_f = timed(lambda i: B.palquant_fake_quant_forward(xs[i], outs[i], P, G, Cg, c.bits_a, 0, l, u, stream=stream), 2)
+    ms_b = timed(lambda i: B.palquant_fake_quant_backward(xs[i], dys[i], outs[i], dl, du, P, G, Cg, c.bits_a, 0, l, u,
+                                                          scratch, sb, stream=stream), 2)
+    res = {}
+    for key, ms, byt in (("qat_forward_config1", ms_f, 8 * n), ("qat_backward_config1", ms_b, 12 * n)):
+        gbs = byt / (ms / 1e3) / 1e9
+        res[key] = {"shape": f"{c.N}x{c.H}x{c.W}x{G * Cg} fp32, G={G}, b={c.bits_a}", "us": ms * 1e3, "gbs": gbs,
+                    "frac_hbm": gbs / pk["hbm_gbs"], "algorithmic_bytes": byt, "buffer_sets": 2}
+    del xs, dys, outs
+    torch.cuda.empty_cache()
+    return res
 
 
 def measure_bitsplit_vs_palquant(dev, stream, timed, pk, fp8_peak):

@@ -383,6 +383,52 @@ pq_status palquant_linear_f32(const float* x_dev, const float* w_dev, float* y_d
                               int32_t Cout, pq_stream_t stream);
 
 /* ------------------------------------------------------------------------ */
+/* Quantisation-aware training of the quantiser (Sec. 3.2 Eq. 2-3, Sec. 5).  */
+/* ------------------------------------------------------------------------ */
+
+/* Fake quantisation with learned per-group bounds (the training-time form of
+ * Eq. 2-3; Sec. 5 learns l and u through back-propagation).  x_dev is
+ * [P][G*Cg] fp32 (group g = channel / Cg: NHWC activations with P = N*H*W, or
+ * weights with P = 1 and Cg = the group's weight count); l_host, u_host hold G
+ * floats with l[g] < u[g] (finite).  Per element, in fp32 with one rounding per
+ * operation and the divisions taken as multiplies by fp32 reciprocals:
+ *   t   = (x - l) * fl(1 / fl(u - l)),   x_n = min(max(t, 0), 1)   (NaN -> 0)
+ *   x_q = rint(x_n * (2^bits - 1))                                 (half to even)
+ *   kind 0 (activations): xhat = x_q * fl(1 / (2^bits - 1))              in [0, 1]
+ *   kind 1 (weights):     xhat = 2 * (x_q * fl(1 / (2^bits - 1)) - 0.5)  in [-1, 1]
+ * (Eq. 3 is printed with its two cases swapped; the activations are the
+ * non-negative ones.)  Requires Cg % 4 == 0, 16-byte aligned pointers,
+ * 1 <= bits <= 8, G <= 64 and P * Cg / 4 < 2^32 (else PQ_EUNSUPPORTED); P = 0
+ * does nothing.  Bound by HBM: 8 bytes per element.  Asynchronous on the
+ * stream. */
+pq_status palquant_fake_quant_forward(const float* x_dev, float* xhat_dev, int64_t P, int32_t G, int32_t Cg,
+                                      int32_t bits, int32_t kind, const float* l_host, const float* u_host,
+                                      pq_stream_t stream);
+
+/* Bytes of device scratch palquant_fake_quant_backward needs (16-byte aligned). */
+size_t palquant_fake_quant_scratch_bytes(int64_t P, int32_t G, int32_t Cg);
+
+/* Its backward with the straight-through estimator: the rounding passes the
+ * gradient unchanged, the clip does not.  With c = 1 (kind 0) or 2 (kind 1),
+ * r = u - l and t as in the forward:
+ *   dx[i] = dy[i] * (c * fl(1 / fl(r)))     if 0 < t < 1, else 0    (fp32)
+ *   dl[g] =  c / r^2 * sum over group g's elements with 0 < t < 1 of dy * (x - u)
+ *   du[g] = -c / r^2 * sum over the same elements of dy * (x - l)
+ * dl_dev and du_dev receive G doubles each (device).  The sums take each product
+ * in fp32, add four in fp32, accumulate a thread's share in a compensated fp32
+ * sum and the threads in double, over a partition fixed by the problem size, so
+ * they are deterministic; their error is below 1e-6 of
+ * c / r^2 * sum |dy (x - u)| (resp. |dy (x - l)|).  Bound by HBM: 12 bytes per
+ * element.  Same requirements as the forward; scratch_dev holds
+ * palquant_fake_quant_scratch_bytes(P, G, Cg) bytes.  P = 0 gives zero
+ * gradients (the element pointers and the scratch may then be NULL).
+ * Asynchronous. */
+pq_status palquant_fake_quant_backward(const float* x_dev, const float* dy_dev, float* dx_dev, double* dl_dev,
+                                       double* du_dev, int64_t P, int32_t G, int32_t Cg, int32_t bits, int32_t kind,
+                                       const float* l_host, const float* u_host, void* scratch_dev,
+                                       size_t scratch_bytes, pq_stream_t stream);
+
+/* ------------------------------------------------------------------------ */
 /* Introspection (host only; no GPU needed).                                */
 /* ------------------------------------------------------------------------ */
 

@@ -32,7 +32,8 @@ EXPORTS = [
     "palquant_conv2d_f32", "palquant_maxpool2d_f32", "palquant_avgpool_f32", "palquant_linear_f32",
     "palquant_cyclic_shuffle_module", "palquant_bitsplit_desc", "palquant_bitsplit_scratch_bytes",
     "palquant_bitsplit_pack_weight_codes_host", "palquant_bitsplit_act", "palquant_bitsplit_conv",
-    "palquant_pack_weights_odd_host",
+    "palquant_pack_weights_odd_host", "palquant_fake_quant_forward", "palquant_fake_quant_scratch_bytes",
+    "palquant_fake_quant_backward",
 ]
 
 
@@ -131,6 +132,13 @@ def _load():
                        ("palquant_linear_f32", [_P, _P, _P, _I64, _I32, _I32, _P])):
         getattr(L, name).restype = _I32
         getattr(L, name).argtypes = args
+    L.palquant_fake_quant_forward.restype = _I32
+    L.palquant_fake_quant_forward.argtypes = [_P, _P, _I64, _I32, _I32, _I32, _I32, _P, _P, _P]
+    L.palquant_fake_quant_scratch_bytes.restype = ctypes.c_size_t
+    L.palquant_fake_quant_scratch_bytes.argtypes = [_I64, _I32, _I32]
+    L.palquant_fake_quant_backward.restype = _I32
+    L.palquant_fake_quant_backward.argtypes = [_P, _P, _P, _P, _P, _I64, _I32, _I32, _I32, _I32, _P, _P, _P,
+                                               ctypes.c_size_t, _P]
     return L
 
 
@@ -388,3 +396,24 @@ def palquant_pack_weights_odd_host(w_host, d: LayerDesc, u) -> np.ndarray:
     _check(lib.palquant_pack_weights_odd_host(_ptr(w), ctypes.byref(d), _ptr(uu), _ptr(out), n),
            "palquant_pack_weights_odd_host")
     return out
+
+
+# ---------------------------------------------------------------- quantisation-aware training
+def palquant_fake_quant_forward(x_dev, xhat_dev, P, G, Cg, bits, kind, l, u, stream=None) -> None:
+    """Fake quantisation with learned per-group bounds (Eq. 2-3); kind 0 activations, 1 weights."""
+    lf, uf = _f32(l), _f32(u)
+    _check(lib.palquant_fake_quant_forward(_ptr(x_dev), _ptr(xhat_dev), P, G, Cg, bits, kind, _ptr(lf), _ptr(uf),
+                                           _stream(stream)), "palquant_fake_quant_forward")
+
+
+def palquant_fake_quant_scratch_bytes(P, G, Cg) -> int:
+    return lib.palquant_fake_quant_scratch_bytes(P, G, Cg)
+
+
+def palquant_fake_quant_backward(x_dev, dy_dev, dx_dev, dl_dev, du_dev, P, G, Cg, bits, kind, l, u, scratch_dev,
+                                 scratch_bytes, stream=None) -> None:
+    """Straight-through backward: dx (fp32) and the per-group gradients of l and u (G doubles each, device)."""
+    lf, uf = _f32(l), _f32(u)
+    _check(lib.palquant_fake_quant_backward(_ptr(x_dev), _ptr(dy_dev), _ptr(dx_dev), _ptr(dl_dev), _ptr(du_dev), P, G,
+                                            Cg, bits, kind, _ptr(lf), _ptr(uf), _ptr(scratch_dev), scratch_bytes,
+                                            _stream(stream)), "palquant_fake_quant_backward")

@@ -353,3 +353,33 @@ def test_quantize_layer_fused_rules():
     wq = synth.random_codes((2, 32, 3, 3, 64), 2, gen, signed=True)
     d2 = B.layer_desc(1, 8, 8, 2, 64, 32, 3, 1, 1, 2, 2, 2, code_format=B.PQ_CODES_C16)
     assert np.array_equal(B.palquant_unpack_weight_codes_host(B.palquant_pack_weight_codes_host(wq, d2), d2), wq)
+
+
+# ------------------------------------------------ quantisation-aware training (host checks)
+def test_fake_quant_argument_rules():
+    """Invalid arguments return before any launch (no device memory is touched)."""
+    A = 0x10000  # a 16-byte aligned stand-in address: every case below fails its checks first
+    ok = dict(P=8, G=2, Cg=8, bits=2, kind=0, l=[0.0, 0.0], u=[1.0, 2.0])
+
+    def fwd(**kw):
+        a = dict(ok, **kw)
+        return B.lib.palquant_fake_quant_forward(A, A, a["P"], a["G"], a["Cg"], a["bits"], a["kind"],
+                                                 B._ptr(B._f32(a["l"])), B._ptr(B._f32(a["u"])), None)
+
+    bad = [dict(Cg=6), dict(Cg=0), dict(G=0), dict(G=65, l=[0.0] * 65, u=[1.0] * 65), dict(bits=0), dict(bits=9),
+           dict(kind=2), dict(P=-1), dict(l=[0.0, 2.0]), dict(l=[0.0, float("nan")]), dict(u=[1.0, float("inf")]),
+           dict(l=[1.0, 0.0], u=[1.0, 2.0])]
+    for kw in bad:
+        assert fwd(**kw) == B.PQ_EINVAL, kw
+    assert B.lib.palquant_fake_quant_forward(A + 4, A, 8, 2, 8, 2, 0, B._ptr(B._f32(ok["l"])),
+                                             B._ptr(B._f32(ok["u"])), None) == B.PQ_EINVAL
+    # more than 2^32 float4s per group
+    assert fwd(P=1 << 31, Cg=16) == B.PQ_EUNSUPPORTED
+    assert B.palquant_fake_quant_scratch_bytes(1 << 31, 1, 16) == 0
+    # backward: a scratch buffer too small, misaligned gradient outputs
+    sb = B.palquant_fake_quant_scratch_bytes(8, 2, 8)
+    assert sb >= 2 * 16
+    lp, up = B._ptr(B._f32(ok["l"])), B._ptr(B._f32(ok["u"]))
+    assert B.lib.palquant_fake_quant_backward(A, A, A, A, A, 8, 2, 8, 2, 0, lp, up, A, sb - 1, None) == B.PQ_EINVAL
+    assert B.lib.palquant_fake_quant_backward(A, A, A, A + 4, A, 8, 2, 8, 2, 0, lp, up, A, sb, None) == B.PQ_EINVAL
+    assert B.lib.palquant_fake_quant_backward(A, A, A, A, A, 8, 2, 6, 2, 0, lp, up, A, sb, None) == B.PQ_EINVAL
