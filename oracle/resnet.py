@@ -20,6 +20,17 @@ oracle's own functions:
 * global average pooling and a full-precision FC layer (the last layer stays in
   full precision, Sec. 5).
 
+Placement "paper" follows Sec. 4.3 instead: a cyclic shuffle module (Eq. 9-10,
+weights "s{k}.csm" [G, c, 1, 1, c]) at the beginning of each stage, on the stage's
+input (X, Q): Z = X + Conv1x1(CyclicPermute(Q)), no ReLU, with Z's codes for the
+stage's first block; inside the stage no group permutation; the channel shuffle
+(kind 2, ShuffleNet's transpose) once per stage (the paper's default), at the end of
+the stage's last block, i.e. in that block's conv2 epilogue after the shortcut add
+and ReLU; that output is fp32 only (a per-channel scatter of codes would mix groups
+with different steps), and the next stage's input codes come from it by the
+quantiser with that stage's module input steps.  Steps keys: "s{k}.csm.in" (module
+input), "s{k}.csm.w", and the blocks' keys as in the plain placement.
+
 Steps.  calibrate() derives every step from fp32 tensors of one forward pass: a
 layer's weight steps from its weights (LSQ init), a block's input steps from X, the
 conv1 output steps from conv1's rescaled output.  forward() takes those steps as
@@ -29,8 +40,8 @@ from __future__ import annotations
 
 import numpy as np
 
-from . import (avgpool_f32, conv2d_f32, epilogue_scales, group_perm, inv_step, layer, linear_f32, maxpool_f32,
-               quantize_act, quantize_weights, act_step, weight_step)
+from . import (avgpool_f32, conv2d_f32, cyclic_shuffle_module, epilogue_scales, group_perm, inv_step, layer,
+               linear_f32, maxpool_f32, quantize_act, quantize_weights, act_step, weight_step)
 
 
 def _blocks(params: dict):
@@ -43,19 +54,24 @@ def _blocks(params: dict):
     return out
 
 
-def calibrate(x: np.ndarray, params: dict, G: int, bits: int) -> dict:
+def calibrate(x: np.ndarray, params: dict, G: int, bits: int, placement: str = "block") -> dict:
     """Steps of every PalQuant layer from one forward pass in fp32 (see module doc)."""
-    return _run(x, params, G, bits, None)["steps"]
+    return _run(x, params, G, bits, None, placement)["steps"]
 
 
-def forward(x: np.ndarray, params: dict, G: int, bits: int, steps: dict) -> dict:
+def forward(x: np.ndarray, params: dict, G: int, bits: int, steps: dict, placement: str = "block") -> dict:
     """Forward pass with the given steps.  Returns every intermediate tensor:
     "stem", "pool", per block "<b>.in_codes", "<b>.mid_codes", "<b>.down" (if any),
-    "<b>.out" (fp32), "<b>.out_codes" (not for the last block), "avg", "logits"."""
-    return _run(x, params, G, bits, steps)
+    "<b>.out" (fp32), "<b>.out_codes" (not for the last block; placement "paper":
+    first blocks of a stage only), "avg", "logits"; placement "paper" also per stage
+    "s{k}.csm.in_codes", "s{k}.csm.out" (fp32 Z) and "s{k}.csm.out_codes"."""
+    return _run(x, params, G, bits, steps, placement)
 
 
-def _run(x, params, G, bits, steps):
+def _run(x, params, G, bits, steps, placement="block"):
+    if placement not in ("block", "paper"):
+        raise ValueError("placement must be 'block' or 'paper'")
+    paper = placement == "paper"
     calib = steps is None
     st = {} if calib else steps
     r = {}
@@ -63,11 +79,29 @@ def _run(x, params, G, bits, steps):
     X = maxpool_f32(stem, 3, 2, 1)
     r["stem"], r["pool"] = stem, X
     blocks = _blocks(params)
+    first_key = "s1.csm.in" if paper else blocks[0][0] + ".in"
     if calib:
-        st[blocks[0][0] + ".in"] = act_step(X, G, bits)
-    Q = quantize_act(X, G, bits, inv_step(st[blocks[0][0] + ".in"]))
+        st[first_key] = act_step(X, G, bits)
+    Q = quantize_act(X, G, bits, inv_step(st[first_key]))
     dst = group_perm(G, 1, 1)
+    src = [(g - 1) % G for g in range(G)]  # the module's conv group g reads input group pi^-1(g)
     for i, (name, stride, has_down) in enumerate(blocks):
+        stage, first_in_stage = int(name[1]), name.endswith("b1")
+        if paper and first_in_stage:
+            # cyclic shuffle module at the beginning of the stage (Eq. 9-10)
+            csm = f"s{stage}.csm"
+            r[csm + ".in_codes"] = Q
+            wc = params[csm]
+            if calib:
+                st[csm + ".w"] = weight_step(wc, bits)
+            wqc = quantize_weights(wc, bits, inv_step(st[csm + ".w"]))
+            m_outc, _ = epilogue_scales(st[csm + ".w"], np.asarray(st[csm + ".in"])[src], None, 1.0, 0, 0)
+            if calib:
+                Z, _ = cyclic_shuffle_module(X, Q, wqc, m_outc, None, 1, False, bits)
+                st[name + ".in"] = act_step(Z, G, bits)
+            Z, Qz = cyclic_shuffle_module(X, Q, wqc, m_outc, inv_step(st[name + ".in"]), 1, False, bits)
+            r[csm + ".out"], r[csm + ".out_codes"] = Z, Qz
+            X, Q = Z, Qz
         s_in = st[name + ".in"]
         r[name + ".in_codes"] = Q
         # conv1: codes for conv2
@@ -100,6 +134,29 @@ def _run(x, params, G, bits, steps):
         wq2 = quantize_weights(w2, bits, inv_step(st[name + ".conv2.w"]))
         m_out2, _ = epilogue_scales(st[name + ".conv2.w"], st[name + ".mid"], None, 1.0, 1, 1)
         last = i == len(blocks) - 1
+        if paper:
+            if first_in_stage:
+                # no permutation inside the stage: codes for the stage's second block
+                nxt = blocks[i + 1][0] + ".in"
+                if calib:
+                    _, Xn, _ = layer(Q1, wq2, 1, 1, m_out2, None, 0, 0, shortcut=S, relu=True, bits_out=bits)
+                    st[nxt] = act_step(Xn, G, bits)
+                _, Xn, Qn = layer(Q1, wq2, 1, 1, m_out2, inv_step(st[nxt]), 0, 0, shortcut=S, relu=True,
+                                  bits_out=bits)
+                r[name + ".out"], r[name + ".out_codes"] = Xn, Qn
+            else:
+                # the stage's last block: channel shuffle after the add and ReLU, fp32 out;
+                # the next stage's input codes from the quantiser
+                _, Xn, _ = layer(Q1, wq2, 1, 1, m_out2, None, 2, 0, shortcut=S, relu=True, bits_out=bits)
+                r[name + ".out"] = Xn
+                Qn = None
+                if not last:
+                    nk = f"s{stage + 1}.csm.in"
+                    if calib:
+                        st[nk] = act_step(Xn, G, bits)
+                    Qn = quantize_act(Xn, G, bits, inv_step(st[nk]))
+            X, Q = Xn, Qn
+            continue
         nxt = None if last else blocks[i + 1][0] + ".in"
         if not last and calib:
             _, Xn, _ = layer(Q1, wq2, 1, 1, m_out2, None, 1, 1, shortcut=S, relu=True, bits_out=bits)

@@ -59,7 +59,7 @@ def random_codes(shape, bits: int, gen: torch.Generator, signed: bool = False) -
 
 
 def resnet18_inputs(N: int, H: int = 224, W: int = 224, G: int = 2, widths=(64, 128, 256, 512), classes: int = 1000,
-                    seed: int = 0):
+                    seed: int = 0, cyclic_modules: bool = False):
     """(x, params) for the ResNet-18-shaped PalQuant network.
 
     x: images N(0, 1), NHWC [N, H, W, 3].  params: name -> fp32 weights, drawn after x
@@ -68,7 +68,9 @@ def resnet18_inputs(N: int, H: int = 224, W: int = 224, G: int = 2, widths=(64, 
     [G, w, 3, 3, w] and, in the first block of stages 2-4 (stride 2, channels change),
     "s{s}b{b}.down" [G, w, 1, 1, cin], all He-initialised per group (w = widths[s-1],
     cin = the block's per-group input width); last "fc" [classes, G*widths[-1]]
-    N(0, 1/fan_in)."""
+    N(0, 1/fan_in).  With cyclic_modules, then per stage k = 1..4 "s{k}.csm"
+    [G, c, 1, 1, c] (the weights of the cyclic shuffle module at the stage's
+    beginning, c = the stage's per-group input width), He-initialised."""
     gen = generator(seed)
     x = normal((N, H, W, 3), gen)
     params = {"stem": normal((G * widths[0], 7, 7, 3), gen, math.sqrt(2.0 / 147.0))}
@@ -82,4 +84,9 @@ def resnet18_inputs(N: int, H: int = 224, W: int = 224, G: int = 2, widths=(64, 
                 params[name + ".down"] = he_weights(G, w, 1, 1, cin, gen)
             cin = w
     params["fc"] = normal((classes, G * widths[-1]), gen, math.sqrt(1.0 / (G * widths[-1])))
+    if cyclic_modules:
+        cin = widths[0]
+        for s, w in enumerate(widths):
+            params[f"s{s + 1}.csm"] = he_weights(G, cin, 1, 1, cin, gen)
+            cin = w
     return x, params

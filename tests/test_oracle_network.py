@@ -269,3 +269,62 @@ def test_prop1_G_minus_1_modules_reach_every_group(G):
             x, _ = oracle.cyclic_shuffle_module(x, q, wq, m_out, None, 1)
             live = {g for g in range(G) if np.any(x[..., g * Cg:(g + 1) * Cg] != 0)}
             assert live == {(s + j) % G for j in range(k + 1)}, (G, s, k, live)
+
+
+# ------------------------------------------- the paper's placement (Sec. 4.3)
+@pytest.fixture(scope="module")
+def net_paper():
+    x, params = synth.resnet18_inputs(2, 32, 32, G, WIDTHS, 10, seed=5, cyclic_modules=True)
+    steps = R.calibrate(x, params, G, BITS, placement="paper")
+    return x, params, steps, R.forward(x, params, G, BITS, steps, placement="paper")
+
+
+def test_paper_placement_rederived_with_float64_library(net_paper):
+    """The paper's placement re-derived stage by stage from the oracle's own tensors:
+    the cyclic shuffle module at each stage's start (Eq. 9-10: torch float64 1x1
+    grouped convolution of the group-rolled codes, one fp32 multiply, + X, no ReLU),
+    no permutation inside the stage, and the channel shuffle (ShuffleNet's
+    reshape/transpose) after the add and ReLU of each stage's last block."""
+    x, params, steps, r = net_paper
+    f32 = lambda a, m: (a.astype(np.float32).reshape(*a.shape[:-1], G, -1) *
+                        np.asarray(m, np.float32)[:, None]).reshape(a.shape)
+    X = r["pool"]
+    for k in range(1, 5):
+        csm = f"s{k}.csm"
+        Q = r[csm + ".in_codes"]
+        assert np.array_equal(Q, oracle.quantize_act(X, G, BITS, oracle.inv_step(steps[csm + ".in"]))), csm
+        swc = steps[csm + ".w"]
+        wqc = oracle.quantize_weights(params[csm], BITS, oracle.inv_step(swc))
+        rolled_q = np.roll(Q.reshape(*Q.shape[:-1], G, -1), 1, axis=-2).reshape(Q.shape)  # Eq. 8
+        accc = torch_group_conv_f64(rolled_q, wqc, 1, 0)
+        src = [(g - 1) % G for g in range(G)]
+        m_c = (np.float64(swc) * np.float64(np.asarray(steps[csm + ".in"])[src])).astype(np.float32)
+        Z = f32(accc, m_c) + X
+        assert np.array_equal(Z, r[csm + ".out"]), csm
+        for b, stride, down, last in ((f"s{k}b1", 1 if k == 1 else 2, k > 1, False), (f"s{k}b2", 1, False, True)):
+            Qb = r[b + ".in_codes"]
+            Xb = Z if not last else r[f"s{k}b1.out"]
+            assert np.array_equal(Qb, oracle.quantize_act(Xb, G, BITS, oracle.inv_step(steps[b + ".in"]))), b
+            sw1, sin, smid = steps[b + ".conv1.w"], steps[b + ".in"], steps[b + ".mid"]
+            wq1 = oracle.quantize_weights(params[b + ".conv1"], BITS, oracle.inv_step(sw1))
+            acc1 = torch_group_conv_f64(Qb, wq1, stride, 1)
+            q1 = np.clip(np.rint(f32(acc1, (np.float64(sw1) * np.float64(sin) / np.float64(smid)).astype(np.float32))),
+                         0, 3).astype(np.uint8)
+            assert np.array_equal(q1, r[b + ".mid_codes"]), b
+            if down:
+                swd = steps[b + ".down.w"]
+                wqd = oracle.quantize_weights(params[b + ".down"], BITS, oracle.inv_step(swd))
+                S = f32(torch_group_conv_f64(Qb, wqd, stride, 0), (np.float64(swd) * np.float64(sin)).astype(np.float32))
+            else:
+                S = Xb
+            sw2 = steps[b + ".conv2.w"]
+            wq2 = oracle.quantize_weights(params[b + ".conv2"], BITS, oracle.inv_step(sw2))
+            acc2 = torch_group_conv_f64(q1, wq2, 1, 1)
+            y = np.maximum(f32(acc2, (np.float64(sw2) * np.float64(smid)).astype(np.float32)) + S, np.float32(0))
+            if last:  # ShuffleNet's channel shuffle: [G, Cg] -> [Cg, G]
+                y = np.swapaxes(y.reshape(*y.shape[:-1], G, -1), -1, -2).reshape(y.shape)
+            assert np.array_equal(y, r[b + ".out"]), b
+        X = r[f"s{k}b2.out"]
+    ref = X.astype(np.float64).mean(axis=(1, 2)) @ params["fc"].astype(np.float64).T
+    assert np.allclose(r["logits"], ref, rtol=1e-4, atol=1e-4)
+
