@@ -518,6 +518,45 @@ def measure_bitsplit_vs_palquant(dev, stream, timed, pk, fp8_peak):
 # ---------------------------------------------------------------------------
 # The ResNet-18-shaped network (config 2): images/s of the whole forward.
 # ---------------------------------------------------------------------------
+def measure_resnet18_paper(dev, world, args):
+    """The same network with the paper's placement of the shuffles (Sec. 4.3): a cyclic
+    shuffle module at each stage's start, the channel shuffle at each stage's end (and
+    the quantiser that re-codes each stage's output), timed the same way."""
+    import torch
+
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300 import synth
+    from paper_2208_01944_gb300.resnet18 import PalQuantResNet18
+
+    N = args.resnet_batch
+    x_np, params = synth.resnet18_inputs(N, seed=0, cyclic_modules=True)
+    net = PalQuantResNet18(params, N, device=dev, placement="paper")
+    xs = [torch.from_numpy(x_np).to(dev)]
+    xs.append(torch.flip(xs[0], dims=[0]).contiguous())
+    net.calibrate(xs[0])
+    graphs = [net.capture(x) for x in xs]
+    for i in range(3):
+        net.replay(graphs[i & 1])
+    torch.cuda.synchronize(dev)
+    R = args.resnet_reps
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(net.stream)
+    for i in range(R):
+        net.replay(graphs[i & 1])
+    e1.record(net.stream)
+    torch.cuda.synchronize(dev)
+    st = B.palquant_sync_check(net.stream)
+    assert st == B.PQ_OK, B.strerror(st)
+    ms = max_over_ranks(e0.elapsed_time(e1) / R, world, dev)
+    res = {"images_per_s": whole_job_rate(N, world, ms), "ms_per_batch": ms,
+           "palquant_body_tops": whole_job_rate(net.body_int_ops(), world, ms) / 1e12,
+           "gpu_launches_per_forward": net.launches_per_forward(),
+           "timed": "CUDA-graph replay; 4 cyclic shuffle modules, 20 PalQuant layers, 4 quantisers"}
+    del graphs, net
+    torch.cuda.empty_cache()
+    return res
+
+
 def measure_resnet18(dev, world, args):
     """Forward of the ResNet-18-shaped PalQuant network (224x224, G = 2, b = 2, per-group
     widths 64/128/256/512, fp32 stem and FC) on a batch of synthetic images, replayed
@@ -564,6 +603,7 @@ def measure_resnet18(dev, world, args):
     out["stages_ms"] = {name: marks[i - 1][1].elapsed_time(ev) for i, (name, ev) in enumerate(marks) if i > 0}
     del graphs, net
     torch.cuda.empty_cache()
+    out["paper_placement"] = measure_resnet18_paper(dev, world, args)
     if not args.no_cpu_baseline and world == 1:
         import time
 

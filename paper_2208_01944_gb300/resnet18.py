@@ -19,6 +19,15 @@ takes the following reading:
            group's input step);
 * global average pooling and an fp32 FC layer.
 
+placement="paper" follows Sec. 4.3 instead (weights from
+synth.resnet18_inputs(..., cyclic_modules=True)): a cyclic shuffle module (Eq. 9-10,
+palquant_cyclic_shuffle_module: 1x1 group convolution of the group-permuted codes +
+the fp32 input, no ReLU) at the beginning of each stage, whose codes feed the stage's
+first block; no group permutation inside a stage; the channel shuffle (ShuffleNet's
+transpose, shuffle kind 2) once per stage, in the epilogue of the stage's last conv2
+after the shortcut add and ReLU, with fp32 output only; the next stage's input codes
+then come from the quantiser with that stage's module input steps.
+
 Every step runs in the library's kernels; this module only owns buffers, derives
 per-layer multipliers through palquant_epilogue_scales and launches the calls on one
 stream, with no host synchronisation inside forward() (which can be captured in a
@@ -43,7 +52,11 @@ def _out(n: int, k: int, s: int, p: int) -> int:
 class PalQuantResNet18:
     def __init__(self, params: dict, N: int, H: int = 224, W: int = 224, G: int = 2, widths=(64, 128, 256, 512),
                  classes: int = 1000, bits: int = 2, device="cuda:0", stream: torch.cuda.Stream | None = None,
-                 code_format: int | None = None):
+                 code_format: int | None = None, placement: str = "block"):
+        if placement not in ("block", "paper"):
+            raise ValueError("placement must be 'block' or 'paper'")
+        self.placement = placement
+        self.paper = paper = placement == "paper"
         self.dev = torch.device(device)
         self.N, self.H, self.W, self.G, self.bits, self.classes = N, H, W, G, bits, classes
         self.stream = stream or torch.cuda.Stream(device=self.dev)
@@ -67,8 +80,17 @@ class PalQuantResNet18:
         self.pool = torch.empty((N, self.Hp, self.Wp, C0), **f32)
         self.in_codes = torch.empty((N, self.Hp, self.Wp, C0 // per_byte), **u8)
         self.blocks = []
+        self.modules = []  # placement "paper": one cyclic shuffle module per stage
         Hc, Wc, cin = self.Hp, self.Wp, widths[0]
         for s, w in enumerate(widths):
+            if paper:
+                m = dict(name=f"s{s + 1}.csm", H=Hc, W=Wc, c=cin)
+                m["d"] = B.layer_desc(N, Hc, Wc, G, cin, cin, 1, 1, 0, bits, bits, bits, 0, code_format=fmt)
+                m["in_codes"] = self.in_codes if s == 0 else torch.empty((N, Hc, Wc, G * cin // per_byte), **u8)
+                m["z"] = torch.empty((N, Hc, Wc, G * cin), **f32)
+                m["codes"] = torch.empty((N, Hc, Wc, G * cin // per_byte), **u8)
+                m["wp"] = torch.empty(B.palquant_packed_weight_bytes(m["d"]), **u8)
+                self.modules.append(m)
             for b in range(2):
                 name = f"s{s + 1}b{b + 1}"
                 stride = 2 if (s > 0 and b == 0) else 1
@@ -92,6 +114,7 @@ class PalQuantResNet18:
         self.logits = torch.empty((N, classes), **f32)
         self.no_shuffle = B.shuffle(0, 0)
         self.cyclic = B.shuffle(1, 1)
+        self.channel_shuffle = B.shuffle(2, 0)
         self.ones = np.ones(G, dtype=np.float32)
         self.steps = None
         self.graph = None
@@ -110,6 +133,8 @@ class PalQuantResNet18:
     def calibrate(self, x_dev: torch.Tensor) -> dict:
         """Steps of every PalQuant layer from one fp32 pass over x (LSQ initialisation:
         weights from their own values, activations from the tensor entering the layer)."""
+        if self.paper:
+            return self._calibrate_paper(x_dev)
         G, bits, st = self.G, self.bits, {}
         s = self.stream
         self._stem(x_dev)
@@ -148,6 +173,77 @@ class PalQuantResNet18:
         self.set_steps(st)
         return st
 
+    def _calibrate_paper(self, x_dev: torch.Tensor) -> dict:
+        """calibrate() for placement "paper", in the order the oracle network takes."""
+        G, bits, st, s = self.G, self.bits, {}, self.stream
+        self._stem(x_dev)
+        st["s1.csm.in"] = self._act_steps(self.pool, self.C0 // G)
+        for blk in self.blocks:
+            n = blk["name"]
+            st[n + ".conv1.w"] = B.palquant_weight_steps(self.params[n + ".conv1"], blk["d1"])
+            st[n + ".conv2.w"] = B.palquant_weight_steps(self.params[n + ".conv2"], blk["d2"])
+            if blk["down"]:
+                st[n + ".down.w"] = B.palquant_weight_steps(self.params[n + ".down"], blk["dd"])
+        for m in self.modules:
+            st[m["name"] + ".w"] = B.palquant_weight_steps(self.params[m["name"]], m["d"])
+        self.steps = st
+        B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, G, self.C0 // G, bits,
+                                self._inv(st["s1.csm.in"]), code_format=self.fmt, stream=s)
+        X = self.pool
+        for k, m in enumerate(self.modules):
+            b1, b2 = self.blocks[2 * k], self.blocks[2 * k + 1]
+            self._pack_module(m, st)
+            B.palquant_cyclic_shuffle_module(m["in_codes"], m["wp"], m["d"], m["m_out"], None, 1, X, m["z"], None,
+                                             stream=s)
+            st[b1["name"] + ".in"] = self._act_steps(m["z"], m["c"])
+            m["m_req"] = self._inv(st[b1["name"] + ".in"])
+            B.palquant_cyclic_shuffle_module(m["in_codes"], m["wp"], m["d"], m["m_out"], m["m_req"], 1, X, m["z"],
+                                             m["codes"], stream=s)
+            for blk, q_in in ((b1, m["codes"]), (b2, b1["out_codes"])):
+                n = blk["name"]
+                self._pack(blk, st)
+                m_out1, _ = B.palquant_epilogue_scales(G, st[n + ".conv1.w"], st[n + ".in"], 1.0, None, self.no_shuffle)
+                y1 = torch.empty((self.N, blk["Ho"], blk["Wo"], G * blk["w"]), dtype=torch.float32, device=self.dev)
+                B.palquant_layer_fused(q_in, blk["wp1"], blk["d1"], m_out1, None, self.no_shuffle, None, None, y1, None,
+                                       stream=s)
+                st[n + ".mid"] = self._act_steps(y1, blk["w"])
+                del y1
+                self._scales(blk, st)
+                self._block_front(blk, q_in)
+                if blk is b1:
+                    sc = b1["down_out"] if b1["down"] else m["z"]
+                    self._conv2_paper(b1, sc, None, False)
+                    st[b2["name"] + ".in"] = self._act_steps(b1["out"], b1["w"])
+                    self._conv2_paper(b1, sc, self._inv(st[b2["name"] + ".in"]), False)
+                else:
+                    self._conv2_paper(b2, b1["out"], None, True)
+                    if k + 1 < len(self.modules):
+                        nxt = self.modules[k + 1]
+                        st[nxt["name"] + ".in"] = self._act_steps(b2["out"], b2["w"])
+                        B.palquant_quantize_act(b2["out"], nxt["in_codes"], self.N, b2["Ho"], b2["Wo"], G, b2["w"],
+                                                bits, self._inv(st[nxt["name"] + ".in"]), code_format=self.fmt,
+                                                stream=s)
+            X = b2["out"]
+        self.set_steps(st)
+        return st
+
+    def _pack_module(self, m, st):
+        """Pack a stage's module weights; its multiplier m_out[g] = fl(s_w[g] s_in[pi^-1(g)])
+        (conv group g reads the permuted input group)."""
+        n, G = m["name"], self.G
+        B.palquant_pack_weights(self.params[n], m["d"], self._inv(st[n + ".w"]), m["wp"], m["wp"].numel(),
+                                stream=self.stream)
+        src = [(g - 1) % G for g in range(G)]
+        s_in = np.asarray(st[n + ".in"], dtype=np.float32)[src]
+        m["m_out"] = B.palquant_epilogue_scales(G, st[n + ".w"], s_in, 1.0, None, self.no_shuffle)[0]
+
+    def _conv2_paper(self, blk, shortcut, m_req2, last):
+        """conv2 of placement "paper": no permutation and the codes of the stage's second
+        block, or (the stage's last block) the channel shuffle and fp32 out only."""
+        B.palquant_layer_fused(blk["mid_codes"], blk["wp2"], blk["d2"], blk["m_out2"], None if last else m_req2,
+                               self.channel_shuffle if last else self.no_shuffle, shortcut, None, blk["out"],
+                               None if (last or m_req2 is None) else blk["out_codes"], stream=self.stream)
+
     def _pack(self, blk, st):
         """Quantise and pack the block's weights with their steps (synchronous)."""
         n = blk["name"]
@@ -170,6 +266,20 @@ class PalQuantResNet18:
     def set_steps(self, steps: dict):
         """Pack every layer's weights and derive the epilogue multipliers from `steps`."""
         self.steps = dict(steps)
+        if self.paper:
+            for k, m in enumerate(self.modules):
+                self._pack_module(m, self.steps)
+                m["inv_in"] = self._inv(self.steps[m["name"] + ".in"])
+                m["m_req"] = self._inv(self.steps[self.blocks[2 * k]["name"] + ".in"])
+            for i, blk in enumerate(self.blocks):
+                self._pack(blk, self.steps)
+                self._scales(blk, self.steps)
+                first = blk["name"].endswith("b1")
+                blk["m_req2"] = self._inv(self.steps[self.blocks[i + 1]["name"] + ".in"]) if first else None
+            self.inv_in = self.modules[0]["inv_in"]
+            self.stream.synchronize()
+            self.graph = None
+            return
         for i, blk in enumerate(self.blocks):
             self._pack(blk, self.steps)
             self._scales(blk, self.steps)
@@ -221,12 +331,34 @@ class PalQuantResNet18:
         B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, self.G, self.C0 // self.G,
                                 self.bits, self.inv_in, code_format=self.fmt, stream=s)
         mark("input quantiser")
-        for i, blk in enumerate(self.blocks):
-            q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]
-            self._block_front(blk, q_in)
-            mark(blk["name"] + " conv1" + (" + down" if blk["down"] else ""))
-            self._conv2(blk, blk["m_req2"])
-            mark(blk["name"] + " conv2")
+        if self.paper:
+            X = self.pool
+            for k, m in enumerate(self.modules):
+                b1, b2 = self.blocks[2 * k], self.blocks[2 * k + 1]
+                B.palquant_cyclic_shuffle_module(m["in_codes"], m["wp"], m["d"], m["m_out"], m["m_req"], 1, X, m["z"],
+                                                 m["codes"], stream=s)
+                mark(m["name"] + " cyclic shuffle module")
+                self._block_front(b1, m["codes"])
+                mark(b1["name"] + " conv1" + (" + down" if b1["down"] else ""))
+                self._conv2_paper(b1, b1["down_out"] if b1["down"] else m["z"], b1["m_req2"], False)
+                mark(b1["name"] + " conv2")
+                self._block_front(b2, b1["out_codes"])
+                mark(b2["name"] + " conv1")
+                self._conv2_paper(b2, b1["out"], None, True)
+                mark(b2["name"] + " conv2 + channel shuffle")
+                if k + 1 < len(self.modules):
+                    nxt = self.modules[k + 1]
+                    B.palquant_quantize_act(b2["out"], nxt["in_codes"], self.N, b2["Ho"], b2["Wo"], self.G, b2["w"],
+                                            self.bits, nxt["inv_in"], code_format=self.fmt, stream=s)
+                    mark(nxt["name"] + " input quantiser")
+                X = b2["out"]
+        else:
+            for i, blk in enumerate(self.blocks):
+                q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]
+                self._block_front(blk, q_in)
+                mark(blk["name"] + " conv1" + (" + down" if blk["down"] else ""))
+                self._conv2(blk, blk["m_req2"])
+                mark(blk["name"] + " conv2")
         last = self.blocks[-1]["out"]
         B.palquant_avgpool_f32(last, self.avg, self.N, self.Hl, self.Wl, self.Cl, stream=s)
         B.palquant_linear_f32(self.avg, self.w_fc, self.logits, self.N, self.Cl, self.classes, stream=s)
@@ -252,7 +384,10 @@ class PalQuantResNet18:
     def launches_per_forward(self) -> int:
         """Kernels one forward launches: stem conv, max pooling, quantiser, per block
         conv1 (+ down) + conv2, average pooling, FC."""
-        return 3 + sum(3 if b["down"] else 2 for b in self.blocks) + 2
+        n = 3 + sum(3 if b["down"] else 2 for b in self.blocks) + 2
+        if self.paper:
+            n += len(self.modules) + len(self.modules) - 1  # a module per stage, a quantiser per stage boundary
+        return n
 
     def body_int_ops(self) -> int:
         """Integer operations (2 per MAC) of the PalQuant layers of one forward."""
@@ -262,4 +397,6 @@ class PalQuantResNet18:
             ops += 2 * N * b["Ho"] * b["Wo"] * G * b["w"] * 9 * b["w"]
             if b["down"]:
                 ops += 2 * N * b["Ho"] * b["Wo"] * G * b["w"] * b["cin"]
+        for m in self.modules:
+            ops += 2 * N * m["H"] * m["W"] * G * m["c"] * m["c"]
         return ops

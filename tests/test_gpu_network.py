@@ -152,3 +152,60 @@ def test_pooling_and_linear_match_oracle():
     B.palquant_linear_f32(torch.from_numpy(v).cuda(), torch.from_numpy(w).cuda(), y, 13, 100, 1000)
     assert B.palquant_sync_check() == B.PQ_OK
     assert np.array_equal(y.cpu().numpy(), ref)
+
+
+def _compare_paper(net, r):
+    f = net.fmt
+    assert np.array_equal(net.pool.cpu().numpy(), r["pool"]), "max pooling"
+    for m in net.modules:
+        n = m["name"]
+        assert np.array_equal(_codes(m["in_codes"], f), r[n + ".in_codes"]), n + " input codes"
+        assert np.array_equal(m["z"].cpu().numpy(), r[n + ".out"]), n + " module output"
+        assert np.array_equal(_codes(m["codes"], f), r[n + ".out_codes"]), n + " module codes"
+    for blk in net.blocks:
+        n = blk["name"]
+        assert np.array_equal(_codes(blk["mid_codes"], f), r[n + ".mid_codes"]), n + " conv1 codes"
+        if blk["down"]:
+            assert np.array_equal(blk["down_out"].cpu().numpy(), r[n + ".down"]), n + " downsample"
+        assert np.array_equal(blk["out"].cpu().numpy(), r[n + ".out"]), n + " block output"
+        if n + ".out_codes" in r:
+            assert np.array_equal(_codes(blk["out_codes"], f), r[n + ".out_codes"]), n + " next-block codes"
+    assert np.array_equal(net.logits.cpu().numpy(), r["logits"]), "logits"
+
+
+@pytest.mark.parametrize("N,H,widths,classes,seed,fmt", [(2, 32, (32, 32, 32, 32), 10, 7, 2),
+                                                         (2, 48, (64, 64, 128, 64), 12, 8, 4),   # FP4 codes
+                                                         (3, 64, (32, 64, 32, 64), 16, 9, 2)])
+def test_paper_placement_matches_oracle(N, H, widths, classes, seed, fmt):
+    """Sec. 4.3's placement: a cyclic shuffle module at each stage's start, the channel
+    shuffle at each stage's end; every tensor bit for bit against the oracle network."""
+    from paper_2208_01944_gb300 import binding as B
+    from paper_2208_01944_gb300.resnet18 import PalQuantResNet18
+
+    x, params = synth.resnet18_inputs(N, H, H, 2, widths, classes, seed=seed, cyclic_modules=True)
+    steps = OR.calibrate(x, params, 2, 2, placement="paper")
+    r = OR.forward(x, params, 2, 2, steps, placement="paper")
+    net = PalQuantResNet18(params, N, H, H, 2, widths, classes, 2, code_format=fmt, placement="paper")
+    net.set_steps(steps)
+    net.forward(torch.from_numpy(x).cuda())
+    net.stream.synchronize()
+    assert B.palquant_sync_check() == B.PQ_OK
+    _compare_paper(net, r)
+
+
+def test_paper_placement_gpu_calibration_matches_oracle():
+    """The library's step initialisation for the paper placement: the first module's
+    input steps and every weight step within one float ulp of the oracle's, the
+    later steps (which depend on codes an ulp can flip) within 1e-3."""
+    from paper_2208_01944_gb300.resnet18 import PalQuantResNet18
+
+    x, params = synth.resnet18_inputs(2, 32, 32, 2, (32, 32, 32, 32), 10, seed=7, cyclic_modules=True)
+    ref = OR.calibrate(x, params, 2, 2, placement="paper")
+    net = PalQuantResNet18(params, 2, 32, 32, 2, (32, 32, 32, 32), 10, 2, code_format=2, placement="paper")
+    got = net.calibrate(torch.from_numpy(x).cuda())
+    assert set(got) == set(ref)
+    for k in ["s1.csm.in"] + [k for k in ref if k.endswith(".w")]:
+        d = np.abs(got[k].view(np.int32).astype(np.int64) - ref[k].view(np.int32).astype(np.int64))
+        assert np.all(d <= 1), k
+    for k in ref:
+        assert np.allclose(got[k], ref[k], rtol=1e-3), k
