@@ -69,6 +69,7 @@ def _declare(lib):
     lib.oracle_epilogue_scales.argtypes = [_I32, _P, _P, ctypes.c_double, _P, _I32, _I32, _P, _P, _P]
     lib.oracle_quantize_weights_odd.argtypes = [_P, _P, _I32, _I64, _I32, _P]
     lib.oracle_fake_quant_fwd.argtypes = [_P, _P, _I64, _I32, _I64, _I32, _I32, _P, _P]
+    lib.oracle_quantize_act_lu.argtypes = [_P, _P, _I64, _I32, _I64, _I32, _P, _P]
     lib.oracle_fake_quant_bwd.argtypes = [_P, _P, _P, _P, _P, _I64, _I32, _I64, _I32, _I32, _P, _P]
     lib.oracle_conv2d_f32.argtypes = [_P, _P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _I32, _I32, _I32]
     lib.oracle_maxpool_f32.argtypes = [_P, _P, _I64, _I64, _I64, _I32, _I32, _I32, _I32]
@@ -409,3 +410,17 @@ def fake_quant_backward(x: np.ndarray, dy: np.ndarray, G: int, bits: int, kind: 
     L.oracle_fake_quant_bwd(_ptr(x), _ptr(dy), _ptr(dx), _ptr(dl), _ptr(du), x.size // C, G, C // G, bits, kind,
                             _ptr(l), _ptr(u))
     return dx, dl, du
+
+
+def quantize_act_lu(x: np.ndarray, G: int, bits: int, l, u, L=None) -> np.ndarray:
+    """Inference codes with learned per-group bounds l < u (Eq. 2): the training
+    forward's x_q, x_q = rint(clamp((x - l) * fl(1/fl(u - l)), 0, 1) * (2^b - 1)).
+    x: [..., G*Cg] fp32 -> uint8 codes of the same shape."""
+    L = L or lib()
+    x = _f32(x)
+    l, u = _f32(l), _f32(u)
+    C = x.shape[-1]
+    assert C % G == 0 and l.shape == (G,) and u.shape == (G,)
+    q = np.empty(x.shape, dtype=np.uint8)
+    L.oracle_quantize_act_lu(_ptr(x), _ptr(q), x.size // C, G, C // G, bits, _ptr(l), _ptr(u))
+    return q

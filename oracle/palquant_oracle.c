@@ -32,6 +32,8 @@
  *   oracle_quantize_weights  pinned (hand cases, code range)
  *   oracle_quantize_weights_odd  pinned (hand cases, odd levels, monotone,
  *                            the clip bounds)
+ *   oracle_quantize_act_lu   pinned (hand cases; equal to the codes of the
+ *                            training forward)
  *   oracle_fake_quant_fwd /
  *   oracle_fake_quant_bwd    pinned (hand cases, levels, monotone; the
  *                            straight-through gradients against central
@@ -167,6 +169,25 @@ void oracle_fake_quant_fwd(const float* x, float* xhat, int64_t P, int G, int64_
                 float xq = rintf(xn * qp);
                 float v = xq * inv_qp;
                 xhat[i] = kind ? 2.0f * (v - 0.5f) : v;
+            }
+        }
+    }
+}
+
+/* Inference codes with learned bounds (Sec. 3.2 Eq. 2 with l, u per group, the
+ * training forward's x_q above): x_q = rint(min(max((x - l) * fl(1/fl(u - l)),
+ * 0), 1) * (2^b - 1)), NaN -> 0, one code per byte, x and q [P][G*Cg]. */
+void oracle_quantize_act_lu(const float* x, uint8_t* q, int64_t P, int G, int64_t Cg, int bits, const float* l,
+                            const float* u) {
+    const float qp = (float)((1 << bits) - 1);
+    const int64_t C = (int64_t)G * Cg;
+    for (int64_t p = 0; p < P; ++p) {
+        for (int g = 0; g < G; ++g) {
+            const float inv_r = 1.0f / (u[g] - l[g]);
+            for (int64_t j = 0; j < Cg; ++j) {
+                const int64_t i = p * C + (int64_t)g * Cg + j;
+                float xn = fminf(fmaxf(fq_t(x[i], l[g], inv_r), 0.0f), 1.0f);
+                q[i] = (uint8_t)(int)rintf(xn * qp);
             }
         }
     }

@@ -127,3 +127,22 @@ def test_backward_hand_case_and_outside_zero():
     np.testing.assert_array_equal(dx[0], [0.25, 0.25, 0.25, 0.25, 0, 0, 0, 0])  # t = 1 is outside (strict)
     assert dl[0] == (0.5 + 1 + 2 + 3.5 - 4 * 4) / 16.0   # sum(x - u) / r^2 over the four inside elements
     assert du[0] == -(0.5 + 1 + 2 + 3.5) / 16.0
+
+
+def test_inference_codes_with_learned_bounds():
+    """Eq. 2 with l, u at inference: hand cases (a negative lower bound shifts code 0
+    below x = 0), and the codes equal the training forward's x_q (x_hat * (2^b - 1))."""
+    x = np.array([[-3.0, -2.0, -1.0, 0.0, 0.5, 1.0, 2.0, 3.0, np.nan]], np.float32)
+    # l = -2, u = 2, b = 2: t = (x + 2) / 4, x_q = rint(3 t): 0, 0, 0.75 -> 1, 1.5 -> 2, 1.875 -> 2, 2.25 -> 2, 3, 3, 0
+    np.testing.assert_array_equal(oracle.quantize_act_lu(x, 1, 2, [-2.0], [2.0])[0], [0, 0, 1, 2, 2, 2, 3, 3, 0])
+    rng = np.random.default_rng(9)
+    G, Cg = 3, 16
+    l = np.array([-0.75, 0.0, 0.5], np.float32)
+    u = np.array([1.25, 3.0, 0.625], np.float32)
+    xs = rng.uniform(-1.5, 3.5, size=(64, G * Cg)).astype(np.float32)
+    for bits in (1, 2, 3, 4, 8):
+        q = oracle.quantize_act_lu(xs, G, bits, l, u)
+        xh = oracle.fake_quant_forward(xs, G, bits, 0, l, u)
+        qp = (1 << bits) - 1
+        assert q.max() <= qp
+        np.testing.assert_array_equal(np.rint(xh.astype(np.float64) * qp).astype(np.uint8), q)
