@@ -270,6 +270,24 @@ pq_status palquant_quantize_layer_fused(const float* x_dev, const float* inv_s_h
                                         pq_shuffle shuf, const float* shortcut_dev, int32_t* acc_out_dev,
                                         float* y_out_dev, void* q_out_dev, pq_stream_t stream);
 
+/* Inference quantisers with learned per-group bounds l[g] < u[g] (Eq. 2 as the
+ * paper trains it, Sec. 5): the codes of palquant_fake_quant_forward,
+ *   code = rint(min(max((x - l) * fl(1 / fl(u - l)), 0), 1) * (2^bits - 1))
+ * (one fp32 rounding per operation, NaN -> 0), so a layer trained with those
+ * kernels runs on exactly the codes its training forward used.  l_host and u_host
+ * hold G finite floats each (PQ_EINVAL otherwise).  Otherwise as
+ * palquant_quantize_act (all code formats) and palquant_quantize_layer_fused; in
+ * the fused form the out-of-image positions of the zero padding are code 0 for any
+ * l (the fp32 tiles are NaN-filled there). */
+pq_status palquant_quantize_act_lu(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G,
+                                   int32_t Cg, int32_t bits, int32_t code_format, const float* l_host,
+                                   const float* u_host, pq_stream_t stream);
+pq_status palquant_quantize_layer_fused_lu(const float* x_dev, const float* l_host, const float* u_host,
+                                           const void* w_packed_dev, const pq_layer_desc* d, const float* m_out_host,
+                                           const float* m_req_host, pq_shuffle shuf, const float* shortcut_dev,
+                                           int32_t* acc_out_dev, float* y_out_dev, void* q_out_dev,
+                                           pq_stream_t stream);
+
 /* Cyclic shuffle module (Sec. 4.2, Eq. 9-10), fused into one kernel:
  *   Y = CyclicPermute(X):  Y[:, pi(i)] = X[:, i] with pi(i) = (i + shift) mod G (Eq. 8,
  *                          group-level; Eq. 6 for shift = 1)

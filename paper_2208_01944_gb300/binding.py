@@ -33,7 +33,7 @@ EXPORTS = [
     "palquant_cyclic_shuffle_module", "palquant_bitsplit_desc", "palquant_bitsplit_scratch_bytes",
     "palquant_bitsplit_pack_weight_codes_host", "palquant_bitsplit_act", "palquant_bitsplit_conv",
     "palquant_pack_weights_odd_host", "palquant_fake_quant_forward", "palquant_fake_quant_scratch_bytes",
-    "palquant_fake_quant_backward",
+    "palquant_fake_quant_backward", "palquant_quantize_act_lu", "palquant_quantize_layer_fused_lu",
 ]
 
 
@@ -132,6 +132,11 @@ def _load():
                        ("palquant_linear_f32", [_P, _P, _P, _I64, _I32, _I32, _P])):
         getattr(L, name).restype = _I32
         getattr(L, name).argtypes = args
+    L.palquant_quantize_act_lu.restype = _I32
+    L.palquant_quantize_act_lu.argtypes = [_P, _P, _I64, _I32, _I32, _I32, _I32, _I32, _I32, _P, _P, _P]
+    L.palquant_quantize_layer_fused_lu.restype = _I32
+    L.palquant_quantize_layer_fused_lu.argtypes = list(L.palquant_quantize_layer_fused.argtypes[:1]) + [_P, _P] + \
+        list(L.palquant_quantize_layer_fused.argtypes[2:])
     L.palquant_fake_quant_forward.restype = _I32
     L.palquant_fake_quant_forward.argtypes = [_P, _P, _I64, _I32, _I32, _I32, _I32, _P, _P, _P]
     L.palquant_fake_quant_scratch_bytes.restype = ctypes.c_size_t
@@ -417,3 +422,24 @@ def palquant_fake_quant_backward(x_dev, dy_dev, dx_dev, dl_dev, du_dev, P, G, Cg
     _check(lib.palquant_fake_quant_backward(_ptr(x_dev), _ptr(dy_dev), _ptr(dx_dev), _ptr(dl_dev), _ptr(du_dev), P, G,
                                             Cg, bits, kind, _ptr(lf), _ptr(uf), _ptr(scratch_dev), scratch_bytes,
                                             _stream(stream)), "palquant_fake_quant_backward")
+
+
+# ---------------------------------------------------------------- learned bounds at inference
+def palquant_quantize_act_lu(x_dev, q_dev, N, H, W, G, Cg, bits, l, u, code_format=PQ_CODES_INT8, stream=None):
+    """Activation codes with learned per-group bounds l < u (the training forward's codes)."""
+    lf, uf = _f32(l), _f32(u)
+    _check(lib.palquant_quantize_act_lu(_ptr(x_dev), _ptr(q_dev), N, H, W, G, Cg, bits, code_format, _ptr(lf),
+                                        _ptr(uf), _stream(stream)), "palquant_quantize_act_lu")
+
+
+def palquant_quantize_layer_fused_lu(x_dev, l, u, w_packed_dev, d: LayerDesc, m_out, m_req=None, shuf=None,
+                                     shortcut_dev=None, acc_out_dev=None, y_out_dev=None, q_out_dev=None,
+                                     stream=None):
+    """Quantise-on-load with learned per-group bounds l < u, then the layer."""
+    lf, uf = _f32(l), _f32(u)
+    mo = None if m_out is None else _f32(m_out)
+    mr = None if m_req is None else _f32(m_req)
+    _check(lib.palquant_quantize_layer_fused_lu(_ptr(x_dev), _ptr(lf), _ptr(uf), _ptr(w_packed_dev), ctypes.byref(d),
+                                                _ptr(mo), _ptr(mr), shuf or shuffle(1, 1), _ptr(shortcut_dev),
+                                                _ptr(acc_out_dev), _ptr(y_out_dev), _ptr(q_out_dev), _stream(stream)),
+           "palquant_quantize_layer_fused_lu")

@@ -503,6 +503,20 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
 
 bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
 
+// Learned bounds usable by the quantisers: finite, l < u, and fl(1 / fl(u - l)) finite.
+bool valid_bounds(int G, const float* l, const float* u) {
+  for (int g = 0; g < G; ++g) {
+    if (!std::isfinite(l[g]) || !std::isfinite(u[g]) || !(u[g] > l[g])) return false;
+    const float r = u[g] - l[g];
+    if (!std::isfinite(r) || !(r > 0.0f) || !std::isfinite(1.0f / r)) return false;
+  }
+  return true;
+}
+
+pq_status quantize_act_impl(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G, int32_t Cg,
+                            int32_t bits, int32_t code_format, const float* inv_s_host, const float* l_host,
+                            const float* u_host, pq_stream_t stream);
+
 // ---------------------------------------------------------------------------
 // Tensor map of channel-blocked activation codes for the TMA operand loads.
 // Element = 8 bytes, so one 16-byte position is 2 elements and a plane row of
@@ -574,11 +588,16 @@ bool encode_c16_map(const pq_layer_desc* d, const ConvParams& p, const void* q_d
 // Tensor map of fp32 NHWC activations for quantise-on-load: boxes of 32 channels
 // (128 bytes, swizzled 128B so the copy warps read them without bank conflicts)
 // x Wd positions x Hd rows (rows mode), or x 128 positions (flat mode, HW as one
-// dimension).  Out-of-range positions are zero-filled: code 0, the zero padding.
+// dimension).  Out-of-range positions are zero-filled (code 0, the zero padding),
+// or with learned bounds NaN-filled, which that quantiser maps to code 0 whatever
+// the lower bound is.
 bool encode_f32_map(const pq_layer_desc* d, const ConvParams& p, const void* x_dev, CUtensorMap* map) {
   EncodeTiledFn enc = encode_fn();
   if (enc == nullptr) return false;
   std::memset(map, 0, sizeof(*map));
+  // learned bounds: NaN padding (code 0 for any lower bound); else zeros (code 0)
+  const CUtensorMapFloatOOBfill fill =
+      p.q_lu ? CU_TENSOR_MAP_FLOAT_OOB_FILL_NAN_REQUEST_ZERO_FMA : CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE;
   const uint64_t C = static_cast<uint64_t>(d->G) * d->Cin_g, H = d->H, W = d->W;
   cuuint32_t es[4] = {1, 1, 1, 1};
   if (p.mode == pq::kModeFlat) {
@@ -587,14 +606,14 @@ bool encode_f32_map(const pq_layer_desc* d, const ConvParams& p, const void* x_d
     cuuint32_t box[3] = {32u, static_cast<cuuint32_t>(p.flat_box), 1};
     return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(x_dev), dims, strides, box, es,
                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+               fill) == CUDA_SUCCESS;
   }
   cuuint64_t dims[4] = {C, W, H, static_cast<cuuint64_t>(d->N)};
   cuuint64_t strides[3] = {C * 4, W * C * 4, H * W * C * 4};
   cuuint32_t box[4] = {32u, static_cast<cuuint32_t>(p.Wd), static_cast<cuuint32_t>(p.Hd), 1};
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<void*>(x_dev), dims, strides, box, es,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+             fill) == CUDA_SUCCESS;
 }
 
 // ---------------------------------------------------------------------------
@@ -668,7 +687,8 @@ void pack_codes(const ConvParams& p, const pq_layer_desc* d, const int8_t* wq, u
 pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
                            const float* m_out_host, const float* m_req_host, pq_shuffle shuf,
                            const float* shortcut_dev, int32_t* acc_out_dev, float* y_out_dev, void* q_out_dev,
-                           const int* src_group, pq_stream_t stream, const float* inv_s_in = nullptr) {
+                           const int* src_group, pq_stream_t stream, const float* inv_s_in = nullptr,
+                           const float* l_in = nullptr, const float* u_in = nullptr) {
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
   if (q_dev == nullptr || w_packed_dev == nullptr) return PQ_EINVAL;
@@ -683,9 +703,20 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
   // Channel-blocked codes as the only output are stored from registers (the
   // per-channel scatter of the channel shuffle is unstaged too).
   const bool direct_out = acc_out_dev == nullptr && y_out_dev == nullptr && d->code_format != PQ_CODES_INT8;
-  st = plan_conv(d, &p, nullptr, &phases, inv_s_in != nullptr, direct_out);
+  const bool quant_in = inv_s_in != nullptr || l_in != nullptr;
+  st = plan_conv(d, &p, nullptr, &phases, quant_in, direct_out);
   if (st != PQ_OK) return st;
-  if (inv_s_in != nullptr) {
+  if (l_in != nullptr) {
+    // learned bounds: the training forward's codes (sat((x - l) * fl(1/fl(u - l))) * Qp, rounded)
+    if (u_in == nullptr || !valid_bounds(d->G, l_in, u_in)) return PQ_EINVAL;
+    p.q_lu = 1;
+    for (int g = 0; g < d->G; ++g) {
+      p.q_neg_l[g] = -l_in[g];
+      p.q_inv_r[g] = 1.0f / (u_in[g] - l_in[g]);
+    }
+    p.q_qp = static_cast<float>((1 << d->bits_a) - 1);
+    p.q_qmax2 = static_cast<uint32_t>((1 << d->bits_a) - 1) * 0x00010001u;
+  } else if (inv_s_in != nullptr) {
     // reciprocal steps scaled by 2^-b (exact: a power of two) for the saturating form
     const float inv_two_b = 1.0f / static_cast<float>(1 << d->bits_a);
     for (int g = 0; g < d->G; ++g) {
@@ -926,7 +957,26 @@ pq_status palquant_pack_weights(const float* w_host, const pq_layer_desc* d, con
 
 pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G, int32_t Cg,
                                 int32_t bits, int32_t code_format, const float* inv_s_host, pq_stream_t stream) {
-  if (x_dev == nullptr || q_dev == nullptr || inv_s_host == nullptr) return PQ_EINVAL;
+  if (inv_s_host == nullptr) return PQ_EINVAL;
+  return quantize_act_impl(x_dev, q_dev, N, H, W, G, Cg, bits, code_format, inv_s_host, nullptr, nullptr, stream);
+}
+
+pq_status palquant_quantize_act_lu(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G,
+                                   int32_t Cg, int32_t bits, int32_t code_format, const float* l_host,
+                                   const float* u_host, pq_stream_t stream) {
+  if (l_host == nullptr || u_host == nullptr) return PQ_EINVAL;
+  if (G >= 1 && G <= pq::kMaxG && !valid_bounds(G, l_host, u_host)) return PQ_EINVAL;
+  return quantize_act_impl(x_dev, q_dev, N, H, W, G, Cg, bits, code_format, nullptr, l_host, u_host, stream);
+}
+
+}  // extern "C"
+
+namespace {
+
+pq_status quantize_act_impl(const float* x_dev, void* q_dev, int64_t N, int32_t H, int32_t W, int32_t G, int32_t Cg,
+                            int32_t bits, int32_t code_format, const float* inv_s_host, const float* l_host,
+                            const float* u_host, pq_stream_t stream) {
+  if (x_dev == nullptr || q_dev == nullptr) return PQ_EINVAL;
   if (N < 0 || H < 1 || W < 1 || G < 1 || Cg < 1 || bits < 1 || bits > 8) return PQ_EINVAL;
   if (G > pq::kMaxG) return PQ_EUNSUPPORTED;
   if (code_format == PQ_CODES_E4M3) return PQ_EUNSUPPORTED;
@@ -941,15 +991,19 @@ pq_status palquant_quantize_act(const float* x_dev, void* q_dev, int64_t N, int3
     if (!aligned16(x_dev) || !aligned16(q_dev)) return PQ_EINVAL;
     const int pack = code_format == PQ_CODES_C16P2 ? 1 : (code_format == PQ_CODES_C32F4 ? 2 : 0);
     if (pq::launch_quantize_c16(x_dev, static_cast<uint8_t*>(q_dev), N, static_cast<int64_t>(H) * W, G, Cg, bits,
-                                inv_s_host, pack, static_cast<cudaStream_t>(stream)) != 0)
+                                inv_s_host, pack, static_cast<cudaStream_t>(stream), l_host, u_host) != 0)
       return PQ_ECUDA;
     return PQ_OK;
   }
   if (pq::launch_quantize(x_dev, static_cast<uint8_t*>(q_dev), P, G, Cg, bits, inv_s_host,
-                          static_cast<cudaStream_t>(stream)) != 0)
+                          static_cast<cudaStream_t>(stream), l_host, u_host) != 0)
     return PQ_ECUDA;
   return PQ_OK;
 }
+
+}  // namespace
+
+extern "C" {
 
 pq_status palquant_layer_fused(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,
                                const float* m_out_host, const float* m_req_host, pq_shuffle shuf,
@@ -966,6 +1020,16 @@ pq_status palquant_quantize_layer_fused(const float* x_dev, const float* inv_s_h
   if (inv_s_host == nullptr) return PQ_EINVAL;
   return layer_fused_impl(x_dev, w_packed_dev, d, m_out_host, m_req_host, shuf, shortcut_dev, acc_out_dev, y_out_dev,
                           q_out_dev, nullptr, stream, inv_s_host);
+}
+
+pq_status palquant_quantize_layer_fused_lu(const float* x_dev, const float* l_host, const float* u_host,
+                                           const void* w_packed_dev, const pq_layer_desc* d, const float* m_out_host,
+                                           const float* m_req_host, pq_shuffle shuf, const float* shortcut_dev,
+                                           int32_t* acc_out_dev, float* y_out_dev, void* q_out_dev,
+                                           pq_stream_t stream) {
+  if (l_host == nullptr || u_host == nullptr) return PQ_EINVAL;
+  return layer_fused_impl(x_dev, w_packed_dev, d, m_out_host, m_req_host, shuf, shortcut_dev, acc_out_dev, y_out_dev,
+                          q_out_dev, nullptr, stream, nullptr, l_host, u_host);
 }
 
 pq_status palquant_cyclic_shuffle_module(const void* q_dev, const void* w_packed_dev, const pq_layer_desc* d,

@@ -654,6 +654,34 @@ __device__ __forceinline__ uint4 epi_codes16(const uint32_t (&v)[16], float m_sa
   return w;
 }
 
+// Quantise-on-load with learned bounds: the codes rint(sat((x - l) * inv_r) * Qp)
+// of 16 fp32 values, one rounding per operation (x - l as x + (-l), exact), the
+// rounding to an integer by the fp32 add of 1.5 * 2^23 (its low 16 bits); sat
+// maps NaN to 0, so NaN-filled padding gives code 0 whatever l is.  The product
+// with Qp is a scalar __fmul_rn: a packed mul.rn.f32x2 followed by the packed add
+// was fused into one FMA by the compiler (the product then not rounded first),
+// which changes the rounding at ties.
+__device__ __forceinline__ uint4 lu_codes16(const uint32_t (&v)[16], float neg_l, float inv_r, float qp,
+                                            uint32_t qmax2) {
+  uint32_t h[8];
+#pragma unroll
+  for (int j = 0; j < 16; j += 2) {
+    float d0, d1, y0, y1, r0, r1;
+    add2_rn(__uint_as_float(v[j]), __uint_as_float(v[j + 1]), neg_l, d0, d1);
+    const float c0 = mul_sat(d0, inv_r), c1 = mul_sat(d1, inv_r);
+    y0 = __fmul_rn(c0, qp);
+    y1 = __fmul_rn(c1, qp);
+    add2_rn(y0, y1, 12582912.0f, r0, r1);
+    h[j >> 1] = __vimin_s16x2_relu(__byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x5410), qmax2);
+  }
+  uint4 w;
+  w.x = __byte_perm(h[0], h[1], 0x6420);
+  w.y = __byte_perm(h[2], h[3], 0x6420);
+  w.z = __byte_perm(h[4], h[5], 0x6420);
+  w.w = __byte_perm(h[6], h[7], 0x6420);
+  return w;
+}
+
 // Code packing of the channel-blocked output: 0 one code per byte, 1 four 2-bit
 // codes per byte, 2 two FP4 nibbles per byte.
 __device__ __forceinline__ int codes_pack(const ConvParams& p) { return p.codes_p2 ? 1 : (p.codes_f4 ? 2 : 0); }
@@ -688,7 +716,7 @@ __device__ __forceinline__ long long codes_offset(const ConvParams& p, int pack,
 // one for the row's 32 FP4 nibbles.  Positions outside the image were
 // zero-filled by the TMA unit: code 0, the zero padding.
 // --------------------------------------------------------------------------
-template <bool F4>
+template <bool F4, bool LU>
 __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t st_base,
                                            int64_t it0, int64_t it1, const WaitCtx& ctx) {
   const int tid = threadIdx.x - 32 * kFirstLoadWarp;
@@ -705,8 +733,15 @@ __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars
   Ring r{0, 0, static_cast<uint32_t>(p.a_stages)};
   bool ok = true;
   Item item = item_begin(p, it0);
+  const float qp = p.q_qp;
   for (int64_t it = it0; it < it1 && ok; ++it, item_next(p, item)) {
-    const float m_sat = p.q_inv_sat[p.src_group[item.g]];
+    const int sg = p.src_group[item.g];
+    const float m_sat = LU ? p.q_inv_r[sg] : p.q_inv_sat[sg];
+    const float neg_l = LU ? p.q_neg_l[sg] : 0.0f;
+    auto codes16 = [&](const uint32_t (&x)[16]) {
+      if constexpr (LU) return lu_codes16(x, neg_l, m_sat, qp, qmax2);
+      else return epi_codes16(x, m_sat, two_b, qmax2);
+    };
     for (int kb = 0; kb < p.n_kb; ++kb) {
       if (!warp_wait(bars.pk_full(r.stage), r.phase, ctx)) { ok = false; break; }
       if (!warp_wait(bars.a_empty(r.stage), r.phase ^ 1u, ctx)) { ok = false; break; }
@@ -731,7 +766,7 @@ __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars
                            : "r"(a)
                            : "memory");
             }
-            packed[h] = pack4_word(epi_codes16(v, m_sat, two_b, qmax2));
+            packed[h] = pack4_word(codes16(v));
           }
           asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(out), "r"(packed[0].x), "r"(packed[0].y),
                        "r"(packed[1].x), "r"(packed[1].y)
@@ -754,8 +789,8 @@ __device__ __forceinline__ void quant_role(const ConvParams& p, const Bars& bars
                          : "r"(b)
                          : "memory");
           }
-          const uint4 w0 = epi_codes16(v, m_sat, two_b, qmax2);
-          const uint4 w1 = epi_codes16(u, m_sat, two_b, qmax2);
+          const uint4 w0 = codes16(v);
+          const uint4 w1 = codes16(u);
           asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(out), "r"(w0.x), "r"(w0.y), "r"(w0.z),
                        "r"(w0.w)
                        : "memory");
@@ -1059,7 +1094,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
 // One instance per operand type (F4: packed FP4 codes and block-scaled FP4 MMAs;
 // else one code per byte or packed 2-bit codes, FP8 MMAs), so that each carries
 // only its own MMA loops and epilogue paths (a smaller instruction footprint).
-template <bool F4>
+template <bool F4, bool LU>
 __global__ void __launch_bounds__(kConvThreads, 1)
     pq_conv_tc_kernel(const __grid_constant__ ConvParams p, const __grid_constant__ CUtensorMap tmA) {
   extern __shared__ uint8_t smem_raw[];
@@ -1136,7 +1171,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   } else if (warp < kFirstEpiWarp && !p.a_tma) {
     loader_role(p, bars, a_base, it0, it1, WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else if (warp < kFirstEpiWarp && p.a_quant) {
-    quant_role<F4>(p, bars, a_base, base + p.smem_pk_off, it0, it1,
+    quant_role<F4, LU>(p, bars, a_base, base + p.smem_pk_off, it0, it1,
                WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else if (warp < kFirstEpiWarp && p.a_unpack) {
     unpack_role(p, bars, a_base, base + p.smem_pk_off, it0, it1,
@@ -1158,22 +1193,30 @@ __global__ void __launch_bounds__(kConvThreads, 1)
 }
 
 int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream) {
-  static int attr_set_for_device[2][64] = {{0}};
+  // one instance per operand type (FP4 or byte codes) and quantiser form (learned
+  // bounds or not); the attribute is set once per instance and device
+  static int attr_set_for_device[4][64] = {{0}};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return -1;
   const int need = static_cast<int>(p.smem_bytes) + 1024;
-  const int f4 = p.codes_f4 ? 1 : 0;
-  if (dev < 64 && attr_set_for_device[f4][dev] < need) {
-    const cudaError_t e =
-        f4 ? cudaFuncSetAttribute(pq_conv_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem)
-           : cudaFuncSetAttribute(pq_conv_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
-    if (e != cudaSuccess) return -1;
-    attr_set_for_device[f4][dev] = kMaxSmem;
+  const int f4 = p.codes_f4 ? 1 : 0, lu = p.q_lu ? 1 : 0;
+  const int v = f4 * 2 + lu;
+  const void* fn = f4 ? (lu ? reinterpret_cast<const void*>(pq_conv_tc_kernel<true, true>)
+                            : reinterpret_cast<const void*>(pq_conv_tc_kernel<true, false>))
+                      : (lu ? reinterpret_cast<const void*>(pq_conv_tc_kernel<false, true>)
+                            : reinterpret_cast<const void*>(pq_conv_tc_kernel<false, false>));
+  if (dev < 64 && attr_set_for_device[v][dev] < need) {
+    if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) != cudaSuccess) return -1;
+    attr_set_for_device[v][dev] = kMaxSmem;
   }
-  if (f4)
-    pq_conv_tc_kernel<true><<<grid, kConvThreads, need, stream>>>(p, tma_a);
+  if (f4 && lu)
+    pq_conv_tc_kernel<true, true><<<grid, kConvThreads, need, stream>>>(p, tma_a);
+  else if (f4)
+    pq_conv_tc_kernel<true, false><<<grid, kConvThreads, need, stream>>>(p, tma_a);
+  else if (lu)
+    pq_conv_tc_kernel<false, true><<<grid, kConvThreads, need, stream>>>(p, tma_a);
   else
-    pq_conv_tc_kernel<false><<<grid, kConvThreads, need, stream>>>(p, tma_a);
+    pq_conv_tc_kernel<false, false><<<grid, kConvThreads, need, stream>>>(p, tma_a);
   return cudaGetLastError() == cudaSuccess ? 0 : -1;
 }
 

@@ -64,6 +64,13 @@ struct ConvParams {
   float q_inv_sat[kMaxG];
   float q_two_b;
   uint32_t q_qmax2;  // Qp in both 16-bit halves
+  // q_lu = 1: learned bounds l < u per group instead (Eq. 2 as trained):
+  // code = rint(sat((x - l) * q_inv_r[g]) * Qp), q_inv_r = fl(1 / fl(u - l)),
+  // q_neg_l = -l, q_qp = Qp; out-of-image positions are NaN-filled (code 0).
+  int q_lu;
+  float q_neg_l[kMaxG];
+  float q_inv_r[kMaxG];
+  float q_qp;
   uint32_t q_box_bytes;  // staging bytes per 32-channel box (a multiple of 1024: the 128B swizzle atom)
   int pk_box_w, pk_off;
   uint32_t pk_stage_bytes, smem_pk_off;
@@ -131,9 +138,10 @@ int launch_bitsplit_act(const uint8_t* q, uint8_t* xs, int64_t N, int64_t HW, in
 // pack: 0 one code per byte [N][C/16][HW][16]; 1 four 2-bit codes per byte
 // [N][C/16][HW][4 B]; 2 two 4-bit codes per byte [N][C/32][HW][16 B].
 int launch_quantize_c16(const float* x, uint8_t* q, int64_t N, int64_t HW, int G, int Cg, int bits, const float* inv_s,
-                        int pack, cudaStream_t stream);
+                        int pack, cudaStream_t stream, const float* l = nullptr, const float* u = nullptr);
+// l non-NULL: learned bounds l, u per group instead of inv_s (see quantize.cu).
 int launch_quantize(const float* x, uint8_t* q, int64_t P, int G, int Cg, int bits, const float* inv_s,
-                    cudaStream_t stream);
+                    cudaStream_t stream, const float* l = nullptr, const float* u = nullptr);
 int launch_act_sum(const float* x, int64_t P, int G, int Cg, double* partial, int nblocks, cudaStream_t stream);
 int launch_act_sum_finish(const double* partial, int nblocks, int G, double* sums, cudaStream_t stream);
 int launch_watchdog_selftest(unsigned int* err, uint64_t limit_ns, cudaStream_t stream);
