@@ -735,7 +735,8 @@ def fp4_summary(r, c, pk, world):
         "ms_per_step": r["ms_per_step"],
         "timed": "one launch per step: quantiser fused into the layer, packed FP4 operands and codes",
         "code_layout": "packed FP4 nibbles [N][C/32][H][W][16 B], two 2-bit codes per byte",
-        "dtype": "fp32 activations -> 2-bit codes as FP4 e2m1 x e2m1 weights, block scales 2^-4 -> f32 (exact)",
+        "dtype": "e2m1",
+        "dtype_detail": "fp32 activations -> 2-bit codes as FP4 e2m1 x e2m1 weights, block scales 2^-4 -> f32 (exact)",
         "roofline_kernels": [
             {"kernel": "pq_conv_tc_kernel<FP4> (quantise on load)", "bound": "hbm", "achieved": gbs,
              "peak": pk["hbm_gbs"], "unit": "GB/s", "frac": gbs / pk["hbm_gbs"],
@@ -902,7 +903,8 @@ def run_ours(args, rank, world, local_rank):
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": K, "warmup": args.warmup,
         "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
-        "dtype": "fp32 activations -> u8 codes, e4m3 x e4m3 -> f32 (exact integer)", "data": "synthetic",
+        "dtype": "e4m3", "dtype_detail": "fp32 activations -> u8 codes, e4m3 x e4m3 -> f32 (exact integer)",
+        "data": "synthetic",
         "config": {"workload": WORKLOAD, "global_batch": c.N * world, "per_gpu_batch": c.N,
                    "timed": "one launch per step: quantiser fused into the layer (fp32 NHWC -> next-layer codes)",
                    "code_layout": "output codes channel-blocked [N][C/16][H][W][16], one byte per code",
