@@ -761,6 +761,7 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
   if (grid <= 0) return PQ_OK;
   CUtensorMap map;
   std::memset(&map, 0, sizeof(map));
+  p.pdl = 1;  // programmatic dependent launch: the set-up overlaps the previous grid's last CTAs
   if (p.a_quant) {
     if (!encode_f32_map(d, p, q_dev, &map)) return PQ_ECUDA;
   } else if (p.a_tma && !encode_c16_map(d, p, q_dev, &map)) {

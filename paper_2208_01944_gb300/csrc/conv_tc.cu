@@ -1110,6 +1110,8 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   uint32_t* tap_a16 = reinterpret_cast<uint32_t*>(bar_block + 8 * bars.words() + 16);  // p.taps entries
   for (int t = threadIdx.x; t < p.taps; t += blockDim.x) tap_a16[t] = p.tap_a16[t];
 
+  // let the next dependent launch on the stream start its CTAs as SMs free up
+  if (p.pdl && threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   if (threadIdx.x == 0) {
     for (int s = 0; s < bars.A; ++s) {
       // TMA, or one arrival per copy warp
@@ -1152,6 +1154,11 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     tc_fence_after();
   }
 
+  // A programmatic dependent launch: the set-up above (barriers, tensor memory,
+  // scale factors) overlaps the previous grid's last CTAs; every global read and
+  // write below waits for that grid to complete (it may produce this launch's
+  // inputs or read its outputs), so stream order holds.
+  if (p.pdl) asm volatile("griddepcontrol.wait;" ::: "memory");
   const int64_t it0 = static_cast<int64_t>(blockIdx.x) * p.items / gridDim.x;
   const int64_t it1 = static_cast<int64_t>(blockIdx.x + 1) * p.items / gridDim.x;
   const uint32_t a_base = base;
@@ -1181,6 +1188,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     // epilogue warpgroup.
     const bool third = p.a_tma && !p.a_unpack && !p.a_quant;
     const int first = third ? kFirstLoadWarp : kFirstEpiWarp;
+
     epilogue_role<F4>(p, bars, tmem_base, gbase + p.smem_stage_off, first, third ? kEpiGroups + 1 : kEpiGroups, it0, it1,
                   WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_EPILOGUE});
   }
@@ -1209,15 +1217,26 @@ int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cuda
     if (cudaFuncSetAttribute(fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem) != cudaSuccess) return -1;
     attr_set_for_device[v][dev] = kMaxSmem;
   }
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(kConvThreads);
+  cfg.dynamicSmemBytes = static_cast<size_t>(need);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = p.pdl ? 1 : 0;
+  cudaError_t e;
   if (f4 && lu)
-    pq_conv_tc_kernel<true, true><<<grid, kConvThreads, need, stream>>>(p, tma_a);
+    e = cudaLaunchKernelEx(&cfg, pq_conv_tc_kernel<true, true>, p, tma_a);
   else if (f4)
-    pq_conv_tc_kernel<true, false><<<grid, kConvThreads, need, stream>>>(p, tma_a);
+    e = cudaLaunchKernelEx(&cfg, pq_conv_tc_kernel<true, false>, p, tma_a);
   else if (lu)
-    pq_conv_tc_kernel<false, true><<<grid, kConvThreads, need, stream>>>(p, tma_a);
+    e = cudaLaunchKernelEx(&cfg, pq_conv_tc_kernel<false, true>, p, tma_a);
   else
-    pq_conv_tc_kernel<false, false><<<grid, kConvThreads, need, stream>>>(p, tma_a);
-  return cudaGetLastError() == cudaSuccess ? 0 : -1;
+    e = cudaLaunchKernelEx(&cfg, pq_conv_tc_kernel<false, false>, p, tma_a);
+  return e == cudaSuccess && cudaGetLastError() == cudaSuccess ? 0 : -1;
 }
 
 }  // namespace pq

@@ -67,6 +67,11 @@ struct ConvParams {
   // q_lu = 1: learned bounds l < u per group instead (Eq. 2 as trained):
   // code = rint(sat((x - l) * q_inv_r[g]) * Qp), q_inv_r = fl(1 / fl(u - l)),
   // q_neg_l = -l, q_qp = Qp; out-of-image positions are NaN-filled (code 0).
+  // pdl = 1: launched as a programmatic dependent of the previous kernel on the
+  // stream: a CTA's set-up (barriers, tensor memory) may run while that kernel's
+  // last CTAs still run; every global access waits for it to complete (stream
+  // order holds), and every CTA lets the next such launch start early.
+  int pdl;
   int q_lu;
   float q_neg_l[kMaxG];
   float q_inv_r[kMaxG];
