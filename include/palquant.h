@@ -111,7 +111,18 @@ typedef struct {
     int32_t bits_out;    /* requantised output code bits, 1..4 */
     int32_t relu;        /* 1: ReLU after the rescale (and the shortcut add) */
     int32_t code_format; /* pq_code_format of the input codes and the output codes */
+    int32_t flags;       /* PQ_LAYER_* bits; 0 for none */
 } pq_layer_desc;
+
+/* pq_layer_desc.flags bit: the kernel launched on the stream immediately before this
+ * call writes neither this layer's input (codes or fp32 activations) nor its packed
+ * weights, e.g. consecutive layers over independent batches.  The layer kernel then
+ * starts loading them and computing on them while that kernel's last blocks still
+ * run; its stores (and its reads of the shortcut) still wait for that kernel to
+ * complete.  The caller answers for the promise: a layer
+ * that consumes the previous kernel's output (the next layer of a network) must
+ * leave the bit clear, and then every access waits.  Other bits: PQ_EINVAL. */
+#define PQ_LAYER_INPUTS_READY 1
 
 /* Human-readable name of a status. */
 const char* palquant_strerror(pq_status s);

@@ -19,6 +19,7 @@ LIB_PATH = os.path.join(HERE, "libpalquant.so")
 
 PQ_OK, PQ_EINVAL, PQ_EUNSUPPORTED, PQ_ECUDA, PQ_ETIMEOUT = 0, -1, -2, -3, -4
 PQ_CODES_INT8, PQ_CODES_E4M3, PQ_CODES_C16, PQ_CODES_C16P2, PQ_CODES_C32F4 = 0, 1, 2, 3, 4
+PQ_LAYER_INPUTS_READY = 1  # pq_layer_desc.flags: the previous kernel on the stream writes neither input nor weights
 
 # Every symbol include/palquant.h declares.
 EXPORTS = [
@@ -46,7 +47,7 @@ class PalquantError(RuntimeError):
 class LayerDesc(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "N", "H", "W", "G", "Cin_g", "Cout_g", "kh", "kw", "stride", "pad", "bits_a", "bits_w", "bits_out", "relu",
-        "code_format")]
+        "code_format", "flags")]
 
 
 class Shuffle(ctypes.Structure):
@@ -190,9 +191,9 @@ def strerror(status: int) -> str:
 
 
 def layer_desc(N, H, W, G, Cin_g, Cout_g, k, stride=1, pad=0, bits_a=2, bits_w=2, bits_out=2, relu=1,
-               code_format=PQ_CODES_INT8, kw=None) -> LayerDesc:
+               code_format=PQ_CODES_INT8, kw=None, flags=0) -> LayerDesc:
     return LayerDesc(N, H, W, G, Cin_g, Cout_g, k, k if kw is None else kw, stride, pad, bits_a, bits_w, bits_out,
-                     int(relu), code_format)
+                     int(relu), code_format, int(flags))
 
 
 def shuffle(kind=1, shift=1, perm=None):

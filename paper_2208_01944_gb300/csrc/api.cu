@@ -87,6 +87,7 @@ pq_status validate_desc(const pq_layer_desc* d) {
   if (d->bits_a < 1 || d->bits_a > 8 || d->bits_w < 2 || d->bits_w > 8 || d->bits_out < 1 || d->bits_out > 8)
     return PQ_EINVAL;
   if (d->relu != 0 && d->relu != 1) return PQ_EINVAL;
+  if ((d->flags & ~PQ_LAYER_INPUTS_READY) != 0) return PQ_EINVAL;
   if (d->code_format != PQ_CODES_INT8 && d->code_format != PQ_CODES_E4M3 && d->code_format != PQ_CODES_C16 &&
       d->code_format != PQ_CODES_C16P2 && d->code_format != PQ_CODES_C32F4)
     return PQ_EINVAL;
@@ -762,6 +763,7 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
   CUtensorMap map;
   std::memset(&map, 0, sizeof(map));
   p.pdl = 1;  // programmatic dependent launch: the set-up overlaps the previous grid's last CTAs
+  p.pdl_early_loads = (d->flags & PQ_LAYER_INPUTS_READY) ? 1 : 0;
   if (p.a_quant) {
     if (!encode_f32_map(d, p, q_dev, &map)) return PQ_ECUDA;
   } else if (p.a_tma && !encode_c16_map(d, p, q_dev, &map)) {

@@ -1157,8 +1157,14 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   // A programmatic dependent launch: the set-up above (barriers, tensor memory,
   // scale factors) overlaps the previous grid's last CTAs; every global read and
   // write below waits for that grid to complete (it may produce this launch's
-  // inputs or read its outputs), so stream order holds.
-  if (p.pdl) asm volatile("griddepcontrol.wait;" ::: "memory");
+  // inputs or read its outputs), so stream order holds.  Where the caller has
+  // promised that the previous kernel writes neither the activations nor the
+  // weights (pdl_early_loads), only the epilogue warps wait: the others' global
+  // accesses are those loads (the producer's copies, the loader warps' reads),
+  // and the quantiser and MMA warps work in shared and tensor memory.
+  const bool third_epi = p.a_tma && !p.a_unpack && !p.a_quant;  // warps 2-5 run the epilogue too
+  const bool epi_warp = warp >= kFirstEpiWarp || (third_epi && warp >= kFirstLoadWarp);
+  if (p.pdl && (epi_warp || !p.pdl_early_loads)) asm volatile("griddepcontrol.wait;" ::: "memory");
   const int64_t it0 = static_cast<int64_t>(blockIdx.x) * p.items / gridDim.x;
   const int64_t it1 = static_cast<int64_t>(blockIdx.x + 1) * p.items / gridDim.x;
   const uint32_t a_base = base;

@@ -72,6 +72,10 @@ struct ConvParams {
   // last CTAs still run; every global access waits for it to complete (stream
   // order holds), and every CTA lets the next such launch start early.
   int pdl;
+  // pdl_early_loads = 1 (the caller's PQ_LAYER_INPUTS_READY): only the epilogue
+  // warps (every global store) wait for the previous kernel; loads, quantisation
+  // and MMAs may start before it completes.
+  int pdl_early_loads;
   int q_lu;
   float q_neg_l[kMaxG];
   float q_inv_r[kMaxG];

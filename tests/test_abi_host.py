@@ -126,11 +126,17 @@ def test_invalid_arguments_rejected_before_launch():
         B.layer_desc(1, 8, 8, 2, 32, 32, 3, 0, 1),       # stride 0
         B.layer_desc(1, 2, 2, 2, 32, 32, 5, 1, 0),       # output would be empty
         B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, bits_a=9),
+        B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, flags=2),    # unknown flag bit
+        B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, flags=-1),
     ]
     for d in bad_descs:
         with pytest.raises(B.PalquantError) as e:
             B.palquant_layer_fused(16, 16, d, [1.0] * 2, [1.0] * 2, acc_out_dev=16)
         assert e.value.status == B.PQ_EINVAL
+    # the inputs-ready promise is a valid flag: planning accepts it and plans the same tiles
+    ready = B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, code_format=B.PQ_CODES_C16, flags=B.PQ_LAYER_INPUTS_READY)
+    plain = B.layer_desc(1, 8, 8, 2, 32, 32, 3, 1, 1, code_format=B.PQ_CODES_C16)
+    assert B.palquant_conv_plan(ready).as_dict() == B.palquant_conv_plan(plain).as_dict()
     # no output requested
     with pytest.raises(B.PalquantError) as e:
         B.palquant_layer_fused(16, 16, good, [1.0] * 2, [1.0] * 2)

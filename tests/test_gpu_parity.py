@@ -539,6 +539,56 @@ def test_quantize_layer_fused_matches_oracle(B, c, fmt):
     assert_layer_parity(c, ref, _run_quant_fused(B, c, ref, fmt))
 
 
+@pytest.mark.parametrize("c,fmt", [(QF_CASES[0], 2), (QF_CASES[2], 2), (QF_CASES[12], 0), (QF_CASES[4], 2),
+                                   (Case(2, 36, 40, 2, 64, 64, 3, 1, 1, seed=136), 4)], ids=str)
+def test_quantize_layer_fused_inputs_ready_overlapped(B, c, fmt):
+    """PQ_LAYER_INPUTS_READY: back-to-back launches over independent inputs, each one's
+    loads starting while the previous launch still runs; two output buffers written
+    in turn, so every store must also wait for the launch before (the last two
+    launches' codes are checked).  Results equal single flagless launches bit for bit
+    and the oracle's codes."""
+    from layer_cases import code_bytes, from_format
+
+    from paper_2208_01944_gb300 import synth
+
+    r0 = prepare(c)
+    x_np = [r0["x"]] + [synth.half_normal(r0["x"].shape, synth.generator(c.seed + 1000 * i)) for i in range(1, 5)]
+    kw = dict(code_format=fmt)
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad, c.bits, c.bits, c.bo, int(c.relu), **kw)
+    dr = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, c.k, c.stride, c.pad, c.bits, c.bits, c.bo, int(c.relu),
+                      flags=B.PQ_LAYER_INPUTS_READY, **kw)
+    # one weight set and one set of steps for all launches (those of the first input)
+    nbytes = B.palquant_packed_weight_bytes(d)
+    wp = torch.empty(nbytes, dtype=torch.uint8, device="cuda")
+    B.palquant_pack_weights(r0["w"], d, r0["inv_sw"], wp, nbytes)
+    shape = (c.N, c.Ho, c.Wo, c.G * c.Cout)
+    n_out = code_bytes(int(np.prod(shape)), fmt)
+    xs = [torch.from_numpy(x).cuda() for x in x_np]
+    shuf = B.shuffle(c.kind, c.shift, c.perm)
+    sc = None if r0["shortcut"] is None else torch.from_numpy(r0["shortcut"]).cuda()
+
+    def launch(x, desc, out):
+        B.palquant_quantize_layer_fused(x, r0["inv_s"], wp, desc, r0["m_out"], r0["m_req"], shuf, sc, None, None, out)
+
+    outs = [torch.full((n_out,), 255, dtype=torch.uint8, device="cuda") for _ in range(2)]
+    for i, x in enumerate(xs):
+        launch(x, dr, outs[i % 2])
+    assert B.palquant_sync_check() == B.PQ_OK
+    for i in (3, 4):
+        single = torch.full((n_out,), 255, dtype=torch.uint8, device="cuda")
+        launch(xs[i], d, single)
+        assert B.palquant_sync_check() == B.PQ_OK
+        assert torch.equal(outs[i % 2], single), i
+        # against the oracle: input i quantised with the first input's steps, the same layer
+        q = oracle.quantize_act(x_np[i], c.G, c.bits, r0["inv_s"])
+        acc = oracle.group_conv(q, oracle.quantize_weights(r0["w"], c.bits, r0["inv_sw"]), c.stride, c.pad)
+        _, _, q_ref = oracle.epilogue(acc.reshape(-1, c.G * c.Cout), c.G, r0["m_out"], r0["m_req"], c.kind, c.shift,
+                                      c.perm, None if sc is None else r0["shortcut"].reshape(-1, c.G * c.Cout),
+                                      c.relu, c.bo)
+        got = from_format(single.cpu().numpy(), fmt, c.N, c.Ho, c.Wo, c.G * c.Cout).reshape(-1, c.G * c.Cout)
+        assert np.array_equal(got, q_ref), i
+
+
 QF_F4_CASES = [
     Case(1, 28, 28, 2, 64, 32, 3, 1, 1, seed=130),
     Case(2, 13, 11, 3, 64, 96, 3, 1, 1, seed=131),                    # odd sizes
