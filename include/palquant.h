@@ -353,7 +353,9 @@ pq_status palquant_watchdog_selftest(uint64_t limit_ns, pq_stream_t stream);
 /* whose M-bit sums could reach 2^24 return PQ_EUNSUPPORTED.                   */
 /* ------------------------------------------------------------------------ */
 
-/* The decomposed layer's descriptor: Cin_g multiplied by Ga Gw, bits_a = B. */
+/* The decomposed layer's descriptor: Cin_g multiplied by Ga Gw, bits_a = B,
+ * PQ_LAYER_INPUTS_READY cleared (the decomposed layer reads the slices that the
+ * kernel launched just before it writes). */
 pq_status palquant_bitsplit_desc(const pq_layer_desc* d, int32_t bits_b, pq_layer_desc* out);
 
 /* Bytes of the slice buffer (N H W Ga Gw Cin_g); 0 if unsupported. */

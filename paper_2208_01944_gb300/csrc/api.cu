@@ -1085,6 +1085,8 @@ pq_status bitsplit_layer(const pq_layer_desc* d, int bits_b, pq_layer_desc* out,
   const int64_t taps = static_cast<int64_t>(d->kh) * d->kw;
   if (taps * d->Cin_g * ((1LL << d->bits_a) - 1) * (1LL << (d->bits_w - 1)) >= (1LL << 24)) return PQ_EUNSUPPORTED;
   *out = *d;
+  // the derived layer reads the split codes the kernel before it writes
+  out->flags = d->flags & ~PQ_LAYER_INPUTS_READY;
   out->Cin_g = d->Cin_g * Ga * Gw;
   out->bits_a = bits_b;
   out->bits_w = bits_b < 2 ? 2 : bits_b;

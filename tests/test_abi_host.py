@@ -187,6 +187,15 @@ def test_bitsplit_weight_blocks_are_shifted_slices(M, Bb):
             assert np.array_equal(blk, ws[j].astype(np.int64) << ((i + j) * B_bits))
 
 
+def test_bitsplit_desc_clears_inputs_ready():
+    """The decomposed convolution reads the slices the kernel before it writes, so the
+    caller's inputs-ready promise does not carry over to it."""
+    d = B.layer_desc(2, 8, 8, 1, 32, 32, 3, 1, 1, bits_a=4, bits_w=4, bits_out=4, code_format=B.PQ_CODES_C16,
+                     flags=B.PQ_LAYER_INPUTS_READY)
+    t = B.palquant_bitsplit_desc(d, 2)
+    assert t.flags == 0 and t.Cin_g == 32 * 4 and t.bits_a == 2
+
+
 def test_bitsplit_unsupported_shapes():
     # 6-bit on 2-bit hardware: shifted slices reach 3 * 2^8, beyond exact E4M3
     d = B.layer_desc(1, 8, 8, 1, 32, 16, 3, 1, 1, 6, 6, 2)
