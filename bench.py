@@ -180,6 +180,55 @@ def whole_job_rate(units_per_rank: float, world: int, ms: float) -> float:
     return units_per_rank * world / (ms / 1e3)
 
 
+def queue_ahead(stream, ms: float = 3.0):
+    """Enqueue a bounded spin kernel (torch's cycle-count sleep, about `ms` at the SM
+    clock) on `stream` just before a timed region.  While it runs, the host queues the
+    region's start event and its first launches, so the region holds device work
+    only: no host launch latency before the first kernel, and no idle GPU entering
+    the region."""
+    import torch
+
+    with torch.cuda.stream(stream):
+        torch.cuda._sleep(int(ms * 1e-3 * 2.0e9))
+
+
+def timed_region(dev, stream, launch, n):
+    """Device time (ms) of `n` back-to-back launches between two CUDA events on
+    `stream`, queued behind queue_ahead(); `launch(i)` enqueues launch i on `stream`."""
+    import torch
+
+    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    queue_ahead(stream)
+    with torch.cuda.stream(stream):
+        start.record(stream)
+        for i in range(n):
+            launch(i)
+        stop.record(stream)
+    torch.cuda.synchronize(dev)
+    return start.elapsed_time(stop)
+
+
+def launch_spread(dev, stream, launch, n):
+    """Diagnostic pass (outside any timed region): `n` launches with an event pair
+    around each, queued behind queue_ahead(); min / median / max device time per
+    launch in microseconds.  The events between launches keep each launch from
+    overlapping its neighbour's tail, so these times sit a little above the
+    region average."""
+    import torch
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(n)]
+    queue_ahead(stream)
+    with torch.cuda.stream(stream):
+        for i in range(n):
+            ev[i][0].record(stream)
+            launch(i)
+            ev[i][1].record(stream)
+    torch.cuda.synchronize(dev)
+    t = sorted(a.elapsed_time(b) * 1e3 for a, b in ev)
+    return {"min_us": t[0], "median_us": t[len(t) // 2], "max_us": t[-1], "launches": n,
+            "how": "separate pass, an event pair around each launch"}
+
+
 class ClockSampler:
     """nvidia-smi clock / throttle sampling while the timed region runs."""
 
@@ -335,16 +384,10 @@ def measure_layer_configs(dev, args):
             for i in range(3):
                 launch(i % n_sets)
         torch.cuda.synchronize(dev)
-        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        with torch.cuda.stream(stream):
-            e0.record(stream)
-            for i in range(reps):
-                launch(i % n_sets)
-            e1.record(stream)
-        torch.cuda.synchronize(dev)
+        ms = timed_region(dev, stream, lambda i: launch(i % n_sets), reps)
         st = B.palquant_sync_check(stream)
         assert st == B.PQ_OK, B.strerror(st)
-        return e0.elapsed_time(e1) / reps
+        return ms / reps
 
     for name, c in workloads.BENCH_CONFIGS.items():
         gen = synth.generator(0)
@@ -543,6 +586,7 @@ def measure_resnet18_paper(dev, world, args):
     torch.cuda.synchronize(dev)
     R = args.resnet_reps
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    queue_ahead(net.stream)
     e0.record(net.stream)
     for i in range(R):
         net.replay(graphs[i & 1])
@@ -583,6 +627,7 @@ def measure_resnet18(dev, world, args):
     torch.cuda.synchronize(dev)
     R = args.resnet_reps
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    queue_ahead(net.stream)
     e0.record(net.stream)
     for i in range(R):
         net.replay(graphs[i & 1])
@@ -643,6 +688,7 @@ def measure_unfused_step(dev, stream, c, xs, q, inv_s, wp, d, m_out, m_req, shuf
     torch.cuda.synchronize(dev)
     ev = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(K)]
     start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    queue_ahead(stream)
     with torch.cuda.stream(stream):
         start.record(stream)
         for i in range(K):
@@ -715,16 +761,9 @@ def measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf
         for i in range(3):
             launch(i)
     torch.cuda.synchronize(dev)
-    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with torch.cuda.stream(stream):
-        start.record(stream)
-        for i in range(K):
-            launch(i)
-        stop.record(stream)
-    torch.cuda.synchronize(dev)
+    t = timed_region(dev, stream, launch, K) / K
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
-    t = start.elapsed_time(stop) / K
     return {"ms_per_step": max_over_ranks(t, world, dev), "t_step": t}
 
 
@@ -781,8 +820,12 @@ def run_ours(args, rank, world, local_rank):
     d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w, c.bits_out,
                      int(c.relu), code_format=fmt)
     s_w = B.palquant_weight_steps(w_np, d)
-    inv_s = np.array([np.float32(1.0 / np.float64(v)) for v in s_a], dtype=np.float32)
-    inv_sw = np.array([np.float32(1.0 / np.float64(v)) for v in s_w], dtype=np.float32)
+    # fl(1 / s) from the library: the requantisation multiplier of s_w = s_a = 1 onto the
+    # step s, with no permutation
+    ones = np.ones(c.G, dtype=np.float32)
+    no_shuffle = B.shuffle(0, 0)
+    inv_s = B.palquant_epilogue_scales(c.G, ones, ones, 1.0, s_a, no_shuffle)[1]
+    inv_sw = B.palquant_epilogue_scales(c.G, ones, ones, 1.0, s_w, no_shuffle)[1]
     nbytes = B.palquant_packed_weight_bytes(d)
     wp = torch.empty(nbytes, dtype=torch.uint8, device=dev)
     B.palquant_pack_weights(w_np, d, inv_sw, wp, nbytes)
@@ -810,33 +853,35 @@ def run_ours(args, rank, world, local_rank):
         B.palquant_quantize_layer_fused(xs[i & 1], inv_s, wp, d_ready, m_out, m_req, shuf, None, None, None, q_out,
                                         stream=s)
 
-    # ---- warm-up
-    with torch.cuda.stream(stream):
-        for i in range(args.warmup):
-            step(i, stream)
-    torch.cuda.synchronize(dev)
+    # ---- warm-up: at least W steps, and the GPU kept busy until the clock sampler
+    # (started first) is running, so the timed region does not start from an idle GPU
+    sampler = ClockSampler(local_rank)
+    sampler.start()
+    t_warm = time.perf_counter()
+    n_warm = 0
+    while n_warm < args.warmup or time.perf_counter() - t_warm < 0.5:
+        with torch.cuda.stream(stream):
+            for _ in range(50):
+                step(n_warm, stream)
+                n_warm += 1
+        torch.cuda.synchronize(dev)
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
 
     # ---- timed region: K steps (one launch each) between two events on the
-    # launching stream; the step's average launch duration is the region / K
-    # (launch gaps included), with no events between the launches
+    # launching stream, queued behind a short spin kernel so that the region holds
+    # the K launches back to back (no host launch latency before the first); the
+    # step's average launch duration is the region / K, with no events between the
+    # launches
     K = args.steps
-    start, stop = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    sampler = ClockSampler(local_rank)
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize(dev)
-    sampler.start()
-    time.sleep(0.3)
-    with torch.cuda.stream(stream):
-        start.record(stream)
-        for i in range(K):
-            step(i, stream)
-        stop.record(stream)
-    torch.cuda.synchronize(dev)
+    elapsed_ms = timed_region(dev, stream, lambda i: step(i, stream), K)
     st = B.palquant_sync_check(stream)
     assert st == B.PQ_OK, B.strerror(st)
+    # per-launch spread, from a separate diagnostic pass (not the timed region)
+    spread = launch_spread(dev, stream, lambda i: step(i, stream), max(3, min(K, 200)))
     unfused = measure_unfused_step(dev, stream, c, xs, q, inv_s, wp, d, m_out, m_req, shuf, q_out, K, world)
     fp4 = measure_fp4_step(dev, stream, c, xs, inv_s, w_np, inv_sw, m_out, m_req, shuf, K, world)
     resnet = None if args.no_resnet else measure_resnet18(dev, world, args)
@@ -844,7 +889,6 @@ def run_ours(args, rank, world, local_rank):
     clocks = sampler.stop()
     if world > 1:
         dist.barrier()
-    elapsed_ms = start.elapsed_time(stop)
     t_step = elapsed_ms / K
     elapsed_ms = max_over_ranks(elapsed_ms, world, dev)
     ms_per_step = elapsed_ms / K
@@ -920,7 +964,9 @@ def run_ours(args, rank, world, local_rank):
         "data": "synthetic",
         "config": {"workload": WORKLOAD, "global_batch": c.N * world, "per_gpu_batch": c.N,
                    "timed": "one launch per step: quantiser fused into the layer (fp32 NHWC -> next-layer codes); "
-                            "independent batches, each launch's loads start while the previous launch finishes",
+                            "independent batches, each launch's loads start while the previous launch finishes; "
+                            "the K launches are queued behind a 3 ms spin kernel that precedes the start event",
+                   "warmup_steps_run": n_warm,
                    "code_layout": "output codes channel-blocked [N][C/16][H][W][16], one byte per code",
                    "l2": "inputs larger than L2 (205.5 MB fp32, two buffers used in turn)",
                    "parallelism": f"replicas x{world}"},
@@ -934,6 +980,7 @@ def run_ours(args, rank, world, local_rank):
                 "timed": "pinned host fp32 -> H2D -> fused step -> D2H of the codes, every step; steps "
                          "pipelined over three streams (copies of neighbouring steps overlap the compute)"},
         "gpu_launches": K,
+        "launch_spread": spread,
     }
     line["unfused_step"] = unfused_summary(unfused, c, pk, world)
     line["fp4_step"] = fp4_summary(fp4, c, pk, world)

@@ -121,7 +121,13 @@ typedef struct {
  * run; its stores (and its reads of the shortcut) still wait for that kernel to
  * complete.  The caller answers for the promise: a layer
  * that consumes the previous kernel's output (the next layer of a network) must
- * leave the bit clear, and then every access waits.  Other bits: PQ_EINVAL. */
+ * leave the bit clear, and then every access waits.  Kernels launched earlier
+ * than that one have completed before the loads start (each layer kernel lets its
+ * dependent launch start only after its own wait for the kernel before it), so a
+ * layer may read what a layer two launches back wrote.  Under the bit, the time
+ * the previous kernel still runs counts against the in-kernel wait limit
+ * (palquant_set_wait_limit_ns) of the waits that depend on it.  Other bits:
+ * PQ_EINVAL. */
 #define PQ_LAYER_INPUTS_READY 1
 
 /* Human-readable name of a status. */
@@ -158,7 +164,9 @@ pq_status palquant_act_steps(const float* x_dev, int64_t N, int32_t H, int32_t W
  * library's own device memory (held by every GPU that loads the library until
  * the process exits), which bounds the group count: G <= 64, else
  * PQ_EUNSUPPORTED.  The first call on a device looks up that array's device
- * address (make it before any stream capture).  All calls share the array and
+ * address and caches it for the process (make that call before any stream
+ * capture); the cached address does not survive cudaDeviceReset, so do not call
+ * this entry point on a device after resetting it.  All calls share the array and
  * overwrite what they read, so calls that run on the GPU at the same time race
  * and must be serialised by the caller.  Results are identical to
  * palquant_act_steps for the same input.  Synchronises the stream. */

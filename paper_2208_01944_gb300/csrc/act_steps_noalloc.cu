@@ -14,7 +14,9 @@
 // code cannot pass the array's name to a kernel (on the host the name is only a
 // stand-in for the symbol, not a device address), so the first call on each
 // device looks up the device address with cudaGetSymbolAddress while that device
-// is current and caches it.  Make that first call before any stream capture.
+// is current and caches it.  Make that first call before any stream capture.  The
+// cache lives as long as the process: after cudaDeviceReset the module may load the
+// array at another address, so the entry point must not be used on a reset device.
 //
 // All calls share the array.  Each call overwrites every partial sum it reads
 // (pass 1 writes all of them before pass 2 adds them), so nothing has to start

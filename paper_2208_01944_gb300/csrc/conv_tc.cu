@@ -1110,8 +1110,6 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   uint32_t* tap_a16 = reinterpret_cast<uint32_t*>(bar_block + 8 * bars.words() + 16);  // p.taps entries
   for (int t = threadIdx.x; t < p.taps; t += blockDim.x) tap_a16[t] = p.tap_a16[t];
 
-  // let the next dependent launch on the stream start its CTAs as SMs free up
-  if (p.pdl && threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   if (threadIdx.x == 0) {
     for (int s = 0; s < bars.A; ++s) {
       // TMA, or one arrival per copy warp
@@ -1165,6 +1163,13 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   const bool third_epi = p.a_tma && !p.a_unpack && !p.a_quant;  // warps 2-5 run the epilogue too
   const bool epi_warp = warp >= kFirstEpiWarp || (third_epi && warp >= kFirstLoadWarp);
   if (p.pdl && (epi_warp || !p.pdl_early_loads)) asm volatile("griddepcontrol.wait;" ::: "memory");
+  // Let the next dependent launch on the stream start its CTAs as SMs free up, but
+  // only once this CTA's own wait has returned: a launch that depends on this one
+  // then starts only after the kernel before this one has completed, so an early
+  // loader two launches on never reads what that kernel is still writing.  The
+  // signal comes from a thread that waited (the first epilogue warp's lane 0).
+  const int first_epi_warp = third_epi ? kFirstLoadWarp : kFirstEpiWarp;
+  if (p.pdl && threadIdx.x == 32 * first_epi_warp) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
   const int64_t it0 = static_cast<int64_t>(blockIdx.x) * p.items / gridDim.x;
   const int64_t it1 = static_cast<int64_t>(blockIdx.x + 1) * p.items / gridDim.x;
   const uint32_t a_base = base;

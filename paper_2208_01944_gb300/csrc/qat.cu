@@ -65,8 +65,7 @@ __device__ __forceinline__ float qat_fwd1(float x, float l, float inv_r, const Q
 
 // Blocks: G per part of the row range, the groups fastest in launch order, so
 // the blocks that run together read whole rows (DRAM pages), not one group's
-// slice of every row.  At most 32 registers per thread: eight blocks per SM, so
-// the grid runs in as few waves as the forward's.
+// slice of every row.
 __global__ void __launch_bounds__(kQatThreads) pq_fake_quant_fwd(const float4* __restrict__ x, float4* __restrict__ y,
                                                                  int G, const __grid_constant__ QatParams q) {
   const int g = static_cast<int>(blockIdx.x % G);
@@ -106,6 +105,8 @@ struct KahanF {
 // products, four summed in fp32, the thread's quads in a compensated fp32 sum,
 // the threads in double), written to partial[g][block].  (Double arithmetic per
 // element would cost more than the memory traffic: the FP64 rate is low here.)
+// At most 32 registers per thread (12 bytes of spills): eight blocks per SM, so
+// the grid runs in as few waves as the forward's.
 __global__ void __launch_bounds__(kQatThreads, 8) pq_fake_quant_bwd(const float4* __restrict__ x,
                                                                  const float4* __restrict__ dy,
                                                                  float4* __restrict__ dx, double2* __restrict__ partial,

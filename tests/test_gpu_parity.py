@@ -589,6 +589,60 @@ def test_quantize_layer_fused_inputs_ready_overlapped(B, c, fmt):
         assert np.array_equal(got, q_ref), i
 
 
+def test_inputs_ready_chain_reads_output_two_launches_back(B):
+    """PQ_LAYER_INPUTS_READY over a chain L1 -> L2 -> L3 in which L2 reads nothing L1
+    writes but L3 reads L1's output codes.  L1 fills every SM; L2 is a few CTAs, so
+    its CTAs start while most of L1 still runs.  Each layer kernel lets its
+    dependent launch start only after its own wait for the kernel before it, so
+    L3's early loads cannot start before L1 has completed.  L3's codes equal the
+    oracle's layer over the oracle's L1 codes, three chains in a row."""
+    from layer_cases import from_format
+
+    fmt = B.PQ_CODES_C16
+    c1 = Case(16, 56, 56, 2, 32, 64, 3, 1, 1, seed=140)
+    c2 = Case(1, 8, 8, 2, 32, 64, 3, 1, 1, seed=141)
+    r1, r2 = prepare(c1), prepare(c2)
+    G, C3 = 2, 32
+    gen = synth.generator(142)
+    w3 = synth.he_weights(G, C3, 3, 3, c1.Cout, gen)
+    inv_sw3 = oracle.inv_step(oracle.weight_step(w3, 2))
+    s_a3 = np.full(G, 0.75, np.float32)
+    m_out3, m_req3 = oracle.epilogue_scales(oracle.weight_step(w3, 2), s_a3, s_a3, 1.0, 1, 1)
+    q1_ref = r1["q_ref"].reshape(c1.N, c1.Ho, c1.Wo, G * c1.Cout)
+    acc3 = oracle.group_conv(q1_ref, oracle.quantize_weights(w3, 2, inv_sw3), 1, 1).reshape(-1, G * C3)
+    _, _, q3_ref = oracle.epilogue(acc3, G, m_out3, m_req3, 1, 1, None, None, True, 2)
+
+    def desc(c, cin, cout, flags):  # 3x3, stride 1, pad 1: the output has the input's size
+        return B.layer_desc(c.N, c.H, c.W, G, cin, cout, 3, 1, 1, 2, 2, 2, 1, code_format=fmt, flags=flags)
+
+    d1 = desc(c1, c1.Cin, c1.Cout, 0)
+    d2 = desc(c2, c2.Cin, c2.Cout, B.PQ_LAYER_INPUTS_READY)
+    d3 = desc(c1, c1.Cout, C3, B.PQ_LAYER_INPUTS_READY)
+    wps = []
+    for d, w, inv in ((d1, r1["w"], r1["inv_sw"]), (d2, r2["w"], r2["inv_sw"]), (d3, w3, inv_sw3)):
+        nb = B.palquant_packed_weight_bytes(d)
+        wp = torch.empty(nb, dtype=torch.uint8, device="cuda")
+        B.palquant_pack_weights(w, d, inv, wp, nb)
+        wps.append(wp)
+    x1, x2 = torch.from_numpy(r1["x"]).cuda(), torch.from_numpy(r2["x"]).cuda()
+    shuf = B.shuffle(1, 1)
+    n1 = c1.N * c1.Ho * c1.Wo * G * c1.Cout
+    o2 = torch.empty(c2.N * c2.Ho * c2.Wo * G * c2.Cout, dtype=torch.uint8, device="cuda")
+    for rep in range(3):
+        o1 = torch.full((n1,), 255, dtype=torch.uint8, device="cuda")
+        o3 = torch.full((c1.N * c1.Ho * c1.Wo * G * C3,), 255, dtype=torch.uint8, device="cuda")
+        B.palquant_quantize_layer_fused(x1, r1["inv_s"], wps[0], d1, r1["m_out"], r1["m_req"], shuf, None, None,
+                                        None, o1)
+        B.palquant_quantize_layer_fused(x2, r2["inv_s"], wps[1], d2, r2["m_out"], r2["m_req"], shuf, None, None,
+                                        None, o2)
+        B.palquant_layer_fused(o1, wps[2], d3, m_out3, m_req3, shuf, None, None, None, o3)
+        assert B.palquant_sync_check() == B.PQ_OK
+        got1 = from_format(o1.cpu().numpy(), fmt, c1.N, c1.Ho, c1.Wo, G * c1.Cout)
+        assert np.array_equal(got1, q1_ref), rep
+        got3 = from_format(o3.cpu().numpy(), fmt, c1.N, c1.Ho, c1.Wo, G * C3).reshape(-1, G * C3)
+        assert np.array_equal(got3, q3_ref), rep
+
+
 QF_F4_CASES = [
     Case(1, 28, 28, 2, 64, 32, 3, 1, 1, seed=130),
     Case(2, 13, 11, 3, 64, 96, 3, 1, 1, seed=131),                    # odd sizes
