@@ -411,8 +411,10 @@ def measure_layer_configs(dev, args):
         plan = B.palquant_conv_plan(d).as_dict()
         out[name] = {"shape": c.name, "us": ms * 1e3, "tops": tops, "frac_fp8_peak": tops / fp8_peak,
                      "algorithmic_gbs": byt / (ms / 1e3) / 1e9, "frac_hbm": byt / (ms / 1e3) / 1e9 / pk["hbm_gbs"],
-                     "buffer_sets": n_sets, "plan": {k: plan[k] for k in ("m_tiles", "n_block", "k_chunk",
-                                                                         "weights_resident", "work_items")}}
+                     "buffer_sets": n_sets,
+                     "kernel": "pq_pointwise_tc_kernel" if plan["pointwise"] else "pq_conv_tc_kernel",
+                     "plan": ({} if plan["pointwise"] else
+                              {k: plan[k] for k in ("m_tiles", "n_block", "k_chunk", "weights_resident", "work_items")})}
         del qs, qo, q, wp
         # the same layer with packed FP4 codes (block-scaled FP4 tensor path), where it applies
         d4 = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin_g, c.Cout_g, c.k, c.stride, c.pad, c.bits_a, c.bits_w,

@@ -488,6 +488,10 @@ typedef struct {
     int32_t smem_bytes;    /* dynamic shared memory per CTA */
     int64_t tiles;         /* tiles per (group, n-block) unit */
     int64_t work_items;    /* tiles * G * n_blocks */
+    int32_t pointwise;     /* 1 if a call writing channel-blocked codes only (no int32 or
+                              fp32 outputs, no shortcut, no channel shuffle, codes in)
+                              runs on the pointwise kernel (1x1 layers); the fields above
+                              describe the general kernel */
 } pq_conv_plan;
 
 pq_status palquant_conv_plan(const pq_layer_desc* d, pq_conv_plan* plan);

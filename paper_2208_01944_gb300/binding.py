@@ -57,7 +57,8 @@ class Shuffle(ctypes.Structure):
 class ConvPlan(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "supported", "mode", "rows_per_tile", "m_tiles", "tile_pitch", "n_block", "n_blocks", "k_chunk", "k_blocks",
-        "taps", "weights_resident", "acc_stages", "smem_bytes")] + [("tiles", ctypes.c_int64), ("work_items", ctypes.c_int64)]
+        "taps", "weights_resident", "acc_stages", "smem_bytes")] + [("tiles", ctypes.c_int64), ("work_items", ctypes.c_int64),
+                                                                     ("pointwise", ctypes.c_int32)]
 
     def as_dict(self):
         return {name: getattr(self, name) for name, _ in self._fields_}

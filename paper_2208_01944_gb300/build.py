@@ -17,8 +17,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libpalquant.so")
-SOURCES = ["api.cu", "conv_tc.cu", "quantize.cu", "watchdog.cu", "act_steps_noalloc.cu", "net_f32.cu", "bitsplit.cu",
-           "qat.cu"]
+SOURCES = ["api.cu", "conv_tc.cu", "pointwise_tc.cu", "quantize.cu", "watchdog.cu", "act_steps_noalloc.cu", "net_f32.cu",
+           "bitsplit.cu", "qat.cu"]
 HEADERS = ["pq_device.cuh", "pq_internal.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-fno-strict-aliasing",

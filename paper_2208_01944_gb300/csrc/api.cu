@@ -502,6 +502,68 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   return PQ_OK;
 }
 
+// ---------------------------------------------------------------------------
+// Planner of the pointwise kernel: 1x1, stride 1, pad 0 layers with
+// channel-blocked byte codes in and codes only out.  Pure host arithmetic; false
+// when the kernel does not cover the layer (the general kernel then runs it).
+//   tiles: up to 256 pixels of one image (two 128-row accumulators) when two
+//   such tiles fit tensor memory, else up to 128; every group's weights resident
+//   in shared memory (at most 96 KB); as many stages of input codes as the rest
+//   of the shared memory holds (2 to kPwMaxStages).  The weights use the general
+//   kernel's packing with one output block per group (Cout_g <= 256).
+// ---------------------------------------------------------------------------
+bool plan_pointwise(const pq_layer_desc* d, pq::PwParams* out) {
+  if (!(d->kh == 1 && d->kw == 1 && d->stride == 1 && d->pad == 0)) return false;
+  if (d->code_format != PQ_CODES_C16) return false;
+  if (d->G < 1 || d->G > pq::kMaxG || d->Cin_g % 32 != 0 || d->Cout_g % 16 != 0 || d->Cout_g > 256) return false;
+  if (d->bits_a > 4 || d->bits_w > 4) return false;
+  const int64_t qa = (1 << d->bits_a) - 1, qw = 1 << (d->bits_w - 1);
+  if (static_cast<int64_t>(d->Cin_g) * qa * qw >= (1LL << 24)) return false;  // exact fp32 sums
+  const int64_t HW = static_cast<int64_t>(d->H) * d->W;
+  if (HW < 1 || HW > (1LL << 22)) return false;  // 32-bit plane offsets in the epilogue
+  pq::PwParams p;
+  std::memset(&p, 0, sizeof(p));
+  p.Npow2 = std::max(32, next_pow2(d->Cout_g));  // the epilogue reads 32 columns at a time
+  p.MT = (HW > 128 && 4 * p.Npow2 <= 512) ? 2 : 1;
+  p.T = static_cast<int>(std::min<int64_t>(HW, 128 * p.MT));
+  p.tiles_per_img = static_cast<int>((HW + p.T - 1) / p.T);
+  const int64_t items = static_cast<int64_t>(d->N) * p.tiles_per_img * d->G;
+  if (items >= (1LL << 31)) return false;
+  p.acc_stages = (512 / (p.MT * p.Npow2) >= 4) ? 4 : 2;
+  p.tmem_cols = static_cast<uint32_t>(std::max(32, next_pow2(p.acc_stages * p.MT * p.Npow2)));
+  p.w_bytes = static_cast<uint32_t>(d->G) * d->Cin_g * d->Cout_g;
+  if (p.w_bytes > 96u * 1024u) return false;
+  p.nch = d->Cin_g / 16;
+  if (p.nch > 256) return false;  // TMA box extent
+  p.ksteps = d->Cin_g / 32;
+  p.a_stage_bytes = static_cast<uint32_t>(p.MT) * p.nch * 2048u;
+  p.a_tx_bytes = p.a_stage_bytes;
+  const uint32_t w_round = round_up(p.w_bytes, 1024);
+  const uint32_t bar_bytes = 1024;
+  const int64_t room = static_cast<int64_t>(pq::kMaxSmem) - 1024 - w_round - bar_bytes;
+  const int stages = static_cast<int>(std::min<int64_t>(pq::kPwMaxStages, room / p.a_stage_bytes));
+  if (stages < 2) return false;
+  p.a_stages = stages;
+  p.N = d->N;
+  p.HW = static_cast<int>(HW);
+  p.G = d->G;
+  p.Cin_g = d->Cin_g;
+  p.Cout_g = d->Cout_g;
+  p.items = static_cast<int>(items);
+  p.smem_w_off = static_cast<uint32_t>(stages) * p.a_stage_bytes;
+  p.smem_bar_off = p.smem_w_off + w_round;
+  p.smem_bytes = p.smem_bar_off + bar_bytes;
+  p.C16_out = d->G * d->Cout_g / 16;
+  p.qmax2 = static_cast<uint32_t>((1 << d->bits_out) - 1) * 0x00010001u;
+  if (out) *out = p;
+  return true;
+}
+
+// Tensor map of the pointwise kernel's input codes, channel-blocked: 8-byte
+// elements, dims (2 HW, C/16, N); box (2 * 128, nch, 1), one accumulator's 128
+// positions of the group's planes.  Positions past the image are zero-filled.
+bool encode_pw_map(const pq_layer_desc* d, const pq::PwParams& p, const void* q_dev, CUtensorMap* map);
+
 bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
 
 // Learned bounds usable by the quantisers: finite, l < u, and fl(1 / fl(u - l)) finite.
@@ -615,6 +677,20 @@ bool encode_f32_map(const pq_layer_desc* d, const ConvParams& p, const void* x_d
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 4, const_cast<void*>(x_dev), dims, strides, box, es,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
              fill) == CUDA_SUCCESS;
+}
+
+bool encode_pw_map(const pq_layer_desc* d, const pq::PwParams& p, const void* q_dev, CUtensorMap* map) {
+  EncodeTiledFn enc = encode_fn();
+  if (enc == nullptr) return false;
+  std::memset(map, 0, sizeof(*map));
+  const uint64_t C16 = static_cast<uint64_t>(d->G) * d->Cin_g / 16, HW = static_cast<uint64_t>(p.HW);
+  cuuint32_t es[3] = {1, 1, 1};
+  cuuint64_t dims[3] = {2 * HW, C16, static_cast<cuuint64_t>(d->N)};
+  cuuint64_t strides[2] = {HW * 16, C16 * HW * 16};
+  cuuint32_t box[3] = {256u, static_cast<cuuint32_t>(p.nch), 1};
+  return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT64, 3, const_cast<void*>(q_dev), dims, strides, box, es,
+             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 // ---------------------------------------------------------------------------
@@ -758,6 +834,27 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
   p.q_in = static_cast<const uint8_t*>(q_dev);
   const int sms = device_sm_count();
   if (sms <= 0) return PQ_ECUDA;
+  // 1x1 layers with codes only out run on the pointwise kernel where it covers them.
+  pq::PwParams pw;
+  if (!quant_in && direct_out && q_out_dev != nullptr && shortcut_dev == nullptr && src_group == nullptr &&
+      !p.channel_shuffle && plan_pointwise(d, &pw)) {
+    for (int g = 0; g < d->G; ++g) {
+      pw.m_req15[g] = p.m_req[g] * (1.0f / 32768.0f);  // exact: m_req is 0 or above 1e-30 in magnitude
+      pw.dst_group[g] = dst[g];
+    }
+    pw.w_packed = p.w_packed;
+    pw.q_out = p.q_out;
+    pw.err = p.err;
+    pw.wait_limit_ns = p.wait_limit_ns;
+    pw.pdl = 1;
+    pw.pdl_early_loads = (d->flags & PQ_LAYER_INPUTS_READY) ? 1 : 0;
+    const int pw_grid = std::min(sms, pw.items);
+    if (pw_grid <= 0) return PQ_OK;
+    CUtensorMap pw_map;
+    if (!encode_pw_map(d, pw, q_dev, &pw_map)) return PQ_ECUDA;
+    if (pq::launch_pointwise_tc(pw, pw_map, pw_grid, static_cast<cudaStream_t>(stream)) != 0) return PQ_ECUDA;
+    return PQ_OK;
+  }
   const int grid = static_cast<int>(std::min<int64_t>(sms, p.items));
   if (grid <= 0) return PQ_OK;
   CUtensorMap map;
@@ -1207,7 +1304,9 @@ pq_status palquant_watchdog_selftest(uint64_t limit_ns, pq_stream_t stream) {
 
 pq_status palquant_conv_plan(const pq_layer_desc* d, pq_conv_plan* plan) {
   if (plan == nullptr) return PQ_EINVAL;
-  return plan_conv(d, nullptr, plan, nullptr);
+  const pq_status st = plan_conv(d, nullptr, plan, nullptr);
+  if (st == PQ_OK) plan->pointwise = plan_pointwise(d, nullptr) ? 1 : 0;
+  return st;
 }
 
 }  // extern "C"

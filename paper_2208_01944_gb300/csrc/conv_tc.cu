@@ -627,33 +627,6 @@ __device__ __forceinline__ int epi_pos(const ConvParams& p, const EpiItem& e, in
   return oh * p.Wo + c;
 }
 
-// Codes-only unit (the timed path): the codes clamp(rint(t), 0, Qp) of
-// t = acc * m_req = raw * (m_req * 2^9), Qp = 2^b - 1, as
-//   c = sat(raw * m_sat), m_sat = m_req * 2^9 / 2^b (a power-of-two scaling, so
-//       c = clamp(t, 0, 2^b) / 2^b exactly; NaN -> 0);
-//   r = c * 2^b + 1.5 * 2^23, one rounding half to even: the low 16 bits of r
-//       hold k = rint(clamp(t, 0, 2^b)), in [0, 2^b];
-//   code = min(k, Qp), two 16-bit halves per instruction.
-// Clamping to [0, 2^b] before rounding and to Qp after it equals clamping the
-// rounded value to [0, Qp] (integer bounds, monotone rounding).
-__device__ __forceinline__ uint4 epi_codes16(const uint32_t (&v)[16], float m_sat, float two_b, uint32_t qmax2) {
-  uint32_t h[8];
-#pragma unroll
-  for (int j = 0; j < 16; j += 2) {
-    const float c0 = mul_sat(__uint_as_float(v[j]), m_sat);
-    const float c1 = mul_sat(__uint_as_float(v[j + 1]), m_sat);
-    float r0, r1;
-    fma2_rn(c0, c1, two_b, 12582912.0f, r0, r1);
-    h[j >> 1] = __vimin_s16x2_relu(__byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x5410), qmax2);
-  }
-  uint4 w;
-  w.x = __byte_perm(h[0], h[1], 0x6420);
-  w.y = __byte_perm(h[2], h[3], 0x6420);
-  w.z = __byte_perm(h[4], h[5], 0x6420);
-  w.w = __byte_perm(h[6], h[7], 0x6420);
-  return w;
-}
-
 // Quantise-on-load with learned bounds: the codes rint(sat((x - l) * inv_r) * Qp)
 // of 16 fp32 values, one rounding per operation (x - l as x + (-l), exact), the
 // rounding to an integer by the fp32 add of 1.5 * 2^23 (its low 16 bits); sat

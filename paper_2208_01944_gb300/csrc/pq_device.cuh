@@ -194,6 +194,71 @@ __device__ __forceinline__ void fma2_rn(float a, float b, float m, float c, floa
       : "f"(a), "f"(b), "f"(m), "f"(c));
 }
 
+// Codes-only unit (the timed path): the codes clamp(rint(t), 0, Qp) of
+// t = acc * m_req = raw * (m_req * 2^9), Qp = 2^b - 1, as
+//   c = sat(raw * m_sat), m_sat = m_req * 2^9 / 2^b (a power-of-two scaling, so
+//       c = clamp(t, 0, 2^b) / 2^b exactly; NaN -> 0);
+//   r = c * 2^b + 1.5 * 2^23, one rounding half to even: the low 16 bits of r
+//       hold k = rint(clamp(t, 0, 2^b)), in [0, 2^b];
+//   code = min(k, Qp), two 16-bit halves per instruction.
+// Clamping to [0, 2^b] before rounding and to Qp after it equals clamping the
+// rounded value to [0, Qp] (integer bounds, monotone rounding).
+// (v: 16 accumulator columns, or 16 of a larger array starting at OFF.)
+template <int NV = 16, int OFF = 0>
+__device__ __forceinline__ uint4 epi_codes16(const uint32_t (&v)[NV], float m_sat, float two_b, uint32_t qmax2) {
+  static_assert(OFF + 16 <= NV, "16 columns of the array");
+  uint32_t h[8];
+#pragma unroll
+  for (int j = 0; j < 16; j += 2) {
+    const float c0 = mul_sat(__uint_as_float(v[OFF + j]), m_sat);
+    const float c1 = mul_sat(__uint_as_float(v[OFF + j + 1]), m_sat);
+    float r0, r1;
+    fma2_rn(c0, c1, two_b, 12582912.0f, r0, r1);
+    h[j >> 1] = __vimin_s16x2_relu(__byte_perm(__float_as_uint(r0), __float_as_uint(r1), 0x5410), qmax2);
+  }
+  uint4 w;
+  w.x = __byte_perm(h[0], h[1], 0x6420);
+  w.y = __byte_perm(h[2], h[3], 0x6420);
+  w.z = __byte_perm(h[4], h[5], 0x6420);
+  w.w = __byte_perm(h[6], h[7], 0x6420);
+  return w;
+}
+
+// Requantised codes of 16 accumulator columns through the fp16 conversion, for
+// output codes of at most 8 bits:
+//   y = fl(raw * m_req 2^-15) with raw = acc * 2^-9, so y = fl(acc * m_req) * 2^-24
+//       = t * 2^-24 exactly (power-of-two scalings commute with rounding; where y
+//       would be an fp32 subnormal, |t| < 2^-102 and the code is 0 either way);
+//   the fp16 conversion with .relu rounds y half to even onto the fp16 grid,
+//       which below 2^-14 is the integers times 2^-24 (the subnormals), so the
+//       16-bit pattern is rint(t) for t in [0, 1024], any larger t gives a larger
+//       pattern (the positive encodings are ordered, up to +inf), and negative t
+//       gives +0;
+//   code = min(pattern, Qp) on both 16-bit halves in one instruction.
+// This equals clamp(rint(t), 0, Qp): integer bounds, monotone rounding.  Per
+// pair of values: one packed multiply, one packed conversion, one packed min,
+// against two multiplies, a packed multiply-add and two integer steps in
+// epi_codes16.  m_req15 = m_req * 2^-15 (the caller's exact scaling).
+__device__ __forceinline__ uint32_t cvt_f16x2_relu(float hi, float lo) {
+  uint32_t r;
+  asm("cvt.rn.relu.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+template <int NV = 16, int OFF = 0>
+__device__ __forceinline__ uint4 epi_codes16_f16(const uint32_t (&v)[NV], float m_req15, uint32_t qmax2) {
+  static_assert(OFF + 16 <= NV, "16 columns of the array");
+  uint32_t h[8];
+#pragma unroll
+  for (int q = 0; q < 8; ++q) {
+    float y0, y1;
+    mul2_rn(__uint_as_float(v[OFF + 2 * q]), __uint_as_float(v[OFF + 2 * q + 1]), m_req15, y0, y1);
+    h[q] = __vimin_s16x2_relu(cvt_f16x2_relu(y1, y0), qmax2);
+  }
+  return make_uint4(__byte_perm(h[0], h[1], 0x6420), __byte_perm(h[2], h[3], 0x6420), __byte_perm(h[4], h[5], 0x6420),
+                    __byte_perm(h[6], h[7], 0x6420));
+}
+
 // ------------------------------------------------------------- packed codes
 // Sixteen 2-bit codes (one per byte of w, each <= 3) packed into one 32-bit word,
 // code k at bits 2k: the product of a byte quadruple with 2^24 + 2^18 + 2^12 + 2^6
@@ -405,6 +470,19 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
       "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
       : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
         "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr)
+      : "memory");
+}
+
+// Each lane of the warp reads 32 consecutive 32-bit columns of its own TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+        "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]), "=r"(r[16]),
+        "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]),
+        "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
       : "r"(taddr)
       : "memory");
 }

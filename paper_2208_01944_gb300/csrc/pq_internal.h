@@ -140,8 +140,42 @@ struct ConvParams {
   uint64_t wait_limit_ns;
 };
 
+// The pointwise kernel (1x1, stride 1, pad 0 layers, channel-blocked codes in
+// and codes only out); filled by the host planner.  A work item is (image,
+// pixel tile, group), the group fastest.
+constexpr int kPwEpiGroups = 4;                             // epilogue warpgroups, taking accumulators in turn
+constexpr int kPwFirstEpiWarp = 2;                          // warp 0 loads, warp 1 issues the MMAs
+constexpr int kPwThreads = 32 * (kPwFirstEpiWarp + 4 * kPwEpiGroups);
+constexpr int kPwMaxStages = 8;
+
+struct PwParams {
+  int N, HW, G, Cin_g, Cout_g;
+  int T;                  // pixels per tile (at most 256; the last tile of an image may be shorter)
+  int MT;                 // 128-row accumulators per tile (1 or 2)
+  int tiles_per_img;
+  int items;              // N * tiles_per_img * G
+  int nch;                // Cin_g / 16: 16-channel planes of an item's input
+  int ksteps;             // Cin_g / 32: MMAs per accumulator
+  int Npow2;              // tensor-memory columns per accumulator
+  int a_stages, acc_stages;
+  uint32_t a_stage_bytes; // MT * nch * 2048: per accumulator one TMA box of nch planes x 128 positions
+  uint32_t a_tx_bytes;    // bytes a stage receives (whole boxes, out-of-image rows zero-filled)
+  uint32_t w_bytes;       // every group's packed weights, G * Cout_g * Cin_g
+  uint32_t smem_w_off, smem_bar_off, smem_bytes, tmem_cols;
+  int C16_out;            // 16-channel planes of an output image: G * Cout_g / 16
+  uint32_t qmax2;         // Qp_out in both 16-bit halves
+  float m_req15[kMaxG];   // m_req * 2^-15, applied to the raw accumulator acc * 2^-9 (fl(acc m_req) * 2^-24)
+  int dst_group[kMaxG];
+  const uint8_t* w_packed;
+  uint8_t* q_out;
+  unsigned int* err;
+  uint64_t wait_limit_ns;
+  int pdl, pdl_early_loads;
+};
+
 // Host-side launch helpers implemented in the .cu files.
 int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream);
+int launch_pointwise_tc(const PwParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream);
 int launch_bitsplit_act(const uint8_t* q, uint8_t* xs, int64_t N, int64_t HW, int C, int Ga, int Gw, int B, int c16,
                         cudaStream_t stream);
 // pack: 0 one code per byte [N][C/16][HW][16]; 1 four 2-bit codes per byte

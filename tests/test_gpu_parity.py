@@ -230,6 +230,106 @@ def test_full_size_codes_only_c16_sampled(B, name, cfg):
     assert_layer_parity(c, ref, got, pix)
 
 
+# ------------------------------- the pointwise kernel (1x1 layers, codes only out)
+PW_CASES = [
+    Case(2, 7, 7, 4, 32, 16, 1, seed=150),                            # 49 pixels: one accumulator, ragged
+    Case(3, 14, 14, 4, 96, 96, 1, seed=151),                          # the config-4 shape: 196 of 256 rows
+    Case(2, 20, 20, 2, 64, 64, 1, seed=152),                          # 400 pixels: tiles of 256 and 144
+    Case(1, 16, 16, 1, 32, 256, 1, kind=0, seed=153),                 # N = 256: tiles of 128 pixels
+    Case(2, 9, 13, 8, 32, 48, 1, kind=3, perm=(3, 0, 7, 1, 6, 2, 5, 4), seed=154),  # odd plane count
+    Case(2, 12, 12, 2, 64, 32, 1, bits=4, bits_out=3, relu=False, shift=-1, seed=155),
+    Case(1, 1, 1, 2, 32, 16, 1, seed=156),                            # one pixel
+    Case(4, 8, 8, 1, 256, 64, 1, kind=0, seed=157),                   # eight K steps
+    Case(1, 30, 30, 3, 32, 32, 1, seed=158),                          # 900 pixels, three groups
+    Case(5, 11, 23, 2, 128, 16, 1, bits_out=1, seed=159),             # N = 16: four accumulator stages, 1-bit codes out
+]
+
+
+@pytest.mark.parametrize("c", PW_CASES, ids=str)
+def test_pointwise_kernel_matches_oracle(B, c):
+    """1x1 layers with channel-blocked codes in and codes only out run on the
+    pointwise kernel; its codes equal the oracle's bit for bit."""
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, 1, 1, 0, c.bits, c.bits, c.bo, int(c.relu),
+                     code_format=B.PQ_CODES_C16)
+    assert B.palquant_conv_plan(d).pointwise == 1
+    ref = prepare(c)
+    assert_layer_parity(c, ref, run_gpu(c, ref, outputs=("q",), fmt=2))
+
+
+def test_pointwise_not_taken_when_weights_do_not_fit(B):
+    """Weights beyond the pointwise kernel's resident budget (96 KB) go to the
+    general kernel, with the same results."""
+    c = Case(1, 9, 9, 4, 128, 256, 1, seed=160)                      # 4 x 128 x 256 = 128 KB of weights
+    d = B.layer_desc(c.N, c.H, c.W, c.G, c.Cin, c.Cout, 1, 1, 0, c.bits, c.bits, c.bo, int(c.relu),
+                     code_format=B.PQ_CODES_C16)
+    assert B.palquant_conv_plan(d).pointwise == 0
+    ref = prepare(c)
+    assert_layer_parity(c, ref, run_gpu(c, ref, outputs=("q",), fmt=2))
+
+
+def test_pointwise_inputs_ready_chain(B):
+    """PQ_LAYER_INPUTS_READY over a chain of pointwise layers L1 -> L2 -> L3: L2
+    reads nothing L1 writes, L3 reads L1's codes.  L1 fills every SM, L2 is a few
+    CTAs.  L3's codes equal the oracle's layer over the oracle's L1 codes, and
+    back-to-back flagged launches over independent inputs equal flagless ones."""
+    from layer_cases import from_format, to_format
+
+    fmt = B.PQ_CODES_C16
+    G = 4
+    c1 = Case(64, 14, 14, G, 96, 96, 1, seed=161)
+    c2 = Case(1, 4, 4, G, 96, 96, 1, seed=162)
+    r1, r2 = prepare(c1), prepare(c2)
+    gen = synth.generator(163)
+    w3 = synth.he_weights(G, 32, 1, 1, c1.Cout, gen)
+    s_w3 = oracle.weight_step(w3, 2)
+    inv_sw3 = oracle.inv_step(s_w3)
+    s_a3 = np.full(G, 0.75, np.float32)
+    m_out3, m_req3 = oracle.epilogue_scales(s_w3, s_a3, s_a3, 1.0, 1, 1)
+    q1_ref = r1["q_ref"].reshape(c1.N, c1.H, c1.W, G * c1.Cout)
+    acc3 = oracle.group_conv(q1_ref, oracle.quantize_weights(w3, 2, inv_sw3), 1, 0).reshape(-1, G * 32)
+    _, _, q3_ref = oracle.epilogue(acc3, G, m_out3, m_req3, 1, 1, None, None, True, 2)
+
+    def desc(c, cin, cout, flags):
+        return B.layer_desc(c.N, c.H, c.W, G, cin, cout, 1, 1, 0, 2, 2, 2, 1, code_format=fmt, flags=flags)
+
+    d1 = desc(c1, 96, 96, 0)
+    d2 = desc(c2, 96, 96, B.PQ_LAYER_INPUTS_READY)
+    d3 = desc(c1, 96, 32, B.PQ_LAYER_INPUTS_READY)
+    assert all(B.palquant_conv_plan(d).pointwise == 1 for d in (d1, d2, d3))
+    wps = []
+    for d, w, inv in ((d1, r1["w"], r1["inv_sw"]), (d2, r2["w"], r2["inv_sw"]), (d3, w3, inv_sw3)):
+        nb = B.palquant_packed_weight_bytes(d)
+        wp = torch.empty(nb, dtype=torch.uint8, device="cuda")
+        B.palquant_pack_weights(w, d, inv, wp, nb)
+        wps.append(wp)
+    q1 = torch.from_numpy(to_format(r1["q"], fmt)).cuda()
+    q2 = torch.from_numpy(to_format(r2["q"], fmt)).cuda()
+    shuf = B.shuffle(1, 1)
+    o2 = torch.empty(c2.N * c2.H * c2.W * G * 96, dtype=torch.uint8, device="cuda")
+    for rep in range(3):
+        o1 = torch.full((c1.N * c1.H * c1.W * G * 96,), 255, dtype=torch.uint8, device="cuda")
+        o3 = torch.full((c1.N * c1.H * c1.W * G * 32,), 255, dtype=torch.uint8, device="cuda")
+        B.palquant_layer_fused(q1, wps[0], d1, r1["m_out"], r1["m_req"], shuf, None, None, None, o1)
+        B.palquant_layer_fused(q2, wps[1], d2, r2["m_out"], r2["m_req"], shuf, None, None, None, o2)
+        B.palquant_layer_fused(o1, wps[2], d3, m_out3, m_req3, shuf, None, None, None, o3)
+        assert B.palquant_sync_check() == B.PQ_OK
+        assert np.array_equal(from_format(o1.cpu().numpy(), fmt, c1.N, c1.H, c1.W, G * 96), q1_ref), rep
+        got3 = from_format(o3.cpu().numpy(), fmt, c1.N, c1.H, c1.W, G * 32).reshape(-1, G * 32)
+        assert np.array_equal(got3, q3_ref), rep
+    # back to back over independent inputs (five launches, two output buffers in turn)
+    d1r = desc(c1, 96, 96, B.PQ_LAYER_INPUTS_READY)
+    outs = [torch.full((c1.N * c1.H * c1.W * G * 96,), 255, dtype=torch.uint8, device="cuda") for _ in range(2)]
+    qs = [q1, torch.flip(q1, dims=[0]).contiguous()]
+    for i in range(5):
+        B.palquant_layer_fused(qs[i % 2], wps[0], d1r, r1["m_out"], r1["m_req"], shuf, None, None, None, outs[i % 2])
+    assert B.palquant_sync_check() == B.PQ_OK
+    for i in (3, 4):
+        single = torch.full_like(outs[0], 255)
+        B.palquant_layer_fused(qs[i % 2], wps[0], d1, r1["m_out"], r1["m_req"], shuf, None, None, None, single)
+        assert B.palquant_sync_check() == B.PQ_OK
+        assert torch.equal(outs[i % 2], single), i
+
+
 # ------------------------------------------------------ failure detection
 def test_watchdog_times_out_and_context_survives(B):
     assert B.palquant_watchdog_selftest(2_000_000) == B.PQ_ETIMEOUT  # a 2 ms wait nobody completes
@@ -257,13 +357,15 @@ def test_layer_codes_only_matches_oracle(B, c, fmt):
     assert_layer_parity(c, ref, got)
 
 
+@pytest.mark.parametrize("k", [3, 1], ids=["3x3", "1x1"])
 @pytest.mark.parametrize("fmt,bits", [(0, 4), (2, 4), (2, 1), (4, 2)], ids=["nhwc4", "c16_4", "c16_1", "fp4_2"])
 @pytest.mark.parametrize("mult", [0.5, 0.25, 1.0 / 3.0, 1e4, -0.5, 1e-3])
-def test_requant_ties_round_half_even(B, mult, fmt, bits):
+def test_requant_ties_round_half_even(B, mult, fmt, bits, k):
     """Multipliers that put many products exactly on .5 (ties must round to even),
     that saturate every positive sum, that make every product negative, and that
-    round almost everything to 0; codes only, in every code format."""
-    c = Case(2, 10, 10, 2, 64, 64, 3, 1, 1, bits=bits if bits > 1 else 2, bits_out=bits, seed=44)
+    round almost everything to 0; codes only, in every code format (1x1 layers
+    with channel-blocked byte codes run on the pointwise kernel)."""
+    c = Case(2, 10, 10, 2, 64, 64, k, 1, (k - 1) // 2, bits=bits if bits > 1 else 2, bits_out=bits, seed=44)
     ref = prepare(c)
     m_req = np.array([mult, mult * 0.75], dtype=np.float32)
     acc = oracle.group_conv(ref["q"], ref["wq"], c.stride, c.pad).reshape(-1, c.G * c.Cout)
