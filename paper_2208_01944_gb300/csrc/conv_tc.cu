@@ -607,7 +607,7 @@ __device__ __forceinline__ int requant_code(float t, float qmax_f, int qmax) {
 struct EpiItem {
   uint32_t tbase;        // TMEM address of accumulator 0, this warp's lanes
   float m_out512, m_req512, m_req;
-  float m_sat;           // m_req512 / 2^b_out (codes-only conversion)
+  float m_req15;         // m_req * 2^-15 (codes-only conversion through fp16, see epi_codes16_f16)
   int g, src_c0, dst_c0;
   int n, rb, oh0;
   int nb;
@@ -900,15 +900,12 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
   Ring racc{0, 0, static_cast<uint32_t>(p.acc_stages)};
   const int nchunks = p.Nblk >> 4;
   const int n_units = p.MT * nchunks;
-  const float qmax_f = static_cast<float>(p.qmax_out);
   const bool codes_only = p.shortcut == nullptr && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle;
   // The group's multipliers and destination stay in registers while consecutive
   // items share the group (items run group by group); a dynamically indexed
   // kernel-parameter array costs a long-latency constant load.
   int cur_g = -1, dst_g = 0;
-  float g_m_out512 = 0.0f, g_m_req512 = 0.0f, g_m_req = 0.0f, g_m_sat = 0.0f;
-  const float two_b = static_cast<float>(p.qmax_out + 1);  // 2^b_out
-  const float inv_two_b = 1.0f / two_b;                     // exact: a power of two
+  float g_m_out512 = 0.0f, g_m_req512 = 0.0f, g_m_req = 0.0f, g_m_req15 = 0.0f;
   const uint32_t qmax2 = static_cast<uint32_t>(p.qmax_out) * 0x00010001u;
   Item item = item_begin(p, it0);
   for (int64_t it = it0; it < it1; ++it, item_next(p, item)) {
@@ -917,7 +914,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
       g_m_out512 = p.m_out512[cur_g];
       g_m_req512 = p.m_req512[cur_g];
       g_m_req = p.m_req[cur_g];
-      g_m_sat = __fmul_rn(g_m_req512, inv_two_b);
+      g_m_req15 = __fmul_rn(g_m_req, 1.0f / 32768.0f);  // exact: |m_req| is 0 or above 1e-30
       dst_g = p.dst_group[cur_g];
     }
     if (!warp_wait(bars.acc_full(racc.stage), racc.phase, ctx)) break;
@@ -931,7 +928,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
     e.m_out512 = g_m_out512;
     e.m_req512 = g_m_req512;
     e.m_req = g_m_req;
-    e.m_sat = g_m_sat;
+    e.m_req15 = g_m_req15;
     e.src_c0 = e.g * p.Cout_g + item.nb * p.Nblk;     // source channel of column 0
     e.dst_c0 = dst_g * p.Cout_g + item.nb * p.Nblk;  // destination channel of column 0
     e.tbase = tmem_base + (static_cast<uint32_t>(quarter * 32) << 16) + racc.stage * p.MT * p.Npow2;
@@ -972,12 +969,12 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
       }
       while (c_mt < MT) {
         tmem_ld16(col(c_mt, c_b) + 16, vb);
-        const uint2 lo = pack4_word(epi_codes16(va, e.m_sat, two_b, qmax2));
+        const uint2 lo = pack4_word(epi_codes16_f16(va, e.m_req15, qmax2));
         tmem_wait_ld();
         int n_mt = c_mt, n_b = c_b;
         step(n_mt, n_b);
         if (n_mt < MT) tmem_ld16(col(n_mt, n_b), va);
-        const uint2 hi = pack4_word(epi_codes16(vb, e.m_sat, two_b, qmax2));
+        const uint2 hi = pack4_word(epi_codes16_f16(vb, e.m_req15, qmax2));
         tmem_wait_ld();  // before the store: a TMEM-load wait right after a store stalls on the store
         if (c_row) *reinterpret_cast<uint4*>(c_row + c_b * blk_bytes) = make_uint4(lo.x, lo.y, hi.x, hi.y);
         c_row = n_mt == c_mt ? c_row : row_ptr(n_mt);
@@ -1034,8 +1031,8 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         uint8_t* c_row = row_ptr(c_mt);
         uint8_t* n_row = two ? (n_mt == c_mt ? c_row : row_ptr(n_mt)) : nullptr;
         tmem_wait_ld();
-        const uint4 w0 = epi_codes16(va, e.m_sat, two_b, qmax2);
-        const uint4 w1 = epi_codes16(vb, e.m_sat, two_b, qmax2);
+        const uint4 w0 = epi_codes16_f16(va, e.m_req15, qmax2);
+        const uint4 w1 = epi_codes16_f16(vb, e.m_req15, qmax2);
         if (c_row) store_codes16(c_row + coff(c_ch), w0, pack);
         if (n_row) store_codes16(n_row + coff(n_ch), w1, pack);
         if (!two) break;
