@@ -558,7 +558,8 @@ def measure_bitsplit_vs_palquant(dev, stream, timed, pk, fp8_peak):
         "palquant_2bit_G2_us": ms_pal * 1e3,
         "speedup_palquant_vs_bit_decomposed": ms_split / ms_pal,
         "int_ops": {"direct_4bit": ops4, "bit_decomposed_2bit_products": 4 * ops4, "palquant_G2": 2 * ops4},
-        "note": "the 4 products of Eq. 4 form one tensor-core pass (K = 4C) after a slice kernel",
+        "note": "the 4 products of Eq. 4 form one tensor-core pass after a slice kernel that writes each "
+                "activation slice once (K = 2C slice channels, each meeting its 2 weight slices as taps)",
     })
     return res
 

@@ -112,6 +112,12 @@ typedef struct {
     int32_t relu;        /* 1: ReLU after the rescale (and the shortcut add) */
     int32_t code_format; /* pq_code_format of the input codes and the output codes */
     int32_t flags;       /* PQ_LAYER_* bits; 0 for none */
+    int32_t wslices;     /* weight slices per input channel and tap: 0 or 1 for a plain
+                            layer.  R > 1 (set by palquant_bitsplit_desc, 2..8) makes
+                            every input code meet R weight codes, the sum running over
+                            them: acc = sum_{tap, r, ci} q[...] w[g, co, tap, r, ci],
+                            weights [G][Cout_g][kh][kw][R][Cin_g] (Eq. 4's G^2 products
+                            with each activation slice stored once) */
 } pq_layer_desc;
 
 /* pq_layer_desc.flags bit: the kernel launched on the stream immediately before this
@@ -361,12 +367,13 @@ pq_status palquant_watchdog_selftest(uint64_t limit_ns, pq_stream_t stream);
 /* whose M-bit sums could reach 2^24 return PQ_EUNSUPPORTED.                   */
 /* ------------------------------------------------------------------------ */
 
-/* The decomposed layer's descriptor: Cin_g multiplied by Ga Gw, bits_a = B,
- * PQ_LAYER_INPUTS_READY cleared (the decomposed layer reads the slices that the
- * kernel launched just before it writes). */
+/* The decomposed layer's descriptor: Cin_g multiplied by Ga (the activation
+ * slices, each stored once), wslices = Gw (every slice meets the Gw shifted
+ * weight slices), bits_a = B, PQ_LAYER_INPUTS_READY cleared (the decomposed layer
+ * reads the slices that the kernel launched just before it writes). */
 pq_status palquant_bitsplit_desc(const pq_layer_desc* d, int32_t bits_b, pq_layer_desc* out);
 
-/* Bytes of the slice buffer (N H W Ga Gw Cin_g); 0 if unsupported. */
+/* Bytes of the slice buffer (N H W Ga Cin_g); 0 if unsupported. */
 size_t palquant_bitsplit_scratch_bytes(const pq_layer_desc* d, int32_t bits_b);
 
 /* Pack the decomposed weights from the M-bit signed codes wq_host

@@ -47,7 +47,7 @@ class PalquantError(RuntimeError):
 class LayerDesc(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int32) for n in (
         "N", "H", "W", "G", "Cin_g", "Cout_g", "kh", "kw", "stride", "pad", "bits_a", "bits_w", "bits_out", "relu",
-        "code_format", "flags")]
+        "code_format", "flags", "wslices")]
 
 
 class Shuffle(ctypes.Structure):
@@ -194,7 +194,7 @@ def strerror(status: int) -> str:
 def layer_desc(N, H, W, G, Cin_g, Cout_g, k, stride=1, pad=0, bits_a=2, bits_w=2, bits_out=2, relu=1,
                code_format=PQ_CODES_INT8, kw=None, flags=0) -> LayerDesc:
     return LayerDesc(N, H, W, G, Cin_g, Cout_g, k, k if kw is None else kw, stride, pad, bits_a, bits_w, bits_out,
-                     int(relu), code_format, int(flags))
+                     int(relu), code_format, int(flags), 0)
 
 
 def shuffle(kind=1, shift=1, perm=None):
@@ -277,7 +277,10 @@ def palquant_pack_weight_codes_host(wq_host, d: LayerDesc) -> np.ndarray:
 
 
 def palquant_unpack_weight_codes_host(packed_host, d: LayerDesc) -> np.ndarray:
-    out = np.empty((d.G, d.Cout_g, d.kh, d.kw, d.Cin_g), dtype=np.int8)
+    """[G][Cout_g][kh][kw][Cin_g], or [G][Cout_g][kh][kw][R][Cin_g] with R = d.wslices > 1 weight slices."""
+    R = d.wslices if d.wslices > 1 else 1
+    shape = (d.G, d.Cout_g, d.kh, d.kw, d.Cin_g) if R == 1 else (d.G, d.Cout_g, d.kh, d.kw, R, d.Cin_g)
+    out = np.empty(shape, dtype=np.int8)
     pk = np.ascontiguousarray(packed_host, dtype=np.uint8)
     _check(lib.palquant_unpack_weight_codes_host(_ptr(pk), ctypes.byref(d), _ptr(out)), "palquant_unpack_weight_codes_host")
     return out

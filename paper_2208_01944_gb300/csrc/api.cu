@@ -88,6 +88,7 @@ pq_status validate_desc(const pq_layer_desc* d) {
     return PQ_EINVAL;
   if (d->relu != 0 && d->relu != 1) return PQ_EINVAL;
   if ((d->flags & ~PQ_LAYER_INPUTS_READY) != 0) return PQ_EINVAL;
+  if (d->wslices < 0 || d->wslices > 8) return PQ_EINVAL;
   if (d->code_format != PQ_CODES_INT8 && d->code_format != PQ_CODES_E4M3 && d->code_format != PQ_CODES_C16 &&
       d->code_format != PQ_CODES_C16P2 && d->code_format != PQ_CODES_C32F4)
     return PQ_EINVAL;
@@ -95,6 +96,12 @@ pq_status validate_desc(const pq_layer_desc* d) {
   if (d->G > pq::kMaxG) return PQ_EUNSUPPORTED;
   return PQ_OK;
 }
+
+// Weight slices per input channel and tap (pq_layer_desc.wslices; 0 means 1).
+int wslices_of(const pq_layer_desc* d) { return d->wslices > 1 ? d->wslices : 1; }
+
+// Taps of the weight operand: kh kw positions, each with R weight slices.
+int weight_taps(const pq_layer_desc* d) { return d->kh * d->kw * wslices_of(d); }
 
 int device_sm_count() {
   int dev = 0, sms = 0;
@@ -125,7 +132,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   std::memset(&p, 0, sizeof(p));
   const int Ho = static_cast<int>(out_dim(d->H, d->kh, d->stride, d->pad));
   const int Wo = static_cast<int>(out_dim(d->W, d->kw, d->stride, d->pad));
-  const int taps = d->kh * d->kw;
+  // R weight slices per kernel position: R consecutive taps with the same
+  // activation offset (the operand's tap t = position * R + slice)
+  const int R = wslices_of(d);
+  const int taps = d->kh * d->kw * R;
   const int qa = (1 << d->bits_a) - 1;
   const int qw = 1 << (d->bits_w - 1);
   // Coverage of the tensor-core kernel.
@@ -191,16 +201,20 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
           phases.push_back({a, b});
           idx = static_cast<int>(phases.size()) - 1;
         }
-        const int t = i * d->kw + j;
-        p.tap_phase[t] = idx;
-        p.tap_off[t] = (floor_div(i - d->pad, s) - rmin) * Wh + (floor_div(j - d->pad, s) - cmin);
-        off_max = std::max(off_max, p.tap_off[t]);
+        for (int r = 0; r < R; ++r) {
+          const int t = (i * d->kw + j) * R + r;
+          p.tap_phase[t] = idx;
+          p.tap_off[t] = (floor_div(i - d->pad, s) - rmin) * Wh + (floor_div(j - d->pad, s) - cmin);
+          off_max = std::max(off_max, p.tap_off[t]);
+        }
       }
     }
   } else {
     phases.push_back({0, 0});
-    p.tap_phase[0] = 0;
-    p.tap_off[0] = 0;
+    for (int r = 0; r < R; ++r) {
+      p.tap_phase[r] = 0;
+      p.tap_off[r] = 0;
+    }
   }
   p.nph = static_cast<int>(phases.size());
   // Tile shape: MT accumulators of 128 rows; rows mode packs Ht whole output
@@ -513,7 +527,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
 //   kernel's packing with one output block per group (Cout_g <= 256).
 // ---------------------------------------------------------------------------
 bool plan_pointwise(const pq_layer_desc* d, pq::PwParams* out) {
-  if (!(d->kh == 1 && d->kw == 1 && d->stride == 1 && d->pad == 0)) return false;
+  if (!(d->kh == 1 && d->kw == 1 && d->stride == 1 && d->pad == 0) || wslices_of(d) != 1) return false;
   if (d->code_format != PQ_CODES_C16) return false;
   if (d->G < 1 || d->G > pq::kMaxG || d->Cin_g % 32 != 0 || d->Cout_g % 16 != 0 || d->Cout_g > 256) return false;
   if (d->bits_a > 4 || d->bits_w > 4) return false;
@@ -743,19 +757,21 @@ int int_of_e2m1(uint8_t b) {
 
 // Bytes of the packed weight operand: one per code, or one per two (FP4).
 size_t packed_weight_bytes_of(const pq_layer_desc* d, const ConvParams& p) {
-  const size_t elems = static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
+  const size_t elems = static_cast<size_t>(d->G) * d->Cout_g * weight_taps(d) * d->Cin_g;
   return p.codes_f4 ? elems / 2 : elems;
 }
 
-// Write the signed codes wq [G][Cout_g][kh][kw][Cin_g] in the operand layout.
+// Write the signed codes wq [G][Cout_g][kh][kw][R][Cin_g] in the operand layout
+// (a tap of the operand is a kernel position and weight slice: kw R per row).
 void pack_codes(const ConvParams& p, const pq_layer_desc* d, const int8_t* wq, uint8_t* out) {
+  const int kwr = d->kw * wslices_of(d);
   if (p.codes_f4) {
     std::memset(out, 0, packed_weight_bytes_of(d, p));
-    for_each_packed(p, d->kw, [&](size_t dst, size_t src) {
+    for_each_packed(p, kwr, [&](size_t dst, size_t src) {
       out[dst >> 1] = static_cast<uint8_t>(out[dst >> 1] | (e2m1_of_int(wq[src]) << (4 * (dst & 1))));
     });
   } else {
-    for_each_packed(p, d->kw, [&](size_t dst, size_t src) { out[dst] = e4m3_of_int(wq[src]); });
+    for_each_packed(p, kwr, [&](size_t dst, size_t src) { out[dst] = e4m3_of_int(wq[src]); });
   }
 }
 
@@ -923,6 +939,7 @@ pq_status palquant_weight_steps(const float* w_host, const pq_layer_desc* d, flo
   if (w_host == nullptr || s_w_out_host == nullptr) return PQ_EINVAL;
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
+  if (wslices_of(d) != 1) return PQ_EINVAL;  // float weights belong to plain layers
   const int64_t per_group = static_cast<int64_t>(d->Cout_g) * d->kh * d->kw * d->Cin_g;
   const double qp = static_cast<double>((1 << (d->bits_w - 1)) - 1);
   for (int g = 0; g < d->G; ++g) {
@@ -959,7 +976,7 @@ pq_status palquant_pack_weight_codes_host(const int8_t* wq_host, const pq_layer_
   ConvParams p;
   pq_status st = plan_conv(d, &p, nullptr, nullptr);
   if (st != PQ_OK) return st;
-  const size_t elems = static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
+  const size_t elems = static_cast<size_t>(d->G) * d->Cout_g * weight_taps(d) * d->Cin_g;
   if (packed_bytes < packed_weight_bytes_of(d, p)) return PQ_EINVAL;
   const int lo = -(1 << (d->bits_w - 1)), hi = (1 << (d->bits_w - 1)) - 1;
   for (size_t i = 0; i < elems; ++i)
@@ -974,12 +991,13 @@ pq_status palquant_unpack_weight_codes_host(const void* packed_host, const pq_la
   pq_status st = plan_conv(d, &p, nullptr, nullptr);
   if (st != PQ_OK) return st;
   const uint8_t* in = static_cast<const uint8_t*>(packed_host);
+  const int kwr = d->kw * wslices_of(d);
   if (p.codes_f4)
-    for_each_packed(p, d->kw, [&](size_t dst, size_t src) {
+    for_each_packed(p, kwr, [&](size_t dst, size_t src) {
       wq_host[src] = static_cast<int8_t>(int_of_e2m1(static_cast<uint8_t>(in[dst >> 1] >> (4 * (dst & 1)))));
     });
   else
-    for_each_packed(p, d->kw, [&](size_t dst, size_t src) { wq_host[src] = static_cast<int8_t>(int_of_e4m3(in[dst])); });
+    for_each_packed(p, kwr, [&](size_t dst, size_t src) { wq_host[src] = static_cast<int8_t>(int_of_e4m3(in[dst])); });
   return PQ_OK;
 }
 
@@ -988,6 +1006,7 @@ pq_status palquant_pack_weights_host(const float* w_host, const pq_layer_desc* d
   if (w_host == nullptr || inv_sw_host == nullptr || packed_host == nullptr) return PQ_EINVAL;
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
+  if (wslices_of(d) != 1) return PQ_EINVAL;  // float weights belong to plain layers
   const size_t per_group = static_cast<size_t>(d->Cout_g) * d->kh * d->kw * d->Cin_g;
   std::vector<int8_t> wq(per_group * d->G);
   const float lo = static_cast<float>(-(1 << (d->bits_w - 1))), hi = static_cast<float>((1 << (d->bits_w - 1)) - 1);
@@ -1010,6 +1029,7 @@ pq_status palquant_pack_weights_odd_host(const float* w_host, const pq_layer_des
   ConvParams p;
   pq_status st = plan_conv(d, &p, nullptr, nullptr);
   if (st != PQ_OK) return st;
+  if (wslices_of(d) != 1) return PQ_EINVAL;  // float weights belong to plain layers
   const size_t per_group = static_cast<size_t>(d->Cout_g) * d->kh * d->kw * d->Cin_g;
   const size_t need = per_group * d->G;
   if (packed_bytes < packed_weight_bytes_of(d, p)) return PQ_EINVAL;
@@ -1181,10 +1201,14 @@ pq_status bitsplit_layer(const pq_layer_desc* d, int bits_b, pq_layer_desc* out,
   if (wmax > 448) return PQ_EUNSUPPORTED;
   const int64_t taps = static_cast<int64_t>(d->kh) * d->kw;
   if (taps * d->Cin_g * ((1LL << d->bits_a) - 1) * (1LL << (d->bits_w - 1)) >= (1LL << 24)) return PQ_EUNSUPPORTED;
+  if (wslices_of(d) != 1) return PQ_EINVAL;  // an M-bit plain layer
   *out = *d;
   // the derived layer reads the split codes the kernel before it writes
   out->flags = d->flags & ~PQ_LAYER_INPUTS_READY;
-  out->Cin_g = d->Cin_g * Ga * Gw;
+  // input channel block i holds activation slice X_i (stored once); each of its
+  // codes meets the Gw weight slices of its tap
+  out->Cin_g = d->Cin_g * Ga;
+  out->wslices = Gw;
   out->bits_a = bits_b;
   out->bits_w = bits_b < 2 ? 2 : bits_b;
   *ga = Ga;
@@ -1228,17 +1252,19 @@ pq_status palquant_bitsplit_pack_weight_codes_host(const int8_t* wq_host, const 
   const size_t n_codes = static_cast<size_t>(d->G) * d->Cout_g * d->kh * d->kw * d->Cin_g;
   for (size_t i = 0; i < n_codes; ++i)
     if (wq_host[i] < lo || wq_host[i] > hi) return PQ_EINVAL;
-  // Weight block (i, j) holds 2^((i+j)B) w_j (w_j: slice j of w, the lower
-  // slices unsigned B-bit, the top one the signed rest), encoded as E4M3 (exact:
-  // bitsplit_layer bounded the magnitude).
+  // Weight slice j of input channel block i (activation slice X_i) holds
+  // 2^((i+j)B) w_j (w_j: slice j of w, the lower slices unsigned B-bit, the top
+  // one the signed rest), encoded as E4M3 (exact: bitsplit_layer bounded the
+  // magnitude).  The derived weights are [Cout][kh][kw][Gw][Ga Cin_g].
   uint8_t* out = static_cast<uint8_t*>(packed_host);
   const int Cin_t = t.Cin_g;
-  for_each_packed(p, t.kw, [&](size_t dst, size_t src) {
-    const size_t r = src / Cin_t;
+  for_each_packed(p, t.kw * Gw, [&](size_t dst, size_t src) {
+    const size_t r = src / Cin_t;                  // (co, kernel position, weight slice)
     const int k = static_cast<int>(src - r * Cin_t);
-    const int blk = k / d->Cin_g, c = k - blk * d->Cin_g;
-    const int i = blk / Gw, j = blk - i * Gw;
-    const int w = wq_host[r * d->Cin_g + c];
+    const int i = k / d->Cin_g, c = k - i * d->Cin_g;
+    const size_t pos = r / Gw;                     // (co, kernel position)
+    const int j = static_cast<int>(r - pos * Gw);
+    const int w = wq_host[pos * d->Cin_g + c];
     const int wj = (j < Gw - 1) ? ((w >> (j * bits_b)) & ((1 << bits_b) - 1)) : (w >> (j * bits_b));
     out[dst] = e4m3_of_int(wj * (1 << ((i + j) * bits_b)));
   });
@@ -1259,7 +1285,7 @@ pq_status palquant_bitsplit_act(const void* q_dev, void* xs_dev, size_t xs_bytes
   if (d->N == 0) return PQ_OK;
   if (d->G != 1) return PQ_EUNSUPPORTED;  // one group: the M-bit layer of Eq. 4
   return pq::launch_bitsplit_act(static_cast<const uint8_t*>(q_dev), static_cast<uint8_t*>(xs_dev), d->N,
-                                 static_cast<int64_t>(d->H) * d->W, C, Ga, Gw, bits_b,
+                                 static_cast<int64_t>(d->H) * d->W, C, Ga, bits_b,
                                  d->code_format == PQ_CODES_C16 ? 1 : 0, static_cast<cudaStream_t>(stream)) == 0
              ? PQ_OK
              : PQ_ECUDA;

@@ -176,7 +176,7 @@ struct PwParams {
 // Host-side launch helpers implemented in the .cu files.
 int launch_conv_tc(const ConvParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream);
 int launch_pointwise_tc(const PwParams& p, const CUtensorMap& tma_a, int grid, cudaStream_t stream);
-int launch_bitsplit_act(const uint8_t* q, uint8_t* xs, int64_t N, int64_t HW, int C, int Ga, int Gw, int B, int c16,
+int launch_bitsplit_act(const uint8_t* q, uint8_t* xs, int64_t N, int64_t HW, int C, int Ga, int B, int c16,
                         cudaStream_t stream);
 // pack: 0 one code per byte [N][C/16][HW][16]; 1 four 2-bit codes per byte
 // [N][C/16][HW][4 B]; 2 two 4-bit codes per byte [N][C/32][HW][16 B].

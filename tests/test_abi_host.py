@@ -177,13 +177,15 @@ def test_bitsplit_weight_blocks_are_shifted_slices(M, Bb):
     B_bits = Bb
     t = B.palquant_bitsplit_desc(d, B_bits)
     Ga = Gw = -(-M // B_bits)
-    assert t.Cin_g == 32 * Ga * Gw and t.bits_a == B_bits
+    # each activation slice once (Ga channel blocks), Gw weight slices per tap
+    assert t.Cin_g == 32 * Ga and t.wslices == Gw and t.bits_a == B_bits
     packed = B.palquant_bitsplit_pack_weight_codes_host(wq, d, B_bits)
-    vals = B.palquant_unpack_weight_codes_host(packed, t).astype(np.int64)  # [1,16,3,3,Ga*Gw*32]
+    vals = B.palquant_unpack_weight_codes_host(packed, t).astype(np.int64)  # [1,16,3,3,Gw,Ga*32]
+    assert vals.shape == (1, 16, 3, 3, Gw, Ga * 32)
     ws = oracle.bit_slices_weights(wq, M, B_bits)
     for i in range(Ga):
         for j in range(Gw):
-            blk = vals[..., (i * Gw + j) * 32:(i * Gw + j + 1) * 32]
+            blk = vals[..., j, i * 32:(i + 1) * 32]
             assert np.array_equal(blk, ws[j].astype(np.int64) << ((i + j) * B_bits))
 
 
@@ -193,7 +195,7 @@ def test_bitsplit_desc_clears_inputs_ready():
     d = B.layer_desc(2, 8, 8, 1, 32, 32, 3, 1, 1, bits_a=4, bits_w=4, bits_out=4, code_format=B.PQ_CODES_C16,
                      flags=B.PQ_LAYER_INPUTS_READY)
     t = B.palquant_bitsplit_desc(d, 2)
-    assert t.flags == 0 and t.Cin_g == 32 * 4 and t.bits_a == 2
+    assert t.flags == 0 and t.Cin_g == 32 * 2 and t.wslices == 2 and t.bits_a == 2
 
 
 def test_bitsplit_unsupported_shapes():

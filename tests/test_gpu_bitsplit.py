@@ -1,5 +1,6 @@
 """Bit-level decomposition (Sec. 3.3, Eq. 4) on the GPU: the M-bit layer computed as the
-G^2 shifted B-bit slice products in one tensor-core pass equals the oracle's M-bit
+G^2 shifted B-bit slice products in one tensor-core pass (each activation slice stored
+and read once, meeting the Gw weight slices as extra taps) equals the oracle's M-bit
 convolution (and its own decomposition) exactly."""
 import numpy as np
 import pytest
@@ -47,9 +48,10 @@ def test_bitsplit_conv_matches_oracle(M, Bb, shape, fmt):
     B.palquant_bitsplit_conv(qd, xs, nbytes, wp, acc, d, Bb)
     assert B.palquant_sync_check() == B.PQ_OK
     assert np.array_equal(acc.cpu().numpy().astype(np.int64), ref)
-    # the slices in the scratch buffer are the oracle's
-    Ga = Gw = -(-M // Bb)
+    # the slices in the scratch buffer are the oracle's, each stored once
+    Ga = -(-M // Bb)
+    assert t.Cin_g == Ga * C and t.wslices == Ga
     got = xs.cpu().numpy()
     slices = oracle.bit_slices_act(q, M, Bb)
-    want = np.concatenate([slices[i] for i in range(Ga) for _ in range(Gw)], axis=-1)
+    want = np.concatenate([slices[i] for i in range(Ga)], axis=-1)
     assert np.array_equal(got.reshape(want.shape) if fmt == 0 else got, _to_fmt(want, fmt).ravel() if fmt == 2 else want)
