@@ -40,6 +40,9 @@ def parse():
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--min-warmup-s", type=float, default=0.5,
+                    help="keep warming up (and the GPU busy) for at least this long after the clock sampler starts; "
+                         "0 for profilers")
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="target CPU time of the oracle baseline sample")
@@ -862,9 +865,9 @@ def run_ours(args, rank, world, local_rank):
     sampler.start()
     t_warm = time.perf_counter()
     n_warm = 0
-    while n_warm < args.warmup or time.perf_counter() - t_warm < 0.5:
+    while n_warm < args.warmup or time.perf_counter() - t_warm < args.min_warmup_s:
         with torch.cuda.stream(stream):
-            for _ in range(50):
+            for _ in range(min(50, max(1, args.warmup - n_warm)) if args.min_warmup_s <= 0 else 50):
                 step(n_warm, stream)
                 n_warm += 1
         torch.cuda.synchronize(dev)
