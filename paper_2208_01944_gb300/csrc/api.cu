@@ -520,10 +520,11 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
 // Planner of the pointwise kernel: 1x1, stride 1, pad 0 layers with
 // channel-blocked byte codes in and codes only out.  Pure host arithmetic; false
 // when the kernel does not cover the layer (the general kernel then runs it).
-//   tiles: up to 256 pixels of one image (two 128-row accumulators) when two
-//   such tiles fit tensor memory, else up to 128; every group's weights resident
+//   tiles: up to 256 pixels of one image (two 128-row accumulators) when they
+//   fit the CTA's tensor memory, else up to 128; every group's weights resident
 //   in shared memory (at most 96 KB); as many stages of input codes as the rest
-//   of the shared memory holds (2 to kPwMaxStages).  The weights use the general
+//   of the CTA's shared memory holds (up to kPwMaxStages); two CTAs per SM when
+//   each fits half the SM.  The weights use the general
 //   kernel's packing with one output block per group (Cout_g <= 256).
 // ---------------------------------------------------------------------------
 bool plan_pointwise(const pq_layer_desc* d, pq::PwParams* out) {
@@ -538,25 +539,36 @@ bool plan_pointwise(const pq_layer_desc* d, pq::PwParams* out) {
   pq::PwParams p;
   std::memset(&p, 0, sizeof(p));
   p.Npow2 = std::max(32, next_pow2(d->Cout_g));  // the epilogue reads 32 columns at a time
-  p.MT = (HW > 128 && 4 * p.Npow2 <= 512) ? 2 : 1;
-  p.T = static_cast<int>(std::min<int64_t>(HW, 128 * p.MT));
-  p.tiles_per_img = static_cast<int>((HW + p.T - 1) / p.T);
-  const int64_t items = static_cast<int64_t>(d->N) * p.tiles_per_img * d->G;
-  if (items >= (1LL << 31)) return false;
-  p.acc_stages = (512 / (p.MT * p.Npow2) >= 4) ? 4 : 2;
-  p.tmem_cols = static_cast<uint32_t>(std::max(32, next_pow2(p.acc_stages * p.MT * p.Npow2)));
   p.w_bytes = static_cast<uint32_t>(d->G) * d->Cin_g * d->Cout_g;
   if (p.w_bytes > 96u * 1024u) return false;
   p.nch = d->Cin_g / 16;
   if (p.nch > 256) return false;  // TMA box extent
   p.ksteps = d->Cin_g / 32;
-  p.a_stage_bytes = static_cast<uint32_t>(p.MT) * p.nch * 2048u;
-  p.a_tx_bytes = p.a_stage_bytes;
   const uint32_t w_round = round_up(p.w_bytes, 1024);
   const uint32_t bar_bytes = 1024;
-  const int64_t room = static_cast<int64_t>(pq::kMaxSmem) - 1024 - w_round - bar_bytes;
-  const int stages = static_cast<int>(std::min<int64_t>(pq::kPwMaxStages, room / p.a_stage_bytes));
+  // Two CTAs per SM where each fits half of the SM's shared memory (three or more
+  // stages) and half of its tensor memory: a CTA of the next launch then starts
+  // loading as soon as one of this launch's two CTAs on the SM finishes, and the
+  // two CTAs' pipelines overlap.  Else one CTA with the whole SM.
+  int stages = 0;
+  for (int pair = 1; pair >= 0 && stages < 2; --pair) {
+    const int tmem = pair ? 256 : 512;
+    p.ctas_per_sm = pair ? 2 : 1;
+    p.MT = (HW > 128 && 2 * p.Npow2 <= tmem / (pair ? 1 : 2)) ? 2 : 1;
+    p.acc_stages = std::max(1, std::min(4, tmem / (p.MT * p.Npow2)));
+    if (p.acc_stages == 3) p.acc_stages = 2;
+    p.a_stage_bytes = static_cast<uint32_t>(p.MT) * p.nch * 2048u;
+    const int64_t room = static_cast<int64_t>(pair ? pq::kPwHalfSmem : pq::kMaxSmem) - 1024 - w_round - bar_bytes;
+    stages = static_cast<int>(std::min<int64_t>(pq::kPwMaxStages, room / p.a_stage_bytes));
+    if (pair && stages < 3) stages = 0;
+  }
   if (stages < 2) return false;
+  p.tmem_cols = static_cast<uint32_t>(std::max(32, next_pow2(p.acc_stages * p.MT * p.Npow2)));
+  p.T = static_cast<int>(std::min<int64_t>(HW, 128 * p.MT));
+  p.tiles_per_img = static_cast<int>((HW + p.T - 1) / p.T);
+  const int64_t items = static_cast<int64_t>(d->N) * p.tiles_per_img * d->G;
+  if (items >= (1LL << 31)) return false;
+  p.a_tx_bytes = p.a_stage_bytes;
   p.a_stages = stages;
   p.N = d->N;
   p.HW = static_cast<int>(HW);
@@ -864,7 +876,7 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
     pw.wait_limit_ns = p.wait_limit_ns;
     pw.pdl = 1;
     pw.pdl_early_loads = (d->flags & PQ_LAYER_INPUTS_READY) ? 1 : 0;
-    const int pw_grid = std::min(sms, pw.items);
+    const int pw_grid = std::min(sms * pw.ctas_per_sm, pw.items);
     if (pw_grid <= 0) return PQ_OK;
     CUtensorMap pw_map;
     if (!encode_pw_map(d, pw, q_dev, &pw_map)) return PQ_ECUDA;

@@ -285,7 +285,8 @@ __device__ __forceinline__ void pw_epilogue(const PwParams& p, const PwBars& bar
 
 }  // namespace
 
-__global__ void __launch_bounds__(kPwThreads, 1)
+// At most 102 registers a thread, so that two CTAs fit an SM's register file.
+__global__ void __launch_bounds__(kPwThreads, 2)
     pq_pointwise_tc_kernel(const __grid_constant__ PwParams p, const __grid_constant__ CUtensorMap tmA) {
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);

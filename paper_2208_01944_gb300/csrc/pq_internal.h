@@ -143,10 +143,11 @@ struct ConvParams {
 // The pointwise kernel (1x1, stride 1, pad 0 layers, channel-blocked codes in
 // and codes only out); filled by the host planner.  A work item is (image,
 // pixel tile, group), the group fastest.
-constexpr int kPwEpiGroups = 4;                             // epilogue warpgroups, taking accumulators in turn
+constexpr int kPwEpiGroups = 2;                             // epilogue warpgroups, taking accumulators in turn
 constexpr int kPwFirstEpiWarp = 2;                          // warp 0 loads, warp 1 issues the MMAs
 constexpr int kPwThreads = 32 * (kPwFirstEpiWarp + 4 * kPwEpiGroups);
 constexpr int kPwMaxStages = 8;
+constexpr int kPwHalfSmem = 113 * 1024;                     // dynamic shared memory of one of two CTAs on an SM
 
 struct PwParams {
   int N, HW, G, Cin_g, Cout_g;
@@ -158,6 +159,7 @@ struct PwParams {
   int ksteps;             // Cin_g / 32: MMAs per accumulator
   int Npow2;              // tensor-memory columns per accumulator
   int a_stages, acc_stages;
+  int ctas_per_sm;        // 2: two CTAs share an SM (each at most half its shared memory and tensor memory)
   uint32_t a_stage_bytes; // MT * nch * 2048: per accumulator one TMA box of nch planes x 128 positions
   uint32_t a_tx_bytes;    // bytes a stage receives (whole boxes, out-of-image rows zero-filled)
   uint32_t w_bytes;       // every group's packed weights, G * Cout_g * Cin_g
