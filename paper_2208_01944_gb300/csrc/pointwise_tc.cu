@@ -8,10 +8,11 @@
 //   q'[n, p, dst(g) Cout_g + co] = clamp(rint(m_req[g] sum_ci q[n, p, g Cin_g + ci] w[g, co, ci]), 0, Qp)
 // with channel-blocked codes [N][C/16][H*W][16] in and out.
 //
-// How (one persistent CTA per SM, warp-specialised):
+// How (persistent CTAs, two per SM where each fits half the SM, warp-specialised):
 //  * A work item is (image, tile of up to 256 pixels, group), the group
 //    fastest, and a CTA takes a contiguous range of items, so its loads walk
-//    through consecutive bytes of each image.
+//    through consecutive bytes of each image.  With two CTAs per SM, a CTA of
+//    the next launch starts loading as soon as one of the two finishes.
 //  * Warp 0 (one lane) bulk-copies every group's packed weights into shared
 //    memory once, then loads each item's input codes with one TMA box per
 //    128-row accumulator (the group's 16-channel planes x 128 positions;
@@ -21,7 +22,7 @@
 //    item, tcgen05.mma kind::f8f6f4 with M = 128 and N = Cout_g on the codes read
 //    in place as E4M3 subnormals (a code byte v <= 15 is the E4M3 encoding of
 //    v 2^-9, so every sum is exact), into a tensor-memory accumulator stage.
-//  * Four epilogue warpgroups take the accumulators in turn: tcgen05.ld (the
+//  * Two epilogue warpgroups take the accumulators in turn: tcgen05.ld (the
 //    next 32 columns in flight while the current ones are converted), the
 //    requantisation in registers (through the fp16 conversion, two values per
 //    instruction), and the codes stored straight from registers
@@ -117,7 +118,7 @@ __device__ __forceinline__ void pw_producer(const PwParams& p, const CUtensorMap
 // Tensor-core issue role (warp 1, converged; one elected lane issues).  The
 // issue loop is compiled for the accumulators per item (MT) and the K steps
 // (KS, 0: a runtime loop), so that an item's MMAs go out back to back: the
-// warp shares its scheduler with four busy epilogue warps, and every
+// warp shares its scheduler with busy epilogue warps, and every
 // instruction per MMA delays the next item's accumulator.
 template <int MT, int KS>
 __device__ __forceinline__ void pw_mma(const PwParams& p, const PwBars& bars, uint32_t a_base, uint32_t w_base,
@@ -196,11 +197,11 @@ __device__ __forceinline__ void pw_mma_dispatch(const PwParams& p, const PwBars&
   return pw_mma<1, 0>(p, bars, a_base, w_base, tmem_base, it0, it1, ctx);
 }
 
-// Epilogue role (warps 2-17: four warpgroups).  The tasks are the items'
+// Epilogue role (warps 2-9: two warpgroups).  The tasks are the items'
 // accumulators in order (item i, accumulator mt is task i MT + mt), and
-// warpgroup w takes tasks w, w + 4, ... (w, w + 2, ... when only two
-// accumulators fit tensor memory): with two accumulators per item, two
-// warpgroups share an item and two items are in flight.  Warp w reads
+// warpgroup w takes tasks w, w + 2, ... (only warpgroup 0 when the CTA's tensor
+// memory holds a single accumulator): with two accumulators per item, the two
+// warpgroups share each item.  Warp w reads
 // tensor-memory lanes 32 (w % 4) .. 32 (w % 4) + 31, the accumulator rows that
 // are consecutive pixels of the tile, and takes the accumulator 32 columns at a
 // time (two 16-channel planes of codes), the next 32 columns loading while the
