@@ -366,7 +366,13 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
     if (pub) *pub = plan;
     return PQ_EUNSUPPORTED;
   }
+  // Stride 2 with channel-blocked codes: TMA stages the tile's input window (2 Hd
+  // rows x 2 Wd positions, both stride phases) and the copy warps split it into
+  // the phase planes; the window's row of 2 Wd positions is one box row of
+  // 4 Wd 8-byte elements (at most 256).
+  const bool split = c16 && !p2 && !quant_in && d->stride == 2 && !flat && 4 * p.Wd <= 256 && 2 * p.Hd <= 256;
   auto pk_stage_bytes = [&](int KC) -> uint32_t {
+    if (split) return round_up(static_cast<uint64_t>(KC / (16 * cpb)) * (2 * p.Hd) * (2 * p.Wd) * 16, 1024);
     if (quant_in) {
       // KC/32 fp32 boxes of 32 channels x all positions of the stage (128-byte rows),
       // each starting on a 1024-byte swizzle atom
@@ -434,17 +440,21 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   p.codes_f4 = f4 ? 1 : 0;
   p.chunk_shift = f4 ? 5 : 4;
   p.a_unpack = p2 ? 1 : 0;
+  p.a_split = split ? 1 : 0;
   p.a_quant = quant_in ? 1 : 0;
   p.q_box_bytes = quant_in ? round_up(static_cast<uint64_t>(flat ? p.flat_box : p.Hd * p.Wd) * 128, 1024) : 0;
   p.pk_box_w = pk_box_w;
   p.pk_off = pk_off;
   p.pk_stage_bytes = pk_stage_bytes(KC);
   // The A operand comes by TMA when every plane row is one contiguous run in
-  // global memory: channel-blocked codes, stride 1, rows of at most 128 positions.
-  p.a_tma = (quant_in || p2 || (c16 && d->stride == 1 && (flat ? p.flat_box <= 256 : p.Wd <= 128))) ? 1 : 0;
+  // global memory (channel-blocked codes, stride 1, rows of at most 128
+  // positions), or through the staging ring (packed codes, quantise-on-load,
+  // stride-2 windows).
+  p.a_tma = (quant_in || p2 || split || (c16 && d->stride == 1 && (flat ? p.flat_box <= 256 : p.Wd <= 128))) ? 1 : 0;
   p.a_mt16 = (flat && c16 && !p2 && !quant_in) ? static_cast<uint32_t>(p.nch) * 128u : 128u;
   p.a_tx_bytes = quant_in ? static_cast<uint32_t>(KC) * 4u * (flat ? p.flat_box : p.Hd * p.Wd)
                  : p2 ? static_cast<uint32_t>(p.nch) * pk_box_w * (flat ? 1 : p.Hd) * 4u
+                 : split ? static_cast<uint32_t>(p.nch) * (2 * p.Hd) * (2 * p.Wd) * 16u
                  : flat ? static_cast<uint32_t>(p.nch) * p.flat_box * 16u
                         : static_cast<uint32_t>(p.nph) * p.nch * p.Hd * p.Wd * 16u;
   {
@@ -667,7 +677,9 @@ bool encode_c16_map(const pq_layer_desc* d, const ConvParams& p, const void* q_d
   }
   cuuint64_t dims[4] = {2 * W, H, C16, static_cast<cuuint64_t>(d->N)};
   cuuint64_t strides[3] = {W * 16, H * W * 16, C16 * H * W * 16};
-  cuuint32_t box[4] = {2u * static_cast<cuuint32_t>(p.Wd), static_cast<cuuint32_t>(p.Hd),
+  // stride 2 (a_split): the window of 2 Hd rows x 2 Wd positions
+  const cuuint32_t sw = p.a_split ? 2u : 1u;
+  cuuint32_t box[4] = {2u * sw * static_cast<cuuint32_t>(p.Wd), sw * static_cast<cuuint32_t>(p.Hd),
                        static_cast<cuuint32_t>(p.nch), 1};
   return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT64, 4, const_cast<void*>(q_dev), dims, strides, box, es,
              CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,

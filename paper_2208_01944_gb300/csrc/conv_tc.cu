@@ -179,6 +179,18 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
         }
         ra.advance();
         ++a_issued;
+      } else if (a_tma && p.a_split) {
+        // Stride 2: the tile's whole input window (both stride phases of its rows
+        // and columns) into the staging ring; the copy warps split it into the
+        // phase planes.
+        if (!mbar_wait(bars.pk_empty(ra.stage), ra.phase ^ 1u, ctx)) { ok = false; break; }
+        const uint32_t full = bars.pk_full(ra.stage);
+        mbar_arrive_expect_tx(full, p.a_tx_bytes);
+        const int chi = (p.src_group[item.g] * p.Cin_g + kb * p.KC) >> p.chunk_shift;
+        tma_load_4d(pk_base + ra.stage * p.pk_stage_bytes, tmA, 4 * p.w_coord, 2 * (item.oh0(p.Ht) + p.h_off), chi,
+                    item.n, full);
+        ra.advance();
+        ++a_issued;
       } else if (a_tma && p.a_unpack) {
         // Packed codes: the box of 32-bit words into the staging ring; the copy
         // warps unpack it into the operand stage.
@@ -225,7 +237,7 @@ __device__ __forceinline__ void producer_role(const ConvParams& p, const CUtenso
   // Drain: the last min(stages, issued) copies of each ring may still be in flight.
   const int64_t na = p.a_stages, nbs = p.b_resident ? 1 : p.b_stages;
   for (int64_t k = (a_issued > na ? a_issued - na : 0); k < a_issued; ++k)
-    mbar_wait_drain((p.a_unpack || p.a_quant) ? bars.pk_full(static_cast<int>(k % na)) : bars.a_full(static_cast<int>(k % na)),
+    mbar_wait_drain((p.a_unpack || p.a_quant || p.a_split) ? bars.pk_full(static_cast<int>(k % na)) : bars.a_full(static_cast<int>(k % na)),
                     static_cast<uint32_t>((k / na) & 1), ctx.limit_ns, ctx.err);
   for (int64_t k = (b_issued > nbs ? b_issued - nbs : 0); k < b_issued; ++k)
     mbar_wait_drain(bars.b_full(static_cast<int>(k % nbs)), static_cast<uint32_t>((k / nbs) & 1), ctx.limit_ns, ctx.err);
@@ -401,6 +413,67 @@ __device__ __forceinline__ void unpack_role(const ConvParams& p, const Bars& bar
           const uint4 u = unpack2_word(v);
           asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(drow + static_cast<uint32_t>(w) * 16u),
                        "r"(u.x), "r"(u.y), "r"(u.z), "r"(u.w)
+                       : "memory");
+        }
+      }
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        mbar_arrive(bars.a_full(r.stage));
+        mbar_arrive(bars.pk_empty(r.stage));
+      }
+      r.advance();
+    }
+  }
+}
+
+// --------------------------------------------------------------------------
+// Split role for stride 2 (warps 2-5): a staged window holds, per 16-byte chunk
+// j, 2 Hd input rows of 2 Wd positions (16 bytes each) starting at input row
+// 2 (oh0 + h_off) and column 2 w_coord; staged row y = 2 r + a and column
+// x = 2 w + b go to row r, position w of the plane of stride phase (a, b) (the
+// phases no tap uses are skipped).  Warp wi takes staged rows wi, wi + 4, ...
+// and its lanes consecutive columns: conflict-free 16-byte reads, and 16-byte
+// writes in two runs of consecutive positions.  Positions outside the image were
+// zero-filled by the TMA unit (the zero padding).  The stage goes to the tensor
+// core after a proxy fence, the staging stage back to the producer.
+// --------------------------------------------------------------------------
+__device__ __forceinline__ void split_role(const ConvParams& p, const Bars& bars, uint32_t a_base, uint32_t pk_base,
+                                           int64_t it0, int64_t it1, const WaitCtx& ctx) {
+  const int tid = threadIdx.x - 32 * kFirstLoadWarp;
+  const int wi = tid >> 5, lane = tid & 31;
+  const int Hd = p.Hd, Wd = p.Wd, Ws = 2 * p.Wd;
+  const int n_rows = p.nch * 2 * Hd;
+  const uint32_t plane = p.lbo_a;
+  // destination offset of phase (a, b), or -1 where no tap reads it
+  int ph_off[2][2] = {{-1, -1}, {-1, -1}};
+  for (int q = 0; q < p.nph && q < kMaxPhases; ++q) ph_off[p.phase_a[q] & 1][p.phase_b[q] & 1] = q * p.a_phase_bytes;
+  Ring r{0, 0, static_cast<uint32_t>(p.a_stages)};
+  bool ok = true;
+  for (int64_t it = it0; it < it1 && ok; ++it) {
+    for (int kb = 0; kb < p.n_kb; ++kb) {
+      if (!warp_wait(bars.pk_full(r.stage), r.phase, ctx)) { ok = false; break; }
+      if (!warp_wait(bars.a_empty(r.stage), r.phase ^ 1u, ctx)) { ok = false; break; }
+      const uint32_t src = pk_base + r.stage * p.pk_stage_bytes;
+      const uint32_t dst = a_base + r.stage * p.a_stage_bytes;
+      for (int row = wi; row < n_rows; row += kLoadWarps) {
+        const int j = row / (2 * Hd), y = row - j * 2 * Hd;
+        const int a = y & 1, rr = y >> 1;
+        const int off0 = ph_off[a][0], off1 = ph_off[a][1];
+        if (off0 < 0 && off1 < 0) continue;
+        const uint32_t srow = src + static_cast<uint32_t>(row * Ws) * 16u;
+        const uint32_t drow = dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(rr * Wd) * 16u;
+        for (int x = lane; x < Ws; x += 32) {
+          const int off = (x & 1) ? off1 : off0;
+          if (off < 0) continue;
+          uint32_t v0, v1, v2, v3;
+          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                       : "=r"(v0), "=r"(v1), "=r"(v2), "=r"(v3)
+                       : "r"(srow + static_cast<uint32_t>(x) * 16u)
+                       : "memory");
+          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(drow + static_cast<uint32_t>(off) +
+                                                                         static_cast<uint32_t>(x >> 1) * 16u),
+                       "r"(v0), "r"(v1), "r"(v2), "r"(v3)
                        : "memory");
         }
       }
@@ -802,84 +875,54 @@ __device__ __forceinline__ void epi_store_codes(const ConvParams& p, const EpiIt
   }
 }
 
-// General unit: int32 sums, fp32 outputs (with the shortcut) and codes, or the
-// per-channel scatter of the channel shuffle.
-__device__ __forceinline__ void epi_general16(const ConvParams& p, const EpiItem& e, uint8_t* stg, int lane, int m, int ch,
-                                           const uint32_t* v) {
+// The 16 shortcut values of accumulator row m, 16-column chunk ch (the source
+// channels of the unit), or zeros for a row outside the output.
+__device__ __forceinline__ void epi_load_shortcut(const ConvParams& p, const EpiItem& e, int m, int ch,
+                                                  float (&sc)[16]) {
   bool valid;
   const int pos = epi_pos(p, e, m, valid);
+  if (valid) {
+    const long long pix = static_cast<long long>(e.n) * p.Ho * p.Wo + pos;
+    const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + pix * p.C_out_total + e.src_c0 + ch * 16);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float4 t = s4[j];
+      sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
+    }
+  } else {
+#pragma unroll
+    for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
+  }
+}
+
+// Channel-shuffle unit: int32 sums, fp32 outputs (with the shortcut, loaded by
+// the caller into sc) and codes, each channel scattered to destination channel
+// co * G + g (unstaged, one element at a time).
+__device__ __forceinline__ void epi_general16(const ConvParams& p, const EpiItem& e, int m, int ch, const uint32_t* v,
+                                              const float (&sc)[16]) {
+  bool valid;
+  const int pos = epi_pos(p, e, m, valid);
+  if (!valid) return;
   const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
   const long long pix = static_cast<long long>(e.n) * hw_out + pos;
-  const long long row_elem = valid ? pix * p.C_out_total : -1;
   const bool has_sc = p.shortcut != nullptr;
   const int qmax = p.qmax_out;
   const float qmax_f = static_cast<float>(qmax);
-  float sc[16];
-  if (has_sc) {
-    if (valid) {
-      const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + pix * p.C_out_total + e.src_c0 + ch * 16);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float4 t = s4[j];
-        sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
-      }
-    } else {
-#pragma unroll
-      for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
-    }
-  }
-  float y[16];
-  int code[16];
-#pragma unroll
   for (int j = 0; j < 16; ++j) {
     const float raw = __uint_as_float(v[j]);
     float t = __fmul_rn(raw, e.m_out512);  // = (float)acc * m_out, one rounding
     if (has_sc) t = __fadd_rn(t, sc[j]);
     if (p.relu) t = fmaxf(t, 0.0f);
-    y[j] = t;
-    code[j] = requant_code(has_sc ? __fmul_rn(t, e.m_req) : __fmul_rn(raw, e.m_req512), qmax_f, qmax);
-  }
-  if (p.channel_shuffle) {
-    // Per-channel scatter (destination channel co * G + g); rarely used, unstaged.
-    if (valid) {
-      for (int j = 0; j < 16; ++j) {
-        const int co = e.nb * p.Nblk + ch * 16 + j;
-        const long long dc = static_cast<long long>(co) * p.G + e.g;
-        const long long o = pix * p.C_out_total + dc;
-        if (p.acc_out) p.acc_out[o] = __float2int_rn(__fmul_rn(__uint_as_float(v[j]), 512.0f));
-        if (p.y_out) p.y_out[o] = y[j];
-        if (p.q_out) {
-          const long long c16o = (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (dc >> 4)) * hw_out + pos;
-          p.q_out[p.codes_c16 ? c16o * 16 + (dc & 15) : o] = static_cast<uint8_t>(code[j]);
-        }
-      }
+    const int code = requant_code(has_sc ? __fmul_rn(t, e.m_req) : __fmul_rn(raw, e.m_req512), qmax_f, qmax);
+    const int co = e.nb * p.Nblk + ch * 16 + j;
+    const long long dc = static_cast<long long>(co) * p.G + e.g;
+    const long long o = pix * p.C_out_total + dc;
+    if (p.acc_out) p.acc_out[o] = __float2int_rn(__fmul_rn(raw, 512.0f));
+    if (p.y_out) p.y_out[o] = t;
+    if (p.q_out) {
+      const long long c16o = (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (dc >> 4)) * hw_out + pos;
+      p.q_out[p.codes_c16 ? c16o * 16 + (dc & 15) : o] = static_cast<uint8_t>(code);
     }
-    return;
-  }
-  if (p.acc_out) {
-    uint32_t* row = reinterpret_cast<uint32_t*>(stg + lane * p.stage_q_pitch);
-    for (int j = 0; j < 16; j += 4)
-      *reinterpret_cast<int4*>(row + j) =
-          make_int4(__float2int_rn(__fmul_rn(__uint_as_float(v[j]), 512.0f)),
-                    __float2int_rn(__fmul_rn(__uint_as_float(v[j + 1]), 512.0f)),
-                    __float2int_rn(__fmul_rn(__uint_as_float(v[j + 2]), 512.0f)),
-                    __float2int_rn(__fmul_rn(__uint_as_float(v[j + 3]), 512.0f)));
-    warp_store_rows(stg, p.stage_q_pitch, 64, reinterpret_cast<uint8_t*>(p.acc_out),
-                    row_elem < 0 ? -1 : (row_elem + e.dst_c0 + ch * 16) * 4, lane);
-  }
-  if (p.y_out) {
-    float* row = reinterpret_cast<float*>(stg + lane * p.stage_q_pitch);
-    for (int j = 0; j < 16; j += 4) *reinterpret_cast<float4*>(row + j) = make_float4(y[j], y[j + 1], y[j + 2], y[j + 3]);
-    warp_store_rows(stg, p.stage_q_pitch, 64, reinterpret_cast<uint8_t*>(p.y_out),
-                    row_elem < 0 ? -1 : (row_elem + e.dst_c0 + ch * 16) * 4, lane);
-  }
-  if (p.q_out) {
-    uint4 w;
-    w.x = __byte_perm(__byte_perm(code[0], code[1], 0x0040), __byte_perm(code[2], code[3], 0x0040), 0x5410);
-    w.y = __byte_perm(__byte_perm(code[4], code[5], 0x0040), __byte_perm(code[6], code[7], 0x0040), 0x5410);
-    w.z = __byte_perm(__byte_perm(code[8], code[9], 0x0040), __byte_perm(code[10], code[11], 0x0040), 0x5410);
-    w.w = __byte_perm(__byte_perm(code[12], code[13], 0x0040), __byte_perm(code[14], code[15], 0x0040), 0x5410);
-    epi_store_codes(p, e, stg, lane, valid, pos, ch, w);
   }
 }
 
@@ -1040,13 +1083,98 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         c_mt = n_mt;
         c_ch = n_ch;
       }
-    } else {
+    } else if (!p.channel_shuffle) {
+      // General units (int32 sums, fp32 outputs with or without the shortcut,
+      // codes): lane r's 16 values of a unit are 64 contiguous bytes of its
+      // pixel's NHWC row, loaded and stored straight from registers.  The codes
+      // go through the fp16 conversion (epi_codes16_f16) where no NaN can reach
+      // it: without a shortcut the value is fl(raw * m_req * 2^-15) =
+      // fl(acc * m_req) * 2^-24; with one, fl(y * m_req * 2^-24) =
+      // fl(y * m_req) * 2^-24 (a power-of-two factor, exact while the product is
+      // normal, and both round to code 0 below that), and ReLU has removed NaN
+      // (fmaxf(NaN, 0) = 0).  A shortcut without ReLU keeps the scalar form,
+      // which maps NaN to code 0.
+      const bool has_sc = p.shortcut != nullptr;
+      const bool f16q = !has_sc || p.relu;
+      const float m_q = has_sc ? __fmul_rn(e.m_req, 1.0f / 16777216.0f) : e.m_req15;
+      const int qmax = p.qmax_out;
+      const float qmax_f = static_cast<float>(qmax);
+      const int m_lane = quarter * 32 + lane;
+      const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
       for (int u = wg; u < n_units; u += n_groups) {
         const int mt = u / nchunks, ch = u - mt * nchunks;
+        bool valid;
+        const int pos = epi_pos(p, e, mt * 128 + m_lane, valid);
+        const long long rowc = (static_cast<long long>(e.n) * hw_out + pos) * p.C_out_total;
+        uint32_t v[16];
+        tmem_ld16(e.tbase + mt * p.Npow2 + ch * 16, v);
+        float sc[16];
+        if (has_sc) {
+          if (valid) {
+            const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + rowc + e.src_c0 + ch * 16);
+#pragma unroll
+            for (int j = 0; j < 4; ++j) {
+              const float4 t = s4[j];
+              sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
+            }
+          } else {
+#pragma unroll
+            for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
+          }
+        }
+        tmem_wait_ld();
+        uint32_t y[16];
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          float t = __fmul_rn(__uint_as_float(v[j]), e.m_out512);  // = (float)acc * m_out, one rounding
+          if (has_sc) t = __fadd_rn(t, sc[j]);
+          if (p.relu) t = fmaxf(t, 0.0f);
+          y[j] = __float_as_uint(t);
+        }
+        if (valid) {
+          const long long o = rowc + e.dst_c0 + ch * 16;
+          if (p.acc_out) {
+            int4* a4 = reinterpret_cast<int4*>(p.acc_out + o);
+#pragma unroll
+            for (int j = 0; j < 16; j += 4)
+              a4[j >> 2] = make_int4(__float2int_rn(__fmul_rn(__uint_as_float(v[j]), 512.0f)),
+                                     __float2int_rn(__fmul_rn(__uint_as_float(v[j + 1]), 512.0f)),
+                                     __float2int_rn(__fmul_rn(__uint_as_float(v[j + 2]), 512.0f)),
+                                     __float2int_rn(__fmul_rn(__uint_as_float(v[j + 3]), 512.0f)));
+          }
+          if (p.y_out) {
+            uint4* y4 = reinterpret_cast<uint4*>(p.y_out + o);
+#pragma unroll
+            for (int j = 0; j < 16; j += 4) y4[j >> 2] = make_uint4(y[j], y[j + 1], y[j + 2], y[j + 3]);
+          }
+        }
+        if (p.q_out) {
+          uint4 w;
+          if (f16q) {
+            w = epi_codes16_f16(has_sc ? y : v, m_q, qmax2);
+          } else {
+            int code[16];
+#pragma unroll
+            for (int j = 0; j < 16; ++j) code[j] = requant_code(__fmul_rn(__uint_as_float(y[j]), e.m_req), qmax_f, qmax);
+            w.x = __byte_perm(__byte_perm(code[0], code[1], 0x0040), __byte_perm(code[2], code[3], 0x0040), 0x5410);
+            w.y = __byte_perm(__byte_perm(code[4], code[5], 0x0040), __byte_perm(code[6], code[7], 0x0040), 0x5410);
+            w.z = __byte_perm(__byte_perm(code[8], code[9], 0x0040), __byte_perm(code[10], code[11], 0x0040), 0x5410);
+            w.w = __byte_perm(__byte_perm(code[12], code[13], 0x0040), __byte_perm(code[14], code[15], 0x0040), 0x5410);
+          }
+          epi_store_codes(p, e, stg, lane, valid, pos, ch, w);
+        }
+      }
+    } else {
+      // The channel shuffle's per-channel scatter (rarely used).
+      const int m_lane = quarter * 32 + lane;
+      for (int u = wg; u < n_units; u += n_groups) {
+        const int mt = u / nchunks, ch = u - mt * nchunks;
+        float sc[16];
+        if (p.shortcut != nullptr) epi_load_shortcut(p, e, mt * 128 + m_lane, ch, sc);
         uint32_t v[16];
         tmem_ld16(e.tbase + mt * p.Npow2 + ch * 16, v);
         tmem_wait_ld();
-        epi_general16(p, e, stg, lane, mt * 128 + quarter * 32 + lane, ch, v);
+        epi_general16(p, e, mt * 128 + m_lane, ch, v, sc);
       }
     }
     // One arrival per warp: the warp's tensor-memory reads are complete (each
@@ -1083,9 +1211,9 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < bars.A; ++s) {
       // TMA, or one arrival per copy warp
-      mbar_init(bars.a_full(s), (p.a_tma && !p.a_unpack && !p.a_quant) ? 1 : kLoadWarps);
+      mbar_init(bars.a_full(s), (p.a_tma && !p.a_unpack && !p.a_quant && !p.a_split) ? 1 : kLoadWarps);
       mbar_init(bars.a_empty(s), 1);
-      if (p.a_unpack || p.a_quant) {
+      if (p.a_unpack || p.a_quant || p.a_split) {
         mbar_init(bars.pk_full(s), 1);
         mbar_init(bars.pk_empty(s), kLoadWarps);
       }
@@ -1097,7 +1225,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
     for (int s = 0; s < p.acc_stages; ++s) {
       mbar_init(bars.acc_full(s), 1);
       mbar_init(bars.acc_empty(s),
-                (p.a_tma && !p.a_unpack && !p.a_quant) ? kEpiWarps + kLoadWarps : kEpiWarps);  // one per warp
+                (p.a_tma && !p.a_unpack && !p.a_quant && !p.a_split) ? kEpiWarps + kLoadWarps : kEpiWarps);  // one per warp
     }
     mbar_init(bars.drain(), 1);
     *abort_flag = 0;
@@ -1130,7 +1258,7 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   // weights (pdl_early_loads), only the epilogue warps wait: the others' global
   // accesses are those loads (the producer's copies, the loader warps' reads),
   // and the quantiser and MMA warps work in shared and tensor memory.
-  const bool third_epi = p.a_tma && !p.a_unpack && !p.a_quant;  // warps 2-5 run the epilogue too
+  const bool third_epi = p.a_tma && !p.a_unpack && !p.a_quant && !p.a_split;  // warps 2-5 run the epilogue too
   const bool epi_warp = warp >= kFirstEpiWarp || (third_epi && warp >= kFirstLoadWarp);
   if (p.pdl && (epi_warp || !p.pdl_early_loads)) asm volatile("griddepcontrol.wait;" ::: "memory");
   // Let the next dependent launch on the stream start its CTAs as SMs free up, but
@@ -1161,13 +1289,16 @@ __global__ void __launch_bounds__(kConvThreads, 1)
   } else if (warp < kFirstEpiWarp && p.a_quant) {
     quant_role<F4, LU>(p, bars, a_base, base + p.smem_pk_off, it0, it1,
                WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
+  } else if (warp < kFirstEpiWarp && p.a_split) {
+    split_role(p, bars, a_base, base + p.smem_pk_off, it0, it1,
+               WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else if (warp < kFirstEpiWarp && p.a_unpack) {
     unpack_role(p, bars, a_base, base + p.smem_pk_off, it0, it1,
                 WaitCtx{abort_flag, p.err, p.wait_limit_ns, PQ_ERR_PRODUCER});
   } else {
     // With TMA loading the activations as they are, the copy warps form a third
     // epilogue warpgroup.
-    const bool third = p.a_tma && !p.a_unpack && !p.a_quant;
+    const bool third = p.a_tma && !p.a_unpack && !p.a_quant && !p.a_split;
     const int first = third ? kFirstLoadWarp : kFirstEpiWarp;
 
     epilogue_role<F4>(p, bars, tmem_base, gbase + p.smem_stage_off, first, third ? kEpiGroups + 1 : kEpiGroups, it0, it1,

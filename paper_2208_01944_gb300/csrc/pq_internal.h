@@ -56,6 +56,10 @@ struct ConvParams {
   // them into the operand stages (a_unpack = 1): staged rows of pk_box_w 32-bit
   // words starting pk_off words left of the tile's first position.
   int a_unpack;
+  // Stride 2 (a_split = 1): TMA stages the input window of the tile (2 Hd rows x
+  // 2 Wd positions x nch chunks, every stride phase interleaved) into the staging
+  // ring and the copy warps split it into the phase planes of the operand stage.
+  int a_split;
   // Quantise-on-load (a_quant = 1): the input is fp32 NHWC; TMA stages boxes of 32
   // channels x all positions of a stage (128-byte rows, 128-byte swizzle) into the
   // staging ring and the copy warps quantise them into the operand stage:

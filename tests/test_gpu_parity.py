@@ -96,6 +96,7 @@ SMALL_CASES = [
     Case(1, 40, 30, 2, 64, 64, 3, 2, 1, seed=18),                     # three accumulators, stride 2
     Case(2, 20, 20, 2, 64, 64, 1, 1, 0, seed=19),                     # flat, two boxes per tile, ragged
     Case(2, 17, 17, 2, 64, 64, 1, 1, 0, shortcut=True, seed=20),      # flat, second box wholly past the image
+    Case(1, 6, 140, 2, 32, 32, 3, 2, 1, seed=21),                     # stride 2, window wider than one TMA box row
 ]
 
 
@@ -473,7 +474,7 @@ def test_layer_with_odd_weight_levels_matches_oracle(B, fmt, bits_w):
 F4_CASES = [
     Case(1, 28, 28, 2, 64, 32, 3, 1, 1, seed=80),
     Case(2, 13, 11, 3, 64, 96, 3, 1, 1, seed=81),                     # odd sizes, six 16-column chunks
-    Case(3, 9, 17, 4, 64, 64, 3, 2, 1, seed=82),                      # stride 2 (copy warps)
+    Case(3, 9, 17, 4, 64, 64, 3, 2, 1, seed=82),                      # stride 2 (staged window split into phases)
     Case(2, 10, 10, 2, 64, 128, 1, 2, 0, kind=0, relu=False, seed=83),  # 1x1 stride-2 downsample
     Case(2, 7, 9, 4, 128, 96, 1, 1, 0, seed=84),                      # flat mode, ragged last tile
     Case(2, 14, 14, 8, 64, 32, 3, 1, 1, kind=3, perm=(3, 0, 7, 1, 6, 2, 5, 4), seed=85),
@@ -492,6 +493,7 @@ F4_CASES = [
     Case(2, 20, 42, 2, 128, 64, 3, 1, 1, seed=98),                    # three accumulators, two K steps
     Case(2, 20, 20, 2, 64, 64, 1, 1, 0, seed=99),                     # flat, two boxes per tile
     Case(2, 17, 17, 2, 128, 64, 1, 1, 0, seed=100),                   # flat, second box wholly past the image
+    Case(1, 6, 140, 2, 64, 32, 3, 2, 1, seed=101),                    # stride 2, window wider than one TMA box row
 ]
 
 
