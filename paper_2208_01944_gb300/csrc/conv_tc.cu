@@ -926,6 +926,157 @@ __device__ __forceinline__ void epi_general16(const ConvParams& p, const EpiItem
   }
 }
 
+// General units (int32 sums, fp32 outputs with or without the shortcut, codes)
+// of UC accumulator columns.  TMEM gives each lane one row (pixel), but a global
+// access instruction costs about one cycle per cache line it touches, so rows
+// of 4 UC bytes per lane would cost 32 lines per instruction.  The shortcut,
+// the fp32 outputs and the int32 sums therefore pass through the warp's staging
+// buffer (32 rows of 4 UC bytes; 16-byte chunk c of row r at chunk c ^ sw(r),
+// which keeps both access patterns conflict-free): a global access instruction
+// takes whole rows, 512 bytes in 4 rows of 128 (UC = 32) or 8 rows of 64
+// (UC = 16), and each lane reads or writes its own row in shared memory.  The shortcut comes by
+// cp.async (zero-filled for rows outside the output).  Codes go through the
+// fp16 conversion (epi_codes16_f16) where no NaN can reach it: without a
+// shortcut the value is fl(raw * m_req * 2^-15) = fl(acc * m_req) * 2^-24; with
+// one, fl(y * m_req * 2^-24) = fl(y * m_req) * 2^-24 (a power-of-two factor,
+// exact while the product is normal; both give code 0 below that), and ReLU has
+// removed NaN (fmaxf(NaN, 0) = 0).  A shortcut without ReLU keeps the scalar
+// form, which maps NaN to code 0.
+template <int UC>
+__device__ __forceinline__ uint32_t stg_chunk(uint32_t base, int r, int c) {
+  constexpr int CPR = UC / 4;  // 16-byte chunks per staged row
+  const int sw = (UC == 32 ? r : r >> 1) & (CPR - 1);
+  return base + static_cast<uint32_t>(r * (UC * 4) + ((c ^ sw) << 4));
+}
+
+template <int UC>
+__device__ __forceinline__ void epi_general_units(const ConvParams& p, const EpiItem& e, uint8_t* stg, int wg,
+                                                  int n_groups, int quarter, int lane, uint32_t qmax2) {
+  constexpr int CPR = UC / 4, RPP = 32 / CPR;  // chunks per row, rows per coalesced pass
+  const uint32_t sbase = smem_u32(stg);
+  const bool has_sc = p.shortcut != nullptr;
+  const bool f16q = !has_sc || p.relu;
+  const float m_q = has_sc ? __fmul_rn(e.m_req, 1.0f / 16777216.0f) : e.m_req15;
+  const int qmax = p.qmax_out;
+  const float qmax_f = static_cast<float>(qmax);
+  const int m_lane = quarter * 32 + lane;
+  const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
+  const int per_acc = p.Nblk / UC;
+  const int n_units = p.MT * per_acc;
+  const int pr = lane / CPR, pc = lane % CPR;  // row within a pass, chunk: coalesced role
+  for (int u = wg; u < n_units; u += n_groups) {
+    const int mt = u / per_acc, col0 = (u - mt * per_acc) * UC;
+    bool valid;
+    const int pos = epi_pos(p, e, mt * 128 + m_lane, valid);
+    const long long rowc = valid ? (static_cast<long long>(e.n) * hw_out + pos) * p.C_out_total : -1;
+    uint32_t v[UC];
+    if constexpr (UC == 32)
+      tmem_ld32(e.tbase + mt * p.Npow2 + col0, v);
+    else
+      tmem_ld16(e.tbase + mt * p.Npow2 + col0, v);
+    // Whole staged rows to global memory (row r's element offset is lane r's rowc).
+    auto store_rows = [&](void* out, int c0) {
+      __syncwarp();
+#pragma unroll
+      for (int ps = 0; ps < CPR; ++ps) {
+        const int r = ps * RPP + pr;
+        const long long off = __shfl_sync(0xffffffffu, rowc, r);
+        uint32_t x0, x1, x2, x3;
+        asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(x0), "=r"(x1), "=r"(x2), "=r"(x3)
+                     : "r"(stg_chunk<UC>(sbase, r, pc))
+                     : "memory");
+        if (off >= 0)
+          *reinterpret_cast<uint4*>(reinterpret_cast<uint32_t*>(out) + off + c0 + col0 + 4 * pc) =
+              make_uint4(x0, x1, x2, x3);
+      }
+      __syncwarp();
+    };
+    // This lane's row of UC 32-bit values into the staging buffer.
+    auto stage_row = [&](const uint32_t (&x)[UC]) {
+#pragma unroll
+      for (int c = 0; c < CPR; ++c)
+        asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(stg_chunk<UC>(sbase, lane, c)), "r"(x[4 * c]),
+                     "r"(x[4 * c + 1]), "r"(x[4 * c + 2]), "r"(x[4 * c + 3])
+                     : "memory");
+    };
+    if (p.acc_out) {
+      tmem_wait_ld();
+      uint32_t a[UC];
+#pragma unroll
+      for (int j = 0; j < UC; ++j) a[j] = static_cast<uint32_t>(__float2int_rn(__fmul_rn(__uint_as_float(v[j]), 512.0f)));
+      __syncwarp();
+      stage_row(a);
+      store_rows(p.acc_out, e.dst_c0);
+    }
+    if (has_sc) {
+      // the rows' shortcut values (the unit's source channels) into the staging buffer
+#pragma unroll
+      for (int ps = 0; ps < CPR; ++ps) {
+        const int r = ps * RPP + pr;
+        const long long off = __shfl_sync(0xffffffffu, rowc, r);
+        cp_async_16(stg_chunk<UC>(sbase, r, pc), off >= 0 ? p.shortcut + off + e.src_c0 + col0 + 4 * pc : p.shortcut,
+                    off >= 0 ? 16u : 0u);
+      }
+      cp_async_commit();
+      cp_async_wait<0>();
+      __syncwarp();
+    }
+    tmem_wait_ld();
+    uint4 w[UC / 16];
+    if (p.q_out && !has_sc) {
+      w[0] = epi_codes16_f16<UC, 0>(v, m_q, qmax2);
+      if constexpr (UC == 32) w[1] = epi_codes16_f16<UC, 16>(v, m_q, qmax2);
+    }
+    // y = relu(fl(acc * m_out) + shortcut), in place
+#pragma unroll
+    for (int c = 0; c < CPR; ++c) {
+      float sc0 = 0.0f, sc1 = 0.0f, sc2 = 0.0f, sc3 = 0.0f;
+      if (has_sc)
+        asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];"
+                     : "=f"(sc0), "=f"(sc1), "=f"(sc2), "=f"(sc3)
+                     : "r"(stg_chunk<UC>(sbase, lane, c))
+                     : "memory");
+      const float scv[4] = {sc0, sc1, sc2, sc3};
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        float t = __fmul_rn(__uint_as_float(v[4 * c + k]), e.m_out512);  // = (float)acc * m_out, one rounding
+        if (has_sc) t = __fadd_rn(t, scv[k]);
+        if (p.relu) t = fmaxf(t, 0.0f);
+        v[4 * c + k] = __float_as_uint(t);
+      }
+    }
+    if (p.q_out && has_sc) {
+      if (f16q) {
+        w[0] = epi_codes16_f16<UC, 0>(v, m_q, qmax2);
+        if constexpr (UC == 32) w[1] = epi_codes16_f16<UC, 16>(v, m_q, qmax2);
+      } else {
+#pragma unroll
+        for (int h = 0; h < UC / 16; ++h) {
+          int code[16];
+#pragma unroll
+          for (int j = 0; j < 16; ++j)
+            code[j] = requant_code(__fmul_rn(__uint_as_float(v[16 * h + j]), e.m_req), qmax_f, qmax);
+          w[h].x = __byte_perm(__byte_perm(code[0], code[1], 0x0040), __byte_perm(code[2], code[3], 0x0040), 0x5410);
+          w[h].y = __byte_perm(__byte_perm(code[4], code[5], 0x0040), __byte_perm(code[6], code[7], 0x0040), 0x5410);
+          w[h].z = __byte_perm(__byte_perm(code[8], code[9], 0x0040), __byte_perm(code[10], code[11], 0x0040), 0x5410);
+          w[h].w = __byte_perm(__byte_perm(code[12], code[13], 0x0040), __byte_perm(code[14], code[15], 0x0040), 0x5410);
+        }
+      }
+    }
+    if (p.y_out) {
+      __syncwarp();  // every lane has read its shortcut row
+      stage_row(v);
+      store_rows(p.y_out, e.dst_c0);
+    }
+    if (p.q_out) {
+      __syncwarp();
+#pragma unroll
+      for (int h = 0; h < UC / 16; ++h) epi_store_codes(p, e, stg, lane, valid, pos, col0 / 16 + h, w[h]);
+    }
+  }
+}
+
 // The epilogue's work per tile is a list of units, one per (accumulator mt,
 // 16-column chunk); epilogue warpgroup wg of n_groups takes units wg,
 // wg + n_groups, ...  Each warp handles the 32 TMEM lanes (rows) it may access.
@@ -1084,86 +1235,10 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         c_ch = n_ch;
       }
     } else if (!p.channel_shuffle) {
-      // General units (int32 sums, fp32 outputs with or without the shortcut,
-      // codes): lane r's 16 values of a unit are 64 contiguous bytes of its
-      // pixel's NHWC row, loaded and stored straight from registers.  The codes
-      // go through the fp16 conversion (epi_codes16_f16) where no NaN can reach
-      // it: without a shortcut the value is fl(raw * m_req * 2^-15) =
-      // fl(acc * m_req) * 2^-24; with one, fl(y * m_req * 2^-24) =
-      // fl(y * m_req) * 2^-24 (a power-of-two factor, exact while the product is
-      // normal, and both round to code 0 below that), and ReLU has removed NaN
-      // (fmaxf(NaN, 0) = 0).  A shortcut without ReLU keeps the scalar form,
-      // which maps NaN to code 0.
-      const bool has_sc = p.shortcut != nullptr;
-      const bool f16q = !has_sc || p.relu;
-      const float m_q = has_sc ? __fmul_rn(e.m_req, 1.0f / 16777216.0f) : e.m_req15;
-      const int qmax = p.qmax_out;
-      const float qmax_f = static_cast<float>(qmax);
-      const int m_lane = quarter * 32 + lane;
-      const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
-      for (int u = wg; u < n_units; u += n_groups) {
-        const int mt = u / nchunks, ch = u - mt * nchunks;
-        bool valid;
-        const int pos = epi_pos(p, e, mt * 128 + m_lane, valid);
-        const long long rowc = (static_cast<long long>(e.n) * hw_out + pos) * p.C_out_total;
-        uint32_t v[16];
-        tmem_ld16(e.tbase + mt * p.Npow2 + ch * 16, v);
-        float sc[16];
-        if (has_sc) {
-          if (valid) {
-            const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + rowc + e.src_c0 + ch * 16);
-#pragma unroll
-            for (int j = 0; j < 4; ++j) {
-              const float4 t = s4[j];
-              sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
-            }
-          } else {
-#pragma unroll
-            for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
-          }
-        }
-        tmem_wait_ld();
-        uint32_t y[16];
-#pragma unroll
-        for (int j = 0; j < 16; ++j) {
-          float t = __fmul_rn(__uint_as_float(v[j]), e.m_out512);  // = (float)acc * m_out, one rounding
-          if (has_sc) t = __fadd_rn(t, sc[j]);
-          if (p.relu) t = fmaxf(t, 0.0f);
-          y[j] = __float_as_uint(t);
-        }
-        if (valid) {
-          const long long o = rowc + e.dst_c0 + ch * 16;
-          if (p.acc_out) {
-            int4* a4 = reinterpret_cast<int4*>(p.acc_out + o);
-#pragma unroll
-            for (int j = 0; j < 16; j += 4)
-              a4[j >> 2] = make_int4(__float2int_rn(__fmul_rn(__uint_as_float(v[j]), 512.0f)),
-                                     __float2int_rn(__fmul_rn(__uint_as_float(v[j + 1]), 512.0f)),
-                                     __float2int_rn(__fmul_rn(__uint_as_float(v[j + 2]), 512.0f)),
-                                     __float2int_rn(__fmul_rn(__uint_as_float(v[j + 3]), 512.0f)));
-          }
-          if (p.y_out) {
-            uint4* y4 = reinterpret_cast<uint4*>(p.y_out + o);
-#pragma unroll
-            for (int j = 0; j < 16; j += 4) y4[j >> 2] = make_uint4(y[j], y[j + 1], y[j + 2], y[j + 3]);
-          }
-        }
-        if (p.q_out) {
-          uint4 w;
-          if (f16q) {
-            w = epi_codes16_f16(has_sc ? y : v, m_q, qmax2);
-          } else {
-            int code[16];
-#pragma unroll
-            for (int j = 0; j < 16; ++j) code[j] = requant_code(__fmul_rn(__uint_as_float(y[j]), e.m_req), qmax_f, qmax);
-            w.x = __byte_perm(__byte_perm(code[0], code[1], 0x0040), __byte_perm(code[2], code[3], 0x0040), 0x5410);
-            w.y = __byte_perm(__byte_perm(code[4], code[5], 0x0040), __byte_perm(code[6], code[7], 0x0040), 0x5410);
-            w.z = __byte_perm(__byte_perm(code[8], code[9], 0x0040), __byte_perm(code[10], code[11], 0x0040), 0x5410);
-            w.w = __byte_perm(__byte_perm(code[12], code[13], 0x0040), __byte_perm(code[14], code[15], 0x0040), 0x5410);
-          }
-          epi_store_codes(p, e, stg, lane, valid, pos, ch, w);
-        }
-      }
+      if ((p.Nblk & 31) == 0)
+        epi_general_units<32>(p, e, stg, wg, n_groups, quarter, lane, qmax2);
+      else
+        epi_general_units<16>(p, e, stg, wg, n_groups, quarter, lane, qmax2);
     } else {
       // The channel shuffle's per-channel scatter (rarely used).
       const int m_lane = quarter * 32 + lane;
