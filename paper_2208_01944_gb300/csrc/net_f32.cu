@@ -103,130 +103,156 @@ __device__ __forceinline__ void fma2_rn(float& d0, float& d1, float a, float b0,
       : "f"(a), "f"(b0), "f"(b1));
 }
 
-// The 7x7 stride-2 convolution of a 3-channel image (the network's first layer),
-// for Cout = 16 * CG channels (CG <= 8).  A block computes an output tile of
-// 8 rows x 16 columns: warp w takes channels [16 w, 16 w + 16) and lane l the
-// 4 consecutive pixels (row l / 4, columns 4 (l % 4) .. + 3), so the 16 weights
-// of a term are one broadcast read.  The input tile (21 x 37 x 3 floats, zero
-// outside the image) and all weights ([147][Cout]) sit in shared memory; the next
-// tile's input is copied asynchronously while the current one is computed.
-// Per output the terms are added in (kh, kw, ci) order like the generic kernel;
-// the zero taps outside the image change nothing: fma(0, w, acc) = acc for
-// finite w, since a sum started at +0 is never -0 under round-to-nearest.
-constexpr int kStemK = 7, kStemS = 2, kStemP = 3, kStemCin = 3;
+// The 7x7 stride-2 convolution of a 3-channel image to 128 channels (the
+// network's first layer).  A block of 256 threads computes an output tile of
+// 8 rows x 16 columns; thread (pixel group p, channel group g) the 8
+// consecutive pixels 8 (p % 2) .. + 7 of row p / 2 and the 8 channels
+// 8 g .. 8 g + 7: 64 sums, so that a term costs two 16-byte loads of inputs,
+// two of weights and 32 packed FMAs.  The input tile (21 x 37 x 3 floats, zero
+// outside the image) is held split by column parity, channel-planar, in four
+// copies shifted by 0..3 positions: copy s of parity b holds at row r, position
+// k the tile's column 2 (k + s) + b, so the 8 inputs of a thread for tap
+// (kh, kw) are positions 8 (p % 2) .. + 7, aligned, of copy kw / 2, parity
+// kw % 2, row 2 (p / 2) + kh.  The weights of a term are stored as two halves of
+// 4 channels per group ([147][2][16][4]), so that the 16 groups of a warp read
+// 256 contiguous bytes.  The next tile's inputs are loaded into registers while
+// the current one's outputs are stored, and the two CTAs of an SM take turns at
+// the barriers.  Per output the terms are added in (kh, kw, ci) order like the
+// generic kernel; the zero taps outside the image change nothing:
+// fma(0, w, acc) = acc for finite w, since a sum started at +0 is never -0
+// under round-to-nearest.
+constexpr int kStemK = 7, kStemS = 2, kStemP = 3, kStemCin = 3, kStemCout = 128;
 constexpr int kStemTH = 8, kStemTW = 16;
-constexpr int kStemIR = (kStemTH - 1) * kStemS + kStemK;  // 21
-constexpr int kStemIC = (kStemTW - 1) * kStemS + kStemK;  // 37
+constexpr int kStemThreads = 256;
+constexpr int kStemIR = (kStemTH - 1) * kStemS + kStemK;  // 21 input rows
+constexpr int kStemIC = (kStemTW - 1) * kStemS + kStemK;  // 37 input columns
 constexpr int kStemTerms = kStemK * kStemK * kStemCin;    // 147
+constexpr int kStemRowF = 16;                             // positions per copy row
+constexpr int kStemPlaneF = kStemIR * kStemRowF;          // one (copy, parity, channel) plane
+constexpr int kStemCopyF = 2 * kStemCin * kStemPlaneF;    // one shifted copy
+constexpr int kStemXFloats = 4 * kStemCopyF;
+constexpr int kStemTileElems = kStemIR * kStemIC * kStemCin;                     // 2331
+constexpr int kStemLoads = (kStemTileElems + kStemThreads - 1) / kStemThreads;  // 10 per thread
+constexpr size_t kStemSmem = (static_cast<size_t>(kStemTerms) * kStemCout + kStemXFloats) * sizeof(float);
 
-__device__ __forceinline__ void cp_async4(float* dst, const float* src, bool valid) {
-  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
-  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(d), "l"(src), "r"(valid ? 4 : 0) : "memory");
-}
-
-__global__ void __launch_bounds__(256, 2) pq_stem7x7s2_kernel(const float* __restrict__ x, const float* __restrict__ w,
-                                                           float* __restrict__ y, int64_t N, int H, int W, int Cout,
-                                                           int Ho, int Wo, int relu) {
-  extern __shared__ float smem[];
-  constexpr int kTileFloats = kStemIR * kStemIC * kStemCin;
-  float* ws = smem;                          // [147][Cout]
-  float* xs0 = smem + kStemTerms * Cout;     // two input tiles [21][37][3]
+__global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const float* __restrict__ x,
+                                                                     const float* __restrict__ w,
+                                                                     float* __restrict__ y, int64_t N, int H, int W,
+                                                                     int Ho, int Wo, int relu) {
+  extern __shared__ float4 smem4[];
+  float* ws = reinterpret_cast<float*>(smem4);  // [147][2][16][4]
+  float* xs = ws + kStemTerms * kStemCout;      // [copy 4][parity 2][ci 3][row 21][16]
   const int tiles_h = (Ho + kStemTH - 1) / kStemTH, tiles_w = (Wo + kStemTW - 1) / kStemTW;
   const int64_t n_tiles = N * tiles_h * tiles_w;
-  // Input tile t into buffer b with 4-byte asynchronous copies; taps outside the
-  // image are zero-filled (source size 0).
-  auto load_tile = [&](int64_t t, int b) {
+  float pre[kStemLoads];
+  // Global loads of tile t's inputs (element i = (row, column, channel) of the
+  // 21 x 37 x 3 window, i = threadIdx.x + 256 e), zero outside the image.
+  auto fetch = [&](int64_t t) {
     const int tw = static_cast<int>(t % tiles_w);
     const int64_t r = t / tiles_w;
     const int th = static_cast<int>(r % tiles_h);
     const int64_t n = r / tiles_h;
     const int ih0 = th * kStemTH * kStemS - kStemP, iw0 = tw * kStemTW * kStemS - kStemP;
-    float* xs = xs0 + b * kTileFloats;
-    for (int i = threadIdx.x; i < kTileFloats; i += blockDim.x) {
-      const int ci = i % kStemCin;
-      const int rc = i / kStemCin;
-      const int c = rc % kStemIC, rr = rc / kStemIC;
+#pragma unroll
+    for (int e = 0; e < kStemLoads; ++e) {
+      const int i = threadIdx.x + e * kStemThreads;
+      const int rr = i / (kStemIC * kStemCin), rem = i - rr * (kStemIC * kStemCin);
+      const int c = rem / kStemCin, ci = rem - c * kStemCin;
       const int ih = ih0 + rr, iw = iw0 + c;
-      const bool valid = ih >= 0 && ih < H && iw >= 0 && iw < W;
-      cp_async4(xs + i, valid ? x + ((n * H + ih) * W + iw) * kStemCin + ci : x, valid);
+      const bool valid = i < kStemTileElems && ih >= 0 && ih < H && iw >= 0 && iw < W;
+      pre[e] = valid ? x[((n * H + ih) * W + iw) * kStemCin + ci] : 0.0f;
     }
-    asm volatile("cp.async.commit_group;" ::: "memory");
+  };
+  // The fetched window into the four shifted copies of its parity planes.
+  auto scatter = [&]() {
+#pragma unroll
+    for (int e = 0; e < kStemLoads; ++e) {
+      const int i = threadIdx.x + e * kStemThreads;
+      if (i < kStemTileElems) {
+        const int rr = i / (kStemIC * kStemCin), rem = i - rr * (kStemIC * kStemCin);
+        const int c = rem / kStemCin, ci = rem - c * kStemCin;
+        const int k0 = c >> 1;
+        float* dst = xs + ((c & 1) * kStemCin + ci) * kStemPlaneF + rr * kStemRowF + k0;
+#pragma unroll
+        for (int sh = 0; sh < 4; ++sh)
+          if (k0 - sh >= 0 && k0 - sh < kStemRowF) dst[sh * kStemCopyF - sh] = pre[e];
+      }
+    }
   };
   int64_t t = blockIdx.x;
-  if (t < n_tiles) load_tile(t, 0);
-  // transposed to [term][Cout]: consecutive threads write consecutive words
-  // (conflict-free) and gather from the [Cout][term] weights through L2
-  for (int i = threadIdx.x; i < kStemTerms * Cout; i += blockDim.x) {
-    const int r = i / Cout, co = i - r * Cout;
-    ws[i] = w[co * kStemTerms + r];
+  if (t < n_tiles) fetch(t);
+  // weights [Cout][147] to [147][2][16][4]: channel co = 8 g + 4 h + k at
+  // term * 128 + h * 64 + g * 4 + k (consecutive threads write consecutive words)
+  for (int i = threadIdx.x; i < kStemTerms * kStemCout; i += kStemThreads) {
+    const int term = i >> 7, rem = i & 127;
+    const int h = rem >> 6, g = (rem >> 2) & 15, k = rem & 3;
+    ws[i] = w[(g * 8 + h * 4 + k) * kStemTerms + term];
   }
-  const int cg = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int ohl = lane >> 2, owl = (lane & 3) * 4;
-  const float* wcol = ws + cg * 16;
-  int buf = 0;
-  for (; t < n_tiles; t += gridDim.x, buf ^= 1) {
-    __syncthreads();  // every thread is done with the buffer the next load overwrites
-    if (t + gridDim.x < n_tiles) {
-      load_tile(t + gridDim.x, buf ^ 1);
-      asm volatile("cp.async.wait_group 1;" ::: "memory");
-    } else {
-      asm volatile("cp.async.wait_group 0;" ::: "memory");
-    }
-    __syncthreads();  // tile t (and the weights) visible to all threads
+  const int cg = threadIdx.x & 15, pg = threadIdx.x >> 4;
+  const int ohl = pg >> 1, q = pg & 1;
+  const float* xthr = xs + (2 * ohl) * kStemRowF + 8 * q;
+  const float* wthr = ws + cg * 4;
+  for (; t < n_tiles; t += gridDim.x) {
+    __syncthreads();  // every thread is done with the copies of the previous tile
+    scatter();
+    __syncthreads();  // the copies (and, the first time, the weights) visible to all threads
     const int tw = static_cast<int>(t % tiles_w);
     const int64_t r = t / tiles_w;
     const int th = static_cast<int>(r % tiles_h);
     const int64_t n = r / tiles_h;
-    const int oh0 = th * kStemTH, ow0 = tw * kStemTW;
-    float acc[4][16];
+    float acc[8][8];
 #pragma unroll
-    for (int j = 0; j < 4; ++j)
+    for (int j = 0; j < 8; ++j)
 #pragma unroll
-      for (int c = 0; c < 16; ++c) acc[j][c] = 0.0f;
-    const float* xrow = xs0 + buf * kTileFloats + ((ohl * kStemS) * kStemIC + owl * kStemS) * kStemCin;
+      for (int c = 0; c < 8; ++c) acc[j][c] = 0.0f;
 #pragma unroll 1
     for (int kh = 0; kh < kStemK; ++kh) {
+      const float* xk = xthr + kh * kStemRowF;
+      const float* wk = wthr + kh * (kStemK * kStemCin) * kStemCout;
 #pragma unroll
       for (int kw = 0; kw < kStemK; ++kw) {
 #pragma unroll
         for (int ci = 0; ci < kStemCin; ++ci) {
-          const int term = (kh * kStemK + kw) * kStemCin + ci;
-          const float4* w4 = reinterpret_cast<const float4*>(wcol + term * Cout);
-          const float4 wa = w4[0], wb = w4[1], wc = w4[2], wd = w4[3];
-          const float wv[16] = {wa.x, wa.y, wa.z, wa.w, wb.x, wb.y, wb.z, wb.w,
-                                wc.x, wc.y, wc.z, wc.w, wd.x, wd.y, wd.z, wd.w};
+          const float4* xp =
+              reinterpret_cast<const float4*>(xk + (kw >> 1) * kStemCopyF + ((kw & 1) * kStemCin + ci) * kStemPlaneF);
+          const float4 xa = xp[0], xb = xp[1];
+          const float* wt = wk + (kw * kStemCin + ci) * kStemCout;
+          const float4 wa = *reinterpret_cast<const float4*>(wt), wb = *reinterpret_cast<const float4*>(wt + 64);
+          const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
 #pragma unroll
-          for (int j = 0; j < 4; ++j) {
-            const float xv = xrow[(kh * kStemIC + kw + j * kStemS) * kStemCin + ci];
-#pragma unroll
-            for (int c = 0; c < 16; c += 2) fma2_rn(acc[j][c], acc[j][c + 1], xv, wv[c], wv[c + 1]);
+          for (int j = 0; j < 8; ++j) {
+            fma2_rn(acc[j][0], acc[j][1], xv[j], wa.x, wa.y);
+            fma2_rn(acc[j][2], acc[j][3], xv[j], wa.z, wa.w);
+            fma2_rn(acc[j][4], acc[j][5], xv[j], wb.x, wb.y);
+            fma2_rn(acc[j][6], acc[j][7], xv[j], wb.z, wb.w);
           }
         }
       }
     }
-    const int oh = oh0 + ohl;
+    // the next tile's loads are in flight while this one's outputs are stored
+    if (t + gridDim.x < n_tiles) fetch(t + gridDim.x);
+    const int oh = th * kStemTH + ohl;
     if (oh < Ho) {
 #pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const int ow = ow0 + owl + j;
+      for (int j = 0; j < 8; ++j) {
+        const int ow = tw * kStemTW + 8 * q + j;
         if (ow < Wo) {
-          float4* yp = reinterpret_cast<float4*>(y + ((n * Ho + oh) * Wo + ow) * Cout + cg * 16);
+          float4* yp = reinterpret_cast<float4*>(y + ((n * Ho + oh) * Wo + ow) * kStemCout + cg * 8);
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            float4 o = make_float4(acc[j][4 * q], acc[j][4 * q + 1], acc[j][4 * q + 2], acc[j][4 * q + 3]);
+          for (int h = 0; h < 2; ++h) {
+            float4 o = make_float4(acc[j][4 * h], acc[j][4 * h + 1], acc[j][4 * h + 2], acc[j][4 * h + 3]);
             if (relu) {
               o.x = fmaxf(o.x, 0.0f);
               o.y = fmaxf(o.y, 0.0f);
               o.z = fmaxf(o.z, 0.0f);
               o.w = fmaxf(o.w, 0.0f);
             }
-            yp[q] = o;
+            yp[h] = o;
           }
         }
       }
     }
   }
-  asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
 
 // Max over the in-image taps of each window, fmaxf in (kh, kw) order from -inf.
@@ -367,14 +393,12 @@ pq_status palquant_conv2d_f32(const float* x_dev, const float* w_dev, float* y_d
   const int64_t wbytes = static_cast<int64_t>(k) * k * Cin * Cout * 4;
   const int64_t work = N * Ho * Wo * (Cout / pq::kCoT);
   auto s = static_cast<cudaStream_t>(stream);
-  const size_t stem_smem =
-      static_cast<size_t>(pq::kStemTerms * Cout + 2 * pq::kStemIR * pq::kStemIC * pq::kStemCin) * sizeof(float);
-  if (k == pq::kStemK && stride == pq::kStemS && pad == pq::kStemP && Cin == pq::kStemCin && Cout <= 128 &&
-      stem_smem <= 200 * 1024) {
+  if (k == pq::kStemK && stride == pq::kStemS && pad == pq::kStemP && Cin == pq::kStemCin && Cout == pq::kStemCout &&
+      pq::aligned16(y_dev)) {
     static bool stem_attr = false;
     if (!stem_attr) {
-      if (cudaFuncSetAttribute(pq::pq_stem7x7s2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024) !=
-          cudaSuccess)
+      if (cudaFuncSetAttribute(pq::pq_stem7x7s2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               static_cast<int>(pq::kStemSmem)) != cudaSuccess)
         return PQ_ECUDA;
       stem_attr = true;
     }
@@ -382,10 +406,9 @@ pq_status palquant_conv2d_f32(const float* x_dev, const float* w_dev, float* y_d
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const int per_sm = stem_smem <= 100 * 1024 ? 2 : 1;
-    const unsigned grid = static_cast<unsigned>(tiles < static_cast<int64_t>(sms) * per_sm ? tiles : sms * per_sm);
-    pq::pq_stem7x7s2_kernel<<<grid, 32 * (Cout / 16), stem_smem, s>>>(x_dev, w_dev, y_dev, N, H, W, Cout,
-                                                                       static_cast<int>(Ho), static_cast<int>(Wo), relu);
+    const unsigned grid = static_cast<unsigned>(tiles < static_cast<int64_t>(sms) * 2 ? tiles : sms * 2);
+    pq::pq_stem7x7s2_kernel<<<grid, pq::kStemThreads, pq::kStemSmem, s>>>(
+        x_dev, w_dev, y_dev, N, H, W, static_cast<int>(Ho), static_cast<int>(Wo), relu);
     return cudaGetLastError() == cudaSuccess ? PQ_OK : PQ_ECUDA;
   }
   if (wbytes <= 96 * 1024) {
