@@ -412,6 +412,20 @@ pq_status palquant_conv2d_f32(const float* x_dev, const float* w_dev, float* y_d
                               int32_t Cin, int32_t Cout, int32_t k, int32_t stride, int32_t pad, int32_t relu,
                               pq_stream_t stream);
 
+/* The network's first layer and the pooling after it in one pass (Sec. 5 keeps
+ * the first layer in full precision): stem = max(conv2d_f32(x, w, stride 2,
+ * pad 3, 7 x 7), 0) exactly as palquant_conv2d_f32 with relu computes it, and
+ * pool = palquant_maxpool2d_f32(stem, 3 x 3, stride 2, pad 1).  x NHWC
+ * [N,H,W,3], w [Cout][7][7][3], pool NHWC [N,Hp,Wp,Cout] with Ho = (H - 1) / 2 + 1,
+ * Hp = (Ho - 1) / 2 + 1 (likewise W); stem_dev, NHWC [N,Ho,Wo,Cout], may be NULL
+ * (the stem output is then never written to memory).  Outputs 16-byte aligned.
+ * The call zeroes pool on the stream first (windows that span two tiles of the
+ * kernel are combined by atomic maxima); the result is exact, so it equals the
+ * two separate calls bit for bit.  Cout must be 128 (PQ_EUNSUPPORTED otherwise:
+ * use the two calls); PQ_EINVAL on bad sizes or pointers. */
+pq_status palquant_stem_pool_f32(const float* x_dev, const float* w_dev, float* stem_dev, float* pool_dev, int64_t N,
+                                 int32_t H, int32_t W, int32_t Cout, pq_stream_t stream);
+
 /* Max pooling, NHWC: y[n,oh,ow,c] = max over the in-image taps of the k x k
  * window at (oh*stride - pad, ow*stride - pad) (padding taps are ignored);
  * pad < k. */

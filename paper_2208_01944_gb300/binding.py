@@ -30,7 +30,8 @@ EXPORTS = [
     "palquant_unpack_weight_codes_host", "palquant_quantize_act", "palquant_group_conv", "palquant_layer_fused",
     "palquant_quantize_layer_fused",
     "palquant_sync_check", "palquant_set_wait_limit_ns", "palquant_watchdog_selftest", "palquant_conv_plan",
-    "palquant_conv2d_f32", "palquant_maxpool2d_f32", "palquant_avgpool_f32", "palquant_linear_f32",
+    "palquant_conv2d_f32", "palquant_stem_pool_f32", "palquant_maxpool2d_f32", "palquant_avgpool_f32",
+    "palquant_linear_f32",
     "palquant_cyclic_shuffle_module", "palquant_bitsplit_desc", "palquant_bitsplit_scratch_bytes",
     "palquant_bitsplit_pack_weight_codes_host", "palquant_bitsplit_act", "palquant_bitsplit_conv",
     "palquant_pack_weights_odd_host", "palquant_fake_quant_forward", "palquant_fake_quant_scratch_bytes",
@@ -129,6 +130,7 @@ def _load():
     L.palquant_cyclic_shuffle_module.restype = _I32
     L.palquant_cyclic_shuffle_module.argtypes = [_P, _P, ctypes.POINTER(LayerDesc), _P, _P, _I32, _P, _P, _P, _P]
     for name, args in (("palquant_conv2d_f32", [_P, _P, _P, _I64] + [_I32] * 8 + [_P]),
+                       ("palquant_stem_pool_f32", [_P, _P, _P, _P, _I64, _I32, _I32, _I32, _P]),
                        ("palquant_maxpool2d_f32", [_P, _P, _I64] + [_I32] * 6 + [_P]),
                        ("palquant_avgpool_f32", [_P, _P, _I64, _I32, _I32, _I32, _P]),
                        ("palquant_linear_f32", [_P, _P, _P, _I64, _I32, _I32, _P])):
@@ -350,6 +352,12 @@ def palquant_conv_plan(d: LayerDesc) -> ConvPlan:
 def palquant_conv2d_f32(x_dev, w_dev, y_dev, N, H, W, Cin, Cout, k, stride, pad, relu=False, stream=None):
     _check(lib.palquant_conv2d_f32(_ptr(x_dev), _ptr(w_dev), _ptr(y_dev), N, H, W, Cin, Cout, k, stride, pad,
                                    int(bool(relu)), _stream(stream)), "palquant_conv2d_f32")
+
+
+def palquant_stem_pool_f32(x_dev, w_dev, stem_dev, pool_dev, N, H, W, Cout, stream=None):
+    """7x7/2 stem + ReLU and 3x3/2 max pooling in one pass; stem_dev may be None."""
+    _check(lib.palquant_stem_pool_f32(_ptr(x_dev), _ptr(w_dev), _ptr(stem_dev) if stem_dev is not None else None,
+                                      _ptr(pool_dev), N, H, W, Cout, _stream(stream)), "palquant_stem_pool_f32")
 
 
 def palquant_maxpool2d_f32(x_dev, y_dev, N, H, W, C, k, stride, pad, stream=None):

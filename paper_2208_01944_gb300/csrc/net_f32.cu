@@ -135,10 +135,88 @@ constexpr int kStemTileElems = kStemIR * kStemIC * kStemCin;                    
 constexpr int kStemLoads = (kStemTileElems + kStemThreads - 1) / kStemThreads;  // 10 per thread
 constexpr size_t kStemSmem = (static_cast<size_t>(kStemTerms) * kStemCout + kStemXFloats) * sizeof(float);
 
+// 3x3 stride-2 pad-1 max pooling of the stem tile held in registers (ReLU
+// outputs, so every value is >= 0, and pixels outside the output are 0).
+// Pooled row pr (0..4) of the tile covers stem rows 2 pr - 1 .. 2 pr + 1 and
+// pooled column pc (0..8) stem columns 2 pc - 1 .. 2 pc + 1 (tile-relative).
+// Columns: each thread reduces its 8 pixels to the windows it sees (slots
+// s = 0..4, pooled column 4 q + s) and the pixel-half q = 0 takes q = 1's part of
+// pooled column 4 by a shuffle.  Rows: warp w holds stem row w; the odd rows go
+// through shared memory (the input copies' space, free after the FMAs) to the
+// even warps, which complete pooled rows 1..3.  Windows that reach into a
+// neighbouring tile (pooled row 0 and 4, pooled column 0 and 8) are combined
+// across tiles by an integer atomic maximum on the float bits (the order of
+// non-negative floats), into an output the launcher zeroed; the others are
+// stored.  The maximum is exact, so the result does not depend on the order.
+__device__ __forceinline__ void stem_pool_tile(const float (&acc)[8][8], float* xs, float* __restrict__ pool, int64_t n,
+                                               int th, int tw, int ohl, int q, int cg, int Hp, int Wp) {
+  float h[5][8];
+#pragma unroll
+  for (int c = 0; c < 8; ++c) {
+    h[0][c] = fmaxf(acc[0][c], acc[1][c]);
+    h[1][c] = fmaxf(fmaxf(acc[1][c], acc[2][c]), acc[3][c]);
+    h[2][c] = fmaxf(fmaxf(acc[3][c], acc[4][c]), acc[5][c]);
+    h[3][c] = fmaxf(fmaxf(acc[5][c], acc[6][c]), acc[7][c]);
+    h[4][c] = acc[7][c];
+    const float other = __shfl_xor_sync(0xffffffffu, h[0][c], 16);  // q = 1's columns 8, 9 of the tile
+    if (q == 0) h[4][c] = fmaxf(h[4][c], other);
+  }
+  constexpr int kRowF = 9 * kStemCout;  // one staged row: 9 pooled columns x 128 channels
+  __syncthreads();                      // every warp is done reading the input copies
+  if (ohl & 1) {
+#pragma unroll
+    for (int sl = 0; sl < 5; ++sl) {
+      if (q == 1 && sl == 0) continue;
+      float4* d = reinterpret_cast<float4*>(xs + (ohl >> 1) * kRowF + (4 * q + sl) * kStemCout + cg * 8);
+      d[0] = make_float4(h[sl][0], h[sl][1], h[sl][2], h[sl][3]);
+      d[1] = make_float4(h[sl][4], h[sl][5], h[sl][6], h[sl][7]);
+    }
+  }
+  __syncthreads();  // the odd rows staged
+  if ((ohl & 1) == 0 || ohl == kStemTH - 1) {
+    const int pr = (ohl + 1) >> 1;  // even rows: ohl / 2; the last row: pooled row 4
+    const int64_t pi = static_cast<int64_t>(th) * (kStemTH / 2) + pr;
+    if (pi < Hp) {
+#pragma unroll
+      for (int sl = 0; sl < 5; ++sl) {
+        if (q == 1 && sl == 0) continue;
+        const int pc = 4 * q + sl;
+        const int pj = tw * (kStemTW / 2) + pc;
+        if (pj >= Wp) continue;
+        float v[8];
+#pragma unroll
+        for (int c = 0; c < 8; ++c) v[c] = h[sl][c];
+        if ((ohl & 1) == 0) {
+          // rows ohl - 1 and ohl + 1 from the staged odd rows
+#pragma unroll
+          for (int rr = -1; rr <= 1; rr += 2) {
+            const int ro = ohl + rr;
+            if (ro < 0) continue;
+            const float4* sp = reinterpret_cast<const float4*>(xs + (ro >> 1) * kRowF + pc * kStemCout + cg * 8);
+            const float4 a = sp[0], b = sp[1];
+            v[0] = fmaxf(v[0], a.x); v[1] = fmaxf(v[1], a.y); v[2] = fmaxf(v[2], a.z); v[3] = fmaxf(v[3], a.w);
+            v[4] = fmaxf(v[4], b.x); v[5] = fmaxf(v[5], b.y); v[6] = fmaxf(v[6], b.z); v[7] = fmaxf(v[7], b.w);
+          }
+        }
+        float* dst = pool + ((n * Hp + pi) * Wp + pj) * kStemCout + cg * 8;
+        const bool whole = pr >= 1 && pr <= 3 && pc >= 1 && pc <= 7;
+        if (whole) {
+          reinterpret_cast<float4*>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
+          reinterpret_cast<float4*>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
+        } else {
+#pragma unroll
+          for (int c = 0; c < 8; ++c) atomicMax(reinterpret_cast<unsigned int*>(dst) + c, __float_as_uint(v[c]));
+        }
+      }
+    }
+  }
+}
+
 __global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const float* __restrict__ x,
                                                                      const float* __restrict__ w,
-                                                                     float* __restrict__ y, int64_t N, int H, int W,
-                                                                     int Ho, int Wo, int relu) {
+                                                                     float* __restrict__ y, float* __restrict__ pool,
+                                                                     int64_t N, int H, int W, int Ho, int Wo, int Hp,
+                                                                     int Wp, int relu) {
   extern __shared__ float4 smem4[];
   float* ws = reinterpret_cast<float*>(smem4);  // [147][2][16][4]
   float* xs = ws + kStemTerms * kStemCout;      // [copy 4][parity 2][ci 3][row 21][16]
@@ -232,26 +310,23 @@ __global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const flo
     // the next tile's loads are in flight while this one's outputs are stored
     if (t + gridDim.x < n_tiles) fetch(t + gridDim.x);
     const int oh = th * kStemTH + ohl;
-    if (oh < Ho) {
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const int ow = tw * kStemTW + 8 * q + j;
-        if (ow < Wo) {
-          float4* yp = reinterpret_cast<float4*>(y + ((n * Ho + oh) * Wo + ow) * kStemCout + cg * 8);
+    for (int j = 0; j < 8; ++j) {
+      const bool in_out = oh < Ho && tw * kStemTW + 8 * q + j < Wo;
 #pragma unroll
-          for (int h = 0; h < 2; ++h) {
-            float4 o = make_float4(acc[j][4 * h], acc[j][4 * h + 1], acc[j][4 * h + 2], acc[j][4 * h + 3]);
-            if (relu) {
-              o.x = fmaxf(o.x, 0.0f);
-              o.y = fmaxf(o.y, 0.0f);
-              o.z = fmaxf(o.z, 0.0f);
-              o.w = fmaxf(o.w, 0.0f);
-            }
-            yp[h] = o;
-          }
-        }
+      for (int c = 0; c < 8; ++c) {
+        if (relu) acc[j][c] = fmaxf(acc[j][c], 0.0f);
+        // a pixel outside the output takes no part in a pooling window (with
+        // ReLU every value is >= 0, and 0 leaves a window's maximum unchanged)
+        if (pool != nullptr && !in_out) acc[j][c] = 0.0f;
+      }
+      if (y != nullptr && in_out) {
+        float4* yp = reinterpret_cast<float4*>(y + ((n * Ho + oh) * Wo + tw * kStemTW + 8 * q + j) * kStemCout + cg * 8);
+        yp[0] = make_float4(acc[j][0], acc[j][1], acc[j][2], acc[j][3]);
+        yp[1] = make_float4(acc[j][4], acc[j][5], acc[j][6], acc[j][7]);
       }
     }
+    if (pool != nullptr) stem_pool_tile(acc, xs, pool, n, th, tw, ohl, q, cg, Hp, Wp);
   }
 }
 
@@ -377,6 +452,19 @@ int64_t out_dim(int64_t n, int k, int s, int p) { return (n + 2 * p - k) / s + 1
 bool aligned16(const void* ptr) { return (reinterpret_cast<uintptr_t>(ptr) & 15u) == 0; }
 
 }  // namespace
+// The stem kernel's dynamic shared memory above the default limit, once per
+// process (the network runs on one device).
+bool stem_smem_attribute() {
+  static bool done = false;
+  if (!done) {
+    if (cudaFuncSetAttribute(pq_stem7x7s2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(kStemSmem)) != cudaSuccess)
+      return false;
+    done = true;
+  }
+  return true;
+}
+
 }  // namespace pq
 
 extern "C" {
@@ -395,20 +483,14 @@ pq_status palquant_conv2d_f32(const float* x_dev, const float* w_dev, float* y_d
   auto s = static_cast<cudaStream_t>(stream);
   if (k == pq::kStemK && stride == pq::kStemS && pad == pq::kStemP && Cin == pq::kStemCin && Cout == pq::kStemCout &&
       pq::aligned16(y_dev)) {
-    static bool stem_attr = false;
-    if (!stem_attr) {
-      if (cudaFuncSetAttribute(pq::pq_stem7x7s2_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                               static_cast<int>(pq::kStemSmem)) != cudaSuccess)
-        return PQ_ECUDA;
-      stem_attr = true;
-    }
+    if (!pq::stem_smem_attribute()) return PQ_ECUDA;
     const int64_t tiles = N * ((Ho + pq::kStemTH - 1) / pq::kStemTH) * ((Wo + pq::kStemTW - 1) / pq::kStemTW);
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
     const unsigned grid = static_cast<unsigned>(tiles < static_cast<int64_t>(sms) * 2 ? tiles : sms * 2);
     pq::pq_stem7x7s2_kernel<<<grid, pq::kStemThreads, pq::kStemSmem, s>>>(
-        x_dev, w_dev, y_dev, N, H, W, static_cast<int>(Ho), static_cast<int>(Wo), relu);
+        x_dev, w_dev, y_dev, nullptr, N, H, W, static_cast<int>(Ho), static_cast<int>(Wo), 0, 0, relu);
     return cudaGetLastError() == cudaSuccess ? PQ_OK : PQ_ECUDA;
   }
   if (wbytes <= 96 * 1024) {
@@ -425,6 +507,31 @@ pq_status palquant_conv2d_f32(const float* x_dev, const float* w_dev, float* y_d
     pq::pq_conv2d_f32_kernel<false><<<pq::grid_for(work, 8), pq::kF32Threads, 0, s>>>(
         x_dev, w_dev, y_dev, N, H, W, Cin, Cout, k, stride, pad, static_cast<int>(Ho), static_cast<int>(Wo), relu);
   }
+  return cudaGetLastError() == cudaSuccess ? PQ_OK : PQ_ECUDA;
+}
+
+pq_status palquant_stem_pool_f32(const float* x_dev, const float* w_dev, float* stem_dev, float* pool_dev, int64_t N,
+                                 int32_t H, int32_t W, int32_t Cout, pq_stream_t stream) {
+  if (N < 0 || H <= 0 || W <= 0 || Cout <= 0 || !x_dev || !w_dev || !pool_dev) return PQ_EINVAL;
+  if (!pq::aligned16(pool_dev) || (stem_dev && !pq::aligned16(stem_dev))) return PQ_EINVAL;
+  if (Cout != pq::kStemCout) return PQ_EUNSUPPORTED;
+  const int64_t Ho = pq::out_dim(H, pq::kStemK, pq::kStemS, pq::kStemP), Wo = pq::out_dim(W, pq::kStemK, pq::kStemS, pq::kStemP);
+  if (Ho <= 0 || Wo <= 0) return PQ_EINVAL;
+  const int64_t Hp = pq::out_dim(Ho, 3, 2, 1), Wp = pq::out_dim(Wo, 3, 2, 1);
+  if (N == 0) return PQ_OK;
+  auto s = static_cast<cudaStream_t>(stream);
+  if (!pq::stem_smem_attribute()) return PQ_ECUDA;
+  // border windows are combined by atomic maxima over non-negative values: start from 0
+  if (cudaMemsetAsync(pool_dev, 0, static_cast<size_t>(N * Hp * Wp * Cout) * sizeof(float), s) != cudaSuccess)
+    return PQ_ECUDA;
+  const int64_t tiles = N * ((Ho + pq::kStemTH - 1) / pq::kStemTH) * ((Wo + pq::kStemTW - 1) / pq::kStemTW);
+  int dev = 0, sms = 148;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const unsigned grid = static_cast<unsigned>(tiles < static_cast<int64_t>(sms) * 2 ? tiles : sms * 2);
+  pq::pq_stem7x7s2_kernel<<<grid, pq::kStemThreads, pq::kStemSmem, s>>>(
+      x_dev, w_dev, stem_dev, pool_dev, N, H, W, static_cast<int>(Ho), static_cast<int>(Wo), static_cast<int>(Hp),
+      static_cast<int>(Wp), 1);
   return cudaGetLastError() == cudaSuccess ? PQ_OK : PQ_ECUDA;
 }
 

@@ -7,7 +7,8 @@ in full precision (Sec. 5).  The paper's network figure is not available; this d
 takes the following reading:
 
 * stem: 7x7 stride-2 pad-3 fp32 convolution (3 -> G*w_1 channels) + ReLU, then 3x3
-  stride-2 pad-1 max pooling; the pooled tensor is quantised once into codes;
+  stride-2 pad-1 max pooling (one kernel for 128 stem channels); the pooled tensor
+  is quantised once into codes;
 * four stages of two basic blocks (per-group widths w_1..w_4).  In block (X, Q):
     conv1  PalQuant 3x3 (stride 2 in the first block of stages 2-4), ReLU, no
            permutation, codes out (requantised with conv2's input steps);
@@ -52,7 +53,7 @@ def _out(n: int, k: int, s: int, p: int) -> int:
 class PalQuantResNet18:
     def __init__(self, params: dict, N: int, H: int = 224, W: int = 224, G: int = 2, widths=(64, 128, 256, 512),
                  classes: int = 1000, bits: int = 2, device="cuda:0", stream: torch.cuda.Stream | None = None,
-                 code_format: int | None = None, placement: str = "block"):
+                 code_format: int | None = None, placement: str = "block", keep_stem: bool = False):
         if placement not in ("block", "paper"):
             raise ValueError("placement must be 'block' or 'paper'")
         self.placement = placement
@@ -76,7 +77,10 @@ class PalQuantResNet18:
         self.C0 = C0
         self.w_stem = torch.from_numpy(np.ascontiguousarray(params["stem"])).to(self.dev)
         self.w_fc = torch.from_numpy(np.ascontiguousarray(params["fc"])).to(self.dev)
-        self.stem_out = torch.empty((N, self.Hs, self.Ws, C0), **f32)
+        # The stem and the max pooling run as one kernel for 128 stem channels (the
+        # stem output then stays on chip unless keep_stem asks for it), else as two.
+        self.fused_stem = C0 == 128
+        self.stem_out = torch.empty((N, self.Hs, self.Ws, C0), **f32) if keep_stem or not self.fused_stem else None
         self.pool = torch.empty((N, self.Hp, self.Wp, C0), **f32)
         self.in_codes = torch.empty((N, self.Hp, self.Wp, C0 // per_byte), **u8)
         self.blocks = []
@@ -293,6 +297,10 @@ class PalQuantResNet18:
     # --------------------------------------------------------------- forward
     def _stem(self, x_dev):
         s = self.stream
+        if self.fused_stem:
+            B.palquant_stem_pool_f32(x_dev, self.w_stem, self.stem_out, self.pool, self.N, self.H, self.W, self.C0,
+                                     stream=s)
+            return
         B.palquant_conv2d_f32(x_dev, self.w_stem, self.stem_out, self.N, self.H, self.W, 3, self.C0, 7, 2, 3, relu=True,
                               stream=s)
         B.palquant_maxpool2d_f32(self.stem_out, self.pool, self.N, self.Hs, self.Ws, self.C0, 3, 2, 1, stream=s)
@@ -382,9 +390,10 @@ class PalQuantResNet18:
         return self.logits
 
     def launches_per_forward(self) -> int:
-        """Kernels one forward launches: stem conv, max pooling, quantiser, per block
-        conv1 (+ down) + conv2, average pooling, FC."""
-        n = 3 + sum(3 if b["down"] else 2 for b in self.blocks) + 2
+        """Kernels one forward launches: the stem with its max pooling (one kernel for
+        128 stem channels, else two), quantiser, per block conv1 (+ down) + conv2,
+        average pooling, FC."""
+        n = (2 if self.fused_stem else 3) + sum(3 if b["down"] else 2 for b in self.blocks) + 2
         if self.paper:
             n += len(self.modules) + len(self.modules) - 1  # a module per stage, a quantiser per stage boundary
         return n

@@ -23,7 +23,8 @@ def _codes(t, fmt):
 
 def _compare(net, r):
     f = net.fmt
-    assert np.array_equal(net.stem_out.cpu().numpy(), r["stem"]), "stem"
+    if net.stem_out is not None:
+        assert np.array_equal(net.stem_out.cpu().numpy(), r["stem"]), "stem"
     assert np.array_equal(net.pool.cpu().numpy(), r["pool"]), "max pooling"
     assert np.array_equal(_codes(net.in_codes, f), r[net.blocks[0]["name"] + ".in_codes"]), "input codes"
     for i, blk in enumerate(net.blocks):
@@ -69,8 +70,11 @@ def test_resnet18_224_matches_oracle():
     steps = OR.calibrate(x, params, 2, 2)
     r = OR.forward(x, params, 2, 2, steps)
     xd = torch.from_numpy(x).cuda()
-    for fmt in (B.PQ_CODES_C32F4, B.PQ_CODES_C16):  # the default (FP4 nibbles), and one code per byte
-        net = PalQuantResNet18(params, 1, code_format=None if fmt == B.PQ_CODES_C32F4 else fmt)
+    # the default (FP4 nibbles, the stem output kept for the comparison), and one code
+    # per byte with the stem output never written
+    for fmt, keep in ((B.PQ_CODES_C32F4, True), (B.PQ_CODES_C16, False)):
+        net = PalQuantResNet18(params, 1, code_format=None if fmt == B.PQ_CODES_C32F4 else fmt, keep_stem=keep)
+        assert net.fused_stem and (net.stem_out is not None) == keep
         assert net.fmt == fmt
         net.set_steps(steps)
         net.forward(xd)
@@ -124,6 +128,38 @@ def test_conv2d_f32_matches_oracle(shape, Cout, k, s, p, relu):
                           shape[3], Cout, k, s, p, relu)
     assert B.palquant_sync_check() == B.PQ_OK
     assert np.array_equal(y.cpu().numpy(), ref)
+
+
+@pytest.mark.parametrize("N,H,W,keep", [(2, 224, 224, True), (2, 37, 29, True), (3, 50, 46, False), (1, 13, 9, True)])
+def test_stem_pool_f32_matches_oracle(N, H, W, keep):
+    """The fused stem + max pooling: the pooled output (and the stem output when asked
+    for) bit for bit against the oracle's separate convolution and pooling; tiles
+    ragged at the image's right and bottom edges, and images of one tile."""
+    import oracle
+    from paper_2208_01944_gb300 import binding as B
+
+    gen = synth.generator(N * 1000 + H + W)
+    x = synth.normal((N, H, W, 3), gen)
+    w = synth.normal((128, 7, 7, 3), gen, 0.2)
+    stem = oracle.conv2d_f32(x, w, 2, 3, True)
+    ref = oracle.maxpool_f32(stem, 3, 2, 1)
+    pool = torch.full(ref.shape, float("nan"), dtype=torch.float32, device="cuda")  # the call zeroes it
+    st = torch.empty(stem.shape, dtype=torch.float32, device="cuda") if keep else None
+    B.palquant_stem_pool_f32(torch.from_numpy(x).cuda(), torch.from_numpy(w).cuda(), st, pool, N, H, W, 128)
+    assert B.palquant_sync_check() == B.PQ_OK
+    assert np.array_equal(pool.cpu().numpy(), ref)
+    if keep:
+        assert np.array_equal(st.cpu().numpy(), stem)
+
+
+def test_stem_pool_f32_rejects_other_widths():
+    from paper_2208_01944_gb300 import binding as B
+
+    x = torch.zeros((1, 16, 16, 3), device="cuda")
+    w = torch.zeros((64, 7, 7, 3), device="cuda")
+    pool = torch.empty((1, 4, 4, 64), device="cuda")
+    with pytest.raises(RuntimeError):
+        B.palquant_stem_pool_f32(x, w, None, pool, 1, 16, 16, 64)
 
 
 def test_pooling_and_linear_match_oracle():
