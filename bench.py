@@ -109,8 +109,9 @@ def run_profile_layer(name: str, reps: int, fmt_name: str = "c16"):
 
 
 def run_profile_stem(N: int, reps: int):
-    """The network's stem alone (7x7 stride-2 pad-3 fp32 convolution 3 -> 128 channels
-    + ReLU) on N synthetic 224x224 images, for profiling."""
+    """The network's stem with its max pooling (7x7 stride-2 pad-3 fp32 convolution
+    3 -> 128 channels + ReLU, then 3x3 stride-2 pad-1 max pooling, one kernel) on N
+    synthetic 224x224 images, for profiling."""
     import torch
 
     from paper_2208_01944_gb300 import binding as B
@@ -120,9 +121,9 @@ def run_profile_stem(N: int, reps: int):
     x, params = synth.resnet18_inputs(N, seed=0)
     xd = torch.from_numpy(x).to(dev)
     wd = torch.from_numpy(params["stem"]).to(dev)
-    y = torch.empty((N, 112, 112, wd.shape[0]), dtype=torch.float32, device=dev)
+    pool = torch.empty((N, 56, 56, wd.shape[0]), dtype=torch.float32, device=dev)
     for _ in range(reps):
-        B.palquant_conv2d_f32(xd, wd, y, N, 224, 224, 3, wd.shape[0], 7, 2, 3, relu=True)
+        B.palquant_stem_pool_f32(xd, wd, None, pool, N, 224, 224, wd.shape[0])
     st = B.palquant_sync_check()
     assert st == B.PQ_OK, B.strerror(st)
 
@@ -605,6 +606,10 @@ def measure_resnet18_paper(dev, world, args):
            "palquant_body_tops": whole_job_rate(net.body_int_ops(), world, ms) / 1e12,
            "gpu_launches_per_forward": net.launches_per_forward(),
            "timed": "CUDA-graph replay; 4 cyclic shuffle modules, 20 PalQuant layers, 4 quantisers"}
+    marks = []
+    net.forward(xs[0], marks)
+    torch.cuda.synchronize(dev)
+    res["stages_ms"] = {name: marks[i - 1][1].elapsed_time(ev) for i, (name, ev) in enumerate(marks) if i > 0}
     del graphs, net
     torch.cuda.empty_cache()
     return res

@@ -875,57 +875,6 @@ __device__ __forceinline__ void epi_store_codes(const ConvParams& p, const EpiIt
   }
 }
 
-// The 16 shortcut values of accumulator row m, 16-column chunk ch (the source
-// channels of the unit), or zeros for a row outside the output.
-__device__ __forceinline__ void epi_load_shortcut(const ConvParams& p, const EpiItem& e, int m, int ch,
-                                                  float (&sc)[16]) {
-  bool valid;
-  const int pos = epi_pos(p, e, m, valid);
-  if (valid) {
-    const long long pix = static_cast<long long>(e.n) * p.Ho * p.Wo + pos;
-    const float4* s4 = reinterpret_cast<const float4*>(p.shortcut + pix * p.C_out_total + e.src_c0 + ch * 16);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float4 t = s4[j];
-      sc[4 * j] = t.x; sc[4 * j + 1] = t.y; sc[4 * j + 2] = t.z; sc[4 * j + 3] = t.w;
-    }
-  } else {
-#pragma unroll
-    for (int j = 0; j < 16; ++j) sc[j] = 0.0f;
-  }
-}
-
-// Channel-shuffle unit: int32 sums, fp32 outputs (with the shortcut, loaded by
-// the caller into sc) and codes, each channel scattered to destination channel
-// co * G + g (unstaged, one element at a time).
-__device__ __forceinline__ void epi_general16(const ConvParams& p, const EpiItem& e, int m, int ch, const uint32_t* v,
-                                              const float (&sc)[16]) {
-  bool valid;
-  const int pos = epi_pos(p, e, m, valid);
-  if (!valid) return;
-  const long long hw_out = static_cast<long long>(p.Ho) * p.Wo;
-  const long long pix = static_cast<long long>(e.n) * hw_out + pos;
-  const bool has_sc = p.shortcut != nullptr;
-  const int qmax = p.qmax_out;
-  const float qmax_f = static_cast<float>(qmax);
-  for (int j = 0; j < 16; ++j) {
-    const float raw = __uint_as_float(v[j]);
-    float t = __fmul_rn(raw, e.m_out512);  // = (float)acc * m_out, one rounding
-    if (has_sc) t = __fadd_rn(t, sc[j]);
-    if (p.relu) t = fmaxf(t, 0.0f);
-    const int code = requant_code(has_sc ? __fmul_rn(t, e.m_req) : __fmul_rn(raw, e.m_req512), qmax_f, qmax);
-    const int co = e.nb * p.Nblk + ch * 16 + j;
-    const long long dc = static_cast<long long>(co) * p.G + e.g;
-    const long long o = pix * p.C_out_total + dc;
-    if (p.acc_out) p.acc_out[o] = __float2int_rn(__fmul_rn(raw, 512.0f));
-    if (p.y_out) p.y_out[o] = t;
-    if (p.q_out) {
-      const long long c16o = (static_cast<long long>(e.n) * (p.C_out_total >> 4) + (dc >> 4)) * hw_out + pos;
-      p.q_out[p.codes_c16 ? c16o * 16 + (dc & 15) : o] = static_cast<uint8_t>(code);
-    }
-  }
-}
-
 // General units (int32 sums, fp32 outputs with or without the shortcut, codes)
 // of UC accumulator columns.  TMEM gives each lane one row (pixel), but a global
 // access instruction costs about one cycle per cache line it touches, so rows
@@ -964,6 +913,11 @@ __device__ __forceinline__ void epi_general_units(const ConvParams& p, const Epi
   const int per_acc = p.Nblk / UC;
   const int n_units = p.MT * per_acc;
   const int pr = lane / CPR, pc = lane % CPR;  // row within a pass, chunk: coalesced role
+  // Channel shuffle (kind 2): column j of the unit goes to destination channel
+  // (nb Nblk + col0 + j) G + g, so a staged row leaves as UC values G apart:
+  // lane j of a store instruction takes column j of 32 / UC rows.
+  const bool shuf = p.channel_shuffle != 0;
+  const int sj = lane % UC, sr = lane / UC;
   for (int u = wg; u < n_units; u += n_groups) {
     const int mt = u / per_acc, col0 = (u - mt * per_acc) * UC;
     bool valid;
@@ -977,6 +931,19 @@ __device__ __forceinline__ void epi_general_units(const ConvParams& p, const Epi
     // Whole staged rows to global memory (row r's element offset is lane r's rowc).
     auto store_rows = [&](void* out, int c0) {
       __syncwarp();
+      if (shuf) {
+        const long long dcl = static_cast<long long>(e.nb * p.Nblk + col0 + sj) * p.G + e.g;
+#pragma unroll 4
+        for (int r0 = 0; r0 < 32; r0 += 32 / UC) {
+          const int r = r0 + sr;
+          const long long off = __shfl_sync(0xffffffffu, rowc, r);
+          uint32_t x;
+          asm volatile("ld.shared.b32 %0, [%1];" : "=r"(x) : "r"(stg_chunk<UC>(sbase, r, sj >> 2) + 4u * (sj & 3)) : "memory");
+          if (off >= 0) reinterpret_cast<uint32_t*>(out)[off + dcl] = x;
+        }
+        __syncwarp();
+        return;
+      }
 #pragma unroll
       for (int ps = 0; ps < CPR; ++ps) {
         const int r = ps * RPP + pr;
@@ -1069,10 +1036,23 @@ __device__ __forceinline__ void epi_general_units(const ConvParams& p, const Epi
       stage_row(v);
       store_rows(p.y_out, e.dst_c0);
     }
-    if (p.q_out) {
+    if (p.q_out && !shuf) {
       __syncwarp();
 #pragma unroll
       for (int h = 0; h < UC / 16; ++h) epi_store_codes(p, e, stg, lane, valid, pos, col0 / 16 + h, w[h]);
+    } else if (p.q_out && valid) {
+      // byte codes scattered one by one (the API takes no packed codes here)
+#pragma unroll
+      for (int h = 0; h < UC / 16; ++h) {
+        const uint32_t wd[4] = {w[h].x, w[h].y, w[h].z, w[h].w};
+#pragma unroll
+        for (int j = 0; j < 16; ++j) {
+          const long long dc = static_cast<long long>(e.nb * p.Nblk + col0 + 16 * h + j) * p.G + e.g;
+          const long long o = p.codes_c16 ? ((static_cast<long long>(e.n) * (p.C_out_total >> 4) + (dc >> 4)) * hw_out + pos) * 16 + (dc & 15)
+                                          : rowc + dc;
+          p.q_out[o] = static_cast<uint8_t>(wd[j >> 2] >> (8 * (j & 3)));
+        }
+      }
     }
   }
 }
@@ -1234,23 +1214,11 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
         c_mt = n_mt;
         c_ch = n_ch;
       }
-    } else if (!p.channel_shuffle) {
+    } else {
       if ((p.Nblk & 31) == 0)
         epi_general_units<32>(p, e, stg, wg, n_groups, quarter, lane, qmax2);
       else
         epi_general_units<16>(p, e, stg, wg, n_groups, quarter, lane, qmax2);
-    } else {
-      // The channel shuffle's per-channel scatter (rarely used).
-      const int m_lane = quarter * 32 + lane;
-      for (int u = wg; u < n_units; u += n_groups) {
-        const int mt = u / nchunks, ch = u - mt * nchunks;
-        float sc[16];
-        if (p.shortcut != nullptr) epi_load_shortcut(p, e, mt * 128 + m_lane, ch, sc);
-        uint32_t v[16];
-        tmem_ld16(e.tbase + mt * p.Npow2 + ch * 16, v);
-        tmem_wait_ld();
-        epi_general16(p, e, mt * 128 + m_lane, ch, v, sc);
-      }
     }
     // One arrival per warp: the warp's tensor-memory reads are complete (each
     // thread waited for its loads) and ordered before the arrive by the fence
