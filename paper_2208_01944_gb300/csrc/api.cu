@@ -121,9 +121,15 @@ struct Phase {
 // copy warps quantise TMA-staged 32-channel fp32 boxes into the operand stages).
 // direct_out: the call reads no shortcut and writes channel-blocked codes only
 // (no int32 or fp32 outputs), which the epilogue stores straight from registers,
-// so the plan reserves no per-warp staging for it.
+// so the plan reserves no per-warp staging for it.  shortcut: the call reads a
+// shortcut (two staging buffers per warp).
 pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, std::vector<Phase>* phases_out,
-                    bool quant_in = false, bool direct_out = false) {
+                    bool quant_in = false, bool direct_out = false, bool shortcut = false) {
+  // Epilogue staging per warp: 32 rows of up to 32 fp32/int32 values (128 bytes,
+  // chunk-swizzled), twice with a shortcut (the next unit's rows are fetched into
+  // the second buffer), or 32 rows of 16 code bytes at a pitch of 80 bytes (an odd
+  // number of 16-byte bank groups).
+  const uint32_t warp_stage = direct_out ? 0u : (shortcut ? 2u : 1u) * 32u * 128u;
   pq_status st = validate_desc(d);
   if (st != PQ_OK) return st;
   pq_conv_plan plan;
@@ -270,7 +276,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
       const uint64_t w_unit = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk / cpb;
       const uint64_t w_min = w_unit <= 112u * 1024u ? round_up(w_unit, 1024) : 2ull * round_up(32ull * p.Nblk, 1024);
       const uint64_t need = 2ull * (cpb * round_up(npos * 128, 1024) + round_up(npos * 32, 1024)) + w_min +
-                            (direct_out ? 0ull : pq::kEpiWarps * 4096ull) + 1024;
+                            static_cast<uint64_t>(pq::kEpiWarps) * warp_stage + 1024;
       if (need > pq::kMaxSmem - 1024) continue;
     }
     const int units = MT * units_per_acc;
@@ -343,12 +349,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
                              16ull * (p.MT * 128 + off_max);
     return round_up(std::max<uint64_t>(static_cast<uint64_t>(p.nph) * (*phase_bytes), overrun), 1024);
   };
-  // Epilogue staging per warp: 32 rows of up to 32 fp32/int32 values (128 bytes,
-  // chunk-swizzled), or 32 rows of 16 code bytes at a pitch of 80 bytes (an odd
-  // number of 16-byte bank groups).
   const uint32_t q_pitch = 80;
   const uint32_t f_pitch = 128;
-  const uint32_t warp_stage = 32u * 128u;
   // Staging for every warp that runs the epilogue: the copy warps join it only when
   // TMA loads the activation operand as it is (not unpacked, not quantised).
   const bool third_group =
@@ -823,7 +825,7 @@ pq_status layer_fused_impl(const void* q_dev, const void* w_packed_dev, const pq
   const bool direct_out =
       acc_out_dev == nullptr && y_out_dev == nullptr && shortcut_dev == nullptr && d->code_format != PQ_CODES_INT8;
   const bool quant_in = inv_s_in != nullptr || l_in != nullptr;
-  st = plan_conv(d, &p, nullptr, &phases, quant_in, direct_out);
+  st = plan_conv(d, &p, nullptr, &phases, quant_in, direct_out, shortcut_dev != nullptr);
   if (st != PQ_OK) return st;
   if (l_in != nullptr) {
     // learned bounds: the training forward's codes (sat((x - l) * fl(1/fl(u - l))) * Qp, rounded)

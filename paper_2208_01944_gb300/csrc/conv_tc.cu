@@ -902,8 +902,12 @@ template <int UC>
 __device__ __forceinline__ void epi_general_units(const ConvParams& p, const EpiItem& e, uint8_t* stg, int wg,
                                                   int n_groups, int quarter, int lane, uint32_t qmax2) {
   constexpr int CPR = UC / 4, RPP = 32 / CPR;  // chunks per row, rows per coalesced pass
-  const uint32_t sbase = smem_u32(stg);
+  constexpr uint32_t kBuf = 32u * UC * 4u;     // one staging buffer: 32 rows of UC values
   const bool has_sc = p.shortcut != nullptr;
+  // With a shortcut (and no int32 output, which would need the buffer first) the
+  // next unit's shortcut rows are fetched into the warp's second buffer while
+  // this unit computes and stores: the fetch latency then runs under the stores.
+  const bool pre = has_sc && p.acc_out == nullptr;
   const bool f16q = !has_sc || p.relu;
   const float m_q = has_sc ? __fmul_rn(e.m_req, 1.0f / 16777216.0f) : e.m_req15;
   const int qmax = p.qmax_out;
@@ -918,11 +922,49 @@ __device__ __forceinline__ void epi_general_units(const ConvParams& p, const Epi
   // lane j of a store instruction takes column j of 32 / UC rows.
   const bool shuf = p.channel_shuffle != 0;
   const int sj = lane % UC, sr = lane / UC;
-  for (int u = wg; u < n_units; u += n_groups) {
+  // this lane's row offset (elements; -1 outside the output) of unit u
+  auto row_of = [&](int u, bool& valid, int& pos) -> long long {
+    const int mt = u / per_acc;
+    pos = epi_pos(p, e, mt * 128 + m_lane, valid);
+    return valid ? (static_cast<long long>(e.n) * hw_out + pos) * p.C_out_total : -1;
+  };
+  // unit u's shortcut rows (its source channels) into buffer `buf` by cp.async,
+  // whole rows per instruction, zero-filled outside the output
+  auto fetch_sc = [&](int u, long long rc, uint32_t buf) {
+    const int col0 = (u - (u / per_acc) * per_acc) * UC;
+#pragma unroll
+    for (int ps = 0; ps < CPR; ++ps) {
+      const int r = ps * RPP + pr;
+      const long long off = __shfl_sync(0xffffffffu, rc, r);
+      cp_async_16(stg_chunk<UC>(buf, r, pc), off >= 0 ? p.shortcut + off + e.src_c0 + col0 + 4 * pc : p.shortcut,
+                  off >= 0 ? 16u : 0u);
+    }
+    cp_async_commit();
+  };
+  int cur = 0;
+  if (pre && wg < n_units) {
+    bool v0;
+    int p0;
+    fetch_sc(wg, row_of(wg, v0, p0), smem_u32(stg));
+  }
+  for (int u = wg; u < n_units; u += n_groups, cur ^= 1) {
     const int mt = u / per_acc, col0 = (u - mt * per_acc) * UC;
     bool valid;
-    const int pos = epi_pos(p, e, mt * 128 + m_lane, valid);
-    const long long rowc = valid ? (static_cast<long long>(e.n) * hw_out + pos) * p.C_out_total : -1;
+    int pos;
+    const long long rowc = row_of(u, valid, pos);
+    const uint32_t sbase = smem_u32(stg) + (pre ? static_cast<uint32_t>(cur) * kBuf : 0u);
+    uint8_t* const stg_cur = stg + (pre ? cur * kBuf : 0u);
+    if (pre) {
+      if (u + n_groups < n_units) {
+        bool vn;
+        int pn;
+        fetch_sc(u + n_groups, row_of(u + n_groups, vn, pn), smem_u32(stg) + static_cast<uint32_t>(cur ^ 1) * kBuf);
+        cp_async_wait<1>();  // this unit's rows have landed; the next unit's may still be in flight
+      } else {
+        cp_async_wait<0>();
+      }
+      __syncwarp();
+    }
     uint32_t v[UC];
     if constexpr (UC == 32)
       tmem_ld32(e.tbase + mt * p.Npow2 + col0, v);
@@ -976,16 +1018,9 @@ __device__ __forceinline__ void epi_general_units(const ConvParams& p, const Epi
       stage_row(a);
       store_rows(p.acc_out, e.dst_c0);
     }
-    if (has_sc) {
-      // the rows' shortcut values (the unit's source channels) into the staging buffer
-#pragma unroll
-      for (int ps = 0; ps < CPR; ++ps) {
-        const int r = ps * RPP + pr;
-        const long long off = __shfl_sync(0xffffffffu, rowc, r);
-        cp_async_16(stg_chunk<UC>(sbase, r, pc), off >= 0 ? p.shortcut + off + e.src_c0 + col0 + 4 * pc : p.shortcut,
-                    off >= 0 ? 16u : 0u);
-      }
-      cp_async_commit();
+    if (has_sc && !pre) {
+      // the rows' shortcut values into the staging buffer, after the int32 sums left it
+      fetch_sc(u, rowc, sbase);
       cp_async_wait<0>();
       __syncwarp();
     }
@@ -1039,7 +1074,7 @@ __device__ __forceinline__ void epi_general_units(const ConvParams& p, const Epi
     if (p.q_out && !shuf) {
       __syncwarp();
 #pragma unroll
-      for (int h = 0; h < UC / 16; ++h) epi_store_codes(p, e, stg, lane, valid, pos, col0 / 16 + h, w[h]);
+      for (int h = 0; h < UC / 16; ++h) epi_store_codes(p, e, stg_cur, lane, valid, pos, col0 / 16 + h, w[h]);
     } else if (p.q_out && valid) {
       // byte codes scattered one by one (the API takes no packed codes here)
 #pragma unroll
