@@ -66,3 +66,35 @@ def test_module_rejects_non_1x1():
         with pytest.raises(B.PalquantError) as e:
             B.palquant_cyclic_shuffle_module(16, 16, d, [1.0, 1.0], [1.0, 1.0], 1, 16, 16, None)
         assert e.value.status == B.PQ_EINVAL
+
+
+@pytest.mark.parametrize("G", [2, 3, 4])
+def test_prop1_chained_modules_reach_every_group(G):
+    """Prop. 1 on the device: G - 1 cyclic shuffle modules chained through the library
+    (each module's fp32 output quantised by the library for the next) spread one
+    non-zero input group to every group; every intermediate tensor bit for bit
+    against the oracle's chain."""
+    from paper_2208_01944_gb300 import binding as B
+
+    Cg, N, H, W = 32, 1, 4, 6
+    wq = np.ones((G, Cg, 1, 1, Cg), dtype=np.int8)
+    m_out = np.full(G, 0.1, np.float32)
+    inv = np.ones(G, np.float32)
+    d = B.layer_desc(N, H, W, G, Cg, Cg, 1, 1, 0, 2, 2, 2, 0, code_format=2)
+    wp = torch.from_numpy(B.palquant_pack_weight_codes_host(wq, d)).cuda()
+    for s in range(G):
+        x = np.zeros((N, H, W, G * Cg), dtype=np.float32)
+        x[..., s * Cg:(s + 1) * Cg] = 2.0
+        xd = torch.from_numpy(x).cuda()
+        for k in range(1, G):
+            q_ref = oracle.quantize_act(x, G, 2, inv)
+            x, _ = oracle.cyclic_shuffle_module(x, q_ref, wq, m_out, None, 1)
+            qd = torch.empty((N, H, W, G * Cg), dtype=torch.uint8, device="cuda")
+            B.palquant_quantize_act(xd, qd, N, H, W, G, Cg, 2, inv, code_format=2)
+            zd = torch.empty_like(xd)
+            B.palquant_cyclic_shuffle_module(qd, wp, d, m_out, None, 1, xd, zd, None)
+            assert B.palquant_sync_check() == B.PQ_OK
+            assert np.array_equal(zd.cpu().numpy(), x), (G, s, k)
+            live = {g for g in range(G) if np.any(x[..., g * Cg:(g + 1) * Cg] != 0)}
+            assert live == {(s + j) % G for j in range(k + 1)}, (G, s, k, live)
+            xd = zd
