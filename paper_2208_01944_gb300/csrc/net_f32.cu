@@ -104,127 +104,99 @@ __device__ __forceinline__ void fma2_rn(float& d0, float& d1, float a, float b0,
 }
 
 // The 7x7 stride-2 convolution of a 3-channel image to 128 channels (the
-// network's first layer).  A block of 256 threads computes an output tile of
-// 8 rows x 16 columns; thread (pixel group p, channel group g) the 8
-// consecutive pixels 8 (p % 2) .. + 7 of row p / 2 and the 8 channels
-// 8 g .. 8 g + 7: 64 sums, so that a term costs two 16-byte loads of inputs,
-// two of weights and 32 packed FMAs.  The input tile (21 x 37 x 3 floats, zero
-// outside the image) is held split by column parity, channel-planar, in four
-// copies shifted by 0..3 positions: copy s of parity b holds at row r, position
-// k the tile's column 2 (k + s) + b, so the 8 inputs of a thread for tap
-// (kh, kw) are positions 8 (p % 2) .. + 7, aligned, of copy kw / 2, parity
-// kw % 2, row 2 (p / 2) + kh.  The weights of a term are stored as two halves of
-// 4 channels per group ([147][2][16][4]), so that the 16 groups of a warp read
-// 256 contiguous bytes.  The next tile's inputs are loaded into registers while
-// the current one's outputs are stored, and the two CTAs of an SM take turns at
-// the barriers.  Per output the terms are added in (kh, kw, ci) order like the
-// generic kernel; the zero taps outside the image change nothing:
-// fma(0, w, acc) = acc for finite w, since a sum started at +0 is never -0
-// under round-to-nearest.
+// network's first layer).  One block of 256 threads per SM computes output
+// tiles of 16 rows x 16 columns; thread (row r, channel group g) holds the 16
+// pixels of tile row r and the 8 channels 8 g .. 8 g + 7: 128 sums, so that a
+// term costs four 16-byte input loads, two 16-byte weight loads and 64 packed
+// FMAs, with the registers to load the next term's operands while the current
+// one's FMAs run.  The input window of a tile (37 x 37 x 3 floats, zero outside
+// the image) is held split by column parity, channel-planar, in four copies
+// shifted by 0..3 positions: copy s of parity b holds at row i, position k the
+// window's column 2 (k + s) + b, so the 16 inputs of a thread for tap (kh, kw)
+// are positions 0..15, aligned, of copy kw / 2, parity kw % 2, row 2 r + kh.
+// The next tile's window comes into a plain copy in shared memory by cp.async
+// while the current one is computed, and is split into the copies between the
+// tile's two barriers.  The weights of a term are stored as two
+// halves of 4 channels per group ([147][2][16][4]): the 16 groups of a warp
+// read 256 contiguous bytes.  Per output the terms are added in (kh, kw, ci)
+// order like the generic kernel; the zero taps outside the image change
+// nothing: fma(0, w, acc) = acc for finite w, since a sum started at +0 is
+// never -0 under round-to-nearest.
 constexpr int kStemK = 7, kStemS = 2, kStemP = 3, kStemCin = 3, kStemCout = 128;
-constexpr int kStemTH = 8, kStemTW = 16;
+constexpr int kStemTH = 16, kStemTW = 16;
 constexpr int kStemThreads = 256;
-constexpr int kStemIR = (kStemTH - 1) * kStemS + kStemK;  // 21 input rows
+constexpr int kStemIR = (kStemTH - 1) * kStemS + kStemK;  // 37 input rows
 constexpr int kStemIC = (kStemTW - 1) * kStemS + kStemK;  // 37 input columns
 constexpr int kStemTerms = kStemK * kStemK * kStemCin;    // 147
 constexpr int kStemRowF = 16;                             // positions per copy row
 constexpr int kStemPlaneF = kStemIR * kStemRowF;          // one (copy, parity, channel) plane
 constexpr int kStemCopyF = 2 * kStemCin * kStemPlaneF;    // one shifted copy
-constexpr int kStemXFloats = 4 * kStemCopyF;
-constexpr int kStemTileElems = kStemIR * kStemIC * kStemCin;                     // 2331
-constexpr int kStemLoads = (kStemTileElems + kStemThreads - 1) / kStemThreads;  // 10 per thread
-constexpr size_t kStemSmem = (static_cast<size_t>(kStemTerms) * kStemCout + kStemXFloats) * sizeof(float);
+constexpr int kStemXFloats = 4 * kStemCopyF;              // one window
+constexpr int kStemTileElems = kStemIR * kStemIC * kStemCin;                     // 4107
+constexpr int kStemLoads = (kStemTileElems + kStemThreads - 1) / kStemThreads;  // 17 per thread
+constexpr int kStemPoolRowF = 9 * kStemCout;  // a staged row of pooled columns (max pooling)
+constexpr int kStemRawF = (kStemTileElems + 3) / 4 * 4;  // the next window as it lies in the image
+constexpr size_t kStemSmem = (static_cast<size_t>(kStemTerms) * kStemCout + kStemXFloats + kStemRawF +
+                              (kStemTH / 2) * kStemPoolRowF) * sizeof(float);
+
+// Packed fp32 pairs in one 64-bit register (the low half first), and the packed
+// fused multiply-add on them: d = a b + d lane by lane, each lane with a single
+// IEEE rounding like __fmaf_rn.
+__device__ __forceinline__ unsigned long long f32x2_pair(float lo, float hi) {
+  unsigned long long r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f32x2_unpair(unsigned long long v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ void ffma2(unsigned long long& d, unsigned long long a, unsigned long long b) {
+  asm("fma.rn.f32x2 %0, %1, %2, %0;" : "+l"(d) : "l"(a), "l"(b));
+}
+
+// One 4-byte asynchronous copy global -> shared, zero-filled when !valid.
+__device__ __forceinline__ void cp_async4(float* dst, const float* src, bool valid) {
+  const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+  asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(d), "l"(src), "r"(valid ? 4 : 0) : "memory");
+}
 
 // 3x3 stride-2 pad-1 max pooling of the stem tile held in registers (ReLU
 // outputs, so every value is >= 0, and pixels outside the output are 0).
-// Pooled row pr (0..4) of the tile covers stem rows 2 pr - 1 .. 2 pr + 1 and
+// Pooled row pr (0..8) of the tile covers stem rows 2 pr - 1 .. 2 pr + 1 and
 // pooled column pc (0..8) stem columns 2 pc - 1 .. 2 pc + 1 (tile-relative).
-// Columns: each thread reduces its 8 pixels to the windows it sees (slots
-// s = 0..4, pooled column 4 q + s) and the pixel-half q = 0 takes q = 1's part of
-// pooled column 4 by a shuffle.  Rows: warp w holds stem row w; the odd rows go
-// through shared memory (the input copies' space, free after the FMAs) to the
-// even warps, which complete pooled rows 1..3.  Windows that reach into a
-// neighbouring tile (pooled row 0 and 4, pooled column 0 and 8) are combined
+// Columns: each thread reduces its row's 16 pixels to the 9 windows it sees.
+// Rows: the odd rows go through shared memory (`stage`) to the even rows'
+// threads, which complete pooled rows 1..7.  Windows that reach into a
+// neighbouring tile (pooled row 0 and 8, pooled column 0 and 8) are combined
 // across tiles by an integer atomic maximum on the float bits (the order of
 // non-negative floats), into an output the launcher zeroed; the others are
 // stored.  The maximum is exact, so the result does not depend on the order.
-__device__ __forceinline__ void stem_pool_tile(const float (&acc)[8][8], float* xs, float* __restrict__ pool, int64_t n,
-                                               int th, int tw, int ohl, int q, int cg, int Hp, int Wp) {
-  float h[5][8];
+// `staged` runs between the caller's two barriers: odd rows write, even rows read.
+__device__ __forceinline__ void stem_pool_rows(const float (&acc)[16][8], float (&h)[9][8]) {
 #pragma unroll
   for (int c = 0; c < 8; ++c) {
     h[0][c] = fmaxf(acc[0][c], acc[1][c]);
-    h[1][c] = fmaxf(fmaxf(acc[1][c], acc[2][c]), acc[3][c]);
-    h[2][c] = fmaxf(fmaxf(acc[3][c], acc[4][c]), acc[5][c]);
-    h[3][c] = fmaxf(fmaxf(acc[5][c], acc[6][c]), acc[7][c]);
-    h[4][c] = acc[7][c];
-    const float other = __shfl_xor_sync(0xffffffffu, h[0][c], 16);  // q = 1's columns 8, 9 of the tile
-    if (q == 0) h[4][c] = fmaxf(h[4][c], other);
-  }
-  constexpr int kRowF = 9 * kStemCout;  // one staged row: 9 pooled columns x 128 channels
-  __syncthreads();                      // every warp is done reading the input copies
-  if (ohl & 1) {
 #pragma unroll
-    for (int sl = 0; sl < 5; ++sl) {
-      if (q == 1 && sl == 0) continue;
-      float4* d = reinterpret_cast<float4*>(xs + (ohl >> 1) * kRowF + (4 * q + sl) * kStemCout + cg * 8);
-      d[0] = make_float4(h[sl][0], h[sl][1], h[sl][2], h[sl][3]);
-      d[1] = make_float4(h[sl][4], h[sl][5], h[sl][6], h[sl][7]);
-    }
-  }
-  __syncthreads();  // the odd rows staged
-  if ((ohl & 1) == 0 || ohl == kStemTH - 1) {
-    const int pr = (ohl + 1) >> 1;  // even rows: ohl / 2; the last row: pooled row 4
-    const int64_t pi = static_cast<int64_t>(th) * (kStemTH / 2) + pr;
-    if (pi < Hp) {
-#pragma unroll
-      for (int sl = 0; sl < 5; ++sl) {
-        if (q == 1 && sl == 0) continue;
-        const int pc = 4 * q + sl;
-        const int pj = tw * (kStemTW / 2) + pc;
-        if (pj >= Wp) continue;
-        float v[8];
-#pragma unroll
-        for (int c = 0; c < 8; ++c) v[c] = h[sl][c];
-        if ((ohl & 1) == 0) {
-          // rows ohl - 1 and ohl + 1 from the staged odd rows
-#pragma unroll
-          for (int rr = -1; rr <= 1; rr += 2) {
-            const int ro = ohl + rr;
-            if (ro < 0) continue;
-            const float4* sp = reinterpret_cast<const float4*>(xs + (ro >> 1) * kRowF + pc * kStemCout + cg * 8);
-            const float4 a = sp[0], b = sp[1];
-            v[0] = fmaxf(v[0], a.x); v[1] = fmaxf(v[1], a.y); v[2] = fmaxf(v[2], a.z); v[3] = fmaxf(v[3], a.w);
-            v[4] = fmaxf(v[4], b.x); v[5] = fmaxf(v[5], b.y); v[6] = fmaxf(v[6], b.z); v[7] = fmaxf(v[7], b.w);
-          }
-        }
-        float* dst = pool + ((n * Hp + pi) * Wp + pj) * kStemCout + cg * 8;
-        const bool whole = pr >= 1 && pr <= 3 && pc >= 1 && pc <= 7;
-        if (whole) {
-          reinterpret_cast<float4*>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
-          reinterpret_cast<float4*>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
-        } else {
-#pragma unroll
-          for (int c = 0; c < 8; ++c) atomicMax(reinterpret_cast<unsigned int*>(dst) + c, __float_as_uint(v[c]));
-        }
-      }
-    }
+    for (int k = 1; k < 8; ++k) h[k][c] = fmaxf(fmaxf(acc[2 * k - 1][c], acc[2 * k][c]), acc[2 * k + 1][c]);
+    h[8][c] = acc[15][c];
   }
 }
 
-__global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const float* __restrict__ x,
+__global__ void __launch_bounds__(kStemThreads, 1) pq_stem7x7s2_kernel(const float* __restrict__ x,
                                                                      const float* __restrict__ w,
                                                                      float* __restrict__ y, float* __restrict__ pool,
                                                                      int64_t N, int H, int W, int Ho, int Wo, int Hp,
                                                                      int Wp, int relu) {
   extern __shared__ float4 smem4[];
   float* ws = reinterpret_cast<float*>(smem4);  // [147][2][16][4]
-  float* xs = ws + kStemTerms * kStemCout;      // [copy 4][parity 2][ci 3][row 21][16]
+  float* xs = ws + kStemTerms * kStemCout;      // the window [copy 4][parity 2][ci 3][row 37][16]
+  float* raw = xs + kStemXFloats;               // the next window [row 37][column 37][ci 3]
+  float* pstage = raw + kStemRawF;              // odd rows' pooled columns [8][9][128]
   const int tiles_h = (Ho + kStemTH - 1) / kStemTH, tiles_w = (Wo + kStemTW - 1) / kStemTW;
   const int64_t n_tiles = N * tiles_h * tiles_w;
-  float pre[kStemLoads];
-  // Global loads of tile t's inputs (element i = (row, column, channel) of the
-  // 21 x 37 x 3 window, i = threadIdx.x + 256 e), zero outside the image.
+  // Tile t's window (element i = (row, column, channel) of the 37 x 37 x 3
+  // window, i = threadIdx.x + 256 e) into `raw` by 4-byte cp.async, zero-filled
+  // outside the image.
   auto fetch = [&](int64_t t) {
     const int tw = static_cast<int>(t % tiles_w);
     const int64_t r = t / tiles_w;
@@ -237,9 +209,10 @@ __global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const flo
       const int rr = i / (kStemIC * kStemCin), rem = i - rr * (kStemIC * kStemCin);
       const int c = rem / kStemCin, ci = rem - c * kStemCin;
       const int ih = ih0 + rr, iw = iw0 + c;
-      const bool valid = i < kStemTileElems && ih >= 0 && ih < H && iw >= 0 && iw < W;
-      pre[e] = valid ? x[((n * H + ih) * W + iw) * kStemCin + ci] : 0.0f;
+      const bool valid = ih >= 0 && ih < H && iw >= 0 && iw < W;
+      if (i < kStemTileElems) cp_async4(raw + i, valid ? x + ((n * H + ih) * W + iw) * kStemCin + ci : x, valid);
     }
+    asm volatile("cp.async.commit_group;" ::: "memory");
   };
   // The fetched window into the four shifted copies of its parity planes.
   auto scatter = [&]() {
@@ -247,13 +220,14 @@ __global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const flo
     for (int e = 0; e < kStemLoads; ++e) {
       const int i = threadIdx.x + e * kStemThreads;
       if (i < kStemTileElems) {
+        const float v = raw[i];
         const int rr = i / (kStemIC * kStemCin), rem = i - rr * (kStemIC * kStemCin);
         const int c = rem / kStemCin, ci = rem - c * kStemCin;
         const int k0 = c >> 1;
         float* dst = xs + ((c & 1) * kStemCin + ci) * kStemPlaneF + rr * kStemRowF + k0;
 #pragma unroll
         for (int sh = 0; sh < 4; ++sh)
-          if (k0 - sh >= 0 && k0 - sh < kStemRowF) dst[sh * kStemCopyF - sh] = pre[e];
+          if (k0 - sh >= 0 && k0 - sh < kStemRowF) dst[sh * kStemCopyF - sh] = v;
       }
     }
   };
@@ -266,23 +240,22 @@ __global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const flo
     const int h = rem >> 6, g = (rem >> 2) & 15, k = rem & 3;
     ws[i] = w[(g * 8 + h * 4 + k) * kStemTerms + term];
   }
-  const int cg = threadIdx.x & 15, pg = threadIdx.x >> 4;
-  const int ohl = pg >> 1, q = pg & 1;
-  const float* xthr = xs + (2 * ohl) * kStemRowF + 8 * q;
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
+  __syncthreads();  // the first window landed
+  scatter();
+  __syncthreads();  // the first window's copies and the weights visible to all threads
+  const int cg = threadIdx.x & 15, r = threadIdx.x >> 4;  // channel group, tile row
   const float* wthr = ws + cg * 4;
+  const float* xthr = xs + (2 * r) * kStemRowF;
   for (; t < n_tiles; t += gridDim.x) {
-    __syncthreads();  // every thread is done with the copies of the previous tile
-    scatter();
-    __syncthreads();  // the copies (and, the first time, the weights) visible to all threads
-    const int tw = static_cast<int>(t % tiles_w);
-    const int64_t r = t / tiles_w;
-    const int th = static_cast<int>(r % tiles_h);
-    const int64_t n = r / tiles_h;
-    float acc[8][8];
+    const bool more = t + gridDim.x < n_tiles;
+    if (more) fetch(t + gridDim.x);  // in flight during the FMAs
+    // the sums of pixel j, channels 2 k and 2 k + 1, as one 64-bit register pair
+    unsigned long long a2[16][4];
 #pragma unroll
-    for (int j = 0; j < 8; ++j)
+    for (int j = 0; j < 16; ++j)
 #pragma unroll
-      for (int c = 0; c < 8; ++c) acc[j][c] = 0.0f;
+      for (int k = 0; k < 4; ++k) a2[j][k] = 0ull;
 #pragma unroll 1
     for (int kh = 0; kh < kStemK; ++kh) {
       const float* xk = xthr + kh * kStemRowF;
@@ -293,26 +266,37 @@ __global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const flo
         for (int ci = 0; ci < kStemCin; ++ci) {
           const float4* xp =
               reinterpret_cast<const float4*>(xk + (kw >> 1) * kStemCopyF + ((kw & 1) * kStemCin + ci) * kStemPlaneF);
-          const float4 xa = xp[0], xb = xp[1];
+          const float4 x0 = xp[0], x1 = xp[1], x2 = xp[2], x3 = xp[3];
           const float* wt = wk + (kw * kStemCin + ci) * kStemCout;
-          const float4 wa = *reinterpret_cast<const float4*>(wt), wb = *reinterpret_cast<const float4*>(wt + 64);
-          const float xv[8] = {xa.x, xa.y, xa.z, xa.w, xb.x, xb.y, xb.z, xb.w};
+          // the weight pairs (channels 2 k, 2 k + 1) as they lie in shared memory
+          const ulonglong2 wa = *reinterpret_cast<const ulonglong2*>(wt);
+          const ulonglong2 wb = *reinterpret_cast<const ulonglong2*>(wt + 64);
+          const float xv[16] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w,
+                                x2.x, x2.y, x2.z, x2.w, x3.x, x3.y, x3.z, x3.w};
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            fma2_rn(acc[j][0], acc[j][1], xv[j], wa.x, wa.y);
-            fma2_rn(acc[j][2], acc[j][3], xv[j], wa.z, wa.w);
-            fma2_rn(acc[j][4], acc[j][5], xv[j], wb.x, wb.y);
-            fma2_rn(acc[j][6], acc[j][7], xv[j], wb.z, wb.w);
+          for (int j = 0; j < 16; ++j) {
+            const unsigned long long xx = f32x2_pair(xv[j], xv[j]);
+            ffma2(a2[j][0], xx, wa.x);
+            ffma2(a2[j][1], xx, wa.y);
+            ffma2(a2[j][2], xx, wb.x);
+            ffma2(a2[j][3], xx, wb.y);
           }
         }
       }
     }
-    // the next tile's loads are in flight while this one's outputs are stored
-    if (t + gridDim.x < n_tiles) fetch(t + gridDim.x);
-    const int oh = th * kStemTH + ohl;
+    float acc[16][8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-      const bool in_out = oh < Ho && tw * kStemTW + 8 * q + j < Wo;
+    for (int j = 0; j < 16; ++j)
+#pragma unroll
+      for (int k = 0; k < 4; ++k) f32x2_unpair(a2[j][k], acc[j][2 * k], acc[j][2 * k + 1]);
+    const int tw = static_cast<int>(t % tiles_w);
+    const int64_t rt = t / tiles_w;
+    const int th = static_cast<int>(rt % tiles_h);
+    const int64_t n = rt / tiles_h;
+    const int oh = th * kStemTH + r;
+#pragma unroll
+    for (int j = 0; j < 16; ++j) {
+      const bool in_out = oh < Ho && tw * kStemTW + j < Wo;
 #pragma unroll
       for (int c = 0; c < 8; ++c) {
         if (relu) acc[j][c] = fmaxf(acc[j][c], 0.0f);
@@ -321,13 +305,67 @@ __global__ void __launch_bounds__(kStemThreads, 2) pq_stem7x7s2_kernel(const flo
         if (pool != nullptr && !in_out) acc[j][c] = 0.0f;
       }
       if (y != nullptr && in_out) {
-        float4* yp = reinterpret_cast<float4*>(y + ((n * Ho + oh) * Wo + tw * kStemTW + 8 * q + j) * kStemCout + cg * 8);
+        float4* yp = reinterpret_cast<float4*>(y + ((n * Ho + oh) * Wo + tw * kStemTW + j) * kStemCout + cg * 8);
         yp[0] = make_float4(acc[j][0], acc[j][1], acc[j][2], acc[j][3]);
         yp[1] = make_float4(acc[j][4], acc[j][5], acc[j][6], acc[j][7]);
       }
     }
-    if (pool != nullptr) stem_pool_tile(acc, xs, pool, n, th, tw, ohl, q, cg, Hp, Wp);
+    // Every warp is done with this window and, from the previous tile, with the
+    // pooling stage, and every thread's copies of the next window have landed.
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+    __syncthreads();
+    if (more) scatter();
+    if (pool != nullptr) {
+      float h[9][8];
+      stem_pool_rows(acc, h);
+      if (r & 1) {
+#pragma unroll
+        for (int pc = 0; pc < 9; ++pc) {
+          float4* d = reinterpret_cast<float4*>(pstage + (r >> 1) * kStemPoolRowF + pc * kStemCout + cg * 8);
+          d[0] = make_float4(h[pc][0], h[pc][1], h[pc][2], h[pc][3]);
+          d[1] = make_float4(h[pc][4], h[pc][5], h[pc][6], h[pc][7]);
+        }
+      }
+      __syncthreads();  // the odd rows staged and the next window's copies written
+      if ((r & 1) == 0 || r == kStemTH - 1) {
+        const int pr = (r + 1) >> 1;  // even rows: r / 2; the last row: pooled row 8
+        const int64_t pi = static_cast<int64_t>(th) * (kStemTH / 2) + pr;
+        if (pi < Hp) {
+#pragma unroll
+          for (int pc = 0; pc < 9; ++pc) {
+            const int pj = tw * (kStemTW / 2) + pc;
+            if (pj >= Wp) continue;
+            float v[8];
+#pragma unroll
+            for (int c = 0; c < 8; ++c) v[c] = h[pc][c];
+            if ((r & 1) == 0) {
+#pragma unroll
+              for (int rr = -1; rr <= 1; rr += 2) {
+                const int ro = r + rr;
+                if (ro < 0) continue;
+                const float4* sp = reinterpret_cast<const float4*>(pstage + (ro >> 1) * kStemPoolRowF + pc * kStemCout + cg * 8);
+                const float4 pa = sp[0], pb = sp[1];
+                v[0] = fmaxf(v[0], pa.x); v[1] = fmaxf(v[1], pa.y); v[2] = fmaxf(v[2], pa.z); v[3] = fmaxf(v[3], pa.w);
+                v[4] = fmaxf(v[4], pb.x); v[5] = fmaxf(v[5], pb.y); v[6] = fmaxf(v[6], pb.z); v[7] = fmaxf(v[7], pb.w);
+              }
+            }
+            float* dst = pool + ((n * Hp + pi) * Wp + pj) * kStemCout + cg * 8;
+            const bool whole = pr >= 1 && pr <= kStemTH / 2 - 1 && pc >= 1 && pc <= 7;
+            if (whole) {
+              reinterpret_cast<float4*>(dst)[0] = make_float4(v[0], v[1], v[2], v[3]);
+              reinterpret_cast<float4*>(dst)[1] = make_float4(v[4], v[5], v[6], v[7]);
+            } else {
+#pragma unroll
+              for (int c = 0; c < 8; ++c) atomicMax(reinterpret_cast<unsigned int*>(dst) + c, __float_as_uint(v[c]));
+            }
+          }
+        }
+      }
+    } else {
+      __syncthreads();  // the next window's copies written
+    }
   }
+  asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
 
 // Max over the in-image taps of each window, fmaxf in (kh, kw) order from -inf.
@@ -488,7 +526,7 @@ pq_status palquant_conv2d_f32(const float* x_dev, const float* w_dev, float* y_d
     int dev = 0, sms = 148;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-    const unsigned grid = static_cast<unsigned>(tiles < static_cast<int64_t>(sms) * 2 ? tiles : sms * 2);
+    const unsigned grid = static_cast<unsigned>(tiles < static_cast<int64_t>(sms) ? tiles : sms);
     pq::pq_stem7x7s2_kernel<<<grid, pq::kStemThreads, pq::kStemSmem, s>>>(
         x_dev, w_dev, y_dev, nullptr, N, H, W, static_cast<int>(Ho), static_cast<int>(Wo), 0, 0, relu);
     return cudaGetLastError() == cudaSuccess ? PQ_OK : PQ_ECUDA;
@@ -528,7 +566,7 @@ pq_status palquant_stem_pool_f32(const float* x_dev, const float* w_dev, float* 
   int dev = 0, sms = 148;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const unsigned grid = static_cast<unsigned>(tiles < static_cast<int64_t>(sms) * 2 ? tiles : sms * 2);
+  const unsigned grid = static_cast<unsigned>(tiles < static_cast<int64_t>(sms) ? tiles : sms);
   pq::pq_stem7x7s2_kernel<<<grid, pq::kStemThreads, pq::kStemSmem, s>>>(
       x_dev, w_dev, stem_dev, pool_dev, N, H, W, static_cast<int>(Ho), static_cast<int>(Wo), static_cast<int>(Hp),
       static_cast<int>(Wp), 1);
