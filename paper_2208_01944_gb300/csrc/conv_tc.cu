@@ -432,8 +432,8 @@ __device__ __forceinline__ void unpack_role(const ConvParams& p, const Bars& bar
 // j, 2 Hd input rows of 2 Wd positions (16 bytes each) starting at input row
 // 2 (oh0 + h_off) and column 2 w_coord; staged row y = 2 r + a and column
 // x = 2 w + b go to row r, position w of the plane of stride phase (a, b) (the
-// phases no tap uses are skipped).  Warp wi takes staged rows wi, wi + 4, ...
-// and its lanes consecutive columns: conflict-free 16-byte reads, and 16-byte
+// phases no tap uses are skipped).  Warp wi takes window rows wi, wi + 4, ...
+// of every chunk and its lanes consecutive columns: conflict-free 16-byte reads, and 16-byte
 // writes in two runs of consecutive positions.  Positions outside the image were
 // zero-filled by the TMA unit (the zero padding).  The stage goes to the tensor
 // core after a proxy fence, the staging stage back to the producer.
@@ -442,12 +442,23 @@ __device__ __forceinline__ void split_role(const ConvParams& p, const Bars& bars
                                            int64_t it0, int64_t it1, const WaitCtx& ctx) {
   const int tid = threadIdx.x - 32 * kFirstLoadWarp;
   const int wi = tid >> 5, lane = tid & 31;
-  const int Hd = p.Hd, Wd = p.Wd, Ws = 2 * p.Wd;
-  const int n_rows = p.nch * 2 * Hd;
+  const int Hd = p.Hd, Wd = p.Wd, Ws = 2 * p.Wd, nch = p.nch;
   const uint32_t plane = p.lbo_a;
-  // destination offset of phase (a, b), or -1 where no tap reads it
-  int ph_off[2][2] = {{-1, -1}, {-1, -1}};
-  for (int q = 0; q < p.nph && q < kMaxPhases; ++q) ph_off[p.phase_a[q] & 1][p.phase_b[q] & 1] = q * p.a_phase_bytes;
+  // destination offset of phase (a, b), or -1 where no tap reads it, in
+  // registers (a dynamically indexed local array would live in local memory,
+  // one long-latency load per staged row)
+  int o00 = -1, o01 = -1, o10 = -1, o11 = -1;
+#pragma unroll
+  for (int q = 0; q < kMaxPhases; ++q) {
+    if (q >= p.nph) break;
+    const int v = q * static_cast<int>(p.a_phase_bytes);
+    const int pa = p.phase_a[q] & 1, pb = p.phase_b[q] & 1;
+    if (pa == 0) {
+      if (pb == 0) o00 = v; else o01 = v;
+    } else {
+      if (pb == 0) o10 = v; else o11 = v;
+    }
+  }
   Ring r{0, 0, static_cast<uint32_t>(p.a_stages)};
   bool ok = true;
   for (int64_t it = it0; it < it1 && ok; ++it) {
@@ -456,25 +467,26 @@ __device__ __forceinline__ void split_role(const ConvParams& p, const Bars& bars
       if (!warp_wait(bars.a_empty(r.stage), r.phase ^ 1u, ctx)) { ok = false; break; }
       const uint32_t src = pk_base + r.stage * p.pk_stage_bytes;
       const uint32_t dst = a_base + r.stage * p.a_stage_bytes;
-      for (int row = wi; row < n_rows; row += kLoadWarps) {
-        const int j = row / (2 * Hd), y = row - j * 2 * Hd;
+      for (int y = wi; y < 2 * Hd; y += kLoadWarps) {
         const int a = y & 1, rr = y >> 1;
-        const int off0 = ph_off[a][0], off1 = ph_off[a][1];
+        const int off0 = a ? o10 : o00, off1 = a ? o11 : o01;
         if (off0 < 0 && off1 < 0) continue;
-        const uint32_t srow = src + static_cast<uint32_t>(row * Ws) * 16u;
-        const uint32_t drow = dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(rr * Wd) * 16u;
-        for (int x = lane; x < Ws; x += 32) {
-          const int off = (x & 1) ? off1 : off0;
-          if (off < 0) continue;
-          uint32_t v0, v1, v2, v3;
-          asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
-                       : "=r"(v0), "=r"(v1), "=r"(v2), "=r"(v3)
-                       : "r"(srow + static_cast<uint32_t>(x) * 16u)
-                       : "memory");
-          asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(drow + static_cast<uint32_t>(off) +
-                                                                         static_cast<uint32_t>(x >> 1) * 16u),
-                       "r"(v0), "r"(v1), "r"(v2), "r"(v3)
-                       : "memory");
+        for (int j = 0; j < nch; ++j) {
+          const uint32_t srow = src + static_cast<uint32_t>((j * 2 * Hd + y) * Ws) * 16u;
+          const uint32_t drow = dst + static_cast<uint32_t>(j) * plane + static_cast<uint32_t>(rr * Wd) * 16u;
+          for (int x = lane; x < Ws; x += 32) {
+            const int off = (x & 1) ? off1 : off0;
+            if (off < 0) continue;
+            uint32_t v0, v1, v2, v3;
+            asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(v0), "=r"(v1), "=r"(v2), "=r"(v3)
+                         : "r"(srow + static_cast<uint32_t>(x) * 16u)
+                         : "memory");
+            asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(drow + static_cast<uint32_t>(off) +
+                                                                           static_cast<uint32_t>(x >> 1) * 16u),
+                         "r"(v0), "r"(v1), "r"(v2), "r"(v3)
+                         : "memory");
+          }
         }
       }
       fence_proxy_async_smem();
