@@ -236,9 +236,10 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // taking one warpgroup about 430 ns (550 ns for a 32-column FP4 unit), and its
   // warpgroups (three when TMA loads the operand, else two) take the units in
   // turn, so an uneven split costs a whole unit; an item costs 500 ns of
-  // overhead; weights too large to stay in shared memory are streamed again for
-  // every item, from L2 at about 40 B/ns per SM when all SMs stream (config 3,
-  // b=2, G=4: 147 KB per item).  Double-buffered accumulators come first.
+  // overhead; a unit's weights stay in shared memory up to 160 KB (beside two
+  // operand stages: config 3 at G=4 ran 63 -> 45 us once its 147 KB stayed),
+  // larger ones are streamed again for every item, from L2 at about 40 B/ns per SM
+  // when all SMs stream.  Double-buffered accumulators come first.
   const double ns_per_clk = 1.0 / 1.9;
   const double mma_ns = std::max(32.0 + p.Npow2 / 4.0, p.Npow2 / 2.0) * ns_per_clk;
   const double mma_acc_ns = static_cast<double>(p.taps) * (d->Cin_g / (32 * cpb)) * mma_ns;  // one accumulator
@@ -249,7 +250,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   const int units_per_acc = p.Nblk / unit_cols;
   const double unit_ns = unit_cols == 32 ? 550.0 : 430.0;
   const double w_unit_bytes = static_cast<double>(p.taps) * d->Cin_g * p.Nblk / cpb;
-  const double w_stream_ns = w_unit_bytes > 112.0 * 1024.0 ? w_unit_bytes / 40.0 : 0.0;  // per item
+  const double w_stream_ns = w_unit_bytes > 160.0 * 1024.0 ? w_unit_bytes / 40.0 : 0.0;  // per item
   const int tmem_avail = f4 ? 512 - 32 : 512;  // FP4: 32 columns hold the scale factors
   int best_mt = 0, best_ht = 0, best_tpi = 0, best_acc = 0;
   double best_cost = 0.0;
@@ -274,7 +275,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
       // two-slice ring) and the epilogue staging
       const uint64_t npos = flat ? 128u : static_cast<uint64_t>(ht + rmax - rmin) * Wh;
       const uint64_t w_unit = static_cast<uint64_t>(taps) * d->Cin_g * p.Nblk / cpb;
-      const uint64_t w_min = w_unit <= 112u * 1024u ? round_up(w_unit, 1024) : 2ull * round_up(32ull * p.Nblk, 1024);
+      const uint64_t w_min = 2ull * round_up(32ull * p.Nblk, 1024);  // a streamed ring at least (resident when it fits)
       const uint64_t need = 2ull * (cpb * round_up(npos * 128, 1024) + round_up(npos * 32, 1024)) + w_min +
                             static_cast<uint64_t>(pq::kEpiWarps) * warp_stage + 1024;
       if (need > pq::kMaxSmem - 1024) continue;
@@ -403,7 +404,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
     sb = a_stage_bytes(kc, &pb, &l);
     if (sb > 64u * 1024u) continue;
     for (int res = 1; res >= 0 && !found; --res) {
-      if (res && unit_bytes > 112u * 1024u) continue;
+      if (res && unit_bytes > 160u * 1024u) continue;
       const uint64_t slice = static_cast<uint64_t>(kc) * p.Nblk / cpb;
       if (!res && slice > 32u * 1024u) continue;
       for (int na = 4; na >= 2 && !found; --na) {
