@@ -914,7 +914,9 @@ template <int UC>
 __device__ __forceinline__ void epi_general_units(const ConvParams& p, const EpiItem& e, uint8_t* stg, int wg,
                                                   int n_groups, int quarter, int lane, uint32_t qmax2) {
   constexpr int CPR = UC / 4, RPP = 32 / CPR;  // chunks per row, rows per coalesced pass
-  constexpr uint32_t kBuf = 32u * UC * 4u;     // one staging buffer: 32 rows of UC values
+  // one staging buffer: 32 rows of 128 bytes whatever UC is, so that the NHWC code
+  // rows staged by epi_store_codes (32 rows at an 80-byte pitch) stay inside it
+  constexpr uint32_t kBuf = 32u * 128u;
   const bool has_sc = p.shortcut != nullptr;
   // With a shortcut (and no int32 output, which would need the buffer first) the
   // next unit's shortcut rows are fetched into the warp's second buffer while

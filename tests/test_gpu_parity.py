@@ -350,6 +350,28 @@ CODES_ONLY = [
 ]
 
 
+# Shortcut layers writing fp32 and codes but no int32 sums: the epilogue fetches the
+# next unit's shortcut rows while the current unit computes (two staging buffers a
+# warp).  16-column units (48 and 80 output channels), several units per warpgroup,
+# rows outside the output, stride 2, the channel shuffle and the cyclic shuffle.
+SHORTCUT_YQ = [
+    Case(2, 13, 11, 2, 32, 48, 3, 1, 1, shortcut=True, seed=50),
+    Case(1, 9, 10, 2, 64, 80, 3, 1, 1, shortcut=True, kind=1, shift=-1, seed=51),
+    Case(2, 36, 40, 2, 64, 64, 3, 1, 1, shortcut=True, seed=52),
+    Case(2, 12, 14, 2, 64, 128, 3, 2, 1, shortcut=True, seed=53),
+    Case(2, 9, 9, 4, 32, 32, 3, 1, 1, shortcut=True, kind=2, seed=54),
+    Case(2, 7, 9, 2, 96, 96, 1, 1, 0, shortcut=True, relu=False, seed=55),
+]
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=["nhwc", "c16"])
+@pytest.mark.parametrize("c", SHORTCUT_YQ, ids=str)
+def test_layer_shortcut_y_and_codes_matches_oracle(B, c, fmt):
+    ref = prepare(c)
+    got = run_gpu(c, ref, outputs=("y", "q"), fmt=fmt)
+    assert_layer_parity(c, ref, got)
+
+
 @pytest.mark.parametrize("fmt", FORMATS, ids=["nhwc", "c16"])
 @pytest.mark.parametrize("c", CODES_ONLY, ids=str)
 def test_layer_codes_only_matches_oracle(B, c, fmt):
