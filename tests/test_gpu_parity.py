@@ -97,6 +97,8 @@ SMALL_CASES = [
     Case(2, 20, 20, 2, 64, 64, 1, 1, 0, seed=19),                     # flat, two boxes per tile, ragged
     Case(2, 17, 17, 2, 64, 64, 1, 1, 0, shortcut=True, seed=20),      # flat, second box wholly past the image
     Case(1, 6, 140, 2, 32, 32, 3, 2, 1, seed=21),                     # stride 2, window wider than one TMA box row
+    Case(2, 11, 10, 2, 32, 48, 3, 1, 1, shortcut=True, seed=22),      # shortcut with int32 sums, 16-column units
+    Case(2, 13, 15, 2, 32, 32, 5, 2, 2, seed=23),                     # 5x5 stride 2: a window of 4 phases, 3 taps each way
 ]
 
 
