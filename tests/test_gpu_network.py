@@ -110,8 +110,9 @@ def test_device_calibration_close_to_oracle():
 
 # ------------------------------------------------------------ full-precision layers alone
 @pytest.mark.parametrize("shape,Cout,k,s,p,relu", [
-    ((2, 37, 29, 3), 64, 7, 2, 3, True),     # the stem kernel, ragged tiles
-    ((1, 224, 224, 3), 128, 7, 2, 3, True),  # the network's stem shape
+    ((2, 37, 29, 3), 64, 7, 2, 3, True),     # the stem shape at 64 channels (the generic kernel)
+    ((1, 224, 224, 3), 128, 7, 2, 3, True),  # the network's stem shape (the stem kernel)
+    ((2, 30, 34, 3), 128, 7, 2, 3, False),   # the stem kernel without ReLU, ragged tiles
     ((2, 9, 11, 5), 32, 3, 1, 1, False),     # the generic kernel, weights in shared memory
     ((1, 12, 10, 64), 48, 5, 2, 2, True),    # the generic kernel, weights from global memory
 ])
