@@ -387,13 +387,16 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
     const uint64_t rows = flat ? 1 : p.Hd;
     return round_up(static_cast<uint64_t>(pk_box_w) * rows * (KC / 16) * 4, 1024);
   };
-  // Largest K block (input channels per pipeline stage) that fits: the whole
-  // unit's weights resident if they fit, else a ring of (K block, tap) slices.
+  // Largest K block (input channels per pipeline stage) that fits with the whole
+  // unit's weights resident, else the largest with a ring of (K block, tap)
+  // slices (the stage-4 conv1 of the network: 84 -> 72 us with conv1 + down once
+  // its 147 KB of weights stayed at half the K block).
   bool found = false, resident = false;
   int KC = d->Cin_g, a_stages = 0, b_stages = 0;
   uint32_t stage_bytes = 0, phase_bytes = 0, lbo = 0;
   // K blocks of {8, 4, 3, 2, 1} MMA K steps (32 channels each, 64 for FP4): the
   // MMA issue loop is compiled for these K-step counts.
+  for (int pass = 1; pass >= 0 && !found; --pass)
   for (int kc1 : {256, 128, 96, 64, 32}) {
     if (found) break;
     // at most four 32-channel fp32 boxes per stage, a power-of-two chunk count
@@ -403,7 +406,7 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
     uint32_t sb, pb, l;
     sb = a_stage_bytes(kc, &pb, &l);
     if (sb > 64u * 1024u) continue;
-    for (int res = 1; res >= 0 && !found; --res) {
+    for (int res = pass; res >= pass && !found; --res) {
       if (res && unit_bytes > 160u * 1024u) continue;
       const uint64_t slice = static_cast<uint64_t>(kc) * p.Nblk / cpb;
       if (!res && slice > 32u * 1024u) continue;
