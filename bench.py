@@ -363,6 +363,15 @@ def run_reference(args, rank, world):
 # ---------------------------------------------------------------------------
 L2_BYTES = 126 * 1024 * 1024
 
+# Tensor-core rates (TFLOP/s, 2 x MACs) that an MMA issue-loop probe measured on
+# this GB300 by the MMA's N (M = 128, cta_group::1, one CTA per SM issuing nine
+# taps of shifted A addresses with nothing else running): the ceiling of the MMA
+# shape a layer's plan uses.  N = 64 is bound by shared-memory operand reads (6 KB
+# per MMA, 24.6 ns for FP8 K = 32 and block-scaled FP4 K = 64 alike); N >= 128 by
+# the tensor core (FP8 4.86, FP4 9.73 PFLOP/s).
+MMA_PROBE_TFLOPS = {"fp8": {64: 3238.0, 128: 4843.0, 256: 4858.0},
+                    "fp4": {64: 6486.0, 128: 9708.0, 256: 9732.0}}
+
 
 def measure_layer_configs(dev, args):
     """Each config's fused layer in timed mode (channel-blocked codes in, codes out)
@@ -413,7 +422,9 @@ def measure_layer_configs(dev, args):
         byt = c.in_elems + c.out_elems + c.weight_elems
         tops = c.int_ops / (ms / 1e3) / 1e12
         plan = B.palquant_conv_plan(d).as_dict()
+        probe = None if plan["pointwise"] else MMA_PROBE_TFLOPS["fp8"].get(plan["n_block"])
         out[name] = {"shape": c.name, "us": ms * 1e3, "tops": tops, "frac_fp8_peak": tops / fp8_peak,
+                     "frac_mma_probe": tops / probe if probe else None,
                      "algorithmic_gbs": byt / (ms / 1e3) / 1e9, "frac_hbm": byt / (ms / 1e3) / 1e9 / pk["hbm_gbs"],
                      "buffer_sets": n_sets,
                      "kernel": "pq_pointwise_tc_kernel" if plan["pointwise"] else "pq_conv_tc_kernel",
@@ -437,8 +448,10 @@ def measure_layer_configs(dev, args):
             tops4 = c.int_ops / (ms4 / 1e3) / 1e12
             byt4 = nin + nout + c.weight_elems // 2
             plan4 = B.palquant_conv_plan(d4).as_dict()
+            probe4 = MMA_PROBE_TFLOPS["fp4"].get(plan4["n_block"])
             out[name + "_fp4"] = {"shape": c.name + ", packed FP4 codes", "us": ms4 * 1e3, "tops": tops4,
                                   "frac_fp4_peak": tops4 / fp4_peak, "frac_fp8_peak": tops4 / fp8_peak,
+                                  "frac_mma_probe": tops4 / probe4 if probe4 else None,
                                   "algorithmic_gbs": byt4 / (ms4 / 1e3) / 1e9,
                                   "frac_hbm": byt4 / (ms4 / 1e3) / 1e9 / pk["hbm_gbs"], "buffer_sets": n4,
                                   "plan": {k: plan4[k] for k in ("m_tiles", "n_block", "k_chunk", "weights_resident",
