@@ -1122,6 +1122,7 @@ __device__ __forceinline__ void epilogue_role(const ConvParams& p, const Bars& b
   uint8_t* stg = stage_base + ew * p.stage_warp_bytes;
   Ring racc{0, 0, static_cast<uint32_t>(p.acc_stages)};
   const int nchunks = p.Nblk >> 4;
+  const int n_units = p.MT * nchunks;
   const bool codes_only = p.shortcut == nullptr && p.y_out == nullptr && p.acc_out == nullptr && !p.channel_shuffle;
   // The group's multipliers and destination stay in registers while consecutive
   // items share the group (items run group by group); a dynamically indexed
