@@ -506,7 +506,10 @@ typedef struct {
     int32_t taps;          /* kh*kw */
     int32_t weights_resident; /* 1 if a group's weights stay in shared memory */
     int32_t acc_stages;    /* tensor-memory accumulator buffers */
-    int32_t smem_bytes;    /* dynamic shared memory per CTA */
+    int32_t smem_bytes;    /* dynamic shared memory per CTA of a call that stages its
+                              outputs; a call writing channel-blocked codes only (no
+                              int32 or fp32 outputs, no shortcut) reserves no per-warp
+                              staging and launches with less */
     int64_t tiles;         /* tiles per (group, n-block) unit */
     int64_t work_items;    /* tiles * G * n_blocks */
     int32_t pointwise;     /* 1 if a call writing channel-blocked codes only (no int32 or
