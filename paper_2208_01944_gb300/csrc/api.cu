@@ -237,7 +237,8 @@ pq_status plan_conv(const pq_layer_desc* d, ConvParams* P, pq_conv_plan* pub, st
   // warpgroups (three when TMA loads the operand, else two) take the units in
   // turn, so an uneven split costs a whole unit; an item costs 500 ns of
   // overhead; a unit's weights stay in shared memory up to 160 KB (beside two
-  // operand stages: config 3 at G=4 ran 63 -> 45 us once its 147 KB stayed),
+  // operand stages: a 3x3 layer of 128x28x28 with 4 groups of 128 ran 63 -> 45 us
+  // once its 147 KB stayed),
   // larger ones are streamed again for every item, from L2 at about 40 B/ns per SM
   // when all SMs stream.  Double-buffered accumulators come first.
   const double ns_per_clk = 1.0 / 1.9;
