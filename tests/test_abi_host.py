@@ -61,6 +61,23 @@ def test_plan_invariants(c):
     assert plan.acc_stages * plan.m_tiles * plan.n_block <= 512
 
 
+def test_plan_weight_residency():
+    """A (group, output block) unit's packed weights stay in shared memory only up to
+    160 KB; the 3x3 layers of 128x28x28 with 4 groups of 128 (147 KB a unit) keep
+    theirs, the 2-group ones (590 KB at 256 columns) stream them."""
+    for c in ALL_LAYERS:
+        plan = B.palquant_conv_plan(_desc(c))
+        unit_bytes = c.k * c.k * c.Cin_g * plan.n_block
+        if unit_bytes > 160 * 1024:
+            assert plan.weights_resident == 0, c
+    for name in ("config3_1", "config3_4"):
+        c = workloads.BENCH_CONFIGS[name]
+        plan = B.palquant_conv_plan(_desc(c))
+        assert (c.G, c.Cin_g, plan.n_block, plan.weights_resident) == (4, 128, 128, 1)
+    plan = B.palquant_conv_plan(_desc(workloads.BENCH_CONFIGS["config3_0"]))
+    assert plan.weights_resident == 0
+
+
 @pytest.mark.parametrize("shape", [(2, 48, 3, 64, 4), (4, 96, 1, 96, 2), (1, 272, 3, 32, 2), (3, 64, 3, 128, 4)])
 def test_pack_unpack_roundtrip_and_fp8_encoding(shape):
     G, Co, k, Ci, bits = shape
