@@ -440,40 +440,111 @@ __global__ void __launch_bounds__(256) pq_avgpool_f32_kernel(const float* __rest
   }
 }
 
-// y[n, o] = fma over i in order of x[n, i] w[o, i] (no bias).  A block computes
-// 32 outputs x 8 images (warp = one image, lane = one output); 64-wide chunks of
-// x and w are staged in shared memory (w rows at pitch 65, so the lanes' reads of
-// one column fall in distinct banks).  Every output keeps one running sum in
-// register across the chunks, so the order of its terms is i = 0, 1, 2, ...
-constexpr int kFcO = 32, kFcN = 8, kFcK = 64;
-
-__global__ void __launch_bounds__(kFcO * kFcN) pq_linear_f32_kernel(const float* __restrict__ x,
-                                                                   const float* __restrict__ w,
-                                                                   float* __restrict__ y, int64_t N, int Cin,
-                                                                   int Cout) {
-  __shared__ float xs[kFcN][kFcK];
-  __shared__ float wsh[kFcO][kFcK + 1];
-  const int lane = threadIdx.x & 31, wn = threadIdx.x >> 5;
-  const int o = blockIdx.x * kFcO + lane;
-  const int64_t n = static_cast<int64_t>(blockIdx.y) * kFcN + wn;
-  float acc = 0.0f;
-  for (int c0 = 0; c0 < Cin; c0 += kFcK) {
-    const int kc = min(kFcK, Cin - c0);
-    __syncthreads();
-    for (int i = threadIdx.x; i < kFcN * kFcK; i += blockDim.x) {
-      const int r = i / kFcK, c = i - r * kFcK;
-      const int64_t nn = static_cast<int64_t>(blockIdx.y) * kFcN + r;
-      xs[r][c] = (c < kc && nn < N) ? x[nn * Cin + c0 + c] : 0.0f;
+// The same sums for four consecutive channels per thread (C % 4 == 0, 16-byte
+// aligned rows): each channel's terms are still added in (h, w) order from 0; the
+// loop is unrolled so that the loads of several positions are in flight at once.
+__global__ void __launch_bounds__(128) pq_avgpool_f32_vec4_kernel(const float4* __restrict__ x,
+                                                                 float4* __restrict__ y, int64_t N, int HW, int C4) {
+  const int64_t total = N * C4;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < total;
+       i += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+    const int64_t n = i / C4;
+    const int64_t c4 = i - n * C4;
+    const float4* p = x + n * HW * C4 + c4;
+    float4 a = make_float4(0.0f, 0.0f, 0.0f, 0.0f);
+#pragma unroll 7
+    for (int j = 0; j < HW; ++j) {
+      const float4 v = __ldg(p + static_cast<int64_t>(j) * C4);
+      a.x = __fadd_rn(a.x, v.x);
+      a.y = __fadd_rn(a.y, v.y);
+      a.z = __fadd_rn(a.z, v.z);
+      a.w = __fadd_rn(a.w, v.w);
     }
-    for (int i = threadIdx.x; i < kFcO * kFcK; i += blockDim.x) {
-      const int r = i / kFcK, c = i - r * kFcK;
-      const int oo = blockIdx.x * kFcO + r;
-      wsh[r][c] = (c < kc && oo < Cout) ? w[static_cast<int64_t>(oo) * Cin + c0 + c] : 0.0f;
-    }
-    __syncthreads();
-    for (int c = 0; c < kc; ++c) acc = __fmaf_rn(xs[wn][c], wsh[lane][c], acc);
+    const float hw = static_cast<float>(HW);
+    y[i] = make_float4(__fdiv_rn(a.x, hw), __fdiv_rn(a.y, hw), __fdiv_rn(a.z, hw), __fdiv_rn(a.w, hw));
   }
-  if (o < Cout && n < N) y[n * Cout + o] = acc;
+}
+
+// y[n, o] = fma over i in order of x[n, i] w[o, i] (no bias).  A block computes
+// 32 outputs x 16 images: lane = output, warp w = images 2w and 2w + 1, so a
+// thread keeps two running sums, each over i = 0, 1, 2, ... in order.  128-wide
+// chunks of x (as image pairs) and w (rows at pitch 129, so the lanes' reads of
+// one column fall in distinct banks) are staged in shared memory; the next
+// chunk's global loads are issued into registers before the current chunk's
+// FMAs and stored after them.
+constexpr int kFcO = 32, kFcN = 16, kFcK = 128, kFcThreads = 256;
+constexpr int kFcXPer = kFcN * kFcK / kFcThreads;  // 8 x values a thread loads per chunk
+constexpr int kFcWPer = kFcO * kFcK / kFcThreads;  // 16 w values a thread loads per chunk
+
+__global__ void __launch_bounds__(kFcThreads) pq_linear_f32_kernel(const float* __restrict__ x,
+                                                                  const float* __restrict__ w,
+                                                                  float* __restrict__ y, int64_t N, int Cin,
+                                                                  int Cout) {
+  __shared__ float2 xs[kFcN / 2][kFcK];
+  __shared__ float wsh[kFcO][kFcK + 1];
+  const int t = threadIdx.x, lane = t & 31, wn = t >> 5;
+  const int o = blockIdx.x * kFcO + lane;
+  const int64_t n0 = static_cast<int64_t>(blockIdx.y) * kFcN;
+  float xr[kFcXPer], wr[kFcWPer];
+  // element e = t + kFcThreads * r of a chunk: x row e / kFcK (an image), w row
+  // e / kFcK (an output), column e % kFcK; consecutive threads read consecutive
+  // columns of one row.
+  auto load = [&](int c0) {
+#pragma unroll
+    for (int r = 0; r < kFcXPer; ++r) {
+      const int e = t + kFcThreads * r, img = e / kFcK, c = e % kFcK;
+      xr[r] = (c0 + c < Cin && n0 + img < N) ? __ldg(x + (n0 + img) * Cin + c0 + c) : 0.0f;
+    }
+#pragma unroll
+    for (int r = 0; r < kFcWPer; ++r) {
+      const int e = t + kFcThreads * r, row = e / kFcK, c = e % kFcK;
+      const int oo = blockIdx.x * kFcO + row;
+      wr[r] = (c0 + c < Cin && oo < Cout) ? __ldg(w + static_cast<int64_t>(oo) * Cin + c0 + c) : 0.0f;
+    }
+  };
+  auto store = [&]() {
+#pragma unroll
+    for (int r = 0; r < kFcXPer; ++r) {
+      const int e = t + kFcThreads * r, img = e / kFcK, c = e % kFcK;
+      float* p = reinterpret_cast<float*>(&xs[img >> 1][c]);
+      p[img & 1] = xr[r];
+    }
+#pragma unroll
+    for (int r = 0; r < kFcWPer; ++r) {
+      const int e = t + kFcThreads * r, row = e / kFcK, c = e % kFcK;
+      wsh[row][c] = wr[r];
+    }
+  };
+  float acc0 = 0.0f, acc1 = 0.0f;
+  load(0);
+  for (int c0 = 0; c0 < Cin; c0 += kFcK) {
+    __syncthreads();  // the previous chunk's reads are done
+    store();
+    __syncthreads();
+    if (c0 + kFcK < Cin) load(c0 + kFcK);
+    const int kc = min(kFcK, Cin - c0);
+    if (kc == kFcK) {
+#pragma unroll 16
+      for (int c = 0; c < kFcK; ++c) {
+        const float2 xv = xs[wn][c];
+        const float wv = wsh[lane][c];
+        acc0 = __fmaf_rn(xv.x, wv, acc0);
+        acc1 = __fmaf_rn(xv.y, wv, acc1);
+      }
+    } else {
+      for (int c = 0; c < kc; ++c) {
+        const float2 xv = xs[wn][c];
+        const float wv = wsh[lane][c];
+        acc0 = __fmaf_rn(xv.x, wv, acc0);
+        acc1 = __fmaf_rn(xv.y, wv, acc1);
+      }
+    }
+  }
+  const int64_t na = n0 + 2 * wn;
+  if (o < Cout) {
+    if (na < N) y[na * Cout + o] = acc0;
+    if (na + 1 < N) y[(na + 1) * Cout + o] = acc1;
+  }
 }
 
 unsigned grid_for(int64_t work, int per_sm) {
@@ -596,8 +667,20 @@ pq_status palquant_avgpool_f32(const float* x_dev, float* y_dev, int64_t N, int3
                                pq_stream_t stream) {
   if (N < 0 || H <= 0 || W <= 0 || C <= 0 || !x_dev || !y_dev) return PQ_EINVAL;
   if (N == 0) return PQ_OK;
-  pq::pq_avgpool_f32_kernel<<<pq::grid_for(N * C, 8), 256, 0, static_cast<cudaStream_t>(stream)>>>(x_dev, y_dev, N,
-                                                                                                    H * W, C);
+  if (C % 4 == 0 && pq::aligned16(x_dev) && pq::aligned16(y_dev)) {
+    const int64_t work = N * (C / 4);
+    int dev = 0, sms = 148;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    const int64_t want = (work + 127) / 128, cap = static_cast<int64_t>(sms) * 16;
+    pq::pq_avgpool_f32_vec4_kernel<<<static_cast<unsigned>(want < cap ? want : cap), 128, 0,
+                                     static_cast<cudaStream_t>(stream)>>>(reinterpret_cast<const float4*>(x_dev),
+                                                                          reinterpret_cast<float4*>(y_dev), N, H * W,
+                                                                          C / 4);
+  } else {
+    pq::pq_avgpool_f32_kernel<<<pq::grid_for(N * C, 8), 256, 0, static_cast<cudaStream_t>(stream)>>>(x_dev, y_dev, N,
+                                                                                                      H * W, C);
+  }
   return cudaGetLastError() == cudaSuccess ? PQ_OK : PQ_ECUDA;
 }
 
@@ -608,7 +691,7 @@ pq_status palquant_linear_f32(const float* x_dev, const float* w_dev, float* y_d
   const int64_t gy = (N + pq::kFcN - 1) / pq::kFcN;
   if (gy > 65535) return PQ_EUNSUPPORTED;
   const dim3 grid(static_cast<unsigned>((Cout + pq::kFcO - 1) / pq::kFcO), static_cast<unsigned>(gy));
-  pq::pq_linear_f32_kernel<<<grid, pq::kFcO * pq::kFcN, 0, static_cast<cudaStream_t>(stream)>>>(x_dev, w_dev, y_dev,
+  pq::pq_linear_f32_kernel<<<grid, pq::kFcThreads, 0, static_cast<cudaStream_t>(stream)>>>(x_dev, w_dev, y_dev,
                                                                                                N, Cin, Cout);
   return cudaGetLastError() == cudaSuccess ? PQ_OK : PQ_ECUDA;
 }
