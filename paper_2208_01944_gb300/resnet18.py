@@ -122,6 +122,7 @@ class PalQuantResNet18:
         self.ones = np.ones(G, dtype=np.float32)
         self.steps = None
         self.graph = None
+        self.fuse_input = False  # set by set_steps()
 
     # --------------------------------------------------------------- set-up
     def _inv(self, s, shuf=None):
@@ -291,6 +292,21 @@ class PalQuantResNet18:
             # conv2's codes land in group dst(g) of the next block: multiplier fl(1/s_next[dst(g)])
             blk["m_req2"] = None if nxt is None else self._inv(self.steps[nxt], self.cyclic)
         self.inv_in = self._inv(self.steps[self.blocks[0]["name"] + ".in"])
+        # The input quantiser runs inside the first conv1 (quantise-on-load: the fp32
+        # pooled tensor in, its codes only in shared memory) where that layer can take
+        # it: stride 1 and no downsample reading the input codes.  A shape the fused
+        # call rejects keeps the separate quantiser.
+        b0 = self.blocks[0]
+        self.fuse_input = False
+        if not b0["down"] and b0["stride"] == 1:
+            try:
+                B.palquant_quantize_layer_fused(self.pool, self.inv_in, b0["wp1"], b0["d1"], b0["m_out1"],
+                                                b0["m_req1"], self.no_shuffle, None, None, None, b0["mid_codes"],
+                                                stream=self.stream)
+                self.fuse_input = True
+            except B.PalquantError as e:
+                if e.status not in (B.PQ_EUNSUPPORTED, B.PQ_EINVAL):
+                    raise
         self.stream.synchronize()
         self.graph = None
 
@@ -336,9 +352,11 @@ class PalQuantResNet18:
         mark("start")
         self._stem(x_dev)
         mark("stem conv + max pooling (fp32)")
-        B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, self.G, self.C0 // self.G,
-                                self.bits, self.inv_in, code_format=self.fmt, stream=s)
-        mark("input quantiser")
+        fused_in = self.fuse_input and not self.paper
+        if not fused_in:
+            B.palquant_quantize_act(self.pool, self.in_codes, self.N, self.Hp, self.Wp, self.G, self.C0 // self.G,
+                                    self.bits, self.inv_in, code_format=self.fmt, stream=s)
+            mark("input quantiser")
         if self.paper:
             X = self.pool
             for k, m in enumerate(self.modules):
@@ -362,9 +380,15 @@ class PalQuantResNet18:
                 X = b2["out"]
         else:
             for i, blk in enumerate(self.blocks):
-                q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]
-                self._block_front(blk, q_in)
-                mark(blk["name"] + " conv1" + (" + down" if blk["down"] else ""))
+                if i == 0 and fused_in:
+                    B.palquant_quantize_layer_fused(self.pool, self.inv_in, blk["wp1"], blk["d1"], blk["m_out1"],
+                                                    blk["m_req1"], self.no_shuffle, None, None, None,
+                                                    blk["mid_codes"], stream=s)
+                    mark(blk["name"] + " conv1 (input quantiser fused)")
+                else:
+                    q_in = self.in_codes if i == 0 else self.blocks[i - 1]["out_codes"]
+                    self._block_front(blk, q_in)
+                    mark(blk["name"] + " conv1" + (" + down" if blk["down"] else ""))
                 self._conv2(blk, blk["m_req2"])
                 mark(blk["name"] + " conv2")
         last = self.blocks[-1]["out"]
@@ -394,6 +418,8 @@ class PalQuantResNet18:
         128 stem channels, else two), quantiser, per block conv1 (+ down) + conv2,
         average pooling, FC."""
         n = (2 if self.fused_stem else 3) + sum(3 if b["down"] else 2 for b in self.blocks) + 2
+        if self.fuse_input and not self.paper:
+            n -= 1  # the quantiser runs inside the first conv1
         if self.paper:
             n += len(self.modules) + len(self.modules) - 1  # a module per stage, a quantiser per stage boundary
         return n

@@ -26,7 +26,8 @@ def _compare(net, r):
     if net.stem_out is not None:
         assert np.array_equal(net.stem_out.cpu().numpy(), r["stem"]), "stem"
     assert np.array_equal(net.pool.cpu().numpy(), r["pool"]), "max pooling"
-    assert np.array_equal(_codes(net.in_codes, f), r[net.blocks[0]["name"] + ".in_codes"]), "input codes"
+    if not net.fuse_input:  # else the input codes exist only inside the first conv1
+        assert np.array_equal(_codes(net.in_codes, f), r[net.blocks[0]["name"] + ".in_codes"]), "input codes"
     for i, blk in enumerate(net.blocks):
         n = blk["name"]
         assert np.array_equal(_codes(blk["mid_codes"], f), r[n + ".mid_codes"]), n + " conv1 codes"
