@@ -8,7 +8,8 @@ takes the following reading:
 
 * stem: 7x7 stride-2 pad-3 fp32 convolution (3 -> G*w_1 channels) + ReLU, then 3x3
   stride-2 pad-1 max pooling (one kernel for 128 stem channels); the pooled tensor
-  is quantised once into codes;
+  is quantised once into codes (inside the first conv1, which then reads the pooled
+  fp32 and quantises it on load, where that layer allows it);
 * four stages of two basic blocks (per-group widths w_1..w_4).  In block (X, Q):
     conv1  PalQuant 3x3 (stride 2 in the first block of stages 2-4), ReLU, no
            permutation, codes out (requantised with conv2's input steps);
